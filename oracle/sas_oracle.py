@@ -1,0 +1,286 @@
+"""Plain fp64 CPU oracle for the SAS attention forward and the dense GELU MLP.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import, call or
+execute this module: only the tests, the smoke check and the benchmark's CPU
+baseline leg use it.  It shares no code with the CUDA library; the two meet
+only through the seeded input generator, which holds none of the method's
+arithmetic.
+
+What it computes (SAS, "Simple Attention Sparsification", arXiv 2609.13141):
+
+  a1  block summaries      Kbar_m = mean of the keys of block B_m            (Sec. 7 limitation: "pooling based block summaries")
+  a2  selector scores      s_im = R_theta(q_i, {K_Bm})                       (Alg. 1 step 1; Sec. 4.3)
+  a3  causal log-gates     log g_m = s_m - LSE(s) over the row's history     (Eq. normalized_log_gate)
+  a4  Top-K selection      I = TopK(g, K) = TopK(s, K)                       (Eq. selected_context; Alg. 1 / Alg. 2)
+  a5  gated attention      o = softmax(q K_S^T + log g_S) V_S                (Eq. ours_train; Alg. 2 for the ungated form)
+  a6  dense MLP (not SAS)  Y = GELU(X W1^T + b1) W2^T + b2, exact-erf GELU
+
+Readings of points the paper leaves open (each one is also listed with its
+reasoning in the design notes of the repository):
+
+  * sm_scale multiplies q.k only; the log-gate is added unscaled (Alg. 3,
+    gated_scores).
+  * Token j is in block floor(j / b).  For query i the current block B_0 is
+    block floor(i / b), restricted causally to keys j <= i, always kept with a
+    unit gate; its historical blocks are 0 .. floor(i / b) - 1, so
+    C_i = floor(i / b) (Sec. 4.1, Eq. general_gate).
+  * The gate softmax runs over all C_i historical blocks of the row, not only
+    the selected ones, and is not renormalised after selection (Eq.
+    normalized_log_gate; Eq. scope_grad).
+  * Top-K is exact-K: order by (score descending, block index ascending), so a
+    tie goes to the lower block index.  Rows with C_i <= K keep every
+    historical block; K = 0 keeps none (only the current block).
+  * Selection uses the scores s, never the computed log-gates (the two orders
+    agree because log g = s - const; Alg. 1 vs Alg. 2).
+  * Selector R_theta (MEANPOOL_PROJ): the paper names the AttnGate of
+    SeerAttention-R without describing it.  The reading used here is
+    q~_i = bf16(q_i Wq), K~_m = bf16(Kbar_m Wk), s_im = q~_i . K~_m / sqrt(d_s).
+    The two projections are bf16 activations, as in a bf16 model.
+    PARITY UNPINNED for the selector architecture itself: no paper value
+    exists to check it against; only its arithmetic is pinned.
+  * MLP: the hidden activation GELU(X W1^T + b1) is a bf16 tensor between the
+    two products (the precision of a stored bf16 activation).
+
+Arrays are float64 numpy arrays holding the bf16-rounded inputs the GPU sees.
+One "head" means one (batch, head) pair; Q, K, V of a head are [N, d].
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+MODE_TRAIN_SOFT = 0   # Eq. ours_train: selected historical blocks get + log g
+MODE_INFER_HARD = 1   # Alg. 2: selected historical blocks get no bias
+
+
+# ---------------------------------------------------------------- rounding --
+
+def round_to_bf16(x):
+    """Round float64 values to the nearest bfloat16 value, ties to even.
+
+    bfloat16 keeps 8 significant bits and the float32 exponent range.  For a
+    value with binary exponent e (2**e <= |x| < 2**(e+1)) the spacing of
+    bfloat16 numbers is 2**(e-7); below 2**-126 the spacing stays 2**-133
+    (subnormals).  Division by a power of two is exact, and numpy's rint
+    rounds half to even, so this is a single correctly rounded step.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    out = np.zeros_like(x)
+    nz = x != 0
+    _, e = np.frexp(x[nz])               # x = m * 2**e with 0.5 <= |m| < 1
+    e = np.maximum(e - 1, -126)          # floor(log2|x|), clamped at the subnormal range
+    ulp = np.ldexp(1.0, e - 7)
+    out[nz] = np.rint(x[nz] / ulp) * ulp
+    return out
+
+
+# ----------------------------------------------------------- block layout --
+
+def num_blocks(N, b):
+    """C = ceil(N / b) contiguous token blocks (Sec. 3, block partition)."""
+    return -(-N // b)
+
+
+def historical_count(i, b):
+    """C_i = floor(i / b): blocks strictly before query i's current block (Sec. 4.1)."""
+    return i // b
+
+
+# --------------------------------------------------------------- a1 / a2 --
+
+def block_summaries(K, b):
+    """a1: Kbar[m] = (1/b) * sum of k_j over the b tokens j of block m.
+
+    Only full blocks are summarised (m < floor(N / b)): a partial last block
+    is never historical for any query, because a query's historical blocks all
+    precede its own block.
+    """
+    N, d = K.shape
+    F = N // b
+    out = np.zeros((F, d))
+    for m in range(F):
+        out[m] = K[m * b:(m + 1) * b].sum(axis=0) / b
+    return out
+
+
+def selector_scores(Q, K, Wq, Wk, b):
+    """a2 (MEANPOOL_PROJ reading of R_theta): s[i, m] for every row i, m < F.
+
+    q~_i = bf16(q_i Wq), K~_m = bf16(Kbar_m Wk), s_im = q~_i . K~_m / sqrt(d_s).
+    Entries with m >= C_i are computed but never used by a row (causality).
+    Wq, Wk: [d, d_s].
+    """
+    d_s = Wq.shape[1]
+    qt = round_to_bf16(Q @ Wq)
+    kt = round_to_bf16(block_summaries(K, b) @ Wk)
+    return (qt @ kt.T) / math.sqrt(d_s)
+
+
+# --------------------------------------------------------------- a3 / a4 --
+
+def log_gates(s_hist):
+    """a3, Eq. normalized_log_gate: log g_m = s_m - LSE(s) over the row's history."""
+    s_hist = np.asarray(s_hist, dtype=np.float64)
+    if s_hist.size == 0:
+        return s_hist.copy()
+    mx = s_hist.max()
+    lse = mx + math.log(np.exp(s_hist - mx).sum())
+    return s_hist - lse
+
+
+def topk_blocks(s_hist, K):
+    """a4, Eq. selected_context: the K highest-scoring historical blocks.
+
+    Exact-K with ties to the lower block index; all blocks when C_i <= K.
+    Returned in ascending block order.
+    """
+    s_hist = np.asarray(s_hist)
+    C_i = s_hist.shape[0]
+    if C_i <= K:
+        return np.arange(C_i)
+    # A stable sort on the negated scores keeps equal scores in ascending
+    # block order, which is the tie rule.
+    order = np.argsort(-s_hist, kind="stable")
+    return np.sort(order[:K])
+
+
+# -------------------------------------------------------------------- a5 --
+
+def _row_keys_and_bias(i, s_row, b, topk, mode):
+    """Attended keys of row i and their additive bias (Eq. ours_train).
+
+    Returns (keys, bias, sel_idx, sel_logg) where keys lists token indices:
+    first the tokens of the selected historical blocks, then the causal part
+    of the current block.
+    """
+    c = historical_count(i, b)
+    s_hist = np.asarray(s_row[:c], dtype=np.float64)
+    lg = log_gates(s_hist)
+    sel = topk_blocks(s_hist, topk)
+    keys, bias = [], []
+    for m in sel:
+        toks = np.arange(m * b, (m + 1) * b)
+        keys.append(toks)
+        g = lg[m] if mode == MODE_TRAIN_SOFT else 0.0
+        bias.append(np.full(b, g))
+    cur = np.arange(c * b, i + 1)           # current block, causal, unit gate
+    keys.append(cur)
+    bias.append(np.zeros(cur.shape[0]))
+    return np.concatenate(keys), np.concatenate(bias), sel, lg[sel]
+
+
+def sas_attention_head(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                       rows=None):
+    """a5 for one head: O_i = softmax(z) V, z_j = sm_scale q_i.k_j + bias_j.
+
+    s: [N, >=C-1] selector scores of the head (row i reads s[i, :C_i]).
+    rows: iterable of query indices (default: all).
+    Returns dict with O [R, d], LSE [R], sel_idx [R, topk] (ascending, -1
+    padded) and sel_logg [R, topk] (log g of the selected blocks, 0 padded).
+    LSE is the natural-log log-sum-exp of the logits z (Alg. 3 output).
+    """
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    rows = np.arange(N) if rows is None else np.asarray(rows)
+    R = rows.shape[0]
+    O = np.zeros((R, V.shape[1]))
+    LSE = np.zeros(R)
+    sel_idx = np.full((R, topk), -1, dtype=np.int64)
+    sel_logg = np.zeros((R, topk))
+    for r, i in enumerate(rows):
+        keys, bias, sel, lg = _row_keys_and_bias(int(i), s[i], b, topk, mode)
+        z = sm_scale * (K[keys] @ Q[i]) + bias
+        zmax = z.max()
+        w = np.exp(z - zmax)
+        l = w.sum()
+        O[r] = (w @ V[keys]) / l
+        LSE[r] = zmax + math.log(l)
+        sel_idx[r, :sel.shape[0]] = sel
+        sel_logg[r, :sel.shape[0]] = lg
+    return {"O": O, "LSE": LSE, "sel_idx": sel_idx, "sel_logg": sel_logg}
+
+
+def sas_attention_materialized(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT,
+                               sm_scale=None):
+    """Brute force: the whole N x N gated logit matrix, then a row softmax.
+
+    This is the naive form the paper calls prohibitive (Sec. 4.3, Kernel
+    Design); it exists only to cross-check the per-row oracle on small N.
+    Bias[i, j] = 0 on the causal current block, log g (or 0 in inference
+    mode) on selected historical blocks, -inf elsewhere.
+    """
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    bias = np.full((N, N), -np.inf)
+    for i in range(N):
+        c = historical_count(i, b)
+        s_hist = np.asarray(s[i][:c], dtype=np.float64)
+        lg = log_gates(s_hist)
+        for m in topk_blocks(s_hist, topk):
+            bias[i, m * b:(m + 1) * b] = lg[m] if mode == MODE_TRAIN_SOFT else 0.0
+        bias[i, c * b:i + 1] = 0.0
+    Z = sm_scale * (Q @ K.T) + bias
+    zmax = Z.max(axis=1, keepdims=True)
+    W = np.exp(Z - zmax)
+    l = W.sum(axis=1, keepdims=True)
+    return {"O": (W @ V) / l, "LSE": (zmax + np.log(l))[:, 0], "P": W / l}
+
+
+def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                  scores=None, Wq=None, Wk=None, heads=None, rows=None):
+    """Alg. 1 steps 1-4 (training forward) over [B, H, N, d] inputs.
+
+    Either `scores` [B, H, N, >=C-1] are given (scores-given selector) or the
+    MEANPOOL_PROJ selector weights Wq, Wk [H, d, d_s] are.  heads: list of
+    (batch, head) pairs to evaluate (default all); rows as in
+    sas_attention_head.  Returns {(bi, hi): result-dict}.
+    """
+    Bn, H, N, d = Q.shape
+    heads = [(bi, hi) for bi in range(Bn) for hi in range(H)] if heads is None else heads
+    out = {}
+    for bi, hi in heads:
+        if scores is not None:
+            s = scores[bi, hi]
+        else:
+            s = selector_scores(Q[bi, hi], K[bi, hi], Wq[hi], Wk[hi], b)
+        out[(bi, hi)] = sas_attention_head(Q[bi, hi], K[bi, hi], V[bi, hi], s, b,
+                                           topk, mode, sm_scale, rows)
+    return out
+
+
+# -------------------------------------------------------------------- a6 --
+
+def gelu(x):
+    """Exact GELU: x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2))."""
+    x = np.asarray(x, dtype=np.float64)
+    erf = np.vectorize(math.erf, otypes=[np.float64])
+    return 0.5 * x * (1.0 + erf(x / math.sqrt(2.0)))
+
+
+def gelu_mlp(X, W1, W2, b1=None, b2=None, rows=None):
+    """a6 (dense MLP; SAS does not define one): Y = bf16(GELU(X W1^T + b1)) W2^T + b2.
+
+    X [T, D], W1 [F, D], W2 [D, F] (linear-layer weight layout [out, in]).
+    rows: optional subset of token rows.
+    """
+    Xr = X if rows is None else X[np.asarray(rows)]
+    Hh = Xr @ W1.T
+    if b1 is not None:
+        Hh = Hh + b1
+    G = round_to_bf16(gelu(Hh))
+    Y = G @ W2.T
+    if b2 is not None:
+        Y = Y + b2
+    return Y
+
+
+# ------------------------------------------------------------- accounting --
+
+def attention_flops_row(i, b, topk, d, d_sel=0):
+    """Algorithmic FLOPs of one query row: 4 d (|current| + b min(K, C_i)) + 2 d_s C_i."""
+    c = historical_count(i, b)
+    cur = i - c * b + 1
+    return 4 * d * (cur + b * min(topk, c)) + 2 * d_sel * c

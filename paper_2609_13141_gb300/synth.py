@@ -1,0 +1,83 @@
+"""Seeded synthetic inputs shaped like the SAS workloads.
+
+This module only draws random numbers: it holds none of the method's
+arithmetic, and both the CUDA path and the oracle take their inputs from it.
+Everything is drawn in float32 on the CPU with a seeded torch generator and
+then rounded to the storage dtype (bf16 for activations and weights, fp32 for
+scores), so that every consumer sees the same bits.
+
+Score regimes (the paper does not describe how coherent the selections of
+neighbouring queries are, so the benchmark names three):
+  R1  block-coherent scores: s[i, m] = u[floor(i / b), m] + 0.05 eps[i, m]
+  R2  block-correlated queries for the learned-selector path:
+      q_i = (mu[floor(i / b)] + 0.3 eps_i) / sqrt(1.09), marginally N(0, 1)
+  R3  independent scores: s ~ N(0, 1)
+"""
+from __future__ import annotations
+
+import math
+
+import torch
+
+
+def _gen(seed):
+    g = torch.Generator(device="cpu")
+    g.manual_seed(int(seed))
+    return g
+
+
+def normal(shape, seed, std=1.0):
+    """float32 N(0, std^2) tensor on the CPU."""
+    return torch.randn(*shape, generator=_gen(seed), dtype=torch.float32) * std
+
+
+def qkv(B, H, N, d, seed=0, regime="iid", block=64):
+    """Q, K, V as bf16 [B, H, N, d].  regime 'iid' or 'R2' (block-correlated Q)."""
+    K = normal((B, H, N, d), seed + 1).to(torch.bfloat16)
+    V = normal((B, H, N, d), seed + 2).to(torch.bfloat16)
+    if regime == "R2":
+        nb = -(-N // block)
+        mu = normal((B, H, nb, d), seed + 3)
+        eps = normal((B, H, N, d), seed + 4)
+        idx = torch.arange(N) // block
+        Q = (mu[:, :, idx, :] + 0.3 * eps) / math.sqrt(1.09)
+        Q = Q.to(torch.bfloat16)
+    else:
+        Q = normal((B, H, N, d), seed).to(torch.bfloat16)
+    return Q, K, V
+
+
+def scores(B, H, N, C, seed=0, regime="R1", block=64):
+    """Selector scores as fp32 [B, H, N, C].  regime 'R1' (block-coherent) or 'R3' (iid)."""
+    if regime == "R1":
+        nb = -(-N // block)
+        u = normal((B, H, nb, C), seed + 10)
+        eps = normal((B, H, N, C), seed + 11)
+        idx = torch.arange(N) // block
+        return (u[:, :, idx, :] + 0.05 * eps).contiguous()
+    return normal((B, H, N, C), seed + 12)
+
+
+def integer_scores(B, H, N, C, seed=0, levels=4):
+    """Small-integer fp32 scores: many exact ties, for the tie rule."""
+    g = _gen(seed + 20)
+    return torch.randint(0, levels, (B, H, N, C), generator=g).to(torch.float32)
+
+
+def selector_weights(H, d, d_sel, seed=0, std=0.02):
+    """Wq, Wk as bf16 [H, d, d_sel]."""
+    Wq = normal((H, d, d_sel), seed + 30, std).to(torch.bfloat16)
+    Wk = normal((H, d, d_sel), seed + 31, std).to(torch.bfloat16)
+    return Wq, Wk
+
+
+def mlp(T, D, F, seed=0, std=0.02, bias=False):
+    """X [T, D], W1 [F, D], W2 [D, F] (and b1 [F], b2 [D] if bias) as bf16."""
+    X = normal((T, D), seed + 40).to(torch.bfloat16)
+    W1 = normal((F, D), seed + 41, std).to(torch.bfloat16)
+    W2 = normal((D, F), seed + 42, std).to(torch.bfloat16)
+    if not bias:
+        return X, W1, W2, None, None
+    b1 = normal((F,), seed + 43, std).to(torch.bfloat16)
+    b2 = normal((D,), seed + 44, std).to(torch.bfloat16)
+    return X, W1, W2, b1, b2

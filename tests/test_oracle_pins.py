@@ -1,0 +1,264 @@
+"""Pins for the CPU oracle: each test checks the oracle against something
+other than itself -- hand-derived closed forms (tests/golden), library
+routines that implement a special case independently (torch SDPA, torch's
+bf16 conversion, torch GELU, scipy logsumexp), invariants the paper states,
+and brute force on tiny inputs.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+import torch.nn.functional as F
+
+from oracle import sas_oracle as O
+from paper_2609_13141_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "sas_worked_examples.json")
+
+
+def f64(t):
+    return t.to(torch.float64).numpy()
+
+
+# ------------------------------------------------------------- bf16 rounding
+
+def test_round_to_bf16_matches_torch_conversion():
+    # float32 inputs have one rounding to bf16 in torch; the oracle rounds the
+    # exact float64 value of the same float32 number, so both must agree bit for bit.
+    x = synth.normal((20000,), seed=5, std=3.0)
+    x = torch.cat([x, x * 1e-30, x * 1e30, torch.tensor([0.0, -0.0, 1.0, -2.5])])
+    # exact ties between two bf16 neighbours: 1 + 2^-8 (tie, even -> 1), 1 + 3*2^-8 (tie -> up)
+    x = torch.cat([x, torch.tensor([1 + 2.0**-8, 1 + 3 * 2.0**-8, -(1 + 2.0**-8), 2.0**-130 * 1.5])])
+    ref = x.to(torch.bfloat16).to(torch.float64).numpy()
+    got = O.round_to_bf16(x.to(torch.float64).numpy())
+    assert np.array_equal(ref, got)
+
+
+# ---------------------------------------------------------- a1 block summary
+
+def test_block_summaries_closed_form_ramp_and_partial_block():
+    b, N, d = 8, 8 * 5 + 3, 3
+    j = np.arange(N, dtype=np.float64)
+    K = np.stack([j, 2 * j, np.ones(N)], axis=1)
+    Kbar = O.block_summaries(K, b)
+    assert Kbar.shape == (5, d)            # the 3-token tail block is not summarised
+    m = np.arange(5)
+    mean_j = m * b + (b - 1) / 2.0         # mean of an arithmetic run
+    assert np.allclose(Kbar[:, 0], mean_j)
+    assert np.allclose(Kbar[:, 1], 2 * mean_j)
+    assert np.allclose(Kbar[:, 2], 1.0)
+
+
+def test_selector_worked_example():
+    g = json.load(open(GOLDEN))["selector_example"]
+    K = np.array(g["K"], float)
+    Q = np.array(g["Q"], float)
+    I2 = np.eye(2)
+    assert np.allclose(O.block_summaries(K, g["b"]), g["expect_Kbar"])
+    s = O.selector_scores(Q, K, I2, I2, g["b"])
+    assert np.allclose(s[3], g["expect_s_row3"], rtol=0, atol=1e-15)
+
+
+def test_selector_scores_scaling_and_permutation():
+    # doubling Wq (exact in bf16) doubles every score; permuting key blocks
+    # permutes the score columns.
+    rng = np.random.default_rng(0)
+    b, N, d, ds = 4, 32, 8, 6
+    Q = O.round_to_bf16(rng.standard_normal((N, d)))
+    K = O.round_to_bf16(rng.standard_normal((N, d)))
+    Wq = O.round_to_bf16(rng.standard_normal((d, ds)) * 0.3)
+    Wk = O.round_to_bf16(rng.standard_normal((d, ds)) * 0.3)
+    s = O.selector_scores(Q, K, Wq, Wk, b)
+    assert np.allclose(O.selector_scores(Q, K, 2 * Wq, Wk, b), 2 * s, rtol=1e-12, atol=0)
+    perm = rng.permutation(N // b)
+    Kp = K.reshape(N // b, b, d)[perm].reshape(N, d)
+    assert np.allclose(O.selector_scores(Q, Kp, Wq, Wk, b), s[:, perm], rtol=1e-12, atol=1e-15)
+
+
+# ------------------------------------------------------------------ a3 gates
+
+def test_log_gates_normalised_shift_invariant_and_single_block():
+    rng = np.random.default_rng(1)
+    for C in [1, 2, 7, 100]:
+        s = rng.standard_normal(C) * 3
+        lg = O.log_gates(s)
+        assert math.isclose(np.exp(lg).sum(), 1.0, rel_tol=1e-12)      # softmax gates sum to 1
+        assert np.allclose(O.log_gates(s + 17.25), lg, atol=1e-12)      # Eq. normalized_log_gate shift invariance
+        assert np.allclose(lg, s - scipy.special.logsumexp(s), atol=1e-12)
+    assert O.log_gates(np.array([4.2]))[0] == 0.0                      # one block: g = 1
+    lg = O.log_gates(np.array([0.0, math.log(3.0)]))
+    assert np.allclose(lg, [math.log(0.25), math.log(0.75)], atol=1e-15)
+
+
+# ------------------------------------------------------------------ a4 top-K
+
+def test_topk_brute_force_with_ties():
+    rng = np.random.default_rng(2)
+    for _ in range(300):
+        C = int(rng.integers(0, 40))
+        K = int(rng.integers(0, 12))
+        s = rng.integers(0, 4, size=C).astype(np.float64)       # many exact ties
+        got = list(O.topk_blocks(s, K))
+        ranked = sorted(range(C), key=lambda m: (-s[m], m))       # score desc, index asc
+        assert got == sorted(ranked[:K])
+
+
+def test_topk_all_when_history_short_and_none_when_k0():
+    s = np.array([0.3, -1.0, 2.0])
+    assert list(O.topk_blocks(s, 3)) == [0, 1, 2]
+    assert list(O.topk_blocks(s, 10)) == [0, 1, 2]
+    assert list(O.topk_blocks(s, 0)) == []
+    assert list(O.topk_blocks(s, 1)) == [2]
+
+
+# ------------------------------------------------------------ a5 attention
+
+@pytest.mark.parametrize("case", json.load(open(GOLDEN))["cases"], ids=lambda c: c["name"])
+def test_attention_worked_examples(case):
+    Q = np.array(case["Q"], float)
+    K = np.array(case["K"], float)
+    V = np.array(case["V"], float)
+    N = Q.shape[0]
+    s = np.zeros((N, N))
+    s[case["row"], :len(case["scores_row"])] = case["scores_row"]
+    mode = O.MODE_TRAIN_SOFT if case["mode"] == "train" else O.MODE_INFER_HARD
+    r = O.sas_attention_head(Q, K, V, s, case["b"], case["topk"], mode,
+                             case["sm_scale"], rows=[case["row"]])
+    nsel = len(case["expect_sel_idx"])
+    assert list(r["sel_idx"][0, :nsel]) == case["expect_sel_idx"]
+    assert np.all(r["sel_idx"][0, nsel:] == -1)
+    assert np.allclose(r["sel_logg"][0, :nsel], case["expect_sel_logg"], atol=1e-14)
+    assert np.allclose(r["O"][0], case["expect_O"], atol=1e-14)
+    assert math.isclose(r["LSE"][0], case["expect_LSE"], abs_tol=1e-14)
+
+
+def _rand_head(N, d, seed):
+    rng = np.random.default_rng(seed)
+    q = O.round_to_bf16(rng.standard_normal((N, d)))
+    k = O.round_to_bf16(rng.standard_normal((N, d)))
+    v = O.round_to_bf16(rng.standard_normal((N, d)))
+    return q, k, v, rng
+
+
+def _sdpa(q, k, v, mask, scale):
+    t = lambda a: torch.from_numpy(a)[None, None]
+    return F.scaled_dot_product_attention(t(q), t(k), t(v), attn_mask=t(mask), scale=scale)[0, 0].numpy()
+
+
+@pytest.mark.parametrize("N,b", [(37, 8), (64, 16), (5, 8)])
+def test_infer_keep_all_equals_dense_causal_sdpa(N, b):
+    q, k, v, rng = _rand_head(N, 16, 3)
+    s = rng.standard_normal((N, N))
+    C = O.num_blocks(N, b)
+    r = O.sas_attention_head(q, k, v, s, b, topk=C, mode=O.MODE_INFER_HARD)
+    causal = np.where(np.tril(np.ones((N, N))) > 0, 0.0, -np.inf)
+    ref = _sdpa(q, k, v, causal, 1 / 4.0)
+    assert np.allclose(r["O"], ref, atol=1e-12)
+
+
+def test_train_constant_scores_equals_biased_dense_sdpa():
+    # s = const gives log g_m = -log C_i for every historical block: dense causal
+    # attention with a -log C_i bias on keys before the current block.
+    N, b, d = 50, 8, 16
+    q, k, v, _ = _rand_head(N, d, 4)
+    s = np.full((N, N), 0.7)
+    r = O.sas_attention_head(q, k, v, s, b, topk=64, mode=O.MODE_TRAIN_SOFT)
+    mask = np.full((N, N), -np.inf)
+    for i in range(N):
+        c = i // b
+        if c > 0:
+            mask[i, :c * b] = -math.log(c)
+        mask[i, c * b:i + 1] = 0.0
+    ref = _sdpa(q, k, v, mask, 1 / 4.0)
+    assert np.allclose(r["O"], ref, atol=1e-12)
+    lse_ref = scipy.special.logsumexp(q @ k.T / 4.0 + mask, axis=1)
+    assert np.allclose(r["LSE"], lse_ref, atol=1e-12)
+
+
+def test_k0_equals_block_local_causal_sdpa():
+    N, b, d = 45, 8, 16
+    q, k, v, rng = _rand_head(N, d, 5)
+    s = rng.standard_normal((N, N))
+    r = O.sas_attention_head(q, k, v, s, b, topk=0, mode=O.MODE_TRAIN_SOFT)
+    blk = np.arange(N) // b
+    ok = (blk[:, None] == blk[None, :]) & (np.arange(N)[None, :] <= np.arange(N)[:, None])
+    ref = _sdpa(q, k, v, np.where(ok, 0.0, -np.inf), 1 / 4.0)
+    assert np.allclose(r["O"], ref, atol=1e-12)
+    assert np.all(r["sel_idx"].shape == (N, 0))
+
+
+@pytest.mark.parametrize("mode", [O.MODE_TRAIN_SOFT, O.MODE_INFER_HARD])
+@pytest.mark.parametrize("N,b,K,ties", [(70, 8, 3, False), (64, 16, 2, True), (19, 4, 1, True), (9, 8, 2, False)])
+def test_streaming_rows_equal_materialised_matrix(mode, N, b, K, ties):
+    q, k, v, rng = _rand_head(N, 8, 6 + N)
+    s = rng.integers(0, 3, (N, N)).astype(float) if ties else rng.standard_normal((N, N))
+    r = O.sas_attention_head(q, k, v, s, b, K, mode)
+    m = O.sas_attention_materialized(q, k, v, s, b, K, mode)
+    assert np.allclose(r["O"], m["O"], atol=1e-12)
+    assert np.allclose(r["LSE"], m["LSE"], atol=1e-12)
+    P = m["P"]
+    assert np.allclose(P.sum(axis=1), 1.0)                  # rows sum to 1
+    assert P.max() <= 1.0 + 1e-15                           # soft weights bounded (Eq. rank_unbounded)
+    assert np.all(P[np.triu_indices(N, 1)] == 0)            # causal
+
+
+def test_attention_shift_invariant_in_scores():
+    # Eq. normalized_log_gate: s -> s + c per row leaves gates, selection and output unchanged.
+    N, b = 60, 8
+    q, k, v, rng = _rand_head(N, 8, 9)
+    s = rng.standard_normal((N, N))
+    shift = rng.standard_normal((N, 1)) * 10
+    r1 = O.sas_attention_head(q, k, v, s, b, 2)
+    r2 = O.sas_attention_head(q, k, v, s + shift, b, 2)
+    assert np.array_equal(r1["sel_idx"], r2["sel_idx"])
+    assert np.allclose(r1["O"], r2["O"], atol=1e-12)
+
+
+def test_selected_blocks_change_output_only_through_selected_set():
+    # A row's output must not depend on keys/values of blocks it did not select.
+    N, b = 48, 8
+    q, k, v, rng = _rand_head(N, 8, 10)
+    s = rng.standard_normal((N, N))
+    i = 47
+    r = O.sas_attention_head(q, k, v, s, b, 2, rows=[i])
+    sel = set(r["sel_idx"][0])
+    k2, v2 = k.copy(), v.copy()
+    for m in range(i // b):
+        if m not in sel:
+            k2[m * b:(m + 1) * b] += 5
+            v2[m * b:(m + 1) * b] -= 3
+    r2 = O.sas_attention_head(q, k2, v2, s, b, 2, rows=[i])
+    assert np.allclose(r["O"], r2["O"], atol=1e-14)
+
+
+# ---------------------------------------------------------------------- a6
+
+def test_gelu_matches_torch_exact_gelu():
+    x = np.linspace(-8, 8, 2001)
+    ref = F.gelu(torch.from_numpy(x), approximate="none").numpy()
+    assert np.allclose(O.gelu(x), ref, atol=1e-15)
+    assert O.gelu(np.array([0.0]))[0] == 0.0
+    assert math.isclose(O.gelu(np.array([30.0]))[0], 30.0)
+
+
+def test_gelu_mlp_matches_torch_linear_pipeline():
+    X, W1, W2, b1, b2 = synth.mlp(33, 24, 40, seed=3, std=0.2, bias=True)
+    Y = O.gelu_mlp(f64(X), f64(W1), f64(W2), f64(b1), f64(b2))
+    h = F.linear(X.double(), W1.double(), b1.double())
+    g = F.gelu(h, approximate="none").float().to(torch.bfloat16).double()
+    ref = F.linear(g, W2.double(), b2.double()).numpy()
+    # the two routes may round a hidden value to different bf16 neighbours
+    # (torch rounds via float32): allow a couple of such flips, no more
+    assert np.abs(Y - ref).max() < 2e-3
+    rows = [0, 5, 32]
+    assert np.allclose(O.gelu_mlp(f64(X), f64(W1), f64(W2), f64(b1), f64(b2), rows=rows), Y[rows])
+
+
+def test_flops_accounting_row():
+    # row 130 with b = 64: C_i = 2, current block holds 3 keys (128..130)
+    assert O.attention_flops_row(130, 64, 32, 128, 128) == 4 * 128 * (3 + 64 * 2) + 2 * 128 * 2
+    assert O.attention_flops_row(64 * 40, 64, 32, 128, 0) == 4 * 128 * (1 + 64 * 32)
