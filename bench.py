@@ -1,0 +1,410 @@
+"""Benchmark: one SAS transformer layer on GB300 through the C ABI.
+
+A step is one pass of the whole hot path over one batch of synthetic input:
+the SAS attention forward (block summaries, query projection, selector scores,
+log-gates, Top-K, gated block-sparse attention) followed by the dense GELU MLP
+on the same tokens.  Workload (the DiT-scale layer): B=2, H=24, N=4096+512,
+d=128, b=64, K=32, learned selector with d_sel=128, MLP 9216 x 3072 -> 12288
+-> 3072.  Inputs are seeded synthetic data resident in HBM; L2 is flushed
+(256 MiB write) between timed steps, outside the timed events.
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ms/layer and effective TFLOP/s on 1xGB300; % of bf16 tensor-core roofline"
+UNIT = "TFLOP/s"
+
+WORKLOADS = {
+    "dit": dict(B=2, H=24, N=4096 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
+                name="DiT-scale causal SAS layer: B=2 H=24 N=4096+512 d=128 b=64 K=32, learned selector d_sel=128, "
+                     "GELU MLP 9216x3072->12288->3072"),
+    "tiny": dict(B=1, H=4, N=256, d=64, topk=32, d_sel=64, D=256, F=1024,
+                 name="tiny SAS layer: B=1 H=4 N=256 d=64 K=32, MLP 256->1024->256"),
+    "hires": dict(B=1, H=24, N=16384 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
+                  name="high-resolution causal SAS layer: B=1 H=24 N=16384+512 d=128 K=32, MLP 16896x3072->12288->3072"),
+    "video": dict(B=1, H=24, N=75600 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
+                  name="video-scale causal SAS layer: B=1 H=24 N=75600+512 d=128 K=32, MLP 76112x3072->12288->3072"),
+}
+
+
+def algorithmic_flops(w):
+    """Work the method itself must do for one layer (no tile-union or padding waste).
+
+    Attention per (batch, head) row i with c = floor(i/64):
+      4 d (|current-block keys| + 64 min(K, c))    QK^T and PV over the kept keys
+      2 d_sel c                                    selector scores against c summaries
+      2 d d_sel                                    query projection
+    plus 2 d d_sel per full key block (key projection), and the MLP 4 T D F.
+    """
+    N, d, K, ds = w["N"], w["d"], w["topk"], w["d_sel"]
+    BH = w["B"] * w["H"]
+    attn = sel = 0
+    for c in range((N + 63) // 64):
+        rows = min(64, N - 64 * c)
+        cur = rows * (rows + 1) // 2            # sum over rows of (i - 64c + 1)
+        attn += 4 * d * (cur + rows * 64 * min(K, c))
+        sel += rows * (2 * ds * c + 2 * d * ds)
+    sel += (N // 64) * 2 * d * ds
+    mlp = 4 * w["B"] * N * w["D"] * w["F"]
+    return {"attention": BH * attn, "selector": BH * sel, "mlp": mlp,
+            "total": BH * (attn + sel) + mlp}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"bf16": d.get("bf16_tflops"), "bf16_sustained": d.get("bf16_tflops_sustained"),
+                "hbm": d.get("hbm_gbs"), "source": "measured"}
+    return {"bf16": 1900.0, "bf16_sustained": 1700.0, "hbm": 6800.0, "source": "fallback"}
+
+
+# ----------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "utilization.gpu", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) == len(self.FIELDS):
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons = [], 0.0, set()
+        for r in self.rows:
+            try:
+                clk, cmax, util = float(r[0]), float(r[1]), float(r[2])
+            except ValueError:
+                continue
+            mx = max(mx, cmax)
+            if util > 0:
+                sm.append(clk)
+            for k, name in enumerate(names):
+                if r[3 + k].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx or None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------- our arm
+
+def kernel_traffic(kind):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    if not os.path.exists(p):
+        return None
+    rec = json.load(open(p)).get(kind)
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2609_13141_gb300", "csrc", rec["source"])
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return rec["dram_bytes_per_launch"] if sha == rec["source_sha256_16"] else None
+
+
+def run_ours(args, w, rank, world):
+    import torch
+
+    from paper_2609_13141_gb300 import sas, synth
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
+    T = B * N
+    Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
+    Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
+    X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
+    Qd, Kd, Vd, Wqd, Wkd = (t.to(dev) for t in (Q, Kk, V, Wq, Wk))
+    Xd, W1d, W2d = X.to(dev), W1.to(dev), W2.to(dev)
+    Od = torch.empty_like(Qd)
+    LSEd = torch.empty(B, H, N, device=dev, dtype=torch.float32)
+    Yd = torch.empty(T, D, device=dev, dtype=torch.bfloat16)
+    flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
+
+    layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
+    h = layer.h
+    stream = torch.cuda.current_stream(dev)
+
+    def step(Qx, Kx, Vx, Xx, O, Y):
+        sas.sas_attention_fwd(h, Qx, Kx, Vx, O, None, Wqd, Wkd, LSEd, None, None, stream)
+        sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step(Qd, Kd, Vd, Xd, Od, Yd)
+    torch.cuda.synchronize()
+    # keep the GPU busy for ~1 s so the clock sampler sees it under load
+    t_end = time.time() + 1.0
+    while time.time() < t_end:
+        step(Qd, Kd, Vd, Xd, Od, Yd)
+        torch.cuda.synchronize()
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.2)
+    sas.sas_set_timing(h, True)
+    launches0 = sas.sas_launch_count(h)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for k in range(args.steps):
+        flush.zero_()
+        starts[k].record(stream)
+        step(Qd, Kd, Vd, Xd, Od, Yd)
+        ends[k].record(stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    launches = sas.sas_launch_count(h) - launches0
+    kt = sas.sas_get_timings(h)
+    sas.sas_set_timing(h, False)
+    clocks = sampler.stop()
+    ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    assert sas.sas_get_device_status(h) == 0, "device status word reports a timed-out wait"
+
+    # end to end: pinned host inputs -> device -> layer -> host outputs, every step
+    hQ, hK, hV, hX = (t.pin_memory() for t in (Q, Kk, V, X))
+    hO = torch.empty(Q.shape, dtype=torch.bfloat16).pin_memory()
+    hY = torch.empty(T, D, dtype=torch.bfloat16).pin_memory()
+    dQ, dK, dV, dX = (torch.empty_like(t) for t in (Qd, Kd, Vd, Xd))
+    e_st = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e_en = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    for k in range(-2, args.steps):
+        flush.zero_()
+        if k >= 0:
+            e_st[k].record(stream)
+        for dst, src in ((dQ, hQ), (dK, hK), (dV, hV), (dX, hX)):
+            dst.copy_(src, non_blocking=True)
+        step(dQ, dK, dV, dX, Od, Yd)
+        hO.copy_(Od, non_blocking=True)
+        hY.copy_(Yd, non_blocking=True)
+        if k >= 0:
+            e_en[k].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = sum(s.elapsed_time(e) for s, e in zip(e_st, e_en)) / args.steps
+    h2d = sum(t.numel() * t.element_size() for t in (hQ, hK, hV, hX))
+    d2h = hO.numel() * 2 + hY.numel() * 2
+
+    # tile-union statistics of the last forward (executed vs algorithmic work)
+    Tt = (N + 127) // 128
+    unions = sas.sas_get_tile_union_counts(h, B * H * Tt)
+    layer.close()
+
+    if dist is not None:
+        t = torch.tensor([ms, e2e_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = float(t[0]), float(t[1])
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return None
+
+    fl = algorithmic_flops(w)
+    tflop = fl["total"] / 1e12
+    value = tflop * world / (ms / 1e3)
+    per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None)} for k, (n, t) in kt.items()}
+    flops_per_launch = {"attention": fl["attention"], "mlp_up_gelu": fl["mlp"] / 2, "mlp_down": fl["mlp"] / 2}
+    dom = max((k for k in kt if kt[k][0] > 0), key=lambda k: kt[k][1])
+    peaks = load_peaks()
+    roof = None
+    if dom in flops_per_launch:
+        avg = kt[dom][1] / kt[dom][0]
+        achieved = flops_per_launch[dom] / (avg / 1e3) / 1e12
+        roof = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1), "peak": peaks["bf16"],
+                "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16"], 4), "traffic": kernel_traffic(dom),
+                "peak_source": f"{peaks['source']} bf16 dense burst"}
+    # attention-kernel view (the SAS kernel proper)
+    a_avg = kt["attention"][1] / max(kt["attention"][0], 1)
+    hist_blocks = sum(unions) / max(len(unions), 1)
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; R2 block-correlated queries, N(0,1) K/V/X, "
+        "weights N(0,0.02))",
+        "config": {"workload": w["name"], "B": B, "H": H, "N": N, "d": d, "block": 64, "topk": K, "d_sel": ds,
+                   "mlp": [T, D, F, D], "selector": "meanpool_proj", "l2": "flushed between timed steps (256 MiB write)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roof,
+        "attention_kernel": {"ms": round(a_avg, 4), "algorithmic_tflops": round(fl["attention"] / (a_avg / 1e3) / 1e12, 1),
+                             "frac_of_bf16_peak": round(fl["attention"] / (a_avg / 1e3) / 1e12 / peaks["bf16"], 4),
+                             "mean_union_blocks_per_tile": round(hist_blocks, 2)},
+        "kernels": per_kind,
+        "algorithmic_tflop_per_step": round(tflop, 4),
+        "e2e": {"value": round(tflop * world / (e2e_ms / 1e3), 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    if dist is not None:
+        dist.destroy_process_group()
+    return out
+
+
+# ----------------------------------------------------------- CPU oracle
+
+def _oracle_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 1) for i in threadpool_info()]
+        return max(n) if n else 1
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_sample(w, budget_s, seed=0):
+    """Runs the oracle on a bounded sample of the workload and returns its
+    throughput on the workload's FLOP mix.
+
+    Half the budget goes to query rows of one head (selector scores for the
+    whole head, then the gated attention of random rows), half to random MLP
+    token rows.  Each part's rate (algorithmic FLOPs per second) is measured
+    on its own; the full layer's time is attention FLOPs / attention rate +
+    MLP FLOPs / MLP rate.  Returns (rate_flops_per_s, seconds, desc)."""
+    import numpy as np
+    import torch
+
+    from oracle import sas_oracle as OR
+    from paper_2609_13141_gb300 import synth
+
+    B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
+    Q, Kk, V = synth.qkv(1, 1, N, d, seed=seed, regime="R2")
+    Wq, Wk = synth.selector_weights(1, d, ds, seed=seed)
+    X, W1, W2, _, _ = synth.mlp(256, D, F, seed=seed)
+    f = lambda t: t.to(torch.float64).numpy()
+    q, k, v, wq, wk = f(Q[0, 0]), f(Kk[0, 0]), f(V[0, 0]), f(Wq[0]), f(Wk[0])
+    x, w1, w2 = f(X), f(W1), f(W2)
+    rng = np.random.default_rng(seed)
+
+    t0 = time.perf_counter()
+    s = OR.selector_scores(q, k, wq, wk, 64)
+    a_flops = N * 2 * d * ds + (N // 64) * 2 * d * ds
+    rows_done = 0
+    while time.perf_counter() - t0 < budget_s / 2:
+        rows = rng.integers(0, N, size=32)
+        OR.sas_attention_head(q, k, v, s, 64, K, rows=rows)
+        a_flops += sum(OR.attention_flops_row(int(i), 64, K, d, ds) for i in rows)
+        rows_done += len(rows)
+    a_time = time.perf_counter() - t0
+    # the whole head's selector is amortised over the rows actually run
+    a_rate = a_flops / a_time
+
+    t1 = time.perf_counter()
+    m_flops = 0
+    tok_done = 0
+    while time.perf_counter() - t1 < budget_s / 2:
+        toks = rng.integers(0, 256, size=2)
+        OR.gelu_mlp(x, w1, w2, rows=toks)
+        m_flops += 4 * len(toks) * D * F
+        tok_done += len(toks)
+    m_time = time.perf_counter() - t1
+    m_rate = m_flops / m_time
+
+    fl = algorithmic_flops(w)
+    full_time = (fl["attention"] + fl["selector"]) / a_rate + fl["mlp"] / m_rate
+    rate = fl["total"] / full_time
+    desc = (f"oracle (numpy fp64): {rows_done} random query rows of one head (with that head's selector) "
+            f"in {a_time:.1f} s and {tok_done} MLP token rows in {m_time:.1f} s; the two measured rates are "
+            f"combined by the layer's FLOP mix")
+    return rate, a_time + m_time, desc
+
+
+def cpu_baseline(w, budget_s=12.0):
+    rate, dt, desc = oracle_sample(w, budget_s)
+    return {"value": round(rate / 1e12, 8), "unit": UNIT, "cores": _oracle_threads(), "kind": "oracle",
+            "sample": desc, "seconds": round(dt, 2)}
+
+
+def run_reference(args, w, rank, world):
+    if rank != 0:
+        return None
+    rates = []
+    desc = ""
+    for k in range(args.warmup + args.steps):
+        rate, dt, desc = oracle_sample(w, budget_s=args.ref_step_s, seed=k)
+        if k >= args.warmup:
+            rates.append(rate)
+    # harmonic mean: total FLOPs over total time for equal-work steps
+    value = len(rates) / sum(1.0 / r for r in rates) / 1e12
+    full = algorithmic_flops(w)["total"]
+    ms = full / (value * 1e12) * 1e3
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 8), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+        "config": {"workload": w["name"], "B": w["B"], "H": w["H"], "N": w["N"], "d": w["d"], "topk": w["topk"]},
+        "cpu_baseline": {"value": round(value, 8), "unit": UNIT, "cores": _oracle_threads(), "kind": "oracle",
+                         "sample": desc + f"; each step a {args.ref_step_s:.0f}-second sample"},
+        "e2e": {"value": round(value, 8), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dit")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--ref-step-s", type=float, default=4.0)
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    w = WORKLOADS[args.workload]
+    out = run_reference(args, w, rank, world) if args.impl == "reference" else run_ours(args, w, rank, world)
+    if out is not None and rank == 0:
+        print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()

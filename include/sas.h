@@ -1,0 +1,170 @@
+/*
+ * sas.h -- C ABI of the GB300 (sm_103a) SAS attention forward library.
+ *
+ * SAS ("Simple Attention Sparsification", arXiv 2609.13141) is trainable
+ * block-sparse attention for causal language models.  Keys and values are cut
+ * into blocks of b = 64 tokens.  A selector scores the historical blocks of
+ * every query, the scores become gates g = softmax(s) (Sec. 4.3), the Top-K
+ * blocks are kept (Eq. selected_context) and attention runs over the query's
+ * own block B_0 (causal, unit gate) plus the kept blocks, with log g added
+ * to the logits of the kept blocks (Eq. ours_train; Alg. 1 step 4).  The
+ * inference form (Alg. 2) drops the log g bias.
+ *
+ * Conventions shared by every entry point:
+ *   - All tensor arguments are DEVICE pointers owned by the caller.  The
+ *     library never frees them and keeps no reference after the call.
+ *   - bf16 tensors are passed as void* and hold IEEE bfloat16 values.
+ *   - Layouts are dense row-major with the shapes given; Q, K, V, O are
+ *     [B, H, N, d] ("BHND").  Base pointers must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *     asynchronous on that stream; the library synchronises only inside
+ *     sas_create / sas_destroy / sas_mlp_fwd's first use of a larger size /
+ *     the sas_get_* readers.
+ *   - Arguments are checked before anything is launched; on an argument error
+ *     nothing is written and the call returns SAS_ERR_INVALID_ARG or
+ *     SAS_ERR_UNSUPPORTED.  sas_last_error(h) then describes the problem.
+ *   - Every wait inside a kernel is bounded.  A wait that runs out sets a
+ *     device status word (read with sas_get_device_status) and the kernel
+ *     returns early; nothing traps.
+ *   - There is no CPU fallback: without a usable sm_103a device, calls return
+ *     SAS_ERR_CUDA.
+ */
+#ifndef SAS_H
+#define SAS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SAS_OK = 0,
+    SAS_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size, bad enum   */
+    SAS_ERR_UNSUPPORTED = 2,   /* valid but outside what the kernels implement  */
+    SAS_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed             */
+    SAS_ERR_TIMEOUT = 4,       /* a bounded in-kernel wait ran out              */
+    SAS_ERR_OOM = 5            /* workspace allocation failed                   */
+} sas_status;
+
+/* Gate form of the historical blocks.
+ *   TRAIN_SOFT : Eq. ours_train, logits of a kept block get + log g_m.
+ *   INFER_HARD : Alg. 2, kept blocks enter unbiased (the forward of the hard
+ *                Top-K gate, Sec. 4.2 "ranking preservation"). */
+typedef enum { SAS_MODE_TRAIN_SOFT = 0, SAS_MODE_INFER_HARD = 1 } sas_mode;
+
+/* Where the selector scores s come from (Alg. 1 step 1).
+ *   SCORES_GIVEN  : the caller passes s as a [B, H, N, C] fp32 table.
+ *   MEANPOOL_PROJ : s_im = bf16(Wq q_i) . bf16(Wk mean(K_Bm)) / sqrt(d_sel),
+ *                   a mean-pooled block-summary selector (the paper relies on
+ *                   pooled block summaries, App. B, and a gate-query projection
+ *                   dotted against them, Sec. 6.3; its exact AttnGate is not
+ *                   described, this is the library's reading). */
+typedef enum { SAS_SEL_SCORES_GIVEN = 0, SAS_SEL_MEANPOOL_PROJ = 1 } sas_selector;
+
+typedef struct {
+    int32_t B, H, N, d;   /* batch, heads, tokens, head dim (d in {64, 128})          */
+    int32_t block;        /* block size b; must be 64 (Sec. 4.2.1 setup)             */
+    int32_t topk;         /* K historical blocks kept per query, 0 <= K <= 1024       */
+    float sm_scale;       /* softmax scale on q.k; 0 selects 1/sqrt(d) (Alg. 3)       */
+    int32_t mode;         /* sas_mode                                                 */
+    int32_t selector;     /* sas_selector                                             */
+    int32_t d_sel;        /* selector dim d_sel in {64, 128}; 0 selects d             */
+} sas_config;
+
+typedef struct sas_handle sas_handle;
+
+/* Validates cfg, allocates the handle's device workspace (block summaries,
+ * projected queries, per-tile block lists, internal selection buffers) on the
+ * current device and returns the handle in *out.  Synchronous. */
+sas_status sas_create(const sas_config* cfg, sas_handle** out);
+
+/* Frees the workspace.  Waits for the device first.  NULL is a no-op. */
+void sas_destroy(sas_handle* h);
+
+/* SAS training-mode forward of one attention layer: Alg. 1 steps 1-4
+ * (selector scores, gates g = softmax(s), Top-K, gated sparse attention),
+ * with the fused-kernel structure of Alg. 3 (skip blocks no query in a tile
+ * keeps, online softmax, O and LSE outputs).
+ *
+ *   Q, K, V   bf16 [B, H, N, d]                                       (in)
+ *   scores    fp32 [B, H, N, C], C = ceil(N / 64); row i reads entries
+ *             0 .. floor(i/64)-1 and ignores the rest.  Required for
+ *             SCORES_GIVEN, must be NULL for MEANPOOL_PROJ.  Scores must
+ *             be finite.                                              (in)
+ *   Wq, Wk    bf16 [H, d_sel, d] selector projections (linear-layer
+ *             layout [out, in]); required for MEANPOOL_PROJ, NULL
+ *             otherwise.                                              (in)
+ *   O         bf16 [B, H, N, d]                                       (out)
+ *   LSE       fp32 [B, H, N] natural-log log-sum-exp of each row's
+ *             gated logits (Alg. 3 output); may be NULL.              (out)
+ *   sel_idx   int32 [B, H, N, topk]: each row's kept historical blocks in
+ *             ascending order, padded with -1; may be NULL.           (out)
+ *   sel_logg  fp32 [B, H, N, topk]: log g of the kept blocks (same order,
+ *             0 where padded); may be NULL.                           (out)
+ *
+ * Top-K is exact-K: ties go to the lower block index; rows with at most K
+ * historical blocks keep all of them. */
+sas_status sas_attention_fwd(sas_handle* h,
+                             const void* Q, const void* K, const void* V,
+                             const float* scores,
+                             const void* Wq, const void* Wk,
+                             void* O, float* LSE,
+                             int32_t* sel_idx, float* sel_logg,
+                             void* stream);
+
+/* Dense MLP sublayer Y = GELU(X W1^T + b1) W2^T + b2 with the exact (erf)
+ * GELU.  SAS itself does not define or change the MLP; this is the plain
+ * transformer MLP that completes a layer.
+ *   X  bf16 [T, D]; W1 bf16 [F, D]; b1 bf16 [F] or NULL;
+ *   W2 bf16 [D, F]; b2 bf16 [D] or NULL; Y bf16 [T, D].
+ * D and F must be multiples of 64; T >= 1.  The hidden activation
+ * GELU(X W1^T + b1) is kept as a bf16 [T, F] tensor in handle-owned
+ * memory, allocated (synchronously) the first time a call needs more. */
+sas_status sas_mlp_fwd(sas_handle* h,
+                       const void* X, const void* W1, const void* b1,
+                       const void* W2, const void* b2, void* Y,
+                       int64_t T, int64_t D, int64_t F,
+                       void* stream);
+
+/* Static text for a status code. */
+const char* sas_status_str(sas_status s);
+
+/* Text of the last error recorded on this handle ("" if none). */
+const char* sas_last_error(const sas_handle* h);
+
+/* Reads and clears the device status word (SAS_OK or SAS_ERR_TIMEOUT).
+ * Synchronises the device first. */
+sas_status sas_get_device_status(sas_handle* h, int32_t* out_status);
+
+/* Per-kernel timing with CUDA events recorded on the launch stream around
+ * every kernel.  sas_set_timing(h, 1) starts recording (and clears earlier
+ * records); sas_get_timings synchronises, then writes, for each kernel kind,
+ * the number of launches and the summed milliseconds.  Kinds, in order:
+ * 0 block summaries, 1 query projection, 2 selection, 3 attention,
+ * 4 MLP up-projection + GELU, 5 MLP down-projection.  n_kinds <= 6. */
+#define SAS_NUM_KERNEL_KINDS 6
+sas_status sas_set_timing(sas_handle* h, int32_t enable);
+sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds);
+
+/* Total number of kernels this handle has launched since creation. */
+int64_t sas_launch_count(const sas_handle* h);
+
+/* Copies the per-tile count of historical blocks the attention kernel
+ * processes (the union of the kept blocks of the tile's 128 query rows,
+ * excluding the tile's own two diagonal blocks) from the last
+ * sas_attention_fwd: out[B * H * ceil(N/128)].  Synchronises. */
+sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n);
+
+/* Failure-path self-test: launches one block that waits on an mbarrier that
+ * nothing completes, with the library's bounded wait and a limit of
+ * `limit_cycles` SM clock cycles, and returns in *host_status what the
+ * device recorded (SAS_ERR_TIMEOUT expected).  Synchronises. */
+sas_status sas_selftest_wait_timeout(int64_t limit_cycles, int32_t* host_status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SAS_H */

@@ -8,7 +8,7 @@ arithmetic.
 
 What it computes (SAS, "Simple Attention Sparsification", arXiv 2609.13141):
 
-  a1  block summaries      Kbar_m = mean of the keys of block B_m            (Sec. 7 limitation: "pooling based block summaries")
+  a1  block summaries      Kbar_m = mean of the keys of block B_m            (App. B, Limitation: pooled block summaries)
   a2  selector scores      s_im = R_theta(q_i, {K_Bm})                       (Alg. 1 step 1; Sec. 4.3)
   a3  causal log-gates     log g_m = s_m - LSE(s) over the row's history     (Eq. normalized_log_gate)
   a4  Top-K selection      I = TopK(g, K) = TopK(s, K)                       (Eq. selected_context; Alg. 1 / Alg. 2)
@@ -34,8 +34,9 @@ reasoning in the design notes of the repository):
     agree because log g = s - const; Alg. 1 vs Alg. 2).
   * Selector R_theta (MEANPOOL_PROJ): the paper names the AttnGate of
     SeerAttention-R without describing it.  The reading used here is
-    q~_i = bf16(q_i Wq), K~_m = bf16(Kbar_m Wk), s_im = q~_i . K~_m / sqrt(d_s).
-    The two projections are bf16 activations, as in a bf16 model.
+    q~_i = bf16(Wq q_i), K~_m = bf16(Wk Kbar_m), s_im = q~_i . K~_m / sqrt(d_s),
+    with Wq, Wk in linear-layer layout [d_s, d].  The two projections are
+    bf16 activations, as in a bf16 model.
     PARITY UNPINNED for the selector architecture itself: no paper value
     exists to check it against; only its arithmetic is pinned.
   * MLP: the hidden activation GELU(X W1^T + b1) is a bf16 tensor between the
@@ -107,13 +108,13 @@ def block_summaries(K, b):
 def selector_scores(Q, K, Wq, Wk, b):
     """a2 (MEANPOOL_PROJ reading of R_theta): s[i, m] for every row i, m < F.
 
-    q~_i = bf16(q_i Wq), K~_m = bf16(Kbar_m Wk), s_im = q~_i . K~_m / sqrt(d_s).
+    q~_i = bf16(Wq q_i), K~_m = bf16(Wk Kbar_m), s_im = q~_i . K~_m / sqrt(d_s).
     Entries with m >= C_i are computed but never used by a row (causality).
-    Wq, Wk: [d, d_s].
+    Wq, Wk: [d_s, d] (linear-layer layout [out, in]).
     """
-    d_s = Wq.shape[1]
-    qt = round_to_bf16(Q @ Wq)
-    kt = round_to_bf16(block_summaries(K, b) @ Wk)
+    d_s = Wq.shape[0]
+    qt = round_to_bf16(Q @ Wq.T)
+    kt = round_to_bf16(block_summaries(K, b) @ Wk.T)
     return (qt @ kt.T) / math.sqrt(d_s)
 
 
@@ -234,7 +235,7 @@ def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
     """Alg. 1 steps 1-4 (training forward) over [B, H, N, d] inputs.
 
     Either `scores` [B, H, N, >=C-1] are given (scores-given selector) or the
-    MEANPOOL_PROJ selector weights Wq, Wk [H, d, d_s] are.  heads: list of
+    MEANPOOL_PROJ selector weights Wq, Wk [H, d_s, d] are.  heads: list of
     (batch, head) pairs to evaluate (default all); rows as in
     sas_attention_head.  Returns {(bi, hi): result-dict}.
     """

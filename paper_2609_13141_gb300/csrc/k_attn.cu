@@ -1,0 +1,386 @@
+// a5: fused gated block-sparse attention forward (Eq. ours_train; Alg. 3).
+//
+// For query row i with current block c = floor(i/64) the logits are
+//   z_ij = sm_scale q_i.k_j + beta_ij,
+//   beta_ij = 0                for j in block c with j <= i   (unit gate, causal)
+//           = log g_{i,m}      for j in a kept historical block m (0 in Alg. 2 mode)
+//           = -inf             otherwise,
+// and O_i = sum_j softmax(z_i)_j v_j, LSE_i = log sum_j exp(z_ij).
+//
+// One CTA handles one 128-row query tile t (query blocks 2t and 2t+1) of one
+// (batch, head).  It visits only the key blocks some row of the tile needs:
+// the tile's union list from the selection pass (blocks < 2t, ascending),
+// then the diagonal blocks 2t and 2t+1.  Per visited 64-key block:
+//   * warp 0 TMA-loads K (two-stage ring), warp 1 TMA-loads V (own ring);
+//   * warp 2 (one lane) issues S = Q K^T into one of two TMEM score buffers
+//     (tcgen05.mma M=128 N=64 K=16 steps), and later O += P V into the TMEM
+//     output accumulator (M=128 N=d, V as an MN-major operand);
+//   * warps 4-7, one thread per query row (TMEM lane), read the score row,
+//     add the row's gate or mask (each thread walks its own ascending list of
+//     kept blocks), run the online softmax in the log2 domain, write P as bf16
+//     into a 128-byte-swizzled shared tile for the next MMA and rescale the
+//     TMEM output row when the running maximum grows by more than 2^8.
+// The epilogue divides by the row sum and writes bf16 O and fp32 LSE.
+#include <math_constants.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace sas {
+namespace {
+
+constexpr int kBM = 128;          // query rows per tile
+constexpr int kBN = 64;           // keys per block
+constexpr int kThreads = 256;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.69314718055994531f;
+constexpr float kRescaleThreshold = 8.0f;   // log2 units
+
+template <int D>
+struct AttnCfg {
+    static constexpr int Q_BYTES = kBM * D * 2;
+    static constexpr int KV_BYTES = kBN * D * 2;
+    static constexpr int P_BYTES = kBM * kBN * 2;
+    static constexpr int KST = 2;
+    static constexpr int VST = 1;
+    static constexpr int OFF_K = Q_BYTES;
+    static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
+    static constexpr int OFF_P = OFF_V + VST * KV_BYTES;
+    static constexpr int SMEM = OFF_P + P_BYTES + 1024;
+    static constexpr int TMEM_COLS = 256;    // S0 [0,64) S1 [64,128) O [128,128+D)
+    static constexpr int TMEM_O = 128;
+    static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, 0, 0);
+    static constexpr uint32_t IDESC_O = idesc_bf16(kBM, D, 0, 1);
+};
+
+struct AttnParams {
+    bf16* O;
+    float* LSE;
+    const int32_t* union_idx;
+    const int32_t* union_cnt;
+    const int32_t* sel_idx;
+    const float* sel_logg;
+    int N, C, T, topk, mode;
+    float scale_log2;
+    int* status;
+    long long limit;
+};
+
+__device__ __forceinline__ int block_at(const AttnParams& p, const int32_t* ulist, int U, int j, int t) {
+    return j < U ? __ldg(ulist + j) : 2 * t + (j - U);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 2)
+attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
+            const __grid_constant__ CUtensorMap mapV, AttnParams p) {
+    using Cfg = AttnCfg<D>;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    __shared__ uint64_t q_full, k_full[Cfg::KST], k_empty[Cfg::KST], v_full[Cfg::VST], v_empty[Cfg::VST];
+    __shared__ uint64_t s_full[2], s_free[2], p_full, o_ready, drain_bar;
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ int abort_flag;
+
+    const uint32_t warp = warp_id(), lane = lane_id();
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
+
+    const int t = p.T - 1 - static_cast<int>(blockIdx.x);   // heavy tiles first
+    const int bh = blockIdx.y;
+    const int32_t* ulist = p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C;
+    const int U = __ldg(p.union_cnt + static_cast<long long>(bh) * p.T + t);
+    const int n_diag = (2 * t + 1 < p.C) ? 2 : 1;
+    const int n = U + n_diag;
+
+    if (threadIdx.x == 0) {
+        mbar_init(&q_full, 1);
+        for (int s = 0; s < Cfg::KST; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
+        for (int s = 0; s < Cfg::VST; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
+        for (int s = 0; s < 2; ++s) { mbar_init(&s_full[s], 1); mbar_init(&s_free[s], 128); }
+        mbar_init(&p_full, 128);
+        mbar_init(&o_ready, 1);
+        mbar_init(&drain_bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 3) {
+        tmem_alloc(&tmem_base_sh, Cfg::TMEM_COLS);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = tmem_base_sh;
+    const WaitCtl wc{&abort_flag, p.status, p.limit};
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- K producer (and the Q tile)
+        tma_prefetch_desc(&mapQ);
+        tma_prefetch_desc(&mapK);
+        mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
+#pragma unroll
+        for (int a = 0; a < D / 64; ++a) tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, t * kBM, bh);
+        int issued = 0;
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int s = j % Cfg::KST;
+            if (!mbar_wait(&k_empty[s], ((j / Cfg::KST) & 1) ^ 1u, wc)) { ok = false; break; }
+            const int m = block_at(p, ulist, U, j, t);
+            uint8_t* dst = smem + Cfg::OFF_K + s * Cfg::KV_BYTES;
+            mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
+#pragma unroll
+            for (int a = 0; a < D / 64; ++a) tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, bh);
+            ++issued;
+        }
+        if (!ok) {
+            mbar_wait_drain(&q_full, 0, p.limit, p.status);
+            for (int q = issued - 1; q >= 0 && q >= issued - Cfg::KST; --q)
+                mbar_wait_drain(&k_full[q % Cfg::KST], (q / Cfg::KST) & 1, p.limit, p.status);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- V producer
+        tma_prefetch_desc(&mapV);
+        int issued = 0;
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int s = j % Cfg::VST;
+            if (!mbar_wait(&v_empty[s], ((j / Cfg::VST) & 1) ^ 1u, wc)) { ok = false; break; }
+            const int m = block_at(p, ulist, U, j, t);
+            uint8_t* dst = smem + Cfg::OFF_V + s * Cfg::KV_BYTES;
+            mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
+#pragma unroll
+            for (int a = 0; a < D / 64; ++a) tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, bh);
+            ++issued;
+        }
+        if (!ok) {
+            for (int q = issued - 1; q >= 0 && q >= issued - Cfg::VST; --q)
+                mbar_wait_drain(&v_full[q % Cfg::VST], (q / Cfg::VST) & 1, p.limit, p.status);
+        }
+    } else if (warp == 2 && lane == 0) {
+        // ---------------- MMA issuer
+        const uint32_t q_addr = smem_u32(smem);
+        const uint32_t p_addr = smem_u32(smem + Cfg::OFF_P);
+        bool ok = mbar_wait(&q_full, 0, wc);
+        for (int j = 0; ok && j <= n; ++j) {
+            if (j < n) {
+                // S[j%2] = Q K_j^T
+                const int s = j % Cfg::KST;
+                const int sb = j & 1;
+                if (!mbar_wait(&k_full[s], (j / Cfg::KST) & 1, wc)) break;
+                if (!mbar_wait(&s_free[sb], ((j >> 1) & 1) ^ 1u, wc)) break;
+                tc_fence_after();
+                const uint32_t k_addr = smem_u32(smem + Cfg::OFF_K + s * Cfg::KV_BYTES);
+#pragma unroll
+                for (int k = 0; k < D / 16; ++k) {
+                    const uint32_t off_q = (k >> 2) * (kBM * 128) + (k & 3) * 32;
+                    const uint32_t off_k = (k >> 2) * (kBN * 128) + (k & 3) * 32;
+                    umma_bf16(tmem_base + sb * 64, smem_desc_sw128(q_addr + off_q, 16, 1024),
+                              smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                }
+                umma_commit(&s_full[sb]);
+                umma_commit(&k_empty[s]);
+            }
+            if (j >= 1) {
+                // O += P_{j-1} V_{j-1}
+                const int jj = j - 1;
+                const int vs = jj % Cfg::VST;
+                if (!mbar_wait(&p_full, jj & 1, wc)) break;
+                if (!mbar_wait(&v_full[vs], (jj / Cfg::VST) & 1, wc)) break;
+                tc_fence_after();
+                const uint32_t v_addr = smem_u32(smem + Cfg::OFF_V + vs * Cfg::KV_BYTES);
+#pragma unroll
+                for (int k = 0; k < kBN / 16; ++k) {
+                    // P: K-major, 16 keys = 32 bytes along the swizzled row.
+                    // V: MN-major (d contiguous), 16 keys = two 8-row atoms;
+                    //    the two 64-wide d halves sit kBN*128 bytes apart.
+                    umma_bf16(tmem_base + Cfg::TMEM_O, smem_desc_sw128(p_addr + k * 32, 16, 1024),
+                              smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
+                              (jj > 0 || k > 0) ? 1u : 0u);
+                }
+                umma_commit(&o_ready);
+                umma_commit(&v_empty[vs]);
+            }
+        }
+        umma_commit(&drain_bar);
+        mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+    } else if (warp >= 4) {
+        // ---------------- softmax / correction / epilogue: one thread per row
+        const int q = warp - 4;
+        const int r = q * 32 + lane;
+        const int i = t * kBM + r;
+        const bool valid = i < p.N;
+        const int c = i >> 6;
+        const int nsel = valid ? min(p.topk, c) : 0;
+        const long long row_off = static_cast<long long>(bh) * p.N + i;
+        const int32_t* my_idx = p.sel_idx + row_off * p.topk;
+        const float* my_lg = p.sel_logg + row_off * p.topk;
+        int sp = 0;
+        int next_m = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
+        float next_lg = nsel > 0 ? __ldg(my_lg) : 0.f;
+        const bool train = p.mode == 0;
+
+        const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+        uint8_t* p_row = smem + Cfg::OFF_P + r * 128;
+        const int sw = r & 7;
+
+        float m_use = -CUDART_INF_F;
+        float l = 0.f;
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int sb = j & 1;
+            const int m = block_at(p, ulist, U, j, t);
+            // additive gate (log2 units) and the last visible key column of this block for the row
+            float bias = 0.f;
+            int lim;
+            if (m < c) {
+                if (m == next_m) {
+                    bias = train ? next_lg * kLog2e : 0.f;
+                    lim = kBN - 1;
+                    ++sp;
+                    next_m = sp < nsel ? __ldg(my_idx + sp) : 0x7fffffff;
+                    next_lg = sp < nsel ? __ldg(my_lg + sp) : 0.f;
+                } else {
+                    lim = -1;
+                }
+            } else if (m == c) {
+                lim = i & (kBN - 1);
+            } else {
+                lim = -1;
+            }
+
+            if (!mbar_wait_warp(&s_full[sb], (j >> 1) & 1, wc)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t u0[32], u1[32];
+            tmem_ld32(lane_addr + sb * 64, u0);
+            tmem_ld32(lane_addr + sb * 64 + 32, u1);
+            tmem_wait_ld();
+            tc_fence_before();
+            mbar_arrive(&s_free[sb]);
+
+            float x[64];
+            float mb = -CUDART_INF_F;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+                x[k] = k <= lim ? fmaf(__uint_as_float(u0[k]), p.scale_log2, bias) : -CUDART_INF_F;
+                x[k + 32] = k + 32 <= lim ? fmaf(__uint_as_float(u1[k]), p.scale_log2, bias) : -CUDART_INF_F;
+                mb = fmaxf(mb, fmaxf(x[k], x[k + 32]));
+            }
+            const bool need = mb > m_use + kRescaleThreshold;
+            const float m_new = need ? mb : m_use;
+            const float base = m_new == -CUDART_INF_F ? 0.f : m_new;
+            float rs = 0.f;
+#pragma unroll
+            for (int k = 0; k < 64; ++k) {
+                x[k] = fast_exp2(x[k] - base);
+                rs += x[k];
+            }
+            float factor = 1.f;
+            if (need) factor = m_use == -CUDART_INF_F ? 0.f : fast_exp2(m_use - m_new);
+
+            if (j > 0) {
+                // PV_{j-1} must be done before P is overwritten and O rescaled.
+                if (!mbar_wait_warp(&o_ready, (j - 1) & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, need)) {
+#pragma unroll 1
+                    for (int cc = 0; cc < D / 32; ++cc) {
+                        uint32_t o[32];
+                        tmem_ld32(lane_addr + Cfg::TMEM_O + cc * 32, o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
+                        tmem_st32(lane_addr + Cfg::TMEM_O + cc * 32, o);
+                    }
+                    tmem_wait_st();
+                }
+            }
+            l = l * factor + rs;
+            m_use = m_new;
+
+            // P row (64 bf16 = 8 chunks of 16 bytes), 128-byte swizzle: chunk k at k ^ (row & 7)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                uint4 w;
+                w.x = pack_bf16x2(x[8 * k + 0], x[8 * k + 1]);
+                w.y = pack_bf16x2(x[8 * k + 2], x[8 * k + 3]);
+                w.z = pack_bf16x2(x[8 * k + 4], x[8 * k + 5]);
+                w.w = pack_bf16x2(x[8 * k + 6], x[8 * k + 7]);
+                *reinterpret_cast<uint4*>(p_row + ((k ^ sw) << 4)) = w;
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&p_full);
+        }
+
+        if (ok && mbar_wait_warp(&o_ready, (n - 1) & 1, wc)) {
+            tc_fence_after();
+            const float inv = 1.f / l;
+            bf16* orow = p.O + row_off * D;
+#pragma unroll 1
+            for (int cc = 0; cc < D / 32; ++cc) {
+                uint32_t o[32];
+                tmem_ld32(lane_addr + Cfg::TMEM_O + cc * 32, o);
+                tmem_wait_ld();
+                if (valid) {
+                    uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(o[8 * e + 0]) * inv, __uint_as_float(o[8 * e + 1]) * inv);
+                        w.y = pack_bf16x2(__uint_as_float(o[8 * e + 2]) * inv, __uint_as_float(o[8 * e + 3]) * inv);
+                        w.z = pack_bf16x2(__uint_as_float(o[8 * e + 4]) * inv, __uint_as_float(o[8 * e + 5]) * inv);
+                        w.w = pack_bf16x2(__uint_as_float(o[8 * e + 6]) * inv, __uint_as_float(o[8 * e + 7]) * inv);
+                        dst[e] = w;
+                    }
+                }
+            }
+            if (valid && p.LSE != nullptr) p.LSE[row_off] = m_use * kLn2 + logf(l);
+        }
+    }
+    __syncthreads();
+    if (warp == 3) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    }
+}
+
+template <int D>
+cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) {
+    using Cfg = AttnCfg<D>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+        if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
+        attr_set = true;
+    }
+    CUtensorMap mq, mk, mv;
+    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kBM) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mk, a.K, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mv, a.V, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map V"; return cudaErrorInvalidValue; }
+    AttnParams p;
+    p.O = static_cast<bf16*>(a.O);
+    p.LSE = a.LSE;
+    p.union_idx = a.union_idx;
+    p.union_cnt = a.union_cnt;
+    p.sel_idx = a.sel_idx;
+    p.sel_logg = a.sel_logg;
+    p.N = a.N; p.C = a.C; p.T = a.T; p.topk = a.topk; p.mode = a.mode;
+    p.scale_log2 = a.sm_scale * kLog2e;
+    p.status = env.status;
+    p.limit = env.limit;
+    dim3 grid(a.T, a.BH);
+    attn_kernel<D><<<grid, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) *err = "attention launch";
+    return e;
+}
+
+}  // namespace
+
+cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err) {
+    if (a.d == 128) return launch_d<128>(a, env, err);
+    if (a.d == 64) return launch_d<64>(a, env, err);
+    *err = "attention: unsupported head dim";
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace sas

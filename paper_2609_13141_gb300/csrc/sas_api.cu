@@ -1,0 +1,439 @@
+// C ABI of the SAS library: argument checking, workspace ownership, launch
+// sequencing on the caller's stream, per-kernel event timing and the device
+// status word.  All arithmetic happens in the kernels of k_*.cu.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "../../include/sas.h"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace sas {
+
+// ------------------------------------------------------------ tensor maps
+
+namespace {
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+void resolve_encode() {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+}
+}  // namespace
+
+int make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t outer,
+                      uint32_t box_inner, uint32_t box_rows) {
+    std::call_once(g_encode_once, resolve_encode);
+    if (g_encode == nullptr) return -1;
+    cuuint64_t dims[3] = {inner, rows, outer};
+    cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
+    cuuint32_t box[3] = {box_inner, box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return static_cast<int>(r);
+}
+
+// ------------------------------------------------------- failure self test
+
+namespace {
+__global__ void wait_selftest_kernel(int* status, long long limit) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);   // nothing ever arrives
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const WaitCtl wc{&abort_flag, status, limit};
+        mbar_wait(&bar, 0, wc);
+    }
+}
+}  // namespace
+
+cudaError_t launch_wait_selftest(int* status, long long limit, cudaStream_t stream) {
+    wait_selftest_kernel<<<1, 32, 0, stream>>>(status, limit);
+    return cudaGetLastError();
+}
+
+}  // namespace sas
+
+// ================================================================ handle
+
+namespace {
+
+constexpr long long kDefaultWaitLimit = 4000000000LL;   // ~2 s of SM clock per wait
+
+struct TimeRec {
+    int kind;
+    cudaEvent_t a, b;
+};
+
+}  // namespace
+
+struct sas_handle {
+    sas_config cfg;
+    int device = 0;
+    int d_sel = 0;
+    float sm_scale = 0.f;
+    int BH = 0, C = 0, T = 0, F = 0;
+    // workspace
+    void* Kt = nullptr;         // bf16 [BH][max(F,1)][d_sel]
+    void* Qt = nullptr;         // bf16 [BH][N][d_sel]
+    int32_t* union_idx = nullptr;
+    int32_t* union_cnt = nullptr;
+    int32_t* sel_idx = nullptr;
+    float* sel_logg = nullptr;
+    int* status = nullptr;
+    // MLP hidden activation
+    void* hidden = nullptr;
+    size_t hidden_bytes = 0;
+    // timing
+    bool timing = false;
+    std::vector<TimeRec> recs;
+    std::vector<cudaEvent_t> events;
+    size_t events_used = 0;
+    int64_t launches = 0;
+    long long limit = kDefaultWaitLimit;
+    std::string last_error;
+};
+
+namespace {
+
+sas_status fail(sas_handle* h, sas_status s, const std::string& msg) {
+    if (h) h->last_error = msg;
+    return s;
+}
+
+sas_status cuda_fail(sas_handle* h, cudaError_t e, const char* what) {
+    std::string m = std::string(what ? what : "cuda") + ": " + cudaGetErrorString(e);
+    return fail(h, e == cudaErrorMemoryAllocation ? SAS_ERR_OOM : SAS_ERR_CUDA, m);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+
+cudaEvent_t next_event(sas_handle* h) {
+    if (h->events_used == h->events.size()) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        h->events.push_back(e);
+    }
+    return h->events[h->events_used++];
+}
+
+// Runs one kernel launch, bracketed by events when timing is on.
+template <class Fn>
+cudaError_t timed_launch(sas_handle* h, int kind, cudaStream_t s, Fn&& fn) {
+    cudaEvent_t a = nullptr, b = nullptr;
+    if (h->timing) {
+        a = next_event(h);
+        b = next_event(h);
+        if (a) cudaEventRecord(a, s);
+    }
+    cudaError_t e = fn();
+    if (e == cudaSuccess) ++h->launches;
+    if (h->timing && a && b) {
+        cudaEventRecord(b, s);
+        h->recs.push_back({kind, a, b});
+    }
+    return e;
+}
+
+template <class T>
+cudaError_t alloc(T** p, size_t bytes) {
+    void* v = nullptr;
+    cudaError_t e = cudaMalloc(&v, bytes < 16 ? 16 : bytes);
+    *p = static_cast<T*>(v);
+    return e;
+}
+
+sas_status check_device(sas_handle* h) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaGetDevice");
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (major != 10 || minor != 3)
+        return fail(h, SAS_ERR_UNSUPPORTED, "device is not sm_103 (GB300); the kernels are built for sm_103a only");
+    return SAS_OK;
+}
+
+}  // namespace
+
+// ================================================================ C ABI
+
+extern "C" {
+
+const char* sas_status_str(sas_status s) {
+    switch (s) {
+        case SAS_OK: return "ok";
+        case SAS_ERR_INVALID_ARG: return "invalid argument";
+        case SAS_ERR_UNSUPPORTED: return "unsupported";
+        case SAS_ERR_CUDA: return "cuda error";
+        case SAS_ERR_TIMEOUT: return "device wait timed out";
+        case SAS_ERR_OOM: return "out of device memory";
+    }
+    return "unknown status";
+}
+
+const char* sas_last_error(const sas_handle* h) { return h ? h->last_error.c_str() : ""; }
+
+sas_status sas_create(const sas_config* cfg, sas_handle** out) {
+    if (out == nullptr || cfg == nullptr) return SAS_ERR_INVALID_ARG;
+    *out = nullptr;
+    const sas_config& c = *cfg;
+    if (c.B < 1 || c.H < 1 || c.N < 1) return SAS_ERR_INVALID_ARG;
+    if (c.block != 64) return SAS_ERR_UNSUPPORTED;
+    if (c.d != 64 && c.d != 128) return SAS_ERR_UNSUPPORTED;
+    if (c.topk < 0) return SAS_ERR_INVALID_ARG;
+    if (c.topk > 128) return SAS_ERR_UNSUPPORTED;
+    if (c.mode != SAS_MODE_TRAIN_SOFT && c.mode != SAS_MODE_INFER_HARD) return SAS_ERR_INVALID_ARG;
+    if (c.selector != SAS_SEL_SCORES_GIVEN && c.selector != SAS_SEL_MEANPOOL_PROJ) return SAS_ERR_INVALID_ARG;
+    if (!(c.sm_scale >= 0.f) || !std::isfinite(c.sm_scale)) return SAS_ERR_INVALID_ARG;
+    const int d_sel = c.d_sel == 0 ? c.d : c.d_sel;
+    if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
+    const long long BH = static_cast<long long>(c.B) * c.H;
+    if (BH > (1LL << 30) || BH * c.N > (1LL << 40)) return SAS_ERR_UNSUPPORTED;
+
+    sas_handle* h = new sas_handle();
+    h->cfg = c;
+    h->d_sel = d_sel;
+    h->sm_scale = c.sm_scale > 0.f ? c.sm_scale : 1.0f / std::sqrt(static_cast<float>(c.d));
+    h->BH = static_cast<int>(BH);
+    h->C = (c.N + 63) / 64;
+    h->T = (c.N + 127) / 128;
+    h->F = c.N / 64;
+    sas_status st = check_device(h);
+    if (st != SAS_OK) { delete h; return st; }
+    cudaGetDevice(&h->device);
+
+    cudaError_t e = cudaSuccess;
+    const size_t rows = static_cast<size_t>(BH) * c.N;
+    if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
+        if (e == cudaSuccess) e = alloc(&h->Kt, static_cast<size_t>(BH) * (h->F > 0 ? h->F : 1) * d_sel * 2);
+        if (e == cudaSuccess) e = alloc(&h->Qt, rows * d_sel * 2);
+    }
+    if (e == cudaSuccess) e = alloc(&h->union_idx, static_cast<size_t>(BH) * h->T * h->C * 4);
+    if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BH) * h->T * 4);
+    if (e == cudaSuccess) e = alloc(&h->sel_idx, rows * (c.topk > 0 ? c.topk : 1) * 4);
+    if (e == cudaSuccess) e = alloc(&h->sel_logg, rows * (c.topk > 0 ? c.topk : 1) * 4);
+    if (e == cudaSuccess) e = alloc(&h->status, 16);
+    if (e == cudaSuccess) e = cudaMemset(h->status, 0, 16);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        sas_status s = e == cudaErrorMemoryAllocation ? SAS_ERR_OOM : SAS_ERR_CUDA;
+        sas_destroy(h);
+        return s;
+    }
+    *out = h;
+    return SAS_OK;
+}
+
+void sas_destroy(sas_handle* h) {
+    if (h == nullptr) return;
+    cudaDeviceSynchronize();
+    cudaFree(h->Kt);
+    cudaFree(h->Qt);
+    cudaFree(h->union_idx);
+    cudaFree(h->union_cnt);
+    cudaFree(h->sel_idx);
+    cudaFree(h->sel_logg);
+    cudaFree(h->status);
+    cudaFree(h->hidden);
+    for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
+    delete h;
+}
+
+sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
+                             const void* Wq, const void* Wk, void* O, float* LSE, int32_t* sel_idx,
+                             float* sel_logg, void* stream) {
+    if (h == nullptr) return SAS_ERR_INVALID_ARG;
+    const sas_config& c = h->cfg;
+    if (!Q || !K || !V || !O) return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O are required");
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O must be 16-byte aligned");
+    if (c.selector == SAS_SEL_SCORES_GIVEN) {
+        if (!scores || !aligned4(scores)) return fail(h, SAS_ERR_INVALID_ARG, "scores required (4-byte aligned)");
+        if (Wq || Wk) return fail(h, SAS_ERR_INVALID_ARG, "Wq/Wk must be NULL with given scores");
+    } else {
+        if (scores) return fail(h, SAS_ERR_INVALID_ARG, "scores must be NULL with the learned selector");
+        if (!Wq || !Wk || !aligned16(Wq) || !aligned16(Wk))
+            return fail(h, SAS_ERR_INVALID_ARG, "Wq and Wk required (16-byte aligned)");
+    }
+    if ((LSE && !aligned4(LSE)) || (sel_idx && !aligned4(sel_idx)) || (sel_logg && !aligned4(sel_logg)))
+        return fail(h, SAS_ERR_INVALID_ARG, "LSE / sel_idx / sel_logg must be 4-byte aligned");
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const sas::KernelEnv env{s, h->status, h->limit};
+    const char* err = "";
+    int32_t* out_idx = sel_idx ? sel_idx : h->sel_idx;
+    float* out_lg = sel_logg ? sel_logg : h->sel_logg;
+    cudaError_t e = cudaSuccess;
+
+    if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
+        // a1: block summaries -> projected summaries
+        if (h->F > 0) {
+            e = timed_launch(h, 0, s, [&] { return sas::launch_pool(K, Wk, h->Kt, h->BH, c.H, c.N, c.d, h->d_sel, env); });
+            if (e != cudaSuccess) return cuda_fail(h, e, "block summaries");
+        }
+        // a2 (first half): per-head query projection Qt = bf16(Q Wq^T) on the tensor cores
+        sas::GemmProblem g{};
+        g.A = Q; g.B = Wq; g.C = h->Qt; g.bias = nullptr;
+        g.M = c.N; g.N = h->d_sel; g.K = c.d;
+        g.batches = h->BH; g.b_mod = c.H;
+        g.c_batch_stride = static_cast<long long>(c.N) * h->d_sel; g.ldc = h->d_sel;
+        g.gelu = 0; g.bn = h->d_sel; g.max_ctas = 0;
+        e = timed_launch(h, 1, s, [&] { return sas::launch_gemm(g, env, &err); });
+        if (e != cudaSuccess) return cuda_fail(h, e, err);
+    }
+    // a2-a4: scores, log-gates, Top-K, tile unions
+    sas::SelectArgs sa{};
+    sa.BH = h->BH; sa.H = c.H; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.score_scale = c.selector == SAS_SEL_MEANPOOL_PROJ ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
+    sa.scores = scores;
+    sa.Qt = h->Qt; sa.Kt = h->Kt; sa.F = h->F;
+    sa.sel_idx = out_idx; sa.sel_logg = out_lg;
+    sa.union_idx = h->union_idx; sa.union_cnt = h->union_cnt;
+    e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    // a5: gated sparse attention
+    sas::AttnArgs aa{};
+    aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
+    aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
+    aa.sel_idx = out_idx; aa.sel_logg = out_lg;
+    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.sm_scale = h->sm_scale;
+    e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    return SAS_OK;
+}
+
+sas_status sas_mlp_fwd(sas_handle* h, const void* X, const void* W1, const void* b1, const void* W2, const void* b2,
+                       void* Y, int64_t T, int64_t D, int64_t F, void* stream) {
+    if (h == nullptr) return SAS_ERR_INVALID_ARG;
+    if (!X || !W1 || !W2 || !Y) return fail(h, SAS_ERR_INVALID_ARG, "X, W1, W2 and Y are required");
+    if (!aligned16(X) || !aligned16(W1) || !aligned16(W2) || !aligned16(Y) || (b1 && !aligned16(b1)) ||
+        (b2 && !aligned16(b2)))
+        return fail(h, SAS_ERR_INVALID_ARG, "MLP tensors must be 16-byte aligned");
+    if (T < 1 || D < 64 || F < 64) return fail(h, SAS_ERR_INVALID_ARG, "T >= 1, D >= 64, F >= 64 required");
+    if (D % 64 != 0 || F % 64 != 0) return fail(h, SAS_ERR_UNSUPPORTED, "D and F must be multiples of 64");
+    if (T > (1LL << 31) - 1 || D > 65536 || F > 262144) return fail(h, SAS_ERR_UNSUPPORTED, "MLP size too large");
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t need = static_cast<size_t>(T) * F * 2;
+    if (need > h->hidden_bytes) {
+        cudaError_t e = cudaStreamSynchronize(s);
+        if (e == cudaSuccess) {
+            cudaFree(h->hidden);
+            h->hidden = nullptr;
+            h->hidden_bytes = 0;
+            e = cudaMalloc(&h->hidden, need);
+        }
+        if (e != cudaSuccess) return cuda_fail(h, e, "MLP hidden buffer");
+        h->hidden_bytes = need;
+    }
+    const sas::KernelEnv env{s, h->status, h->limit};
+    const char* err = "";
+    auto pick_bn = [](int64_t n) { return n % 256 == 0 ? 256 : (n % 128 == 0 ? 128 : 64); };
+
+    sas::GemmProblem g1{};
+    g1.A = X; g1.B = W1; g1.C = h->hidden; g1.bias = b1;
+    g1.M = static_cast<int>(T); g1.N = static_cast<int>(F); g1.K = static_cast<int>(D);
+    g1.batches = 1; g1.b_mod = 1; g1.c_batch_stride = 0; g1.ldc = static_cast<int>(F);
+    g1.gelu = 1; g1.bn = pick_bn(F); g1.max_ctas = 0;
+    cudaError_t e = timed_launch(h, 4, s, [&] { return sas::launch_gemm(g1, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+
+    sas::GemmProblem g2{};
+    g2.A = h->hidden; g2.B = W2; g2.C = Y; g2.bias = b2;
+    g2.M = static_cast<int>(T); g2.N = static_cast<int>(D); g2.K = static_cast<int>(F);
+    g2.batches = 1; g2.b_mod = 1; g2.c_batch_stride = 0; g2.ldc = static_cast<int>(D);
+    g2.gelu = 0; g2.bn = pick_bn(D); g2.max_ctas = 0;
+    e = timed_launch(h, 5, s, [&] { return sas::launch_gemm(g2, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    return SAS_OK;
+}
+
+sas_status sas_get_device_status(sas_handle* h, int32_t* out_status) {
+    if (h == nullptr || out_status == nullptr) return SAS_ERR_INVALID_ARG;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(h, e, "synchronize");
+    int v = 0;
+    e = cudaMemcpy(&v, h->status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemset(h->status, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(h, e, "status word");
+    *out_status = v;
+    return SAS_OK;
+}
+
+sas_status sas_set_timing(sas_handle* h, int32_t enable) {
+    if (h == nullptr) return SAS_ERR_INVALID_ARG;
+    cudaDeviceSynchronize();
+    h->timing = enable != 0;
+    h->recs.clear();
+    h->events_used = 0;
+    return SAS_OK;
+}
+
+sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds) {
+    if (h == nullptr || launches == nullptr || total_ms == nullptr || n_kinds < 0 || n_kinds > SAS_NUM_KERNEL_KINDS)
+        return SAS_ERR_INVALID_ARG;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(h, e, "synchronize");
+    for (int k = 0; k < n_kinds; ++k) { launches[k] = 0; total_ms[k] = 0.0; }
+    for (const TimeRec& r : h->recs) {
+        if (r.kind >= n_kinds) continue;
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, r.a, r.b) == cudaSuccess) {
+            launches[r.kind] += 1;
+            total_ms[r.kind] += ms;
+        }
+    }
+    return SAS_OK;
+}
+
+int64_t sas_launch_count(const sas_handle* h) { return h ? h->launches : 0; }
+
+sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n) {
+    if (h == nullptr || host_out == nullptr) return SAS_ERR_INVALID_ARG;
+    const int64_t total = static_cast<int64_t>(h->BH) * h->T;
+    if (n < total) return fail(h, SAS_ERR_INVALID_ARG, "output too small");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpy(host_out, h->union_cnt, total * 4, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(h, e, "union counts");
+    return SAS_OK;
+}
+
+sas_status sas_selftest_wait_timeout(int64_t limit_cycles, int32_t* host_status) {
+    if (host_status == nullptr || limit_cycles < 0) return SAS_ERR_INVALID_ARG;
+    if (check_device(nullptr) != SAS_OK) return SAS_ERR_UNSUPPORTED;
+    int* d = nullptr;
+    cudaError_t e = cudaMalloc(&d, 16);
+    if (e == cudaSuccess) e = cudaMemset(d, 0, 16);
+    if (e == cudaSuccess) e = sas::launch_wait_selftest(d, limit_cycles, nullptr);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    int v = 0;
+    if (e == cudaSuccess) e = cudaMemcpy(&v, d, sizeof(int), cudaMemcpyDeviceToHost);
+    cudaFree(d);
+    if (e != cudaSuccess) return SAS_ERR_CUDA;
+    *host_status = v;
+    return SAS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,242 @@
+"""ctypes binding of the SAS C ABI (include/sas.h).
+
+Argument marshalling only: every function here converts torch tensors to
+device pointers, checks dtype/device/contiguity, and calls the entry point
+of the same name in libsas.so.  No arithmetic of the method happens here, and
+there is no fallback: if the library is missing or the device is not sm_103,
+the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import torch
+
+from . import _build
+
+SAS_OK = 0
+SAS_ERR_INVALID_ARG = 1
+SAS_ERR_UNSUPPORTED = 2
+SAS_ERR_CUDA = 3
+SAS_ERR_TIMEOUT = 4
+SAS_ERR_OOM = 5
+
+SAS_MODE_TRAIN_SOFT = 0
+SAS_MODE_INFER_HARD = 1
+SAS_SEL_SCORES_GIVEN = 0
+SAS_SEL_MEANPOOL_PROJ = 1
+SAS_NUM_KERNEL_KINDS = 6
+KERNEL_KINDS = ["block_summaries", "query_projection", "selection", "attention", "mlp_up_gelu", "mlp_down"]
+
+HEADER = os.path.join(_build.ROOT, "include", "sas.h")
+
+
+class SasConfig(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("block", ctypes.c_int32), ("topk", ctypes.c_int32), ("sm_scale", ctypes.c_float),
+                ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32)]
+
+
+class SasError(RuntimeError):
+    def __init__(self, status, message):
+        super().__init__(f"{message} (status {status})")
+        self.status = status
+
+
+_lib = None
+
+
+def lib():
+    """Loads libsas.so (built in-tree by _build.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_build.LIB_PATH):
+        raise RuntimeError("libsas.so is not built; run paper_2609_13141_gb300._build.build() first")
+    L = ctypes.CDLL(_build.LIB_PATH)
+    vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    L.sas_create.argtypes = [ctypes.POINTER(SasConfig), ctypes.POINTER(vp)]
+    L.sas_create.restype = i32
+    L.sas_destroy.argtypes = [vp]
+    L.sas_destroy.restype = None
+    L.sas_attention_fwd.argtypes = [vp] * 12
+    L.sas_attention_fwd.restype = i32
+    L.sas_mlp_fwd.argtypes = [vp] * 7 + [i64, i64, i64, vp]
+    L.sas_mlp_fwd.restype = i32
+    L.sas_status_str.argtypes = [i32]
+    L.sas_status_str.restype = ctypes.c_char_p
+    L.sas_last_error.argtypes = [vp]
+    L.sas_last_error.restype = ctypes.c_char_p
+    L.sas_get_device_status.argtypes = [vp, ctypes.POINTER(i32)]
+    L.sas_get_device_status.restype = i32
+    L.sas_set_timing.argtypes = [vp, i32]
+    L.sas_set_timing.restype = i32
+    L.sas_get_timings.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(ctypes.c_double), i32]
+    L.sas_get_timings.restype = i32
+    L.sas_launch_count.argtypes = [vp]
+    L.sas_launch_count.restype = i64
+    L.sas_get_tile_union_counts.argtypes = [vp, ctypes.POINTER(i32), i64]
+    L.sas_get_tile_union_counts.restype = i32
+    L.sas_selftest_wait_timeout.argtypes = [i64, ctypes.POINTER(i32)]
+    L.sas_selftest_wait_timeout.restype = i32
+    _lib = L
+    return L
+
+
+def header_functions():
+    """Names of the functions include/sas.h declares."""
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(sas_[a-z_]+)\s*\(", text)))
+
+
+def _ptr(t, dtype, name, required=True):
+    if t is None:
+        if required:
+            raise ValueError(f"{name} is required")
+        return None
+    if not isinstance(t, torch.Tensor) or t.device.type != "cuda":
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _check(status, handle=None, what="sas"):
+    if status != SAS_OK:
+        L = lib()
+        msg = L.sas_status_str(status).decode()
+        if handle is not None:
+            detail = L.sas_last_error(handle).decode()
+            if detail:
+                msg += ": " + detail
+        raise SasError(status, f"{what}: {msg}")
+
+
+def sas_status_str(status):
+    return lib().sas_status_str(int(status)).decode()
+
+
+def sas_create(B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
+               sm_scale=0.0, block=64):
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel)
+    h = ctypes.c_void_p()
+    _check(lib().sas_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_create")
+    return h
+
+
+def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64):
+    """Raw status of sas_create (for argument-check tests); destroys the handle on success."""
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel)
+    h = ctypes.c_void_p()
+    st = lib().sas_create(ctypes.byref(cfg), ctypes.byref(h))
+    if st == SAS_OK:
+        lib().sas_destroy(h)
+    return st
+
+
+def sas_destroy(h):
+    lib().sas_destroy(h)
+
+
+def sas_attention_fwd(h, Q, K, V, O, scores=None, Wq=None, Wk=None, LSE=None, sel_idx=None, sel_logg=None,
+                      stream=None):
+    bf = torch.bfloat16
+    st = lib().sas_attention_fwd(
+        h, _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"),
+        _ptr(scores, torch.float32, "scores", False), _ptr(Wq, bf, "Wq", False), _ptr(Wk, bf, "Wk", False),
+        _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False), _ptr(sel_idx, torch.int32, "sel_idx", False),
+        _ptr(sel_logg, torch.float32, "sel_logg", False), _stream(stream))
+    _check(st, h, "sas_attention_fwd")
+
+
+def sas_mlp_fwd(h, X, W1, W2, Y, b1=None, b2=None, stream=None):
+    bf = torch.bfloat16
+    T, D = X.shape
+    F = W1.shape[0]
+    st = lib().sas_mlp_fwd(h, _ptr(X, bf, "X"), _ptr(W1, bf, "W1"), _ptr(b1, bf, "b1", False), _ptr(W2, bf, "W2"),
+                           _ptr(b2, bf, "b2", False), _ptr(Y, bf, "Y"), T, D, F, _stream(stream))
+    _check(st, h, "sas_mlp_fwd")
+
+
+def sas_get_device_status(h):
+    v = ctypes.c_int32(0)
+    _check(lib().sas_get_device_status(h, ctypes.byref(v)), h, "sas_get_device_status")
+    return v.value
+
+
+def sas_set_timing(h, enable):
+    _check(lib().sas_set_timing(h, 1 if enable else 0), h, "sas_set_timing")
+
+
+def sas_get_timings(h):
+    """{kind: (launches, total_ms)} for the kernel kinds of sas.h."""
+    n = SAS_NUM_KERNEL_KINDS
+    launches = (ctypes.c_int64 * n)()
+    ms = (ctypes.c_double * n)()
+    _check(lib().sas_get_timings(h, launches, ms, n), h, "sas_get_timings")
+    return {KERNEL_KINDS[k]: (launches[k], ms[k]) for k in range(n)}
+
+
+def sas_launch_count(h):
+    return lib().sas_launch_count(h)
+
+
+def sas_get_tile_union_counts(h, n):
+    out = (ctypes.c_int32 * n)()
+    _check(lib().sas_get_tile_union_counts(h, out, n), h, "sas_get_tile_union_counts")
+    return list(out)
+
+
+def sas_selftest_wait_timeout(limit_cycles):
+    v = ctypes.c_int32(-1)
+    _check(lib().sas_selftest_wait_timeout(int(limit_cycles), ctypes.byref(v)), None, "sas_selftest_wait_timeout")
+    return v.value
+
+
+class SasLayer:
+    """Owns one handle; allocates outputs and calls the C ABI."""
+
+    def __init__(self, B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
+                 sm_scale=0.0):
+        self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
+        self.selector = selector
+        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale)
+
+    def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
+        dev = Q.device
+        O = torch.empty_like(Q)
+        LSE = torch.empty(self.B, self.H, self.N, device=dev, dtype=torch.float32)
+        sel_idx = sel_logg = None
+        if want_sel:
+            k = max(self.topk, 1)
+            sel_idx = torch.empty(self.B, self.H, self.N, k, device=dev, dtype=torch.int32)
+            sel_logg = torch.empty(self.B, self.H, self.N, k, device=dev, dtype=torch.float32)
+        sas_attention_fwd(self.h, Q, K, V, O, scores, Wq, Wk, LSE, sel_idx, sel_logg, stream)
+        return O, LSE, sel_idx, sel_logg
+
+    def mlp(self, X, W1, W2, b1=None, b2=None, stream=None):
+        Y = torch.empty(X.shape[0], W2.shape[0], device=X.device, dtype=torch.bfloat16)
+        sas_mlp_fwd(self.h, X, W1, W2, Y, b1, b2, stream)
+        return Y
+
+    def close(self):
+        if self.h is not None:
+            sas_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

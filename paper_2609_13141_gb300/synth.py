@@ -64,10 +64,31 @@ def integer_scores(B, H, N, C, seed=0, levels=4):
     return torch.randint(0, levels, (B, H, N, C), generator=g).to(torch.float32)
 
 
+def integer_selector_inputs(B, H, N, d, d_sel, seed=0, nnz=4):
+    """Q, K with integer entries in [-3, 3], V ~ N(0, 1), and sparse selector
+    projections with entries in {-1, 0, 1} (nnz non-zeros per output row).
+
+    With these inputs every sum the learned selector forms is exactly
+    representable in fp32, so any two correct implementations see identical
+    scores (and identical ties)."""
+    g = _gen(seed + 50)
+    Q = torch.randint(-3, 4, (B, H, N, d), generator=g).to(torch.bfloat16)
+    K = torch.randint(-3, 4, (B, H, N, d), generator=g).to(torch.bfloat16)
+    V = normal((B, H, N, d), seed + 51).to(torch.bfloat16)
+    W = []
+    for _ in range(2):
+        w = torch.zeros(H, d_sel, d)
+        cols = torch.stack([torch.randperm(d, generator=g)[:nnz] for _ in range(H * d_sel)]).view(H, d_sel, nnz)
+        sign = torch.randint(0, 2, (H, d_sel, nnz), generator=g).float() * 2 - 1
+        w.scatter_(2, cols, sign)
+        W.append(w.to(torch.bfloat16))
+    return Q, K, V, W[0], W[1]
+
+
 def selector_weights(H, d, d_sel, seed=0, std=0.02):
-    """Wq, Wk as bf16 [H, d, d_sel]."""
-    Wq = normal((H, d, d_sel), seed + 30, std).to(torch.bfloat16)
-    Wk = normal((H, d, d_sel), seed + 31, std).to(torch.bfloat16)
+    """Wq, Wk as bf16 [H, d_sel, d] (linear-layer layout [out, in])."""
+    Wq = normal((H, d_sel, d), seed + 30, std).to(torch.bfloat16)
+    Wk = normal((H, d_sel, d), seed + 31, std).to(torch.bfloat16)
     return Wq, Wk
 
 

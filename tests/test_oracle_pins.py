@@ -70,8 +70,8 @@ def test_selector_scores_scaling_and_permutation():
     b, N, d, ds = 4, 32, 8, 6
     Q = O.round_to_bf16(rng.standard_normal((N, d)))
     K = O.round_to_bf16(rng.standard_normal((N, d)))
-    Wq = O.round_to_bf16(rng.standard_normal((d, ds)) * 0.3)
-    Wk = O.round_to_bf16(rng.standard_normal((d, ds)) * 0.3)
+    Wq = O.round_to_bf16(rng.standard_normal((ds, d)) * 0.3)
+    Wk = O.round_to_bf16(rng.standard_normal((ds, d)) * 0.3)
     s = O.selector_scores(Q, K, Wq, Wk, b)
     assert np.allclose(O.selector_scores(Q, K, 2 * Wq, Wk, b), 2 * s, rtol=1e-12, atol=0)
     perm = rng.permutation(N // b)
