@@ -128,6 +128,36 @@ sas_status sas_mlp_fwd(sas_handle* h,
                        int64_t T, int64_t D, int64_t F,
                        void* stream);
 
+/* Handle-free variant of sas_mlp_fwd that allocates no device memory.
+ * (The paper has no counterpart: this serves callers, not the method.)
+ *
+ * Who needs it: callers that cannot call cudaMalloc while they run the
+ * layer -- code recording a CUDA graph on its stream, plug-ins whose host
+ * framework owns all device memory, services that must keep a fixed device
+ * footprint.  sas_mlp_fwd would allocate its hidden buffer through a handle;
+ * this entry point instead keeps the bf16 hidden activation [T, F] in a fixed
+ * array of SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES (32 MiB) compiled into the
+ * library, which every GPU that loads the library reserves until the process
+ * exits.  It calls no allocator (neither CUDA's nor any library's).
+ *
+ * Arguments, layouts and result are those of sas_mlp_fwd (X, W1, b1, W2, b2,
+ * Y are caller-owned device buffers).  T * F * 2 must not exceed
+ * SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES; larger sizes are rejected with
+ * SAS_ERR_UNSUPPORTED before anything runs.
+ *
+ * The first call on each device looks the array's device address up with
+ * cudaGetSymbolAddress (with that device current); make that first call
+ * before any stream capture starts.  All calls on a device share the one
+ * array, and it keeps whatever the last call left in it: two calls whose
+ * work overlaps on the GPU (different streams without ordering between
+ * them) race on it and may corrupt each other's results.  Calls ordered on
+ * one stream are safe. */
+#define SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES (32u * 1024u * 1024u)
+sas_status sas_mlp_fwd_noalloc(const void* X, const void* W1, const void* b1,
+                               const void* W2, const void* b2, void* Y,
+                               int64_t T, int64_t D, int64_t F,
+                               void* stream);
+
 /* Static text for a status code. */
 const char* sas_status_str(sas_status s);
 

@@ -79,6 +79,8 @@ def lib():
     L.sas_launch_count.restype = i64
     L.sas_get_tile_union_counts.argtypes = [vp, ctypes.POINTER(i32), i64]
     L.sas_get_tile_union_counts.restype = i32
+    L.sas_mlp_fwd_noalloc.argtypes = [vp] * 6 + [i64, i64, i64, vp]
+    L.sas_mlp_fwd_noalloc.restype = i32
     L.sas_selftest_wait_timeout.argtypes = [i64, ctypes.POINTER(i32)]
     L.sas_selftest_wait_timeout.restype = i32
     _lib = L
@@ -167,6 +169,25 @@ def sas_mlp_fwd(h, X, W1, W2, Y, b1=None, b2=None, stream=None):
     st = lib().sas_mlp_fwd(h, _ptr(X, bf, "X"), _ptr(W1, bf, "W1"), _ptr(b1, bf, "b1", False), _ptr(W2, bf, "W2"),
                            _ptr(b2, bf, "b2", False), _ptr(Y, bf, "Y"), T, D, F, _stream(stream))
     _check(st, h, "sas_mlp_fwd")
+
+
+SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES = 32 * 1024 * 1024
+
+
+def sas_mlp_fwd_noalloc(X, W1, W2, Y, b1=None, b2=None, stream=None):
+    """The MLP without a handle and without any device allocation (see sas.h):
+    the hidden activation lives in a fixed 32 MiB array inside the library,
+    shared by every call on the device."""
+    bf = torch.bfloat16
+    T, D = X.shape
+    F = W1.shape[0]
+    st = lib().sas_mlp_fwd_noalloc(_ptr(X, bf, "X"), _ptr(W1, bf, "W1"), _ptr(b1, bf, "b1", False),
+                                   _ptr(W2, bf, "W2"), _ptr(b2, bf, "b2", False), _ptr(Y, bf, "Y"), T, D, F,
+                                   _stream(stream))
+    if st == SAS_ERR_UNSUPPORTED and T * F * 2 > SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES:
+        raise SasError(st, f"sas_mlp_fwd_noalloc: hidden activation of {T}x{F} bf16 ({T * F * 2} bytes) exceeds "
+                           f"the fixed {SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES}-byte array")
+    _check(st, None, "sas_mlp_fwd_noalloc")
 
 
 def sas_get_device_status(h):
