@@ -96,8 +96,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         mbar_init(&q_full, 1);
         for (int s = 0; s < Cfg::KST; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
         for (int s = 0; s < Cfg::VST; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
-        for (int s = 0; s < 2; ++s) { mbar_init(&s_full[s], 1); mbar_init(&s_free[s], 128); }
-        mbar_init(&p_full, 128);
+        for (int s = 0; s < 2; ++s) { mbar_init(&s_full[s], 1); mbar_init(&s_free[s], 4); }
+        mbar_init(&p_full, 4);
         mbar_init(&o_ready, 1);
         mbar_init(&drain_bar, 1);
         abort_flag = 0;
@@ -213,31 +213,39 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         const long long row_off = static_cast<long long>(bh) * p.N + i;
         const int32_t* my_idx = p.sel_idx + row_off * p.topk;
         const float* my_lg = p.sel_logg + row_off * p.topk;
-        int sp = 0;
-        int next_m = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
-        float next_lg = nsel > 0 ? __ldg(my_lg) : 0.f;
         const bool train = p.mode == 0;
+        // the row's next two kept blocks (a two-entry queue keeps the loads ahead of their use)
+        int sp = 0;
+        int km0 = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
+        float kl0 = nsel > 0 ? __ldg(my_lg) : 0.f;
+        int km1 = nsel > 1 ? __ldg(my_idx + 1) : 0x7fffffff;
+        float kl1 = nsel > 1 ? __ldg(my_lg + 1) : 0.f;
 
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         uint8_t* p_row = smem + Cfg::OFF_P + r * 128;
         const int sw = r & 7;
+        const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2);
 
         float m_use = -CUDART_INF_F;
         float l = 0.f;
         bool ok = true;
+        int m_next = block_at(p, ulist, U, 0, t);
         for (int j = 0; j < n; ++j) {
             const int sb = j & 1;
-            const int m = block_at(p, ulist, U, j, t);
-            // additive gate (log2 units) and the last visible key column of this block for the row
+            const int m = m_next;
+            if (j + 1 < n) m_next = block_at(p, ulist, U, j + 1, t);
+            // gate (log2 units) and the last visible key column of block m for this row
             float bias = 0.f;
             int lim;
             if (m < c) {
-                if (m == next_m) {
-                    bias = train ? next_lg * kLog2e : 0.f;
+                if (m == km0) {
+                    bias = train ? kl0 * kLog2e : 0.f;
                     lim = kBN - 1;
                     ++sp;
-                    next_m = sp < nsel ? __ldg(my_idx + sp) : 0x7fffffff;
-                    next_lg = sp < nsel ? __ldg(my_lg + sp) : 0.f;
+                    km0 = km1;
+                    kl0 = kl1;
+                    km1 = sp + 1 < nsel ? __ldg(my_idx + sp + 1) : 0x7fffffff;
+                    kl1 = sp + 1 < nsel ? __ldg(my_lg + sp + 1) : 0.f;
                 } else {
                     lim = -1;
                 }
@@ -246,32 +254,61 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             } else {
                 lim = -1;
             }
+            const bool active = lim >= 0;
 
             if (!mbar_wait_warp(&s_full[sb], (j >> 1) & 1, wc)) { ok = false; break; }
             tc_fence_after();
-            uint32_t u0[32], u1[32];
-            tmem_ld32(lane_addr + sb * 64, u0);
-            tmem_ld32(lane_addr + sb * 64 + 32, u1);
-            tmem_wait_ld();
-            tc_fence_before();
-            mbar_arrive(&s_free[sb]);
-
+            const bool warp_active = __any_sync(0xffffffffu, active);
             float x[64];
-            float mb = -CUDART_INF_F;
+            if (warp_active) {
+                uint32_t u0[32], u1[32];
+                tmem_ld32(lane_addr + sb * 64, u0);
+                tmem_ld32(lane_addr + sb * 64 + 32, u1);
+                tmem_wait_ld();
 #pragma unroll
-            for (int k = 0; k < 32; ++k) {
-                x[k] = k <= lim ? fmaf(__uint_as_float(u0[k]), p.scale_log2, bias) : -CUDART_INF_F;
-                x[k + 32] = k + 32 <= lim ? fmaf(__uint_as_float(u1[k]), p.scale_log2, bias) : -CUDART_INF_F;
-                mb = fmaxf(mb, fmaxf(x[k], x[k + 32]));
+                for (int k = 0; k < 32; ++k) {
+                    x[k] = __uint_as_float(u0[k]);
+                    x[k + 32] = __uint_as_float(u1[k]);
+                }
             }
-            const bool need = mb > m_use + kRescaleThreshold;
-            const float m_new = need ? mb : m_use;
-            const float base = m_new == -CUDART_INF_F ? 0.f : m_new;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_free[sb]);
+
+            bool need = false;
+            float m_new = m_use;
             float rs = 0.f;
+            if (warp_active) {
+                // causal mask on the diagonal block only
+                if (__any_sync(0xffffffffu, lim >= 0 && lim < kBN - 1)) {
 #pragma unroll
-            for (int k = 0; k < 64; ++k) {
-                x[k] = fast_exp2(x[k] - base);
-                rs += x[k];
+                    for (int k = 0; k < 64; ++k) x[k] = k <= lim ? x[k] : -CUDART_INF_F;
+                }
+                float mx = -CUDART_INF_F;
+#pragma unroll
+                for (int k = 0; k < 64; k += 2) mx = max3f(mx, x[k], x[k + 1]);
+                // max of the gated logits (log2 units): the gate is constant over the block
+                const float mb = active ? fmaf(mx, p.scale_log2, bias) : -CUDART_INF_F;
+                need = mb > m_use + kRescaleThreshold;
+                m_new = need ? mb : m_use;
+                const float base = m_new == -CUDART_INF_F ? 0.f : m_new;
+                const float off = active ? bias - base : -CUDART_INF_F;
+                const uint64_t off2 = f32x2(off, off);
+                uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+                for (int k = 0; k < 64; k += 2) {
+                    float a0, a1;
+                    f32x2_split(fma_f32x2(f32x2(x[k], x[k + 1]), scale2, off2), a0, a1);
+                    x[k] = fast_exp2(a0);
+                    x[k + 1] = fast_exp2(a1);
+                    acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(x[k], x[k + 1]));
+                }
+                float s0, s1, s2, s3, s4, s5, s6, s7;
+                f32x2_split(acc[0], s0, s1);
+                f32x2_split(acc[1], s2, s3);
+                f32x2_split(acc[2], s4, s5);
+                f32x2_split(acc[3], s6, s7);
+                rs = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
             }
             float factor = 1.f;
             if (need) factor = m_use == -CUDART_INF_F ? 0.f : fast_exp2(m_use - m_new);
@@ -297,18 +334,25 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             m_use = m_new;
 
             // P row (64 bf16 = 8 chunks of 16 bytes), 128-byte swizzle: chunk k at k ^ (row & 7)
+            if (warp_active) {
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                uint4 w;
-                w.x = pack_bf16x2(x[8 * k + 0], x[8 * k + 1]);
-                w.y = pack_bf16x2(x[8 * k + 2], x[8 * k + 3]);
-                w.z = pack_bf16x2(x[8 * k + 4], x[8 * k + 5]);
-                w.w = pack_bf16x2(x[8 * k + 6], x[8 * k + 7]);
-                *reinterpret_cast<uint4*>(p_row + ((k ^ sw) << 4)) = w;
+                for (int k = 0; k < 8; ++k) {
+                    uint4 w;
+                    w.x = pack_bf16x2(x[8 * k + 0], x[8 * k + 1]);
+                    w.y = pack_bf16x2(x[8 * k + 2], x[8 * k + 3]);
+                    w.z = pack_bf16x2(x[8 * k + 4], x[8 * k + 5]);
+                    w.w = pack_bf16x2(x[8 * k + 6], x[8 * k + 7]);
+                    *reinterpret_cast<uint4*>(p_row + ((k ^ sw) << 4)) = w;
+                }
+            } else {
+                const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) *reinterpret_cast<uint4*>(p_row + (k << 4)) = z;
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            mbar_arrive(&p_full);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full);
         }
 
         if (ok && mbar_wait_warp(&o_ready, (n - 1) & 1, wc)) {

@@ -14,10 +14,8 @@
 // never depends on how LSE was rounded.
 //
 // One CTA owns one (batch*head, 128-row tile); one thread owns one row and
-// keeps its running max/sum and its Top-K candidates (a column of a shared
-// array, so the 32 rows of a warp never share a bank).  Candidates arrive in
-// ascending block order, so a later candidate with an equal score is worse
-// and only a strictly larger score evicts the current worst entry.
+// keeps its running max/sum and its Top-K candidates (registers for K <= 32,
+// a shared-memory column otherwise) with replace-the-worst updates.
 //
 // Two score sources:
 //   * scores given: 32x32 score sub-tiles are staged through shared memory
@@ -50,93 +48,288 @@ struct SelParams {
     long long limit;
 };
 
-// Per-row selection state.  ts/tm point at this row's column of the shared
-// candidate arrays (element e of the column at offset e * kRows).
-struct RowSel {
+// Online log-sum-exp of a row's scores.
+struct RowLse {
     float mx, sum;
-    float* ts;
-    int* tm;
-    int K, cnt;
-    float worst_s;
-    int worst_m, worst_pos;
 };
 
-__device__ __forceinline__ void rescan_worst(RowSel& r) {
-    float ws = CUDART_INF_F;
-    int wm = -1, wp = 0;
-    for (int e = 0; e < r.K; ++e) {
-        const float s = r.ts[e * kRows];
-        const int m = r.tm[e * kRows];
-        if (s < ws || (s == ws && m > wm)) { ws = s; wm = m; wp = e; }
-    }
-    r.worst_s = ws;
-    r.worst_m = wm;
-    r.worst_pos = wp;
-}
-
-__device__ __forceinline__ void topk_push(RowSel& r, float s, int m) {
-    if (r.cnt < r.K) {
-        r.ts[r.cnt * kRows] = s;
-        r.tm[r.cnt * kRows] = m;
-        if (++r.cnt == r.K) rescan_worst(r);
-    } else if (s > r.worst_s) {
-        r.ts[r.worst_pos * kRows] = s;
-        r.tm[r.worst_pos * kRows] = m;
-        rescan_worst(r);
-    }
-}
-
-// Consumes 32 scores of blocks m0 .. m0+31; entries at or past C_i are ignored.
-__device__ __forceinline__ void row_consume32(RowSel& r, const float (&v)[32], int m0, int Ci) {
-    const int lim = Ci - m0;
-    if (lim <= 0) return;
+__device__ __forceinline__ void lse_update(RowLse& l, const float (&v)[32], int lim) {
     float cm = -CUDART_INF_F;
 #pragma unroll
     for (int j = 0; j < 32; ++j)
         if (j < lim) cm = fmaxf(cm, v[j]);
-    const float nm = fmaxf(r.mx, cm);
+    const float nm = fmaxf(l.mx, cm);
     float acc = 0.f;
 #pragma unroll
     for (int j = 0; j < 32; ++j)
         if (j < lim) acc += fast_exp2((v[j] - nm) * kLog2e);
-    r.sum = r.sum * fast_exp2((r.mx - nm) * kLog2e) + acc;
-    r.mx = nm;
-    if (r.K > 0) {
+    l.sum = l.sum * fast_exp2((l.mx - nm) * kLog2e) + acc;
+    l.mx = nm;
+}
+
+// ---- Top-K for K <= 32: the kept (score, block) pairs live in registers.
+// Slot e holds block e while the row's first K blocks stream in, so a row
+// with C_i <= K never reorders anything.  Later blocks replace the current
+// worst entry (lowest score; among equal scores the highest block) when
+// strictly better: a later block with an equal score ranks below every kept
+// one because ties go to the lower block.  The work grows with the number of
+// replacements (about K ln(C_i / K) for scores in random order), not with C_i.
+struct RegTopK {
+    float s[32];
+    int m[32];
+    float ws;
+    int wm, wpos;
+    bool replaced;
+};
+
+__device__ __forceinline__ void reg_init(RegTopK& t) {
+    t.replaced = false;
+    t.ws = -CUDART_INF_F;
+    t.wm = 0;
+    t.wpos = 0;
+}
+
+__device__ __forceinline__ void reg_rescan(RegTopK& t, int K) {
+    float ws = CUDART_INF_F;
+    int wm = -1, wp = 0;
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (j < lim) topk_push(r, v[j], m0 + j);
+    for (int e = 0; e < 32; ++e) {
+        if (e < K && (t.s[e] < ws || (t.s[e] == ws && t.m[e] > wm))) {
+            ws = t.s[e];
+            wm = t.m[e];
+            wp = e;
+        }
+    }
+    t.ws = ws;
+    t.wm = wm;
+    t.wpos = wp;
+}
+
+__device__ __forceinline__ void reg_offer(RegTopK& t, float x, int idx, int K) {
+    if (x > t.ws) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+            if (e == t.wpos) {
+                t.s[e] = x;
+                t.m[e] = idx;
+            }
+        }
+        t.replaced = true;
+        reg_rescan(t, K);
     }
 }
 
-// Sorts the kept blocks by index, writes sel_idx / sel_logg for row i and
-// marks kept blocks below `diag` (= 2t) in the tile's union bitmap.
-__device__ __forceinline__ void row_finish(RowSel& r, const SelParams& p, long long row_off, int Ci, int diag,
-                                           uint32_t* bitmap) {
-    const int n = r.cnt;
-    const float lse = Ci > 0 ? r.mx + logf(r.sum) : 0.f;
+// Positions j (within a 32-block chunk) whose score beats `thr`; j < lim only.
+__device__ __forceinline__ uint32_t beats_mask(const float (&v)[32], int lo, int lim, float thr) {
+    uint32_t mask = 0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+        if (j >= lo && j < lim && v[j] > thr) mask |= 1u << j;
+    return mask;
+}
+
+// Consumes the scores of blocks 32c .. 32c+31 (entries at or past C_i ignored).
+// v holds them in registers; col[j * stride] holds the same values in shared
+// memory, read only for the few positions that can enter the Top-K.
+__device__ __forceinline__ void reg_consume(RegTopK& t, RowLse& l, const float (&v)[32], const float* col,
+                                            int stride, int c, int Ci, int K) {
+    const int lim = Ci - 32 * c;
+    if (lim <= 0) return;
+    lse_update(l, v, lim);
+    if (K == 0) return;
+    int lo = 0;
+    if (c == 0) {
+        const int nf = min(K, lim);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            // unused slots carry the largest block index so that sorting sinks them
+            t.s[j] = j < nf ? v[j] : CUDART_INF_F;
+            t.m[j] = j < nf ? j : 0x7fffffff;
+        }
+        if (Ci <= K) return;
+        reg_rescan(t, K);
+        lo = K;
+    }
+    // The threshold only rises while the chunk is consumed, so this mask is a
+    // superset of the entries that will actually replace one.
+    uint32_t mask = beats_mask(v, lo, lim, t.ws);
+    while (mask) {
+        const int j = __ffs(mask) - 1;
+        mask &= mask - 1;
+        reg_offer(t, col[j * stride], 32 * c + j, K);
+    }
+}
+
+// Sorts the kept entries by block index (bitonic network; empty slots carry
+// the largest index and sink to the end).
+__device__ __forceinline__ void reg_sort_by_block(RegTopK& t) {
+#pragma unroll
+    for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int l = i ^ j;
+                if (l > i) {
+                    const bool up = (i & k) == 0;
+                    const bool sw = up ? (t.m[i] > t.m[l]) : (t.m[i] < t.m[l]);
+                    const float si = t.s[i], sl = t.s[l];
+                    const int mi = t.m[i], ml = t.m[l];
+                    t.s[i] = sw ? sl : si;
+                    t.s[l] = sw ? si : sl;
+                    t.m[i] = sw ? ml : mi;
+                    t.m[l] = sw ? mi : ml;
+                }
+            }
+        }
+    }
+}
+
+// ---- Top-K for 32 < K <= 128: the kept pairs live in a shared-memory column
+// of this row (element e at offset e * kRows, so a warp's rows use distinct
+// banks), with the same fill / replace rule.
+struct SmemTopK {
+    float* s;
+    int* m;
+    float ws;
+    int wm, wpos;
+    bool replaced;
+};
+
+__device__ __forceinline__ void smem_rescan(SmemTopK& t, int K) {
+    float ws = CUDART_INF_F;
+    int wm = -1, wp = 0;
+#pragma unroll 8
+    for (int e = 0; e < K; ++e) {
+        const float se = t.s[e * kRows];
+        const int me = t.m[e * kRows];
+        if (se < ws || (se == ws && me > wm)) {
+            ws = se;
+            wm = me;
+            wp = e;
+        }
+    }
+    t.ws = ws;
+    t.wm = wm;
+    t.wpos = wp;
+}
+
+__device__ __forceinline__ void smem_consume(SmemTopK& t, RowLse& l, const float (&v)[32], const float* col,
+                                             int stride, int c, int Ci, int K) {
+    const int lim = Ci - 32 * c;
+    if (lim <= 0) return;
+    lse_update(l, v, lim);
+    const int m0 = 32 * c;
+    // fill: the row's first K blocks take slots 0 .. K-1 in order
+    const int nfill = min(lim, K - m0);
+    for (int j = 0; j < nfill; ++j) {
+        t.s[(m0 + j) * kRows] = col[j * stride];
+        t.m[(m0 + j) * kRows] = m0 + j;
+    }
+    if (Ci <= K || m0 + 32 <= K - 1) return;
+    int lo = 0;
+    if (m0 < K) {
+        smem_rescan(t, K);
+        lo = K - m0;
+    }
+    uint32_t mask = beats_mask(v, lo, lim, t.ws);
+    while (mask) {
+        const int j = __ffs(mask) - 1;
+        mask &= mask - 1;
+        const float x = col[j * stride];
+        if (x > t.ws) {
+            t.s[t.wpos * kRows] = x;
+            t.m[t.wpos * kRows] = m0 + j;
+            t.replaced = true;
+            smem_rescan(t, K);
+        }
+    }
+}
+
+__device__ __forceinline__ void smem_sort_by_block(SmemTopK& t, int n) {
     for (int a = 1; a < n; ++a) {
-        const int km = r.tm[a * kRows];
-        const float ks = r.ts[a * kRows];
+        const int km = t.m[a * kRows];
+        const float ks = t.s[a * kRows];
         int b = a - 1;
-        while (b >= 0 && r.tm[b * kRows] > km) {
-            r.tm[(b + 1) * kRows] = r.tm[b * kRows];
-            r.ts[(b + 1) * kRows] = r.ts[b * kRows];
+        while (b >= 0 && t.m[b * kRows] > km) {
+            t.m[(b + 1) * kRows] = t.m[b * kRows];
+            t.s[(b + 1) * kRows] = t.s[b * kRows];
             --b;
         }
-        r.tm[(b + 1) * kRows] = km;
-        r.ts[(b + 1) * kRows] = ks;
+        t.m[(b + 1) * kRows] = km;
+        t.s[(b + 1) * kRows] = ks;
     }
-    int32_t* oi = p.sel_idx + row_off * p.topk;
-    float* ol = p.sel_logg + row_off * p.topk;
-    for (int e = 0; e < p.topk; ++e) {
+}
+
+// Output staging: each row's K entries are written to shared memory (row
+// stride K + 1 words, so a warp's rows hit distinct banks) and then copied to
+// global memory with coalesced stores.
+struct Staging {
+    int32_t* idx;
+    float* lg;
+    int stride;
+};
+
+__device__ __forceinline__ void stage_entry(const Staging& st, int r, int e, int m, float lg) {
+    st.idx[r * st.stride + e] = m;
+    st.lg[r * st.stride + e] = lg;
+}
+
+// Copies the staged rows of tile t to sel_idx / sel_logg (rows >= N skipped).
+// Consecutive threads take consecutive entries of a row, so stores coalesce.
+__device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, int bh, int t, int tid, int nthreads) {
+    const int K = p.topk;
+    if (K == 0) return;
+    const int rows = min(kRows, p.N - t * kRows);
+    const long long base = (static_cast<long long>(bh) * p.N + static_cast<long long>(t) * kRows) * K;
+    int r = tid / K, e = tid - r * K;
+    const int dr = nthreads / K, de = nthreads - dr * K;
+    for (int q = tid; q < rows * K; q += nthreads) {
+        p.sel_idx[base + q] = st.idx[r * st.stride + e];
+        p.sel_logg[base + q] = st.lg[r * st.stride + e];
+        r += dr;
+        e += de;
+        if (e >= K) {
+            e -= K;
+            ++r;
+        }
+    }
+}
+
+// Finishes one row: log-gates, ascending order, staging, tile-union bits.
+template <class TK>
+__device__ __forceinline__ void row_emit(TK& t, const RowLse& l, const Staging& st, int r, int Ci, int K, int diag,
+                                         uint32_t* bitmap);
+
+template <>
+__device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, const Staging& st, int r, int Ci,
+                                                  int K, int diag, uint32_t* bitmap) {
+    const int n = min(K, Ci);
+    const float lse = Ci > 0 ? l.mx + logf(l.sum) : 0.f;
+    if (t.replaced) reg_sort_by_block(t);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+        if (e < K) {
+            const bool kept = e < n;
+            stage_entry(st, r, e, kept ? t.m[e] : -1, kept ? t.s[e] - lse : 0.f);
+            if (kept && t.m[e] < diag) atomicOr(&bitmap[t.m[e] >> 5], 1u << (t.m[e] & 31));
+        }
+    }
+}
+
+template <>
+__device__ __forceinline__ void row_emit<SmemTopK>(SmemTopK& t, const RowLse& l, const Staging& st, int r, int Ci,
+                                                   int K, int diag, uint32_t* bitmap) {
+    const int n = min(K, Ci);
+    const float lse = Ci > 0 ? l.mx + logf(l.sum) : 0.f;
+    if (t.replaced) smem_sort_by_block(t, n);
+    for (int e = 0; e < K; ++e) {
         if (e < n) {
-            const int m = r.tm[e * kRows];
-            oi[e] = m;
-            ol[e] = r.ts[e * kRows] - lse;
+            const int m = t.m[e * kRows];
+            stage_entry(st, r, e, m, t.s[e * kRows] - lse);
             if (m < diag) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
         } else {
-            oi[e] = -1;
-            ol[e] = 0.f;
+            stage_entry(st, r, e, -1, 0.f);
         }
     }
 }
@@ -167,9 +360,15 @@ __device__ __forceinline__ void compact_union(const uint32_t* bitmap, int diag, 
     if (lane == 0) *out_cnt = base;
 }
 
+// Shared-memory plan of the per-row state and outputs (bytes).
+__host__ __device__ constexpr size_t smem_topk_bytes(int K) { return K > 32 ? size_t(K) * kRows * 8 : 0; }
+__host__ __device__ constexpr size_t staging_bytes(int K) { return size_t(kRows) * (K + 1) * 8; }
+__host__ __device__ constexpr size_t bitmap_bytes(int C) { return size_t((C + 31) / 32) * 4; }
+
 // ------------------------------------------------------------ scores given
 
-__global__ void __launch_bounds__(128) select_given_kernel(SelParams p) {
+template <bool REG>
+__global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ float stage[4][32][33];
 
@@ -181,22 +380,34 @@ __global__ void __launch_bounds__(128) select_given_kernel(SelParams p) {
     const bool valid = i < p.N;
     const int Ci = valid ? (i >> 6) : 0;
     const int diag = 2 * t;
+    const int K = p.topk;
 
-    float* ts = reinterpret_cast<float*>(dsm);
-    int* tm = reinterpret_cast<int*>(ts + p.topk * kRows);
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(tm + p.topk * kRows);
+    uint8_t* ptr = dsm;
+    SmemTopK stk{};
+    if constexpr (!REG) {
+        stk.s = reinterpret_cast<float*>(ptr) + r;
+        stk.m = reinterpret_cast<int*>(ptr + size_t(K) * kRows * 4) + r;
+        stk.ws = -CUDART_INF_F;
+        ptr += smem_topk_bytes(K);
+    }
+    const Staging st{reinterpret_cast<int32_t*>(ptr), reinterpret_cast<float*>(ptr + size_t(kRows) * (K + 1) * 4),
+                     K + 1};
+    ptr += staging_bytes(K);
+    uint32_t* bitmap = reinterpret_cast<uint32_t*>(ptr);
     const int nwords = (p.C + 31) >> 5;
     for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
     __syncthreads();
 
-    RowSel rs{-CUDART_INF_F, 0.f, ts + r, tm + r, p.topk, 0, 0.f, 0, 0};
+    RegTopK rtk;
+    reg_init(rtk);
+    RowLse lse{-CUDART_INF_F, 0.f};
 
     const int row0 = t * kRows + warp * 32;
     const int last = min(row0 + 31, p.N - 1);
     const int Cw = row0 < p.N ? (last >> 6) : 0;   // largest C_i among the warp's rows
     const float* sbase = p.scores + static_cast<long long>(bh) * p.N * p.C;
-    for (int m0 = 0; m0 < Cw; m0 += 32) {
-        const int m = m0 + lane;
+    for (int c = 0; 32 * c < Cw; ++c) {
+        const int m = 32 * c + lane;
 #pragma unroll 4
         for (int rho = 0; rho < 32; ++rho) {
             const int row = row0 + rho;
@@ -207,12 +418,21 @@ __global__ void __launch_bounds__(128) select_given_kernel(SelParams p) {
         __syncwarp();
         float v[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = stage[warp][j][lane] * p.score_scale;
+        for (int j = 0; j < 32; ++j) {
+            v[j] = stage[warp][j][lane] * p.score_scale;
+            stage[warp][j][lane] = v[j];
+        }
+        const float* col = &stage[warp][0][lane];
+        if constexpr (REG) reg_consume(rtk, lse, v, col, 33, c, Ci, K);
+        else smem_consume(stk, lse, v, col, 33, c, Ci, K);
         __syncwarp();
-        row_consume32(rs, v, m0, Ci);
     }
-    if (valid) row_finish(rs, p, static_cast<long long>(bh) * p.N + i, Ci, diag, bitmap);
+    if (valid) {
+        if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap);
+        else row_emit(stk, lse, st, r, Ci, K, diag, bitmap);
+    }
     __syncthreads();
+    copy_out(st, p, bh, t, threadIdx.x, 128);
     if (warp == 0)
         compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
                       p.union_cnt + static_cast<long long>(bh) * p.T + t);
@@ -228,8 +448,16 @@ struct SelProjCfg {
     static constexpr uint32_t IDESC = idesc_bf16(kRows, 64, 0, 0);
 };
 
+// Dynamic shared memory: [operand tiles, later reused for output staging]
+// [Top-K columns when K > 32] [current 32 scores of each row] [tile-union bitmap].
+constexpr size_t kValuesBytes = size_t(32) * kRows * 4;
 template <int DS>
-__global__ void __launch_bounds__(192, 1)
+__host__ __device__ constexpr size_t proj_region0(int K) {
+    return SelProjCfg<DS>::TILE_BYTES > staging_bytes(K) ? size_t(SelProjCfg<DS>::TILE_BYTES) : staging_bytes(K);
+}
+
+template <int DS, bool REG>
+__global__ void __launch_bounds__(192, 2)
 select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_constant__ CUtensorMap mapKt, SelParams p) {
     using Cfg = SelProjCfg<DS>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -240,11 +468,12 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     const uint32_t warp = warp_id(), lane = lane_id();
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
+    const int K = p.topk;
     uint8_t* q_s = smem;
     uint8_t* kc_s = smem + Cfg::Q_BYTES;
-    float* ts = reinterpret_cast<float*>(smem + Cfg::TILE_BYTES);
-    int* tm = reinterpret_cast<int*>(ts + p.topk * kRows);
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(tm + p.topk * kRows);
+    uint8_t* topk_s = smem + proj_region0<DS>(K);
+    float* values_s = reinterpret_cast<float*>(topk_s + smem_topk_bytes(K));
+    uint32_t* bitmap = reinterpret_cast<uint32_t*>(topk_s + smem_topk_bytes(K) + kValuesBytes);
 
     const int t = p.T - 1 - static_cast<int>(blockIdx.x);
     const int bh = blockIdx.y;
@@ -332,28 +561,51 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
         const int i = t * kRows + r;
         const bool valid = i < p.N;
         const int Ci = valid ? (i >> 6) : 0;
-        RowSel rs{-CUDART_INF_F, 0.f, ts + r, tm + r, p.topk, 0, 0.f, 0, 0};
+        RegTopK rtk;
+        reg_init(rtk);
+        SmemTopK stk{};
+        if constexpr (!REG) {
+            stk.s = reinterpret_cast<float*>(topk_s) + r;
+            stk.m = reinterpret_cast<int*>(topk_s + size_t(K) * kRows * 4) + r;
+            stk.ws = -CUDART_INF_F;
+        }
+        RowLse lse{-CUDART_INF_F, 0.f};
+        float* vcol = values_s + r;   // this row's current 32 scores, element j at j * kRows
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         for (int c = 0; c < nchunks; ++c) {
             const int b = c & 1;
             if (!mbar_wait_warp(&s_full[b], (c >> 1) & 1, wc)) break;
             tc_fence_after();
-            uint32_t u0[32], u1[32];
-            tmem_ld32(lane_addr + b * 64, u0);
-            tmem_ld32(lane_addr + b * 64 + 32, u1);
-            tmem_wait_ld();
-            tc_fence_before();
-            mbar_arrive(&s_free[b]);
-            float v[32];
+#pragma unroll 1
+            for (int half = 0; half < 2; ++half) {
+                uint32_t u[32];
+                tmem_ld32(lane_addr + b * 64 + half * 32, u);
+                tmem_wait_ld();
+                if (half == 1) {
+                    tc_fence_before();
+                    mbar_arrive(&s_free[b]);
+                }
+                float v[32];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(u0[j]) * p.score_scale;
-            row_consume32(rs, v, c * 64, Ci);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(u1[j]) * p.score_scale;
-            row_consume32(rs, v, c * 64 + 32, Ci);
+                for (int j = 0; j < 32; ++j) {
+                    v[j] = __uint_as_float(u[j]) * p.score_scale;
+                    vcol[j * kRows] = v[j];
+                }
+                if constexpr (REG) reg_consume(rtk, lse, v, vcol, kRows, 2 * c + half, Ci, K);
+                else smem_consume(stk, lse, v, vcol, kRows, 2 * c + half, Ci, K);
+            }
         }
-        if (valid && !abort_flag) row_finish(rs, p, static_cast<long long>(bh) * p.N + i, Ci, diag, bitmap);
+        // Every score MMA has completed once the last chunk was read, so the
+        // operand tiles are free and become the output staging area.
+        const Staging st{reinterpret_cast<int32_t*>(smem),
+                         reinterpret_cast<float*>(smem + size_t(kRows) * (K + 1) * 4), K + 1};
+        const bool ok = !abort_flag;
+        if (valid && ok) {
+            if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap);
+            else row_emit(stk, lse, st, r, Ci, K, diag, bitmap);
+        }
         named_bar_sync(1, 128);
+        if (ok) copy_out(st, p, bh, t, static_cast<int>(threadIdx.x) - 64, 128);
         if (warp == 2)
             compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
                           p.union_cnt + static_cast<long long>(bh) * p.T + t);
@@ -365,20 +617,32 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     }
 }
 
-template <int DS>
-cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, size_t extra, const KernelEnv& env,
-                        const char** err) {
-    using Cfg = SelProjCfg<DS>;
-    const size_t smem = 1024 + Cfg::TILE_BYTES + extra;
+template <int DS, bool REG>
+cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
+    const size_t smem = 1024 + proj_region0<DS>(a.topk) + smem_topk_bytes(a.topk) + kValuesBytes + bitmap_bytes(a.C);
     if (smem > 227 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = cudaFuncSetAttribute(select_proj_kernel<DS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(select_proj_kernel<DS, REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mk;
     if (make_tmap_bf16_3d(&mq, a.Qt, DS, a.N, a.BH, 64, kRows) != 0) { *err = "tensor map Qt"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
     dim3 grid(a.T, a.BH);
-    select_proj_kernel<DS><<<grid, 192, smem, env.stream>>>(mq, mk, p);
+    select_proj_kernel<DS, REG><<<grid, 192, smem, env.stream>>>(mq, mk, p);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) *err = "select launch";
+    return e;
+}
+
+template <bool REG>
+cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
+    const size_t smem = smem_topk_bytes(a.topk) + staging_bytes(a.topk) + bitmap_bytes(a.C);
+    if (smem > 200 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
+    cudaError_t e = cudaFuncSetAttribute(select_given_kernel<REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select_given)"; return e; }
+    dim3 grid(a.T, a.BH);
+    select_given_kernel<REG><<<grid, 128, smem, env.stream>>>(p);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;
@@ -394,20 +658,10 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     p.sel_idx = a.sel_idx; p.sel_logg = a.sel_logg;
     p.union_idx = a.union_idx; p.union_cnt = a.union_cnt;
     p.status = env.status; p.limit = env.limit;
-    const size_t extra = static_cast<size_t>(a.topk) * kRows * 8 + static_cast<size_t>((a.C + 31) / 32) * 4;
-    if (a.scores != nullptr) {
-        if (extra > 180 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-        cudaError_t e = cudaFuncSetAttribute(select_given_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(extra));
-        if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select_given)"; return e; }
-        dim3 grid(a.T, a.BH);
-        select_given_kernel<<<grid, 128, extra, env.stream>>>(p);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) *err = "select launch";
-        return e;
-    }
-    if (a.d_sel == 128) return launch_proj<128>(a, p, extra, env, err);
-    if (a.d_sel == 64) return launch_proj<64>(a, p, extra, env, err);
+    const bool reg = a.topk <= 32;
+    if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
+    if (a.d_sel == 128) return reg ? launch_proj<128, true>(a, p, env, err) : launch_proj<128, false>(a, p, env, err);
+    if (a.d_sel == 64) return reg ? launch_proj<64, true>(a, p, env, err) : launch_proj<64, false>(a, p, env, err);
     *err = "selection: unsupported d_sel";
     return cudaErrorInvalidValue;
 }

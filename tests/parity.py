@@ -84,9 +84,10 @@ def _flip_size(x, delta):
     return np.where(dist_to_mid <= delta, 2 * step, 0.0)
 
 
-def selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel):
+def selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel, rows=None):
     """Per-row bound on |s_gpu - s_oracle| over the row's history, times two
-    (the K-th and the (K+1)-th score may both move).
+    (the K-th and the (K+1)-th score may both move).  Returned for `rows`
+    (default: all rows).
 
     The learned selector computes q~ = bf16(Wq q) and K~ = bf16(Wk mean(K_B))
     with fp32 accumulation (at most 128 terms, error <= 2^-17 of the sum of
@@ -95,6 +96,8 @@ def selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel):
     its exact value sits within that accumulation error of a rounding midpoint.
     """
     q, k, wq, wk = f64(Q[bi, hi]), f64(K[bi, hi]), f64(Wq[hi]), f64(Wk[hi])
+    rows = np.arange(q.shape[0]) if rows is None else np.asarray(rows)
+    q = q[rows]
     qe = q @ wq.T
     dq = 2.0 ** -17 * (np.abs(q) @ np.abs(wq).T)
     kbar = OR.block_summaries(k, 64)
@@ -103,15 +106,14 @@ def selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel):
     fq, fk = _flip_size(qe, dq), _flip_size(ke, dk)
     qt, kt = np.abs(OR.round_to_bf16(qe)), np.abs(OR.round_to_bf16(ke))
     if kt.shape[0] == 0:
-        return np.full(q.shape[0], 1e-30)
+        return np.full(len(rows), 1e-30)
     bound = (fq @ kt.T + qt @ fk.T + fq @ fk.T + 2.0 ** -17 * (qt @ kt.T)) / np.sqrt(d_sel)
     bound += 2.0 ** -22 * np.abs(OR.round_to_bf16(qe) @ OR.round_to_bf16(ke).T) / np.sqrt(d_sel)
-    N = q.shape[0]
-    tol = np.zeros(N)
-    for i in range(N):
-        c = i // 64
+    tol = np.zeros(len(rows))
+    for r, i in enumerate(rows):
+        c = int(i) // 64
         if c > 0:
-            tol[i] = 2 * bound[i, :c].max()
+            tol[r] = 2 * bound[r, :c].max()
     return tol + 1e-30
 
 

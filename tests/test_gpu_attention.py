@@ -90,7 +90,7 @@ def _learned_case(B, H, N, d, topk, mode=TRAIN, d_sel=0, seed=0, heads=None, row
         s = P.oracle_scores(Q, K, Wq, Wk, bi, hi)
         ref = OR.sas_attention_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s, 64, topk, mode,
                                     rows=rr)
-        tol = None if exact_inputs else P.selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel)[rr]
+        tol = None if exact_inputs else P.selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel, rows=rr)
         gi = g["sel_idx"][bi, hi].numpy()[rr][:, :topk]
         exact, near, mism = P.check_selection_rows(gi, s[rr], rr, topk, tol)
         total_mismatch += int(mism.sum())
@@ -131,6 +131,17 @@ def test_full_size_dit_layer_sampled():
     # the benchmark workload: B=2, H=24, N=4096+512, d=128, K=32, learned selector
     N = 4608
     _learned_case(2, 24, N, 128, 32, heads=[(0, 0), (1, 23)], rows=P.sample_rows(N))
+
+
+def test_video_scale_learned_selector_sampled():
+    # video-scale layer: B=1, H=24, N=75600+512 (last block holds 16 tokens), K=32
+    N = 75600 + 512
+    _learned_case(1, 24, N, 128, 32, heads=[(0, 0), (0, 13)], rows=P.sample_rows(N, n_random=512), seed=21)
+
+
+def test_hires_learned_selector_sampled():
+    N = 16384 + 512
+    _learned_case(1, 24, N, 128, 32, heads=[(0, 5), (0, 23)], rows=P.sample_rows(N), seed=22)
 
 
 @pytest.mark.parametrize("topk", [16, 32, 64])
