@@ -164,8 +164,10 @@ const char* sas_status_str(sas_status s);
 /* Text of the last error recorded on this handle ("" if none). */
 const char* sas_last_error(const sas_handle* h);
 
-/* Reads and clears the device status word (SAS_OK or SAS_ERR_TIMEOUT).
- * Synchronises the device first. */
+/* Reads and clears the device status word: SAS_OK, SAS_ERR_TIMEOUT (a
+ * bounded wait ran out) or SAS_ERR_CUDA (a kernel found its shared memory
+ * not 1024-byte aligned and returned without computing).  Synchronises the
+ * device first. */
 sas_status sas_get_device_status(sas_handle* h, int32_t* out_status);
 
 /* Per-kernel timing with CUDA events recorded on the launch stream around

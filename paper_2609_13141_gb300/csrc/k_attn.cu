@@ -40,18 +40,30 @@ template <int D>
 struct AttnCfg {
     static constexpr int Q_BYTES = kBM * D * 2;
     static constexpr int KV_BYTES = kBN * D * 2;
-    static constexpr int P_BYTES = kBM * kBN * 2;
     static constexpr int KST = 2;
-    static constexpr int VST = 1;
+    static constexpr int VST = 2;
     static constexpr int OFF_K = Q_BYTES;
     static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-    static constexpr int OFF_P = OFF_V + VST * KV_BYTES;
-    static constexpr int SMEM = OFF_P + P_BYTES + 1024;
+    static constexpr int OFF_CTL = OFF_V + VST * KV_BYTES;
+    // All shared state lives in the dynamic region (no static shared memory),
+    // so that two CTAs fit on one SM.
+    static constexpr int SMEM = OFF_CTL + 256;
     static constexpr int TMEM_COLS = 256;    // S0 [0,64) S1 [64,128) O [128,128+D)
     static constexpr int TMEM_O = 128;
     static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, 0, 0);
     static constexpr uint32_t IDESC_O = idesc_bf16(kBM, D, 0, 1);
 };
+
+// Barriers and flags at the end of the dynamic shared-memory region.
+struct AttnCtl {
+    uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2];
+    uint64_t s_full[2], s_free[2], p_full[2], o_ready[2], drain_bar;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+static_assert(sizeof(AttnCtl) <= 256, "control block");
+
+constexpr int kStatusLayout = 3;   // == SAS_ERR_CUDA: shared-memory base not 1024-byte aligned
 
 struct AttnParams {
     bf16* O;
@@ -75,15 +87,27 @@ __global__ void __launch_bounds__(kThreads, 2)
 attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
             const __grid_constant__ CUtensorMap mapV, AttnParams p) {
     using Cfg = AttnCfg<D>;
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
-    __shared__ uint64_t q_full, k_full[Cfg::KST], k_empty[Cfg::KST], v_full[Cfg::VST], v_empty[Cfg::VST];
-    __shared__ uint64_t s_full[2], s_free[2], p_full, o_ready, drain_bar;
-    __shared__ uint32_t tmem_base_sh;
-    __shared__ int abort_flag;
+    extern __shared__ __align__(1024) uint8_t smem[];
+    if ((smem_u32(smem) & 1023u) != 0) {
+        // The 128-byte swizzle atoms need 1024-byte alignment; report, never fault.
+        if (threadIdx.x == 0) atomicExch(p.status, kStatusLayout);
+        return;
+    }
+    AttnCtl& ctl = *reinterpret_cast<AttnCtl*>(smem + Cfg::OFF_CTL);
+    uint64_t& q_full = ctl.q_full;
+    uint64_t* k_full = ctl.k_full;
+    uint64_t* k_empty = ctl.k_empty;
+    uint64_t* v_full = ctl.v_full;
+    uint64_t* v_empty = ctl.v_empty;
+    uint64_t* s_full = ctl.s_full;
+    uint64_t* s_free = ctl.s_free;
+    uint64_t* p_full = ctl.p_full;
+    uint64_t* o_ready = ctl.o_ready;
+    uint64_t& drain_bar = ctl.drain_bar;
+    uint32_t& tmem_base_sh = ctl.tmem_base;
+    int& abort_flag = ctl.abort_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
-    const uint32_t raw = smem_u32(smem_raw);
-    uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
 
     const int t = p.T - 1 - static_cast<int>(blockIdx.x);   // heavy tiles first
     const int bh = blockIdx.y;
@@ -96,9 +120,12 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         mbar_init(&q_full, 1);
         for (int s = 0; s < Cfg::KST; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
         for (int s = 0; s < Cfg::VST; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
-        for (int s = 0; s < 2; ++s) { mbar_init(&s_full[s], 1); mbar_init(&s_free[s], 4); }
-        mbar_init(&p_full, 4);
-        mbar_init(&o_ready, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_free[s], 1);
+            mbar_init(&o_ready[s], 1);
+            mbar_init(&p_full[s], 4);
+        }
         mbar_init(&drain_bar, 1);
         abort_flag = 0;
         fence_barrier_init();
@@ -158,7 +185,6 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     } else if (warp == 2 && lane == 0) {
         // ---------------- MMA issuer
         const uint32_t q_addr = smem_u32(smem);
-        const uint32_t p_addr = smem_u32(smem + Cfg::OFF_P);
         bool ok = mbar_wait(&q_full, 0, wc);
         for (int j = 0; ok && j <= n; ++j) {
             if (j < n) {
@@ -183,21 +209,24 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 // O += P_{j-1} V_{j-1}
                 const int jj = j - 1;
                 const int vs = jj % Cfg::VST;
-                if (!mbar_wait(&p_full, jj & 1, wc)) break;
+                // p_full[jj&1] cannot run two phases ahead: the softmax needs QK_{jj+2},
+                // issued only after this wait, before it can arrive there again.
+                if (!mbar_wait(&p_full[jj & 1], (jj >> 1) & 1, wc)) break;
                 if (!mbar_wait(&v_full[vs], (jj / Cfg::VST) & 1, wc)) break;
                 tc_fence_after();
                 const uint32_t v_addr = smem_u32(smem + Cfg::OFF_V + vs * Cfg::KV_BYTES);
 #pragma unroll
                 for (int k = 0; k < kBN / 16; ++k) {
-                    // P: K-major, 16 keys = 32 bytes along the swizzled row.
-                    // V: MN-major (d contiguous), 16 keys = two 8-row atoms;
-                    //    the two 64-wide d halves sit kBN*128 bytes apart.
-                    umma_bf16(tmem_base + Cfg::TMEM_O, smem_desc_sw128(p_addr + k * 32, 16, 1024),
-                              smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
-                              (jj > 0 || k > 0) ? 1u : 0u);
+                    // P_{jj} sits in TMEM over the first 32 columns of score buffer jj & 1
+                    // (16 keys = 8 packed columns per step).  V is MN-major (d contiguous):
+                    // 16 keys = two 8-row atoms; the two 64-wide d halves sit kBN*128 bytes apart.
+                    umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + (jj & 1) * 64 + k * 8,
+                                 smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
+                                 (jj > 0 || k > 0) ? 1u : 0u);
                 }
-                umma_commit(&o_ready);
+                umma_commit(&o_ready[jj & 1]);
                 umma_commit(&v_empty[vs]);
+                umma_commit(&s_free[jj & 1]);   // score buffer (and P in it) free for QK_{jj+2}
             }
         }
         umma_commit(&drain_bar);
@@ -222,8 +251,6 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         float kl1 = nsel > 1 ? __ldg(my_lg + 1) : 0.f;
 
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-        uint8_t* p_row = smem + Cfg::OFF_P + r * 128;
-        const int sw = r & 7;
         const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2);
 
         float m_use = -CUDART_INF_F;
@@ -271,22 +298,23 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                     x[k + 32] = __uint_as_float(u1[k]);
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_free[sb]);
-
             bool need = false;
             float m_new = m_use;
             float rs = 0.f;
+            uint32_t pk[32];   // P row as packed bf16 pairs
             if (warp_active) {
                 // causal mask on the diagonal block only
                 if (__any_sync(0xffffffffu, lim >= 0 && lim < kBN - 1)) {
 #pragma unroll
                     for (int k = 0; k < 64; ++k) x[k] = k <= lim ? x[k] : -CUDART_INF_F;
                 }
-                float mx = -CUDART_INF_F;
+                float mx0 = -CUDART_INF_F, mx1 = -CUDART_INF_F;
 #pragma unroll
-                for (int k = 0; k < 64; k += 2) mx = max3f(mx, x[k], x[k + 1]);
+                for (int k = 0; k < 64; k += 4) {
+                    mx0 = max3f(mx0, x[k], x[k + 1]);
+                    mx1 = max3f(mx1, x[k + 2], x[k + 3]);
+                }
+                const float mx = fmaxf(mx0, mx1);
                 // max of the gated logits (log2 units): the gate is constant over the block
                 const float mb = active ? fmaf(mx, p.scale_log2, bias) : -CUDART_INF_F;
                 need = mb > m_use + kRescaleThreshold;
@@ -299,9 +327,9 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 for (int k = 0; k < 64; k += 2) {
                     float a0, a1;
                     f32x2_split(fma_f32x2(f32x2(x[k], x[k + 1]), scale2, off2), a0, a1);
-                    x[k] = fast_exp2(a0);
-                    x[k + 1] = fast_exp2(a1);
-                    acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(x[k], x[k + 1]));
+                    const float e0 = fast_exp2(a0), e1 = fast_exp2(a1);
+                    acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(e0, e1));
+                    pk[k >> 1] = pack_bf16x2(e0, e1);
                 }
                 float s0, s1, s2, s3, s4, s5, s6, s7;
                 f32x2_split(acc[0], s0, s1);
@@ -309,15 +337,19 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 f32x2_split(acc[2], s4, s5);
                 f32x2_split(acc[3], s6, s7);
                 rs = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+            } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) pk[k] = 0u;
             }
             float factor = 1.f;
             if (need) factor = m_use == -CUDART_INF_F ? 0.f : fast_exp2(m_use - m_new);
 
-            if (j > 0) {
-                // PV_{j-1} must be done before P is overwritten and O rescaled.
-                if (!mbar_wait_warp(&o_ready, (j - 1) & 1, wc)) { ok = false; break; }
+            if (j > 0 && __any_sync(0xffffffffu, need)) {
+                // Rescaling O needs PV_{j-1} done.  PV_{j-1} is the ((j-1)/2)-th phase of
+                // o_ready[(j-1)&1]; that barrier cannot move past it before p_full(j+1).
+                if (!mbar_wait_warp(&o_ready[(j - 1) & 1], ((j - 1) >> 1) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, need)) {
+                {
 #pragma unroll 1
                     for (int cc = 0; cc < D / 32; ++cc) {
                         uint32_t o[32];
@@ -333,29 +365,15 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             l = l * factor + rs;
             m_use = m_new;
 
-            // P row (64 bf16 = 8 chunks of 16 bytes), 128-byte swizzle: chunk k at k ^ (row & 7)
-            if (warp_active) {
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    uint4 w;
-                    w.x = pack_bf16x2(x[8 * k + 0], x[8 * k + 1]);
-                    w.y = pack_bf16x2(x[8 * k + 2], x[8 * k + 3]);
-                    w.z = pack_bf16x2(x[8 * k + 4], x[8 * k + 5]);
-                    w.w = pack_bf16x2(x[8 * k + 6], x[8 * k + 7]);
-                    *reinterpret_cast<uint4*>(p_row + ((k ^ sw) << 4)) = w;
-                }
-            } else {
-                const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-                for (int k = 0; k < 8; ++k) *reinterpret_cast<uint4*>(p_row + (k << 4)) = z;
-            }
-            fence_proxy_async_smem();
+            // P row (64 bf16, packed in pairs) into TMEM over this row's scores
+            tmem_st32(lane_addr + sb * 64, pk);
+            tmem_wait_st();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&p_full);
+            if (lane == 0) mbar_arrive(&p_full[sb]);
         }
 
-        if (ok && mbar_wait_warp(&o_ready, (n - 1) & 1, wc)) {
+        if (ok && mbar_wait_warp(&o_ready[(n - 1) & 1], ((n - 1) >> 1) & 1, wc)) {
             tc_fence_after();
             const float inv = 1.f / l;
             bf16* orow = p.O + row_off * D;
