@@ -66,7 +66,7 @@ typedef enum { SAS_SEL_SCORES_GIVEN = 0, SAS_SEL_MEANPOOL_PROJ = 1 } sas_selecto
 typedef struct {
     int32_t B, H, N, d;   /* batch, heads, tokens, head dim (d in {64, 128})          */
     int32_t block;        /* block size b; must be 64 (Sec. 4.2.1 setup)             */
-    int32_t topk;         /* K historical blocks kept per query, 0 <= K <= 1024       */
+    int32_t topk;         /* K historical blocks kept per query, 0 <= K <= 64         */
     float sm_scale;       /* softmax scale on q.k; 0 selects 1/sqrt(d) (Alg. 3)       */
     int32_t mode;         /* sas_mode                                                 */
     int32_t selector;     /* sas_selector                                             */

@@ -220,8 +220,9 @@ __device__ __forceinline__ void smem_consume(SmemTopK& t, RowLse& l, const float
     if (lim <= 0) return;
     lse_update(l, v, lim);
     const int m0 = 32 * c;
-    // fill: the row's first K blocks take slots 0 .. K-1 in order
-    const int nfill = min(lim, K - m0);
+    // fill: the row's first K blocks take slots 0 .. K-1 in order (at most
+    // the 32 blocks of this chunk)
+    const int nfill = min(min(lim, 32), K - m0);
     for (int j = 0; j < nfill; ++j) {
         t.s[(m0 + j) * kRows] = col[j * stride];
         t.m[(m0 + j) * kRows] = m0 + j;
@@ -312,7 +313,8 @@ __device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, c
         if (e < K) {
             const bool kept = e < n;
             stage_entry(st, r, e, kept ? t.m[e] : -1, kept ? t.s[e] - lse : 0.f);
-            if (kept && t.m[e] < diag) atomicOr(&bitmap[t.m[e] >> 5], 1u << (t.m[e] & 31));
+            if (kept && static_cast<unsigned>(t.m[e]) < static_cast<unsigned>(diag))
+                atomicOr(&bitmap[t.m[e] >> 5], 1u << (t.m[e] & 31));
         }
     }
 }
@@ -327,7 +329,7 @@ __device__ __forceinline__ void row_emit<SmemTopK>(SmemTopK& t, const RowLse& l,
         if (e < n) {
             const int m = t.m[e * kRows];
             stage_entry(st, r, e, m, t.s[e * kRows] - lse);
-            if (m < diag) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
+            if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
         } else {
             stage_entry(st, r, e, -1, 0.f);
         }

@@ -202,7 +202,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (c.block != 64) return SAS_ERR_UNSUPPORTED;
     if (c.d != 64 && c.d != 128) return SAS_ERR_UNSUPPORTED;
     if (c.topk < 0) return SAS_ERR_INVALID_ARG;
-    if (c.topk > 128) return SAS_ERR_UNSUPPORTED;
+    if (c.topk > 64) return SAS_ERR_UNSUPPORTED;
     if (c.mode != SAS_MODE_TRAIN_SOFT && c.mode != SAS_MODE_INFER_HARD) return SAS_ERR_INVALID_ARG;
     if (c.selector != SAS_SEL_SCORES_GIVEN && c.selector != SAS_SEL_MEANPOOL_PROJ) return SAS_ERR_INVALID_ARG;
     if (!(c.sm_scale >= 0.f) || !std::isfinite(c.sm_scale)) return SAS_ERR_INVALID_ARG;

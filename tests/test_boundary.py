@@ -40,7 +40,7 @@ def test_status_strings(lib):
     (dict(B=1, H=1, N=128, d=96, topk=2), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=1, N=128, d=64, topk=2, block=32), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=1, N=128, d=64, topk=-1), sas.SAS_ERR_INVALID_ARG),
-    (dict(B=1, H=1, N=128, d=64, topk=129), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, H=1, N=128, d=64, topk=65), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=1, N=128, d=64, topk=2, mode=7), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=1, N=128, d=64, topk=2, selector=5), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=1, N=128, d=64, topk=2, d_sel=32), sas.SAS_ERR_UNSUPPORTED),

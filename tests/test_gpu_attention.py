@@ -127,6 +127,11 @@ def test_learned_selector_dsel64_with_d128():
     _learned_case(1, 1, 640, 128, 2, d_sel=64, seed=3)
 
 
+def test_learned_selector_k64_shared_memory_topk():
+    # K > 32 keeps the Top-K in shared memory; integer inputs make the kept sets exact
+    _learned_case(1, 2, 5000, 128, 64, exact_inputs=True, seed=13)
+
+
 def test_full_size_dit_layer_sampled():
     # the benchmark workload: B=2, H=24, N=4096+512, d=128, K=32, learned selector
     N = 4608
