@@ -130,16 +130,18 @@ class ClockSampler:
 # --------------------------------------------------------------- our arm
 
 def kernel_traffic(kind):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's
+    sources are unchanged since the capture (else None)."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
         return None
     rec = json.load(open(p)).get(kind)
     if not rec:
         return None
-    src = os.path.join(ROOT, "paper_2609_13141_gb300", "csrc", rec["source"])
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return rec["dram_bytes_per_launch"] if sha == rec["source_sha256_16"] else None
+    m = hashlib.sha256()
+    for f in rec["sources"]:
+        m.update(open(os.path.join(ROOT, "paper_2609_13141_gb300", "csrc", f), "rb").read())
+    return rec["dram_bytes_per_launch"] if m.hexdigest()[:16] == rec["sources_sha256_16"] else None
 
 
 def run_ours(args, w, rank, world):

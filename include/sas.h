@@ -75,8 +75,8 @@ typedef struct {
 
 typedef struct sas_handle sas_handle;
 
-/* Validates cfg, allocates the handle's device workspace (block summaries,
- * projected queries, per-tile block lists, internal selection buffers) on the
+/* Validates cfg, allocates the handle's device workspace (projected block
+ * summaries, per-tile block lists, internal selection buffers) on the
  * current device and returns the handle in *out.  Synchronous. */
 sas_status sas_create(const sas_config* cfg, sas_handle** out);
 
@@ -174,8 +174,9 @@ sas_status sas_get_device_status(sas_handle* h, int32_t* out_status);
  * every kernel.  sas_set_timing(h, 1) starts recording (and clears earlier
  * records); sas_get_timings synchronises, then writes, for each kernel kind,
  * the number of launches and the summed milliseconds.  Kinds, in order:
- * 0 block summaries, 1 query projection, 2 selection, 3 attention,
- * 4 MLP up-projection + GELU, 5 MLP down-projection.  n_kinds <= 6. */
+ * 0 block summaries, 1 (unused: the selector's query projection runs inside
+ * the selection kernel), 2 selection, 3 attention, 4 MLP up-projection +
+ * GELU, 5 MLP down-projection.  n_kinds <= 6. */
 #define SAS_NUM_KERNEL_KINDS 6
 sas_status sas_set_timing(sas_handle* h, int32_t enable);
 sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds);

@@ -24,7 +24,7 @@ struct KernelEnv {
     long long limit;    // bounded-wait budget in SM cycles
 };
 
-// ---- tcgen05 GEMM:  C[b] = epi(A[b] @ B[b % b_mod]^T (+ bias)), bf16 out.
+// ---- tcgen05 GEMM:  C[b] = epi(A[b] @ B[b % b_mod]^T (+ bias)), bf16 out (the MLP).
 // A: [batches][M][K], B: [nb][N][K], C: [batches][M][ldc] (row stride ldc).
 // N must be a multiple of bn (64, 128 or 256), K a multiple of 64.
 struct GemmProblem {
@@ -54,8 +54,10 @@ struct SelectArgs {
     int BH, H, N, C, T, topk, d_sel;
     float score_scale;              // 1/sqrt(d_sel) for projected scores, 1 for given scores
     const float* scores;            // SCORES_GIVEN: [BH][N][C]
-    const void* Qt;                 // MEANPOOL_PROJ: projected queries bf16 [BH][N][d_sel]
+    const void* Q;                  // MEANPOOL_PROJ: queries bf16 [BH][N][d]
+    const void* Wq;                 // MEANPOOL_PROJ: query projection bf16 [H][d_sel][d]
     const void* Kt;                 // MEANPOOL_PROJ: projected block summaries bf16 [BH][F][d_sel]
+    int d;
     int F;
     int32_t* sel_idx;               // [BH][N][topk]
     float* sel_logg;                // [BH][N][topk]

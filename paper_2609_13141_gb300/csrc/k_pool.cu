@@ -6,7 +6,7 @@
 // for the F = floor(N/64) full blocks of every (batch, head): a partial last
 // block is never historical for any query, so it is never summarised.  One
 // CTA handles 8 consecutive blocks of one head: warp w streams block w's 64
-// key rows with coalesced 8-byte loads (a warp covers one 256-byte row) and
+// key rows with coalesced 16-byte loads (sixteen in flight per lane) and
 // keeps fp32 column sums in registers; the CTA then projects the 8 summaries
 // with Wk[h] staged row-major in shared memory (rows padded by one word so
 // that the 32 threads of a warp, one output each, hit distinct banks).  The pass is HBM-bound: it
@@ -23,45 +23,64 @@ template <int D, int DS>
 __global__ void __launch_bounds__(256) pool_kernel(const bf16* __restrict__ K, const bf16* __restrict__ Wk,
                                                     bf16* __restrict__ Kt, int H, int N, int F) {
     __shared__ float kbar[kGroup][D];
-    __shared__ __align__(16) bf16 ws[DS][D + 2];   // ws[j][k] = Wk[h][j][k]
+    __shared__ __align__(16) bf16 ws[DS][D + 2];   // ws[j][k] = Wk[h][j][k]; rows 4-byte aligned
 
     const int bh = blockIdx.y;
     const int h = bh % H;
     const int m0 = blockIdx.x * kGroup;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+    // Wk[h] rows (D bf16 = D/8 16-byte pieces each) into the padded shared copy
     const bf16* w = Wk + static_cast<long long>(h) * DS * D;
-    for (int e = threadIdx.x; e < DS * D; e += blockDim.x) {
-        const int j = e / D, k = e - j * D;
-        ws[j][k] = w[e];
+    for (int e = threadIdx.x; e < DS * (D / 8); e += blockDim.x) {
+        const int j = e / (D / 8), k8 = (e - j * (D / 8)) * 8;
+        const uint4 u = __ldg(reinterpret_cast<const uint4*>(w + j * D + k8));
+        const uint32_t* uw = reinterpret_cast<const uint32_t*>(&u);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) *reinterpret_cast<uint32_t*>(&ws[j][k8 + 2 * q]) = uw[q];
     }
 
+    // Warp w sums block m0 + w.  A key row is D * 2 bytes: D / 8 lanes cover it
+    // with 16-byte loads, so one warp instruction reads LPR = 256 / D rows and
+    // each lane keeps fp32 sums of 8 dims over its rows.
     const int m = m0 + warp;
-    constexpr int PER = D / 32;
+    constexpr int LANES_PER_ROW = D / 8;
+    constexpr int ROWS_PER_STEP = 32 / LANES_PER_ROW;
     if (m < F) {
-        float acc[PER];
+        const int sub = lane / LANES_PER_ROW;            // which of the step's rows
+        const int dl = (lane % LANES_PER_ROW) * 8;       // first of this lane's 8 dims
+        float acc[8];
 #pragma unroll
-        for (int q = 0; q < PER; ++q) acc[q] = 0.f;
-        const bf16* base = K + (static_cast<long long>(bh) * N + static_cast<long long>(m) * 64) * D + lane * PER;
-#pragma unroll 4
-        for (int t = 0; t < 64; ++t) {
-            const bf16* rp = base + static_cast<long long>(t) * D;
-            if constexpr (PER == 4) {
-                const uint2 u = *reinterpret_cast<const uint2*>(rp);
-                const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
-                const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
-                acc[0] += __low2float(a);
-                acc[1] += __high2float(a);
-                acc[2] += __low2float(b);
-                acc[3] += __high2float(b);
-            } else {
-                const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(rp);
-                acc[0] += __low2float(a);
-                acc[1] += __high2float(a);
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        const bf16* base = K + (static_cast<long long>(bh) * N + static_cast<long long>(m) * 64 + sub) * D + dl;
+        // issue all of the lane's row loads before summing (16 in flight)
+        constexpr int STEPS = 64 / ROWS_PER_STEP;
+#pragma unroll
+        for (int t0 = 0; t0 < STEPS; t0 += 16) {
+            uint4 u[16];
+#pragma unroll
+            for (int t = 0; t < 16; ++t)
+                u[t] = __ldg(reinterpret_cast<const uint4*>(base + static_cast<long long>(t0 + t) * ROWS_PER_STEP * D));
+#pragma unroll
+            for (int t = 0; t < 16; ++t) {
+                const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&u[t]);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    acc[2 * q] += __low2float(h2[q]);
+                    acc[2 * q + 1] += __high2float(h2[q]);
+                }
             }
         }
+        // fold the partial sums of the lanes that share dims
 #pragma unroll
-        for (int q = 0; q < PER; ++q) kbar[warp][lane * PER + q] = acc[q] * (1.0f / 64.0f);
+        for (int off = LANES_PER_ROW; off < 32; off <<= 1) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], off);
+        }
+        if (sub == 0) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) kbar[warp][dl + q] = acc[q] * (1.0f / 64.0f);
+        }
     }
     __syncthreads();
 

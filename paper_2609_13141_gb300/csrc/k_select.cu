@@ -20,11 +20,12 @@
 // Two score sources:
 //   * scores given: 32x32 score sub-tiles are staged through shared memory
 //     with coalesced 128-byte row loads;
-//   * learned selector: s = Qt Kt^T / sqrt(d_sel) is computed on the tensor
-//     cores -- TMA brings the tile's 128 projected queries once and 64-block
-//     chunks of projected block summaries in a double-buffered ring, one
-//     thread issues tcgen05.mma (M=128, N=64) into two TMEM buffers, and the
-//     row threads read their scores back with tcgen05.ld.
+//   * learned selector: on the tensor cores, one thread first projects the
+//     tile's 128 queries (q~ = Q Wq^T into TMEM); the row threads round q~
+//     to bf16 into shared memory as the A operand of the score product; then
+//     s = q~ Kt^T / sqrt(d_sel) runs chunk by chunk (M=128, N=64) over
+//     64-block chunks of projected summaries in a double-buffered TMA ring,
+//     and the row threads read their scores back with tcgen05.ld.
 #include <math_constants.h>
 
 #include "internal.h"
@@ -442,28 +443,39 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 
 // --------------------------------------------------------- learned selector
 
-template <int DS>
+// Shared memory of the learned-selector kernel (offsets from a 1024-aligned base):
+//   region A: the 128-row Q tile, overwritten by the bf16 projected queries q~;
+//   region B: the tile's Wq[h], then (once the projection has run) the
+//             double-buffered 64-block chunks of projected block summaries;
+//   after the last chunk, regions A and B hold the output staging;
+//   then the Top-K columns, the current 32 scores of each row, the union bitmap.
+template <int D, int DS>
 struct SelProjCfg {
-    static constexpr int Q_BYTES = kRows * DS * 2;
+    static constexpr int Q_BYTES = kRows * D * 2;
+    static constexpr int QT_BYTES = kRows * DS * 2;
+    static constexpr int A_BYTES = Q_BYTES > QT_BYTES ? Q_BYTES : QT_BYTES;
+    static constexpr int WQ_BYTES = DS * D * 2;
     static constexpr int KC_BYTES = 64 * DS * 2;   // 64 blocks per chunk
-    static constexpr int TILE_BYTES = Q_BYTES + 2 * KC_BYTES;
-    static constexpr uint32_t IDESC = idesc_bf16(kRows, 64, 0, 0);
+    static constexpr int B_BYTES = WQ_BYTES > 2 * KC_BYTES ? WQ_BYTES : 2 * KC_BYTES;
+    static constexpr uint32_t IDESC_PROJ = idesc_bf16(kRows, DS, 0, 0);
+    static constexpr uint32_t IDESC_S = idesc_bf16(kRows, 64, 0, 0);
+    static constexpr int TMEM_S = 128;            // score buffers at columns 128 and 192
 };
-
-// Dynamic shared memory: [operand tiles, later reused for output staging]
-// [Top-K columns when K > 32] [current 32 scores of each row] [tile-union bitmap].
 constexpr size_t kValuesBytes = size_t(32) * kRows * 4;
-template <int DS>
+template <int D, int DS>
 __host__ __device__ constexpr size_t proj_region0(int K) {
-    return SelProjCfg<DS>::TILE_BYTES > staging_bytes(K) ? size_t(SelProjCfg<DS>::TILE_BYTES) : staging_bytes(K);
+    return size_t(SelProjCfg<D, DS>::A_BYTES + SelProjCfg<D, DS>::B_BYTES) > staging_bytes(K)
+               ? size_t(SelProjCfg<D, DS>::A_BYTES + SelProjCfg<D, DS>::B_BYTES)
+               : staging_bytes(K);
 }
 
-template <int DS, bool REG>
+template <int D, int DS, bool REG>
 __global__ void __launch_bounds__(192, 2)
-select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_constant__ CUtensorMap mapKt, SelParams p) {
-    using Cfg = SelProjCfg<DS>;
+select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapWq,
+                   const __grid_constant__ CUtensorMap mapKt, SelParams p, int H) {
+    using Cfg = SelProjCfg<D, DS>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    __shared__ uint64_t q_full, kc_full[2], kc_empty[2], s_full[2], s_free[2], drain_bar;
+    __shared__ uint64_t in_full, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2], drain_bar;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
 
@@ -471,9 +483,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
     const int K = p.topk;
-    uint8_t* q_s = smem;
-    uint8_t* kc_s = smem + Cfg::Q_BYTES;
-    uint8_t* topk_s = smem + proj_region0<DS>(K);
+    uint8_t* a_s = smem;                        // Q tile, then q~
+    uint8_t* b_s = smem + Cfg::A_BYTES;         // Wq, then summary chunks
+    uint8_t* topk_s = smem + proj_region0<D, DS>(K);
     float* values_s = reinterpret_cast<float*>(topk_s + smem_topk_bytes(K));
     uint32_t* bitmap = reinterpret_cast<uint32_t*>(topk_s + smem_topk_bytes(K) + kValuesBytes);
 
@@ -486,7 +498,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     const int nwords = (p.C + 31) >> 5;
     for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
     if (threadIdx.x == 0) {
-        mbar_init(&q_full, 1);
+        mbar_init(&in_full, 1);
+        mbar_init(&proj_done, 1);
+        mbar_init(&qt_ready, 4);
         for (int b = 0; b < 2; ++b) {
             mbar_init(&kc_full[b], 1);
             mbar_init(&kc_empty[b], 1);
@@ -498,7 +512,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
         fence_barrier_init();
     }
     if (warp == 1) {
-        tmem_alloc(&tmem_base_sh, 128);
+        tmem_alloc(&tmem_base_sh, 256);
         tmem_relinquish();
     }
     __syncthreads();
@@ -509,49 +523,65 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
         if (nchunks > 0) {
-            tma_prefetch_desc(&mapQt);
+            tma_prefetch_desc(&mapQ);
+            tma_prefetch_desc(&mapWq);
             tma_prefetch_desc(&mapKt);
-            mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
+            mbar_arrive_expect_tx(&in_full, Cfg::Q_BYTES + Cfg::WQ_BYTES);
 #pragma unroll
-            for (int a = 0; a < DS / 64; ++a)
-                tma_load_3d(q_s + a * (kRows * 128), &mapQt, &q_full, a * 64, t * kRows, bh);
+            for (int a = 0; a < D / 64; ++a) {
+                tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, t * kRows, bh);
+                tma_load_3d(b_s + a * (DS * 128), &mapWq, &in_full, a * 64, 0, bh % H);
+            }
             int issued = 0;
-            bool ok = true;
-            for (int c = 0; c < nchunks; ++c) {
+            bool ok = mbar_wait(&proj_done, 0, wc);   // region B is free once the projection ran
+            for (int c = 0; ok && c < nchunks; ++c) {
                 const int b = c & 1;
                 if (!mbar_wait(&kc_empty[b], ((c >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
                 mbar_arrive_expect_tx(&kc_full[b], Cfg::KC_BYTES);
 #pragma unroll
                 for (int a = 0; a < DS / 64; ++a)
-                    tma_load_3d(kc_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, c * 64, bh);
+                    tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, c * 64, bh);
                 ++issued;
             }
             if (!ok) {
-                mbar_wait_drain(&q_full, 0, p.limit, p.status);
+                mbar_wait_drain(&in_full, 0, p.limit, p.status);
                 for (int q = issued - 1; q >= 0 && q >= issued - 2; --q)
                     mbar_wait_drain(&kc_full[q & 1], (q >> 1) & 1, p.limit, p.status);
             }
         }
     } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer: S[c&1] = Qt (128 x DS) * Kt_chunk (64 x DS)^T
-        if (nchunks > 0 && mbar_wait(&q_full, 0, wc)) {
-            const uint32_t q_addr = smem_u32(q_s);
-            for (int c = 0; c < nchunks; ++c) {
-                const int b = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                if (!mbar_wait(&kc_full[b], ph, wc)) break;
-                if (!mbar_wait(&s_free[b], ph ^ 1u, wc)) break;
-                tc_fence_after();
-                const uint32_t k_addr = smem_u32(kc_s + b * Cfg::KC_BYTES);
+        // ---------------- MMA issuer
+        if (nchunks > 0 && mbar_wait(&in_full, 0, wc)) {
+            tc_fence_after();
+            // q~ (fp32, TMEM columns 0 .. DS-1) = Q (128 x D) * Wq[h] (DS x D)^T
+            const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);
 #pragma unroll
-                for (int k = 0; k < DS / 16; ++k) {
-                    const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
-                    const uint32_t off_k = (k >> 2) * (64 * 128) + (k & 3) * 32;
-                    umma_bf16(tmem_base + b * 64, smem_desc_sw128(q_addr + off_q, 16, 1024),
-                              smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC, k > 0);
+            for (int k = 0; k < D / 16; ++k) {
+                const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                const uint32_t off_w = (k >> 2) * (DS * 128) + (k & 3) * 32;
+                umma_bf16(tmem_base, smem_desc_sw128(q_addr + off_q, 16, 1024),
+                          smem_desc_sw128(w_addr + off_w, 16, 1024), Cfg::IDESC_PROJ, k > 0);
+            }
+            umma_commit(&proj_done);
+            // S[c&1] = q~ (128 x DS, bf16 in region A) * Kt_chunk (64 x DS)^T
+            if (mbar_wait(&qt_ready, 0, wc)) {
+                for (int c = 0; c < nchunks; ++c) {
+                    const int b = c & 1;
+                    const uint32_t ph = (c >> 1) & 1;
+                    if (!mbar_wait(&kc_full[b], ph, wc)) break;
+                    if (!mbar_wait(&s_free[b], ph ^ 1u, wc)) break;
+                    tc_fence_after();
+                    const uint32_t k_addr = smem_u32(b_s + b * Cfg::KC_BYTES);
+#pragma unroll
+                    for (int k = 0; k < DS / 16; ++k) {
+                        const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                        const uint32_t off_k = (k >> 2) * (64 * 128) + (k & 3) * 32;
+                        umma_bf16(tmem_base + Cfg::TMEM_S + b * 64, smem_desc_sw128(q_addr + off_q, 16, 1024),
+                                  smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                    }
+                    umma_commit(&s_full[b]);
+                    umma_commit(&kc_empty[b]);
                 }
-                umma_commit(&s_full[b]);
-                umma_commit(&kc_empty[b]);
             }
         }
         umma_commit(&drain_bar);
@@ -563,6 +593,37 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
         const int i = t * kRows + r;
         const bool valid = i < p.N;
         const int Ci = valid ? (i >> 6) : 0;
+        const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+        bool ok = true;
+        if (nchunks > 0) {
+            // q~ row: fp32 from TMEM -> bf16 -> region A in the 128-byte-swizzled
+            // K-major layout of an MMA operand (16-byte chunk k of the row at k ^ (r & 7))
+            ok = mbar_wait_warp(&proj_done, 0, wc);
+            if (ok) {
+                tc_fence_after();
+#pragma unroll 1
+                for (int cc = 0; cc < DS / 32; ++cc) {
+                    uint32_t u[32];
+                    tmem_ld32(lane_addr + cc * 32, u);
+                    tmem_wait_ld();
+                    uint8_t* row = a_s + (cc >> 1) * (kRows * 128) + r * 128;
+#pragma unroll
+                    for (int k4 = 0; k4 < 4; ++k4) {
+                        const int k = (cc & 1) * 4 + k4;
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(u[8 * k4 + 0]), __uint_as_float(u[8 * k4 + 1]));
+                        w.y = pack_bf16x2(__uint_as_float(u[8 * k4 + 2]), __uint_as_float(u[8 * k4 + 3]));
+                        w.z = pack_bf16x2(__uint_as_float(u[8 * k4 + 4]), __uint_as_float(u[8 * k4 + 5]));
+                        w.w = pack_bf16x2(__uint_as_float(u[8 * k4 + 6]), __uint_as_float(u[8 * k4 + 7]));
+                        *reinterpret_cast<uint4*>(row + ((k ^ (r & 7)) << 4)) = w;
+                    }
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&qt_ready);
+        }
         RegTopK rtk;
         reg_init(rtk);
         SmemTopK stk{};
@@ -573,15 +634,14 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
         }
         RowLse lse{-CUDART_INF_F, 0.f};
         float* vcol = values_s + r;   // this row's current 32 scores, element j at j * kRows
-        const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-        for (int c = 0; c < nchunks; ++c) {
+        for (int c = 0; ok && c < nchunks; ++c) {
             const int b = c & 1;
             if (!mbar_wait_warp(&s_full[b], (c >> 1) & 1, wc)) break;
             tc_fence_after();
 #pragma unroll 1
             for (int half = 0; half < 2; ++half) {
                 uint32_t u[32];
-                tmem_ld32(lane_addr + b * 64 + half * 32, u);
+                tmem_ld32(lane_addr + Cfg::TMEM_S + b * 64 + half * 32, u);
                 tmem_wait_ld();
                 if (half == 1) {
                     tc_fence_before();
@@ -597,11 +657,11 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
                 else smem_consume(stk, lse, v, vcol, kRows, 2 * c + half, Ci, K);
             }
         }
-        // Every score MMA has completed once the last chunk was read, so the
-        // operand tiles are free and become the output staging area.
+        // Every MMA has completed once the last chunk was read, so regions A
+        // and B are free and become the output staging area.
         const Staging st{reinterpret_cast<int32_t*>(smem),
                          reinterpret_cast<float*>(smem + size_t(kRows) * (K + 1) * 4), K + 1};
-        const bool ok = !abort_flag;
+        ok = !abort_flag;
         if (valid && ok) {
             if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap);
             else row_emit(stk, lse, st, r, Ci, K, diag, bitmap);
@@ -615,22 +675,23 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQt, const __grid_const
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, 128);
+        tmem_dealloc(tmem_base, 256);
     }
 }
 
-template <int DS, bool REG>
+template <int D, int DS, bool REG>
 cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
-    const size_t smem = 1024 + proj_region0<DS>(a.topk) + smem_topk_bytes(a.topk) + kValuesBytes + bitmap_bytes(a.C);
+    const size_t smem = 1024 + proj_region0<D, DS>(a.topk) + smem_topk_bytes(a.topk) + kValuesBytes + bitmap_bytes(a.C);
     if (smem > 227 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = cudaFuncSetAttribute(select_proj_kernel<DS, REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(select_proj_kernel<D, DS, REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
-    CUtensorMap mq, mk;
-    if (make_tmap_bf16_3d(&mq, a.Qt, DS, a.N, a.BH, 64, kRows) != 0) { *err = "tensor map Qt"; return cudaErrorInvalidValue; }
+    CUtensorMap mq, mw, mk;
+    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kRows) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mw, a.Wq, D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
     dim3 grid(a.T, a.BH);
-    select_proj_kernel<DS, REG><<<grid, 192, smem, env.stream>>>(mq, mk, p);
+    select_proj_kernel<D, DS, REG><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;
@@ -650,6 +711,11 @@ cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEn
     return e;
 }
 
+template <int D, int DS>
+cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
+    return a.topk <= 32 ? launch_proj<D, DS, true>(a, p, env, err) : launch_proj<D, DS, false>(a, p, env, err);
+}
+
 }  // namespace
 
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
@@ -662,9 +728,11 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     p.status = env.status; p.limit = env.limit;
     const bool reg = a.topk <= 32;
     if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
-    if (a.d_sel == 128) return reg ? launch_proj<128, true>(a, p, env, err) : launch_proj<128, false>(a, p, env, err);
-    if (a.d_sel == 64) return reg ? launch_proj<64, true>(a, p, env, err) : launch_proj<64, false>(a, p, env, err);
-    *err = "selection: unsupported d_sel";
+    if (a.d == 128 && a.d_sel == 128) return launch_proj_k<128, 128>(a, p, env, err);
+    if (a.d == 128 && a.d_sel == 64) return launch_proj_k<128, 64>(a, p, env, err);
+    if (a.d == 64 && a.d_sel == 64) return launch_proj_k<64, 64>(a, p, env, err);
+    if (a.d == 64 && a.d_sel == 128) return launch_proj_k<64, 128>(a, p, env, err);
+    *err = "selection: unsupported head / selector dims";
     return cudaErrorInvalidValue;
 }
 

@@ -93,7 +93,6 @@ struct sas_handle {
     int BH = 0, C = 0, T = 0, F = 0;
     // workspace
     void* Kt = nullptr;         // bf16 [BH][max(F,1)][d_sel]
-    void* Qt = nullptr;         // bf16 [BH][N][d_sel]
     int32_t* union_idx = nullptr;
     int32_t* union_cnt = nullptr;
     int32_t* sel_idx = nullptr;
@@ -227,7 +226,6 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     const size_t rows = static_cast<size_t>(BH) * c.N;
     if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
         if (e == cudaSuccess) e = alloc(&h->Kt, static_cast<size_t>(BH) * (h->F > 0 ? h->F : 1) * d_sel * 2);
-        if (e == cudaSuccess) e = alloc(&h->Qt, rows * d_sel * 2);
     }
     if (e == cudaSuccess) e = alloc(&h->union_idx, static_cast<size_t>(BH) * h->T * h->C * 4);
     if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BH) * h->T * 4);
@@ -249,7 +247,6 @@ void sas_destroy(sas_handle* h) {
     if (h == nullptr) return;
     cudaDeviceSynchronize();
     cudaFree(h->Kt);
-    cudaFree(h->Qt);
     cudaFree(h->union_idx);
     cudaFree(h->union_cnt);
     cudaFree(h->sel_idx);
@@ -292,22 +289,13 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
             e = timed_launch(h, 0, s, [&] { return sas::launch_pool(K, Wk, h->Kt, h->BH, c.H, c.N, c.d, h->d_sel, env); });
             if (e != cudaSuccess) return cuda_fail(h, e, "block summaries");
         }
-        // a2 (first half): per-head query projection Qt = bf16(Q Wq^T) on the tensor cores
-        sas::GemmProblem g{};
-        g.A = Q; g.B = Wq; g.C = h->Qt; g.bias = nullptr;
-        g.M = c.N; g.N = h->d_sel; g.K = c.d;
-        g.batches = h->BH; g.b_mod = c.H;
-        g.c_batch_stride = static_cast<long long>(c.N) * h->d_sel; g.ldc = h->d_sel;
-        g.gelu = 0; g.bn = h->d_sel; g.max_ctas = 0;
-        e = timed_launch(h, 1, s, [&] { return sas::launch_gemm(g, env, &err); });
-        if (e != cudaSuccess) return cuda_fail(h, e, err);
     }
-    // a2-a4: scores, log-gates, Top-K, tile unions
+    // a2-a4: query projection (learned selector), scores, log-gates, Top-K, tile unions
     sas::SelectArgs sa{};
     sa.BH = h->BH; sa.H = c.H; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
     sa.score_scale = c.selector == SAS_SEL_MEANPOOL_PROJ ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
     sa.scores = scores;
-    sa.Qt = h->Qt; sa.Kt = h->Kt; sa.F = h->F;
+    sa.Q = Q; sa.Wq = Wq; sa.d = c.d; sa.Kt = h->Kt; sa.F = h->F;
     sa.sel_idx = out_idx; sa.sel_logg = out_lg;
     sa.union_idx = h->union_idx; sa.union_cnt = h->union_cnt;
     e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });

@@ -169,7 +169,7 @@ def test_launch_count_and_status_word():
     Q, K, V = synth.qkv(1, 1, 300, 64)
     Wq, Wk = synth.selector_weights(1, 64, 64)
     g = P.run_gpu(1, 1, 300, 64, 2, TRAIN, Q, K, V, Wq=Wq, Wk=Wk)
-    assert g["launches"] == 4          # pool, query projection, selection, attention
+    assert g["launches"] == 3          # block summaries, selection (with the query projection), attention
     assert g["status"] == 0
 
 
