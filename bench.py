@@ -127,6 +127,24 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ------------------------------------------------------- multi-rank helpers
+
+def reduce_max(values, dist, device):
+    """Max of each value over all ranks (identity without a process group):
+    the slowest rank sets the job's time."""
+    if dist is None:
+        return list(values)
+    import torch
+    t = torch.tensor(list(values), device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def job_throughput(tflop_per_step, world, ms_per_step):
+    """Whole-job TFLOP/s: every rank runs one replica of the step (weak scaling)."""
+    return tflop_per_step * world / (ms_per_step / 1e3)
+
+
 # --------------------------------------------------------------- our arm
 
 def kernel_traffic(kind):
@@ -239,10 +257,7 @@ def run_ours(args, w, rank, world):
     unions = sas.sas_get_tile_union_counts(h, B * H * Tt)
     layer.close()
 
-    if dist is not None:
-        t = torch.tensor([ms, e2e_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+    ms, e2e_ms = reduce_max([ms, e2e_ms], dist, dev)
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
@@ -250,7 +265,7 @@ def run_ours(args, w, rank, world):
 
     fl = algorithmic_flops(w)
     tflop = fl["total"] / 1e12
-    value = tflop * world / (ms / 1e3)
+    value = job_throughput(tflop, world, ms)
     per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None)} for k, (n, t) in kt.items()}
     flops_per_launch = {"attention": fl["attention"], "mlp_up_gelu": fl["mlp"] / 2, "mlp_down": fl["mlp"] / 2}
     dom = max((k for k in kt if kt[k][0] > 0), key=lambda k: kt[k][1])
@@ -279,7 +294,7 @@ def run_ours(args, w, rank, world):
                              "mean_union_blocks_per_tile": round(hist_blocks, 2)},
         "kernels": per_kind,
         "algorithmic_tflop_per_step": round(tflop, 4),
-        "e2e": {"value": round(tflop * world / (e2e_ms / 1e3), 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
+        "e2e": {"value": round(job_throughput(tflop, world, e2e_ms), 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clocks,

@@ -56,7 +56,7 @@ struct AttnCfg {
 
 // Barriers and flags at the end of the dynamic shared-memory region.
 struct AttnCtl {
-    uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2];
+    uint64_t q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2];
     uint64_t s_full[2], s_free[2], p_full[2], o_ready[2], drain_bar;
     uint32_t tmem_base;
     int abort_flag;
@@ -72,14 +72,41 @@ struct AttnParams {
     const int32_t* union_cnt;
     const int32_t* sel_idx;
     const float* sel_logg;
-    int N, C, T, topk, mode;
+    int N, C, T, BH, topk, mode;
     float scale_log2;
     int* status;
     long long limit;
 };
 
-__device__ __forceinline__ int block_at(const AttnParams& p, const int32_t* ulist, int U, int j, int t) {
-    return j < U ? __ldg(ulist + j) : 2 * t + (j - U);
+// The work list: item w is tile t = T-1 - w / BH of head bh = w % BH, so the
+// tiles with the longest key histories come first.  The grid is persistent:
+// CTA k of G takes the items r*G + k for even rounds r and r*G + G-1-k for odd
+// ones (a snake, which evens out the per-CTA totals of a cost-sorted list).
+__device__ __forceinline__ int work_item(int r, int k, int G) { return r * G + ((r & 1) ? G - 1 - k : k); }
+
+struct TileRef {
+    int t, bh;
+    const int32_t* ulist;   // the tile's union list (ascending historical blocks)
+    int U;                  // its length
+};
+
+__device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w) {
+    TileRef x;
+    x.t = p.T - 1 - w / p.BH;
+    x.bh = w % p.BH;
+    const long long tb = static_cast<long long>(x.bh) * p.T + x.t;
+    x.ulist = p.union_idx + tb * p.C;
+    x.U = __ldg(p.union_cnt + tb);
+    return x;
+}
+
+// visited blocks of a tile: its union list, then the diagonal block(s)
+__device__ __forceinline__ int tile_blocks(const AttnParams& p, const TileRef& x) {
+    return x.U + ((2 * x.t + 1 < p.C) ? 2 : 1);
+}
+
+__device__ __forceinline__ int block_at(const TileRef& x, int j) {
+    return j < x.U ? __ldg(x.ulist + j) : 2 * x.t + (j - x.U);
 }
 
 template <int D>
@@ -95,6 +122,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     }
     AttnCtl& ctl = *reinterpret_cast<AttnCtl*>(smem + Cfg::OFF_CTL);
     uint64_t& q_full = ctl.q_full;
+    uint64_t& q_empty = ctl.q_empty;
     uint64_t* k_full = ctl.k_full;
     uint64_t* k_empty = ctl.k_empty;
     uint64_t* v_full = ctl.v_full;
@@ -108,16 +136,14 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     int& abort_flag = ctl.abort_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
-
-    const int t = p.T - 1 - static_cast<int>(blockIdx.x);   // heavy tiles first
-    const int bh = blockIdx.y;
-    const int32_t* ulist = p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C;
-    const int U = __ldg(p.union_cnt + static_cast<long long>(bh) * p.T + t);
-    const int n_diag = (2 * t + 1 < p.C) ? 2 : 1;
-    const int n = U + n_diag;
+    const int G = static_cast<int>(gridDim.x);
+    const int k_cta = static_cast<int>(blockIdx.x);
+    const int W = p.T * p.BH;
+    const int rounds = (W + G - 1) / G;
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
+        mbar_init(&q_empty, 1);
         for (int s = 0; s < Cfg::KST; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
         for (int s = 0; s < Cfg::VST; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
         for (int s = 0; s < 2; ++s) {
@@ -139,60 +165,121 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     const uint32_t tmem_base = tmem_base_sh;
     const WaitCtl wc{&abort_flag, p.status, p.limit};
 
+    // Every role walks the same work items and counts visited blocks over all of
+    // them (g): ring slots, score buffers and barrier phases follow g, so the
+    // pipeline runs on across tile boundaries.
     if (warp == 0 && lane == 0) {
-        // ---------------- K producer (and the Q tile)
-        tma_prefetch_desc(&mapQ);
+        // ---------------- K producer
         tma_prefetch_desc(&mapK);
-        mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
-#pragma unroll
-        for (int a = 0; a < D / 64; ++a) tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, t * kBM, bh);
-        int issued = 0;
+        int g = 0, nk = 0;
         bool ok = true;
-        for (int j = 0; j < n; ++j) {
-            const int s = j % Cfg::KST;
-            if (!mbar_wait(&k_empty[s], ((j / Cfg::KST) & 1) ^ 1u, wc)) { ok = false; break; }
-            const int m = block_at(p, ulist, U, j, t);
-            uint8_t* dst = smem + Cfg::OFF_K + s * Cfg::KV_BYTES;
-            mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
+        for (int r = 0; ok && r < rounds; ++r) {
+            const int w = work_item(r, k_cta, G);
+            if (w >= W) continue;
+            const TileRef x = tile_ref(p, w);
+            const int n = tile_blocks(p, x);
+            for (int j = 0; j < n; ++j) {
+                const int gb = g + j;
+                const int s = gb % Cfg::KST;
+                const int m = block_at(x, j);
+                if (!mbar_wait(&k_empty[s], ((gb / Cfg::KST) & 1) ^ 1u, wc)) { ok = false; break; }
+                uint8_t* dst = smem + Cfg::OFF_K + s * Cfg::KV_BYTES;
+                mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
 #pragma unroll
-            for (int a = 0; a < D / 64; ++a) tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, bh);
-            ++issued;
+                for (int a = 0; a < D / 64; ++a)
+                    tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, x.bh);
+                ++nk;
+            }
+            g += n;
         }
         if (!ok) {
-            mbar_wait_drain(&q_full, 0, p.limit, p.status);
-            for (int q = issued - 1; q >= 0 && q >= issued - Cfg::KST; --q)
+            // loads are issued in block order, one per block: the last KST may be in flight
+            for (int q = nk - 1; q >= 0 && q >= nk - Cfg::KST; --q)
                 mbar_wait_drain(&k_full[q % Cfg::KST], (q / Cfg::KST) & 1, p.limit, p.status);
         }
     } else if (warp == 1 && lane == 0) {
-        // ---------------- V producer
+        // ---------------- V producer and the Q tile.  Q_{i+1} waits until the last
+        // QK of tile i has run; that falls between the V slots it waits on, so
+        // neither stream holds the other up.
+        tma_prefetch_desc(&mapQ);
         tma_prefetch_desc(&mapV);
-        int issued = 0;
+        int g = 0, tc = 0;
+        int nv = 0, nq = 0;
         bool ok = true;
-        for (int j = 0; j < n; ++j) {
-            const int s = j % Cfg::VST;
-            if (!mbar_wait(&v_empty[s], ((j / Cfg::VST) & 1) ^ 1u, wc)) { ok = false; break; }
-            const int m = block_at(p, ulist, U, j, t);
-            uint8_t* dst = smem + Cfg::OFF_V + s * Cfg::KV_BYTES;
-            mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
+        for (int r = 0; ok && r < rounds; ++r) {
+            const int w = work_item(r, k_cta, G);
+            if (w >= W) continue;
+            const TileRef x = tile_ref(p, w);
+            const int n = tile_blocks(p, x);
+            if (!mbar_wait(&q_empty, (tc & 1) ^ 1u, wc)) { ok = false; break; }
+            mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
 #pragma unroll
-            for (int a = 0; a < D / 64; ++a) tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, bh);
-            ++issued;
+            for (int a = 0; a < D / 64; ++a)
+                tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, x.t * kBM, x.bh);
+            ++nq;
+            for (int j = 0; j < n; ++j) {
+                const int gb = g + j;
+                const int s = gb % Cfg::VST;
+                const int m = block_at(x, j);
+                if (!mbar_wait(&v_empty[s], ((gb / Cfg::VST) & 1) ^ 1u, wc)) { ok = false; break; }
+                uint8_t* dst = smem + Cfg::OFF_V + s * Cfg::KV_BYTES;
+                mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
+#pragma unroll
+                for (int a = 0; a < D / 64; ++a)
+                    tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, x.bh);
+                ++nv;
+            }
+            g += n;
+            ++tc;
         }
         if (!ok) {
-            for (int q = issued - 1; q >= 0 && q >= issued - Cfg::VST; --q)
+            if (nq > 0) mbar_wait_drain(&q_full, (nq - 1) & 1, p.limit, p.status);
+            for (int q = nv - 1; q >= 0 && q >= nv - Cfg::VST; --q)
                 mbar_wait_drain(&v_full[q % Cfg::VST], (q / Cfg::VST) & 1, p.limit, p.status);
         }
     } else if (warp == 2 && lane == 0) {
-        // ---------------- MMA issuer
+        // ---------------- MMA issuer: QK of block g, then PV of block g-1; a tile's
+        // last PV is issued before the next tile starts, so that the softmax
+        // warps' epilogue does not wait for the next Q tile to arrive.
         const uint32_t q_addr = smem_u32(smem);
-        bool ok = mbar_wait(&q_full, 0, wc);
-        for (int j = 0; ok && j <= n; ++j) {
-            if (j < n) {
-                // S[j%2] = Q K_j^T
-                const int s = j % Cfg::KST;
-                const int sb = j & 1;
-                if (!mbar_wait(&k_full[s], (j / Cfg::KST) & 1, wc)) break;
-                if (!mbar_wait(&s_free[sb], ((j >> 1) & 1) ^ 1u, wc)) break;
+        // O += P_gb V_gb; `first` starts a new tile's accumulator
+        auto issue_pv = [&](int gb, bool first) -> bool {
+            const int vs = gb % Cfg::VST;
+            // p_full[gb&1] cannot run two phases ahead: the softmax needs QK_{gb+2},
+            // issued only after this wait, before it can arrive there again.
+            if (!mbar_wait(&p_full[gb & 1], (gb >> 1) & 1, wc)) return false;
+            if (!mbar_wait(&v_full[vs], (gb / Cfg::VST) & 1, wc)) return false;
+            tc_fence_after();
+            const uint32_t v_addr = smem_u32(smem + Cfg::OFF_V + vs * Cfg::KV_BYTES);
+#pragma unroll
+            for (int k = 0; k < kBN / 16; ++k) {
+                // P_gb sits in TMEM over the first 32 columns of score buffer gb & 1
+                // (16 keys = 8 packed columns per step).  V is MN-major (d contiguous):
+                // 16 keys = two 8-row atoms; the two 64-wide d halves sit kBN*128 bytes apart.
+                umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + (gb & 1) * 64 + k * 8,
+                             smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
+                             (!first || k > 0) ? 1u : 0u);
+            }
+            umma_commit(&o_ready[gb & 1]);
+            umma_commit(&v_empty[vs]);
+            umma_commit(&s_free[gb & 1]);   // score buffer (and P in it) free for QK_{gb+2}
+            return true;
+        };
+        int g = 0, tc = 0;
+        bool ok = true;
+        for (int r = 0; ok && r < rounds; ++r) {
+            const int w = work_item(r, k_cta, G);
+            if (w >= W) continue;
+            const TileRef x = tile_ref(p, w);
+            const int n = tile_blocks(p, x);
+            if (!mbar_wait(&q_full, tc & 1, wc)) { ok = false; break; }
+            for (int j = 0; j < n; ++j) {
+                // S[gb%2] = Q K_gb^T
+                const int gb = g + j;
+                const int s = gb % Cfg::KST;
+                const int sb = gb & 1;
+                if (!mbar_wait(&k_full[s], (gb / Cfg::KST) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait(&s_free[sb], ((gb >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t k_addr = smem_u32(smem + Cfg::OFF_K + s * Cfg::KV_BYTES);
 #pragma unroll
@@ -204,152 +291,144 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 }
                 umma_commit(&s_full[sb]);
                 umma_commit(&k_empty[s]);
+                if (j == n - 1) umma_commit(&q_empty);   // Q slot free for the next tile
+                if (j >= 1 && !issue_pv(gb - 1, j == 1)) { ok = false; break; }
             }
-            if (j >= 1) {
-                // O += P_{j-1} V_{j-1}
-                const int jj = j - 1;
-                const int vs = jj % Cfg::VST;
-                // p_full[jj&1] cannot run two phases ahead: the softmax needs QK_{jj+2},
-                // issued only after this wait, before it can arrive there again.
-                if (!mbar_wait(&p_full[jj & 1], (jj >> 1) & 1, wc)) break;
-                if (!mbar_wait(&v_full[vs], (jj / Cfg::VST) & 1, wc)) break;
-                tc_fence_after();
-                const uint32_t v_addr = smem_u32(smem + Cfg::OFF_V + vs * Cfg::KV_BYTES);
-#pragma unroll
-                for (int k = 0; k < kBN / 16; ++k) {
-                    // P_{jj} sits in TMEM over the first 32 columns of score buffer jj & 1
-                    // (16 keys = 8 packed columns per step).  V is MN-major (d contiguous):
-                    // 16 keys = two 8-row atoms; the two 64-wide d halves sit kBN*128 bytes apart.
-                    umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + (jj & 1) * 64 + k * 8,
-                                 smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
-                                 (jj > 0 || k > 0) ? 1u : 0u);
-                }
-                umma_commit(&o_ready[jj & 1]);
-                umma_commit(&v_empty[vs]);
-                umma_commit(&s_free[jj & 1]);   // score buffer (and P in it) free for QK_{jj+2}
-            }
+            if (ok && !issue_pv(g + n - 1, n == 1)) ok = false;
+            g += n;
+            ++tc;
         }
         umma_commit(&drain_bar);
         mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
     } else if (warp >= 4) {
         // ---------------- softmax / correction / epilogue: one thread per row
         const int q = warp - 4;
-        const int r = q * 32 + lane;
-        const int i = t * kBM + r;
-        const bool valid = i < p.N;
-        const int c = i >> 6;
-        const int nsel = valid ? min(p.topk, c) : 0;
-        const long long row_off = static_cast<long long>(bh) * p.N + i;
-        const int32_t* my_idx = p.sel_idx + row_off * p.topk;
-        const float* my_lg = p.sel_logg + row_off * p.topk;
-        const bool train = p.mode == 0;
-        // the row's next two kept blocks (a two-entry queue keeps the loads ahead of their use)
-        int sp = 0;
-        int km0 = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
-        float kl0 = nsel > 0 ? __ldg(my_lg) : 0.f;
-        int km1 = nsel > 1 ? __ldg(my_idx + 1) : 0x7fffffff;
-        float kl1 = nsel > 1 ? __ldg(my_lg + 1) : 0.f;
-
+        const int r_row = q * 32 + lane;
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2);
-
-        float m_use = -CUDART_INF_F;
-        float l = 0.f;
+        const bool train = p.mode == 0;
+        int g = 0;
         bool ok = true;
-        int m_next = block_at(p, ulist, U, 0, t);
-        for (int j = 0; j < n; ++j) {
-            const int sb = j & 1;
-            const int m = m_next;
-            if (j + 1 < n) m_next = block_at(p, ulist, U, j + 1, t);
-            // gate (log2 units) and the last visible key column of block m for this row
-            float bias = 0.f;
-            int lim;
-            if (m < c) {
-                if (m == km0) {
-                    bias = train ? kl0 * kLog2e : 0.f;
-                    lim = kBN - 1;
-                    ++sp;
-                    km0 = km1;
-                    kl0 = kl1;
-                    km1 = sp + 1 < nsel ? __ldg(my_idx + sp + 1) : 0x7fffffff;
-                    kl1 = sp + 1 < nsel ? __ldg(my_lg + sp + 1) : 0.f;
+        for (int r = 0; ok && r < rounds; ++r) {
+            const int w = work_item(r, k_cta, G);
+            if (w >= W) continue;
+            const TileRef x = tile_ref(p, w);
+            const int n = tile_blocks(p, x);
+            const int t = x.t;
+            const int i = t * kBM + r_row;
+            const bool valid = i < p.N;
+            const int c = i >> 6;
+            const int nsel = valid ? min(p.topk, c) : 0;
+            const long long row_off = static_cast<long long>(x.bh) * p.N + i;
+            const int32_t* my_idx = p.sel_idx + row_off * p.topk;
+            const float* my_lg = p.sel_logg + row_off * p.topk;
+            // The row's next two kept blocks (a two-entry queue).  Loads are
+            // predicated into pre-set registers and read one or more iterations
+            // later, so their latency is not paid where they are issued.
+            int sp = 0;
+            int km0 = 0x7fffffff, km1 = 0x7fffffff;
+            float kl0 = 0.f, kl1 = 0.f;
+            if (nsel > 0) { km0 = __ldg(my_idx); kl0 = __ldg(my_lg); }
+            if (nsel > 1) { km1 = __ldg(my_idx + 1); kl1 = __ldg(my_lg + 1); }
+
+            float m_use = -CUDART_INF_F;
+            float l = 0.f;
+            // raw list entry for the next iteration (entries past the union are the diagonal blocks)
+            int raw_next = 0;
+            if (x.U > 0) raw_next = __ldg(x.ulist);
+            for (int j = 0; j < n; ++j) {
+                const int gb = g + j;
+                const int sb = gb & 1;
+                const int m = j < x.U ? raw_next : 2 * t + (j - x.U);
+                if (j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
+                // gate (log2 units) and the last visible key column of block m for this row
+                float bias = 0.f;
+                int lim;
+                if (m < c) {
+                    if (m == km0) {
+                        bias = train ? kl0 * kLog2e : 0.f;
+                        lim = kBN - 1;
+                        ++sp;
+                        km0 = km1;
+                        kl0 = kl1;
+                        km1 = 0x7fffffff;
+                        if (sp + 1 < nsel) { km1 = __ldg(my_idx + sp + 1); kl1 = __ldg(my_lg + sp + 1); }
+                    } else {
+                        lim = -1;
+                    }
+                } else if (m == c) {
+                    lim = i & (kBN - 1);
                 } else {
                     lim = -1;
                 }
-            } else if (m == c) {
-                lim = i & (kBN - 1);
-            } else {
-                lim = -1;
-            }
-            const bool active = lim >= 0;
+                const bool active = lim >= 0;
 
-            if (!mbar_wait_warp(&s_full[sb], (j >> 1) & 1, wc)) { ok = false; break; }
-            tc_fence_after();
-            const bool warp_active = __any_sync(0xffffffffu, active);
-            float x[64];
-            if (warp_active) {
-                uint32_t u0[32], u1[32];
-                tmem_ld32(lane_addr + sb * 64, u0);
-                tmem_ld32(lane_addr + sb * 64 + 32, u1);
-                tmem_wait_ld();
-#pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    x[k] = __uint_as_float(u0[k]);
-                    x[k + 32] = __uint_as_float(u1[k]);
-                }
-            }
-            bool need = false;
-            float m_new = m_use;
-            float rs = 0.f;
-            uint32_t pk[32];   // P row as packed bf16 pairs
-            if (warp_active) {
-                // causal mask on the diagonal block only
-                if (__any_sync(0xffffffffu, lim >= 0 && lim < kBN - 1)) {
-#pragma unroll
-                    for (int k = 0; k < 64; ++k) x[k] = k <= lim ? x[k] : -CUDART_INF_F;
-                }
-                float mx0 = -CUDART_INF_F, mx1 = -CUDART_INF_F;
-#pragma unroll
-                for (int k = 0; k < 64; k += 4) {
-                    mx0 = max3f(mx0, x[k], x[k + 1]);
-                    mx1 = max3f(mx1, x[k + 2], x[k + 3]);
-                }
-                const float mx = fmaxf(mx0, mx1);
-                // max of the gated logits (log2 units): the gate is constant over the block
-                const float mb = active ? fmaf(mx, p.scale_log2, bias) : -CUDART_INF_F;
-                need = mb > m_use + kRescaleThreshold;
-                m_new = need ? mb : m_use;
-                const float base = m_new == -CUDART_INF_F ? 0.f : m_new;
-                const float off = active ? bias - base : -CUDART_INF_F;
-                const uint64_t off2 = f32x2(off, off);
-                uint64_t acc[4] = {0, 0, 0, 0};
-#pragma unroll
-                for (int k = 0; k < 64; k += 2) {
-                    float a0, a1;
-                    f32x2_split(fma_f32x2(f32x2(x[k], x[k + 1]), scale2, off2), a0, a1);
-                    const float e0 = fast_exp2(a0), e1 = fast_exp2(a1);
-                    acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(e0, e1));
-                    pk[k >> 1] = pack_bf16x2(e0, e1);
-                }
-                float s0, s1, s2, s3, s4, s5, s6, s7;
-                f32x2_split(acc[0], s0, s1);
-                f32x2_split(acc[1], s2, s3);
-                f32x2_split(acc[2], s4, s5);
-                f32x2_split(acc[3], s6, s7);
-                rs = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
-            } else {
-#pragma unroll
-                for (int k = 0; k < 32; ++k) pk[k] = 0u;
-            }
-            float factor = 1.f;
-            if (need) factor = m_use == -CUDART_INF_F ? 0.f : fast_exp2(m_use - m_new);
-
-            if (j > 0 && __any_sync(0xffffffffu, need)) {
-                // Rescaling O needs PV_{j-1} done.  PV_{j-1} is the ((j-1)/2)-th phase of
-                // o_ready[(j-1)&1]; that barrier cannot move past it before p_full(j+1).
-                if (!mbar_wait_warp(&o_ready[(j - 1) & 1], ((j - 1) >> 1) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait_warp(&s_full[sb], (gb >> 1) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
-                {
+                const bool warp_active = __any_sync(0xffffffffu, active);
+                float xs[64];
+                if (warp_active) {
+                    uint32_t u0[32], u1[32];
+                    tmem_ld32(lane_addr + sb * 64, u0);
+                    tmem_ld32(lane_addr + sb * 64 + 32, u1);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) {
+                        xs[k] = __uint_as_float(u0[k]);
+                        xs[k + 32] = __uint_as_float(u1[k]);
+                    }
+                }
+                bool need = false;
+                float m_new = m_use;
+                float rs = 0.f;
+                uint32_t pk[32];   // P row as packed bf16 pairs
+                if (warp_active) {
+                    // causal mask on the diagonal block only
+                    if (__any_sync(0xffffffffu, lim >= 0 && lim < kBN - 1)) {
+#pragma unroll
+                        for (int k = 0; k < 64; ++k) xs[k] = k <= lim ? xs[k] : -CUDART_INF_F;
+                    }
+                    float mx0 = -CUDART_INF_F, mx1 = -CUDART_INF_F;
+#pragma unroll
+                    for (int k = 0; k < 64; k += 4) {
+                        mx0 = max3f(mx0, xs[k], xs[k + 1]);
+                        mx1 = max3f(mx1, xs[k + 2], xs[k + 3]);
+                    }
+                    const float mx = fmaxf(mx0, mx1);
+                    // max of the gated logits (log2 units): the gate is constant over the block
+                    const float mb = active ? fmaf(mx, p.scale_log2, bias) : -CUDART_INF_F;
+                    need = mb > m_use + kRescaleThreshold;
+                    m_new = need ? mb : m_use;
+                    const float base = m_new == -CUDART_INF_F ? 0.f : m_new;
+                    const float off = active ? bias - base : -CUDART_INF_F;
+                    const uint64_t off2 = f32x2(off, off);
+                    uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+                    for (int k = 0; k < 64; k += 2) {
+                        float a0, a1;
+                        f32x2_split(fma_f32x2(f32x2(xs[k], xs[k + 1]), scale2, off2), a0, a1);
+                        const float e0 = fast_exp2(a0), e1 = fast_exp2(a1);
+                        acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(e0, e1));
+                        pk[k >> 1] = pack_bf16x2(e0, e1);
+                    }
+                    float s0, s1, s2, s3, s4, s5, s6, s7;
+                    f32x2_split(acc[0], s0, s1);
+                    f32x2_split(acc[1], s2, s3);
+                    f32x2_split(acc[2], s4, s5);
+                    f32x2_split(acc[3], s6, s7);
+                    rs = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) pk[k] = 0u;
+                }
+                float factor = 1.f;
+                if (need) factor = m_use == -CUDART_INF_F ? 0.f : fast_exp2(m_use - m_new);
+
+                if (j > 0 && __any_sync(0xffffffffu, need)) {
+                    // Rescaling O needs PV_{gb-1} done.  PV_{gb-1} is the ((gb-1)/2)-th phase of
+                    // o_ready[(gb-1)&1]; that barrier cannot move past it before p_full(gb+1).
+                    if (!mbar_wait_warp(&o_ready[(gb - 1) & 1], ((gb - 1) >> 1) & 1, wc)) { ok = false; break; }
+                    tc_fence_after();
 #pragma unroll 1
                     for (int cc = 0; cc < D / 32; ++cc) {
                         uint32_t o[32];
@@ -361,19 +440,23 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                     }
                     tmem_wait_st();
                 }
+                l = l * factor + rs;
+                m_use = m_new;
+
+                // P row (64 bf16, packed in pairs) into TMEM over this row's scores
+                tmem_st32(lane_addr + sb * 64, pk);
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_full[sb]);
             }
-            l = l * factor + rs;
-            m_use = m_new;
+            if (!ok) break;
 
-            // P row (64 bf16, packed in pairs) into TMEM over this row's scores
-            tmem_st32(lane_addr + sb * 64, pk);
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&p_full[sb]);
-        }
-
-        if (ok && mbar_wait_warp(&o_ready[(n - 1) & 1], ((n - 1) >> 1) & 1, wc)) {
+            // Epilogue.  The next tile's first PV overwrites O; it is issued only after
+            // this warp has arrived on p_full for that tile's first block, i.e. after
+            // the reads below have completed.  (Its first QK may already run.)
+            const int gl = g + n - 1;
+            if (!mbar_wait_warp(&o_ready[gl & 1], (gl >> 1) & 1, wc)) { ok = false; break; }
             tc_fence_after();
             const float inv = 1.f / l;
             bf16* orow = p.O + row_off * D;
@@ -386,16 +469,18 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                     uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(o[8 * e + 0]) * inv, __uint_as_float(o[8 * e + 1]) * inv);
-                        w.y = pack_bf16x2(__uint_as_float(o[8 * e + 2]) * inv, __uint_as_float(o[8 * e + 3]) * inv);
-                        w.z = pack_bf16x2(__uint_as_float(o[8 * e + 4]) * inv, __uint_as_float(o[8 * e + 5]) * inv);
-                        w.w = pack_bf16x2(__uint_as_float(o[8 * e + 6]) * inv, __uint_as_float(o[8 * e + 7]) * inv);
-                        dst[e] = w;
+                        uint4 v;
+                        v.x = pack_bf16x2(__uint_as_float(o[8 * e + 0]) * inv, __uint_as_float(o[8 * e + 1]) * inv);
+                        v.y = pack_bf16x2(__uint_as_float(o[8 * e + 2]) * inv, __uint_as_float(o[8 * e + 3]) * inv);
+                        v.z = pack_bf16x2(__uint_as_float(o[8 * e + 4]) * inv, __uint_as_float(o[8 * e + 5]) * inv);
+                        v.w = pack_bf16x2(__uint_as_float(o[8 * e + 6]) * inv, __uint_as_float(o[8 * e + 7]) * inv);
+                        dst[e] = v;
                     }
                 }
             }
             if (valid && p.LSE != nullptr) p.LSE[row_off] = m_use * kLn2 + logf(l);
+            tc_fence_before();
+            g += n;
         }
     }
     __syncthreads();
@@ -414,6 +499,10 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
         attr_set = true;
     }
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) { *err = "SM count"; return e; }
     CUtensorMap mq, mk, mv;
     if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kBM) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.K, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
@@ -425,13 +514,15 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.union_cnt = a.union_cnt;
     p.sel_idx = a.sel_idx;
     p.sel_logg = a.sel_logg;
-    p.N = a.N; p.C = a.C; p.T = a.T; p.topk = a.topk; p.mode = a.mode;
+    p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
     p.scale_log2 = a.sm_scale * kLog2e;
     p.status = env.status;
     p.limit = env.limit;
-    dim3 grid(a.T, a.BH);
-    attn_kernel<D><<<grid, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
-    cudaError_t e = cudaGetLastError();
+    // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
+    const long long items = static_cast<long long>(a.T) * a.BH;
+    const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);
+    attn_kernel<D><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
+    e = cudaGetLastError();
     if (e != cudaSuccess) *err = "attention launch";
     return e;
 }
