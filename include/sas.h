@@ -64,7 +64,7 @@ typedef enum { SAS_MODE_TRAIN_SOFT = 0, SAS_MODE_INFER_HARD = 1 } sas_mode;
 typedef enum { SAS_SEL_SCORES_GIVEN = 0, SAS_SEL_MEANPOOL_PROJ = 1 } sas_selector;
 
 typedef struct {
-    int32_t B, H, N, d;   /* batch, heads, tokens, head dim (d in {64, 128})          */
+    int32_t B, H, N, d;   /* batch, heads, tokens (N <= 2^30), head dim (d in {64, 128}) */
     int32_t block;        /* block size b; must be 64 (Sec. 4.2.1 setup)             */
     int32_t topk;         /* K historical blocks kept per query, 0 <= K <= 64         */
     float sm_scale;       /* softmax scale on q.k; 0 selects 1/sqrt(d) (Alg. 3)       */

@@ -79,6 +79,7 @@ struct AttnArgs {
     const float* sel_logg;
     int BH, N, d, C, T, topk, mode;
     float sm_scale;
+    int* sched;                 // 16 zeroed bytes owned by the caller, left zeroed after each launch
 };
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err);
 

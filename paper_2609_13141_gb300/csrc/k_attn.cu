@@ -35,6 +35,9 @@ constexpr int kThreads = 256;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.69314718055994531f;
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
+constexpr int kMaxStages = 4;                // capacity of the K / V ring barrier arrays
+constexpr int kItemSlots = 4;                // work items in flight between the fetching thread and the other roles
+constexpr int kItemReaders = 7;              // K producer, V producer, MMA issuer, four softmax warps
 
 template <int D>
 struct AttnCfg {
@@ -42,12 +45,13 @@ struct AttnCfg {
     static constexpr int KV_BYTES = kBN * D * 2;
     static constexpr int KST = 2;
     static constexpr int VST = 2;
+    static_assert(KST <= kMaxStages && VST <= kMaxStages, "ring barrier arrays");
     static constexpr int OFF_K = Q_BYTES;
     static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
     static constexpr int OFF_CTL = OFF_V + VST * KV_BYTES;
     // All shared state lives in the dynamic region (no static shared memory),
     // so that two CTAs fit on one SM.
-    static constexpr int SMEM = OFF_CTL + 256;
+    static constexpr int SMEM = OFF_CTL + 512;
     static constexpr int TMEM_COLS = 256;    // S0 [0,64) S1 [64,128) O [128,128+D)
     static constexpr int TMEM_O = 128;
     static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, 0, 0);
@@ -56,12 +60,14 @@ struct AttnCfg {
 
 // Barriers and flags at the end of the dynamic shared-memory region.
 struct AttnCtl {
-    uint64_t q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2];
+    uint64_t q_full, q_empty, k_full[kMaxStages], k_empty[kMaxStages], v_full[kMaxStages], v_empty[kMaxStages];
     uint64_t s_full[2], s_free[2], p_full[2], o_ready[2], drain_bar;
+    uint64_t item_full[kItemSlots], item_empty[kItemSlots];
+    int item[kItemSlots];   // work item (or -1: no more work) published to the other roles
     uint32_t tmem_base;
     int abort_flag;
 };
-static_assert(sizeof(AttnCtl) <= 256, "control block");
+static_assert(sizeof(AttnCtl) <= 512, "control block");
 
 constexpr int kStatusLayout = 3;   // == SAS_ERR_CUDA: shared-memory base not 1024-byte aligned
 
@@ -73,16 +79,20 @@ struct AttnParams {
     const int32_t* sel_idx;
     const float* sel_logg;
     int N, C, T, BH, topk, mode;
+    int group;              // heads per group of the work list
+    int* sched;             // [0] next work item, [1] CTAs finished; both zero between launches
     float scale_log2;
     int* status;
     long long limit;
 };
 
-// The work list: item w is tile t = T-1 - w / BH of head bh = w % BH, so the
-// tiles with the longest key histories come first.  The grid is persistent:
-// CTA k of G takes the items r*G + k for even rounds r and r*G + G-1-k for odd
-// ones (a snake, which evens out the per-CTA totals of a cost-sorted list).
-__device__ __forceinline__ int work_item(int r, int k, int G) { return r * G + ((r & 1) ? G - 1 - k : k); }
+// The work list: heads are taken in groups whose K and V fit in about half of
+// L2 together (all heads at once when they fit), and within a group the tiles
+// with the longest key histories come first, the head varying fastest.  The
+// grid is persistent and the list is handed out dynamically: a CTA's K
+// producer takes the next item from a global counter when it starts a tile
+// (tile costs vary with their union lists, so a fixed split would leave SMs
+// idle) and passes it to the CTA's other roles through a small shared ring.
 
 struct TileRef {
     int t, bh;
@@ -92,12 +102,26 @@ struct TileRef {
 
 __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w) {
     TileRef x;
-    x.t = p.T - 1 - w / p.BH;
-    x.bh = w % p.BH;
+    const int per_group = p.group * p.T;                  // items of a full group
+    const int g0 = w / per_group;                         // group index
+    const int h0 = g0 * p.group;                          // its first head
+    const int gs = min(p.group, p.BH - h0);               // heads in this group
+    const int wi = w - g0 * per_group;
+    x.t = p.T - 1 - wi / gs;
+    x.bh = h0 + wi % gs;
     const long long tb = static_cast<long long>(x.bh) * p.T + x.t;
     x.ulist = p.union_idx + tb * p.C;
     x.U = __ldg(p.union_cnt + tb);
     return x;
+}
+
+// Reader side of the item ring: the r-th work item of this CTA, or -1.
+// The caller arrives on item_empty once its lanes have read the value.
+__device__ __forceinline__ bool read_item(AttnCtl& ctl, int r, const WaitCtl& wc, int& w) {
+    const int slot = r % kItemSlots;
+    if (!mbar_wait(&ctl.item_full[slot], (r / kItemSlots) & 1, wc)) return false;
+    w = *reinterpret_cast<volatile int*>(&ctl.item[slot]);
+    return true;
 }
 
 // visited blocks of a tile: its union list, then the diagonal block(s)
@@ -136,10 +160,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     int& abort_flag = ctl.abort_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
-    const int G = static_cast<int>(gridDim.x);
-    const int k_cta = static_cast<int>(blockIdx.x);
     const int W = p.T * p.BH;
-    const int rounds = (W + G - 1) / G;
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
@@ -153,6 +174,10 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             mbar_init(&p_full[s], 4);
         }
         mbar_init(&drain_bar, 1);
+        for (int s = 0; s < kItemSlots; ++s) {
+            mbar_init(&ctl.item_full[s], 1);
+            mbar_init(&ctl.item_empty[s], kItemReaders);
+        }
         abort_flag = 0;
         fence_barrier_init();
     }
@@ -173,9 +198,17 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         tma_prefetch_desc(&mapK);
         int g = 0, nk = 0;
         bool ok = true;
-        for (int r = 0; ok && r < rounds; ++r) {
-            const int w = work_item(r, k_cta, G);
-            if (w >= W) continue;
+        for (int r = 0; ok; ++r) {
+            // take the next item and publish it (the slot is free once all readers
+            // have taken the item published kItemSlots tiles earlier)
+            const int slot = r % kItemSlots;
+            if (!mbar_wait(&ctl.item_empty[slot], ((r / kItemSlots) & 1) ^ 1u, wc)) { ok = false; break; }
+            int w = atomicAdd(p.sched, 1);
+            if (w >= W) w = -1;
+            *reinterpret_cast<volatile int*>(&ctl.item[slot]) = w;
+            mbar_arrive(&ctl.item_full[slot]);
+            mbar_arrive(&ctl.item_empty[slot]);   // this thread has read it too
+            if (w < 0) break;
             const TileRef x = tile_ref(p, w);
             const int n = tile_blocks(p, x);
             for (int j = 0; j < n; ++j) {
@@ -206,9 +239,11 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         int g = 0, tc = 0;
         int nv = 0, nq = 0;
         bool ok = true;
-        for (int r = 0; ok && r < rounds; ++r) {
-            const int w = work_item(r, k_cta, G);
-            if (w >= W) continue;
+        for (int r = 0; ok; ++r) {
+            int w;
+            if (!read_item(ctl, r, wc, w)) { ok = false; break; }
+            mbar_arrive(&ctl.item_empty[r % kItemSlots]);
+            if (w < 0) break;
             const TileRef x = tile_ref(p, w);
             const int n = tile_blocks(p, x);
             if (!mbar_wait(&q_empty, (tc & 1) ^ 1u, wc)) { ok = false; break; }
@@ -267,9 +302,11 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         };
         int g = 0, tc = 0;
         bool ok = true;
-        for (int r = 0; ok && r < rounds; ++r) {
-            const int w = work_item(r, k_cta, G);
-            if (w >= W) continue;
+        for (int r = 0; ok; ++r) {
+            int w;
+            if (!read_item(ctl, r, wc, w)) { ok = false; break; }
+            mbar_arrive(&ctl.item_empty[r % kItemSlots]);
+            if (w < 0) break;
             const TileRef x = tile_ref(p, w);
             const int n = tile_blocks(p, x);
             if (!mbar_wait(&q_full, tc & 1, wc)) { ok = false; break; }
@@ -309,9 +346,13 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         const bool train = p.mode == 0;
         int g = 0;
         bool ok = true;
-        for (int r = 0; ok && r < rounds; ++r) {
-            const int w = work_item(r, k_cta, G);
-            if (w >= W) continue;
+        for (int r = 0; ok; ++r) {
+            const int slot = r % kItemSlots;
+            if (!mbar_wait_warp(&ctl.item_full[slot], (r / kItemSlots) & 1, wc)) { ok = false; break; }
+            const int w = *reinterpret_cast<volatile int*>(&ctl.item[slot]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
+            if (w < 0) break;
             const TileRef x = tile_ref(p, w);
             const int n = tile_blocks(p, x);
             const int t = x.t;
@@ -484,6 +525,15 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         }
     }
     __syncthreads();
+    if (threadIdx.x == 0) {
+        // This CTA takes no more items.  The last CTA to get here returns the
+        // counters to zero for the next launch.
+        __threadfence();
+        if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+            atomicExch(p.sched, 0);
+            atomicExch(p.sched + 1, 0);
+        }
+    }
     if (warp == 3) {
         tc_fence_after();
         tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
@@ -499,10 +549,11 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
         attr_set = true;
     }
-    int dev = 0, sms = 0;
+    int dev = 0, sms = 0, l2 = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) { *err = "SM count"; return e; }
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev);
+    if (e != cudaSuccess) { *err = "device attributes"; return e; }
     CUtensorMap mq, mk, mv;
     if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kBM) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.K, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
@@ -515,9 +566,14 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.sel_idx = a.sel_idx;
     p.sel_logg = a.sel_logg;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
+    // heads whose K and V (2 * N * d bf16 each) fit in half of L2 together, at least one
+    const long long kv_head = 4LL * a.N * D;
+    const long long fit = kv_head > 0 ? (static_cast<long long>(l2) / 2) / kv_head : a.BH;
+    p.group = static_cast<int>(fit < 1 ? 1 : (fit > a.BH ? a.BH : fit));
     p.scale_log2 = a.sm_scale * kLog2e;
     p.status = env.status;
     p.limit = env.limit;
+    p.sched = a.sched;
     // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
     const long long items = static_cast<long long>(a.T) * a.BH;
     const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);

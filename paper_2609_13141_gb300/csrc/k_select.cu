@@ -38,7 +38,7 @@ constexpr int kRows = 128;
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct SelParams {
-    int N, C, T, F, topk;
+    int BH, N, C, T, F, topk;
     float score_scale;
     const float* scores;
     int32_t* sel_idx;
@@ -48,6 +48,12 @@ struct SelParams {
     int* status;
     long long limit;
 };
+
+// One CTA per (head, 128-row tile) on a 1-D grid: the tile index falls with
+// the block index and the head varies fastest, so the tiles with the longest
+// histories of every head are dispatched first and the light ones fill the tail.
+__device__ __forceinline__ int tile_of_block(int T, int BH) { return T - 1 - static_cast<int>(blockIdx.x / BH); }
+__device__ __forceinline__ int head_of_block(int BH) { return static_cast<int>(blockIdx.x % BH); }
 
 // Online log-sum-exp of a row's scores.
 struct RowLse {
@@ -75,48 +81,59 @@ __device__ __forceinline__ void lse_update(RowLse& l, const float (&v)[32], int 
 // strictly better: a later block with an equal score ranks below every kept
 // one because ties go to the lower block.  The work grows with the number of
 // replacements (about K ln(C_i / K) for scores in random order), not with C_i.
+// Block indices are kept as floats (exact: the C ABI caps N at 2^30 tokens, so
+// blocks stay below 2^24); the worst entry is found with two shallow reduction
+// trees (minimum score, then the highest block among the slots at that score)
+// instead of a serial scan, and replaced by its block index, which is unique.
 struct RegTopK {
     float s[32];
-    int m[32];
-    float ws;
-    int wm, wpos;
+    float mf[32];   // block index; slots at or past K hold +inf / kEmptyBlock
+    float ws;       // worst kept score
+    float wmf;      // its block
     bool replaced;
 };
+
+constexpr float kEmptyBlock = 1073741824.f;   // 2^30: above every block index, sorts last
 
 __device__ __forceinline__ void reg_init(RegTopK& t) {
     t.replaced = false;
     t.ws = -CUDART_INF_F;
-    t.wm = 0;
-    t.wpos = 0;
+    t.wmf = 0.f;
 }
 
-__device__ __forceinline__ void reg_rescan(RegTopK& t, int K) {
-    float ws = CUDART_INF_F;
-    int wm = -1, wp = 0;
+__device__ __forceinline__ void reg_rescan(RegTopK& t) {
+    // minimum score: 3-input min tree (slots past K hold +inf and never win)
+    float a[11];
 #pragma unroll
-    for (int e = 0; e < 32; ++e) {
-        if (e < K && (t.s[e] < ws || (t.s[e] == ws && t.m[e] > wm))) {
-            ws = t.s[e];
-            wm = t.m[e];
-            wp = e;
-        }
-    }
+    for (int g = 0; g < 10; ++g) a[g] = min3f(t.s[3 * g], t.s[3 * g + 1], t.s[3 * g + 2]);
+    a[10] = fminf(t.s[30], t.s[31]);
+    const float b0 = min3f(a[0], a[1], a[2]), b1 = min3f(a[3], a[4], a[5]);
+    const float b2 = min3f(a[6], a[7], a[8]), b3 = fminf(a[9], a[10]);
+    const float ws = fminf(min3f(b0, b1, b2), b3);
+    // the highest block among the slots holding that score
+    float c[11];
+#pragma unroll
+    for (int g = 0; g < 10; ++g)
+        c[g] = max3f(t.s[3 * g] == ws ? t.mf[3 * g] : -1.f, t.s[3 * g + 1] == ws ? t.mf[3 * g + 1] : -1.f,
+                     t.s[3 * g + 2] == ws ? t.mf[3 * g + 2] : -1.f);
+    c[10] = fmaxf(t.s[30] == ws ? t.mf[30] : -1.f, t.s[31] == ws ? t.mf[31] : -1.f);
+    const float d0 = max3f(c[0], c[1], c[2]), d1 = max3f(c[3], c[4], c[5]);
+    const float d2 = max3f(c[6], c[7], c[8]), d3 = fmaxf(c[9], c[10]);
     t.ws = ws;
-    t.wm = wm;
-    t.wpos = wp;
+    t.wmf = fmaxf(max3f(d0, d1, d2), d3);
 }
 
-__device__ __forceinline__ void reg_offer(RegTopK& t, float x, int idx, int K) {
+__device__ __forceinline__ void reg_offer(RegTopK& t, float x, int idx) {
     if (x > t.ws) {
+        const float xf = static_cast<float>(idx);
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-            if (e == t.wpos) {
-                t.s[e] = x;
-                t.m[e] = idx;
-            }
+            const bool hit = t.mf[e] == t.wmf;
+            t.s[e] = hit ? x : t.s[e];
+            t.mf[e] = hit ? xf : t.mf[e];
         }
         t.replaced = true;
-        reg_rescan(t, K);
+        reg_rescan(t);
     }
 }
 
@@ -145,10 +162,10 @@ __device__ __forceinline__ void reg_consume(RegTopK& t, RowLse& l, const float (
         for (int j = 0; j < 32; ++j) {
             // unused slots carry the largest block index so that sorting sinks them
             t.s[j] = j < nf ? v[j] : CUDART_INF_F;
-            t.m[j] = j < nf ? j : 0x7fffffff;
+            t.mf[j] = j < nf ? static_cast<float>(j) : kEmptyBlock;
         }
         if (Ci <= K) return;
-        reg_rescan(t, K);
+        reg_rescan(t);
         lo = K;
     }
     // The threshold only rises while the chunk is consumed, so this mask is a
@@ -157,7 +174,7 @@ __device__ __forceinline__ void reg_consume(RegTopK& t, RowLse& l, const float (
     while (mask) {
         const int j = __ffs(mask) - 1;
         mask &= mask - 1;
-        reg_offer(t, col[j * stride], 32 * c + j, K);
+        reg_offer(t, col[j * stride], 32 * c + j);
     }
 }
 
@@ -173,13 +190,13 @@ __device__ __forceinline__ void reg_sort_by_block(RegTopK& t) {
                 const int l = i ^ j;
                 if (l > i) {
                     const bool up = (i & k) == 0;
-                    const bool sw = up ? (t.m[i] > t.m[l]) : (t.m[i] < t.m[l]);
+                    const bool sw = up ? (t.mf[i] > t.mf[l]) : (t.mf[i] < t.mf[l]);
                     const float si = t.s[i], sl = t.s[l];
-                    const int mi = t.m[i], ml = t.m[l];
+                    const float mi = t.mf[i], ml = t.mf[l];
                     t.s[i] = sw ? sl : si;
                     t.s[l] = sw ? si : sl;
-                    t.m[i] = sw ? ml : mi;
-                    t.m[l] = sw ? mi : ml;
+                    t.mf[i] = sw ? ml : mi;
+                    t.mf[l] = sw ? mi : ml;
                 }
             }
         }
@@ -313,9 +330,10 @@ __device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, c
     for (int e = 0; e < 32; ++e) {
         if (e < K) {
             const bool kept = e < n;
-            stage_entry(st, r, e, kept ? t.m[e] : -1, kept ? t.s[e] - lse : 0.f);
-            if (kept && static_cast<unsigned>(t.m[e]) < static_cast<unsigned>(diag))
-                atomicOr(&bitmap[t.m[e] >> 5], 1u << (t.m[e] & 31));
+            const int m = static_cast<int>(t.mf[e]);
+            stage_entry(st, r, e, kept ? m : -1, kept ? t.s[e] - lse : 0.f);
+            if (kept && static_cast<unsigned>(m) < static_cast<unsigned>(diag))
+                atomicOr(&bitmap[m >> 5], 1u << (m & 31));
         }
     }
 }
@@ -375,8 +393,8 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ float stage[4][32][33];
 
-    const int t = p.T - 1 - static_cast<int>(blockIdx.x);
-    const int bh = blockIdx.y;
+    const int t = tile_of_block(p.T, p.BH);
+    const int bh = head_of_block(p.BH);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int r = threadIdx.x;
     const int i = t * kRows + r;
@@ -489,8 +507,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     float* values_s = reinterpret_cast<float*>(topk_s + smem_topk_bytes(K));
     uint32_t* bitmap = reinterpret_cast<uint32_t*>(topk_s + smem_topk_bytes(K) + kValuesBytes);
 
-    const int t = p.T - 1 - static_cast<int>(blockIdx.x);
-    const int bh = blockIdx.y;
+    const int t = tile_of_block(p.T, p.BH);
+    const int bh = head_of_block(p.BH);
     const int diag = 2 * t;
     const int nb = min(2 * t + 1, p.F);          // blocks scored for this tile
     const int nchunks = (nb + 63) >> 6;
@@ -690,7 +708,7 @@ cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv
     if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kRows) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mw, a.Wq, D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
-    dim3 grid(a.T, a.BH);
+    const dim3 grid(a.BH * a.T);
     select_proj_kernel<D, DS, REG><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
@@ -704,7 +722,7 @@ cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEn
     cudaError_t e = cudaFuncSetAttribute(select_given_kernel<REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select_given)"; return e; }
-    dim3 grid(a.T, a.BH);
+    const dim3 grid(a.BH * a.T);
     select_given_kernel<REG><<<grid, 128, smem, env.stream>>>(p);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
@@ -720,7 +738,7 @@ cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelE
 
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
     SelParams p;
-    p.N = a.N; p.C = a.C; p.T = a.T; p.F = a.F; p.topk = a.topk;
+    p.BH = a.BH; p.N = a.N; p.C = a.C; p.T = a.T; p.F = a.F; p.topk = a.topk;
     p.score_scale = a.score_scale;
     p.scores = a.scores;
     p.sel_idx = a.sel_idx; p.sel_logg = a.sel_logg;

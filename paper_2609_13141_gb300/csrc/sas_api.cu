@@ -98,6 +98,7 @@ struct sas_handle {
     int32_t* sel_idx = nullptr;
     float* sel_logg = nullptr;
     int* status = nullptr;
+    int* sched = nullptr;       // attention work counters (zero between launches)
     // MLP hidden activation
     void* hidden = nullptr;
     size_t hidden_bytes = 0;
@@ -198,6 +199,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     *out = nullptr;
     const sas_config& c = *cfg;
     if (c.B < 1 || c.H < 1 || c.N < 1) return SAS_ERR_INVALID_ARG;
+    if (c.N > (1 << 30)) return SAS_ERR_UNSUPPORTED;   // block indices stay below 2^24
     if (c.block != 64) return SAS_ERR_UNSUPPORTED;
     if (c.d != 64 && c.d != 128) return SAS_ERR_UNSUPPORTED;
     if (c.topk < 0) return SAS_ERR_INVALID_ARG;
@@ -209,6 +211,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
     const long long BH = static_cast<long long>(c.B) * c.H;
     if (BH > (1LL << 30) || BH * c.N > (1LL << 40)) return SAS_ERR_UNSUPPORTED;
+    if (BH * ((c.N + 127) / 128) > 0x7fffffffLL) return SAS_ERR_UNSUPPORTED;   // (head, tile) pairs index a 1-D grid
 
     sas_handle* h = new sas_handle();
     h->cfg = c;
@@ -233,6 +236,8 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (e == cudaSuccess) e = alloc(&h->sel_logg, rows * (c.topk > 0 ? c.topk : 1) * 4);
     if (e == cudaSuccess) e = alloc(&h->status, 16);
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, 16);
+    if (e == cudaSuccess) e = alloc(&h->sched, 16);
+    if (e == cudaSuccess) e = cudaMemset(h->sched, 0, 16);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         sas_status s = e == cudaErrorMemoryAllocation ? SAS_ERR_OOM : SAS_ERR_CUDA;
@@ -252,6 +257,7 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->sel_idx);
     cudaFree(h->sel_logg);
     cudaFree(h->status);
+    cudaFree(h->sched);
     cudaFree(h->hidden);
     for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
     delete h;
@@ -307,6 +313,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
     aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
     aa.sm_scale = h->sm_scale;
+    aa.sched = h->sched;
     e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     return SAS_OK;

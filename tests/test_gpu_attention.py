@@ -54,6 +54,14 @@ def test_given_scores_iid_worst_case_union():
     _given_case(1, 2, 900, 128, 5, TRAIN, regime="R3", seed=4)
 
 
+@pytest.mark.parametrize("d,mode", [(128, TRAIN), (64, INFER)])
+def test_persistent_grid_many_tiles_per_cta(d, mode):
+    # 2 x 96 heads x 5 tiles = 960 work items, more than two per SM, so every CTA
+    # runs several tiles back to back; N = 8*64 + 30 makes C = 9 odd, so the last
+    # tile of every head visits a single (diagonal) block
+    _given_case(2, 96, 542, d, 3, mode, seed=31)
+
+
 def test_k0_is_local_attention():
     _given_case(1, 1, 600, 128, 0, TRAIN, seed=5)
 
