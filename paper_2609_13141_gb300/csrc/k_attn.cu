@@ -12,14 +12,20 @@
 // the tile's union list from the selection pass (blocks < 2t, ascending),
 // then the diagonal blocks 2t and 2t+1.  Per visited 64-key block:
 //   * warp 0 TMA-loads K (two-stage ring), warp 1 TMA-loads V (own ring);
-//   * warp 2 (one lane) issues S = Q K^T into one of two TMEM score buffers
-//     (tcgen05.mma M=128 N=64 K=16 steps), and later O += P V into the TMEM
-//     output accumulator (M=128 N=d, V as an MN-major operand);
+//   * warp 2 (one lane) issues S = Q K^T into the TMEM score buffer
+//     (tcgen05.mma M=128 N=64 K=16 steps); warp 3 (one lane) issues
+//     O += P V into the TMEM output accumulator (M=128 N=d, P read from TMEM,
+//     V as an MN-major operand).  The two streams use different accumulators
+//     and are issued independently: one thread cannot issue the small score
+//     MMAs as fast as the tensor pipe runs them;
 //   * warps 4-7, one thread per query row (TMEM lane), read the score row,
 //     add the row's gate or mask (each thread walks its own ascending list of
-//     kept blocks), run the online softmax in the log2 domain, write P as bf16
-//     into a 128-byte-swizzled shared tile for the next MMA and rescale the
-//     TMEM output row when the running maximum grows by more than 2^8.
+//     kept blocks), run the online softmax in the log2 domain, write P as
+//     packed bf16 into one of two TMEM P buffers and rescale the TMEM output
+//     row when the running maximum grows by more than 2^8.
+// The score buffer is released as soon as the softmax warps have loaded it,
+// so the next block's QK runs during this block's softmax; a P buffer is
+// reused once the PV two blocks back has read it.
 // The epilogue divides by the row sum and writes bf16 O and fp32 LSE.
 #include <math_constants.h>
 
@@ -37,7 +43,8 @@ constexpr float kLn2 = 0.69314718055994531f;
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
 constexpr int kMaxStages = 4;                // capacity of the K / V ring barrier arrays
 constexpr int kItemSlots = 4;                // work items in flight between the fetching thread and the other roles
-constexpr int kItemReaders = 7;              // K producer, V producer, MMA issuer, four softmax warps
+constexpr int kItemReaders = 8;              // K and V producers, QK and PV issuers, four softmax warps
+constexpr int kRing = 8;                     // kept-list entries staged ahead per row
 
 template <int D>
 struct AttnCfg {
@@ -48,12 +55,16 @@ struct AttnCfg {
     static_assert(KST <= kMaxStages && VST <= kMaxStages, "ring barrier arrays");
     static constexpr int OFF_K = Q_BYTES;
     static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
-    static constexpr int OFF_CTL = OFF_V + VST * KV_BYTES;
+    // per row, the next kRing kept blocks and log-gates: int/float [kRing][kBM] each
+    static constexpr int OFF_RING = OFF_V + VST * KV_BYTES;
+    static constexpr int OFF_CTL = OFF_RING + 2 * kRing * kBM * 4;
     // All shared state lives in the dynamic region (no static shared memory),
     // so that two CTAs fit on one SM.
     static constexpr int SMEM = OFF_CTL + 512;
-    static constexpr int TMEM_COLS = 256;    // S0 [0,64) S1 [64,128) O [128,128+D)
-    static constexpr int TMEM_O = 128;
+    static constexpr int TMEM_COLS = 256;    // O [0,D)  S [128,192)  P0 [192,224)  P1 [224,256)
+    static constexpr int TMEM_O = 0;
+    static constexpr int TMEM_S = 128;
+    static constexpr int TMEM_P = 192;       // P buffer b at TMEM_P + 32 b (64 keys packed in pairs)
     static constexpr uint32_t IDESC_S = idesc_bf16(kBM, kBN, 0, 0);
     static constexpr uint32_t IDESC_O = idesc_bf16(kBM, D, 0, 1);
 };
@@ -61,7 +72,7 @@ struct AttnCfg {
 // Barriers and flags at the end of the dynamic shared-memory region.
 struct AttnCtl {
     uint64_t q_full, q_empty, k_full[kMaxStages], k_empty[kMaxStages], v_full[kMaxStages], v_empty[kMaxStages];
-    uint64_t s_full[2], s_free[2], p_full[2], o_ready[2], drain_bar;
+    uint64_t s_full, s_free, p_full[2], pv_done[2], drain_bar;
     uint64_t item_full[kItemSlots], item_empty[kItemSlots];
     int item[kItemSlots];   // work item (or -1: no more work) published to the other roles
     uint32_t tmem_base;
@@ -151,10 +162,10 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     uint64_t* k_empty = ctl.k_empty;
     uint64_t* v_full = ctl.v_full;
     uint64_t* v_empty = ctl.v_empty;
-    uint64_t* s_full = ctl.s_full;
-    uint64_t* s_free = ctl.s_free;
-    uint64_t* p_full = ctl.p_full;
-    uint64_t* o_ready = ctl.o_ready;
+    uint64_t& s_full = ctl.s_full;     // QK of block g done
+    uint64_t& s_free = ctl.s_free;     // all four softmax warps have loaded the scores of block g
+    uint64_t* p_full = ctl.p_full;     // P of block g written to P buffer g % 2
+    uint64_t* pv_done = ctl.pv_done;   // PV of block g done (O updated, P buffer g % 2 read)
     uint64_t& drain_bar = ctl.drain_bar;
     uint32_t& tmem_base_sh = ctl.tmem_base;
     int& abort_flag = ctl.abort_flag;
@@ -167,13 +178,13 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
         mbar_init(&q_empty, 1);
         for (int s = 0; s < Cfg::KST; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
         for (int s = 0; s < Cfg::VST; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
+        mbar_init(&s_full, 1);
+        mbar_init(&s_free, 4);
         for (int s = 0; s < 2; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 1);
-            mbar_init(&o_ready[s], 1);
+            mbar_init(&pv_done[s], 1);
             mbar_init(&p_full[s], 4);
         }
-        mbar_init(&drain_bar, 1);
+        mbar_init(&drain_bar, 2);   // both MMA issuers
         for (int s = 0; s < kItemSlots; ++s) {
             mbar_init(&ctl.item_full[s], 1);
             mbar_init(&ctl.item_empty[s], kItemReaders);
@@ -273,33 +284,10 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 mbar_wait_drain(&v_full[q % Cfg::VST], (q / Cfg::VST) & 1, p.limit, p.status);
         }
     } else if (warp == 2 && lane == 0) {
-        // ---------------- MMA issuer: QK of block g, then PV of block g-1; a tile's
-        // last PV is issued before the next tile starts, so that the softmax
-        // warps' epilogue does not wait for the next Q tile to arrive.
-        const uint32_t q_addr = smem_u32(smem);
-        // O += P_gb V_gb; `first` starts a new tile's accumulator
-        auto issue_pv = [&](int gb, bool first) -> bool {
-            const int vs = gb % Cfg::VST;
-            // p_full[gb&1] cannot run two phases ahead: the softmax needs QK_{gb+2},
-            // issued only after this wait, before it can arrive there again.
-            if (!mbar_wait(&p_full[gb & 1], (gb >> 1) & 1, wc)) return false;
-            if (!mbar_wait(&v_full[vs], (gb / Cfg::VST) & 1, wc)) return false;
-            tc_fence_after();
-            const uint32_t v_addr = smem_u32(smem + Cfg::OFF_V + vs * Cfg::KV_BYTES);
-#pragma unroll
-            for (int k = 0; k < kBN / 16; ++k) {
-                // P_gb sits in TMEM over the first 32 columns of score buffer gb & 1
-                // (16 keys = 8 packed columns per step).  V is MN-major (d contiguous):
-                // 16 keys = two 8-row atoms; the two 64-wide d halves sit kBN*128 bytes apart.
-                umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + (gb & 1) * 64 + k * 8,
-                             smem_desc_sw128(v_addr + k * 2048, kBN * 128, 1024), Cfg::IDESC_O,
-                             (!first || k > 0) ? 1u : 0u);
-            }
-            umma_commit(&o_ready[gb & 1]);
-            umma_commit(&v_empty[vs]);
-            umma_commit(&s_free[gb & 1]);   // score buffer (and P in it) free for QK_{gb+2}
-            return true;
-        };
+        // ---------------- QK issuer: S = Q K_g^T for every visited block g, once the
+        // softmax warps have loaded S_{g-1}
+        const uint64_t dq0 = smem_desc_sw128(smem_u32(smem), 16, 1024);
+        const uint64_t dk0 = smem_desc_sw128(smem_u32(smem + Cfg::OFF_K), 16, 1024);
         int g = 0, tc = 0;
         bool ok = true;
         for (int r = 0; ok; ++r) {
@@ -307,33 +295,64 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (!read_item(ctl, r, wc, w)) { ok = false; break; }
             mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
-            const TileRef x = tile_ref(p, w);
-            const int n = tile_blocks(p, x);
+            const int n = tile_blocks(p, tile_ref(p, w));
             if (!mbar_wait(&q_full, tc & 1, wc)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
-                // S[gb%2] = Q K_gb^T
                 const int gb = g + j;
                 const int s = gb % Cfg::KST;
-                const int sb = gb & 1;
                 if (!mbar_wait(&k_full[s], (gb / Cfg::KST) & 1, wc)) { ok = false; break; }
-                if (!mbar_wait(&s_free[sb], ((gb >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
+                if (gb >= 1 && !mbar_wait(&s_free, (gb - 1) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t k_addr = smem_u32(smem + Cfg::OFF_K + s * Cfg::KV_BYTES);
+                // descriptors advance by (byte offset >> 4) in their start-address field
+                const uint64_t dk = dk0 + static_cast<uint64_t>((s * Cfg::KV_BYTES) >> 4);
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
                     const uint32_t off_q = (k >> 2) * (kBM * 128) + (k & 3) * 32;
                     const uint32_t off_k = (k >> 2) * (kBN * 128) + (k & 3) * 32;
-                    umma_bf16(tmem_base + sb * 64, smem_desc_sw128(q_addr + off_q, 16, 1024),
-                              smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                    umma_bf16(tmem_base + Cfg::TMEM_S, dq0 + (off_q >> 4), dk + (off_k >> 4), Cfg::IDESC_S, k > 0);
                 }
-                umma_commit(&s_full[sb]);
+                umma_commit(&s_full);
                 umma_commit(&k_empty[s]);
                 if (j == n - 1) umma_commit(&q_empty);   // Q slot free for the next tile
-                if (j >= 1 && !issue_pv(gb - 1, j == 1)) { ok = false; break; }
             }
-            if (ok && !issue_pv(g + n - 1, n == 1)) ok = false;
             g += n;
             ++tc;
+        }
+        umma_commit(&drain_bar);
+        mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+    } else if (warp == 3 && lane == 0) {
+        // ---------------- PV issuer: O += P_g V_g for every visited block g; the first
+        // block of a tile starts a new accumulator
+        const uint64_t dv0 = smem_desc_sw128(smem_u32(smem + Cfg::OFF_V), kBN * 128, 1024);
+        int g = 0;
+        bool ok = true;
+        for (int r = 0; ok; ++r) {
+            int w;
+            if (!read_item(ctl, r, wc, w)) { ok = false; break; }
+            mbar_arrive(&ctl.item_empty[r % kItemSlots]);
+            if (w < 0) break;
+            const int n = tile_blocks(p, tile_ref(p, w));
+            for (int j = 0; j < n; ++j) {
+                const int gb = g + j;
+                const int vs = gb % Cfg::VST;
+                // p_full[gb&1] cannot run two phases ahead: the softmax writes P_{gb+2}
+                // only after PV_gb (issued after this wait) has read the buffer.
+                if (!mbar_wait(&p_full[gb & 1], (gb >> 1) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait(&v_full[vs], (gb / Cfg::VST) & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+                const uint64_t dv = dv0 + static_cast<uint64_t>((vs * Cfg::KV_BYTES) >> 4);
+#pragma unroll
+                for (int k = 0; k < kBN / 16; ++k) {
+                    // P_gb sits in P buffer gb & 1 (16 keys = 8 packed columns per step).
+                    // V is MN-major (d contiguous): 16 keys = two 8-row atoms (2048 bytes);
+                    // the two 64-wide d halves sit kBN*128 bytes apart.
+                    umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + Cfg::TMEM_P + (gb & 1) * 32 + k * 8,
+                                 dv + ((k * 2048) >> 4), Cfg::IDESC_O, (j > 0 || k > 0) ? 1u : 0u);
+                }
+                umma_commit(&pv_done[gb & 1]);
+                umma_commit(&v_empty[vs]);
+            }
+            g += n;
         }
         umma_commit(&drain_bar);
         mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
@@ -363,14 +382,28 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             const long long row_off = static_cast<long long>(x.bh) * p.N + i;
             const int32_t* my_idx = p.sel_idx + row_off * p.topk;
             const float* my_lg = p.sel_logg + row_off * p.topk;
-            // The row's next two kept blocks (a two-entry queue).  Loads are
-            // predicated into pre-set registers and read one or more iterations
-            // later, so their latency is not paid where they are issued.
-            int sp = 0;
-            int km0 = 0x7fffffff, km1 = 0x7fffffff;
-            float kl0 = 0.f, kl1 = 0.f;
-            if (nsel > 0) { km0 = __ldg(my_idx); kl0 = __ldg(my_lg); }
-            if (nsel > 1) { km1 = __ldg(my_idx + 1); kl1 = __ldg(my_lg + 1); }
+            // The row's kept list is staged kRing entries ahead in a shared ring
+            // (entry e in slot e % kRing, one commit group per entry), so the walk
+            // below only reads entries that have landed long ago.  Every entry of
+            // the list is consumed within the tile (each kept block is visited).
+            int* ring_i = reinterpret_cast<int*>(smem + Cfg::OFF_RING) + r_row;
+            float* ring_l = reinterpret_cast<float*>(smem + Cfg::OFF_RING + kRing * kBM * 4) + r_row;
+#pragma unroll
+            for (int e = 0; e < kRing; ++e) {
+                if (e < nsel) {
+                    cp_async4(ring_i + e * kBM, my_idx + e);
+                    cp_async4(ring_l + e * kBM, my_lg + e);
+                }
+                cp_async_commit();
+            }
+            int sp = 0;   // current entry; groups issued so far = sp + kRing
+            int km0 = 0x7fffffff;
+            float kl0 = 0.f;
+            if (nsel > 0) {
+                cp_async_wait<kRing - 1>();
+                km0 = ring_i[0];
+                kl0 = ring_l[0];
+            }
 
             float m_use = -CUDART_INF_F;
             float l = 0.f;
@@ -379,7 +412,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (x.U > 0) raw_next = __ldg(x.ulist);
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
-                const int sb = gb & 1;
+                const int pb = gb & 1;
                 const int m = j < x.U ? raw_next : 2 * t + (j - x.U);
                 if (j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
                 // gate (log2 units) and the last visible key column of block m for this row
@@ -389,11 +422,20 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                     if (m == km0) {
                         bias = train ? kl0 * kLog2e : 0.f;
                         lim = kBN - 1;
+                        // refill the finished slot with entry sp + kRing, then step to sp + 1
+                        const int e = sp + kRing;
+                        if (e < nsel) {
+                            cp_async4(ring_i + (sp % kRing) * kBM, my_idx + e);
+                            cp_async4(ring_l + (sp % kRing) * kBM, my_lg + e);
+                        }
+                        cp_async_commit();
                         ++sp;
-                        km0 = km1;
-                        kl0 = kl1;
-                        km1 = 0x7fffffff;
-                        if (sp + 1 < nsel) { km1 = __ldg(my_idx + sp + 1); kl1 = __ldg(my_lg + sp + 1); }
+                        km0 = 0x7fffffff;
+                        if (sp < nsel) {
+                            cp_async_wait<kRing - 1>();
+                            km0 = ring_i[(sp % kRing) * kBM];
+                            kl0 = ring_l[(sp % kRing) * kBM];
+                        }
                     } else {
                         lim = -1;
                     }
@@ -404,26 +446,33 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 }
                 const bool active = lim >= 0;
 
-                if (!mbar_wait_warp(&s_full[sb], (gb >> 1) & 1, wc)) { ok = false; break; }
+                // s_full cannot run a phase ahead: QK_{gb+1} waits for this warp's s_free arrival
+                if (!mbar_wait_warp(&s_full, gb & 1, wc)) { ok = false; break; }
+                // P buffer gb & 1 is free once PV_{gb-2} has read it
+                if (gb >= 2 && !mbar_wait_warp(&pv_done[pb], ((gb - 2) >> 1) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
                 const bool warp_active = __any_sync(0xffffffffu, active);
-                float xs[64];
-                if (warp_active) {
-                    uint32_t u0[32], u1[32];
-                    tmem_ld32(lane_addr + sb * 64, u0);
-                    tmem_ld32(lane_addr + sb * 64 + 32, u1);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int k = 0; k < 32; ++k) {
-                        xs[k] = __uint_as_float(u0[k]);
-                        xs[k + 32] = __uint_as_float(u1[k]);
-                    }
-                }
                 bool need = false;
                 float m_new = m_use;
                 float rs = 0.f;
                 uint32_t pk[32];   // P row as packed bf16 pairs
                 if (warp_active) {
+                    float xs[64];
+                    {
+                        uint32_t u0[32], u1[32];
+                        tmem_ld32(lane_addr + Cfg::TMEM_S, u0);
+                        tmem_ld32(lane_addr + Cfg::TMEM_S + 32, u1);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) {
+                            xs[k] = __uint_as_float(u0[k]);
+                            xs[k + 32] = __uint_as_float(u1[k]);
+                        }
+                    }
+                    // the score buffer is free for the next block's QK
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&s_free);
                     // causal mask on the diagonal block only
                     if (__any_sync(0xffffffffu, lim >= 0 && lim < kBN - 1)) {
 #pragma unroll
@@ -459,6 +508,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                     f32x2_split(acc[3], s6, s7);
                     rs = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
                 } else {
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&s_free);
 #pragma unroll
                     for (int k = 0; k < 32; ++k) pk[k] = 0u;
                 }
@@ -467,8 +518,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
 
                 if (j > 0 && __any_sync(0xffffffffu, need)) {
                     // Rescaling O needs PV_{gb-1} done.  PV_{gb-1} is the ((gb-1)/2)-th phase of
-                    // o_ready[(gb-1)&1]; that barrier cannot move past it before p_full(gb+1).
-                    if (!mbar_wait_warp(&o_ready[(gb - 1) & 1], ((gb - 1) >> 1) & 1, wc)) { ok = false; break; }
+                    // pv_done[(gb-1)&1]; that barrier cannot move past it before p_full(gb+1).
+                    if (!mbar_wait_warp(&pv_done[(gb - 1) & 1], ((gb - 1) >> 1) & 1, wc)) { ok = false; break; }
                     tc_fence_after();
 #pragma unroll 1
                     for (int cc = 0; cc < D / 32; ++cc) {
@@ -484,12 +535,12 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 l = l * factor + rs;
                 m_use = m_new;
 
-                // P row (64 bf16, packed in pairs) into TMEM over this row's scores
-                tmem_st32(lane_addr + sb * 64, pk);
+                // P row (64 bf16, packed in pairs) into P buffer gb & 1
+                tmem_st32(lane_addr + Cfg::TMEM_P + pb * 32, pk);
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&p_full[sb]);
+                if (lane == 0) mbar_arrive(&p_full[pb]);
             }
             if (!ok) break;
 
@@ -497,7 +548,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             // this warp has arrived on p_full for that tile's first block, i.e. after
             // the reads below have completed.  (Its first QK may already run.)
             const int gl = g + n - 1;
-            if (!mbar_wait_warp(&o_ready[gl & 1], (gl >> 1) & 1, wc)) { ok = false; break; }
+            if (!mbar_wait_warp(&pv_done[gl & 1], (gl >> 1) & 1, wc)) { ok = false; break; }
             tc_fence_after();
             const float inv = 1.f / l;
             bf16* orow = p.O + row_off * D;
