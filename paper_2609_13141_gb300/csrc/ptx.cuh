@@ -47,15 +47,28 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
         : "memory");
 }
 
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+// suspend_ns > 0 lets the waiting thread sleep (up to that many ns, woken when
+// the phase completes) instead of returning at once; a thread that polls can
+// take issue slots from the warps doing the work.
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity, uint32_t suspend_ns = 0) {
     uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
+    if (suspend_ns == 0) {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+    } else {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity), "r"(suspend_ns)
+            : "memory");
+    }
     return ok != 0;
 }
 
@@ -69,11 +82,12 @@ struct WaitCtl {
 // Waits for the phase with the given parity to complete.  Returns false if
 // the CTA is aborting (another wait ran out) or this wait ran out, in which
 // case the status word and the abort flag are set.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const WaitCtl& w) {
-    if (mbar_try_wait(bar, parity)) return true;
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const WaitCtl& w,
+                                          uint32_t suspend_ns = 0) {
+    if (mbar_try_wait(bar, parity, suspend_ns)) return true;
     const long long t0 = clock64();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait(bar, parity, suspend_ns)) return true;
         if (*w.abort_flag) return false;
         if (clock64() - t0 > w.limit) {
             *w.abort_flag = 1;
@@ -85,15 +99,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
 
 // Warp-uniform wait for code that follows with warp-collective instructions
 // (tcgen05.ld/st, vote): every lane gets the same answer.
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, const WaitCtl& w) {
-    const bool ok = mbar_wait(bar, parity, w);
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, const WaitCtl& w,
+                                               uint32_t suspend_ns = 0) {
+    const bool ok = mbar_wait(bar, parity, w, suspend_ns);
     return __all_sync(0xffffffffu, ok);
 }
 
 // Wait used only while draining at exit: ignores the abort flag.
-__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity, long long limit, int* status) {
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity, long long limit, int* status,
+                                                uint32_t suspend_ns = 0) {
     const long long t0 = clock64();
-    while (!mbar_try_wait(bar, parity)) {
+    while (!mbar_try_wait(bar, parity, suspend_ns)) {
         if (clock64() - t0 > limit) {
             atomicExch(status, kStatusTimeout);
             return false;
