@@ -59,3 +59,9 @@ def test_mlp_stress_config_sampled_rows():
     rows = np.random.default_rng(0).choice(16384, size=48, replace=False)
     rows = np.concatenate([rows, [0, 127, 128, 16383]])
     _run(16384, 3072, 12288, bias=False, rows=rows)
+
+
+def test_mlp_multi_tile_ragged_rows_with_bias():
+    # eight 128-row tiles, the last with 104 rows; N = 2048 and 512 give several
+    # 256-wide output tiles per row block
+    _run(1000, 512, 2048, bias=True, seed=3)
