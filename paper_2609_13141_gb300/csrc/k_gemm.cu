@@ -12,7 +12,10 @@
 //   * warp 1 (one lane) issues tcgen05.mma (M=128, N=BN, K=16) into one of
 //     two TMEM accumulators and releases stages with tcgen05.commit;
 //   * warps 2-5 drain the other accumulator (tcgen05.ld), apply bias/GELU in
-//     fp32 and store bf16, overlapping the next tile's main loop.
+//     fp32, write bf16 into a per-warp 128-byte-swizzled staging tile and send
+//     each 32 x 64 block out with a TMA tensor store (per-thread row stores
+//     scattered over 32 rows cost 6% of the GEMM), overlapping the next tile's
+//     main loop.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -30,7 +33,10 @@ struct GemmCfg {
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
     static constexpr int TMEM_COLS = 2 * BN;
-    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;
+    // per epilogue warp two 32-row x 64-column bf16 staging tiles (4 KB each)
+    static constexpr int OFF_STAGING = STAGES * STAGE_BYTES;
+    static constexpr int STAGING_BYTES = 4 * 2 * 4096;
+    static constexpr int SMEM = OFF_STAGING + STAGING_BYTES + 1024;
     static constexpr uint32_t IDESC = idesc_bf16(kBM, BN, 0, 0);
 };
 
@@ -70,7 +76,8 @@ __device__ __forceinline__ float gelu_erf(float x) {
 
 template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
-gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, GemmParams p) {
+gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+            const __grid_constant__ CUtensorMap mapC, GemmParams p) {
     using Cfg = GemmCfg<BN>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ uint64_t full_bar[Cfg::STAGES], empty_bar[Cfg::STAGES];
@@ -168,11 +175,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         umma_commit(&drain_bar);
         mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
     } else if (warp >= 2) {
-        // ---------------- epilogue: TMEM -> registers -> bias/GELU -> bf16 global
+        // ---------------- epilogue: TMEM -> registers -> bias/GELU -> bf16 -> staging -> TMA store
         const int q = warp & 3;
-        const int row_in_tile = q * 32 + lane;
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+        uint8_t* staging = smem + Cfg::OFF_STAGING + q * 2 * 4096;
+        if (lane == 0) tma_prefetch_desc(&mapC);
         int it = 0;
+        int nst = 0;   // stores issued by this warp (staging buffer = nst & 1)
         for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
             const int acc = it & 1;
             const uint32_t aph = (it >> 1) & 1;
@@ -180,28 +189,32 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
             tc_fence_after();
             int b, m, n;
             tile_coords(t, m_tiles, n_tiles, b, m, n);
-            const int grow = m * kBM + row_in_tile;
-            const bool valid = grow < p.M;
-            bf16* crow = p.C + b * p.c_batch_stride + static_cast<long long>(grow) * p.ldc + n * BN;
 #pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(lane_addr + acc * BN + c * 32, r);
-                tmem_wait_ld();
-                float v[32];
+            for (int cg = 0; cg < BN / 64; ++cg, ++nst) {
+                uint8_t* buf = staging + (nst & 1) * 4096;
+                // the store issued from this buffer two groups ago has finished reading it
+                if (lane == 0) bulk_wait_read<1>();
+                __syncwarp();
+#pragma unroll 1
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int c = cg * 2 + hh;
+                    uint32_t r[32];
+                    tmem_ld32(lane_addr + acc * BN + c * 32, r);
+                    tmem_wait_ld();
+                    float v[32];
 #pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-                if (p.bias != nullptr) {
-                    const bf16* bp = p.bias + n * BN + c * 32;
+                    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+                    if (p.bias != nullptr) {
+                        const bf16* bp = p.bias + n * BN + c * 32;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] += __bfloat162float(bp[j]);
-                }
-                if (p.gelu) {
+                        for (int j = 0; j < 32; ++j) v[j] += __bfloat162float(bp[j]);
+                    }
+                    if (p.gelu) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] = gelu_erf(v[j]);
-                }
-                if (valid) {
-                    uint4* dst = reinterpret_cast<uint4*>(crow + c * 32);
+                        for (int j = 0; j < 32; ++j) v[j] = gelu_erf(v[j]);
+                    }
+                    // row `lane` of the staging tile: 16-byte chunk k of the row at k ^ (lane & 7)
+                    uint8_t* row = buf + lane * 128;
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         uint4 w;
@@ -209,13 +222,22 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
                         w.y = pack_bf16x2(v[8 * j + 2], v[8 * j + 3]);
                         w.z = pack_bf16x2(v[8 * j + 4], v[8 * j + 5]);
                         w.w = pack_bf16x2(v[8 * j + 6], v[8 * j + 7]);
-                        dst[j] = w;
+                        const int k = hh * 4 + j;
+                        *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) = w;
                     }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                // rows past M are clipped by the tensor store
+                if (lane == 0) {
+                    tma_store_3d(&mapC, buf, n * BN + cg * 64, m * kBM + q * 32, b);
+                    bulk_commit();
                 }
             }
             tc_fence_before();
             mbar_arrive(&tempty_bar[acc]);
         }
+        if (lane == 0) bulk_wait_all();
     }
     __syncthreads();
     if (warp == 1) {
@@ -244,10 +266,15 @@ cudaError_t launch_bn(const GemmProblem& p, const KernelEnv& env, const char** e
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(gemm)"; return e; }
         attr_set = true;
     }
-    CUtensorMap ma, mb;
+    if (p.ldc != p.N || (p.batches > 1 && p.c_batch_stride != static_cast<long long>(p.M) * p.N)) {
+        *err = "gemm: C must be a dense [batches][M][N] tensor";
+        return cudaErrorInvalidValue;
+    }
+    CUtensorMap ma, mb, mc;
     const int nb = p.b_mod;
     if (make_tmap_bf16_3d(&ma, p.A, p.K, p.M, p.batches, kBK, kBM) != 0) { *err = "tensor map A"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mb, p.B, p.K, p.N, nb, kBK, BN) != 0) { *err = "tensor map B"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mc, p.C, p.N, p.M, p.batches, 64, 32) != 0) { *err = "tensor map C"; return cudaErrorInvalidValue; }
     GemmParams gp;
     gp.C = static_cast<bf16*>(p.C);
     gp.bias = static_cast<const bf16*>(p.bias);
@@ -258,7 +285,7 @@ cudaError_t launch_bn(const GemmProblem& p, const KernelEnv& env, const char** e
     const long long tiles = static_cast<long long>(p.batches) * ((p.M + kBM - 1) / kBM) * (p.N / BN);
     int grid = p.max_ctas > 0 ? p.max_ctas : sm_count();
     if (tiles < grid) grid = static_cast<int>(tiles);
-    gemm_kernel<BN><<<grid, kThreads, Cfg::SMEM, env.stream>>>(ma, mb, gp);
+    gemm_kernel<BN><<<grid, kThreads, Cfg::SMEM, env.stream>>>(ma, mb, mc, gp);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) *err = "gemm launch";
     return e;
