@@ -43,7 +43,7 @@ WORKLOADS = {
 }
 
 
-def algorithmic_flops(w):
+def algorithmic_flops(w, learned=True):
     """Work the method itself must do for one layer (no tile-union or padding waste).
 
     Attention per (batch, head) row i with c = floor(i/64):
@@ -51,6 +51,7 @@ def algorithmic_flops(w):
       2 d_sel c                                    selector scores against c summaries
       2 d d_sel                                    query projection
     plus 2 d d_sel per full key block (key projection), and the MLP 4 T D F.
+    With given scores (learned=False) the selector terms are not part of the layer.
     """
     N, d, K, ds = w["N"], w["d"], w["topk"], w["d_sel"]
     BH = w["B"] * w["H"]
@@ -61,6 +62,8 @@ def algorithmic_flops(w):
         attn += 4 * d * (cur + rows * 64 * min(K, c))
         sel += rows * (2 * ds * c + 2 * d * ds)
     sel += (N // 64) * 2 * d * ds
+    if not learned:
+        sel = 0
     mlp = 4 * w["B"] * N * w["D"] * w["F"]
     return {"attention": BH * attn, "selector": BH * sel, "mlp": mlp,
             "total": BH * (attn + sel) + mlp}
@@ -177,31 +180,46 @@ def run_ours(args, w, rank, world):
 
     B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
     T = B * N
-    Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
+    learned = args.regime == "R2"
+    if learned:
+        # R2: block-correlated queries through the learned selector
+        Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
+        S = None
+    else:
+        # R1: block-coherent selector scores supplied by the caller
+        Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="iid")
+        S = synth.scores(B, H, N, (N + 63) // 64, seed=rank, regime="R1")
     Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
     X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
     Qd, Kd, Vd, Wqd, Wkd = (t.to(dev) for t in (Q, Kk, V, Wq, Wk))
+    Sd = None if S is None else S.to(dev)
     Xd, W1d, W2d = X.to(dev), W1.to(dev), W2.to(dev)
     Od = torch.empty_like(Qd)
     LSEd = torch.empty(B, H, N, device=dev, dtype=torch.float32)
     Yd = torch.empty(T, D, device=dev, dtype=torch.bfloat16)
     flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
 
-    layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
+    if learned:
+        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
+    else:
+        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN)
     h = layer.h
     stream = torch.cuda.current_stream(dev)
 
-    def step(Qx, Kx, Vx, Xx, O, Y):
-        sas.sas_attention_fwd(h, Qx, Kx, Vx, O, None, Wqd, Wkd, LSEd, None, None, stream)
+    def step(Qx, Kx, Vx, Xx, O, Y, Sx=None):
+        if learned:
+            sas.sas_attention_fwd(h, Qx, Kx, Vx, O, None, Wqd, Wkd, LSEd, None, None, stream)
+        else:
+            sas.sas_attention_fwd(h, Qx, Kx, Vx, O, Sx, None, None, LSEd, None, None, stream)
         sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
 
     for _ in range(max(args.warmup, 3)):
-        step(Qd, Kd, Vd, Xd, Od, Yd)
+        step(Qd, Kd, Vd, Xd, Od, Yd, Sd)
     torch.cuda.synchronize()
     # keep the GPU busy for ~1 s so the clock sampler sees it under load
     t_end = time.time() + 1.0
     while time.time() < t_end:
-        step(Qd, Kd, Vd, Xd, Od, Yd)
+        step(Qd, Kd, Vd, Xd, Od, Yd, Sd)
         torch.cuda.synchronize()
 
     sampler = ClockSampler(local)
@@ -217,7 +235,7 @@ def run_ours(args, w, rank, world):
     for k in range(args.steps):
         flush.zero_()
         starts[k].record(stream)
-        step(Qd, Kd, Vd, Xd, Od, Yd)
+        step(Qd, Kd, Vd, Xd, Od, Yd, Sd)
         ends[k].record(stream)
     torch.cuda.synchronize()
     if dist is not None:
@@ -234,22 +252,25 @@ def run_ours(args, w, rank, world):
     hO = torch.empty(Q.shape, dtype=torch.bfloat16).pin_memory()
     hY = torch.empty(T, D, dtype=torch.bfloat16).pin_memory()
     dQ, dK, dV, dX = (torch.empty_like(t) for t in (Qd, Kd, Vd, Xd))
+    hS = None if S is None else S.pin_memory()
+    dS = None if S is None else torch.empty_like(Sd)
+    copies = [(dQ, hQ), (dK, hK), (dV, hV), (dX, hX)] + ([] if S is None else [(dS, hS)])
     e_st = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     e_en = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for k in range(-2, args.steps):
         flush.zero_()
         if k >= 0:
             e_st[k].record(stream)
-        for dst, src in ((dQ, hQ), (dK, hK), (dV, hV), (dX, hX)):
+        for dst, src in copies:
             dst.copy_(src, non_blocking=True)
-        step(dQ, dK, dV, dX, Od, Yd)
+        step(dQ, dK, dV, dX, Od, Yd, dS)
         hO.copy_(Od, non_blocking=True)
         hY.copy_(Yd, non_blocking=True)
         if k >= 0:
             e_en[k].record(stream)
     torch.cuda.synchronize()
     e2e_ms = sum(s.elapsed_time(e) for s, e in zip(e_st, e_en)) / args.steps
-    h2d = sum(t.numel() * t.element_size() for t in (hQ, hK, hV, hX))
+    h2d = sum(src.numel() * src.element_size() for _, src in copies)
     d2h = hO.numel() * 2 + hY.numel() * 2
 
     # tile-union statistics of the last forward (executed vs algorithmic work)
@@ -263,7 +284,7 @@ def run_ours(args, w, rank, world):
             dist.destroy_process_group()
         return None
 
-    fl = algorithmic_flops(w)
+    fl = algorithmic_flops(w, learned)
     tflop = fl["total"] / 1e12
     value = job_throughput(tflop, world, ms)
     per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None)} for k, (n, t) in kt.items()}
@@ -283,10 +304,13 @@ def run_ours(args, w, rank, world):
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; R2 block-correlated queries, N(0,1) K/V/X, "
-        "weights N(0,0.02))",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": ("synthetic (seeded; R2 block-correlated queries, N(0,1) K/V/X, weights N(0,0.02))" if learned else
+                 "synthetic (seeded; R1 block-coherent selector scores s = u[block] + 0.05 eps given by the caller, "
+                 "N(0,1) Q/K/V/X, weights N(0,0.02))"),
         "config": {"workload": w["name"], "B": B, "H": H, "N": N, "d": d, "block": 64, "topk": K, "d_sel": ds,
-                   "mlp": [T, D, F, D], "selector": "meanpool_proj", "l2": "flushed between timed steps (256 MiB write)",
+                   "mlp": [T, D, F, D], "selector": "meanpool_proj" if learned else "scores_given (R1)",
+                   "l2": "flushed between timed steps (256 MiB write)",
                    "parallelism": f"replicas x{world}"},
         "roofline": roof,
         "attention_kernel": {"ms": round(a_avg, 4), "algorithmic_tflops": round(fl["attention"] / (a_avg / 1e3) / 1e12, 1),
@@ -300,7 +324,7 @@ def run_ours(args, w, rank, world):
         "clocks": clocks,
     }
     if not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget, learned=learned)
     if dist is not None:
         dist.destroy_process_group()
     return out
@@ -317,13 +341,13 @@ def _oracle_threads():
         return os.cpu_count() or 1
 
 
-def oracle_sample(w, budget_s, seed=0):
+def oracle_sample(w, budget_s, seed=0, learned=True):
     """Runs the oracle on a bounded sample of the workload and returns its
     throughput on the workload's FLOP mix.
 
     Half the budget goes to query rows of one head (selector scores for the
-    whole head, then the gated attention of random rows), half to random MLP
-    token rows.  Each part's rate (algorithmic FLOPs per second) is measured
+    whole head, or the head's given R1 scores, then the gated attention of
+    random rows), half to random MLP token rows.  Each part's rate (algorithmic FLOPs per second) is measured
     on its own; the full layer's time is attention FLOPs / attention rate +
     MLP FLOPs / MLP rate.  Returns (rate_flops_per_s, seconds, desc)."""
     import numpy as np
@@ -341,14 +365,19 @@ def oracle_sample(w, budget_s, seed=0):
     x, w1, w2 = f(X), f(W1), f(W2)
     rng = np.random.default_rng(seed)
 
-    t0 = time.perf_counter()
-    s = OR.selector_scores(q, k, wq, wk, 64)
-    a_flops = N * 2 * d * ds + (N // 64) * 2 * d * ds
+    if learned:
+        t0 = time.perf_counter()
+        s = OR.selector_scores(q, k, wq, wk, 64)
+        a_flops = N * 2 * d * ds + (N // 64) * 2 * d * ds
+    else:
+        s = f(synth.scores(1, 1, N, (N + 63) // 64, seed=seed, regime="R1")[0, 0])
+        t0 = time.perf_counter()
+        a_flops = 0
     rows_done = 0
     while time.perf_counter() - t0 < budget_s / 2:
         rows = rng.integers(0, N, size=32)
         OR.sas_attention_head(q, k, v, s, 64, K, rows=rows)
-        a_flops += sum(OR.attention_flops_row(int(i), 64, K, d, ds) for i in rows)
+        a_flops += sum(OR.attention_flops_row(int(i), 64, K, d, ds if learned else 0) for i in rows)
         rows_done += len(rows)
     a_time = time.perf_counter() - t0
     # the whole head's selector is amortised over the rows actually run
@@ -365,17 +394,18 @@ def oracle_sample(w, budget_s, seed=0):
     m_time = time.perf_counter() - t1
     m_rate = m_flops / m_time
 
-    fl = algorithmic_flops(w)
+    fl = algorithmic_flops(w, learned)
     full_time = (fl["attention"] + fl["selector"]) / a_rate + fl["mlp"] / m_rate
     rate = fl["total"] / full_time
-    desc = (f"oracle (numpy fp64): {rows_done} random query rows of one head (with that head's selector) "
+    how = "with that head's selector" if learned else "with that head's given R1 scores"
+    desc = (f"oracle (numpy fp64): {rows_done} random query rows of one head ({how}) "
             f"in {a_time:.1f} s and {tok_done} MLP token rows in {m_time:.1f} s; the two measured rates are "
             f"combined by the layer's FLOP mix")
     return rate, a_time + m_time, desc
 
 
-def cpu_baseline(w, budget_s=12.0):
-    rate, dt, desc = oracle_sample(w, budget_s)
+def cpu_baseline(w, budget_s=12.0, learned=True):
+    rate, dt, desc = oracle_sample(w, budget_s, learned=learned)
     return {"value": round(rate / 1e12, 8), "unit": UNIT, "cores": _oracle_threads(), "kind": "oracle",
             "sample": desc, "seconds": round(dt, 2)}
 
@@ -411,13 +441,21 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dit")
+    ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
+                    help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
+    ap.add_argument("--topk", type=int, default=None, help="override the workload's K")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=4.0)
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
-    w = WORKLOADS[args.workload]
+    w = dict(WORKLOADS[args.workload])
+    if args.topk is not None:
+        w["topk"] = args.topk
+        w["name"] = w["name"].replace("K=32", f"K={args.topk}")
+    if args.impl == "reference" and args.regime != "R2":
+        ap.error("the reference arm times the oracle on the learned-selector workload only")
     out = run_reference(args, w, rank, world) if args.impl == "reference" else run_ours(args, w, rank, world)
     if out is not None and rank == 0:
         print(json.dumps(out))
