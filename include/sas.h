@@ -20,6 +20,11 @@
  *     asynchronous on that stream; the library synchronises only inside
  *     sas_create / sas_destroy / sas_mlp_fwd's first use of a larger size /
  *     the sas_get_* readers.
+ *   - A handle's device workspace (kept lists, tile union lists, the attention
+ *     kernel's work counter, the MLP hidden activation) is reused by every
+ *     call on it, so calls on one handle must not overlap on the GPU: issue
+ *     them on one stream (or order the streams with events), and use one
+ *     handle per concurrently running stream.
  *   - Arguments are checked before anything is launched; on an argument error
  *     nothing is written and the call returns SAS_ERR_INVALID_ARG or
  *     SAS_ERR_UNSUPPORTED.  sas_last_error(h) then describes the problem.
