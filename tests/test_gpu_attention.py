@@ -62,6 +62,30 @@ def test_persistent_grid_many_tiles_per_cta(d, mode):
     _given_case(2, 96, 542, d, 3, mode, seed=31)
 
 
+def test_repeated_calls_on_one_handle_are_identical():
+    # Tiles are handed out from a counter in the handle; the last CTA of each
+    # launch returns it to zero.  Three calls in a row must give bit-identical
+    # outputs (and parity with the oracle on sampled rows).
+    B, H, N, d, topk = 2, 40, 1000, 128, 4
+    Q, K, V = synth.qkv(B, H, N, d, seed=41)
+    C = -(-N // 64)
+    S = synth.scores(B, H, N, C, seed=41, regime="R1")
+    dev = torch.device("cuda:0")
+    layer = sas.SasLayer(B, H, N, d, topk, mode=TRAIN, selector=sas.SAS_SEL_SCORES_GIVEN)
+    args = [t.to(dev) for t in (Q, K, V)]
+    outs = [layer.attention(*args, scores=S.to(dev)) for _ in range(3)]
+    torch.cuda.synchronize()
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    for o in outs[1:]:
+        assert torch.equal(o[0], outs[0][0]) and torch.equal(o[1], outs[0][1])
+    rows = P.sample_rows(N, n_random=64)
+    for bi, hi in [(0, 0), (1, 39)]:
+        ref = OR.sas_attention_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), P.f64(S[bi, hi]), 64,
+                                    topk, TRAIN, rows=rows)
+        P.compare_o(P.f64(outs[2][0][bi, hi].cpu())[rows], ref["O"], f"O[{bi},{hi}]")
+
+
 def test_k0_is_local_attention():
     _given_case(1, 1, 600, 128, 0, TRAIN, seed=5)
 
