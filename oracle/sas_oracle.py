@@ -13,6 +13,8 @@ What it computes (SAS, "Simple Attention Sparsification", arXiv 2609.13141):
   a3  causal log-gates     log g_m = s_m - LSE(s) over the row's history     (Eq. normalized_log_gate)
   a4  Top-K selection      I = TopK(g, K) = TopK(s, K)                       (Eq. selected_context; Alg. 1 / Alg. 2)
   a5  gated attention      o = softmax(q K_S^T + log g_S) V_S                (Eq. ours_train; Alg. 2 for the ungated form)
+      ablation forms       gate activation softmax / sigmoid / logit and gate position inner / outer
+                           (Sec. 4.2, Components of learnable ranking; Eq. general_gate)
   a6  dense MLP (not SAS)  Y = GELU(X W1^T + b1) W2^T + b2, exact-erf GELU
 
 Readings of points the paper leaves open (each one is also listed with its
@@ -53,6 +55,14 @@ import numpy as np
 
 MODE_TRAIN_SOFT = 0   # Eq. ours_train: selected historical blocks get + log g
 MODE_INFER_HARD = 1   # Alg. 2: selected historical blocks get no bias
+
+# Gate activation phi of Eq. general_gate (Sec. 4.2, gate activation):
+GATE_SOFTMAX = 0      # g = softmax(s) over the row's historical blocks (the SAS default)
+GATE_SIGMOID = 1      # g = sigmoid(s), independent gates
+GATE_LOGIT = 2        # s added to the logits directly, i.e. log g = s
+# Gate position (Sec. 4.2, gate position):
+GATE_INNER = 0        # o = softmax(q K^T + log g) V  (the SAS default)
+GATE_OUTER = 1        # o = softmax(q K^T) (g . V): gates scale the value rows after the softmax
 
 
 # ---------------------------------------------------------------- rounding --
@@ -120,10 +130,19 @@ def selector_scores(Q, K, Wq, Wk, b):
 
 # --------------------------------------------------------------- a3 / a4 --
 
-def log_gates(s_hist):
-    """a3, Eq. normalized_log_gate: log g_m = s_m - LSE(s) over the row's history."""
+def log_gates(s_hist, act=GATE_SOFTMAX):
+    """a3, log g_m for the row's historical blocks.
+
+    GATE_SOFTMAX: Eq. normalized_log_gate, log g_m = s_m - LSE(s) over the row's history.
+    GATE_SIGMOID: g_m = sigmoid(s_m), so log g_m = -log(1 + exp(-s_m)).
+    GATE_LOGIT:   s_m is injected into the logits unnormalised, log g_m = s_m.
+    (Sec. 4.2, gate activation.)"""
     s_hist = np.asarray(s_hist, dtype=np.float64)
     if s_hist.size == 0:
+        return s_hist.copy()
+    if act == GATE_SIGMOID:
+        return -np.logaddexp(0.0, -s_hist)
+    if act == GATE_LOGIT:
         return s_hist.copy()
     mx = s_hist.max()
     lse = mx + math.log(np.exp(s_hist - mx).sum())
@@ -148,32 +167,41 @@ def topk_blocks(s_hist, K):
 
 # -------------------------------------------------------------------- a5 --
 
-def _row_keys_and_bias(i, s_row, b, topk, mode):
-    """Attended keys of row i and their additive bias (Eq. ours_train).
+def _row_keys_and_bias(i, s_row, b, topk, mode, act=GATE_SOFTMAX, pos=GATE_INNER):
+    """Attended keys of row i, their additive logit bias and their
+    multiplicative weight on the probabilities.
 
-    Returns (keys, bias, sel_idx, sel_logg) where keys lists token indices:
-    first the tokens of the selected historical blocks, then the causal part
-    of the current block.
+    Inner position (Eq. ours_train): bias log g on the selected historical
+    blocks, weight 1.  Outer position: bias 0, weight g (the gate scales the
+    value rows after the softmax).  Inference mode (Alg. 2): neither.  The
+    current block always has bias 0 and weight 1 (g_0 = 1, Eq. general_gate).
+
+    Returns (keys, bias, weight, sel_idx, sel_logg) where keys lists token
+    indices: first the tokens of the selected historical blocks, then the
+    causal part of the current block.
     """
     c = historical_count(i, b)
     s_hist = np.asarray(s_row[:c], dtype=np.float64)
-    lg = log_gates(s_hist)
+    lg = log_gates(s_hist, act)
     sel = topk_blocks(s_hist, topk)
-    keys, bias = [], []
+    keys, bias, weight = [], [], []
     for m in sel:
         toks = np.arange(m * b, (m + 1) * b)
         keys.append(toks)
-        g = lg[m] if mode == MODE_TRAIN_SOFT else 0.0
-        bias.append(np.full(b, g))
+        gated = mode == MODE_TRAIN_SOFT
+        bias.append(np.full(b, lg[m] if gated and pos == GATE_INNER else 0.0))
+        weight.append(np.full(b, math.exp(lg[m]) if gated and pos == GATE_OUTER else 1.0))
     cur = np.arange(c * b, i + 1)           # current block, causal, unit gate
     keys.append(cur)
     bias.append(np.zeros(cur.shape[0]))
-    return np.concatenate(keys), np.concatenate(bias), sel, lg[sel]
+    weight.append(np.ones(cur.shape[0]))
+    return np.concatenate(keys), np.concatenate(bias), np.concatenate(weight), sel, lg[sel]
 
 
 def sas_attention_head(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
-                       rows=None):
-    """a5 for one head: O_i = softmax(z) V, z_j = sm_scale q_i.k_j + bias_j.
+                       rows=None, act=GATE_SOFTMAX, pos=GATE_INNER):
+    """a5 for one head: O_i = sum_j softmax(z)_j w_j v_j, z_j = sm_scale q_i.k_j + bias_j
+    (w_j = 1 except for the outer gate position, where w_j = g of key j's block).
 
     s: [N, >=C-1] selector scores of the head (row i reads s[i, :C_i]).
     rows: iterable of query indices (default: all).
@@ -191,12 +219,12 @@ def sas_attention_head(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
     sel_idx = np.full((R, topk), -1, dtype=np.int64)
     sel_logg = np.zeros((R, topk))
     for r, i in enumerate(rows):
-        keys, bias, sel, lg = _row_keys_and_bias(int(i), s[i], b, topk, mode)
+        keys, bias, weight, sel, lg = _row_keys_and_bias(int(i), s[i], b, topk, mode, act, pos)
         z = sm_scale * (K[keys] @ Q[i]) + bias
         zmax = z.max()
         w = np.exp(z - zmax)
         l = w.sum()
-        O[r] = (w @ V[keys]) / l
+        O[r] = ((w * weight) @ V[keys]) / l
         LSE[r] = zmax + math.log(l)
         sel_idx[r, :sel.shape[0]] = sel
         sel_logg[r, :sel.shape[0]] = lg
@@ -204,7 +232,7 @@ def sas_attention_head(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
 
 
 def sas_attention_materialized(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT,
-                               sm_scale=None):
+                               sm_scale=None, act=GATE_SOFTMAX, pos=GATE_INNER):
     """Brute force: the whole N x N gated logit matrix, then a row softmax.
 
     This is the naive form the paper calls prohibitive (Sec. 4.3, Kernel
@@ -216,22 +244,27 @@ def sas_attention_materialized(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT,
     if sm_scale is None:
         sm_scale = 1.0 / math.sqrt(d)
     bias = np.full((N, N), -np.inf)
+    gate = np.ones((N, N))
     for i in range(N):
         c = historical_count(i, b)
         s_hist = np.asarray(s[i][:c], dtype=np.float64)
-        lg = log_gates(s_hist)
+        lg = log_gates(s_hist, act)
         for m in topk_blocks(s_hist, topk):
-            bias[i, m * b:(m + 1) * b] = lg[m] if mode == MODE_TRAIN_SOFT else 0.0
+            gated = mode == MODE_TRAIN_SOFT
+            bias[i, m * b:(m + 1) * b] = lg[m] if gated and pos == GATE_INNER else 0.0
+            if gated and pos == GATE_OUTER:
+                gate[i, m * b:(m + 1) * b] = math.exp(lg[m])
         bias[i, c * b:i + 1] = 0.0
     Z = sm_scale * (Q @ K.T) + bias
     zmax = Z.max(axis=1, keepdims=True)
     W = np.exp(Z - zmax)
     l = W.sum(axis=1, keepdims=True)
-    return {"O": (W @ V) / l, "LSE": (zmax + np.log(l))[:, 0], "P": W / l}
+    return {"O": (W * gate @ V) / l, "LSE": (zmax + np.log(l))[:, 0], "P": W / l}
 
 
 def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
-                  scores=None, Wq=None, Wk=None, heads=None, rows=None):
+                  scores=None, Wq=None, Wk=None, heads=None, rows=None,
+                  act=GATE_SOFTMAX, pos=GATE_INNER):
     """Alg. 1 steps 1-4 (training forward) over [B, H, N, d] inputs.
 
     Either `scores` [B, H, N, >=C-1] are given (scores-given selector) or the
@@ -248,7 +281,7 @@ def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
         else:
             s = selector_scores(Q[bi, hi], K[bi, hi], Wq[hi], Wk[hi], b)
         out[(bi, hi)] = sas_attention_head(Q[bi, hi], K[bi, hi], V[bi, hi], s, b,
-                                           topk, mode, sm_scale, rows)
+                                           topk, mode, sm_scale, rows, act, pos)
     return out
 
 

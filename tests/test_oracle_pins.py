@@ -262,3 +262,80 @@ def test_flops_accounting_row():
     # row 130 with b = 64: C_i = 2, current block holds 3 keys (128..130)
     assert O.attention_flops_row(130, 64, 32, 128, 128) == 4 * 128 * (3 + 64 * 2) + 2 * 128 * 2
     assert O.attention_flops_row(64 * 40, 64, 32, 128, 0) == 4 * 128 * (1 + 64 * 32)
+
+
+# ------------------------------------------------- ablation gate forms (Sec. 4.2)
+
+def test_sigmoid_and_logit_log_gates_closed_forms():
+    s = np.array([0.0, 40.0, -40.0, math.log(3.0)])
+    lg = O.log_gates(s, O.GATE_SIGMOID)
+    assert lg[0] == pytest.approx(math.log(0.5), abs=1e-15)            # sigmoid(0) = 1/2
+    assert lg[1] == pytest.approx(0.0, abs=1e-15)                      # sigmoid(s) -> 1
+    assert lg[2] == pytest.approx(-40.0, abs=1e-15)                    # log sigmoid(s) ~ s for s << 0
+    assert lg[3] == pytest.approx(math.log(0.75), abs=1e-15)           # sigmoid(log 3) = 3/4
+    assert np.array_equal(O.log_gates(s, O.GATE_LOGIT), s)             # logit injection: log g = s
+    # sigmoid gates are independent: one block's gate ignores the others
+    assert O.log_gates(np.array([0.0, 5.0]), O.GATE_SIGMOID)[0] == O.log_gates(np.array([0.0, -5.0]), O.GATE_SIGMOID)[0]
+
+
+def _one_row_case():
+    # Query i = 64 (current block 1, one historical block 0, C_i = 1): all keys
+    # zero, so every logit is 0; block 0's 64 values are 1, the query's own
+    # value is 0.  With gate g on block 0:
+    #   inner: weights g (x64) and 1 -> O = 64 g / (64 g + 1)
+    #   outer: probabilities 1/65 each, block 0 rows scaled by g -> O = 64 g / 65
+    N, d = 65, 1
+    Q = np.ones((N, d))
+    K = np.zeros((N, d))
+    V = np.zeros((N, d))
+    V[:64] = 1.0
+    return Q, K, V
+
+
+@pytest.mark.parametrize("act,s0,g", [(O.GATE_SOFTMAX, 1.7, 1.0), (O.GATE_SIGMOID, 0.0, 0.5),
+                                      (O.GATE_SIGMOID, math.log(3.0), 0.75), (O.GATE_LOGIT, math.log(0.25), 0.25)])
+def test_inner_and_outer_gate_positions_worked_example(act, s0, g):
+    Q, K, V = _one_row_case()
+    s = np.full((65, 2), s0)
+    inner = O.sas_attention_head(Q, K, V, s, 64, 1, O.MODE_TRAIN_SOFT, rows=[64], act=act, pos=O.GATE_INNER)
+    outer = O.sas_attention_head(Q, K, V, s, 64, 1, O.MODE_TRAIN_SOFT, rows=[64], act=act, pos=O.GATE_OUTER)
+    assert inner["O"][0, 0] == pytest.approx(64 * g / (64 * g + 1), rel=1e-12)
+    assert outer["O"][0, 0] == pytest.approx(64 * g / 65, rel=1e-12)
+    assert inner["sel_logg"][0, 0] == pytest.approx(math.log(g), abs=1e-12)
+    # inner LSE is over the gated logits, outer LSE over the plain ones (all 0 here)
+    assert inner["LSE"][0] == pytest.approx(math.log(64 * g + 1), rel=1e-12)
+    assert outer["LSE"][0] == pytest.approx(math.log(65.0), rel=1e-12)
+    # the hard (inference) forward ignores the gate in both positions
+    hard = O.sas_attention_head(Q, K, V, s, 64, 1, O.MODE_INFER_HARD, rows=[64], act=act, pos=O.GATE_OUTER)
+    assert hard["O"][0, 0] == pytest.approx(64 / 65, rel=1e-12)
+
+
+def test_outer_position_is_affine_in_a_common_gate():
+    # With every historical gate equal to g (logit gates, constant scores s =
+    # log g, K >= C), the outer output is O_cur + g * O_hist: linear in g, so
+    # O(2g) - O(g) = O(g) - O(0) (a gate inside the softmax would not be).
+    rng = np.random.default_rng(7)
+    N, d = 200, 4
+    Q, K, V = (O.round_to_bf16(rng.standard_normal((N, d))) for _ in range(3))
+    rows = [70, 150, 199]
+    def out(g):
+        s = np.full((N, 4), math.log(g)) if g > 0 else np.full((N, 4), -1e300)
+        return O.sas_attention_head(Q, K, V, s, 64, 4, rows=rows, act=O.GATE_LOGIT, pos=O.GATE_OUTER)["O"]
+    o0, o1, o2 = out(0.0), out(0.8), out(1.6)
+    assert np.allclose(o2 - o1, o1 - o0, atol=1e-12)
+    inner1 = O.sas_attention_head(Q, K, V, np.full((N, 4), math.log(0.8)), 64, 4, rows=rows,
+                                  act=O.GATE_LOGIT, pos=O.GATE_INNER)["O"]
+    assert not np.allclose(inner1, o1, atol=1e-3)
+
+
+def test_ablation_forms_match_materialized_matrix():
+    rng = np.random.default_rng(8)
+    N, d = 300, 8
+    Q, K, V = (O.round_to_bf16(rng.standard_normal((N, d))) for _ in range(3))
+    s = rng.standard_normal((N, 5))
+    for act in (O.GATE_SOFTMAX, O.GATE_SIGMOID, O.GATE_LOGIT):
+        for pos in (O.GATE_INNER, O.GATE_OUTER):
+            row = O.sas_attention_head(Q, K, V, s, 64, 2, act=act, pos=pos)
+            mat = O.sas_attention_materialized(Q, K, V, s, 64, 2, act=act, pos=pos)
+            assert np.allclose(row["O"], mat["O"], atol=1e-12)
+            assert np.allclose(row["LSE"], mat["LSE"], atol=1e-12)
