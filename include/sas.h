@@ -68,6 +68,21 @@ typedef enum { SAS_MODE_TRAIN_SOFT = 0, SAS_MODE_INFER_HARD = 1 } sas_mode;
  *                   described, this is the library's reading). */
 typedef enum { SAS_SEL_SCORES_GIVEN = 0, SAS_SEL_MEANPOOL_PROJ = 1 } sas_selector;
 
+/* Gate activation phi of Eq. general_gate, g = phi(s) over the row's
+ * historical blocks (Sec. 4.2 "gate activation"; the current block keeps
+ * g_0 = 1).  Selection is the same for all three (Top-K of s).
+ *   SOFTMAX : g = softmax(s) over the C_i historical blocks (the SAS form).
+ *   SIGMOID : g = sigmoid(s), independent gates.
+ *   LOGIT   : s itself is added to the logits, i.e. log g = s. */
+typedef enum { SAS_GATE_SOFTMAX = 0, SAS_GATE_SIGMOID = 1, SAS_GATE_LOGIT = 2 } sas_gate_act;
+
+/* Gate position (Sec. 4.2 "gate position"), TRAIN_SOFT mode only:
+ *   INNER : o = softmax(q K^T + log g) V (Eq. ours_train, the SAS form).
+ *   OUTER : o = softmax(q K^T) (g . V): the softmax runs over the plain
+ *           logits and each kept block's value rows are scaled by its g;
+ *           LSE is then that of the plain logits. */
+typedef enum { SAS_GATE_INNER = 0, SAS_GATE_OUTER = 1 } sas_gate_pos;
+
 typedef struct {
     int32_t B, H, N, d;   /* batch, heads, tokens (N <= 2^30), head dim (d in {64, 128}) */
     int32_t block;        /* block size b; must be 64 (Sec. 4.2.1 setup)             */
@@ -76,6 +91,8 @@ typedef struct {
     int32_t mode;         /* sas_mode                                                 */
     int32_t selector;     /* sas_selector                                             */
     int32_t d_sel;        /* selector dim d_sel in {64, 128}; 0 selects d             */
+    int32_t gate_act;     /* sas_gate_act (0 = SOFTMAX, the SAS default)               */
+    int32_t gate_pos;     /* sas_gate_pos (0 = INNER, the SAS default)                 */
 } sas_config;
 
 typedef struct sas_handle sas_handle;
@@ -106,8 +123,9 @@ void sas_destroy(sas_handle* h);
  *             gated logits (Alg. 3 output); may be NULL.              (out)
  *   sel_idx   int32 [B, H, N, topk]: each row's kept historical blocks in
  *             ascending order, padded with -1; may be NULL.           (out)
- *   sel_logg  fp32 [B, H, N, topk]: log g of the kept blocks (same order,
- *             0 where padded); may be NULL.                           (out)
+ *   sel_logg  fp32 [B, H, N, topk]: log g of the kept blocks under the
+ *             handle's gate activation (same order, 0 where padded);
+ *             may be NULL.                                            (out)
  *
  * Top-K is exact-K: ties go to the lower block index; rows with at most K
  * historical blocks keep all of them. */

@@ -52,6 +52,7 @@ cudaError_t launch_pool(const void* K, const void* Wk, void* Kt, int BH, int H, 
 // per 128-row tile the sorted union of kept blocks below the tile's diagonal.
 struct SelectArgs {
     int BH, H, N, C, T, topk, d_sel;
+    int gate_act;                   // 0 softmax (log g = s - LSE), 1 sigmoid, 2 logit (log g = s)
     float score_scale;              // 1/sqrt(d_sel) for projected scores, 1 for given scores
     const float* scores;            // SCORES_GIVEN: [BH][N][C]
     const void* Q;                  // MEANPOOL_PROJ: queries bf16 [BH][N][d]
@@ -78,6 +79,7 @@ struct AttnArgs {
     const int32_t* sel_idx;
     const float* sel_logg;
     int BH, N, d, C, T, topk, mode;
+    int gate_pos;               // 0 inner (+ log g in the logits), 1 outer (g scales P after the softmax)
     float sm_scale;
     int* sched;                 // 16 zeroed bytes owned by the caller, left zeroed after each launch
 };

@@ -144,7 +144,10 @@ __device__ __forceinline__ int block_at(const TileRef& x, int j) {
     return j < x.U ? __ldg(x.ulist + j) : 2 * x.t + (j - x.U);
 }
 
-template <int D>
+// OUTER: the gate of a kept block multiplies its probabilities after the
+// softmax (gate position "outer" of Sec. 4.2) instead of adding log g to its
+// logits; the row sum and LSE then stay those of the ungated logits.
+template <int D, bool OUTER>
 __global__ void __launch_bounds__(kThreads, 2)
 attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
             const __grid_constant__ CUtensorMap mapV, AttnParams p) {
@@ -417,10 +420,12 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 if (j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
                 // gate (log2 units) and the last visible key column of block m for this row
                 float bias = 0.f;
+                float gsc = 1.f;   // outer position: gate applied to the probabilities
                 int lim;
                 if (m < c) {
                     if (m == km0) {
-                        bias = train ? kl0 * kLog2e : 0.f;
+                        if constexpr (OUTER) gsc = train ? fast_exp2(kl0 * kLog2e) : 1.f;
+                        else bias = train ? kl0 * kLog2e : 0.f;
                         lim = kBN - 1;
                         // refill the finished slot with entry sp + kRing, then step to sp + 1
                         const int e = sp + kRing;
@@ -499,7 +504,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                         f32x2_split(fma_f32x2(f32x2(xs[k], xs[k + 1]), scale2, off2), a0, a1);
                         const float e0 = fast_exp2(a0), e1 = fast_exp2(a1);
                         acc[(k >> 1) & 3] = add_f32x2(acc[(k >> 1) & 3], f32x2(e0, e1));
-                        pk[k >> 1] = pack_bf16x2(e0, e1);
+                        if constexpr (OUTER) pk[k >> 1] = pack_bf16x2(e0 * gsc, e1 * gsc);
+                        else pk[k >> 1] = pack_bf16x2(e0, e1);
                     }
                     float s0, s1, s2, s3, s4, s5, s6, s7;
                     f32x2_split(acc[0], s0, s1);
@@ -591,12 +597,12 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     }
 }
 
-template <int D>
+template <int D, bool OUTER>
 cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) {
     using Cfg = AttnCfg<D>;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, OUTER>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
         attr_set = true;
     }
@@ -628,7 +634,7 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
     const long long items = static_cast<long long>(a.T) * a.BH;
     const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);
-    attn_kernel<D><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
+    attn_kernel<D, OUTER><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "attention launch";
     return e;
@@ -637,8 +643,9 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
 }  // namespace
 
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err) {
-    if (a.d == 128) return launch_d<128>(a, env, err);
-    if (a.d == 64) return launch_d<64>(a, env, err);
+    const bool outer = a.gate_pos == 1;
+    if (a.d == 128) return outer ? launch_d<128, true>(a, env, err) : launch_d<128, false>(a, env, err);
+    if (a.d == 64) return outer ? launch_d<64, true>(a, env, err) : launch_d<64, false>(a, env, err);
     *err = "attention: unsupported head dim";
     return cudaErrorInvalidValue;
 }

@@ -5,6 +5,7 @@
 //   I_i        = the K largest s_im, ties to the lower index   (Eq. selected_context)
 //   sel_idx_i  = I_i in ascending order, -1 padded
 //   sel_logg_i = s_im - LSE_i for m in I_i                      (log g of the kept blocks)
+// (with the ablation activations of Sec. 4.2 instead: log sigmoid(s_im), or s_im itself)
 // and for each 128-row tile t the sorted union of kept blocks below the tile's
 // two diagonal blocks (m < 2t): the list of historical key blocks the
 // attention kernel visits for that tile (Alg. 3 skips the others).
@@ -39,6 +40,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 struct SelParams {
     int BH, N, C, T, F, topk;
+    int gate_act;                 // 0 softmax, 1 sigmoid, 2 logit (see staged_gate)
     float score_scale;
     const float* scores;
     int32_t* sel_idx;
@@ -280,6 +282,18 @@ __device__ __forceinline__ void smem_sort_by_block(SmemTopK& t, int n) {
     }
 }
 
+// log g of a kept block from its score (Eq. general_gate with the activation of
+// Sec. 4.2): softmax s - LSE; logit s; sigmoid log(1/(1+e^-s)).  The row pass
+// stages s - LSE (softmax) or s (the others); copy_out turns a staged s into
+// log sigmoid(s), off the per-row path.
+__device__ __forceinline__ float staged_gate(float s, float lse, int act) {
+    return act == 0 ? s - lse : s;
+}
+
+__device__ __forceinline__ float log_sigmoid(float s) {
+    return -(fmaxf(-s, 0.f) + log1pf(expf(-fabsf(s))));
+}
+
 // Output staging: each row's K entries are written to shared memory (row
 // stride K + 1 words, so a warp's rows hit distinct banks) and then copied to
 // global memory with coalesced stores.
@@ -303,9 +317,12 @@ __device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, 
     const long long base = (static_cast<long long>(bh) * p.N + static_cast<long long>(t) * kRows) * K;
     int r = tid / K, e = tid - r * K;
     const int dr = nthreads / K, de = nthreads - dr * K;
+    const bool sigm = p.gate_act == 1;
     for (int q = tid; q < rows * K; q += nthreads) {
-        p.sel_idx[base + q] = st.idx[r * st.stride + e];
-        p.sel_logg[base + q] = st.lg[r * st.stride + e];
+        const int m = st.idx[r * st.stride + e];
+        const float lg = st.lg[r * st.stride + e];
+        p.sel_idx[base + q] = m;
+        p.sel_logg[base + q] = (sigm && m >= 0) ? log_sigmoid(lg) : lg;
         r += dr;
         e += de;
         if (e >= K) {
@@ -318,11 +335,11 @@ __device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, 
 // Finishes one row: log-gates, ascending order, staging, tile-union bits.
 template <class TK>
 __device__ __forceinline__ void row_emit(TK& t, const RowLse& l, const Staging& st, int r, int Ci, int K, int diag,
-                                         uint32_t* bitmap);
+                                         uint32_t* bitmap, int act);
 
 template <>
 __device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, const Staging& st, int r, int Ci,
-                                                  int K, int diag, uint32_t* bitmap) {
+                                                  int K, int diag, uint32_t* bitmap, int act) {
     const int n = min(K, Ci);
     const float lse = Ci > 0 ? l.mx + logf(l.sum) : 0.f;
     if (t.replaced) reg_sort_by_block(t);
@@ -331,7 +348,7 @@ __device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, c
         if (e < K) {
             const bool kept = e < n;
             const int m = static_cast<int>(t.mf[e]);
-            stage_entry(st, r, e, kept ? m : -1, kept ? t.s[e] - lse : 0.f);
+            stage_entry(st, r, e, kept ? m : -1, kept ? staged_gate(t.s[e], lse, act) : 0.f);
             if (kept && static_cast<unsigned>(m) < static_cast<unsigned>(diag))
                 atomicOr(&bitmap[m >> 5], 1u << (m & 31));
         }
@@ -340,14 +357,14 @@ __device__ __forceinline__ void row_emit<RegTopK>(RegTopK& t, const RowLse& l, c
 
 template <>
 __device__ __forceinline__ void row_emit<SmemTopK>(SmemTopK& t, const RowLse& l, const Staging& st, int r, int Ci,
-                                                   int K, int diag, uint32_t* bitmap) {
+                                                   int K, int diag, uint32_t* bitmap, int act) {
     const int n = min(K, Ci);
     const float lse = Ci > 0 ? l.mx + logf(l.sum) : 0.f;
     if (t.replaced) smem_sort_by_block(t, n);
     for (int e = 0; e < K; ++e) {
         if (e < n) {
             const int m = t.m[e * kRows];
-            stage_entry(st, r, e, m, t.s[e * kRows] - lse);
+            stage_entry(st, r, e, m, staged_gate(t.s[e * kRows], lse, act));
             if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
         } else {
             stage_entry(st, r, e, -1, 0.f);
@@ -449,8 +466,8 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
         __syncwarp();
     }
     if (valid) {
-        if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap);
-        else row_emit(stk, lse, st, r, Ci, K, diag, bitmap);
+        if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
+        else row_emit(stk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
     }
     __syncthreads();
     copy_out(st, p, bh, t, threadIdx.x, 128);
@@ -681,8 +698,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                          reinterpret_cast<float*>(smem + size_t(kRows) * (K + 1) * 4), K + 1};
         ok = !abort_flag;
         if (valid && ok) {
-            if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap);
-            else row_emit(stk, lse, st, r, Ci, K, diag, bitmap);
+            if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
+            else row_emit(stk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
         }
         named_bar_sync(1, 128);
         if (ok) copy_out(st, p, bh, t, static_cast<int>(threadIdx.x) - 64, 128);
@@ -739,6 +756,7 @@ cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelE
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
     SelParams p;
     p.BH = a.BH; p.N = a.N; p.C = a.C; p.T = a.T; p.F = a.F; p.topk = a.topk;
+    p.gate_act = a.gate_act;
     p.score_scale = a.score_scale;
     p.scores = a.scores;
     p.sel_idx = a.sel_idx; p.sel_logg = a.sel_logg;

@@ -206,6 +206,9 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (c.topk > 64) return SAS_ERR_UNSUPPORTED;
     if (c.mode != SAS_MODE_TRAIN_SOFT && c.mode != SAS_MODE_INFER_HARD) return SAS_ERR_INVALID_ARG;
     if (c.selector != SAS_SEL_SCORES_GIVEN && c.selector != SAS_SEL_MEANPOOL_PROJ) return SAS_ERR_INVALID_ARG;
+    if (c.gate_act != SAS_GATE_SOFTMAX && c.gate_act != SAS_GATE_SIGMOID && c.gate_act != SAS_GATE_LOGIT)
+        return SAS_ERR_INVALID_ARG;
+    if (c.gate_pos != SAS_GATE_INNER && c.gate_pos != SAS_GATE_OUTER) return SAS_ERR_INVALID_ARG;
     if (!(c.sm_scale >= 0.f) || !std::isfinite(c.sm_scale)) return SAS_ERR_INVALID_ARG;
     const int d_sel = c.d_sel == 0 ? c.d : c.d_sel;
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
@@ -299,6 +302,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     // a2-a4: query projection (learned selector), scores, log-gates, Top-K, tile unions
     sas::SelectArgs sa{};
     sa.BH = h->BH; sa.H = c.H; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.gate_act = c.gate_act;
     sa.score_scale = c.selector == SAS_SEL_MEANPOOL_PROJ ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
     sa.scores = scores;
     sa.Q = Q; sa.Wq = Wq; sa.d = c.d; sa.Kt = h->Kt; sa.F = h->F;
@@ -312,6 +316,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
     aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
     aa.sched = h->sched;
     e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });

@@ -27,6 +27,11 @@ SAS_MODE_TRAIN_SOFT = 0
 SAS_MODE_INFER_HARD = 1
 SAS_SEL_SCORES_GIVEN = 0
 SAS_SEL_MEANPOOL_PROJ = 1
+SAS_GATE_SOFTMAX = 0
+SAS_GATE_SIGMOID = 1
+SAS_GATE_LOGIT = 2
+SAS_GATE_INNER = 0
+SAS_GATE_OUTER = 1
 SAS_NUM_KERNEL_KINDS = 6
 KERNEL_KINDS = ["block_summaries", "query_projection", "selection", "attention", "mlp_up_gelu", "mlp_down"]
 
@@ -36,7 +41,8 @@ HEADER = os.path.join(_build.ROOT, "include", "sas.h")
 class SasConfig(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("d", ctypes.c_int32),
                 ("block", ctypes.c_int32), ("topk", ctypes.c_int32), ("sm_scale", ctypes.c_float),
-                ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32)]
+                ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32),
+                ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32)]
 
 
 class SasError(RuntimeError):
@@ -130,16 +136,17 @@ def sas_status_str(status):
 
 
 def sas_create(B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-               sm_scale=0.0, block=64):
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel)
+               sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos)
     h = ctypes.c_void_p()
     _check(lib().sas_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_create")
     return h
 
 
-def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64):
+def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64,
+                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
     """Raw status of sas_create (for argument-check tests); destroys the handle on success."""
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel)
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos)
     h = ctypes.c_void_p()
     st = lib().sas_create(ctypes.byref(cfg), ctypes.byref(h))
     if st == SAS_OK:
@@ -229,10 +236,10 @@ class SasLayer:
     """Owns one handle; allocates outputs and calls the C ABI."""
 
     def __init__(self, B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-                 sm_scale=0.0):
+                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
         self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
         self.selector = selector
-        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale)
+        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos)
 
     def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
         dev = Q.device

@@ -42,9 +42,10 @@ def sample_rows(N, n_random=256, seed=0):
     return np.array(sorted(r for r in rows if 0 <= r < N))
 
 
-def run_gpu(B, H, N, d, topk, mode, Q, K, V, scores=None, Wq=None, Wk=None, d_sel=0):
+def run_gpu(B, H, N, d, topk, mode, Q, K, V, scores=None, Wq=None, Wk=None, d_sel=0,
+            act=sas.SAS_GATE_SOFTMAX, pos=sas.SAS_GATE_INNER):
     sel = sas.SAS_SEL_SCORES_GIVEN if scores is not None else sas.SAS_SEL_MEANPOOL_PROJ
-    layer = sas.SasLayer(B, H, N, d, topk, mode=mode, selector=sel, d_sel=d_sel)
+    layer = sas.SasLayer(B, H, N, d, topk, mode=mode, selector=sel, d_sel=d_sel, gate_act=act, gate_pos=pos)
     dev = torch.device("cuda:0")
     cu = lambda t: None if t is None else t.to(dev).contiguous()
     O, LSE, si, sl = layer.attention(cu(Q), cu(K), cu(V), cu(scores), cu(Wq), cu(Wk))
@@ -61,8 +62,11 @@ def oracle_scores(Q, K, Wq, Wk, bi, hi):
     return OR.selector_scores(f64(Q[bi, hi]), f64(K[bi, hi]), f64(Wq[hi]), f64(Wk[hi]), 64)
 
 
-def compare_o(gpu_O, ref_O, what="O"):
-    err = np.abs(gpu_O - ref_O)
+def compare_o(gpu_O, ref_O, what="O", scale=1.0):
+    """Max and mean abs error of O against the oracle; scale > 1 widens both
+    bounds in proportion, for outputs whose magnitude grows past that of V
+    (bf16 rounding error is relative)."""
+    err = np.abs(gpu_O - ref_O) / scale
     mx, mean = float(err.max()), float(err.mean())
     assert mx <= O_MAX_ABS, f"{what}: max abs err {mx:.3e} > {O_MAX_ABS}"
     assert mean <= O_MEAN_ABS, f"{what}: mean abs err {mean:.3e} > {O_MEAN_ABS}"

@@ -46,6 +46,9 @@ def test_status_strings(lib):
     (dict(B=1, H=1, N=128, d=64, topk=2, d_sel=32), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=1, N=128, d=64, topk=2, sm_scale=math.nan), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=1, N=128, d=64, topk=2, sm_scale=-1.0), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=1, N=128, d=64, topk=2, gate_act=3), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=1, N=128, d=64, topk=2, gate_act=-1), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=1, N=128, d=64, topk=2, gate_pos=2), sas.SAS_ERR_INVALID_ARG),
 ])
 def test_create_rejects_bad_configs(lib, kw, expect):
     assert sas.sas_create_status(**kw) == expect

@@ -14,25 +14,25 @@ pytestmark = pytest.mark.gpu
 TRAIN, INFER = sas.SAS_MODE_TRAIN_SOFT, sas.SAS_MODE_INFER_HARD
 
 
-def _given_case(B, H, N, d, topk, mode, regime="R1", seed=0, rows=None):
+def _given_case(B, H, N, d, topk, mode, regime="R1", seed=0, rows=None, act=OR.GATE_SOFTMAX, pos=OR.GATE_INNER):
     Q, K, V = synth.qkv(B, H, N, d, seed=seed)
     C = -(-N // 64)
     if regime == "ties":
         S = synth.integer_scores(B, H, N, C, seed=seed)
     else:
         S = synth.scores(B, H, N, C, seed=seed, regime=regime)
-    g = P.run_gpu(B, H, N, d, topk, mode, Q, K, V, scores=S)
+    g = P.run_gpu(B, H, N, d, topk, mode, Q, K, V, scores=S, act=act, pos=pos)
     assert g["status"] == 0
     for bi in range(B):
         for hi in range(H):
             rr = np.arange(N) if rows is None else rows
             ref = OR.sas_attention_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]),
-                                        P.f64(S[bi, hi]), 64, topk, mode, rows=rr)
+                                        P.f64(S[bi, hi]), 64, topk, mode, rows=rr, act=act, pos=pos)
             gi = g["sel_idx"][bi, hi].numpy()[rr][:, :topk]
             P.check_selection_rows(gi, P.f64(S[bi, hi])[rr], rr, topk)
             lg = g["sel_logg"][bi, hi].numpy()[rr][:, :topk]
             assert np.abs(lg - ref["sel_logg"]).max(initial=0) <= P.LOGG_MAX_ABS
-            P.compare_o(P.f64(g["O"][bi, hi])[rr], ref["O"], f"O[{bi},{hi}]")
+            P.compare_o(P.f64(g["O"][bi, hi])[rr], ref["O"], f"O[{bi},{hi}]", max(1.0, np.abs(ref["O"]).max()))
             assert np.abs(g["LSE"][bi, hi].numpy()[rr] - ref["LSE"]).max() <= P.LSE_MAX_ABS
             if rows is None and topk > 0:
                 full = g["sel_idx"][bi, hi].numpy()[:, :topk]
@@ -106,14 +106,15 @@ def test_tiny_config_defaults():
     _given_case(1, 4, 256, 64, 2, TRAIN, seed=0)
 
 
-def _learned_case(B, H, N, d, topk, mode=TRAIN, d_sel=0, seed=0, heads=None, rows=None, exact_inputs=False):
+def _learned_case(B, H, N, d, topk, mode=TRAIN, d_sel=0, seed=0, heads=None, rows=None, exact_inputs=False,
+                  act=OR.GATE_SOFTMAX, pos=OR.GATE_INNER):
     d_sel = d_sel or d
     if exact_inputs:
         Q, K, V, Wq, Wk = synth.integer_selector_inputs(B, H, N, d, d_sel, seed=seed)
     else:
         Q, K, V = synth.qkv(B, H, N, d, seed=seed, regime="R2")
         Wq, Wk = synth.selector_weights(H, d, d_sel, seed=seed)
-    g = P.run_gpu(B, H, N, d, topk, mode, Q, K, V, Wq=Wq, Wk=Wk, d_sel=d_sel)
+    g = P.run_gpu(B, H, N, d, topk, mode, Q, K, V, Wq=Wq, Wk=Wk, d_sel=d_sel, act=act, pos=pos)
     assert g["status"] == 0
     heads = heads or [(bi, hi) for bi in range(B) for hi in range(H)]
     total_mismatch = total = 0
@@ -121,7 +122,7 @@ def _learned_case(B, H, N, d, topk, mode=TRAIN, d_sel=0, seed=0, heads=None, row
         rr = np.arange(N) if rows is None else rows
         s = P.oracle_scores(Q, K, Wq, Wk, bi, hi)
         ref = OR.sas_attention_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s, 64, topk, mode,
-                                    rows=rr)
+                                    rows=rr, act=act, pos=pos)
         tol = None if exact_inputs else P.selector_score_bound(Q, K, Wq, Wk, bi, hi, d_sel, rows=rr)
         gi = g["sel_idx"][bi, hi].numpy()[rr][:, :topk]
         exact, near, mism = P.check_selection_rows(gi, s[rr], rr, topk, tol)
@@ -162,6 +163,26 @@ def test_learned_selector_dsel64_with_d128():
 def test_learned_selector_k64_shared_memory_topk():
     # K > 32 keeps the Top-K in shared memory; integer inputs make the kept sets exact
     _learned_case(1, 2, 5000, 128, 64, exact_inputs=True, seed=13)
+
+
+# Sec. 4.2 ablations: gate activation (softmax / sigmoid / raw logit) and gate
+# position (inner: + log g on the logits; outer: g scales the probabilities).
+@pytest.mark.parametrize("act", [OR.GATE_SOFTMAX, OR.GATE_SIGMOID, OR.GATE_LOGIT])
+@pytest.mark.parametrize("pos", [OR.GATE_INNER, OR.GATE_OUTER])
+def test_gate_variants_given_scores(act, pos):
+    _given_case(1, 3, 1000, 128, 4, TRAIN, seed=50 + 3 * act + pos, act=act, pos=pos)
+
+
+@pytest.mark.parametrize("act,pos", [(OR.GATE_SIGMOID, OR.GATE_OUTER), (OR.GATE_LOGIT, OR.GATE_INNER)])
+def test_gate_variants_learned_selector(act, pos):
+    _learned_case(1, 2, 900, 64, 3, seed=60 + act, act=act, pos=pos)
+    _learned_case(1, 2, 1000, 128, 4, exact_inputs=True, seed=62 + act, act=act, pos=pos)
+
+
+def test_gate_variants_inference_ignore_gates_but_report_them():
+    # INFER (Alg. 2) uses no gate, so O and LSE match across variants; the
+    # reported log g still follows the activation
+    _given_case(1, 2, 700, 64, 3, INFER, seed=70, act=OR.GATE_SIGMOID, pos=OR.GATE_OUTER)
 
 
 def test_full_size_dit_layer_sampled():
