@@ -219,6 +219,111 @@ sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n
  * device recorded (SAS_ERR_TIMEOUT expected).  Synchronises. */
 sas_status sas_selftest_wait_timeout(int64_t limit_cycles, int32_t* host_status);
 
+/* ===================================================================== decode
+ *
+ * SAS decode step (Alg. 2): one new token per sequence attends to its own
+ * block B_0 plus the Top-K cached blocks chosen by the selector, without gate
+ * bias.  Following the paper's inference implementation (Sec. 5), selection is
+ * made once per query group: the G = Hq / Hkv query heads that share a KV head
+ * share its kept blocks, and only those blocks' keys and values are read.
+ *
+ * Selector of a group (the library's reading; the paper does not describe
+ * how a group forms its gate query):
+ *   q~   = bf16(Wq_g [q_0; q_1; ...; q_{G-1}])   (the group's queries
+ *          concatenated head by head, Wq_g of shape [d_sel, G*d]);
+ *   K~_m = bf16(Wk_g mean(keys of block m))       (kept in a summary cache);
+ *   s_m  = q~ . K~_m / sqrt(d_sel) for the C = floor((n-1)/64) historical
+ *          blocks of a sequence of n tokens (the new token is position n-1).
+ * With G = 1 this is the MEANPOOL_PROJ selector of sas_attention_fwd.
+ * Top-K is exact-K with ties to the lower block; C <= K keeps every block.
+ *
+ * Paged cache (caller-owned device memory):
+ *   K_cache, V_cache  bf16 [num_pages, Hkv, 64, d]: a page holds the 64 tokens
+ *                     of one block for every KV head.
+ *   block_table       int32 [B, max_blocks]: page of logical block m of
+ *                     sequence b (entries of blocks a sequence has not reached
+ *                     are never read).
+ *   seq_lens          int32 [B]: tokens in the cache of each sequence AFTER
+ *                     this step's token is added (1 <= n <= 64 * max_blocks).
+ *   Ksum              bf16 [B, Hkv, max_blocks, d_sel]: block summaries K~_m
+ *                     by logical block; entry m is valid once block m is full.
+ * Lengths and page indices are read on the device, so a CUDA graph of a step
+ * can be replayed while they change.  A length or page index out of range is
+ * not read: that sequence is skipped and the device status word becomes
+ * SAS_ERR_INVALID_ARG (see sas_decode_get_device_status). */
+
+typedef struct {
+    int32_t B;            /* sequences decoded together                               */
+    int32_t Hq, Hkv;      /* query heads and KV heads; G = Hq / Hkv in {1, 2, 4, 8}     */
+    int32_t d;            /* head dim, 64 or 128                                       */
+    int32_t d_sel;        /* selector dim, 64 or 128; 0 selects d                      */
+    int32_t block;        /* must be 64                                                */
+    int32_t topk;         /* K kept blocks per group, 0 <= K <= 64                     */
+    int32_t max_blocks;   /* block-table width: capacity of one sequence, <= 32768     */
+    int32_t num_pages;    /* pages in K_cache / V_cache                                */
+    float sm_scale;       /* scale on q.k; 0 selects 1/sqrt(d)                          */
+    int32_t dense;        /* 1: attend to every cached block (no selector, no summaries:
+                             the dense decode SAS is compared with)                      */
+} sas_decode_config;
+
+typedef struct sas_decode_handle sas_decode_handle;
+
+/* Validates cfg and allocates the handle's workspace (gate queries, scores,
+ * kept lists, split-attention partials, arrival counters, status word) on the
+ * current device.  Synchronous. */
+sas_status sas_decode_create(const sas_decode_config* cfg, sas_decode_handle** out);
+void sas_decode_destroy(sas_decode_handle* h);
+
+/* Fills the summary cache after a prefill: Ksum[b, g, m] = bf16(Wk[g] mean
+ * of the 64 keys of block m) for every full block m < floor(seq_lens[b] / 64).
+ *   K_cache    bf16 [num_pages, Hkv, 64, d]                           (in)
+ *   block_table, seq_lens as above (here seq_lens counts cached tokens) (in)
+ *   Wk         bf16 [Hkv, d_sel, d]                                   (in)
+ *   Ksum       bf16 [B, Hkv, max_blocks, d_sel]                       (out) */
+sas_status sas_decode_summarize(sas_decode_handle* h, const void* K_cache, const int32_t* block_table,
+                                const int32_t* seq_lens, const void* Wk, void* Ksum, void* stream);
+
+/* One decode step for every sequence of the batch (Alg. 2):
+ *   1. appends k_new / v_new (bf16 [B, Hkv, d]; both NULL if the caller has
+ *      already written position n-1 of the cache) at position n-1; when that
+ *      position opens a new block (n-1 = 64c, c >= 1) the now full block c-1 is
+ *      summarised into Ksum; computes each group's gate query from q;
+ *   2. scores the C historical blocks of each group against Ksum and keeps
+ *      the Top-K (ascending, written to sel_idx if given);
+ *   3. attends every query head over its group's kept blocks plus the
+ *      current block (positions 64c .. n-1).
+ *   q        bf16 [B, Hq, d]; query head h belongs to KV head h / G   (in)
+ *   Wq       bf16 [Hkv, d_sel, G*d]; Wk bf16 [Hkv, d_sel, d]          (in)
+ *   Ksum     bf16 [B, Hkv, max_blocks, d_sel]                    (in/out)
+ *   O        bf16 [B, Hq, d]                                         (out)
+ *   LSE      fp32 [B, Hq] natural-log log-sum-exp of the logits, or NULL
+ *   sel_idx  int32 [B, Hkv, topk] kept blocks, -1 padded, or NULL
+ * In dense mode Wq, Wk and Ksum are not used (may be NULL) and sel_idx must be
+ * NULL.  Three kernel launches (two in dense mode); no allocation, no
+ * synchronisation, so the call can be captured in a CUDA graph. */
+sas_status sas_decode_step(sas_decode_handle* h, const void* q, const void* k_new, const void* v_new,
+                           void* K_cache, void* V_cache, const int32_t* block_table, const int32_t* seq_lens,
+                           const void* Wq, const void* Wk, void* Ksum, void* O, float* LSE, int32_t* sel_idx,
+                           void* stream);
+
+/* Text of the last error recorded on this handle ("" if none). */
+const char* sas_decode_last_error(const sas_decode_handle* h);
+
+/* Reads and clears the handle's device status word (SAS_OK,
+ * SAS_ERR_INVALID_ARG for an out-of-range length or page index,
+ * SAS_ERR_TIMEOUT for a bounded wait that ran out).  Synchronises. */
+sas_status sas_decode_get_device_status(sas_decode_handle* h, int32_t* out_status);
+
+/* Event timing per kernel kind, as sas_set_timing / sas_get_timings:
+ * 0 append + summary + gate query, 1 scores + Top-K, 2 attention, 3 summary
+ * fill (sas_decode_summarize).  n_kinds <= 4. */
+#define SAS_DECODE_NUM_KERNEL_KINDS 4
+sas_status sas_decode_set_timing(sas_decode_handle* h, int32_t enable);
+sas_status sas_decode_get_timings(sas_decode_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds);
+
+/* Kernels this handle has launched since creation. */
+int64_t sas_decode_launch_count(const sas_decode_handle* h);
+
 #ifdef __cplusplus
 }
 #endif

@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_PATH = os.path.join(HERE, "libsas.so")
 
-SOURCES = ["sas_api.cu", "k_gemm.cu", "k_pool.cu", "k_select.cu", "k_attn.cu", "sas_noalloc.cu"]
+SOURCES = ["sas_api.cu", "k_gemm.cu", "k_pool.cu", "k_select.cu", "k_attn.cu", "sas_noalloc.cu", "k_decode.cu",
+           "sas_decode.cu"]
 HEADERS = ["ptx.cuh", "internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",

@@ -85,6 +85,48 @@ struct AttnArgs {
 };
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err);
 
+// ---- decode step (Alg. 2, per-group selection over a paged cache).
+struct DecodeArgs {
+    int B, Hq, Hkv, G, d, d_sel, topk, max_blocks, num_pages;
+    int dense;
+    float sm_scale;
+    const void* q;              // bf16 [B][Hq][d]
+    const void* k_new;          // bf16 [B][Hkv][d] or null
+    const void* v_new;
+    void* K_cache;              // bf16 [P][Hkv][64][d]
+    void* V_cache;
+    const int32_t* block_table; // [B][max_blocks]
+    const int32_t* seq_lens;    // [B]
+    const void* Wq;             // bf16 [Hkv][d_sel][G*d]
+    const void* Wk;             // bf16 [Hkv][d_sel][d]
+    void* Ksum;                 // bf16 [B][Hkv][max_blocks][d_sel]
+    void* O;                    // bf16 [B][Hq][d]
+    float* LSE;                 // [B][Hq] or null
+    int32_t* sel_idx;           // [B][Hkv][topk] or null
+    // workspace
+    void* qt;                   // bf16 [B*Hkv][d_sel] gate queries
+    float* scores;              // [B*Hkv][max_blocks]
+    int32_t* list;              // [B*Hkv][64] kept blocks, ascending
+    int32_t* list_n;            // [B*Hkv]
+    float* part;                // [B*Hkv][nsplit_a][G][d + 2] split-attention partials
+    int* cnt_sel;               // [B*Hkv] arrival counters, zero between launches
+    int* cnt_attn;              // [B*Hkv]
+    int nsplit_s;               // score CTAs per group (kDecScoreChunk blocks each)
+    int nsplit_a, bpc;          // attention CTAs per group, list entries per CTA
+};
+constexpr int kDecScoreChunk = 256;
+// Attention split for a group list of at most max_len entries.
+void decode_attn_split(int max_len, int* nsplit, int* bpc);
+// Dynamic shared memory the score and attention kernels need.
+size_t decode_score_smem(int max_blocks, int d_sel);
+size_t decode_attn_smem(int d, int G, int bpc);
+// Sets the kernels' shared-memory limits for these arguments (before any capture).
+cudaError_t decode_prepare(const DecodeArgs& a);
+cudaError_t launch_decode_prep(const DecodeArgs& a, const KernelEnv& env);
+cudaError_t launch_decode_score(const DecodeArgs& a, const KernelEnv& env);
+cudaError_t launch_decode_attn(const DecodeArgs& a, const KernelEnv& env);
+cudaError_t launch_decode_summarize(const DecodeArgs& a, const KernelEnv& env);
+
 // ---- failure-path self test (bounded wait on a barrier nothing completes)
 cudaError_t launch_wait_selftest(int* status, long long limit, cudaStream_t stream);
 

@@ -1,0 +1,820 @@
+// Decode step of SAS (Alg. 2): one new token per sequence, grouped-query
+// attention with one block selection per query group (Sec. 5, inference
+// implementation), over a paged KV cache holding one 64-token block per page.
+//
+//   dec_prep_kernel    appends k_new / v_new at position n-1, summarises the block
+//                      that position closes (K~ = bf16(Wk mean K), App. B) and
+//                      forms the group's gate query q~ = bf16(Wq_g [q_0; ...]).
+//   dec_score_kernel   s_m = q~ . K~_m / sqrt(d_sel) for the C historical blocks
+//                      (Alg. 2 step 1), CTAs of 256 blocks whose summary rows are
+//                      staged in shared memory by bulk async copies; the last CTA
+//                      of a group takes the exact Top-K (step 2) by a radix select
+//                      on the scores' order-preserving bit patterns, ties to the
+//                      lower block, and writes the kept list in ascending order.
+//   dec_attn_kernel    split-KV attention over B_0 and the kept blocks (steps 3-4):
+//                      each CTA streams a few pages (K and V slices of 16 KB at
+//                      d = 128, bulk async copies into a 3-stage ring), keeps an
+//                      online softmax per head, and the last CTA of a group merges
+//                      the partial (max, sum, output) triples.
+// A decode step moves bytes, not flops (a few FMAs per cached element), so the
+// arithmetic runs on CUDA cores with packed fp32x2 FMAs; there is no tensor-core
+// contraction on this path.
+#include <math_constants.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace sas {
+namespace {
+
+constexpr int kBlk = 64;
+constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
+constexpr int kPrepThreads = 256;
+constexpr int kScoreThreads = 256;
+constexpr int kAttnThreads = 128;
+constexpr int kStages = 3;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+__device__ __forceinline__ bool bad_len(int n, const DecodeArgs& a) { return n < 1 || n > a.max_blocks * kBlk; }
+
+// Exclusive prefix sum over the 256 threads of a CTA (scan: 16 shared ints).
+__device__ int block_excl_scan(int v, int* scan) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) scan[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < 8 ? scan[lane] : 0;
+        const int own = w;
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < 8) scan[8 + lane] = w - own;
+    }
+    __syncthreads();
+    const int r = x - v + scan[8 + warp];
+    __syncthreads();
+    return r;
+}
+
+// One full block's summary (App. B): the mean of its 64 keys in fp32, projected
+// by the KV head's Wk [d_sel][d] and rounded to bf16.  256 threads.
+// red: 512 floats, kbar: 128 floats of shared memory.
+__device__ void summarize_block(const bf16* Kt, const bf16* Wk, bf16* out, int d, int d_sel, float* red,
+                                float* kbar) {
+    const int t = threadIdx.x;
+    const int nw = d >> 1;                    // bf16 pairs per key row
+    const int groups = kPrepThreads / nw;     // 4 (d = 128) or 8 (d = 64) row groups
+    const int rows = kBlk / groups;
+    const int wi = t % nw, rg = t / nw;
+    const uint32_t* K32 = reinterpret_cast<const uint32_t*>(Kt);
+    float a0 = 0.f, a1 = 0.f;
+    for (int r = rg * rows; r < (rg + 1) * rows; ++r) {
+        const uint32_t w = __ldg(K32 + r * nw + wi);
+        a0 += bf_lo(w);
+        a1 += bf_hi(w);
+    }
+    red[rg * d + 2 * wi] = a0;
+    red[rg * d + 2 * wi + 1] = a1;
+    __syncthreads();
+    if (t < d) {
+        float s = 0.f;
+        for (int g = 0; g < groups; ++g) s += red[g * d + t];
+        kbar[t] = s * (1.f / kBlk);
+    }
+    __syncthreads();
+    const int warp = t >> 5, lane = t & 31;
+    for (int o = warp; o < d_sel; o += kPrepThreads / 32) {
+        const uint32_t* row = reinterpret_cast<const uint32_t*>(Wk + static_cast<size_t>(o) * d);
+        float acc = 0.f;
+        for (int e = lane; e < nw; e += 32) {
+            const uint32_t w = __ldg(row + e);
+            acc = fmaf(bf_lo(w), kbar[2 * e], acc);
+            acc = fmaf(bf_hi(w), kbar[2 * e + 1], acc);
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) out[o] = __float2bfloat16_rn(acc);
+    }
+}
+
+// grid (B*Hkv, 1 + d_sel/32): y = 0 appends the token and updates the summary
+// cache, y >= 1 computes 32 entries of the group's gate query.
+__global__ void __launch_bounds__(kPrepThreads) dec_prep_kernel(DecodeArgs a, int* status) {
+    __shared__ float red[512];
+    __shared__ __align__(16) float vec[1024];
+    const int bh = blockIdx.x;
+    const int b = bh / a.Hkv, g = bh - b * a.Hkv;
+    const int n = __ldg(a.seq_lens + b);
+    const int t = threadIdx.x;
+    if (bad_len(n, a)) {
+        if (t == 0 && blockIdx.y == 0) atomicExch(status, kStatusBadInput);
+        return;
+    }
+    if (blockIdx.y == 0) {
+        const int pos = n - 1, blk = pos / kBlk, slot = pos - blk * kBlk;
+        const int32_t* row = a.block_table + static_cast<size_t>(b) * a.max_blocks;
+        const int page = __ldg(row + blk);
+        if (page < 0 || page >= a.num_pages) {
+            if (t == 0) atomicExch(status, kStatusBadInput);
+            return;
+        }
+        if (a.k_new != nullptr) {
+            const int nu = a.d / 8;   // 16-byte units per row
+            if (t < 2 * nu) {
+                const bool isv = t >= nu;
+                const int u = isv ? t - nu : t;
+                const uint4* src =
+                    reinterpret_cast<const uint4*>(static_cast<const bf16*>(isv ? a.v_new : a.k_new) +
+                                                   static_cast<size_t>(bh) * a.d) + u;
+                uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16*>(isv ? a.V_cache : a.K_cache) +
+                                                      ((static_cast<size_t>(page) * a.Hkv + g) * kBlk + slot) * a.d) + u;
+                *dst = __ldg(src);
+            }
+        }
+        if (!a.dense && slot == 0 && blk >= 1) {
+            const int pp = __ldg(row + blk - 1);
+            if (pp < 0 || pp >= a.num_pages) {
+                if (t == 0) atomicExch(status, kStatusBadInput);
+                return;
+            }
+            summarize_block(static_cast<const bf16*>(a.K_cache) + (static_cast<size_t>(pp) * a.Hkv + g) * kBlk * a.d,
+                            static_cast<const bf16*>(a.Wk) + static_cast<size_t>(g) * a.d_sel * a.d,
+                            static_cast<bf16*>(a.Ksum) + (static_cast<size_t>(bh) * a.max_blocks + blk - 1) * a.d_sel,
+                            a.d, a.d_sel, red, vec);
+        }
+        return;
+    }
+    // gate query q~[o] = bf16(sum_e Wq_g[o][e] q_cat[e]) for o in [32 (y-1), 32 y)
+    const int GD = a.G * a.d;
+    const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * a.G) * a.d;
+    for (int e = t; e < GD; e += kPrepThreads) vec[e] = __bfloat162float(qg[e]);
+    __syncthreads();
+    const int warp = t >> 5, lane = t & 31;
+    const int o0 = (blockIdx.y - 1) * 32;
+    for (int oo = warp; oo < 32; oo += kPrepThreads / 32) {
+        const int o = o0 + oo;
+        if (o >= a.d_sel) break;
+        const bf16* wrow = static_cast<const bf16*>(a.Wq) + (static_cast<size_t>(g) * a.d_sel + o) * GD;
+        float acc = 0.f;
+        for (int e = lane * 8; e < GD; e += 256) {
+            const uint4 w = __ldg(reinterpret_cast<const uint4*>(wrow + e));
+            const float4 x0 = *reinterpret_cast<const float4*>(vec + e);
+            const float4 x1 = *reinterpret_cast<const float4*>(vec + e + 4);
+            acc = fmaf(bf_lo(w.x), x0.x, acc);
+            acc = fmaf(bf_hi(w.x), x0.y, acc);
+            acc = fmaf(bf_lo(w.y), x0.z, acc);
+            acc = fmaf(bf_hi(w.y), x0.w, acc);
+            acc = fmaf(bf_lo(w.z), x1.x, acc);
+            acc = fmaf(bf_hi(w.z), x1.y, acc);
+            acc = fmaf(bf_lo(w.w), x1.z, acc);
+            acc = fmaf(bf_hi(w.w), x1.w, acc);
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) static_cast<bf16*>(a.qt)[static_cast<size_t>(bh) * a.d_sel + o] = __float2bfloat16_rn(acc);
+    }
+}
+
+// grid (max_blocks, B*Hkv): summary of full block m of every sequence (after a prefill).
+__global__ void __launch_bounds__(kPrepThreads) dec_summarize_kernel(DecodeArgs a, int* status) {
+    __shared__ float red[512];
+    __shared__ float kbar[128];
+    const int m = blockIdx.x, bh = blockIdx.y;
+    const int b = bh / a.Hkv, g = bh - b * a.Hkv;
+    const int n = __ldg(a.seq_lens + b);
+    if (n < 0 || n > a.max_blocks * kBlk) {
+        if (threadIdx.x == 0 && m == 0) atomicExch(status, kStatusBadInput);
+        return;
+    }
+    if (m >= n / kBlk) return;
+    const int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + m);
+    if (page < 0 || page >= a.num_pages) {
+        if (threadIdx.x == 0) atomicExch(status, kStatusBadInput);
+        return;
+    }
+    summarize_block(static_cast<const bf16*>(a.K_cache) + (static_cast<size_t>(page) * a.Hkv + g) * kBlk * a.d,
+                    static_cast<const bf16*>(a.Wk) + static_cast<size_t>(g) * a.d_sel * a.d,
+                    static_cast<bf16*>(a.Ksum) + (static_cast<size_t>(bh) * a.max_blocks + m) * a.d_sel, a.d, a.d_sel,
+                    red, kbar);
+}
+
+// ------------------------------------------------------------ scores + Top-K
+
+struct ScoreSmem {
+    size_t r0;   // staging rows / selection keys
+    size_t qs, bars, misc, hist, scan, total;
+};
+__host__ __device__ inline ScoreSmem score_smem_layout(int max_blocks, int d_sel) {
+    ScoreSmem L;
+    size_t slab = static_cast<size_t>(8) * 32 * d_sel * 2;
+    size_t keys = static_cast<size_t>(max_blocks) * 4;
+    L.r0 = ((slab > keys ? slab : keys) + 127) / 128 * 128;
+    L.qs = L.r0;                  // d_sel bf16 (<= 256 bytes)
+    L.bars = L.qs + 256;          // 8 mbarriers
+    L.misc = L.bars + 64;         // flag + radix broadcast (4 ints)
+    L.hist = L.misc + 64;         // 4096 ints
+    L.scan = L.hist + 4096 * 4;   // 16 ints
+    L.total = L.scan + 128;
+    return L;
+}
+
+// Order-preserving map of a finite float to uint32 (larger float, larger key);
+// -0 is mapped like +0 so that equal scores stay ties.
+__device__ __forceinline__ uint32_t order_key(float f) {
+    const uint32_t u = __float_as_uint(f == 0.f ? 0.f : f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Exact Top-K of the group's C scores (K < C), ties to the lower block:
+// radix select of the K-th largest key tau in digits of 12, 10 and 10 bits,
+// then every key > tau plus the lowest-indexed keys == tau, emitted in
+// ascending block order.  256 threads of the last CTA of the group.
+__device__ void select_group(const DecodeArgs& a, int bh, int C, uint32_t* keys, int* hist, int* scan, int* bc) {
+    const int K = a.topk;
+    const int t = threadIdx.x, lane = t & 31;
+    int32_t* lst = a.list + static_cast<size_t>(bh) * 64;
+    int32_t* so = a.sel_idx ? a.sel_idx + static_cast<size_t>(bh) * K : nullptr;
+    if (C <= K) {
+        for (int e = t; e < K; e += kScoreThreads) {
+            if (e < C) lst[e] = e;
+            if (so) so[e] = e < C ? e : -1;
+        }
+        if (t == 0) a.list_n[bh] = C;
+        return;
+    }
+    if (K == 0) {
+        if (t == 0) a.list_n[bh] = 0;
+        return;
+    }
+    const float* sc = a.scores + static_cast<size_t>(bh) * a.max_blocks;
+    for (int i = t; i < C; i += kScoreThreads) keys[i] = order_key(__ldcg(sc + i));
+    uint32_t prefix = 0, mask = 0;
+    int r = K;
+#pragma unroll 1
+    for (int pass = 0; pass < 3; ++pass) {
+        const int width = pass == 0 ? 12 : 10;
+        const int sh = pass == 0 ? 20 : (pass == 1 ? 10 : 0);
+        const int nb = 1 << width;
+        for (int i = t; i < nb; i += kScoreThreads) hist[i] = 0;
+        __syncthreads();
+        for (int base = 0; base < C; base += kScoreThreads) {
+            const int i = base + t;
+            bool in = false;
+            int bin = 0;
+            if (i < C) {
+                const uint32_t k = keys[i];
+                in = (k & mask) == prefix;
+                bin = static_cast<int>((k >> sh) & static_cast<uint32_t>(nb - 1));
+            }
+            // lanes with the same bin add once (the first pass sees few distinct bins)
+            const uint32_t peers = __match_any_sync(0xffffffffu, in ? bin : -1 - lane);
+            if (in && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+        }
+        __syncthreads();
+        const int per = nb / kScoreThreads;   // 16 or 4 bins per thread, highest digits first
+        int s = 0;
+        for (int j = 0; j < per; ++j) s += hist[nb - 1 - (t * per + j)];
+        const int excl = block_excl_scan(s, scan);
+        if (excl < r && excl + s >= r) {
+            int cum = excl;
+            for (int j = 0; j < per; ++j) {
+                const int bin = nb - 1 - (t * per + j);
+                const int c = hist[bin];
+                if (cum + c >= r) {
+                    bc[0] = bin;
+                    bc[1] = r - cum;
+                    break;
+                }
+                cum += c;
+            }
+        }
+        __syncthreads();
+        prefix |= static_cast<uint32_t>(bc[0]) << sh;
+        mask |= static_cast<uint32_t>(nb - 1) << sh;
+        r = bc[1];
+    }
+    const uint32_t tau = prefix;   // the K-th largest key; take r of the keys equal to it
+    // ascending emission: contiguous index ranges of odd length per thread (conflict-free reads)
+    const int per = ((C + kScoreThreads - 1) / kScoreThreads) | 1;
+    const int lo = min(t * per, C), hi = min(lo + per, C);
+    int eq = 0;
+    for (int i = lo; i < hi; ++i) eq += keys[i] == tau;
+    const int eq_base = block_excl_scan(eq, scan);
+    int cnt = 0, er = eq_base;
+    for (int i = lo; i < hi; ++i) {
+        const uint32_t k = keys[i];
+        if (k > tau) {
+            ++cnt;
+        } else if (k == tau) {
+            if (er < r) ++cnt;
+            ++er;
+        }
+    }
+    int pos = block_excl_scan(cnt, scan);
+    er = eq_base;
+    for (int i = lo; i < hi; ++i) {
+        const uint32_t k = keys[i];
+        bool take = k > tau;
+        if (k == tau) {
+            take = er < r;
+            ++er;
+        }
+        if (take) {
+            lst[pos] = i;
+            if (so) so[pos] = i;
+            ++pos;
+        }
+    }
+    if (t == 0) a.list_n[bh] = K;
+}
+
+// grid (nsplit_s, B*Hkv)
+template <int DSEL>
+__global__ void __launch_bounds__(kScoreThreads) dec_score_kernel(DecodeArgs a, int* status, long long limit,
+                                                                  float score_scale) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    constexpr int kRowBytes = DSEL * 2;
+    constexpr int kSlab = 32 * kRowBytes;
+    const ScoreSmem L = score_smem_layout(a.max_blocks, DSEL);
+    uint8_t* stage = smem;
+    uint4* qs = reinterpret_cast<uint4*>(smem + L.qs);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bars);
+    int* misc = reinterpret_cast<int*>(smem + L.misc);
+    const int bh = blockIdx.y;
+    const int b = bh / a.Hkv;
+    const int n = __ldg(a.seq_lens + b);
+    if (bad_len(n, a)) return;   // recorded by the prep kernel
+    const int C = (n - 1) / kBlk;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int m0 = blockIdx.x * kDecScoreChunk;
+    if (t == 0) {
+        for (int w = 0; w < 8; ++w) mbar_init(&bars[w], 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (m0 < C) {
+        if (t < DSEL / 8) qs[t] = __ldg(reinterpret_cast<const uint4*>(a.qt) + static_cast<size_t>(bh) * (DSEL / 8) + t);
+        const int r0 = m0 + warp * 32;
+        const int rows = max(0, min(32, C - r0));
+        if (rows > 0 && lane == 0) {
+            const uint32_t bytes = static_cast<uint32_t>(rows) * kRowBytes;
+            mbar_arrive_expect_tx(&bars[warp], bytes);
+            bulk_load(stage + warp * kSlab,
+                      static_cast<const bf16*>(a.Ksum) + (static_cast<size_t>(bh) * a.max_blocks + r0) * DSEL, bytes,
+                      &bars[warp]);
+        }
+        __syncthreads();   // q~ in shared memory
+        if (rows > 0) {
+            const bool ok = mbar_wait_drain(&bars[warp], 0, limit, status);
+            if (ok && lane < rows) {
+                const uint4* krow = reinterpret_cast<const uint4*>(stage + warp * kSlab + lane * kRowBytes);
+                constexpr int NCH = DSEL / 8;
+                uint64_t acc = 0;
+#pragma unroll
+                for (int j = 0; j < NCH; ++j) {
+                    const int c = (j + lane) & (NCH - 1);   // rotated: a quarter warp hits distinct banks
+                    const uint4 kv = krow[c], qv = qs[c];
+                    acc = fma_f32x2(f32x2(bf_lo(kv.x), bf_hi(kv.x)), f32x2(bf_lo(qv.x), bf_hi(qv.x)), acc);
+                    acc = fma_f32x2(f32x2(bf_lo(kv.y), bf_hi(kv.y)), f32x2(bf_lo(qv.y), bf_hi(qv.y)), acc);
+                    acc = fma_f32x2(f32x2(bf_lo(kv.z), bf_hi(kv.z)), f32x2(bf_lo(qv.z), bf_hi(qv.z)), acc);
+                    acc = fma_f32x2(f32x2(bf_lo(kv.w), bf_hi(kv.w)), f32x2(bf_lo(qv.w), bf_hi(qv.w)), acc);
+                }
+                float s0, s1;
+                f32x2_split(acc, s0, s1);
+                a.scores[static_cast<size_t>(bh) * a.max_blocks + r0 + lane] = (s0 + s1) * score_scale;
+            }
+        }
+    }
+    // the last CTA of the group to finish selects
+    __threadfence();
+    __syncthreads();
+    if (t == 0) {
+        const int old = atomicAdd(a.cnt_sel + bh, 1);
+        misc[0] = old == static_cast<int>(gridDim.x) - 1;
+    }
+    __syncthreads();
+    if (!misc[0]) return;
+    __threadfence();
+    if (t == 0) a.cnt_sel[bh] = 0;   // zero again for the next launch
+    select_group(a, bh, C, reinterpret_cast<uint32_t*>(stage), reinterpret_cast<int*>(smem + L.hist),
+                 reinterpret_cast<int*>(smem + L.scan), misc + 1);
+}
+
+// ---------------------------------------------------------------- attention
+
+template <int D, int G>
+struct AttnSmem {
+    static constexpr int kTile = kBlk * D * 2;                 // one K or V page slice
+    static constexpr int RING = 0;
+    static constexpr int Q32 = kStages * 2 * kTile;            // fp32 queries [G][D]
+    static constexpr int PS = Q32 + G * D * 4;                 // probabilities [G][64]
+    static constexpr int RED = PS + G * 64 * 4;                // [4 warps][8]
+    static constexpr int ALPHA = RED + 32 * 4;                 // [8]
+    static constexpr int LSUM = ALPHA + 8 * 4;                 // [4 warps][8]
+    static constexpr int BARS = LSUM + 32 * 4;                 // kStages mbarriers
+    static constexpr int MISC = BARS + 64;                     // flag
+    static constexpr int ENT = MISC + 64;                      // entries: block, page (2 ints each)
+};
+
+__host__ __device__ inline size_t attn_smem_bytes(int D, int G, int bpc) {
+    const size_t tile = static_cast<size_t>(kBlk) * D * 2;
+    return kStages * 2 * tile + static_cast<size_t>(G) * D * 4 + static_cast<size_t>(G) * 64 * 4 + (32 + 8 + 32) * 4 +
+           64 + 64 + static_cast<size_t>(bpc) * 8;
+}
+
+// grid (nsplit_a, B*Hkv).  The group's list: the kept blocks (ascending) and then
+// the current block c; this CTA takes entries [x*bpc, (x+1)*bpc).
+template <int D, int G>
+__global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, int* status, long long limit,
+                                                                float scale_log2) {
+    using S = AttnSmem<D, G>;
+    constexpr int kTile = S::kTile;
+    constexpr int kNW = D / 2;                          // bf16 pairs per row
+    constexpr int HP = (G + 1) / 2;                     // heads per thread in the score step
+    constexpr int NHG = kAttnThreads / kNW;             // head groups in the PV step
+    constexpr int HPV = (G + NHG - 1) / NHG;            // heads per thread in the PV step
+    constexpr int NCH = D / 8;                          // 16-byte chunks per row
+    extern __shared__ __align__(128) uint8_t smem[];
+    float* q32 = reinterpret_cast<float*>(smem + S::Q32);
+    float* Ps = reinterpret_cast<float*>(smem + S::PS);
+    float* red = reinterpret_cast<float*>(smem + S::RED);
+    float* alpha_s = reinterpret_cast<float*>(smem + S::ALPHA);
+    float* lsum = reinterpret_cast<float*>(smem + S::LSUM);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::BARS);
+    int* misc = reinterpret_cast<int*>(smem + S::MISC);
+    int* ent = reinterpret_cast<int*>(smem + S::ENT);
+
+    const int bh = blockIdx.y;
+    const int b = bh / a.Hkv, g = bh - b * a.Hkv;
+    const int n = __ldg(a.seq_lens + b);
+    if (bad_len(n, a)) return;   // recorded by the prep kernel
+    const int c = (n - 1) / kBlk;
+    const int L = (a.dense ? c : __ldg(a.list_n + bh)) + 1;
+    const int j0 = blockIdx.x * a.bpc;
+    const int cnt = max(0, min(j0 + a.bpc, L) - j0);
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+
+    for (int jj = t; jj < cnt; jj += kAttnThreads) {
+        const int j = j0 + jj;
+        const int blk = j == L - 1 ? c : (a.dense ? j : __ldg(a.list + static_cast<size_t>(bh) * 64 + j));
+        int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + blk);
+        if (page < 0 || page >= a.num_pages) {
+            atomicExch(status, kStatusBadInput);
+            page = -1;
+        }
+        ent[2 * jj] = blk;
+        ent[2 * jj + 1] = page;
+    }
+    const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G) * D;
+    for (int e = t; e < G * D; e += kAttnThreads) q32[e] = __bfloat162float(qg[e]);
+    if (t == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    const size_t head_off = static_cast<size_t>(g) * kBlk * D;   // this KV head's slice inside a page
+    auto issue = [&](int jj) {
+        const int s = jj % kStages;
+        const int page = ent[2 * jj + 1];
+        uint8_t* dst = smem + S::RING + s * 2 * kTile;
+        if (page < 0) {
+            mbar_arrive(&full[s]);
+            return;
+        }
+        const size_t off = static_cast<size_t>(page) * a.Hkv * kBlk * D + head_off;
+        mbar_arrive_expect_tx(&full[s], 2 * kTile);
+        bulk_load(dst, static_cast<const bf16*>(a.K_cache) + off, kTile, &full[s]);
+        bulk_load(dst + kTile, static_cast<const bf16*>(a.V_cache) + off, kTile, &full[s]);
+    };
+    int issued = 0;
+    if (t == 0) {
+        for (; issued < min(cnt, kStages); ++issued) issue(issued);
+    }
+
+    const int k = t & 63, hh = t >> 6;           // score step: key k, heads hh*HP + u
+    const int wi = t % kNW, hg = t / kNW;        // PV step: column pair wi, heads hg*HPV + u
+    float m_run[HP], l_part[HP];
+#pragma unroll
+    for (int u = 0; u < HP; ++u) {
+        m_run[u] = -CUDART_INF_F;
+        l_part[u] = 0.f;
+    }
+    uint64_t acc[HPV];
+#pragma unroll
+    for (int u = 0; u < HPV; ++u) acc[u] = 0;
+
+    bool ok = true;
+    int jj = 0;
+    for (; jj < cnt; ++jj) {
+        const int s = jj % kStages;
+        const bool got = mbar_wait_drain(&full[s], (jj / kStages) & 1, limit, status);
+        if (!__syncthreads_and(got)) {
+            ok = false;
+            break;
+        }
+        const int page = ent[2 * jj + 1];
+        const int nvalid = page < 0 ? 0 : (ent[2 * jj] == c ? n - c * kBlk : kBlk);
+        const uint8_t* Kt = smem + S::RING + s * 2 * kTile;
+        const uint8_t* Vt = Kt + kTile;
+
+        // z = scale * q_h . k for this thread's key and heads (log2 units)
+        float z[HP];
+        {
+            uint64_t az[HP];
+#pragma unroll
+            for (int u = 0; u < HP; ++u) az[u] = 0;
+            const uint4* krow = reinterpret_cast<const uint4*>(Kt + k * D * 2);
+#pragma unroll
+            for (int jc = 0; jc < NCH; ++jc) {
+                const int cc = (jc + k) & (NCH - 1);    // rotated chunk: no bank conflicts across keys
+                const uint4 kv = krow[cc];
+                const uint64_t k01 = f32x2(bf_lo(kv.x), bf_hi(kv.x));
+                const uint64_t k23 = f32x2(bf_lo(kv.y), bf_hi(kv.y));
+                const uint64_t k45 = f32x2(bf_lo(kv.z), bf_hi(kv.z));
+                const uint64_t k67 = f32x2(bf_lo(kv.w), bf_hi(kv.w));
+#pragma unroll
+                for (int u = 0; u < HP; ++u) {
+                    const int h = hh * HP + u;
+                    if (h < G) {
+                        const float4 qa = *reinterpret_cast<const float4*>(q32 + h * D + cc * 8);
+                        const float4 qb = *reinterpret_cast<const float4*>(q32 + h * D + cc * 8 + 4);
+                        az[u] = fma_f32x2(k01, f32x2(qa.x, qa.y), az[u]);
+                        az[u] = fma_f32x2(k23, f32x2(qa.z, qa.w), az[u]);
+                        az[u] = fma_f32x2(k45, f32x2(qb.x, qb.y), az[u]);
+                        az[u] = fma_f32x2(k67, f32x2(qb.z, qb.w), az[u]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < HP; ++u) {
+                float z0, z1;
+                f32x2_split(az[u], z0, z1);
+                z[u] = k < nvalid ? (z0 + z1) * scale_log2 : -CUDART_INF_F;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < HP; ++u) {
+            const float mx = warp_max(z[u]);
+            if (lane == 0) red[warp * 8 + u] = mx;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < HP; ++u) {
+            const int h = hh * HP + u;
+            if (h < G) {
+                const float mb = fmaxf(red[(2 * hh) * 8 + u], red[(2 * hh + 1) * 8 + u]);
+                const float m_new = fmaxf(m_run[u], mb);
+                const float alpha = m_run[u] == -CUDART_INF_F ? 0.f : fast_exp2(m_run[u] - m_new);
+                const float p = z[u] == -CUDART_INF_F ? 0.f : fast_exp2(z[u] - m_new);
+                l_part[u] = l_part[u] * alpha + p;
+                m_run[u] = m_new;
+                Ps[h * 64 + k] = p;
+                if (k == 0) alpha_s[h] = alpha;
+            }
+        }
+        __syncthreads();
+        // O_h = alpha_h O_h + sum_k p_hk v_k for this thread's column pair
+#pragma unroll
+        for (int u = 0; u < HPV; ++u) {
+            const int h = hg * HPV + u;
+            if (h < G) {
+                const float al = alpha_s[h];
+                acc[u] = fma_f32x2(acc[u], f32x2(al, al), 0ull);
+            }
+        }
+        const uint32_t* V32 = reinterpret_cast<const uint32_t*>(Vt);
+#pragma unroll 4
+        for (int kk = 0; kk < nvalid; ++kk) {
+            const uint32_t w = V32[kk * kNW + wi];
+            const uint64_t v2 = f32x2(bf_lo(w), bf_hi(w));
+#pragma unroll
+            for (int u = 0; u < HPV; ++u) {
+                const int h = hg * HPV + u;
+                if (h < G) {
+                    const float p = Ps[h * 64 + kk];
+                    acc[u] = fma_f32x2(f32x2(p, p), v2, acc[u]);
+                }
+            }
+        }
+        __syncthreads();   // the stage, Ps and red are free
+        if (t == 0 && issued < cnt) {
+            fence_proxy_async_smem();
+            issue(issued);
+            ++issued;
+        }
+    }
+    if (!ok) {
+        // let copies still in flight land before the CTA exits; report nothing
+        if (t == 0)
+            for (int q = jj; q < issued; ++q) mbar_wait_drain(&full[q % kStages], (q / kStages) & 1, limit, status);
+#pragma unroll
+        for (int u = 0; u < HP; ++u) {
+            m_run[u] = -CUDART_INF_F;
+            l_part[u] = 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < HPV; ++u) acc[u] = 0;
+    }
+
+    // partial (max, sum, output) of this CTA per head
+#pragma unroll
+    for (int u = 0; u < HP; ++u) {
+        const float ls = warp_sum(l_part[u]);
+        if (lane == 0) lsum[warp * 8 + u] = ls;
+    }
+    __syncthreads();
+    float* part = a.part + (static_cast<size_t>(bh) * a.nsplit_a + blockIdx.x) * G * (D + 2);
+    if (k == 0) {
+#pragma unroll
+        for (int u = 0; u < HP; ++u) {
+            const int h = hh * HP + u;
+            if (h < G) {
+                part[h * (D + 2)] = m_run[u];
+                part[h * (D + 2) + 1] = lsum[(2 * hh) * 8 + u] + lsum[(2 * hh + 1) * 8 + u];
+            }
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < HPV; ++u) {
+        const int h = hg * HPV + u;
+        if (h < G) {
+            float o0, o1;
+            f32x2_split(acc[u], o0, o1);
+            part[h * (D + 2) + 2 + 2 * wi] = o0;
+            part[h * (D + 2) + 3 + 2 * wi] = o1;
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (t == 0) {
+        const int old = atomicAdd(a.cnt_attn + bh, 1);
+        misc[0] = old == static_cast<int>(gridDim.x) - 1;
+    }
+    __syncthreads();
+    if (!misc[0]) return;
+    __threadfence();
+    if (t == 0) a.cnt_attn[bh] = 0;   // zero again for the next launch
+
+    // merge the nsplit_a partials of every head
+    const float* pg = a.part + static_cast<size_t>(bh) * a.nsplit_a * G * (D + 2);
+#pragma unroll
+    for (int u = 0; u < HPV; ++u) {
+        const int h = hg * HPV + u;
+        if (h >= G) continue;
+        float M = -CUDART_INF_F;
+        for (int x = 0; x < a.nsplit_a; ++x) M = fmaxf(M, __ldcg(pg + (static_cast<size_t>(x) * G + h) * (D + 2)));
+        float lsum_all = 0.f, o0 = 0.f, o1 = 0.f;
+        for (int x = 0; x < a.nsplit_a; ++x) {
+            const float* px = pg + (static_cast<size_t>(x) * G + h) * (D + 2);
+            const float mx = __ldcg(px);
+            if (mx == -CUDART_INF_F) continue;
+            const float w = fast_exp2(mx - M);
+            lsum_all = fmaf(w, __ldcg(px + 1), lsum_all);
+            o0 = fmaf(w, __ldcg(px + 2 + 2 * wi), o0);
+            o1 = fmaf(w, __ldcg(px + 3 + 2 * wi), o1);
+        }
+        const float inv = 1.f / lsum_all;
+        const size_t orow = (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h) * D;
+        reinterpret_cast<uint32_t*>(static_cast<bf16*>(a.O) + orow)[wi] = pack_bf16x2(o0 * inv, o1 * inv);
+        if (a.LSE != nullptr && wi == 0)
+            a.LSE[static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h] = (M + log2f(lsum_all)) / kLog2e;
+    }
+}
+
+// Raises the kernel's dynamic shared-memory limit to what these arguments need
+// (called when a handle is created, so that a captured step sets nothing).
+template <int D, int G>
+cudaError_t prepare_attn_dg(const DecodeArgs& a) {
+    const size_t smem = attn_smem_bytes(D, G, a.bpc);
+    static size_t set = 0;
+    if (smem > set) {
+        cudaError_t e = cudaFuncSetAttribute(dec_attn_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        set = smem;
+    }
+    return cudaSuccess;
+}
+
+template <int D, int G>
+cudaError_t launch_attn_dg(const DecodeArgs& a, const KernelEnv& env) {
+    const size_t smem = attn_smem_bytes(D, G, a.bpc);
+    cudaError_t e = prepare_attn_dg<D, G>(a);
+    if (e != cudaSuccess) return e;
+    dim3 grid(a.nsplit_a, a.B * a.Hkv);
+    dec_attn_kernel<D, G><<<grid, kAttnThreads, smem, env.stream>>>(a, env.status, env.limit,
+                                                                     a.sm_scale * kLog2e);
+    return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_attn_d(const DecodeArgs& a, const KernelEnv& env) {
+    switch (a.G) {
+        case 1: return launch_attn_dg<D, 1>(a, env);
+        case 2: return launch_attn_dg<D, 2>(a, env);
+        case 4: return launch_attn_dg<D, 4>(a, env);
+        case 8: return launch_attn_dg<D, 8>(a, env);
+    }
+    return cudaErrorInvalidValue;
+}
+
+template <int D>
+cudaError_t prepare_attn_d(const DecodeArgs& a) {
+    switch (a.G) {
+        case 1: return prepare_attn_dg<D, 1>(a);
+        case 2: return prepare_attn_dg<D, 2>(a);
+        case 4: return prepare_attn_dg<D, 4>(a);
+        case 8: return prepare_attn_dg<D, 8>(a);
+    }
+    return cudaErrorInvalidValue;
+}
+
+template <int DSEL>
+cudaError_t prepare_score_d(const DecodeArgs& a) {
+    const size_t smem = score_smem_layout(a.max_blocks, DSEL).total;
+    static size_t set = 0;
+    if (smem > set) {
+        cudaError_t e = cudaFuncSetAttribute(dec_score_kernel<DSEL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        set = smem;
+    }
+    return cudaSuccess;
+}
+
+template <int DSEL>
+cudaError_t launch_score_d(const DecodeArgs& a, const KernelEnv& env) {
+    const size_t smem = score_smem_layout(a.max_blocks, DSEL).total;
+    cudaError_t e = prepare_score_d<DSEL>(a);
+    if (e != cudaSuccess) return e;
+    dim3 grid(a.nsplit_s, a.B * a.Hkv);
+    dec_score_kernel<DSEL><<<grid, kScoreThreads, smem, env.stream>>>(a, env.status, env.limit,
+                                                                     static_cast<float>(1.0 / sqrt(static_cast<double>(DSEL))));
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+void decode_attn_split(int max_len, int* nsplit, int* bpc) {
+    const int per = max_len <= 96 ? 2 : (max_len + 63) / 64;
+    *bpc = per;
+    *nsplit = (max_len + per - 1) / per;
+}
+
+size_t decode_score_smem(int max_blocks, int d_sel) { return score_smem_layout(max_blocks, d_sel).total; }
+
+size_t decode_attn_smem(int d, int G, int bpc) { return attn_smem_bytes(d, G, bpc); }
+
+cudaError_t decode_prepare(const DecodeArgs& a) {
+    cudaError_t e = cudaSuccess;
+    if (!a.dense) e = a.d_sel == 128 ? prepare_score_d<128>(a) : prepare_score_d<64>(a);
+    if (e == cudaSuccess) e = a.d == 128 ? prepare_attn_d<128>(a) : prepare_attn_d<64>(a);
+    return e;
+}
+
+cudaError_t launch_decode_prep(const DecodeArgs& a, const KernelEnv& env) {
+    dim3 grid(a.B * a.Hkv, a.dense ? 1 : 1 + (a.d_sel + 31) / 32);
+    dec_prep_kernel<<<grid, kPrepThreads, 0, env.stream>>>(a, env.status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode_summarize(const DecodeArgs& a, const KernelEnv& env) {
+    dim3 grid(a.max_blocks, a.B * a.Hkv);
+    dec_summarize_kernel<<<grid, kPrepThreads, 0, env.stream>>>(a, env.status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode_score(const DecodeArgs& a, const KernelEnv& env) {
+    if (a.d_sel == 128) return launch_score_d<128>(a, env);
+    if (a.d_sel == 64) return launch_score_d<64>(a, env);
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_decode_attn(const DecodeArgs& a, const KernelEnv& env) {
+    if (a.d == 128) return launch_attn_d<128>(a, env);
+    if (a.d == 64) return launch_attn_d<64>(a, env);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace sas

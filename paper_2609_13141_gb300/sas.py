@@ -45,6 +45,17 @@ class SasConfig(ctypes.Structure):
                 ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32)]
 
 
+class SasDecodeConfig(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("d_sel", ctypes.c_int32), ("block", ctypes.c_int32), ("topk", ctypes.c_int32),
+                ("max_blocks", ctypes.c_int32), ("num_pages", ctypes.c_int32), ("sm_scale", ctypes.c_float),
+                ("dense", ctypes.c_int32)]
+
+
+SAS_DECODE_NUM_KERNEL_KINDS = 4
+DECODE_KERNEL_KINDS = ["prep", "score_topk", "attention", "summarize"]
+
+
 class SasError(RuntimeError):
     def __init__(self, status, message):
         super().__init__(f"{message} (status {status})")
@@ -89,6 +100,24 @@ def lib():
     L.sas_mlp_fwd_noalloc.restype = i32
     L.sas_selftest_wait_timeout.argtypes = [i64, ctypes.POINTER(i32)]
     L.sas_selftest_wait_timeout.restype = i32
+    L.sas_decode_create.argtypes = [ctypes.POINTER(SasDecodeConfig), ctypes.POINTER(vp)]
+    L.sas_decode_create.restype = i32
+    L.sas_decode_destroy.argtypes = [vp]
+    L.sas_decode_destroy.restype = None
+    L.sas_decode_summarize.argtypes = [vp] * 7
+    L.sas_decode_summarize.restype = i32
+    L.sas_decode_step.argtypes = [vp] * 15
+    L.sas_decode_step.restype = i32
+    L.sas_decode_last_error.argtypes = [vp]
+    L.sas_decode_last_error.restype = ctypes.c_char_p
+    L.sas_decode_get_device_status.argtypes = [vp, ctypes.POINTER(i32)]
+    L.sas_decode_get_device_status.restype = i32
+    L.sas_decode_set_timing.argtypes = [vp, i32]
+    L.sas_decode_set_timing.restype = i32
+    L.sas_decode_get_timings.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(ctypes.c_double), i32]
+    L.sas_decode_get_timings.restype = i32
+    L.sas_decode_launch_count.argtypes = [vp]
+    L.sas_decode_launch_count.restype = i64
     _lib = L
     return L
 
@@ -261,6 +290,121 @@ class SasLayer:
     def close(self):
         if self.h is not None:
             sas_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# ------------------------------------------------------------------ decode
+
+
+def _dcheck(status, handle, what):
+    if status != SAS_OK:
+        L = lib()
+        msg = L.sas_status_str(status).decode()
+        if handle is not None:
+            detail = L.sas_decode_last_error(handle).decode()
+            if detail:
+                msg += ": " + detail
+        raise SasError(status, f"{what}: {msg}")
+
+
+def sas_decode_create(B, Hq, Hkv, d, topk, max_blocks, num_pages, d_sel=0, sm_scale=0.0, dense=False, block=64):
+    cfg = SasDecodeConfig(B, Hq, Hkv, d, d_sel, block, topk, max_blocks, num_pages, sm_scale, 1 if dense else 0)
+    h = ctypes.c_void_p()
+    _dcheck(lib().sas_decode_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_decode_create")
+    return h
+
+
+def sas_decode_create_status(B, Hq, Hkv, d, topk, max_blocks, num_pages, d_sel=0, sm_scale=0.0, dense=0, block=64):
+    """Raw status of sas_decode_create (argument-check tests); destroys the handle on success."""
+    cfg = SasDecodeConfig(B, Hq, Hkv, d, d_sel, block, topk, max_blocks, num_pages, sm_scale, dense)
+    h = ctypes.c_void_p()
+    st = lib().sas_decode_create(ctypes.byref(cfg), ctypes.byref(h))
+    if st == SAS_OK:
+        lib().sas_decode_destroy(h)
+    return st
+
+
+def sas_decode_destroy(h):
+    lib().sas_decode_destroy(h)
+
+
+def sas_decode_summarize(h, K_cache, block_table, seq_lens, Wk, Ksum, stream=None):
+    bf, i32 = torch.bfloat16, torch.int32
+    st = lib().sas_decode_summarize(h, _ptr(K_cache, bf, "K_cache"), _ptr(block_table, i32, "block_table"),
+                                    _ptr(seq_lens, i32, "seq_lens"), _ptr(Wk, bf, "Wk"), _ptr(Ksum, bf, "Ksum"),
+                                    _stream(stream))
+    _dcheck(st, h, "sas_decode_summarize")
+
+
+def sas_decode_step(h, q, K_cache, V_cache, block_table, seq_lens, O, k_new=None, v_new=None, Wq=None, Wk=None,
+                    Ksum=None, LSE=None, sel_idx=None, stream=None):
+    bf, i32 = torch.bfloat16, torch.int32
+    st = lib().sas_decode_step(
+        h, _ptr(q, bf, "q"), _ptr(k_new, bf, "k_new", False), _ptr(v_new, bf, "v_new", False),
+        _ptr(K_cache, bf, "K_cache"), _ptr(V_cache, bf, "V_cache"), _ptr(block_table, i32, "block_table"),
+        _ptr(seq_lens, i32, "seq_lens"), _ptr(Wq, bf, "Wq", False), _ptr(Wk, bf, "Wk", False),
+        _ptr(Ksum, bf, "Ksum", False), _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False),
+        _ptr(sel_idx, i32, "sel_idx", False), _stream(stream))
+    _dcheck(st, h, "sas_decode_step")
+
+
+def sas_decode_get_device_status(h):
+    v = ctypes.c_int32(0)
+    _dcheck(lib().sas_decode_get_device_status(h, ctypes.byref(v)), h, "sas_decode_get_device_status")
+    return v.value
+
+
+def sas_decode_set_timing(h, enable):
+    _dcheck(lib().sas_decode_set_timing(h, 1 if enable else 0), h, "sas_decode_set_timing")
+
+
+def sas_decode_get_timings(h):
+    n = SAS_DECODE_NUM_KERNEL_KINDS
+    launches = (ctypes.c_int64 * n)()
+    ms = (ctypes.c_double * n)()
+    _dcheck(lib().sas_decode_get_timings(h, launches, ms, n), h, "sas_decode_get_timings")
+    return {DECODE_KERNEL_KINDS[k]: (launches[k], ms[k]) for k in range(n)}
+
+
+def sas_decode_launch_count(h):
+    return lib().sas_decode_launch_count(h)
+
+
+class SasDecoder:
+    """Owns one decode handle; allocates the step's outputs and calls the C ABI."""
+
+    def __init__(self, B, Hq, Hkv, d, topk, max_blocks, num_pages, d_sel=0, sm_scale=0.0, dense=False):
+        self.B, self.Hq, self.Hkv, self.d, self.topk = B, Hq, Hkv, d, topk
+        self.dense = dense
+        self.h = sas_decode_create(B, Hq, Hkv, d, topk, max_blocks, num_pages, d_sel, sm_scale, dense)
+
+    def summarize(self, K_cache, block_table, seq_lens, Wk, Ksum, stream=None):
+        sas_decode_summarize(self.h, K_cache, block_table, seq_lens, Wk, Ksum, stream)
+
+    def step(self, q, K_cache, V_cache, block_table, seq_lens, k_new=None, v_new=None, Wq=None, Wk=None, Ksum=None,
+             out=None, stream=None):
+        """Returns (O, LSE, sel_idx); sel_idx is None in dense mode.  out = (O, LSE, sel_idx)
+        reuses caller buffers (as a captured graph needs)."""
+        if out is None:
+            O = torch.empty(self.B, self.Hq, self.d, device=q.device, dtype=torch.bfloat16)
+            LSE = torch.empty(self.B, self.Hq, device=q.device, dtype=torch.float32)
+            sel = None if self.dense else torch.empty(self.B, self.Hkv, max(self.topk, 1), device=q.device,
+                                                      dtype=torch.int32)
+        else:
+            O, LSE, sel = out
+        sas_decode_step(self.h, q, K_cache, V_cache, block_table, seq_lens, O, k_new, v_new, Wq, Wk, Ksum, LSE,
+                        sel, stream)
+        return O, LSE, sel
+
+    def close(self):
+        if self.h is not None:
+            sas_decode_destroy(self.h)
             self.h = None
 
     def __del__(self):

@@ -102,3 +102,77 @@ def mlp(T, D, F, seed=0, std=0.02, bias=False):
     b1 = normal((F,), seed + 43, std).to(torch.bfloat16)
     b2 = normal((D,), seed + 44, std).to(torch.bfloat16)
     return X, W1, W2, b1, b2
+
+
+# ------------------------------------------------------------------ decode
+
+def _dev_normal(shape, seed, device, std=1.0):
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed))
+    return torch.randn(*shape, generator=g, device=device, dtype=torch.float32) * std
+
+
+def decode_layout(lens, max_blocks, seed=0, spare_pages=3, block=64):
+    """Page assignment of a paged decode cache.
+
+    lens: tokens each sequence will hold.  Every sequence gets ceil(len/64)
+    pages out of a seeded permutation of P = sum + spare_pages pages; block
+    table entries past a sequence's last page are -1.  Returns (block_table
+    int32 [B, max_blocks], P)."""
+    need = [-(-int(n) // block) for n in lens]
+    P = sum(need) + spare_pages
+    perm = torch.randperm(P, generator=_gen(seed + 60))
+    table = torch.full((len(lens), max_blocks), -1, dtype=torch.int32)
+    k = 0
+    for bi, c in enumerate(need):
+        table[bi, :c] = perm[k:k + c].to(torch.int32)
+        k += c
+    return table, P
+
+
+def decode_cache(P, Hkv, d, seed=0, device="cpu", exact=False, block=64):
+    """K, V pages [P, Hkv, 64, d] as bf16.  Keys are block-coherent,
+    k = (mu_page + 0.5 eps) / sqrt(1.25), so block summaries differ from block
+    to block; values N(0, 1).  exact=True: keys are integers in [-3, 3]."""
+    if exact:
+        g = torch.Generator(device=device)
+        g.manual_seed(int(seed + 70))
+        K = torch.randint(-3, 4, (P, Hkv, block, d), generator=g, device=device).to(torch.bfloat16)
+    else:
+        mu = _dev_normal((P, Hkv, 1, d), seed + 71, device)
+        K = ((mu + 0.5 * _dev_normal((P, Hkv, block, d), seed + 72, device)) / math.sqrt(1.25)).to(torch.bfloat16)
+    V = _dev_normal((P, Hkv, block, d), seed + 73, device).to(torch.bfloat16)
+    return K, V
+
+
+def decode_queries(B, Hq, Hkv, d, seed=0, device="cpu", exact=False):
+    """q [B, Hq, d], k_new and v_new [B, Hkv, d] as bf16 (integers in [-3, 3]
+    for q and k_new when exact)."""
+    if exact:
+        g = torch.Generator(device=device)
+        g.manual_seed(int(seed + 80))
+        q = torch.randint(-3, 4, (B, Hq, d), generator=g, device=device).to(torch.bfloat16)
+        kn = torch.randint(-3, 4, (B, Hkv, d), generator=g, device=device).to(torch.bfloat16)
+    else:
+        q = _dev_normal((B, Hq, d), seed + 81, device).to(torch.bfloat16)
+        kn = _dev_normal((B, Hkv, d), seed + 82, device).to(torch.bfloat16)
+    vn = _dev_normal((B, Hkv, d), seed + 83, device).to(torch.bfloat16)
+    return q, kn, vn
+
+
+def decode_selector_weights(Hkv, G, d, d_sel, seed=0, device="cpu", exact=False, std=0.02, nnz=4):
+    """Wq [Hkv, d_sel, G*d] and Wk [Hkv, d_sel, d] as bf16; exact=True gives
+    sparse {-1, 0, 1} rows with nnz non-zeros."""
+    if not exact:
+        Wq = _dev_normal((Hkv, d_sel, G * d), seed + 90, device, std).to(torch.bfloat16)
+        Wk = _dev_normal((Hkv, d_sel, d), seed + 91, device, std).to(torch.bfloat16)
+        return Wq, Wk
+    g = _gen(seed + 92)
+    out = []
+    for width in (G * d, d):
+        w = torch.zeros(Hkv, d_sel, width)
+        cols = torch.stack([torch.randperm(width, generator=g)[:nnz] for _ in range(Hkv * d_sel)])
+        sign = torch.randint(0, 2, (Hkv * d_sel, nnz), generator=g).float() * 2 - 1
+        w.view(Hkv * d_sel, width).scatter_(1, cols, sign)
+        out.append(w.to(torch.bfloat16).to(device))
+    return out[0], out[1]

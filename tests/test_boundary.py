@@ -73,3 +73,35 @@ def test_null_handle_and_null_arguments(lib):
 def test_binding_refuses_cpu_tensors(lib):
     with pytest.raises(ValueError):
         sas._ptr(torch.zeros(4), torch.float32, "x")
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(B=0, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=32), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=12, Hkv=8, d=128, topk=4, max_blocks=16, num_pages=32), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=24, Hkv=8, d=128, topk=4, max_blocks=16, num_pages=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=96, topk=4, max_blocks=16, num_pages=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=128, d_sel=32, topk=4, max_blocks=16, num_pages=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=-1, max_blocks=16, num_pages=32), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=65, max_blocks=16, num_pages=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=0, num_pages=32), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=40000, num_pages=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=0), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=32, dense=2), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=32, block=32), sas.SAS_ERR_UNSUPPORTED),
+    (dict(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=32, sm_scale=math.nan), sas.SAS_ERR_INVALID_ARG),
+])
+def test_decode_create_rejects_bad_configs(lib, kw, expect):
+    assert sas.sas_decode_create_status(**kw) == expect
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU path")
+def test_decode_create_without_gpu_fails_cleanly(lib):
+    st = sas.sas_decode_create_status(B=1, Hq=8, Hkv=2, d=128, topk=4, max_blocks=16, num_pages=32)
+    assert st in (sas.SAS_ERR_CUDA, sas.SAS_ERR_UNSUPPORTED)
+
+
+def test_decode_null_handle(lib):
+    null = ctypes.c_void_p()
+    assert lib.sas_decode_step(null, *([None] * 14)) == sas.SAS_ERR_INVALID_ARG
+    assert lib.sas_decode_summarize(null, *([None] * 6)) == sas.SAS_ERR_INVALID_ARG
+    assert lib.sas_decode_launch_count(null) == 0
