@@ -10,6 +10,12 @@ d=128, b=64, K=32, learned selector with d_sel=128, MLP 9216 x 3072 -> 12288
 
 Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
 bounded sample of the same workload instead.
+
+--workload decode times the SAS decode step instead (Alg. 2 with per-group
+block selection over a paged KV cache): a Qwen3-4B-shaped attention layer
+(32 query heads, 8 KV heads, d=128, b=64, K=32 = a 2048-token budget) at
+--context tokens for --batch sequences, captured in a CUDA graph, next to the
+dense decode of the same cache.
 """
 from __future__ import annotations
 
@@ -434,13 +440,244 @@ def run_reference(args, w, rank, world):
     }
 
 
+# ---------------------------------------------------------------- decode
+
+DECODE_METRIC = "decode step latency of one attention layer (us), SAS vs dense, 1xGB300"
+
+
+def decode_bytes(B, Hq, Hkv, d, ds, K, n, dense):
+    """Algorithmic HBM bytes of one decode step and of each kernel kind for B
+    sequences of n cached tokens (new token included)."""
+    G = Hq // Hkv
+    C = (n - 1) // 64
+    cur = n - 64 * C
+    groups = B * Hkv
+    kv_tokens = (C if dense else min(K, C)) * 64 + cur
+    attn = groups * (2 * 2 * kv_tokens * d + 2 * G * d * 2)           # K, V pages; q in, O out
+    prep = groups * (4 * 2 * d + (0 if dense else 2 * ds * G * d + 2 * G * d))   # append; Wq and q
+    score = 0 if dense else groups * (2 * C * ds + 2 * ds)          # summaries and q~
+    return {"prep": prep, "score_topk": score, "attention": attn, "total": prep + score + attn}
+
+
+def decode_oracle_us(B, Hq, Hkv, d, ds, K, n, budget_s, seed=0):
+    """Oracle (numpy fp64) time of one decode step, from groups run on the host
+    cores until the budget is spent, scaled to the B*Hkv groups of a step."""
+    import numpy as np
+    import torch
+
+    from oracle import decode_oracle as DO
+    from paper_2609_13141_gb300 import synth
+
+    G = Hq // Hkv
+    nb = -(-n // 64)
+    Kc, Vc = synth.decode_cache(nb, 1, d, seed=seed)
+    q, _, _ = synth.decode_queries(1, G, 1, d, seed=seed)
+    Wq, Wk = synth.decode_selector_weights(1, G, d, ds, seed=seed)
+    f = lambda t: t.to(torch.float64).numpy()
+    Kx = f(Kc[:, 0].reshape(-1, d))[:n]
+    Vx = f(Vc[:, 0].reshape(-1, d))[:n]
+    qx, wq, wk = f(q[0]), f(Wq[0]), f(Wk[0])
+    t0 = time.perf_counter()
+    done = 0
+    while time.perf_counter() - t0 < budget_s or done == 0:
+        DO.decode_group(qx, Kx, Vx, wq, wk, 64, K)
+        done += 1
+    per_group = (time.perf_counter() - t0) / done
+    desc = (f"oracle (numpy fp64): {done} decode steps of one KV group ({G} query heads, {n} cached tokens, "
+            f"selector + Top-K + attention) in {per_group * done:.1f} s, scaled to the {B * Hkv} groups of a step")
+    return per_group * B * Hkv * 1e6, per_group * done, desc
+
+
+def run_decode(args, rank, world):
+    import torch
+
+    from paper_2609_13141_gb300 import sas, synth
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    B, Hq, Hkv, d, ds = args.batch, 32, 8, 128, 128
+    K = args.topk if args.topk is not None else 32
+    n = args.context
+    G = Hq // Hkv
+    max_blocks = -(-n // 64)
+    table, P = synth.decode_layout([n] * B, max_blocks, seed=rank)
+    Kc, Vc = synth.decode_cache(P, Hkv, d, seed=rank, device=dev)
+    q, kn, vn = synth.decode_queries(B, Hq, Hkv, d, seed=rank, device=dev)
+    Wq, Wk = synth.decode_selector_weights(Hkv, G, d, ds, seed=rank, device=dev)
+    Ksum = torch.zeros(B, Hkv, max_blocks, ds, device=dev, dtype=torch.bfloat16)
+    tab = table.to(dev)
+    lens = torch.full((B,), n, dtype=torch.int32, device=dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
+    stream = torch.cuda.Stream(dev)
+
+    def measure(dense):
+        dec = sas.SasDecoder(B, Hq, Hkv, d, K, max_blocks, P, d_sel=ds, dense=dense)
+        if not dense:
+            dec.summarize(Kc, tab, lens - 1, Wk, Ksum)
+        out = (torch.empty(B, Hq, d, device=dev, dtype=torch.bfloat16),
+               torch.empty(B, Hq, device=dev, dtype=torch.float32),
+               None if dense else torch.empty(B, Hkv, max(K, 1), device=dev, dtype=torch.int32))
+        args_ = (q, Kc, Vc, tab, lens, kn, vn, Wq, Wk, None if dense else Ksum)
+        with torch.cuda.stream(stream):
+            for _ in range(max(args.warmup, 3)):
+                dec.step(*args_, out=out, stream=stream)
+            # one timed step outside capture creates the timing events, so the
+            # capture below records existing events only
+            sas.sas_decode_set_timing(dec.h, True)
+            dec.step(*args_, out=out, stream=stream)
+        stream.synchronize()
+        # graph_t carries event nodes between the kernels for the per-kernel
+        # breakdown; they serialise the kernels, so the step itself is timed on
+        # a second graph without them (the kernels then overlap their set-up)
+        sas.sas_decode_set_timing(dec.h, True)
+        graph_t = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph_t, stream=stream):
+            dec.step(*args_, out=out, stream=stream)
+        sas.sas_decode_set_timing(dec.h, False)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            dec.step(*args_, out=out, stream=stream)
+        launches_per_step = 2 if dense else 3
+        for _ in range(max(args.warmup, 3)):
+            graph.replay()
+            graph_t.replay()
+        torch.cuda.synchronize()
+        per_kind = {}
+        with torch.cuda.stream(stream):
+            for k in range(args.steps):
+                flush.zero_()
+                graph_t.replay()
+                stream.synchronize()
+                for kind, (cnt, ms) in sas.sas_decode_get_timings(dec.h).items():
+                    if cnt:
+                        per_kind.setdefault(kind, []).append(ms)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        with torch.cuda.stream(stream):
+            for k in range(args.steps):
+                flush.zero_()
+                ev[k][0].record(stream)
+                graph.replay()
+                ev[k][1].record(stream)
+        torch.cuda.synchronize()
+        per_step = sorted(a.elapsed_time(b) * 1e3 for a, b in ev)
+        us = sum(per_step) / args.steps
+        spread = {"min": round(per_step[0], 2), "median": round(per_step[len(per_step) // 2], 2),
+                  "max": round(per_step[-1], 2)}
+        assert sas.sas_decode_get_device_status(dec.h) == 0
+        # end to end: the step's inputs from pinned host memory, its output back
+        hq, hkn, hvn = q.cpu().pin_memory(), kn.cpu().pin_memory(), vn.cpu().pin_memory()
+        hO = torch.empty(B, Hq, d, dtype=torch.bfloat16).pin_memory()
+        e2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        with torch.cuda.stream(stream):
+            for k in range(-2, args.steps):
+                flush.zero_()
+                if k >= 0:
+                    e2[k][0].record(stream)
+                q.copy_(hq, non_blocking=True)
+                kn.copy_(hkn, non_blocking=True)
+                vn.copy_(hvn, non_blocking=True)
+                graph.replay()
+                hO.copy_(out[0], non_blocking=True)
+                if k >= 0:
+                    e2[k][1].record(stream)
+        torch.cuda.synchronize()
+        e2e_us = sum(a.elapsed_time(b) for a, b in e2) / args.steps * 1e3
+        dec.close()
+        kern = {k: sum(v) / len(v) * 1e3 for k, v in per_kind.items()}
+        h2d = (q.numel() + kn.numel() + vn.numel()) * 2
+        return us, e2e_us, kern, launches_per_step * args.steps, h2d, hO.numel() * 2, spread
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.2)
+    us, e2e_us, kern, launches, h2d, d2h, spread = measure(False)
+    dus, de2e_us, dkern, _, _, _, dspread = measure(True)
+    clocks = sampler.stop()
+    us, e2e_us, dus = reduce_max([us, e2e_us, dus], dist, dev)
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return None
+    peaks = load_peaks()
+    by = decode_bytes(B, Hq, Hkv, d, ds, K, n, False)
+    dby = decode_bytes(B, Hq, Hkv, d, ds, K, n, True)
+
+    def roof(kern_us, bytes_):
+        dom = max(kern_us, key=kern_us.get)
+        ach = bytes_[dom] / (kern_us[dom] / 1e6) / 1e9
+        return {"bound": "hbm", "kernel": dom, "achieved": round(ach, 1), "peak": peaks["hbm"], "unit": "GB/s",
+                "frac": round(ach / peaks["hbm"], 4), "traffic": None,
+                "peak_source": f"{peaks['source']} HBM copy bandwidth"}
+
+    wname = (f"Qwen3-4B-shaped decode attention layer: Hq=32 Hkv=8 d=128 b=64, K={K} ({K * 64}-token budget), "
+             f"context {n} tokens, batch {B}, paged KV cache (one 64-token block per page)")
+    out = {
+        "metric": DECODE_METRIC, "value": round(us, 2), "unit": "us", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(us / 1e3, 5), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 (fp32 scores/softmax)",
+        "data": "synthetic (seeded; block-coherent keys, N(0,1) queries/values, selector weights N(0,0.02))",
+        "config": {"workload": wname, "B": B, "Hq": Hq, "Hkv": Hkv, "d": d, "d_sel": ds, "topk": K, "context": n,
+                   "graph": "one CUDA graph per step", "l2": "flushed between timed steps (256 MiB write)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roof(kern, by),
+        "kernels_us": {k: round(v, 2) for k, v in kern.items()},
+        "step_us_spread": spread,
+        "step_algorithmic_bytes": by["total"],
+        "step_gbs": round(by["total"] / (us / 1e6) / 1e9, 1),
+        "dense": {"us": round(dus, 2), "e2e_us": round(de2e_us, 2), "step_us_spread": dspread, "kernels_us": {k: round(v, 2) for k, v in dkern.items()},
+                  "roofline": roof(dkern, dby), "step_algorithmic_bytes": dby["total"],
+                  "step_gbs": round(dby["total"] / (dus / 1e6) / 1e9, 1)},
+        "speedup_vs_dense": round(dus / us, 2),
+        "e2e": {"value": round(e2e_us, 2), "unit": "us", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        v, secs, desc = decode_oracle_us(B, Hq, Hkv, d, ds, K, n, args.cpu_budget / 2)
+        out["cpu_baseline"] = {"value": round(v, 1), "unit": "us", "cores": _oracle_threads(), "kind": "oracle",
+                               "sample": desc, "seconds": round(secs, 2)}
+    if dist is not None:
+        dist.destroy_process_group()
+    return out
+
+
+def run_decode_reference(args, rank, world):
+    if rank != 0:
+        return None
+    K = args.topk if args.topk is not None else 32
+    vals = []
+    desc = ""
+    for k in range(args.warmup + args.steps):
+        v, _, desc = decode_oracle_us(args.batch, 32, 8, 128, 128, K, args.context, args.ref_step_s / 4, seed=k)
+        if k >= args.warmup:
+            vals.append(v)
+    value = sum(vals) / len(vals)
+    return {
+        "impl": "reference", "metric": DECODE_METRIC, "value": round(value, 1), "unit": "us", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(value / 1e3, 3), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+        "config": {"workload": f"Qwen3-4B-shaped decode attention layer, context {args.context}, batch {args.batch}",
+                   "B": args.batch, "context": args.context, "topk": K},
+        "cpu_baseline": {"value": round(value, 1), "unit": "us", "cores": _oracle_threads(), "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": round(value, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dit")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["decode"], default="dit")
+    ap.add_argument("--context", type=int, default=65536, help="decode: cached tokens per sequence")
+    ap.add_argument("--batch", type=int, default=1, help="decode: sequences per step")
     ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
                     help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
     ap.add_argument("--topk", type=int, default=None, help="override the workload's K")
@@ -450,6 +687,11 @@ def main():
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.workload == "decode":
+        out = run_decode_reference(args, rank, world) if args.impl == "reference" else run_decode(args, rank, world)
+        if out is not None and rank == 0:
+            print(json.dumps(out))
+        return
     w = dict(WORKLOADS[args.workload])
     if args.topk is not None:
         w["topk"] = args.topk

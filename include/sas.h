@@ -314,9 +314,14 @@ const char* sas_decode_last_error(const sas_decode_handle* h);
  * SAS_ERR_TIMEOUT for a bounded wait that ran out).  Synchronises. */
 sas_status sas_decode_get_device_status(sas_decode_handle* h, int32_t* out_status);
 
-/* Event timing per kernel kind, as sas_set_timing / sas_get_timings:
- * 0 append + summary + gate query, 1 scores + Top-K, 2 attention, 3 summary
- * fill (sas_decode_summarize).  n_kinds <= 4. */
+/* Event timing per kernel kind: sas_decode_set_timing(h, 1) starts recording
+ * (clearing earlier records), (h, 0) stops and keeps them; sas_decode_get_timings
+ * synchronises and sums launches and milliseconds per kind: 0 append + summary
+ * + gate query, 1 scores + Top-K, 2 attention, 3 summary fill
+ * (sas_decode_summarize).  n_kinds <= 4.  Steps recorded while a stream is
+ * captured get external event nodes in the graph (which serialise the
+ * kernels); each replay re-records them, and the timings then read the latest
+ * replay. */
 #define SAS_DECODE_NUM_KERNEL_KINDS 4
 sas_status sas_decode_set_timing(sas_decode_handle* h, int32_t enable);
 sas_status sas_decode_get_timings(sas_decode_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds);

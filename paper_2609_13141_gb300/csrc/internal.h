@@ -105,21 +105,22 @@ struct DecodeArgs {
     int32_t* sel_idx;           // [B][Hkv][topk] or null
     // workspace
     void* qt;                   // bf16 [B*Hkv][d_sel] gate queries
-    float* scores;              // [B*Hkv][max_blocks]
+    uint32_t* cand_key;         // [B*Hkv][nsplit_s][max(topk,1)] per-CTA Top-K candidates (order keys)
+    int32_t* cand_idx;          // [B*Hkv][nsplit_s][max(topk,1)] their blocks (-1: empty slot)
     int32_t* list;              // [B*Hkv][64] kept blocks, ascending
     int32_t* list_n;            // [B*Hkv]
     float* part;                // [B*Hkv][nsplit_a][G][d + 2] split-attention partials
     int* cnt_sel;               // [B*Hkv] arrival counters, zero between launches
     int* cnt_attn;              // [B*Hkv]
     int nsplit_s;               // score CTAs per group (kDecScoreChunk blocks each)
-    int nsplit_a, bpc;          // attention CTAs per group, list entries per CTA
+    int nsplit_a, bpc, nst;     // attention CTAs per group, list entries per CTA, ring stages
 };
 constexpr int kDecScoreChunk = 256;
 // Attention split for a group list of at most max_len entries.
-void decode_attn_split(int max_len, int* nsplit, int* bpc);
+void decode_attn_split(int max_len, int* nsplit, int* bpc, int* nst);
 // Dynamic shared memory the score and attention kernels need.
-size_t decode_score_smem(int max_blocks, int d_sel);
-size_t decode_attn_smem(int d, int G, int bpc);
+size_t decode_score_smem(int nsplit, int topk, int d_sel);
+size_t decode_attn_smem(int d, int G, int nst, int bpc);
 // Sets the kernels' shared-memory limits for these arguments (before any capture).
 cudaError_t decode_prepare(const DecodeArgs& a);
 cudaError_t launch_decode_prep(const DecodeArgs& a, const KernelEnv& env);

@@ -7,15 +7,21 @@
 //                      forms the group's gate query q~ = bf16(Wq_g [q_0; ...]).
 //   dec_score_kernel   s_m = q~ . K~_m / sqrt(d_sel) for the C historical blocks
 //                      (Alg. 2 step 1), CTAs of 256 blocks whose summary rows are
-//                      staged in shared memory by bulk async copies; the last CTA
-//                      of a group takes the exact Top-K (step 2) by a radix select
-//                      on the scores' order-preserving bit patterns, ties to the
-//                      lower block, and writes the kept list in ascending order.
+//                      staged in shared memory by bulk async copies.  Each CTA keeps
+//                      the exact Top-K of its own blocks (rank by counting); the
+//                      last CTA of a group selects the Top-K of those candidates
+//                      (step 2) by a radix select on the scores' order-preserving
+//                      bit patterns, ties to the lower block, and writes the kept
+//                      list in ascending order.
 //   dec_attn_kernel    split-KV attention over B_0 and the kept blocks (steps 3-4):
-//                      each CTA streams a few pages (K and V slices of 16 KB at
-//                      d = 128, bulk async copies into a 3-stage ring), keeps an
-//                      online softmax per head, and the last CTA of a group merges
-//                      the partial (max, sum, output) triples.
+//                      each CTA streams one or a few pages (K and V slices of 16 KB
+//                      at d = 128, bulk async copies into a ring), keeps an online
+//                      softmax per head, and the last CTA of a group merges the
+//                      partial (max, sum, output) triples.
+// The three kernels are chained with programmatic dependent launch: each one
+// starts while its predecessor runs, does the work that needs none of the
+// predecessor's results (barrier set-up, reading lengths and queries, the page
+// of the current block) and then waits on the grid dependency.
 // A decode step moves bytes, not flops (a few FMAs per cached element), so the
 // arithmetic runs on CUDA cores with packed fp32x2 FMAs; there is no tensor-core
 // contraction on this path.
@@ -31,7 +37,7 @@ constexpr int kBlk = 64;
 constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
 constexpr int kPrepThreads = 256;
 constexpr int kScoreThreads = 256;
-constexpr int kAttnThreads = 128;
+constexpr int kAttnThreads = 256;
 constexpr int kStages = 3;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -50,6 +56,11 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 __device__ __forceinline__ bool bad_len(int n, const DecodeArgs& a) { return n < 1 || n > a.max_blocks * kBlk; }
+
+// Programmatic dependent launch: wait until the preceding grid has completed
+// and its writes are visible; allow the next grid to start launching.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // Exclusive prefix sum over the 256 threads of a CTA (scan: 16 shared ints).
 __device__ int block_excl_scan(int v, int* scan) {
@@ -118,11 +129,12 @@ __device__ void summarize_block(const bf16* Kt, const bf16* Wk, bf16* out, int d
     }
 }
 
-// grid (B*Hkv, 1 + d_sel/32): y = 0 appends the token and updates the summary
-// cache, y >= 1 computes 32 entries of the group's gate query.
+// grid (B*Hkv, 1 + d_sel/8): y = 0 appends the token and updates the summary
+// cache, y >= 1 computes 8 entries of the group's gate query (one per warp).
 __global__ void __launch_bounds__(kPrepThreads) dec_prep_kernel(DecodeArgs a, int* status) {
     __shared__ float red[512];
     __shared__ __align__(16) float vec[1024];
+    grid_dep_launch();   // the score kernel may start its set-up
     const int bh = blockIdx.x;
     const int b = bh / a.Hkv, g = bh - b * a.Hkv;
     const int n = __ldg(a.seq_lens + b);
@@ -165,34 +177,42 @@ __global__ void __launch_bounds__(kPrepThreads) dec_prep_kernel(DecodeArgs a, in
         }
         return;
     }
-    // gate query q~[o] = bf16(sum_e Wq_g[o][e] q_cat[e]) for o in [32 (y-1), 32 y)
+    // gate query q~[o] = bf16(sum_e Wq_g[o][e] q_cat[e]), o = 8 (y-1) + warp.  The
+    // warp's row of Wq_g (G*d <= 1024 bf16) is loaded in one go, 32 bytes a lane.
     const int GD = a.G * a.d;
+    const int warp = t >> 5, lane = t & 31;
+    const int o = (blockIdx.y - 1) * 8 + warp;
+    const bool has_row = o < a.d_sel;
+    const bf16* wrow = static_cast<const bf16*>(a.Wq) + (static_cast<size_t>(g) * a.d_sel + (has_row ? o : 0)) * GD;
+    uint4 w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int e = (k * 32 + lane) * 8;
+        w[k] = (has_row && e < GD) ? __ldg(reinterpret_cast<const uint4*>(wrow + e)) : make_uint4(0, 0, 0, 0);
+    }
     const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * a.G) * a.d;
     for (int e = t; e < GD; e += kPrepThreads) vec[e] = __bfloat162float(qg[e]);
     __syncthreads();
-    const int warp = t >> 5, lane = t & 31;
-    const int o0 = (blockIdx.y - 1) * 32;
-    for (int oo = warp; oo < 32; oo += kPrepThreads / 32) {
-        const int o = o0 + oo;
-        if (o >= a.d_sel) break;
-        const bf16* wrow = static_cast<const bf16*>(a.Wq) + (static_cast<size_t>(g) * a.d_sel + o) * GD;
-        float acc = 0.f;
-        for (int e = lane * 8; e < GD; e += 256) {
-            const uint4 w = __ldg(reinterpret_cast<const uint4*>(wrow + e));
+    if (!has_row) return;
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int e = (k * 32 + lane) * 8;
+        if (e < GD) {
             const float4 x0 = *reinterpret_cast<const float4*>(vec + e);
             const float4 x1 = *reinterpret_cast<const float4*>(vec + e + 4);
-            acc = fmaf(bf_lo(w.x), x0.x, acc);
-            acc = fmaf(bf_hi(w.x), x0.y, acc);
-            acc = fmaf(bf_lo(w.y), x0.z, acc);
-            acc = fmaf(bf_hi(w.y), x0.w, acc);
-            acc = fmaf(bf_lo(w.z), x1.x, acc);
-            acc = fmaf(bf_hi(w.z), x1.y, acc);
-            acc = fmaf(bf_lo(w.w), x1.z, acc);
-            acc = fmaf(bf_hi(w.w), x1.w, acc);
+            acc = fmaf(bf_lo(w[k].x), x0.x, acc);
+            acc = fmaf(bf_hi(w[k].x), x0.y, acc);
+            acc = fmaf(bf_lo(w[k].y), x0.z, acc);
+            acc = fmaf(bf_hi(w[k].y), x0.w, acc);
+            acc = fmaf(bf_lo(w[k].z), x1.x, acc);
+            acc = fmaf(bf_hi(w[k].z), x1.y, acc);
+            acc = fmaf(bf_lo(w[k].w), x1.z, acc);
+            acc = fmaf(bf_hi(w[k].w), x1.w, acc);
         }
-        acc = warp_sum(acc);
-        if (lane == 0) static_cast<bf16*>(a.qt)[static_cast<size_t>(bh) * a.d_sel + o] = __float2bfloat16_rn(acc);
     }
+    acc = warp_sum(acc);
+    if (lane == 0) static_cast<bf16*>(a.qt)[static_cast<size_t>(bh) * a.d_sel + o] = __float2bfloat16_rn(acc);
 }
 
 // grid (max_blocks, B*Hkv): summary of full block m of every sequence (after a prefill).
@@ -221,53 +241,67 @@ __global__ void __launch_bounds__(kPrepThreads) dec_summarize_kernel(DecodeArgs 
 // ------------------------------------------------------------ scores + Top-K
 
 struct ScoreSmem {
-    size_t r0;   // staging rows / selection keys
-    size_t qs, bars, misc, hist, scan, total;
+    size_t r0;   // staged summary rows; in the last CTA the candidates (keys, blocks)
+    size_t qs, bars, misc, xchg, hist, scan, total;
 };
-__host__ __device__ inline ScoreSmem score_smem_layout(int max_blocks, int d_sel) {
+__host__ __device__ inline ScoreSmem score_smem_layout(int nsplit, int topk, int d_sel) {
     ScoreSmem L;
-    size_t slab = static_cast<size_t>(8) * 32 * d_sel * 2;
-    size_t keys = static_cast<size_t>(max_blocks) * 4;
-    L.r0 = ((slab > keys ? slab : keys) + 127) / 128 * 128;
+    const size_t slab = static_cast<size_t>(8) * 32 * d_sel * 2;
+    const size_t cand = static_cast<size_t>(nsplit) * (topk > 0 ? topk : 1) * 8;
+    L.r0 = ((slab > cand ? slab : cand) + 127) / 128 * 128;
     L.qs = L.r0;                  // d_sel bf16 (<= 256 bytes)
     L.bars = L.qs + 256;          // 8 mbarriers
-    L.misc = L.bars + 64;         // flag + radix broadcast (4 ints)
-    L.hist = L.misc + 64;         // 4096 ints
+    L.misc = L.bars + 64;         // flag, radix broadcast, per-warp counts (16 ints)
+    L.xchg = L.misc + 64;         // 256 64-bit sort keys
+    L.hist = L.xchg + 256 * 8;    // 4096 ints
     L.scan = L.hist + 4096 * 4;   // 16 ints
     L.total = L.scan + 128;
     return L;
 }
 
 // Order-preserving map of a finite float to uint32 (larger float, larger key);
-// -0 is mapped like +0 so that equal scores stay ties.
+// -0 is mapped like +0 so that equal scores stay ties.  Every finite float maps
+// above 0, so 0 marks an empty candidate slot.
 __device__ __forceinline__ uint32_t order_key(float f) {
     const uint32_t u = __float_as_uint(f == 0.f ? 0.f : f);
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exact Top-K of the group's C scores (K < C), ties to the lower block:
-// radix select of the K-th largest key tau in digits of 12, 10 and 10 bits,
-// then every key > tau plus the lowest-indexed keys == tau, emitted in
-// ascending block order.  256 threads of the last CTA of the group.
-__device__ void select_group(const DecodeArgs& a, int bh, int C, uint32_t* keys, int* hist, int* scan, int* bc) {
+// Descending bitonic sort of 256 distinct 64-bit keys, one per thread of the
+// CTA; returns the key that ends at position threadIdx.x.  Exchanges within a
+// warp use shuffles, wider ones the 256-entry shared buffer xchg.
+__device__ uint64_t bitonic256_desc(uint64_t c, uint64_t* xchg) {
+    const int t = threadIdx.x;
+#pragma unroll
+    for (int k = 2; k <= 256; k <<= 1) {
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            uint64_t o;
+            if (j >= 32) {
+                xchg[t] = c;
+                __syncthreads();
+                o = xchg[t ^ j];
+                __syncthreads();
+            } else {
+                o = __shfl_xor_sync(0xffffffffu, c, j);
+            }
+            const bool keep_max = ((t & j) == 0) == ((t & k) == 0);
+            c = keep_max ? (c > o ? c : o) : (c < o ? c : o);
+        }
+    }
+    return c;
+}
+
+// Exact Top-K of M candidates (keys[i], block idx[i]) listed in ascending block
+// order, ties to the lower block: radix select of the K-th largest key tau in
+// digits of 12, 10 and 10 bits, then every key > tau plus the first keys == tau,
+// emitted in list order.  256 threads; K < number of non-empty candidates.
+__device__ void select_candidates(const DecodeArgs& a, int bh, int M, const uint32_t* keys, const int32_t* idx,
+                                  int* hist, int* scan, int* bc) {
     const int K = a.topk;
     const int t = threadIdx.x, lane = t & 31;
     int32_t* lst = a.list + static_cast<size_t>(bh) * 64;
     int32_t* so = a.sel_idx ? a.sel_idx + static_cast<size_t>(bh) * K : nullptr;
-    if (C <= K) {
-        for (int e = t; e < K; e += kScoreThreads) {
-            if (e < C) lst[e] = e;
-            if (so) so[e] = e < C ? e : -1;
-        }
-        if (t == 0) a.list_n[bh] = C;
-        return;
-    }
-    if (K == 0) {
-        if (t == 0) a.list_n[bh] = 0;
-        return;
-    }
-    const float* sc = a.scores + static_cast<size_t>(bh) * a.max_blocks;
-    for (int i = t; i < C; i += kScoreThreads) keys[i] = order_key(__ldcg(sc + i));
     uint32_t prefix = 0, mask = 0;
     int r = K;
 #pragma unroll 1
@@ -277,11 +311,11 @@ __device__ void select_group(const DecodeArgs& a, int bh, int C, uint32_t* keys,
         const int nb = 1 << width;
         for (int i = t; i < nb; i += kScoreThreads) hist[i] = 0;
         __syncthreads();
-        for (int base = 0; base < C; base += kScoreThreads) {
+        for (int base = 0; base < M; base += kScoreThreads) {
             const int i = base + t;
             bool in = false;
             int bin = 0;
-            if (i < C) {
+            if (i < M) {
                 const uint32_t k = keys[i];
                 in = (k & mask) == prefix;
                 bin = static_cast<int>((k >> sh) & static_cast<uint32_t>(nb - 1));
@@ -313,10 +347,10 @@ __device__ void select_group(const DecodeArgs& a, int bh, int C, uint32_t* keys,
         mask |= static_cast<uint32_t>(nb - 1) << sh;
         r = bc[1];
     }
-    const uint32_t tau = prefix;   // the K-th largest key; take r of the keys equal to it
-    // ascending emission: contiguous index ranges of odd length per thread (conflict-free reads)
-    const int per = ((C + kScoreThreads - 1) / kScoreThreads) | 1;
-    const int lo = min(t * per, C), hi = min(lo + per, C);
+    const uint32_t tau = prefix;   // the K-th largest key; take the first r keys equal to it
+    // list-order emission: contiguous ranges of odd length per thread (conflict-free reads)
+    const int per = ((M + kScoreThreads - 1) / kScoreThreads) | 1;
+    const int lo = min(t * per, M), hi = min(lo + per, M);
     int eq = 0;
     for (int i = lo; i < hi; ++i) eq += keys[i] == tau;
     const int eq_base = block_excl_scan(eq, scan);
@@ -340,39 +374,46 @@ __device__ void select_group(const DecodeArgs& a, int bh, int C, uint32_t* keys,
             ++er;
         }
         if (take) {
-            lst[pos] = i;
-            if (so) so[pos] = i;
+            lst[pos] = idx[i];
+            if (so) so[pos] = idx[i];
             ++pos;
         }
     }
     if (t == 0) a.list_n[bh] = K;
 }
 
-// grid (nsplit_s, B*Hkv)
+// grid (nsplit_s, B*Hkv), launched as a programmatic dependent of the prep kernel.
 template <int DSEL>
 __global__ void __launch_bounds__(kScoreThreads) dec_score_kernel(DecodeArgs a, int* status, long long limit,
                                                                   float score_scale) {
     extern __shared__ __align__(128) uint8_t smem[];
     constexpr int kRowBytes = DSEL * 2;
     constexpr int kSlab = 32 * kRowBytes;
-    const ScoreSmem L = score_smem_layout(a.max_blocks, DSEL);
+    const ScoreSmem L = score_smem_layout(a.nsplit_s, a.topk, DSEL);
     uint8_t* stage = smem;
     uint4* qs = reinterpret_cast<uint4*>(smem + L.qs);
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bars);
     int* misc = reinterpret_cast<int*>(smem + L.misc);
+    uint64_t* xchg = reinterpret_cast<uint64_t*>(smem + L.xchg);
     const int bh = blockIdx.y;
     const int b = bh / a.Hkv;
-    const int n = __ldg(a.seq_lens + b);
-    if (bad_len(n, a)) return;   // recorded by the prep kernel
-    const int C = (n - 1) / kBlk;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int m0 = blockIdx.x * kDecScoreChunk;
     if (t == 0) {
         for (int w = 0; w < 8; ++w) mbar_init(&bars[w], 1);
         fence_barrier_init();
     }
+    const int n = __ldg(a.seq_lens + b);
+    grid_dep_wait();     // q~ and the summary of a block closed by this step
+    grid_dep_launch();   // the attention kernel may start its set-up
+    if (bad_len(n, a)) return;   // recorded by the prep kernel
+    const int C = (n - 1) / kBlk;
+    const int K = a.topk;
+    const int Kc = K > 0 ? K : 1;
+    const int m0 = blockIdx.x * kDecScoreChunk;
+    const int rows_cta = max(0, min(kDecScoreChunk, C - m0));
     __syncthreads();
-    if (m0 < C) {
+    uint32_t key = 0;
+    if (rows_cta > 0 && K > 0 && C > K) {
         if (t < DSEL / 8) qs[t] = __ldg(reinterpret_cast<const uint4*>(a.qt) + static_cast<size_t>(bh) * (DSEL / 8) + t);
         const int r0 = m0 + warp * 32;
         const int rows = max(0, min(32, C - r0));
@@ -401,8 +442,47 @@ __global__ void __launch_bounds__(kScoreThreads) dec_score_kernel(DecodeArgs a, 
                 }
                 float s0, s1;
                 f32x2_split(acc, s0, s1);
-                a.scores[static_cast<size_t>(bh) * a.max_blocks + r0 + lane] = (s0 + s1) * score_scale;
+                key = order_key((s0 + s1) * score_scale);
             }
+        }
+        // local Top-K of this CTA's blocks: sort the distinct keys (score key, then
+        // the lower block first) and keep those at or above the K-th
+        bool take = t < rows_cta && key != 0;
+        if (rows_cta > K) {
+            const uint64_t comp = (static_cast<uint64_t>(key) << 32) | (0xffffffffu - static_cast<uint32_t>(t));
+            const uint64_t sorted = bitonic256_desc(comp, xchg);
+            __syncthreads();
+            if (t == K - 1) xchg[0] = sorted;
+            __syncthreads();
+            take = take && comp >= xchg[0];
+        }
+        // compact the kept blocks in block order into this CTA's K candidate slots
+        const unsigned bal = __ballot_sync(0xffffffffu, take);
+        if (lane == 0) misc[8 + warp] = __popc(bal);
+        __syncthreads();
+        int off = 0, total = 0;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            const int c = misc[8 + w];
+            off += w < warp ? c : 0;
+            total += c;
+        }
+        const size_t cbase = (static_cast<size_t>(bh) * a.nsplit_s + blockIdx.x) * Kc;
+        if (take) {
+            const int pos = off + __popc(bal & ((1u << lane) - 1u));
+            a.cand_key[cbase + pos] = key;
+            a.cand_idx[cbase + pos] = m0 + t;
+        }
+        for (int e = total + t; e < Kc; e += kScoreThreads) {
+            a.cand_key[cbase + e] = 0;
+            a.cand_idx[cbase + e] = -1;
+        }
+    } else if (K > 0 && C > K) {
+        // no blocks in this CTA's range: empty candidate slots
+        const size_t cbase = (static_cast<size_t>(bh) * a.nsplit_s + blockIdx.x) * Kc;
+        for (int e = t; e < Kc; e += kScoreThreads) {
+            a.cand_key[cbase + e] = 0;
+            a.cand_idx[cbase + e] = -1;
         }
     }
     // the last CTA of the group to finish selects
@@ -416,88 +496,91 @@ __global__ void __launch_bounds__(kScoreThreads) dec_score_kernel(DecodeArgs a, 
     if (!misc[0]) return;
     __threadfence();
     if (t == 0) a.cnt_sel[bh] = 0;   // zero again for the next launch
-    select_group(a, bh, C, reinterpret_cast<uint32_t*>(stage), reinterpret_cast<int*>(smem + L.hist),
-                 reinterpret_cast<int*>(smem + L.scan), misc + 1);
+    int32_t* lst = a.list + static_cast<size_t>(bh) * 64;
+    int32_t* so = a.sel_idx ? a.sel_idx + static_cast<size_t>(bh) * K : nullptr;
+    if (C <= K) {   // short history: every historical block is kept
+        for (int e = t; e < K; e += kScoreThreads) {
+            if (e < C) lst[e] = e;
+            if (so) so[e] = e < C ? e : -1;
+        }
+        if (t == 0) a.list_n[bh] = C;
+        return;
+    }
+    if (K == 0) {
+        if (t == 0) a.list_n[bh] = 0;
+        return;
+    }
+    const int M = a.nsplit_s * Kc;
+    uint32_t* ckeys = reinterpret_cast<uint32_t*>(stage);
+    int32_t* cidx = reinterpret_cast<int32_t*>(stage) + M;
+    const size_t gbase = static_cast<size_t>(bh) * M;
+    for (int i = t; i < M; i += kScoreThreads) {
+        ckeys[i] = __ldcg(a.cand_key + gbase + i);
+        cidx[i] = __ldcg(a.cand_idx + gbase + i);
+    }
+    select_candidates(a, bh, M, ckeys, cidx, reinterpret_cast<int*>(smem + L.hist),
+                      reinterpret_cast<int*>(smem + L.scan), misc + 1);
 }
 
 // ---------------------------------------------------------------- attention
 
-template <int D, int G>
-struct AttnSmem {
-    static constexpr int kTile = kBlk * D * 2;                 // one K or V page slice
-    static constexpr int RING = 0;
-    static constexpr int Q32 = kStages * 2 * kTile;            // fp32 queries [G][D]
-    static constexpr int PS = Q32 + G * D * 4;                 // probabilities [G][64]
-    static constexpr int RED = PS + G * 64 * 4;                // [4 warps][8]
-    static constexpr int ALPHA = RED + 32 * 4;                 // [8]
-    static constexpr int LSUM = ALPHA + 8 * 4;                 // [4 warps][8]
-    static constexpr int BARS = LSUM + 32 * 4;                 // kStages mbarriers
-    static constexpr int MISC = BARS + 64;                     // flag
-    static constexpr int ENT = MISC + 64;                      // entries: block, page (2 ints each)
+// Shared-memory layout of the attention kernel for a ring of nst stages.
+struct AttnLayout {
+    size_t tile, q32, ps, red, alpha, lsum, bars, misc, ent, total;
 };
-
-__host__ __device__ inline size_t attn_smem_bytes(int D, int G, int bpc) {
-    const size_t tile = static_cast<size_t>(kBlk) * D * 2;
-    return kStages * 2 * tile + static_cast<size_t>(G) * D * 4 + static_cast<size_t>(G) * 64 * 4 + (32 + 8 + 32) * 4 +
-           64 + 64 + static_cast<size_t>(bpc) * 8;
+__host__ __device__ inline AttnLayout attn_layout(int D, int G, int nst, int bpc) {
+    AttnLayout L;
+    L.tile = static_cast<size_t>(kBlk) * D * 2;     // one K or V page slice
+    L.q32 = nst * 2 * L.tile;                        // fp32 queries [G][D]
+    L.ps = L.q32 + static_cast<size_t>(G) * D * 4;   // probabilities [G][64]
+    L.red = L.ps + static_cast<size_t>(G) * 64 * 4;  // [8 warps][8]
+    L.alpha = L.red + 64 * 4;                        // [8], then merge max [8] and sum [8]
+    L.lsum = L.alpha + 32 * 4;                       // [8 warps][8]
+    L.bars = L.lsum + 64 * 4;                        // nst mbarriers
+    L.misc = L.bars + 64;                            // flag
+    L.ent = L.misc + 64;                             // entries: block, page (2 ints each)
+    L.total = L.ent + static_cast<size_t>(bpc) * 8;
+    return L;
 }
 
-// grid (nsplit_a, B*Hkv).  The group's list: the kept blocks (ascending) and then
-// the current block c; this CTA takes entries [x*bpc, (x+1)*bpc).
+// grid (nsplit_a, B*Hkv), a programmatic dependent of the score kernel (of the
+// prep kernel in dense mode).  The group's list is the current block c first,
+// then the kept blocks in ascending order (dense: blocks 0 .. c-1); this CTA
+// takes entries [x*bpc, (x+1)*bpc).
 template <int D, int G>
 __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, int* status, long long limit,
                                                                 float scale_log2) {
-    using S = AttnSmem<D, G>;
-    constexpr int kTile = S::kTile;
     constexpr int kNW = D / 2;                          // bf16 pairs per row
-    constexpr int HP = (G + 1) / 2;                     // heads per thread in the score step
+    constexpr int NQG = kAttnThreads / 64;              // head groups in the score step
+    constexpr int HP = (G + NQG - 1) / NQG;             // heads per thread in the score step
     constexpr int NHG = kAttnThreads / kNW;             // head groups in the PV step
     constexpr int HPV = (G + NHG - 1) / NHG;            // heads per thread in the PV step
     constexpr int NCH = D / 8;                          // 16-byte chunks per row
     extern __shared__ __align__(128) uint8_t smem[];
-    float* q32 = reinterpret_cast<float*>(smem + S::Q32);
-    float* Ps = reinterpret_cast<float*>(smem + S::PS);
-    float* red = reinterpret_cast<float*>(smem + S::RED);
-    float* alpha_s = reinterpret_cast<float*>(smem + S::ALPHA);
-    float* lsum = reinterpret_cast<float*>(smem + S::LSUM);
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::BARS);
-    int* misc = reinterpret_cast<int*>(smem + S::MISC);
-    int* ent = reinterpret_cast<int*>(smem + S::ENT);
+    const int nst = a.nst;
+    const AttnLayout Ly = attn_layout(D, G, nst, a.bpc);
+    const int kTile = static_cast<int>(Ly.tile);
+    float* q32 = reinterpret_cast<float*>(smem + Ly.q32);
+    float* Ps = reinterpret_cast<float*>(smem + Ly.ps);
+    float* red = reinterpret_cast<float*>(smem + Ly.red);
+    float* alpha_s = reinterpret_cast<float*>(smem + Ly.alpha);
+    float* lsum = reinterpret_cast<float*>(smem + Ly.lsum);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + Ly.bars);
+    int* misc = reinterpret_cast<int*>(smem + Ly.misc);
+    int* ent = reinterpret_cast<int*>(smem + Ly.ent);
 
     const int bh = blockIdx.y;
     const int b = bh / a.Hkv, g = bh - b * a.Hkv;
-    const int n = __ldg(a.seq_lens + b);
-    if (bad_len(n, a)) return;   // recorded by the prep kernel
-    const int c = (n - 1) / kBlk;
-    const int L = (a.dense ? c : __ldg(a.list_n + bh)) + 1;
-    const int j0 = blockIdx.x * a.bpc;
-    const int cnt = max(0, min(j0 + a.bpc, L) - j0);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-
-    for (int jj = t; jj < cnt; jj += kAttnThreads) {
-        const int j = j0 + jj;
-        const int blk = j == L - 1 ? c : (a.dense ? j : __ldg(a.list + static_cast<size_t>(bh) * 64 + j));
-        int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + blk);
-        if (page < 0 || page >= a.num_pages) {
-            atomicExch(status, kStatusBadInput);
-            page = -1;
-        }
-        ent[2 * jj] = blk;
-        ent[2 * jj + 1] = page;
-    }
-    const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G) * D;
-    for (int e = t; e < G * D; e += kAttnThreads) q32[e] = __bfloat162float(qg[e]);
-    if (t == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
-        fence_barrier_init();
-    }
-    __syncthreads();
-
+    const int n = __ldg(a.seq_lens + b);
+    const bool bad = bad_len(n, a);   // recorded by the prep kernel
+    const int c = bad ? 0 : (n - 1) / kBlk;
+    const int j0 = blockIdx.x * a.bpc;
     const size_t head_off = static_cast<size_t>(g) * kBlk * D;   // this KV head's slice inside a page
     auto issue = [&](int jj) {
-        const int s = jj % kStages;
+        const int s = jj % nst;
         const int page = ent[2 * jj + 1];
-        uint8_t* dst = smem + S::RING + s * 2 * kTile;
+        uint8_t* dst = smem + s * 2 * kTile;
         if (page < 0) {
             mbar_arrive(&full[s]);
             return;
@@ -507,12 +590,47 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
         bulk_load(dst, static_cast<const bf16*>(a.K_cache) + off, kTile, &full[s]);
         bulk_load(dst + kTile, static_cast<const bf16*>(a.V_cache) + off, kTile, &full[s]);
     };
-    int issued = 0;
+
+    // --- set-up that needs nothing from the preceding kernel
     if (t == 0) {
-        for (; issued < min(cnt, kStages); ++issued) issue(issued);
+        for (int s = 0; s < nst; ++s) mbar_init(&full[s], 1);
+        fence_barrier_init();
+        // the current block (entry 0) was appended by the prep kernel, which the
+        // score kernel has waited for before letting this grid start: its page
+        // can load now (in dense mode the prep kernel precedes this one directly)
+        if (!bad && j0 == 0 && !a.dense) {
+            int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + c);
+            if (page < 0 || page >= a.num_pages) page = -1;   // recorded by the prep kernel
+            ent[0] = c;
+            ent[1] = page;
+            issue(0);
+        }
+    }
+    const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G) * D;
+    for (int e = t; e < G * D; e += kAttnThreads) q32[e] = __bfloat162float(qg[e]);
+    grid_dep_wait();   // the kept list
+    if (bad) return;
+    const int L = (a.dense ? c : __ldg(a.list_n + bh)) + 1;
+    const int cnt = max(0, min(j0 + a.bpc, L) - j0);
+    const int first = (j0 == 0 && !a.dense) ? 1 : 0;   // entries set up before the wait
+    for (int jj = first + t; jj < cnt; jj += kAttnThreads) {
+        const int j = j0 + jj;
+        const int blk = j == 0 ? c : (a.dense ? j - 1 : __ldg(a.list + static_cast<size_t>(bh) * 64 + j - 1));
+        int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + blk);
+        if (page < 0 || page >= a.num_pages) {
+            atomicExch(status, kStatusBadInput);
+            page = -1;
+        }
+        ent[2 * jj] = blk;
+        ent[2 * jj + 1] = page;
+    }
+    __syncthreads();
+    int issued = first;
+    if (t == 0) {
+        for (; issued < min(cnt, nst); ++issued) issue(issued);
     }
 
-    const int k = t & 63, hh = t >> 6;           // score step: key k, heads hh*HP + u
+    const int k = t & 63, hh = t >> 6;           // score step: key k, heads hh*HP + u (keys of a head in warps 2hh, 2hh+1)
     const int wi = t % kNW, hg = t / kNW;        // PV step: column pair wi, heads hg*HPV + u
     float m_run[HP], l_part[HP];
 #pragma unroll
@@ -527,15 +645,15 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     bool ok = true;
     int jj = 0;
     for (; jj < cnt; ++jj) {
-        const int s = jj % kStages;
-        const bool got = mbar_wait_drain(&full[s], (jj / kStages) & 1, limit, status);
+        const int s = jj % nst;
+        const bool got = mbar_wait_drain(&full[s], (jj / nst) & 1, limit, status);
         if (!__syncthreads_and(got)) {
             ok = false;
             break;
         }
         const int page = ent[2 * jj + 1];
         const int nvalid = page < 0 ? 0 : (ent[2 * jj] == c ? n - c * kBlk : kBlk);
-        const uint8_t* Kt = smem + S::RING + s * 2 * kTile;
+        const uint8_t* Kt = smem + s * 2 * kTile;
         const uint8_t* Vt = Kt + kTile;
 
         // z = scale * q_h . k for this thread's key and heads (log2 units)
@@ -627,7 +745,7 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     if (!ok) {
         // let copies still in flight land before the CTA exits; report nothing
         if (t == 0)
-            for (int q = jj; q < issued; ++q) mbar_wait_drain(&full[q % kStages], (q / kStages) & 1, limit, status);
+            for (int q = jj; q < issued; ++q) mbar_wait_drain(&full[q % nst], (q / nst) & 1, limit, status);
 #pragma unroll
         for (int u = 0; u < HP; ++u) {
             m_run[u] = -CUDART_INF_F;
@@ -676,37 +794,78 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     __threadfence();
     if (t == 0) a.cnt_attn[bh] = 0;   // zero again for the next launch
 
-    // merge the nsplit_a partials of every head
+    // Merge the partials of every head (only the splits the list reached).  The
+    // (max, sum) pairs are staged in the free ring first, turned into weights
+    // exp2(m_x - M) per head, then every thread sums its columns over the splits
+    // with all loads independent.
+    const int used = (L + a.bpc - 1) / a.bpc;
     const float* pg = a.part + static_cast<size_t>(bh) * a.nsplit_a * G * (D + 2);
+    float* mw = reinterpret_cast<float*>(smem);    // [used][G][2]
+    float* mM = alpha_s + 8;                       // [G] max
+    float* mL = alpha_s + 16;                      // [G] sum
+    for (int i = t; i < used * G; i += kAttnThreads) {
+        const float* px = pg + static_cast<size_t>(i) * (D + 2);
+        mw[2 * i] = __ldcg(px);
+        mw[2 * i + 1] = __ldcg(px + 1);
+    }
+    __syncthreads();
+    if (t < G) {
+        float M = -CUDART_INF_F;
+        for (int x = 0; x < used; ++x) M = fmaxf(M, mw[2 * (x * G + t)]);
+        float ls = 0.f;
+        for (int x = 0; x < used; ++x) {
+            const float mx = mw[2 * (x * G + t)];
+            const float w = mx == -CUDART_INF_F ? 0.f : fast_exp2(mx - M);
+            ls = fmaf(w, mw[2 * (x * G + t) + 1], ls);
+            mw[2 * (x * G + t)] = w;
+        }
+        mM[t] = M;
+        mL[t] = ls;
+    }
+    __syncthreads();
 #pragma unroll
     for (int u = 0; u < HPV; ++u) {
         const int h = hg * HPV + u;
         if (h >= G) continue;
-        float M = -CUDART_INF_F;
-        for (int x = 0; x < a.nsplit_a; ++x) M = fmaxf(M, __ldcg(pg + (static_cast<size_t>(x) * G + h) * (D + 2)));
-        float lsum_all = 0.f, o0 = 0.f, o1 = 0.f;
-        for (int x = 0; x < a.nsplit_a; ++x) {
-            const float* px = pg + (static_cast<size_t>(x) * G + h) * (D + 2);
-            const float mx = __ldcg(px);
-            if (mx == -CUDART_INF_F) continue;
-            const float w = fast_exp2(mx - M);
-            lsum_all = fmaf(w, __ldcg(px + 1), lsum_all);
-            o0 = fmaf(w, __ldcg(px + 2 + 2 * wi), o0);
-            o1 = fmaf(w, __ldcg(px + 3 + 2 * wi), o1);
+        float o0 = 0.f, o1 = 0.f;
+#pragma unroll 16
+        for (int x = 0; x < used; ++x) {
+            const float2 v = __ldcg(reinterpret_cast<const float2*>(pg + (static_cast<size_t>(x) * G + h) * (D + 2) + 2) + wi);
+            const float w = mw[2 * (x * G + h)];
+            o0 = fmaf(w, v.x, o0);
+            o1 = fmaf(w, v.y, o1);
         }
-        const float inv = 1.f / lsum_all;
+        const float inv = 1.f / mL[h];
         const size_t orow = (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h) * D;
         reinterpret_cast<uint32_t*>(static_cast<bf16*>(a.O) + orow)[wi] = pack_bf16x2(o0 * inv, o1 * inv);
         if (a.LSE != nullptr && wi == 0)
-            a.LSE[static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h] = (M + log2f(lsum_all)) / kLog2e;
+            a.LSE[static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h] = (mM[h] + log2f(mL[h])) / kLog2e;
     }
+}
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the preceding kernel on the stream still runs (it waits with griddepcontrol).
+template <class... KArgs, class... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                             Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 // Raises the kernel's dynamic shared-memory limit to what these arguments need
 // (called when a handle is created, so that a captured step sets nothing).
 template <int D, int G>
 cudaError_t prepare_attn_dg(const DecodeArgs& a) {
-    const size_t smem = attn_smem_bytes(D, G, a.bpc);
+    const size_t smem = attn_layout(D, G, a.nst, a.bpc).total;
     static size_t set = 0;
     if (smem > set) {
         cudaError_t e = cudaFuncSetAttribute(dec_attn_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -719,13 +878,12 @@ cudaError_t prepare_attn_dg(const DecodeArgs& a) {
 
 template <int D, int G>
 cudaError_t launch_attn_dg(const DecodeArgs& a, const KernelEnv& env) {
-    const size_t smem = attn_smem_bytes(D, G, a.bpc);
+    const size_t smem = attn_layout(D, G, a.nst, a.bpc).total;
     cudaError_t e = prepare_attn_dg<D, G>(a);
     if (e != cudaSuccess) return e;
     dim3 grid(a.nsplit_a, a.B * a.Hkv);
-    dec_attn_kernel<D, G><<<grid, kAttnThreads, smem, env.stream>>>(a, env.status, env.limit,
-                                                                     a.sm_scale * kLog2e);
-    return cudaGetLastError();
+    return launch_dependent(dec_attn_kernel<D, G>, grid, dim3(kAttnThreads), smem, env.stream, a, env.status,
+                            env.limit, a.sm_scale * kLog2e);
 }
 
 template <int D>
@@ -752,7 +910,7 @@ cudaError_t prepare_attn_d(const DecodeArgs& a) {
 
 template <int DSEL>
 cudaError_t prepare_score_d(const DecodeArgs& a) {
-    const size_t smem = score_smem_layout(a.max_blocks, DSEL).total;
+    const size_t smem = score_smem_layout(a.nsplit_s, a.topk, DSEL).total;
     static size_t set = 0;
     if (smem > set) {
         cudaError_t e = cudaFuncSetAttribute(dec_score_kernel<DSEL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -765,26 +923,28 @@ cudaError_t prepare_score_d(const DecodeArgs& a) {
 
 template <int DSEL>
 cudaError_t launch_score_d(const DecodeArgs& a, const KernelEnv& env) {
-    const size_t smem = score_smem_layout(a.max_blocks, DSEL).total;
+    const size_t smem = score_smem_layout(a.nsplit_s, a.topk, DSEL).total;
     cudaError_t e = prepare_score_d<DSEL>(a);
     if (e != cudaSuccess) return e;
     dim3 grid(a.nsplit_s, a.B * a.Hkv);
-    dec_score_kernel<DSEL><<<grid, kScoreThreads, smem, env.stream>>>(a, env.status, env.limit,
-                                                                     static_cast<float>(1.0 / sqrt(static_cast<double>(DSEL))));
-    return cudaGetLastError();
+    return launch_dependent(dec_score_kernel<DSEL>, grid, dim3(kScoreThreads), smem, env.stream, a, env.status,
+                            env.limit, static_cast<float>(1.0 / sqrt(static_cast<double>(DSEL))));
 }
 
 }  // namespace
 
-void decode_attn_split(int max_len, int* nsplit, int* bpc) {
-    const int per = max_len <= 96 ? 2 : (max_len + 63) / 64;
+void decode_attn_split(int max_len, int* nsplit, int* bpc, int* nst) {
+    // one page per CTA for a SAS list (at most K + 1 pages); long dense lists
+    // are cut into at most 64 pieces streamed through a 3-stage ring
+    const int per = max_len <= 96 ? 1 : (max_len + 63) / 64;
     *bpc = per;
     *nsplit = (max_len + per - 1) / per;
+    *nst = per < kStages ? per : kStages;
 }
 
-size_t decode_score_smem(int max_blocks, int d_sel) { return score_smem_layout(max_blocks, d_sel).total; }
+size_t decode_score_smem(int nsplit, int topk, int d_sel) { return score_smem_layout(nsplit, topk, d_sel).total; }
 
-size_t decode_attn_smem(int d, int G, int bpc) { return attn_smem_bytes(d, G, bpc); }
+size_t decode_attn_smem(int d, int G, int nst, int bpc) { return attn_layout(d, G, nst, bpc).total; }
 
 cudaError_t decode_prepare(const DecodeArgs& a) {
     cudaError_t e = cudaSuccess;
@@ -794,7 +954,7 @@ cudaError_t decode_prepare(const DecodeArgs& a) {
 }
 
 cudaError_t launch_decode_prep(const DecodeArgs& a, const KernelEnv& env) {
-    dim3 grid(a.B * a.Hkv, a.dense ? 1 : 1 + (a.d_sel + 31) / 32);
+    dim3 grid(a.B * a.Hkv, a.dense ? 1 : 1 + (a.d_sel + 7) / 8);
     dec_prep_kernel<<<grid, kPrepThreads, 0, env.stream>>>(a, env.status);
     return cudaGetLastError();
 }

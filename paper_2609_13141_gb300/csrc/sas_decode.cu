@@ -23,10 +23,11 @@ struct sas_decode_handle {
     sas_decode_config cfg;
     int G = 1, d_sel = 0;
     float sm_scale = 0.f;
-    int nsplit_s = 0, nsplit_a = 0, bpc = 0;
+    int nsplit_s = 0, nsplit_a = 0, bpc = 0, nst = 0;
     // workspace
     void* qt = nullptr;
-    float* scores = nullptr;
+    uint32_t* cand_key = nullptr;
+    int32_t* cand_idx = nullptr;
     int32_t* list = nullptr;
     int32_t* list_n = nullptr;
     float* part = nullptr;
@@ -74,20 +75,24 @@ cudaEvent_t dnext_event(sas_decode_handle* h) {
     return h->events[h->events_used++];
 }
 
+// Brackets one launch with events when timing is on.  The events are recorded
+// as external event nodes when the stream is being captured, so a replayed
+// graph re-records them and sas_decode_get_timings reads the latest replay.
 template <class Fn>
 cudaError_t dtimed(sas_decode_handle* h, int kind, cudaStream_t s, Fn&& fn) {
     cudaEvent_t a = nullptr, b = nullptr;
+    unsigned flags = cudaEventRecordDefault;
     if (h->timing) {
         a = dnext_event(h);
         b = dnext_event(h);
-        if (a) cudaEventRecord(a, s);
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(s, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+            flags = cudaEventRecordExternal;
+        if (a && cudaEventRecordWithFlags(a, s, flags) != cudaSuccess) a = nullptr;
     }
     cudaError_t e = fn();
     if (e == cudaSuccess) ++h->launches;
-    if (h->timing && a && b) {
-        cudaEventRecord(b, s);
-        h->recs.push_back({kind, a, b});
-    }
+    if (h->timing && a && b && cudaEventRecordWithFlags(b, s, flags) == cudaSuccess) h->recs.push_back({kind, a, b});
     return e;
 }
 
@@ -96,10 +101,10 @@ sas::DecodeArgs base_args(const sas_decode_handle* h) {
     sas::DecodeArgs a{};
     a.B = c.B; a.Hq = c.Hq; a.Hkv = c.Hkv; a.G = h->G; a.d = c.d; a.d_sel = h->d_sel; a.topk = c.topk;
     a.max_blocks = c.max_blocks; a.num_pages = c.num_pages; a.dense = c.dense; a.sm_scale = h->sm_scale;
-    a.qt = h->qt; a.scores = h->scores; a.list = h->list; a.list_n = h->list_n; a.part = h->part;
+    a.qt = h->qt; a.cand_key = h->cand_key; a.cand_idx = h->cand_idx; a.list = h->list; a.list_n = h->list_n; a.part = h->part;
     a.cnt_sel = h->counters;
     a.cnt_attn = h->counters + static_cast<size_t>(c.B) * c.Hkv;
-    a.nsplit_s = h->nsplit_s; a.nsplit_a = h->nsplit_a; a.bpc = h->bpc;
+    a.nsplit_s = h->nsplit_s; a.nsplit_a = h->nsplit_a; a.bpc = h->bpc; a.nst = h->nst;
     return a;
 }
 
@@ -133,7 +138,7 @@ sas_status sas_decode_create(const sas_decode_config* cfg, sas_decode_handle** o
     h->d_sel = d_sel;
     h->sm_scale = c.sm_scale > 0.f ? c.sm_scale : 1.0f / std::sqrt(static_cast<float>(c.d));
     h->nsplit_s = (c.max_blocks + sas::kDecScoreChunk - 1) / sas::kDecScoreChunk;
-    sas::decode_attn_split(c.dense ? c.max_blocks : c.topk + 1, &h->nsplit_a, &h->bpc);
+    sas::decode_attn_split(c.dense ? c.max_blocks : c.topk + 1, &h->nsplit_a, &h->bpc, &h->nst);
 
     int dev = 0, major = 0, minor = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -148,7 +153,9 @@ sas_status sas_decode_create(const sas_decode_config* cfg, sas_decode_handle** o
         return SAS_ERR_UNSUPPORTED;
     }
     if (e == cudaSuccess) e = dalloc(&h->qt, static_cast<size_t>(BH) * d_sel * 2);
-    if (e == cudaSuccess) e = dalloc(&h->scores, static_cast<size_t>(BH) * c.max_blocks * 4);
+    const size_t ncand = static_cast<size_t>(BH) * h->nsplit_s * (c.topk > 0 ? c.topk : 1);
+    if (e == cudaSuccess) e = dalloc(&h->cand_key, ncand * 4);
+    if (e == cudaSuccess) e = dalloc(&h->cand_idx, ncand * 4);
     if (e == cudaSuccess) e = dalloc(&h->list, static_cast<size_t>(BH) * 64 * 4);
     if (e == cudaSuccess) e = dalloc(&h->list_n, static_cast<size_t>(BH) * 4);
     if (e == cudaSuccess) e = dalloc(&h->part, static_cast<size_t>(BH) * h->nsplit_a * G * (c.d + 2) * 4);
@@ -171,7 +178,8 @@ void sas_decode_destroy(sas_decode_handle* h) {
     if (h == nullptr) return;
     cudaDeviceSynchronize();
     cudaFree(h->qt);
-    cudaFree(h->scores);
+    cudaFree(h->cand_key);
+    cudaFree(h->cand_idx);
     cudaFree(h->list);
     cudaFree(h->list_n);
     cudaFree(h->part);
@@ -256,8 +264,10 @@ sas_status sas_decode_set_timing(sas_decode_handle* h, int32_t enable) {
     if (h == nullptr) return SAS_ERR_INVALID_ARG;
     cudaDeviceSynchronize();
     h->timing = enable != 0;
-    h->recs.clear();
-    h->events_used = 0;
+    if (h->timing) {   // a new recording starts; stopping keeps the records
+        h->recs.clear();
+        h->events_used = 0;
+    }
     return SAS_OK;
 }
 
