@@ -454,9 +454,12 @@ def decode_bytes(B, Hq, Hkv, d, ds, K, n, dense):
     groups = B * Hkv
     kv_tokens = (C if dense else min(K, C)) * 64 + cur
     attn = groups * (2 * 2 * kv_tokens * d + 2 * G * d * 2)           # K, V pages; q in, O out
-    prep = groups * (4 * 2 * d + (0 if dense else 2 * ds * G * d + 2 * G * d))   # append; Wq and q
-    score = 0 if dense else groups * (2 * C * ds + 2 * ds)          # summaries and q~
-    return {"prep": prep, "score_topk": score, "attention": attn, "total": prep + score + attn}
+    prep = groups * 4 * 2 * d                                         # k_new, v_new read and written
+    if dense:
+        return {"prep": prep, "attention": attn, "total": prep + attn}
+    prep += groups * (2 * ds * G * d + 2 * G * d)                    # Wq and q for the gate query
+    select = groups * (2 * C * ds + 2 * ds)                          # the summaries and q~
+    return {"prep": prep, "select": select, "attention": attn, "total": prep + select + attn}
 
 
 def decode_oracle_us(B, Hq, Hkv, d, ds, K, n, budget_s, seed=0):

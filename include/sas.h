@@ -299,7 +299,8 @@ sas_status sas_decode_summarize(sas_decode_handle* h, const void* K_cache, const
  *   LSE      fp32 [B, Hq] natural-log log-sum-exp of the logits, or NULL
  *   sel_idx  int32 [B, Hkv, topk] kept blocks, -1 padded, or NULL
  * In dense mode Wq, Wk and Ksum are not used (may be NULL) and sel_idx must be
- * NULL.  Three kernel launches (two in dense mode); no allocation, no
+ * NULL.  Three kernel launches, one per step above (two in dense mode), each
+ * started early by programmatic dependent launch; no allocation, no
  * synchronisation, so the call can be captured in a CUDA graph. */
 sas_status sas_decode_step(sas_decode_handle* h, const void* q, const void* k_new, const void* v_new,
                            void* K_cache, void* V_cache, const int32_t* block_table, const int32_t* seq_lens,

@@ -117,7 +117,7 @@ struct DecodeArgs {
 };
 constexpr int kDecScoreChunk = 256;
 // Attention split for a group list of at most max_len entries.
-void decode_attn_split(int max_len, int* nsplit, int* bpc, int* nst);
+void decode_attn_split(int max_len, int d, int* nsplit, int* bpc, int* nst);
 // Dynamic shared memory the score and attention kernels need.
 size_t decode_score_smem(int nsplit, int topk, int d_sel);
 size_t decode_attn_smem(int d, int G, int nst, int bpc);

@@ -510,10 +510,20 @@ __global__ void __launch_bounds__(kScoreThreads) dec_score_kernel(DecodeArgs a, 
         if (t == 0) a.list_n[bh] = 0;
         return;
     }
-    const int M = a.nsplit_s * Kc;
+    const size_t gbase = static_cast<size_t>(bh) * a.nsplit_s * Kc;
+    if (C <= kDecScoreChunk) {
+        // one CTA held every block: its local Top-K is the group's, already in block order
+        for (int e = t; e < K; e += kScoreThreads) {
+            const int m = __ldcg(a.cand_idx + gbase + e);
+            lst[e] = m;
+            if (so) so[e] = m;
+        }
+        if (t == 0) a.list_n[bh] = K;
+        return;
+    }
+    const int M = ((C + kDecScoreChunk - 1) / kDecScoreChunk) * Kc;   // the splits that held blocks
     uint32_t* ckeys = reinterpret_cast<uint32_t*>(stage);
     int32_t* cidx = reinterpret_cast<int32_t*>(stage) + M;
-    const size_t gbase = static_cast<size_t>(bh) * M;
     for (int i = t; i < M; i += kScoreThreads) {
         ckeys[i] = __ldcg(a.cand_key + gbase + i);
         cidx[i] = __ldcg(a.cand_idx + gbase + i);
@@ -595,16 +605,6 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     if (t == 0) {
         for (int s = 0; s < nst; ++s) mbar_init(&full[s], 1);
         fence_barrier_init();
-        // the current block (entry 0) was appended by the prep kernel, which the
-        // score kernel has waited for before letting this grid start: its page
-        // can load now (in dense mode the prep kernel precedes this one directly)
-        if (!bad && j0 == 0 && !a.dense) {
-            int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + c);
-            if (page < 0 || page >= a.num_pages) page = -1;   // recorded by the prep kernel
-            ent[0] = c;
-            ent[1] = page;
-            issue(0);
-        }
     }
     const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G) * D;
     for (int e = t; e < G * D; e += kAttnThreads) q32[e] = __bfloat162float(qg[e]);
@@ -612,7 +612,9 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     if (bad) return;
     const int L = (a.dense ? c : __ldg(a.list_n + bh)) + 1;
     const int cnt = max(0, min(j0 + a.bpc, L) - j0);
-    const int first = (j0 == 0 && !a.dense) ? 1 : 0;   // entries set up before the wait
+    // (the current block, entry 0, is written by the preceding kernel, so every
+    // page load waits for the grid dependency)
+    const int first = 0;
     for (int jj = first + t; jj < cnt; jj += kAttnThreads) {
         const int j = j0 + jj;
         const int blk = j == 0 ? c : (a.dense ? j - 1 : __ldg(a.list + static_cast<size_t>(bh) * 64 + j - 1));
@@ -843,6 +845,364 @@ __global__ void __launch_bounds__(kAttnThreads) dec_attn_kernel(DecodeArgs a, in
     }
 }
 
+// -------------------------------------------------- attention on tensor cores (d = 128)
+//
+// A step takes two pages (128 keys) of the CTA's list:
+//   S^T[128 keys][16] = Kpair[128 x 128] . Qpad[16 x 128]^T          tcgen05, M=128 N=16, K-major A and B
+//   softmax over the 128 keys of every head (TMEM lane = key)
+//   O^T[128 d][16]    = Vpair^T[128 d x 128 keys] . Ppad[16 x 128]^T  tcgen05, A MN-major (V as stored)
+// Q and P are padded from G <= 8 heads to N = 16 rows of zeros.  K and V tiles
+// sit in shared memory as [d half][128 keys][128 B] with the 128-byte swizzle,
+// written by four 64 x 64 TMA boxes each (page 0 in rows 0-63, page 1 in
+// rows 64-127); Q is [d half][16][128 B], P [key half][16][128 B], both
+// swizzled by the threads that write them.  Every step's O^T is a fresh
+// accumulator that the threads fold into registers (thread t owns row d = t)
+// with the online-softmax rescale.
+
+constexpr int kTcThreads = 128;
+constexpr int kTcTile = 2 * 128 * 128;          // bytes of one K (or V) tile of a step
+constexpr int kTcStage = 2 * kTcTile;           // K and V
+constexpr uint32_t kTcTmemCols = 64;            // S^T in columns 0-15, O^T in 32-47
+
+struct TcLayout {
+    size_t q, p, red, alpha, lsum, bars, misc, ent, total;
+};
+__host__ __device__ inline TcLayout tc_layout(int nst, int bpc) {
+    TcLayout L;
+    L.q = static_cast<size_t>(nst) * kTcStage;   // 4096: [2][16][128 B]
+    L.p = L.q + 4096;                            // 4096: [2][16][128 B]
+    L.red = L.p + 4096;                          // [4 warps][16]
+    L.alpha = L.red + 64 * 4;                    // [16] alpha, then merge max [16] and sum [16]
+    L.lsum = L.alpha + 48 * 4;                   // [4 warps][16]
+    L.bars = L.lsum + 64 * 4;                    // full[4], qk, pv
+    L.misc = L.bars + 64;                        // flag, TMEM base
+    L.ent = L.misc + 64;                         // entries: block, page
+    L.total = L.ent + static_cast<size_t>(bpc) * 8 + 1024;   // + alignment slack
+    return L;
+}
+
+// TMA loads of list entry e (a page of step e/2) into the step's stage: K and V,
+// two 64 x 64 boxes each (the two halves of d); nothing for a missing page.
+__device__ __forceinline__ void tc_load_page(uint8_t* smem, int nst, const int* ent, int e, const CUtensorMap* mapK,
+                                             const CUtensorMap* mapV, uint64_t* full, int Hkv, int g) {
+    const int page = ent[2 * e + 1];
+    if (page < 0) return;
+    const int s = (e >> 1) % nst, pg = e & 1;
+    uint8_t* st = smem + static_cast<size_t>(s) * kTcStage;
+    const int row = page * Hkv + g;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        tma_load_3d(st + h * 16384 + pg * 8192, mapK, &full[s], h * 64, 0, row);
+        tma_load_3d(st + kTcTile + h * 16384 + pg * 8192, mapV, &full[s], h * 64, 0, row);
+    }
+}
+__device__ __forceinline__ uint32_t tc_page_bytes(const int* ent, int e) {
+    return ent[2 * e + 1] >= 0 ? 4u * 8192u : 0u;
+}
+
+template <int G>
+__global__ void __launch_bounds__(kTcThreads) dec_attn_tc_kernel(const __grid_constant__ CUtensorMap mapK,
+                                                                 const __grid_constant__ CUtensorMap mapV,
+                                                                 DecodeArgs a, int* status, long long limit,
+                                                                 float scale_log2) {
+    constexpr int D = 128;
+    constexpr uint32_t IDESC_S = idesc_bf16(128, 16, 0, 0);
+    constexpr uint32_t IDESC_O = idesc_bf16(128, 16, 1, 0);
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    // the swizzled tiles need 1024-byte alignment
+    uint8_t* smem = dsm + ((1024u - (smem_u32(dsm) & 1023u)) & 1023u);
+    const int nst = a.nst;
+    const TcLayout Ly = tc_layout(nst, a.bpc);
+    uint8_t* qs = smem + Ly.q;
+    uint8_t* ps = smem + Ly.p;
+    float* red = reinterpret_cast<float*>(smem + Ly.red);
+    float* mM = reinterpret_cast<float*>(smem + Ly.alpha) + 16;
+    float* mL = reinterpret_cast<float*>(smem + Ly.alpha) + 32;
+    float* lsum = reinterpret_cast<float*>(smem + Ly.lsum);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + Ly.bars);
+    uint64_t* qk_bar = full + 4;
+    uint64_t* pv_bar = full + 5;
+    int* misc = reinterpret_cast<int*>(smem + Ly.misc);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 4);
+    int* ent = reinterpret_cast<int*>(smem + Ly.ent);
+
+    const int bh = blockIdx.y;
+    const int b = bh / a.Hkv, g = bh - b * a.Hkv;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int n = __ldg(a.seq_lens + b);
+    const bool bad = bad_len(n, a);   // recorded by the prep kernel
+    const int c = bad ? 0 : (n - 1) / kBlk;
+    const int j0 = blockIdx.x * a.bpc;
+
+#define SAS_TC_LOAD(e) tc_load_page(smem, nst, ent, (e), &mapK, &mapV, full, a.Hkv, g)
+
+    // --- set-up that needs nothing from the preceding kernel
+    if (t == 0) {
+        for (int s = 0; s < nst; ++s) mbar_init(&full[s], 1);
+        mbar_init(qk_bar, 1);
+        mbar_init(pv_bar, 1);
+        fence_barrier_init();
+        tma_prefetch_desc(&mapK);
+        tma_prefetch_desc(&mapV);
+        // the current block (entry 0) was appended by the prep kernel, which the
+        // score kernel waited for before letting this grid start, so its page can
+        // load now (dense mode: the prep kernel precedes this one directly)
+        if (!bad && j0 == 0 && !a.dense) {
+            int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + c);
+            if (page < 0 || page >= a.num_pages) page = -1;   // recorded by the prep kernel
+            ent[0] = c;
+            ent[1] = page;
+            mbar_expect_tx(&full[0], tc_page_bytes(ent, 0));
+            SAS_TC_LOAD(0);
+        }
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_slot, kTcTmemCols);
+        tmem_relinquish();
+    }
+    // Q rows (zero past G) and P (rows past G stay zero), 16-byte chunks swizzled
+    const bf16* qg = static_cast<const bf16*>(a.q) + (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G) * D;
+    for (int i = t; i < 2 * 16 * 8; i += kTcThreads) {
+        const int h = i >> 7, row = (i >> 3) & 15, ch = i & 7;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (row < G) v = __ldg(reinterpret_cast<const uint4*>(qg + row * D + h * 64 + ch * 8));
+        *reinterpret_cast<uint4*>(qs + h * 2048 + row * 128 + ((ch ^ (row & 7)) << 4)) = v;
+        *reinterpret_cast<uint4*>(ps + h * 2048 + row * 128 + (ch << 4)) = make_uint4(0, 0, 0, 0);
+    }
+    grid_dep_wait();   // the kept list
+    const int L = bad ? 0 : (a.dense ? c : __ldg(a.list_n + bh)) + 1;
+    const int cnt = bad ? 0 : max(0, min(j0 + a.bpc, L) - j0);
+    const int first = (j0 == 0 && !a.dense) ? 1 : 0;   // entries set up before the wait
+    for (int jj = first + t; jj < cnt; jj += kTcThreads) {
+        const int j = j0 + jj;
+        const int blk = j == 0 ? c : (a.dense ? j - 1 : __ldg(a.list + static_cast<size_t>(bh) * 64 + j - 1));
+        int page = __ldg(a.block_table + static_cast<size_t>(b) * a.max_blocks + blk);
+        if (page < 0 || page >= a.num_pages) {
+            atomicExch(status, kStatusBadInput);
+            page = -1;
+        }
+        ent[2 * jj] = blk;
+        ent[2 * jj + 1] = page;
+    }
+    fence_proxy_async_smem();   // Q and P writes before the tensor cores read them
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int steps = (cnt + 1) >> 1;
+    int issued = 0;   // steps whose loads are issued (thread 0)
+    if (t == 0) {
+        for (; issued < min(steps, nst); ++issued) {
+            const int e0 = 2 * issued, e1 = e0 + 1;
+            uint32_t bytes = 0;
+            if (e0 >= first) bytes += tc_page_bytes(ent, e0);
+            if (e1 < cnt) bytes += tc_page_bytes(ent, e1);
+            mbar_arrive_expect_tx(&full[issued], bytes);
+            if (e0 >= first) SAS_TC_LOAD(e0);
+            if (e1 < cnt) SAS_TC_LOAD(e1);
+        }
+    }
+
+    float m_run[G], l_part[G], o[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+        m_run[h] = -CUDART_INF_F;
+        l_part[h] = 0.f;
+        o[h] = 0.f;
+    }
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    bool ok = true;
+    int j = 0;
+    int pending = 0;   // 1: a QK commit outstanding, 2: a PV commit outstanding
+    for (; j < steps; ++j) {
+        const int s = j % nst;
+        uint8_t* st = smem + static_cast<size_t>(s) * kTcStage;
+        const bool got = mbar_wait_drain(&full[s], (j / nst) & 1, limit, status);
+        if (!__syncthreads_and(got)) {
+            ok = false;
+            break;
+        }
+        // rows of a page past its valid keys (or of a missing page) get zero values,
+        // so P = 0 there cannot meet a non-finite V
+        const int e0 = 2 * j, e1 = e0 + 1;
+        const int nv0 = ent[2 * e0 + 1] < 0 ? 0 : (ent[2 * e0] == c ? n - c * kBlk : kBlk);
+        const int nv1 = (e1 >= cnt || ent[2 * e1 + 1] < 0) ? 0 : (ent[2 * e1] == c ? n - c * kBlk : kBlk);
+        if (nv0 < kBlk || nv1 < kBlk) {
+            for (int i = t; i < 2 * 2 * 64 * 8; i += kTcThreads) {   // (page, half, row, chunk)
+                const int pg = i >> 10, h = (i >> 9) & 1, row = (i >> 3) & 63, ch = i & 7;
+                if (row >= (pg ? nv1 : nv0))
+                    *reinterpret_cast<uint4*>(st + kTcTile + h * 16384 + pg * 8192 + row * 128 + (ch << 4)) =
+                        make_uint4(0, 0, 0, 0);
+            }
+            fence_proxy_async_smem();
+            __syncthreads();
+        }
+        if (t == 0) {
+            tc_fence_after();
+            const uint32_t kb = smem_u32(st), qb = smem_u32(qs);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+                const uint64_t da = smem_desc_sw128(kb + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024);
+                const uint64_t db = smem_desc_sw128(qb + (k >> 2) * 2048 + (k & 3) * 32, 16, 1024);
+                umma_bf16(tmem, da, db, IDESC_S, k > 0);
+            }
+            umma_commit(qk_bar);
+        }
+        pending = 1;
+        if (!mbar_wait_drain(qk_bar, j & 1, limit, status)) ok = false;
+        if (!__syncthreads_and(ok)) break;
+        pending = 0;
+        tc_fence_after();
+        uint32_t sr[16];
+        tmem_ld16(lane_base, sr);
+        tmem_wait_ld();
+        const int key = t;                           // TMEM lane = key of the pair
+        const bool valid = key < 64 ? key < nv0 : key - 64 < nv1;
+        float z[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            z[h] = valid ? __uint_as_float(sr[h]) * scale_log2 : -CUDART_INF_F;
+            const float mx = warp_max(z[h]);
+            if (lane == 0) red[warp * 16 + h] = mx;
+        }
+        __syncthreads();
+        float alpha[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            const float mb = fmaxf(fmaxf(red[h], red[16 + h]), fmaxf(red[32 + h], red[48 + h]));
+            const float m_new = fmaxf(m_run[h], mb);
+            alpha[h] = m_run[h] == -CUDART_INF_F ? 0.f : fast_exp2(m_run[h] - m_new);
+            const float pr = z[h] == -CUDART_INF_F ? 0.f : fast_exp2(z[h] - m_new);
+            l_part[h] = l_part[h] * alpha[h] + pr;
+            m_run[h] = m_new;
+            const int kh = key >> 6, ch = (key & 63) >> 3;
+            *reinterpret_cast<bf16*>(ps + kh * 2048 + h * 128 + ((ch ^ (h & 7)) << 4) + ((key & 7) << 1)) =
+                __float2bfloat16_rn(pr);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (t == 0) {
+            tc_fence_after();
+            const uint32_t vb = smem_u32(st + kTcTile), pb = smem_u32(ps);
+#pragma unroll
+            for (int k = 0; k < 128 / 16; ++k) {
+                const uint64_t da = smem_desc_sw128(vb + k * 2048, 16384, 1024);
+                const uint64_t db = smem_desc_sw128(pb + (k >> 2) * 2048 + (k & 3) * 32, 16, 1024);
+                umma_bf16(tmem + 32, da, db, IDESC_O, k > 0);
+            }
+            umma_commit(pv_bar);
+        }
+        pending = 2;
+        if (!mbar_wait_drain(pv_bar, j & 1, limit, status)) ok = false;
+        if (!__syncthreads_and(ok)) break;
+        pending = 0;
+        tc_fence_after();
+        uint32_t orr[16];
+        tmem_ld16(lane_base + 32, orr);
+        tmem_wait_ld();
+#pragma unroll
+        for (int h = 0; h < G; ++h) o[h] = fmaf(o[h], alpha[h], __uint_as_float(orr[h]));
+        tc_fence_before();
+        __syncthreads();   // the stage, P and the TMEM columns are free
+        if (t == 0 && issued < steps) {
+            const int e0 = 2 * issued, e1 = e0 + 1;
+            const int s2 = issued % nst;
+            uint32_t bytes = tc_page_bytes(ent, e0);
+            if (e1 < cnt) bytes += tc_page_bytes(ent, e1);
+            mbar_arrive_expect_tx(&full[s2], bytes);
+            SAS_TC_LOAD(e0);
+            if (e1 < cnt) SAS_TC_LOAD(e1);
+            ++issued;
+        }
+    }
+    if (!ok) {
+        // let the tensor cores and the copies in flight finish before leaving
+        if (t == 0) {
+            if (pending == 1) mbar_wait_drain(qk_bar, j & 1, limit, status);
+            if (pending == 2) mbar_wait_drain(pv_bar, j & 1, limit, status);
+            for (int q = j; q < issued; ++q) mbar_wait_drain(&full[q % nst], (q / nst) & 1, limit, status);
+        }
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            m_run[h] = -CUDART_INF_F;
+            l_part[h] = 0.f;
+            o[h] = 0.f;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTcTmemCols);
+    }
+
+    // partial (max, sum, output) of this CTA per head
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+        const float ls = warp_sum(l_part[h]);
+        if (lane == 0) lsum[warp * 16 + h] = ls;
+    }
+    __syncthreads();
+    float* part = a.part + (static_cast<size_t>(bh) * a.nsplit_a + blockIdx.x) * G * (D + 2);
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+        if (t == 0) {
+            part[h * (D + 2)] = m_run[h];
+            part[h * (D + 2) + 1] = lsum[h] + lsum[16 + h] + lsum[32 + h] + lsum[48 + h];
+        }
+        part[h * (D + 2) + 2 + t] = o[h];
+    }
+    __threadfence();
+    __syncthreads();
+    if (t == 0) {
+        const int old = atomicAdd(a.cnt_attn + bh, 1);
+        misc[0] = old == static_cast<int>(gridDim.x) - 1;
+    }
+    __syncthreads();
+    if (!misc[0]) return;
+    __threadfence();
+    if (t == 0) a.cnt_attn[bh] = 0;   // zero again for the next launch
+    if (bad) return;
+
+    // merge the partials of the splits the list reached
+    const int used = (L + a.bpc - 1) / a.bpc;
+    const float* pgp = a.part + static_cast<size_t>(bh) * a.nsplit_a * G * (D + 2);
+    float* mw = reinterpret_cast<float*>(smem);    // [used][G][2], in the free stage
+    for (int i = t; i < used * G; i += kTcThreads) {
+        const float* px = pgp + static_cast<size_t>(i) * (D + 2);
+        mw[2 * i] = __ldcg(px);
+        mw[2 * i + 1] = __ldcg(px + 1);
+    }
+    __syncthreads();
+    if (t < G) {
+        float M = -CUDART_INF_F;
+        for (int x = 0; x < used; ++x) M = fmaxf(M, mw[2 * (x * G + t)]);
+        float ls = 0.f;
+        for (int x = 0; x < used; ++x) {
+            const float mx = mw[2 * (x * G + t)];
+            const float w = mx == -CUDART_INF_F ? 0.f : fast_exp2(mx - M);
+            ls = fmaf(w, mw[2 * (x * G + t) + 1], ls);
+            mw[2 * (x * G + t)] = w;
+        }
+        mM[t] = M;
+        mL[t] = ls;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+        float acc = 0.f;
+#pragma unroll 8
+        for (int x = 0; x < used; ++x)
+            acc = fmaf(mw[2 * (x * G + h)], __ldcg(pgp + (static_cast<size_t>(x) * G + h) * (D + 2) + 2 + t), acc);
+        const size_t orow = (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h) * D;
+        static_cast<bf16*>(a.O)[orow + t] = __float2bfloat16_rn(acc / mL[h]);
+        if (a.LSE != nullptr && t == 0)
+            a.LSE[static_cast<size_t>(b) * a.Hq + static_cast<size_t>(g) * G + h] = (mM[h] + log2f(mL[h])) / kLog2e;
+    }
+#undef SAS_TC_LOAD
+}
+
 // Launch with programmatic stream serialization: the kernel may start while
 // the preceding kernel on the stream still runs (it waits with griddepcontrol).
 template <class... KArgs, class... Args>
@@ -886,24 +1246,68 @@ cudaError_t launch_attn_dg(const DecodeArgs& a, const KernelEnv& env) {
                             env.limit, a.sm_scale * kLog2e);
 }
 
+template <int G>
+cudaError_t prepare_attn_tc(const DecodeArgs& a) {
+    const size_t smem = tc_layout(a.nst, a.bpc).total;
+    static size_t set = 0;
+    if (smem > set) {
+        cudaError_t e = cudaFuncSetAttribute(dec_attn_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        set = smem;
+    }
+    return cudaSuccess;
+}
+
+template <int G>
+cudaError_t launch_attn_tc(const DecodeArgs& a, const KernelEnv& env) {
+    cudaError_t e = prepare_attn_tc<G>(a);
+    if (e != cudaSuccess) return e;
+    CUtensorMap mk, mv;
+    const uint64_t rows = static_cast<uint64_t>(a.num_pages) * a.Hkv;
+    if (make_tmap_bf16_3d(&mk, a.K_cache, 128, kBlk, rows, 64, kBlk) != 0) return cudaErrorInvalidValue;
+    if (make_tmap_bf16_3d(&mv, a.V_cache, 128, kBlk, rows, 64, kBlk) != 0) return cudaErrorInvalidValue;
+    dim3 grid(a.nsplit_a, a.B * a.Hkv);
+    return launch_dependent(dec_attn_tc_kernel<G>, grid, dim3(kTcThreads), tc_layout(a.nst, a.bpc).total, env.stream,
+                            mk, mv, a, env.status, env.limit, a.sm_scale * kLog2e);
+}
+
 template <int D>
 cudaError_t launch_attn_d(const DecodeArgs& a, const KernelEnv& env) {
-    switch (a.G) {
-        case 1: return launch_attn_dg<D, 1>(a, env);
-        case 2: return launch_attn_dg<D, 2>(a, env);
-        case 4: return launch_attn_dg<D, 4>(a, env);
-        case 8: return launch_attn_dg<D, 8>(a, env);
+    if constexpr (D == 128) {
+        switch (a.G) {
+            case 1: return launch_attn_tc<1>(a, env);
+            case 2: return launch_attn_tc<2>(a, env);
+            case 4: return launch_attn_tc<4>(a, env);
+            case 8: return launch_attn_tc<8>(a, env);
+        }
+    } else {
+        switch (a.G) {
+            case 1: return launch_attn_dg<D, 1>(a, env);
+            case 2: return launch_attn_dg<D, 2>(a, env);
+            case 4: return launch_attn_dg<D, 4>(a, env);
+            case 8: return launch_attn_dg<D, 8>(a, env);
+        }
     }
     return cudaErrorInvalidValue;
 }
 
 template <int D>
 cudaError_t prepare_attn_d(const DecodeArgs& a) {
-    switch (a.G) {
-        case 1: return prepare_attn_dg<D, 1>(a);
-        case 2: return prepare_attn_dg<D, 2>(a);
-        case 4: return prepare_attn_dg<D, 4>(a);
-        case 8: return prepare_attn_dg<D, 8>(a);
+    if constexpr (D == 128) {
+        switch (a.G) {
+            case 1: return prepare_attn_tc<1>(a);
+            case 2: return prepare_attn_tc<2>(a);
+            case 4: return prepare_attn_tc<4>(a);
+            case 8: return prepare_attn_tc<8>(a);
+        }
+    } else {
+        switch (a.G) {
+            case 1: return prepare_attn_dg<D, 1>(a);
+            case 2: return prepare_attn_dg<D, 2>(a);
+            case 4: return prepare_attn_dg<D, 4>(a);
+            case 8: return prepare_attn_dg<D, 8>(a);
+        }
     }
     return cudaErrorInvalidValue;
 }
@@ -933,18 +1337,29 @@ cudaError_t launch_score_d(const DecodeArgs& a, const KernelEnv& env) {
 
 }  // namespace
 
-void decode_attn_split(int max_len, int* nsplit, int* bpc, int* nst) {
-    // one page per CTA for a SAS list (at most K + 1 pages); long dense lists
-    // are cut into at most 64 pieces streamed through a 3-stage ring
-    const int per = max_len <= 96 ? 1 : (max_len + 63) / 64;
+void decode_attn_split(int max_len, int d, int* nsplit, int* bpc, int* nst) {
+    int per;
+    if (d == 128) {
+        // tensor-core kernel: two pages (one 128-key step) per CTA for a SAS list,
+        // long dense lists cut into at most 64 pieces of whole steps; one stage,
+        // so that three CTAs share an SM and overlap one another's loads
+        per = max_len <= 96 ? 2 : 2 * ((max_len + 127) / 128);
+        *nst = 1;
+    } else {
+        // CUDA-core kernel: one page per CTA for a SAS list; long dense lists in
+        // at most 64 pieces streamed through a 3-stage ring
+        per = max_len <= 96 ? 1 : (max_len + 63) / 64;
+        *nst = per < kStages ? per : kStages;
+    }
     *bpc = per;
     *nsplit = (max_len + per - 1) / per;
-    *nst = per < kStages ? per : kStages;
 }
 
 size_t decode_score_smem(int nsplit, int topk, int d_sel) { return score_smem_layout(nsplit, topk, d_sel).total; }
 
-size_t decode_attn_smem(int d, int G, int nst, int bpc) { return attn_layout(d, G, nst, bpc).total; }
+size_t decode_attn_smem(int d, int G, int nst, int bpc) {
+    return d == 128 ? tc_layout(nst, bpc).total : attn_layout(d, G, nst, bpc).total;
+}
 
 cudaError_t decode_prepare(const DecodeArgs& a) {
     cudaError_t e = cudaSuccess;

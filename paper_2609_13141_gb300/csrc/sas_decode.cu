@@ -138,7 +138,7 @@ sas_status sas_decode_create(const sas_decode_config* cfg, sas_decode_handle** o
     h->d_sel = d_sel;
     h->sm_scale = c.sm_scale > 0.f ? c.sm_scale : 1.0f / std::sqrt(static_cast<float>(c.d));
     h->nsplit_s = (c.max_blocks + sas::kDecScoreChunk - 1) / sas::kDecScoreChunk;
-    sas::decode_attn_split(c.dense ? c.max_blocks : c.topk + 1, &h->nsplit_a, &h->bpc, &h->nst);
+    sas::decode_attn_split(c.dense ? c.max_blocks : c.topk + 1, c.d, &h->nsplit_a, &h->bpc, &h->nst);
 
     int dev = 0, major = 0, minor = 0;
     cudaError_t e = cudaGetDevice(&dev);

@@ -53,7 +53,7 @@ class SasDecodeConfig(ctypes.Structure):
 
 
 SAS_DECODE_NUM_KERNEL_KINDS = 4
-DECODE_KERNEL_KINDS = ["prep", "score_topk", "attention", "summarize"]
+DECODE_KERNEL_KINDS = ["prep", "select", "attention", "summarize"]
 
 
 class SasError(RuntimeError):

@@ -136,7 +136,7 @@ def test_exact_inputs_bit_exact_selection_and_summaries():
     # n = 1 (first token), 65 and 129 (the new token opens a block: the step itself
     # summarises the block it closes), 1000 (ragged current block)
     r = run_case(4, 32, 8, 128, 128, 4, [1, 65, 129, 1000], seed=1, exact=True)
-    assert r["launches"] == 4   # summary fill + prep, scores/Top-K, attention
+    assert r["launches"] == 4   # summary fill, then the step: prep, selection, attention
 
 
 def test_random_inputs_qwen_shape_budget_2048():
