@@ -598,8 +598,14 @@ def run_decode(args, rank, world):
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.2)
-    us, e2e_us, kern, launches, h2d, d2h, spread = measure(False)
-    dus, de2e_us, dkern, _, _, _, dspread = measure(True)
+    if args.decode_only == "dense":
+        us, e2e_us, kern, launches, h2d, d2h, spread = measure(True)
+    else:
+        us, e2e_us, kern, launches, h2d, d2h, spread = measure(False)
+    if args.decode_only is None:
+        dus, de2e_us, dkern, _, _, _, dspread = measure(True)
+    else:   # one arm only (profiling runs): the other arm's fields repeat it
+        dus, de2e_us, dkern, dspread = us, e2e_us, kern, spread
     clocks = sampler.stop()
     us, e2e_us, dus = reduce_max([us, e2e_us, dus], dist, dev)
     if rank != 0:
@@ -607,8 +613,8 @@ def run_decode(args, rank, world):
             dist.destroy_process_group()
         return None
     peaks = load_peaks()
-    by = decode_bytes(B, Hq, Hkv, d, ds, K, n, False)
-    dby = decode_bytes(B, Hq, Hkv, d, ds, K, n, True)
+    by = decode_bytes(B, Hq, Hkv, d, ds, K, n, args.decode_only == "dense")
+    dby = decode_bytes(B, Hq, Hkv, d, ds, K, n, True) if args.decode_only is None else by
 
     def roof(kern_us, bytes_):
         dom = max(kern_us, key=kern_us.get)
@@ -681,6 +687,8 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["decode"], default="dit")
     ap.add_argument("--context", type=int, default=65536, help="decode: cached tokens per sequence")
     ap.add_argument("--batch", type=int, default=1, help="decode: sequences per step")
+    ap.add_argument("--decode-only", choices=["sparse", "dense"], default=None,
+                    help="decode: run one arm only (for profiling)")
     ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
                     help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
     ap.add_argument("--topk", type=int, default=None, help="override the workload's K")

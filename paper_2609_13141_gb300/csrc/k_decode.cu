@@ -1340,10 +1340,12 @@ cudaError_t launch_score_d(const DecodeArgs& a, const KernelEnv& env) {
 void decode_attn_split(int max_len, int d, int* nsplit, int* bpc, int* nst) {
     int per;
     if (d == 128) {
-        // tensor-core kernel: two pages (one 128-key step) per CTA for a SAS list,
-        // long dense lists cut into at most 64 pieces of whole steps; one stage,
-        // so that three CTAs share an SM and overlap one another's loads
-        per = max_len <= 96 ? 2 : 2 * ((max_len + 127) / 128);
+        // tensor-core kernel: two pages (one 128-key step) per CTA for a SAS list;
+        // long dense lists cut into at most 64 (128 past 2048 pages) pieces of
+        // whole steps.  One stage, so that three CTAs share an SM and overlap one
+        // another's loads (two stages and one CTA per SM measured slower).
+        const int pieces = max_len <= 2048 ? 64 : 128;   // long lists: more CTAs pay for the larger merge
+        per = max_len <= 96 ? 2 : 2 * ((max_len + 2 * pieces - 1) / (2 * pieces));
         *nst = 1;
     } else {
         // CUDA-core kernel: one page per CTA for a SAS list; long dense lists in
