@@ -1,0 +1,92 @@
+"""Plain fp64 CPU oracle for the backward pass of the SAS training forward.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import, call or
+execute this module: only the tests, the smoke check and the benchmark's CPU
+baseline leg use it.  It shares no code with the CUDA library.
+
+What it computes (Alg. 4 of App. E, gradients of Eq. ours_train; App. D for the
+gate gradient and the sparse-scope score gradient):
+
+  forward of a row i (gate position inner, softmax gates, training mode):
+    z_j  = sm_scale q_i.k_j + log g_{b(j)}   for j in S_i = B_0 + kept blocks
+    p    = softmax(z),  o_i = sum_j p_j v_j
+  given dO (the loss gradient of O):
+    dp_j    = dO_i . v_j,   Delta_i = dO_i . o_i
+    dz_j    = p_j (dp_j - Delta_i)                      (softmax backward)
+    dQ_i    = sm_scale sum_j dz_j k_j
+    dK_j   += sm_scale dz_j q_i,  dV_j += p_j dO_i
+    dlogg_m = sum_{j in B_m} dz_j  for every kept historical block m
+            (= g_m dg_m with the paper's dg_m = sum_{j in B_m} (p_j / g_m) dO.(v_j - o))
+  sparse-scope score gradient (App. D, training scope; the Top-K choice is a
+  constant of the forward):
+    ds_m = dlogg_m [m kept] - g_m sum_{l kept} dlogg_l,   m < C_i
+  (from ds_m = g_m (dg_m - sum_l g_l dg_l) with dg_l = 0 for dropped blocks).
+
+Selection (which blocks are kept) is taken from the forward: the gradient
+treats it as fixed, as the kernels do.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+from oracle.sas_oracle import _row_keys_and_bias, historical_count, log_gates, MODE_TRAIN_SOFT
+
+
+def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
+    """Gradients of one head's SAS forward (inner softmax gates).
+
+    Q, K, V, dO: [N, d]; s: [N, >=C-1] selector scores (row i reads s[i, :C_i]).
+    Returns dict with dQ, dK, dV [N, d], dlogg [N, topk] (aligned with the
+    forward's ascending kept list, 0 where padded), ds [N, C] (score gradient,
+    0 past each row's history) and Delta [N].
+    """
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    C = -(-N // b)
+    dQ = np.zeros((N, d))
+    dK = np.zeros((N, d))
+    dV = np.zeros((N, V.shape[1]))
+    dlogg = np.zeros((N, max(topk, 1)))
+    ds = np.zeros((N, C))
+    Delta = np.zeros(N)
+    for i in range(N):
+        keys, bias, weight, sel, _ = _row_keys_and_bias(i, s[i], b, topk, mode)
+        z = sm_scale * (K[keys] @ Q[i]) + bias
+        w = np.exp(z - z.max())
+        p = w / w.sum()
+        o = p @ V[keys]
+        dp = V[keys] @ dO[i]
+        Delta[i] = dO[i] @ o
+        dz = p * (dp - Delta[i])
+        dQ[i] = sm_scale * (dz @ K[keys])
+        np.add.at(dK, keys, sm_scale * np.outer(dz, Q[i]))
+        np.add.at(dV, keys, np.outer(p, dO[i]))
+        if mode != MODE_TRAIN_SOFT:
+            continue
+        # kept blocks come first in `keys`, b tokens each, in ascending order
+        c = historical_count(i, b)
+        lg_all = log_gates(np.asarray(s[i][:c], dtype=np.float64))
+        dl = np.zeros(c)
+        for e, m in enumerate(sel):
+            dl[m] = dz[e * b:(e + 1) * b].sum()
+            dlogg[i, e] = dl[m]
+        if c:
+            g = np.exp(lg_all)
+            ds[i, :c] = dl - g * dl.sum()
+    return {"dQ": dQ, "dK": dK, "dV": dV, "dlogg": dlogg[:, :topk], "ds": ds, "Delta": Delta}
+
+
+def backward_flops_head(N, b, topk, d, sel_counts=None):
+    """Algorithmic FLOPs of the backward of one head: per attended (row, key)
+    pair the four products q.k, dO.v, dS k (into dQ) and the two key-side
+    products dS^T q and P^T dO, 2 d FLOPs each -> 10 d per pair (Alg. 4 runs
+    q.k and dO.v in both passes: the kernels execute 14 d)."""
+    pairs = 0
+    for i in range(N):
+        c = i // b
+        kept = min(topk, c)
+        pairs += kept * b + (i - c * b + 1)
+    return 10 * d * pairs
