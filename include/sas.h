@@ -137,6 +137,36 @@ sas_status sas_attention_fwd(sas_handle* h,
                              int32_t* sel_idx, float* sel_logg,
                              void* stream);
 
+/* Backward of sas_attention_fwd (Alg. 4 of App. E; gate and score gradients
+ * of App. D), for d = 128, softmax gates in the inner position, either mode.
+ * The kept sets are those of the forward (the Top-K choice is a constant of
+ * the backward), and the per-tile block lists are read from the handle: call
+ * it after the sas_attention_fwd of the same inputs on this handle, with no
+ * other forward in between.
+ *
+ *   Q, K, V, O bf16 [B, H, N, d]; LSE fp32 [B, H, N]: the forward's     (in)
+ *   dO         bf16 [B, H, N, d] gradient of the loss w.r.t. O          (in)
+ *   sel_idx, sel_logg: the forward's outputs, or NULL if the forward
+ *              was given NULL for them                                   (in)
+ *   scores     fp32 [B, H, N, C] given scores; needed only for dscores   (in)
+ *   dQ, dK, dV bf16 [B, H, N, d]                                         (out)
+ *   dlogg      fp32 [B, H, N, topk] dL/d(log g) of each kept block, in
+ *              the order of sel_idx (0 where padded; all 0 in INFER_HARD
+ *              mode); may be NULL                                        (out)
+ *   dscores    fp32 [B, H, N, C] dL/ds of the given scores, sparse scope:
+ *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
+ *              row's history; SCORES_GIVEN handles only, else NULL       (out)
+ * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
+ * allocates the handle's backward workspace (synchronously). */
+sas_status sas_attention_bwd(sas_handle* h,
+                             const void* Q, const void* K, const void* V,
+                             const float* scores,
+                             const void* O, const float* LSE, const void* dO,
+                             const int32_t* sel_idx, const float* sel_logg,
+                             void* dQ, void* dK, void* dV,
+                             float* dlogg, float* dscores,
+                             void* stream);
+
 /* Dense MLP sublayer Y = GELU(X W1^T + b1) W2^T + b2 with the exact (erf)
  * GELU.  SAS itself does not define or change the MLP; this is the plain
  * transformer MLP that completes a layer.
@@ -199,8 +229,9 @@ sas_status sas_get_device_status(sas_handle* h, int32_t* out_status);
  * the number of launches and the summed milliseconds.  Kinds, in order:
  * 0 block summaries, 1 (unused: the selector's query projection runs inside
  * the selection kernel), 2 selection, 3 attention, 4 MLP up-projection +
- * GELU, 5 MLP down-projection.  n_kinds <= 6. */
-#define SAS_NUM_KERNEL_KINDS 6
+ * GELU, 5 MLP down-projection, 6 attention backward (all its kernels).
+ * n_kinds <= 7. */
+#define SAS_NUM_KERNEL_KINDS 7
 sas_status sas_set_timing(sas_handle* h, int32_t enable);
 sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, int32_t n_kinds);
 

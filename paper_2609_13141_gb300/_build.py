@@ -20,7 +20,7 @@ BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_PATH = os.path.join(HERE, "libsas.so")
 
 SOURCES = ["sas_api.cu", "k_gemm.cu", "k_pool.cu", "k_select.cu", "k_attn.cu", "sas_noalloc.cu", "k_decode.cu",
-           "sas_decode.cu"]
+           "sas_decode.cu", "k_bwd.cu"]
 HEADERS = ["ptx.cuh", "internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",

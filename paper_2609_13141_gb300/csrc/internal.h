@@ -128,6 +128,36 @@ cudaError_t launch_decode_score(const DecodeArgs& a, const KernelEnv& env);
 cudaError_t launch_decode_attn(const DecodeArgs& a, const KernelEnv& env);
 cudaError_t launch_decode_summarize(const DecodeArgs& a, const KernelEnv& env);
 
+// ---- backward of the training forward (Alg. 4), d = 128, inner softmax gates.
+struct AttnBwdArgs {
+    const void* Q;
+    const void* K;
+    const void* V;
+    const void* O;
+    const void* dO;
+    const float* LSE;
+    const int32_t* union_idx;   // the forward's per-tile block lists
+    const int32_t* union_cnt;
+    const int32_t* sel_idx;     // the forward's kept lists and log-gates
+    const float* sel_logg;
+    const float* scores;        // given scores (for ds) or null
+    void* dQ;
+    void* dK;
+    void* dV;
+    float* dlogg;               // [BH][N][topk]
+    float* ds;                  // [BH][N][C] or null
+    // workspace
+    float* delta;               // [BH][N]
+    int32_t* inv_cnt;           // [BH*T]
+    int32_t* inv_off;           // [BH*T + 1]
+    int32_t* inv_cursor;        // [BH*T]
+    int32_t* inv_tiles;         // entries of the inverted lists
+    int N, C, T, BH, topk, mode, d;
+    float sm_scale;
+};
+extern const int kBwdMaxTiles;   // query tiles per head the backward supports
+cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err);
+
 // ---- failure-path self test (bounded wait on a barrier nothing completes)
 cudaError_t launch_wait_selftest(int* status, long long limit, cudaStream_t stream);
 

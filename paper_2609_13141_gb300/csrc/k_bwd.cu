@@ -1,0 +1,729 @@
+// Backward of the SAS training forward (Alg. 4, App. E; gate and score
+// gradients of App. D), d = 128, gate position inner, softmax gates.
+//
+//   bwd_dq_kernel     pass 1, one CTA per (head, 128-row tile) over the tile's
+//                     visited blocks (union of kept blocks + its diagonal
+//                     blocks, the forward's lists): S = Q K^T and dP = dO V^T
+//                     on the tensor cores, P = exp(S + log g - LSE) and
+//                     dS = P (dP - Delta) per row, dS into TMEM as the A
+//                     operand of dQ += dS K; the row sum of dS over a kept
+//                     block is that row's log-gate gradient.
+//   bwd_inv_*         the forward's per-tile block lists inverted into, per
+//                     key pair (blocks 2p, 2p+1), the query tiles that visit
+//                     them (count, scan, fill).
+//   bwd_dkv_kernel    pass 2, one CTA per (head, key pair) over those query
+//                     tiles, 64 rows at a time: S^T = K Q^T, dP^T = V dO^T,
+//                     P^T and dS^T into TMEM, dV += P^T dO and dK += dS^T Q.
+//   bwd_ds_kernel     score gradient of given scores (sparse scope):
+//                     ds_m = dlogg_m [m kept] - g_m sum dlogg.
+// Roles: warps 0-3 are the rows (pass 1) or keys (pass 2) of the tile, one
+// thread per TMEM lane; warp 4 lane 0 issues the TMA loads and the MMAs.
+#include <math_constants.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace sas {
+namespace {
+
+constexpr int kRows = 128;          // query rows per tile
+constexpr int kKeys = 64;           // keys per block
+constexpr int kD = 128;             // head dim
+constexpr int kWorkers = 128;       // row / key threads
+constexpr int kThreadsB = 160;      // + the issuing warp
+constexpr float kLog2eB = 1.4426950408889634f;
+
+__device__ __forceinline__ float bfl(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bfh(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// 16 packed bf16 pairs into 16 TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+// Delta_i = dO_i . O_i for one row (bf16 rows of d = 128).
+__device__ __forceinline__ float row_delta(const bf16* O, const bf16* dO) {
+    const uint4* o4 = reinterpret_cast<const uint4*>(O);
+    const uint4* g4 = reinterpret_cast<const uint4*>(dO);
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < kD / 8; ++i) {
+        const uint4 a = __ldg(o4 + i), b = __ldg(g4 + i);
+        acc = fmaf(bfl(a.x), bfl(b.x), acc); acc = fmaf(bfh(a.x), bfh(b.x), acc);
+        acc = fmaf(bfl(a.y), bfl(b.y), acc); acc = fmaf(bfh(a.y), bfh(b.y), acc);
+        acc = fmaf(bfl(a.z), bfl(b.z), acc); acc = fmaf(bfh(a.z), bfh(b.z), acc);
+        acc = fmaf(bfl(a.w), bfl(b.w), acc); acc = fmaf(bfh(a.w), bfh(b.w), acc);
+    }
+    return acc;
+}
+
+// ------------------------------------------------------------------ pass 1
+
+struct DqCtl {
+    uint64_t q_full, kv_full[2], kv_empty[2], sdp_full, ds_full[2], dq_done[2], fin;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+constexpr int kQBytes = kRows * kD * 2;                 // 32 KB
+constexpr int kKVBytes = kKeys * kD * 2;                // 16 KB
+constexpr int kDqOffDO = kQBytes;
+constexpr int kDqOffKV = 2 * kQBytes;                   // 2 stages x (K, V)
+constexpr int kDqOffCtl = kDqOffKV + 2 * 2 * kKVBytes;
+constexpr int kDqSmem = kDqOffCtl + 256 + 1024;         // + alignment slack
+// TMEM: dQ [0,128), S [128,192), dP [192,256), dS buffers [256,288), [288,320)
+constexpr uint32_t kTmemDQ = 0, kTmemS = 128, kTmemDP = 192, kTmemDS = 256;
+
+struct BwdParams {
+    const bf16* O;
+    const bf16* dO;
+    const float* LSE;
+    const int32_t* union_idx;
+    const int32_t* union_cnt;
+    const int32_t* sel_idx;
+    const float* sel_logg;
+    bf16* dQ;
+    bf16* dK;
+    bf16* dV;
+    float* dlogg;
+    float* delta;
+    const int32_t* inv_off;
+    const int32_t* inv_tiles;
+    int N, C, T, BH, topk, mode;
+    float sm_scale, scale_log2;
+    int* status;
+    long long limit;
+};
+
+__global__ void __launch_bounds__(kThreadsB, 1)
+bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
+              const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapV, BwdParams p) {
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    uint8_t* smem = dsm + ((1024u - (smem_u32(dsm) & 1023u)) & 1023u);
+    DqCtl& ctl = *reinterpret_cast<DqCtl*>(smem + kDqOffCtl);
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int tile = blockIdx.x % p.T, bh = blockIdx.x / p.T;
+    const long long tb = static_cast<long long>(bh) * p.T + tile;
+    const int32_t* ulist = p.union_idx + tb * p.C;
+    const int U = __ldg(p.union_cnt + tb);
+    const int nb = U + ((2 * tile + 1 < p.C) ? 2 : 1);   // visited blocks: union, then the diagonal ones
+    if (t == 0) {
+        mbar_init(&ctl.q_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&ctl.kv_full[s], 1);
+            mbar_init(&ctl.kv_empty[s], 1);
+            mbar_init(&ctl.ds_full[s], kWorkers);
+            mbar_init(&ctl.dq_done[s], 1);
+        }
+        mbar_init(&ctl.sdp_full, 1);
+        mbar_init(&ctl.fin, 1);
+        ctl.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&ctl.tmem_base, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = ctl.tmem_base;
+    const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
+    const int row0 = tile * kRows;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            // ---- issuer: TMA loads and MMAs
+            auto block_at = [&](int j) { return j < U ? __ldg(ulist + j) : 2 * tile + (j - U); };
+            mbar_arrive_expect_tx(&ctl.q_full, 2 * kQBytes);
+            for (int h = 0; h < 2; ++h) {
+                tma_load_3d(smem + h * (kRows * 128), &mapQ, &ctl.q_full, h * 64, row0, bh);
+                tma_load_3d(smem + kDqOffDO + h * (kRows * 128), &mapDO, &ctl.q_full, h * 64, row0, bh);
+            }
+            auto load_kv = [&](int j) {
+                const int s = j & 1;
+                const int m = block_at(j);
+                uint8_t* st = smem + kDqOffKV + s * 2 * kKVBytes;
+                mbar_arrive_expect_tx(&ctl.kv_full[s], 2 * kKVBytes);
+                for (int h = 0; h < 2; ++h) {
+                    tma_load_3d(st + h * (kKeys * 128), &mapK, &ctl.kv_full[s], h * 64, m * kKeys, bh);
+                    tma_load_3d(st + kKVBytes + h * (kKeys * 128), &mapV, &ctl.kv_full[s], h * 64, m * kKeys, bh);
+                }
+            };
+            load_kv(0);
+            if (nb > 1) load_kv(1);
+            constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
+            constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
+            const uint32_t qb = smem_u32(smem), gb = smem_u32(smem + kDqOffDO);
+            bool ok = mbar_wait(&ctl.q_full, 0, wc);
+            for (int j = 0; ok && j < nb; ++j) {
+                const int s = j & 1;
+                if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t kb = smem_u32(smem + kDqOffKV + s * 2 * kKVBytes), vb = kb + kKVBytes;
+#pragma unroll
+                for (int k = 0; k < kD / 16; ++k) {
+                    const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                    const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+                    umma_bf16(tmem + kTmemS, smem_desc_sw128(qb + oq, 16, 1024), smem_desc_sw128(kb + ok2, 16, 1024),
+                              IDESC_S, k > 0);
+                    umma_bf16(tmem + kTmemDP, smem_desc_sw128(gb + oq, 16, 1024), smem_desc_sw128(vb + ok2, 16, 1024),
+                              IDESC_S, k > 0);
+                }
+                umma_commit(&ctl.sdp_full);
+                // dS of block j is in TMEM buffer j & 1 once every row has written it
+                if (!mbar_wait(&ctl.ds_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+#pragma unroll
+                for (int k = 0; k < kKeys / 16; ++k)
+                    umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + s * 32 + k * 8,
+                                 smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ, (j > 0 || k > 0) ? 1u : 0u);
+                umma_commit(&ctl.dq_done[s]);
+                umma_commit(&ctl.kv_empty[s]);
+                if (j + 2 < nb) {
+                    if (!mbar_wait(&ctl.kv_empty[s], (j >> 1) & 1, wc)) { ok = false; break; }
+                    load_kv(j + 2);
+                }
+            }
+            umma_commit(&ctl.fin);
+            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+        }
+    } else {
+        // ---- rows
+        const int r = t;                       // row of the tile = TMEM lane
+        const int i = row0 + r;
+        const bool valid = i < p.N;
+        const int c = i >> 6;                  // the row's current block
+        const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+        const long long roff = static_cast<long long>(bh) * p.N + i;
+        float delta = 0.f, lse2 = 0.f;
+        if (valid) {
+            delta = row_delta(p.O + roff * kD, p.dO + roff * kD);
+            lse2 = __ldg(p.LSE + roff) * kLog2eB;
+            p.delta[roff] = delta;
+        }
+        const int nsel = valid ? min(p.topk, c) : 0;
+        const int32_t* my_idx = p.sel_idx + roff * p.topk;
+        const float* my_lg = p.sel_logg + roff * p.topk;
+        float* my_dlg = p.dlogg + roff * p.topk;
+        int e = 0;                             // next kept entry (ascending)
+        int km = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
+        float kl = nsel > 0 ? __ldg(my_lg) : 0.f;
+        const bool train = p.mode == 0;
+        bool ok = true;
+        for (int j = 0; j < nb; ++j) {
+            const int m = j < U ? __ldg(ulist + j) : 2 * tile + (j - U);
+            float bias = 0.f;
+            int lim = -1;
+            bool kept = false;
+            if (valid) {
+                if (m < c) {
+                    if (m == km) {
+                        kept = true;
+                        bias = train ? kl * kLog2eB : 0.f;
+                        lim = kKeys - 1;
+                    }
+                } else if (m == c) {
+                    lim = i & (kKeys - 1);
+                }
+            }
+            if (!mbar_wait_warp(&ctl.sdp_full, j & 1, wc)) { ok = false; break; }
+            // the dS buffer j & 1 is free once dQ of block j - 2 has read it
+            if (j >= 2 && !mbar_wait_warp(&ctl.dq_done[j & 1], ((j - 2) >> 1) & 1, wc)) { ok = false; break; }
+            tc_fence_after();
+            float sum = 0.f;
+#pragma unroll
+            for (int hk = 0; hk < 2; ++hk) {
+                uint32_t sv[32], dv[32];
+                tmem_ld32(lane_addr + kTmemS + hk * 32, sv);
+                tmem_ld32(lane_addr + kTmemDP + hk * 32, dv);
+                tmem_wait_ld();
+                uint32_t pk[16];
+#pragma unroll
+                for (int k = 0; k < 32; k += 2) {
+                    float ds2[2];
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const int key = hk * 32 + k + u;
+                        const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
+                        const float pr = key <= lim ? fast_exp2(z - lse2) : 0.f;
+                        ds2[u] = pr * (__uint_as_float(dv[k + u]) - delta);
+                        sum += ds2[u];
+                    }
+                    pk[k >> 1] = pack_bf16x2(ds2[0], ds2[1]);
+                }
+                tmem_st16(lane_addr + kTmemDS + (j & 1) * 32 + hk * 16, pk);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(&ctl.ds_full[j & 1]);
+            if (kept) {
+                my_dlg[e] = train ? sum : 0.f;   // no gates in the inference form
+                ++e;
+                km = e < nsel ? __ldg(my_idx + e) : 0x7fffffff;
+                kl = e < nsel ? __ldg(my_lg + e) : 0.f;
+            }
+        }
+        // kept entries never visited cannot exist (every kept block is in the union);
+        // the rest of the row's dlogg slots (padding) are zero
+        if (valid)
+            for (int q = nsel; q < p.topk; ++q) my_dlg[q] = 0.f;
+        if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
+            tc_fence_after();
+#pragma unroll 1
+            for (int cc = 0; cc < kD / 32; ++cc) {
+                uint32_t o[32];
+                tmem_ld32(lane_addr + kTmemDQ + cc * 32, o);
+                tmem_wait_ld();
+                if (valid) {
+                    uint4* dst = reinterpret_cast<uint4*>(p.dQ + roff * kD + cc * 32);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        dst[q] = make_uint4(pack_bf16x2(__uint_as_float(o[8 * q + 0]) * p.sm_scale, __uint_as_float(o[8 * q + 1]) * p.sm_scale),
+                                            pack_bf16x2(__uint_as_float(o[8 * q + 2]) * p.sm_scale, __uint_as_float(o[8 * q + 3]) * p.sm_scale),
+                                            pack_bf16x2(__uint_as_float(o[8 * q + 4]) * p.sm_scale, __uint_as_float(o[8 * q + 5]) * p.sm_scale),
+                                            pack_bf16x2(__uint_as_float(o[8 * q + 6]) * p.sm_scale, __uint_as_float(o[8 * q + 7]) * p.sm_scale));
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// ------------------------------------------------------- inverted block lists
+
+// count: for every tile, the key pairs (2p, 2p+1) its union list touches
+__global__ void bwd_inv_count_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cnt, int BH,
+                                     int T, int C) {
+    const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (tb >= static_cast<long long>(BH) * T) return;
+    const int bh = static_cast<int>(tb / T);
+    const int32_t* u = union_idx + tb * C;
+    const int U = union_cnt[tb];
+    int last = -1;
+    for (int k = 0; k < U; ++k) {
+        const int pr = u[k] >> 1;
+        if (pr == last) continue;
+        last = pr;
+        atomicAdd(cnt + static_cast<long long>(bh) * T + pr, 1);
+    }
+}
+
+// exclusive scan of n counts into off[0..n] (one CTA of 1024 threads)
+__global__ void __launch_bounds__(1024) bwd_inv_scan_kernel(const int32_t* cnt, int32_t* off, int32_t* cursor,
+                                                            long long n) {
+    __shared__ int part[1024];
+    const int t = threadIdx.x;
+    const long long per = (n + 1023) / 1024;
+    const long long lo = min(static_cast<long long>(t) * per, n), hi = min(lo + per, n);
+    int s = 0;
+    for (long long k = lo; k < hi; ++k) s += cnt[k];
+    part[t] = s;
+    __syncthreads();
+    for (int o = 1; o < 1024; o <<= 1) {
+        const int v = t >= o ? part[t - o] : 0;
+        __syncthreads();
+        part[t] += v;
+        __syncthreads();
+    }
+    int run = part[t] - s;
+    for (long long k = lo; k < hi; ++k) {
+        off[k] = run;
+        cursor[k] = run;
+        run += cnt[k];
+    }
+    if (t == 1023) off[n] = part[1023];
+}
+
+__global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cursor,
+                                    int32_t* tiles, int BH, int T, int C) {
+    const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (tb >= static_cast<long long>(BH) * T) return;
+    const int bh = static_cast<int>(tb / T);
+    const int tile = static_cast<int>(tb - static_cast<long long>(bh) * T);
+    const int32_t* u = union_idx + tb * C;
+    const int U = union_cnt[tb];
+    int last = -1;
+    for (int k = 0; k < U; ++k) {
+        const int pr = u[k] >> 1;
+        if (pr == last) continue;
+        last = pr;
+        const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pr, 1);
+        tiles[slot] = tile;
+    }
+}
+
+// ------------------------------------------------------------------ pass 2
+
+struct DkvCtl {
+    uint64_t kv_full, q_full[2], q_empty[2], sdp_full, pds_full, half_done, fin;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+constexpr int kPairBytes = 2 * kKeys * kD * 2;           // 32 KB: K (or V) of the key pair
+constexpr int kDkvOffV = kPairBytes;
+constexpr int kDkvOffQ = 2 * kPairBytes;                 // 2 stages x (Q, dO) tiles
+constexpr int kDkvOffInfo = kDkvOffQ + 2 * 2 * kQBytes;  // 2 stages x [4][128] floats: lse2, delta, bias0, bias1
+constexpr int kDkvOffList = kDkvOffInfo + 2 * 4 * kRows * 4;
+// query tiles of a key pair (sorted list, then the unsorted copy); the host
+// refuses heads of more than kBwdMaxTiles tiles
+constexpr int kDkvListCap = 2048;
+constexpr int kDkvOffCtl = kDkvOffList + 2 * kDkvListCap * 4;
+constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
+// TMEM: dV [0,128), dK [128,256), S^T [256,320), dP^T [320,384), P^T [384,416), dS^T [416,448)
+constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemST = 256, kTmemDPT = 320, kTmemPT = 384, kTmemDST = 416;
+
+// Bias (log2 units, or a marker) of block m for query row i: kept historical
+// block -> log g (training) or 0; the row's own block -> 0 with the causal
+// limit applied by the caller; otherwise -inf.
+__device__ __forceinline__ float row_block_bias(const BwdParams& p, int bh, int i, int m) {
+    if (i >= p.N) return -CUDART_INF_F;
+    const int c = i >> 6;
+    if (m > c) return -CUDART_INF_F;
+    if (m == c) return 0.f;
+    const int nsel = min(p.topk, c);
+    const long long roff = static_cast<long long>(bh) * p.N + i;
+    const int32_t* idx = p.sel_idx + roff * p.topk;
+    int lo = 0, hi = nsel;   // first entry >= m in the ascending kept list
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldg(idx + mid) < m) lo = mid + 1; else hi = mid;
+    }
+    if (lo < nsel && __ldg(idx + lo) == m) return p.mode == 0 ? __ldg(p.sel_logg + roff * p.topk + lo) * kLog2eB : 0.f;
+    return -CUDART_INF_F;
+}
+
+__global__ void __launch_bounds__(kThreadsB, 1)
+bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
+               const __grid_constant__ CUtensorMap mapK2, const __grid_constant__ CUtensorMap mapV2, BwdParams p) {
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    uint8_t* smem = dsm + ((1024u - (smem_u32(dsm) & 1023u)) & 1023u);
+    DkvCtl& ctl = *reinterpret_cast<DkvCtl*>(smem + kDkvOffCtl);
+    int* list = reinterpret_cast<int*>(smem + kDkvOffList);
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int pr = blockIdx.x % p.T, bh = blockIdx.x / p.T;   // key pair = blocks 2pr, 2pr+1 (keys 128 pr ..)
+    const long long pb = static_cast<long long>(bh) * p.T + pr;
+    const int off = __ldg(p.inv_off + pb);
+    const int cnt = min(__ldg(p.inv_off + pb + 1) - off, kDkvListCap - 1);
+    const int nq = cnt + 1;                                    // the diagonal tile pr first
+    if (t == 0) {
+        mbar_init(&ctl.kv_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&ctl.q_full[s], 1);
+            mbar_init(&ctl.q_empty[s], 1);
+        }
+        mbar_init(&ctl.sdp_full, 1);
+        mbar_init(&ctl.pds_full, kWorkers);
+        mbar_init(&ctl.half_done, 1);
+        mbar_init(&ctl.fin, 1);
+        ctl.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&ctl.tmem_base, 512);
+        tmem_relinquish();
+    }
+    // the query tiles: diagonal first, then the others in ascending order (a
+    // fixed summation order); rank sort of the inverted list in shared memory
+    int* raw = list + kDkvListCap;
+    if (t == 0) list[0] = pr;
+    for (int k = t; k < cnt; k += kThreadsB) raw[k] = __ldg(p.inv_tiles + off + k);
+    __syncthreads();
+    for (int k = t; k < cnt; k += kThreadsB) {
+        const int v = raw[k];
+        int rank = 0;
+        for (int q = 0; q < cnt; ++q) rank += raw[q] < v;
+        list[1 + rank] = v;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = ctl.tmem_base;
+    const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
+    float* info = reinterpret_cast<float*>(smem + kDkvOffInfo);
+
+    if (warp == 4) {
+        if (lane == 0) {
+            // ---- issuer
+            mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
+            for (int h = 0; h < 2; ++h) {
+                tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+                tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+            }
+            auto load_q = [&](int q) {
+                const int s = q & 1;
+                const int tq = list[q];
+                uint8_t* st = smem + kDkvOffQ + s * 2 * kQBytes;
+                mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
+                for (int h = 0; h < 2; ++h) {
+                    tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, tq * kRows, bh);
+                    tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, tq * kRows, bh);
+                }
+            };
+            load_q(0);
+            if (nq > 1) load_q(1);
+            constexpr uint32_t IDESC_T = idesc_bf16(2 * kKeys, 64, 0, 0);   // M = 128 keys, N = 64 rows
+            constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
+            const uint32_t kb = smem_u32(smem), vb = smem_u32(smem + kDkvOffV);
+            bool ok = mbar_wait(&ctl.kv_full, 0, wc);
+            int hs = 0;   // halves issued so far
+            for (int q = 0; ok && q < nq; ++q) {
+                const int s = q & 1;
+                if (!mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc)) { ok = false; break; }
+                const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
+                for (int h = 0; h < 2; ++h, ++hs) {
+                    tc_fence_after();
+#pragma unroll
+                    for (int k = 0; k < kD / 16; ++k) {
+                        const uint32_t ok2 = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
+                        const uint32_t oq = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
+                        umma_bf16(tmem + kTmemST, smem_desc_sw128(kb + ok2, 16, 1024), smem_desc_sw128(qb + oq, 16, 1024),
+                                  IDESC_T, k > 0);
+                        umma_bf16(tmem + kTmemDPT, smem_desc_sw128(vb + ok2, 16, 1024), smem_desc_sw128(gb + oq, 16, 1024),
+                                  IDESC_T, k > 0);
+                    }
+                    umma_commit(&ctl.sdp_full);
+                    if (!mbar_wait(&ctl.pds_full, hs & 1, wc)) { ok = false; break; }
+                    tc_fence_after();
+#pragma unroll
+                    for (int k = 0; k < 64 / 16; ++k) {
+                        // B = dO (or Q) rows of this half, MN-major: 16 rows = two 8-row atoms
+                        const uint32_t ob = h * 64 * 128 + k * 2048;
+                        const uint32_t acc = (q > 0 || h > 0 || k > 0) ? 1u : 0u;
+                        umma_bf16_ta(tmem + kTmemDV, tmem + kTmemPT + k * 8, smem_desc_sw128(gb + ob, kRows * 128, 1024),
+                                     IDESC_ACC, acc);
+                        umma_bf16_ta(tmem + kTmemDK, tmem + kTmemDST + k * 8, smem_desc_sw128(qb + ob, kRows * 128, 1024),
+                                     IDESC_ACC, acc);
+                    }
+                    umma_commit(&ctl.half_done);
+                }
+                if (!ok) break;
+                umma_commit(&ctl.q_empty[s]);
+                if (q + 2 < nq) {
+                    if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc)) { ok = false; break; }
+                    load_q(q + 2);
+                }
+            }
+            umma_commit(&ctl.fin);
+            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+        }
+    } else {
+        // ---- keys: thread = key of the pair (TMEM lane)
+        const int key = t;
+        const int kg = pr * 2 * kKeys + key;      // global key index
+        const int kblk = key >> 6;                // 0: block 2pr, 1: block 2pr + 1
+        const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+        bool ok = true;
+        int hs = 0;
+        for (int q = 0; q < nq; ++q) {
+            const int s = q & 1;
+            const int tq = list[q];
+            float* inf = info + s * 4 * kRows;
+            // per-row data of this query tile (thread = row for this part); the
+            // buffer s was last read two tiles ago, before that tile's last pds_full
+            {
+                const int i = tq * kRows + t;
+                const long long roff = static_cast<long long>(bh) * p.N + i;
+                const bool v = i < p.N;
+                inf[t] = v ? __ldg(p.LSE + roff) * kLog2eB : 0.f;
+                inf[kRows + t] = v ? p.delta[roff] : 0.f;
+                inf[2 * kRows + t] = row_block_bias(p, bh, i, 2 * pr);
+                inf[3 * kRows + t] = row_block_bias(p, bh, i, 2 * pr + 1);
+            }
+            named_bar_sync(1, kWorkers);
+            for (int h = 0; h < 2; ++h, ++hs) {
+                if (!mbar_wait_warp(&ctl.sdp_full, hs & 1, wc)) { ok = false; break; }
+                // P^T / dS^T columns are free once the previous half's products have read them
+                if (hs >= 1 && !mbar_wait_warp(&ctl.half_done, (hs - 1) & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    uint32_t sv[32], dv[32];
+                    tmem_ld32(lane_addr + kTmemST + hr * 32, sv);
+                    tmem_ld32(lane_addr + kTmemDPT + hr * 32, dv);
+                    tmem_wait_ld();
+                    uint32_t pp[16], dd[16];
+#pragma unroll
+                    for (int k = 0; k < 32; k += 2) {
+                        float pv[2], dsv[2];
+#pragma unroll
+                        for (int u = 0; u < 2; ++u) {
+                            const int rr = h * 64 + hr * 32 + k + u;        // row of the query tile
+                            const int i = tq * kRows + rr;
+                            const float bias = inf[(2 + kblk) * kRows + rr];
+                            // the row's own block: causal (key <= row); -inf bias: not attended
+                            const bool vis = bias != -CUDART_INF_F && (kg >> 6 != i >> 6 || kg <= i);
+                            const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
+                            const float pr_ = vis ? fast_exp2(z - inf[rr]) : 0.f;
+                            pv[u] = pr_;
+                            dsv[u] = pr_ * (__uint_as_float(dv[k + u]) - inf[kRows + rr]);
+                        }
+                        pp[k >> 1] = pack_bf16x2(pv[0], pv[1]);
+                        dd[k >> 1] = pack_bf16x2(dsv[0], dsv[1]);
+                    }
+                    tmem_st16(lane_addr + kTmemPT + hr * 16, pp);
+                    tmem_st16(lane_addr + kTmemDST + hr * 16, dd);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+                mbar_arrive(&ctl.pds_full);
+            }
+            if (!ok) break;
+        }
+        if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
+            tc_fence_after();
+            const bool kv = kg < p.N;
+            const long long koff = static_cast<long long>(bh) * p.N + kg;
+#pragma unroll 1
+            for (int which = 0; which < 2; ++which) {
+                bf16* dst_row = (which == 0 ? p.dV : p.dK) + koff * kD;
+                const float sc = which == 0 ? 1.f : p.sm_scale;
+#pragma unroll 1
+                for (int cc = 0; cc < kD / 32; ++cc) {
+                    uint32_t o[32];
+                    tmem_ld32(lane_addr + (which == 0 ? kTmemDV : kTmemDK) + cc * 32, o);
+                    tmem_wait_ld();
+                    if (kv) {
+                        uint4* dst = reinterpret_cast<uint4*>(dst_row + cc * 32);
+#pragma unroll
+                        for (int q2 = 0; q2 < 4; ++q2)
+                            dst[q2] = make_uint4(pack_bf16x2(__uint_as_float(o[8 * q2 + 0]) * sc, __uint_as_float(o[8 * q2 + 1]) * sc),
+                                                 pack_bf16x2(__uint_as_float(o[8 * q2 + 2]) * sc, __uint_as_float(o[8 * q2 + 3]) * sc),
+                                                 pack_bf16x2(__uint_as_float(o[8 * q2 + 4]) * sc, __uint_as_float(o[8 * q2 + 5]) * sc),
+                                                 pack_bf16x2(__uint_as_float(o[8 * q2 + 6]) * sc, __uint_as_float(o[8 * q2 + 7]) * sc));
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// --------------------------------------------------------- score gradient
+
+// one warp per row: ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of
+// the row's C_i given scores; 0 past the history
+__global__ void bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* dlogg, float* ds, int BH,
+                              int N, int C, int topk) {
+    const long long w = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= static_cast<long long>(BH) * N) return;
+    const int i = static_cast<int>(w % N);
+    const int c = i >> 6;
+    const float* s = scores + w * C;
+    float* out = ds + w * C;
+    float mx = -CUDART_INF_F;
+    for (int m = lane; m < c; m += 32) mx = fmaxf(mx, s[m]);
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float se = 0.f;
+    for (int m = lane; m < c; m += 32) se += __expf(s[m] - mx);
+    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+    const float lse = mx + __logf(se);
+    const int nsel = min(topk, c);
+    float sum = 0.f;
+    for (int e = lane; e < nsel; e += 32) sum += dlogg[w * topk + e];
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    for (int m = lane; m < C; m += 32) out[m] = m < c ? -__expf(s[m] - lse) * sum : 0.f;
+    __syncwarp();
+    for (int e = lane; e < nsel; e += 32) {
+        const int m = sel_idx[w * topk + e];
+        out[m] += dlogg[w * topk + e];
+    }
+}
+
+}  // namespace
+
+const int kBwdMaxTiles = kDkvListCap - 1;
+
+cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err) {
+    if (a.d != kD) {
+        *err = "backward: head dim must be 128";
+        return cudaErrorInvalidValue;
+    }
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(bwd_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(bwd_dkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDkvSmem);
+        if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(bwd)"; return e; }
+        attr = true;
+    }
+    CUtensorMap mq, mdo, mk, mv, mk2, mv2;
+    if (make_tmap_bf16_3d(&mq, a.Q, kD, a.N, a.BH, 64, kRows) != 0 ||
+        make_tmap_bf16_3d(&mdo, a.dO, kD, a.N, a.BH, 64, kRows) != 0 ||
+        make_tmap_bf16_3d(&mk, a.K, kD, a.N, a.BH, 64, kKeys) != 0 ||
+        make_tmap_bf16_3d(&mv, a.V, kD, a.N, a.BH, 64, kKeys) != 0 ||
+        make_tmap_bf16_3d(&mk2, a.K, kD, a.N, a.BH, 64, 2 * kKeys) != 0 ||
+        make_tmap_bf16_3d(&mv2, a.V, kD, a.N, a.BH, 64, 2 * kKeys) != 0) {
+        *err = "backward tensor maps";
+        return cudaErrorInvalidValue;
+    }
+    BwdParams p{};
+    p.O = static_cast<const bf16*>(a.O);
+    p.dO = static_cast<const bf16*>(a.dO);
+    p.LSE = a.LSE;
+    p.union_idx = a.union_idx;
+    p.union_cnt = a.union_cnt;
+    p.sel_idx = a.sel_idx;
+    p.sel_logg = a.sel_logg;
+    p.dQ = static_cast<bf16*>(a.dQ);
+    p.dK = static_cast<bf16*>(a.dK);
+    p.dV = static_cast<bf16*>(a.dV);
+    p.dlogg = a.dlogg;
+    p.delta = a.delta;
+    p.inv_off = a.inv_off;
+    p.inv_tiles = a.inv_tiles;
+    p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
+    p.sm_scale = a.sm_scale;
+    p.scale_log2 = a.sm_scale * kLog2eB;
+    p.status = env.status;
+    p.limit = env.limit;
+    const long long tiles = static_cast<long long>(a.BH) * a.T;
+    if (tiles > 0x7fffffffLL) { *err = "backward: too many tiles"; return cudaErrorInvalidValue; }
+    // pass 1 (also writes Delta for pass 2)
+    bwd_dq_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
+    // inverted lists
+    e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(tiles) * 4, env.stream);
+    if (e != cudaSuccess) { *err = "backward list counts"; return e; }
+    const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
+    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
+    bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, tiles);
+    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cursor, a.inv_tiles, a.BH, a.T, a.C);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
+    // pass 2
+    bwd_dkv_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
+    if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
+        const long long rows = static_cast<long long>(a.BH) * a.N;
+        bwd_ds_kernel<<<static_cast<unsigned>((rows * 32 + 255) / 256), 256, 0, env.stream>>>(
+            a.scores, a.sel_idx, a.dlogg, a.ds, a.BH, a.N, a.C, a.topk);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
+    } else if (a.ds != nullptr) {
+        e = cudaMemsetAsync(a.ds, 0, static_cast<size_t>(a.BH) * a.N * a.C * 4, env.stream);
+        if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
+    }
+    return cudaSuccess;
+}
+
+}  // namespace sas

@@ -102,6 +102,11 @@ struct sas_handle {
     // MLP hidden activation
     void* hidden = nullptr;
     size_t hidden_bytes = 0;
+    // backward workspace (allocated by the first sas_attention_bwd)
+    float* bwd_delta = nullptr;
+    int32_t* bwd_inv = nullptr;     // counts, offsets, cursors
+    int32_t* bwd_tiles = nullptr;
+    float* bwd_dlogg = nullptr;
     // timing
     bool timing = false;
     std::vector<TimeRec> recs;
@@ -262,6 +267,10 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->status);
     cudaFree(h->sched);
     cudaFree(h->hidden);
+    cudaFree(h->bwd_delta);
+    cudaFree(h->bwd_inv);
+    cudaFree(h->bwd_tiles);
+    cudaFree(h->bwd_dlogg);
     for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
     delete h;
 }
@@ -367,6 +376,68 @@ sas_status sas_mlp_fwd(sas_handle* h, const void* X, const void* W1, const void*
     g2.gelu = 0; g2.bn = pick_bn(D); g2.max_ctas = 0;
     e = timed_launch(h, 5, s, [&] { return sas::launch_gemm(g2, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
+    return SAS_OK;
+}
+
+sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
+                             const void* O, const float* LSE, const void* dO, const int32_t* sel_idx,
+                             const float* sel_logg, void* dQ, void* dK, void* dV, float* dlogg, float* dscores,
+                             void* stream) {
+    if (h == nullptr) return SAS_ERR_INVALID_ARG;
+    const sas_config& c = h->cfg;
+    if (!Q || !K || !V || !O || !LSE || !dO || !dQ || !dK || !dV)
+        return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V, O, LSE, dO, dQ, dK and dV are required");
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(dO) || !aligned16(dQ) ||
+        !aligned16(dK) || !aligned16(dV) || !aligned4(LSE) || (sel_idx && !aligned4(sel_idx)) ||
+        (sel_logg && !aligned4(sel_logg)) || (dlogg && !aligned4(dlogg)) || (dscores && !aligned4(dscores)) ||
+        (scores && !aligned4(scores)))
+        return fail(h, SAS_ERR_INVALID_ARG, "misaligned pointer");
+    if (c.d != 128) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports d = 128");
+    if (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER)
+        return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
+    if (h->T > sas::kBwdMaxTiles) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports N <= 262016");
+    if (dscores) {
+        if (c.selector != SAS_SEL_SCORES_GIVEN || !scores)
+            return fail(h, SAS_ERR_INVALID_ARG, "dscores needs given scores (SCORES_GIVEN)");
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t rows = static_cast<size_t>(h->BH) * c.N;
+    const size_t tiles = static_cast<size_t>(h->BH) * h->T;
+    if (h->bwd_delta == nullptr) {
+        // first backward on this handle: workspace (synchronous)
+        cudaError_t e = cudaStreamSynchronize(s);
+        const size_t pairs = static_cast<size_t>(h->T < h->C ? h->T : h->C);
+        if (e == cudaSuccess) e = alloc(&h->bwd_delta, rows * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_inv, (3 * tiles + 1) * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_tiles, tiles * pairs * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, rows * (c.topk > 0 ? c.topk : 1) * 4);
+        if (e != cudaSuccess) {
+            cudaFree(h->bwd_delta); cudaFree(h->bwd_inv); cudaFree(h->bwd_tiles); cudaFree(h->bwd_dlogg);
+            h->bwd_delta = nullptr; h->bwd_inv = nullptr; h->bwd_tiles = nullptr; h->bwd_dlogg = nullptr;
+            return cuda_fail(h, e, "backward workspace");
+        }
+    }
+    sas::AttnBwdArgs a{};
+    a.Q = Q; a.K = K; a.V = V; a.O = O; a.dO = dO; a.LSE = LSE;
+    a.union_idx = h->union_idx; a.union_cnt = h->union_cnt;
+    a.sel_idx = sel_idx ? sel_idx : h->sel_idx;
+    a.sel_logg = sel_logg ? sel_logg : h->sel_logg;
+    a.scores = dscores ? scores : nullptr;
+    a.dQ = dQ; a.dK = dK; a.dV = dV;
+    a.dlogg = dlogg ? dlogg : h->bwd_dlogg;
+    a.ds = dscores;
+    a.delta = h->bwd_delta;
+    a.inv_cnt = h->bwd_inv;
+    a.inv_cursor = h->bwd_inv + tiles;
+    a.inv_off = h->bwd_inv + 2 * tiles;
+    a.inv_tiles = h->bwd_tiles;
+    a.N = c.N; a.C = h->C; a.T = h->T; a.BH = h->BH; a.topk = c.topk; a.mode = c.mode; a.d = c.d;
+    a.sm_scale = h->sm_scale;
+    const sas::KernelEnv env{s, h->status, h->limit};
+    const char* err = "";
+    cudaError_t e = timed_launch(h, 6, s, [&] { return sas::launch_attn_bwd(a, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    h->launches += (a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 5 : 4;   // six or five kernels in all
     return SAS_OK;
 }
 

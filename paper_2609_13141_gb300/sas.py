@@ -32,8 +32,9 @@ SAS_GATE_SIGMOID = 1
 SAS_GATE_LOGIT = 2
 SAS_GATE_INNER = 0
 SAS_GATE_OUTER = 1
-SAS_NUM_KERNEL_KINDS = 6
-KERNEL_KINDS = ["block_summaries", "query_projection", "selection", "attention", "mlp_up_gelu", "mlp_down"]
+SAS_NUM_KERNEL_KINDS = 7
+KERNEL_KINDS = ["block_summaries", "query_projection", "selection", "attention", "mlp_up_gelu", "mlp_down",
+                "attention_bwd"]
 
 HEADER = os.path.join(_build.ROOT, "include", "sas.h")
 
@@ -80,6 +81,8 @@ def lib():
     L.sas_destroy.restype = None
     L.sas_attention_fwd.argtypes = [vp] * 12
     L.sas_attention_fwd.restype = i32
+    L.sas_attention_bwd.argtypes = [vp] * 16
+    L.sas_attention_bwd.restype = i32
     L.sas_mlp_fwd.argtypes = [vp] * 7 + [i64, i64, i64, vp]
     L.sas_mlp_fwd.restype = i32
     L.sas_status_str.argtypes = [i32]
@@ -198,6 +201,17 @@ def sas_attention_fwd(h, Q, K, V, O, scores=None, Wq=None, Wk=None, LSE=None, se
     _check(st, h, "sas_attention_fwd")
 
 
+def sas_attention_bwd(h, Q, K, V, O, LSE, dO, dQ, dK, dV, scores=None, sel_idx=None, sel_logg=None, dlogg=None,
+                      dscores=None, stream=None):
+    bf, f32 = torch.bfloat16, torch.float32
+    st = lib().sas_attention_bwd(
+        h, _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"), _ptr(scores, f32, "scores", False),
+        _ptr(O, bf, "O"), _ptr(LSE, f32, "LSE"), _ptr(dO, bf, "dO"), _ptr(sel_idx, torch.int32, "sel_idx", False),
+        _ptr(sel_logg, f32, "sel_logg", False), _ptr(dQ, bf, "dQ"), _ptr(dK, bf, "dK"), _ptr(dV, bf, "dV"),
+        _ptr(dlogg, f32, "dlogg", False), _ptr(dscores, f32, "dscores", False), _stream(stream))
+    _check(st, h, "sas_attention_bwd")
+
+
 def sas_mlp_fwd(h, X, W1, W2, Y, b1=None, b2=None, stream=None):
     bf = torch.bfloat16
     T, D = X.shape
@@ -281,6 +295,17 @@ class SasLayer:
             sel_logg = torch.empty(self.B, self.H, self.N, k, device=dev, dtype=torch.float32)
         sas_attention_fwd(self.h, Q, K, V, O, scores, Wq, Wk, LSE, sel_idx, sel_logg, stream)
         return O, LSE, sel_idx, sel_logg
+
+    def attention_bwd(self, Q, K, V, O, LSE, dO, scores=None, sel_idx=None, sel_logg=None, want_ds=False,
+                      stream=None):
+        """Returns (dQ, dK, dV, dlogg, dscores); dscores only with want_ds (given scores)."""
+        dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+        dlogg = torch.empty(self.B, self.H, self.N, max(self.topk, 1), device=Q.device, dtype=torch.float32)
+        ds = None
+        if want_ds:
+            ds = torch.empty(self.B, self.H, self.N, -(-self.N // 64), device=Q.device, dtype=torch.float32)
+        sas_attention_bwd(self.h, Q, K, V, O, LSE, dO, dQ, dK, dV, scores, sel_idx, sel_logg, dlogg, ds, stream)
+        return dQ, dK, dV, dlogg, ds
 
     def mlp(self, X, W1, W2, b1=None, b2=None, stream=None):
         Y = torch.empty(X.shape[0], W2.shape[0], device=X.device, dtype=torch.bfloat16)

@@ -33,7 +33,7 @@ def _worker(rank, world, port, out):
 
 def test_reduce_max_and_job_throughput_two_gloo_ranks():
     port = _free_port()
-    out = mp.Manager().dict()
+    out = mp.get_context("spawn").Manager().dict()
     mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
     for rank in range(2):
         ms, e2e, value = out[rank]
