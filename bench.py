@@ -440,6 +440,97 @@ def run_reference(args, w, rank, world):
     }
 
 
+# ------------------------------------------------------------ training step
+
+TRAIN_METRIC = "SAS attention training step (forward + backward) of one layer: ms and TFLOP/s on 1xGB300"
+
+
+def run_train(args, w, rank, world):
+    """Forward + backward of the SAS attention (Alg. 1 steps 1-4 and Alg. 4) on
+    the workload's attention shape, given block-coherent scores (R1) so that
+    the score gradient is produced too.  Algorithmic FLOPs: the forward's
+    4 d per attended (row, key) pair plus the backward's 10 d (QK^T, dO V^T,
+    dS K, dS^T Q, P^T dO)."""
+    import torch
+
+    from paper_2609_13141_gb300 import sas, synth
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    B, H, N, d, K = (w[k] for k in ("B", "H", "N", "d", "topk"))
+    C = (N + 63) // 64
+    Q, Kk, V = synth.qkv(B, H, N, d, seed=rank)
+    S = synth.scores(B, H, N, C, seed=rank, regime="R1")
+    dO = synth.normal((B, H, N, d), rank + 5).to(torch.bfloat16)
+    Qd, Kd, Vd, Sd, dOd = (t.to(dev) for t in (Q, Kk, V, S, dO))
+    layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN)
+    h = layer.h
+    stream = torch.cuda.current_stream(dev)
+    O = torch.empty_like(Qd)
+    LSE = torch.empty(B, H, N, device=dev, dtype=torch.float32)
+    si = torch.empty(B, H, N, max(K, 1), device=dev, dtype=torch.int32)
+    sl = torch.empty(B, H, N, max(K, 1), device=dev, dtype=torch.float32)
+    dQ, dK, dV = torch.empty_like(Qd), torch.empty_like(Kd), torch.empty_like(Vd)
+    dl = torch.empty_like(sl)
+    ds = torch.empty_like(Sd)
+    flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
+
+    def step():
+        sas.sas_attention_fwd(h, Qd, Kd, Vd, O, Sd, None, None, LSE, si, sl, stream)
+        sas.sas_attention_bwd(h, Qd, Kd, Vd, O, LSE, dOd, dQ, dK, dV, Sd, si, sl, dl, ds, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.2)
+    sas.sas_set_timing(h, True)
+    l0 = sas.sas_launch_count(h)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for k in range(args.steps):
+        flush.zero_()
+        ev[k][0].record(stream)
+        step()
+        ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    launches = sas.sas_launch_count(h) - l0
+    kt = sas.sas_get_timings(h)
+    sas.sas_set_timing(h, False)
+    clocks = sampler.stop()
+    assert sas.sas_get_device_status(h) == 0
+    ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    Tt = (N + 127) // 128
+    unions = sas.sas_get_tile_union_counts(h, B * H * Tt)
+    layer.close()
+    fl = algorithmic_flops(w, learned=False)
+    f_fwd = fl["attention"]
+    f_bwd = f_fwd * 10 // 4
+    tflop = (f_fwd + f_bwd) / 1e12
+    peaks = load_peaks()
+    bwd_ms = kt["attention_bwd"][1] / max(kt["attention_bwd"][0], 1)
+    fwd_ms = kt["attention"][1] / max(kt["attention"][0], 1)
+    sel_ms = kt["selection"][1] / max(kt["selection"][0], 1)
+    ach = f_bwd / (bwd_ms / 1e3) / 1e12
+    return {
+        "metric": TRAIN_METRIC, "value": round(tflop / (ms / 1e3), 2), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 softmax and gradients of log g, s)",
+        "data": "synthetic (seeded; R1 block-coherent scores given, N(0,1) Q/K/V/dO)",
+        "config": {"workload": w["name"] + " (attention only, forward + backward)", "B": B, "H": H, "N": N, "d": d,
+                   "topk": K, "l2": "flushed between timed steps (256 MiB write)", "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "tensor", "kernel": "attention_bwd", "achieved": round(ach, 1), "peak": peaks["bf16"],
+                     "unit": "TFLOP/s", "frac": round(ach / peaks["bf16"], 4), "traffic": None,
+                     "peak_source": f"{peaks['source']} bf16 dense burst"},
+        "mean_union_blocks_per_tile": round(sum(unions) / max(len(unions), 1), 2),
+        "kernels_ms": {"selection": round(sel_ms, 4), "attention_fwd": round(fwd_ms, 4), "attention_bwd": round(bwd_ms, 4)},
+        "algorithmic_tflop_per_step": round(tflop, 4),
+        "gpu_launches": launches,
+        "clocks": clocks,
+    }
+
+
 # ---------------------------------------------------------------- decode
 
 DECODE_METRIC = "decode step latency of one attention layer (us), SAS vs dense, 1xGB300"
@@ -689,6 +780,8 @@ def main():
     ap.add_argument("--batch", type=int, default=1, help="decode: sequences per step")
     ap.add_argument("--decode-only", choices=["sparse", "dense"], default=None,
                     help="decode: run one arm only (for profiling)")
+    ap.add_argument("--train", action="store_true",
+                    help="time the attention training step (forward + backward) of the workload instead")
     ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
                     help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
     ap.add_argument("--topk", type=int, default=None, help="override the workload's K")
@@ -707,6 +800,11 @@ def main():
     if args.topk is not None:
         w["topk"] = args.topk
         w["name"] = w["name"].replace("K=32", f"K={args.topk}")
+    if args.train:
+        out = run_train(args, w, rank, world) if args.impl == "ours" else None
+        if out is not None and rank == 0:
+            print(json.dumps(out))
+        return
     if args.impl == "reference" and args.regime != "R2":
         ap.error("the reference arm times the oracle on the learned-selector workload only")
     out = run_reference(args, w, rank, world) if args.impl == "reference" else run_ours(args, w, rank, world)

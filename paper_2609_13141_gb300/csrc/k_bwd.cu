@@ -29,8 +29,9 @@ namespace {
 constexpr int kRows = 128;          // query rows per tile
 constexpr int kKeys = 64;           // keys per block
 constexpr int kD = 128;             // head dim
-constexpr int kWorkers = 128;       // row / key threads
-constexpr int kThreadsB = 160;      // + the issuing warp
+constexpr int kWorkers = 128;       // key threads (pass 2)
+constexpr int kRowThreads = 256;    // pass 1: two threads per row, 32 keys of a block each
+constexpr int kThreadsB = 288;      // + the issuing warp
 constexpr float kLog2eB = 1.4426950408889634f;
 
 __device__ __forceinline__ float bfl(uint32_t w) { return __uint_as_float(w << 16); }
@@ -65,7 +66,7 @@ __device__ __forceinline__ float row_delta(const bf16* O, const bf16* dO) {
 // ------------------------------------------------------------------ pass 1
 
 struct DqCtl {
-    uint64_t q_full, kv_full[2], kv_empty[2], sdp_full, ds_full[2], dq_done[2], fin;
+    uint64_t q_full, kv_full[2], kv_empty[2], sdp_full[2], ds_full[2], dq_done[2], fin;
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -76,8 +77,9 @@ constexpr int kDqOffDO = kQBytes;
 constexpr int kDqOffKV = 2 * kQBytes;                   // 2 stages x (K, V)
 constexpr int kDqOffCtl = kDqOffKV + 2 * 2 * kKVBytes;
 constexpr int kDqSmem = kDqOffCtl + 256 + 1024;         // + alignment slack
-// TMEM: dQ [0,128), S [128,192), dP [192,256), dS buffers [256,288), [288,320)
-constexpr uint32_t kTmemDQ = 0, kTmemS = 128, kTmemDP = 192, kTmemDS = 256;
+// TMEM: dQ [0,128); S and dP of block j in buffer j & 1: S [128 + 128 b, +64),
+// dP [192 + 128 b, +64); dS buffers [384,416), [416,448)
+constexpr uint32_t kTmemDQ = 0, kTmemS = 128, kTmemDP = 192, kTmemDS = 384;
 
 struct BwdParams {
     const bf16* O;
@@ -117,10 +119,10 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         for (int s = 0; s < 2; ++s) {
             mbar_init(&ctl.kv_full[s], 1);
             mbar_init(&ctl.kv_empty[s], 1);
-            mbar_init(&ctl.ds_full[s], kWorkers);
+            mbar_init(&ctl.ds_full[s], kRowThreads);
             mbar_init(&ctl.dq_done[s], 1);
+            mbar_init(&ctl.sdp_full[s], 1);
         }
-        mbar_init(&ctl.sdp_full, 1);
         mbar_init(&ctl.fin, 1);
         ctl.abort_flag = 0;
         fence_barrier_init();
@@ -136,7 +138,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
     const int row0 = tile * kRows;
 
-    if (warp == 4) {
+    if (warp == 8) {
         if (lane == 0) {
             // ---- issuer: TMA loads and MMAs
             auto block_at = [&](int j) { return j < U ? __ldg(ulist + j) : 2 * tile + (j - U); };
@@ -161,56 +163,66 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
             const uint32_t qb = smem_u32(smem), gb = smem_u32(smem + kDqOffDO);
             bool ok = mbar_wait(&ctl.q_full, 0, wc);
-            for (int j = 0; ok && j < nb; ++j) {
-                const int s = j & 1;
-                if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t kb = smem_u32(smem + kDqOffKV + s * 2 * kKVBytes), vb = kb + kKVBytes;
+            // S and dP of block j go to TMEM buffer j & 1 while the rows still work
+            // on block j - 1; dQ += dS K of block j - 1 follows once its dS is in.
+            for (int j = 0; ok && j <= nb; ++j) {
+                if (j < nb) {
+                    const int s = j & 1;
+                    if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t kb = smem_u32(smem + kDqOffKV + s * 2 * kKVBytes), vb = kb + kKVBytes;
 #pragma unroll
-                for (int k = 0; k < kD / 16; ++k) {
-                    const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
-                    const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
-                    umma_bf16(tmem + kTmemS, smem_desc_sw128(qb + oq, 16, 1024), smem_desc_sw128(kb + ok2, 16, 1024),
-                              IDESC_S, k > 0);
-                    umma_bf16(tmem + kTmemDP, smem_desc_sw128(gb + oq, 16, 1024), smem_desc_sw128(vb + ok2, 16, 1024),
-                              IDESC_S, k > 0);
+                    for (int k = 0; k < kD / 16; ++k) {
+                        const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                        const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+                        umma_bf16(tmem + kTmemS + s * 128, smem_desc_sw128(qb + oq, 16, 1024),
+                                  smem_desc_sw128(kb + ok2, 16, 1024), IDESC_S, k > 0);
+                        umma_bf16(tmem + kTmemDP + s * 128, smem_desc_sw128(gb + oq, 16, 1024),
+                                  smem_desc_sw128(vb + ok2, 16, 1024), IDESC_S, k > 0);
+                    }
+                    umma_commit(&ctl.sdp_full[s]);
                 }
-                umma_commit(&ctl.sdp_full);
-                // dS of block j is in TMEM buffer j & 1 once every row has written it
-                if (!mbar_wait(&ctl.ds_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
-                tc_fence_after();
+                if (j >= 1) {
+                    const int jp = j - 1, sp = jp & 1;
+                    // dS of block jp is in TMEM buffer sp once every row has written it
+                    if (!mbar_wait(&ctl.ds_full[sp], (jp >> 1) & 1, wc)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t kb = smem_u32(smem + kDqOffKV + sp * 2 * kKVBytes);
 #pragma unroll
-                for (int k = 0; k < kKeys / 16; ++k)
-                    umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + s * 32 + k * 8,
-                                 smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ, (j > 0 || k > 0) ? 1u : 0u);
-                umma_commit(&ctl.dq_done[s]);
-                umma_commit(&ctl.kv_empty[s]);
-                if (j + 2 < nb) {
-                    if (!mbar_wait(&ctl.kv_empty[s], (j >> 1) & 1, wc)) { ok = false; break; }
-                    load_kv(j + 2);
+                    for (int k = 0; k < kKeys / 16; ++k)
+                        umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + sp * 32 + k * 8,
+                                     smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ,
+                                     (jp > 0 || k > 0) ? 1u : 0u);
+                    umma_commit(&ctl.dq_done[sp]);
+                    umma_commit(&ctl.kv_empty[sp]);
+                    if (jp + 2 < nb) {
+                        if (!mbar_wait(&ctl.kv_empty[sp], (jp >> 1) & 1, wc)) { ok = false; break; }
+                        load_kv(jp + 2);
+                    }
                 }
             }
             umma_commit(&ctl.fin);
             mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
         }
     } else {
-        // ---- rows
-        const int r = t;                       // row of the tile = TMEM lane
+        // ---- rows: thread t takes row t % 128 (its TMEM lane) and keys
+        // 32 hk .. 32 hk + 31 of every block, hk = t / 128
+        const int r = t & (kRows - 1), hk = t >> 7;
         const int i = row0 + r;
         const bool valid = i < p.N;
         const int c = i >> 6;                  // the row's current block
-        const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+        const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
         const long long roff = static_cast<long long>(bh) * p.N + i;
         float delta = 0.f, lse2 = 0.f;
         if (valid) {
             delta = row_delta(p.O + roff * kD, p.dO + roff * kD);
             lse2 = __ldg(p.LSE + roff) * kLog2eB;
-            p.delta[roff] = delta;
+            if (hk == 0) p.delta[roff] = delta;
         }
         const int nsel = valid ? min(p.topk, c) : 0;
         const int32_t* my_idx = p.sel_idx + roff * p.topk;
         const float* my_lg = p.sel_logg + roff * p.topk;
-        float* my_dlg = p.dlogg + roff * p.topk;
+        float* my_dlg = p.dlogg + roff * p.topk;   // zeroed before this kernel; both halves add
         int e = 0;                             // next kept entry (ascending)
         int km = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
         float kl = nsel > 0 ? __ldg(my_lg) : 0.f;
@@ -232,16 +244,15 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                     lim = i & (kKeys - 1);
                 }
             }
-            if (!mbar_wait_warp(&ctl.sdp_full, j & 1, wc)) { ok = false; break; }
+            if (!mbar_wait_warp(&ctl.sdp_full[j & 1], (j >> 1) & 1, wc)) { ok = false; break; }
             // the dS buffer j & 1 is free once dQ of block j - 2 has read it
             if (j >= 2 && !mbar_wait_warp(&ctl.dq_done[j & 1], ((j - 2) >> 1) & 1, wc)) { ok = false; break; }
             tc_fence_after();
             float sum = 0.f;
-#pragma unroll
-            for (int hk = 0; hk < 2; ++hk) {
+            {
                 uint32_t sv[32], dv[32];
-                tmem_ld32(lane_addr + kTmemS + hk * 32, sv);
-                tmem_ld32(lane_addr + kTmemDP + hk * 32, dv);
+                tmem_ld32(lane_addr + kTmemS + (j & 1) * 128 + hk * 32, sv);
+                tmem_ld32(lane_addr + kTmemDP + (j & 1) * 128 + hk * 32, dv);
                 tmem_wait_ld();
                 uint32_t pk[16];
 #pragma unroll
@@ -263,20 +274,17 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             tc_fence_before();
             mbar_arrive(&ctl.ds_full[j & 1]);
             if (kept) {
-                my_dlg[e] = train ? sum : 0.f;   // no gates in the inference form
+                if (train) atomicAdd(my_dlg + e, sum);   // two halves: a + b, order-independent
                 ++e;
                 km = e < nsel ? __ldg(my_idx + e) : 0x7fffffff;
                 kl = e < nsel ? __ldg(my_lg + e) : 0.f;
             }
         }
-        // kept entries never visited cannot exist (every kept block is in the union);
-        // the rest of the row's dlogg slots (padding) are zero
-        if (valid)
-            for (int q = nsel; q < p.topk; ++q) my_dlg[q] = 0.f;
+        // dQ: columns 64 hk .. 64 hk + 63 of the row
         if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
             tc_fence_after();
 #pragma unroll 1
-            for (int cc = 0; cc < kD / 32; ++cc) {
+            for (int cc = 2 * hk; cc < 2 * hk + 2; ++cc) {
                 uint32_t o[32];
                 tmem_ld32(lane_addr + kTmemDQ + cc * 32, o);
                 tmem_wait_ld();
@@ -366,11 +374,14 @@ __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* uni
 // ------------------------------------------------------------------ pass 2
 
 struct DkvCtl {
-    uint64_t kv_full, q_full[2], q_empty[2], sdp_full, pds_full, half_done, fin;
+    uint64_t kv_full, q_full[2], q_empty[2], info_full[2], info_empty[2];
+    uint64_t sdp_full, sdp_free, pds_full, half_done, fin;
     uint32_t tmem_base;
     int abort_flag;
 };
 
+constexpr int kThreadsD = 224;                           // keys (4 warps), issuer, two row-info warps
+constexpr int kInfoLanes = 64;
 constexpr int kPairBytes = 2 * kKeys * kD * 2;           // 32 KB: K (or V) of the key pair
 constexpr int kDkvOffV = kPairBytes;
 constexpr int kDkvOffQ = 2 * kPairBytes;                 // 2 stages x (Q, dO) tiles
@@ -384,27 +395,61 @@ constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
 // TMEM: dV [0,128), dK [128,256), S^T [256,320), dP^T [320,384), P^T [384,416), dS^T [416,448)
 constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemST = 256, kTmemDPT = 320, kTmemPT = 384, kTmemDST = 416;
 
-// Bias (log2 units, or a marker) of block m for query row i: kept historical
+// Biases (log2 units, or markers) of blocks m and m+1 (m even) for query
+// rows ia and ib, with the two rows' searches interleaved: kept historical
 // block -> log g (training) or 0; the row's own block -> 0 with the causal
-// limit applied by the caller; otherwise -inf.
-__device__ __forceinline__ float row_block_bias(const BwdParams& p, int bh, int i, int m) {
-    if (i >= p.N) return -CUDART_INF_F;
-    const int c = i >> 6;
-    if (m > c) return -CUDART_INF_F;
-    if (m == c) return 0.f;
-    const int nsel = min(p.topk, c);
-    const long long roff = static_cast<long long>(bh) * p.N + i;
-    const int32_t* idx = p.sel_idx + roff * p.topk;
-    int lo = 0, hi = nsel;   // first entry >= m in the ascending kept list
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (__ldg(idx + mid) < m) lo = mid + 1; else hi = mid;
+// limit applied by the caller; otherwise -inf.  One search per row finds the
+// first kept entry >= m, so m+1 is the entry there or the next.
+__device__ __forceinline__ void pair_bias2(const BwdParams& p, int bh, int m, int ia, int ib, float (&ba)[2],
+                                           float (&bb)[2]) {
+    int lo[2] = {0, 0}, hi[2], c[2] = {ia >> 6, ib >> 6};
+    const int32_t* idx[2];
+    long long roff[2];
+    const int rows[2] = {ia, ib};
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const bool v = rows[r] < p.N;
+        roff[r] = static_cast<long long>(bh) * p.N + (v ? rows[r] : 0);
+        idx[r] = p.sel_idx + roff[r] * p.topk;
+        hi[r] = (v && m < c[r]) ? min(p.topk, c[r]) : 0;   // search only where block m is historical
     }
-    if (lo < nsel && __ldg(idx + lo) == m) return p.mode == 0 ? __ldg(p.sel_logg + roff * p.topk + lo) * kLog2eB : 0.f;
-    return -CUDART_INF_F;
+    while (lo[0] < hi[0] || lo[1] < hi[1]) {
+        int val[2];
+#pragma unroll
+        for (int r = 0; r < 2; ++r) val[r] = lo[r] < hi[r] ? __ldg(idx[r] + ((lo[r] + hi[r]) >> 1)) : 0;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            if (lo[r] < hi[r]) {
+                const int mid = (lo[r] + hi[r]) >> 1;
+                if (val[r] < m) lo[r] = mid + 1; else hi[r] = mid;
+            }
+        }
+    }
+    float* outs[2] = {ba, bb};
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int i = rows[r];
+        const int nsel = min(p.topk, c[r]);
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int mq = m + q;
+            float b = -CUDART_INF_F;
+            if (i < p.N) {
+                if (mq == c[r]) {
+                    b = 0.f;
+                } else if (mq < c[r]) {
+                    const int e = lo[r] + q;   // m at lo (if kept), m+1 at lo or lo+1
+                    for (int ee = lo[r]; ee <= e && ee < nsel; ++ee)
+                        if (__ldg(idx[r] + ee) == mq)
+                            b = p.mode == 0 ? __ldg(p.sel_logg + roff[r] * p.topk + ee) * kLog2eB : 0.f;
+                }
+            }
+            outs[r][q] = b;
+        }
+    }
 }
 
-__global__ void __launch_bounds__(kThreadsB, 1)
+__global__ void __launch_bounds__(kThreadsD, 1)
 bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
                const __grid_constant__ CUtensorMap mapK2, const __grid_constant__ CUtensorMap mapV2, BwdParams p) {
     extern __shared__ __align__(1024) uint8_t dsm[];
@@ -422,8 +467,11 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         for (int s = 0; s < 2; ++s) {
             mbar_init(&ctl.q_full[s], 1);
             mbar_init(&ctl.q_empty[s], 1);
+            mbar_init(&ctl.info_full[s], kInfoLanes);
+            mbar_init(&ctl.info_empty[s], kWorkers);
         }
         mbar_init(&ctl.sdp_full, 1);
+        mbar_init(&ctl.sdp_free, kWorkers);
         mbar_init(&ctl.pds_full, kWorkers);
         mbar_init(&ctl.half_done, 1);
         mbar_init(&ctl.fin, 1);
@@ -438,9 +486,9 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     // fixed summation order); rank sort of the inverted list in shared memory
     int* raw = list + kDkvListCap;
     if (t == 0) list[0] = pr;
-    for (int k = t; k < cnt; k += kThreadsB) raw[k] = __ldg(p.inv_tiles + off + k);
+    for (int k = t; k < cnt; k += kThreadsD) raw[k] = __ldg(p.inv_tiles + off + k);
     __syncthreads();
-    for (int k = t; k < cnt; k += kThreadsB) {
+    for (int k = t; k < cnt; k += kThreadsD) {
         const int v = raw[k];
         int rank = 0;
         for (int q = 0; q < cnt; ++q) rank += raw[q] < v;
@@ -452,10 +500,40 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     const uint32_t tmem = ctl.tmem_base;
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
     float* info = reinterpret_cast<float*>(smem + kDkvOffInfo);
+    const int nh = 2 * nq;   // 64-row halves of the query tiles
 
-    if (warp == 4) {
+    if (warp >= 5) {
+        // ---- row information of query tile q (LSE, Delta, bias of both blocks),
+        // one tile ahead of the key threads; two rows per lane, searched together
+        const int il = t - 5 * 32;   // 0 .. 63
+        for (int q = 0; q < nq; ++q) {
+            const int s = q & 1;
+            if (q >= 2 && !mbar_wait(&ctl.info_empty[s], ((q - 2) >> 1) & 1, wc)) break;
+            float* inf = info + s * 4 * kRows;
+            const int tq = list[q];
+            const int ra = il, rb = il + kInfoLanes;
+            const int ia = tq * kRows + ra, ib = tq * kRows + rb;
+            const long long oa = static_cast<long long>(bh) * p.N + ia, ob = static_cast<long long>(bh) * p.N + ib;
+            const float la = ia < p.N ? __ldg(p.LSE + oa) * kLog2eB : 0.f;
+            const float lb = ib < p.N ? __ldg(p.LSE + ob) * kLog2eB : 0.f;
+            const float da = ia < p.N ? p.delta[oa] : 0.f;
+            const float db = ib < p.N ? p.delta[ob] : 0.f;
+            float ba[2], bb[2];
+            pair_bias2(p, bh, 2 * pr, ia, ib, ba, bb);
+            inf[ra] = la;
+            inf[rb] = lb;
+            inf[kRows + ra] = da;
+            inf[kRows + rb] = db;
+            inf[2 * kRows + ra] = ba[0];
+            inf[2 * kRows + rb] = bb[0];
+            inf[3 * kRows + ra] = ba[1];
+            inf[3 * kRows + rb] = bb[1];
+            mbar_arrive(&ctl.info_full[s]);
+        }
+    } else if (warp == 4) {
         if (lane == 0) {
-            // ---- issuer
+            // ---- issuer: S^T, dP^T of half x+1 go in as soon as the keys have read
+            // those of half x; dV, dK of half x once its P^T, dS^T are written
             mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
             for (int h = 0; h < 2; ++h) {
                 tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
@@ -477,42 +555,48 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
             const uint32_t kb = smem_u32(smem), vb = smem_u32(smem + kDkvOffV);
             bool ok = mbar_wait(&ctl.kv_full, 0, wc);
-            int hs = 0;   // halves issued so far
-            for (int q = 0; ok && q < nq; ++q) {
-                const int s = q & 1;
-                if (!mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc)) { ok = false; break; }
+            auto issue_sdp = [&](int x) -> bool {
+                const int q = x >> 1, h = x & 1, s = q & 1;
+                if (h == 0 && !mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc)) return false;
+                tc_fence_after();
                 const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
-                for (int h = 0; h < 2; ++h, ++hs) {
-                    tc_fence_after();
 #pragma unroll
-                    for (int k = 0; k < kD / 16; ++k) {
-                        const uint32_t ok2 = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
-                        const uint32_t oq = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
-                        umma_bf16(tmem + kTmemST, smem_desc_sw128(kb + ok2, 16, 1024), smem_desc_sw128(qb + oq, 16, 1024),
-                                  IDESC_T, k > 0);
-                        umma_bf16(tmem + kTmemDPT, smem_desc_sw128(vb + ok2, 16, 1024), smem_desc_sw128(gb + oq, 16, 1024),
-                                  IDESC_T, k > 0);
-                    }
-                    umma_commit(&ctl.sdp_full);
-                    if (!mbar_wait(&ctl.pds_full, hs & 1, wc)) { ok = false; break; }
-                    tc_fence_after();
-#pragma unroll
-                    for (int k = 0; k < 64 / 16; ++k) {
-                        // B = dO (or Q) rows of this half, MN-major: 16 rows = two 8-row atoms
-                        const uint32_t ob = h * 64 * 128 + k * 2048;
-                        const uint32_t acc = (q > 0 || h > 0 || k > 0) ? 1u : 0u;
-                        umma_bf16_ta(tmem + kTmemDV, tmem + kTmemPT + k * 8, smem_desc_sw128(gb + ob, kRows * 128, 1024),
-                                     IDESC_ACC, acc);
-                        umma_bf16_ta(tmem + kTmemDK, tmem + kTmemDST + k * 8, smem_desc_sw128(qb + ob, kRows * 128, 1024),
-                                     IDESC_ACC, acc);
-                    }
-                    umma_commit(&ctl.half_done);
+                for (int k = 0; k < kD / 16; ++k) {
+                    const uint32_t ok2 = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
+                    const uint32_t oq = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
+                    umma_bf16(tmem + kTmemST, smem_desc_sw128(kb + ok2, 16, 1024), smem_desc_sw128(qb + oq, 16, 1024),
+                              IDESC_T, k > 0);
+                    umma_bf16(tmem + kTmemDPT, smem_desc_sw128(vb + ok2, 16, 1024), smem_desc_sw128(gb + oq, 16, 1024),
+                              IDESC_T, k > 0);
                 }
-                if (!ok) break;
-                umma_commit(&ctl.q_empty[s]);
-                if (q + 2 < nq) {
-                    if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc)) { ok = false; break; }
-                    load_q(q + 2);
+                umma_commit(&ctl.sdp_full);
+                return true;
+            };
+            if (ok) ok = issue_sdp(0);
+            for (int x = 0; ok && x < nh; ++x) {
+                const int q = x >> 1, h = x & 1, s = q & 1;
+                if (!mbar_wait(&ctl.sdp_free, x & 1, wc)) { ok = false; break; }
+                if (x + 1 < nh && !issue_sdp(x + 1)) { ok = false; break; }
+                if (!mbar_wait(&ctl.pds_full, x & 1, wc)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
+#pragma unroll
+                for (int k = 0; k < 64 / 16; ++k) {
+                    // B = dO (or Q) rows of this half, MN-major: 16 rows = two 8-row atoms
+                    const uint32_t ob = h * 64 * 128 + k * 2048;
+                    const uint32_t acc = (x > 0 || k > 0) ? 1u : 0u;
+                    umma_bf16_ta(tmem + kTmemDV, tmem + kTmemPT + k * 8, smem_desc_sw128(gb + ob, kRows * 128, 1024),
+                                 IDESC_ACC, acc);
+                    umma_bf16_ta(tmem + kTmemDK, tmem + kTmemDST + k * 8, smem_desc_sw128(qb + ob, kRows * 128, 1024),
+                                 IDESC_ACC, acc);
+                }
+                umma_commit(&ctl.half_done);
+                if (h == 1) {
+                    umma_commit(&ctl.q_empty[s]);
+                    if (q + 2 < nq) {
+                        if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc)) { ok = false; break; }
+                        load_q(q + 2);
+                    }
                 }
             }
             umma_commit(&ctl.fin);
@@ -525,61 +609,49 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         const int kblk = key >> 6;                // 0: block 2pr, 1: block 2pr + 1
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
         bool ok = true;
-        int hs = 0;
-        for (int q = 0; q < nq; ++q) {
-            const int s = q & 1;
+        for (int x = 0; x < nh; ++x) {
+            const int q = x >> 1, h = x & 1, s = q & 1;
             const int tq = list[q];
-            float* inf = info + s * 4 * kRows;
-            // per-row data of this query tile (thread = row for this part); the
-            // buffer s was last read two tiles ago, before that tile's last pds_full
-            {
-                const int i = tq * kRows + t;
-                const long long roff = static_cast<long long>(bh) * p.N + i;
-                const bool v = i < p.N;
-                inf[t] = v ? __ldg(p.LSE + roff) * kLog2eB : 0.f;
-                inf[kRows + t] = v ? p.delta[roff] : 0.f;
-                inf[2 * kRows + t] = row_block_bias(p, bh, i, 2 * pr);
-                inf[3 * kRows + t] = row_block_bias(p, bh, i, 2 * pr + 1);
-            }
-            named_bar_sync(1, kWorkers);
-            for (int h = 0; h < 2; ++h, ++hs) {
-                if (!mbar_wait_warp(&ctl.sdp_full, hs & 1, wc)) { ok = false; break; }
-                // P^T / dS^T columns are free once the previous half's products have read them
-                if (hs >= 1 && !mbar_wait_warp(&ctl.half_done, (hs - 1) & 1, wc)) { ok = false; break; }
-                tc_fence_after();
+            const float* inf = info + s * 4 * kRows;
+            if (h == 0 && !mbar_wait_warp(&ctl.info_full[s], (q >> 1) & 1, wc)) { ok = false; break; }
+            if (!mbar_wait_warp(&ctl.sdp_full, x & 1, wc)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t sv[64], dv[64];
+            tmem_ld32(lane_addr + kTmemST, *reinterpret_cast<uint32_t(*)[32]>(sv));
+            tmem_ld32(lane_addr + kTmemST + 32, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
+            tmem_ld32(lane_addr + kTmemDPT, *reinterpret_cast<uint32_t(*)[32]>(dv));
+            tmem_ld32(lane_addr + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
+            tmem_wait_ld();
+            tc_fence_before();
+            mbar_arrive(&ctl.sdp_free);   // S^T, dP^T may be overwritten by the next half
+            uint32_t pp[32], dd[32];
 #pragma unroll
-                for (int hr = 0; hr < 2; ++hr) {
-                    uint32_t sv[32], dv[32];
-                    tmem_ld32(lane_addr + kTmemST + hr * 32, sv);
-                    tmem_ld32(lane_addr + kTmemDPT + hr * 32, dv);
-                    tmem_wait_ld();
-                    uint32_t pp[16], dd[16];
+            for (int k = 0; k < 64; k += 2) {
+                float pv[2], dsv[2];
 #pragma unroll
-                    for (int k = 0; k < 32; k += 2) {
-                        float pv[2], dsv[2];
-#pragma unroll
-                        for (int u = 0; u < 2; ++u) {
-                            const int rr = h * 64 + hr * 32 + k + u;        // row of the query tile
-                            const int i = tq * kRows + rr;
-                            const float bias = inf[(2 + kblk) * kRows + rr];
-                            // the row's own block: causal (key <= row); -inf bias: not attended
-                            const bool vis = bias != -CUDART_INF_F && (kg >> 6 != i >> 6 || kg <= i);
-                            const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
-                            const float pr_ = vis ? fast_exp2(z - inf[rr]) : 0.f;
-                            pv[u] = pr_;
-                            dsv[u] = pr_ * (__uint_as_float(dv[k + u]) - inf[kRows + rr]);
-                        }
-                        pp[k >> 1] = pack_bf16x2(pv[0], pv[1]);
-                        dd[k >> 1] = pack_bf16x2(dsv[0], dsv[1]);
-                    }
-                    tmem_st16(lane_addr + kTmemPT + hr * 16, pp);
-                    tmem_st16(lane_addr + kTmemDST + hr * 16, dd);
+                for (int u = 0; u < 2; ++u) {
+                    const int rr = h * 64 + k + u;        // row of the query tile
+                    const int i = tq * kRows + rr;
+                    const float bias = inf[(2 + kblk) * kRows + rr];
+                    // the row's own block: causal (key <= row); -inf bias: not attended
+                    const bool vis = bias != -CUDART_INF_F && (kg >> 6 != i >> 6 || kg <= i);
+                    const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
+                    const float pr_ = vis ? fast_exp2(z - inf[rr]) : 0.f;
+                    pv[u] = pr_;
+                    dsv[u] = pr_ * (__uint_as_float(dv[k + u]) - inf[kRows + rr]);
                 }
-                tmem_wait_st();
-                tc_fence_before();
-                mbar_arrive(&ctl.pds_full);
+                pp[k >> 1] = pack_bf16x2(pv[0], pv[1]);
+                dd[k >> 1] = pack_bf16x2(dsv[0], dsv[1]);
             }
-            if (!ok) break;
+            // P^T / dS^T columns are free once the previous half's products have read them
+            if (x >= 1 && !mbar_wait_warp(&ctl.half_done, (x - 1) & 1, wc)) { ok = false; break; }
+            tc_fence_after();
+            tmem_st32(lane_addr + kTmemPT, pp);
+            tmem_st32(lane_addr + kTmemDST, dd);
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(&ctl.pds_full);
+            if (h == 1) mbar_arrive(&ctl.info_empty[s]);
         }
         if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
             tc_fence_after();
@@ -696,7 +768,10 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     p.limit = env.limit;
     const long long tiles = static_cast<long long>(a.BH) * a.T;
     if (tiles > 0x7fffffffLL) { *err = "backward: too many tiles"; return cudaErrorInvalidValue; }
-    // pass 1 (also writes Delta for pass 2)
+    // pass 1 (also writes Delta for pass 2); both halves of a row add into dlogg
+    cudaError_t e0 = cudaMemsetAsync(a.dlogg, 0, static_cast<size_t>(a.BH) * a.N * (a.topk > 0 ? a.topk : 1) * 4,
+                                     env.stream);
+    if (e0 != cudaSuccess) { *err = "backward dlogg"; return e0; }
     bwd_dq_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
@@ -710,7 +785,7 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
     // pass 2
-    bwd_dkv_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+    bwd_dkv_kernel<<<static_cast<unsigned>(tiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
