@@ -33,6 +33,10 @@ constexpr int kWorkers = 128;       // key threads (pass 2)
 constexpr int kRowThreads = 256;    // pass 1: two threads per row, 32 keys of a block each
 constexpr int kThreadsB = 288;      // + the issuing warp
 constexpr float kLog2eB = 1.4426950408889634f;
+// Waiting threads sleep (woken when the phase completes) instead of spinning:
+// the issuing and row-information warps wait most of the time and would
+// otherwise take issue slots from the row / key warps.
+constexpr uint32_t kSleepNs = 1000;
 
 __device__ __forceinline__ float bfl(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bfh(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -162,13 +166,13 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
             constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
             const uint32_t qb = smem_u32(smem), gb = smem_u32(smem + kDqOffDO);
-            bool ok = mbar_wait(&ctl.q_full, 0, wc);
+            bool ok = mbar_wait(&ctl.q_full, 0, wc, kSleepNs);
             // S and dP of block j go to TMEM buffer j & 1 while the rows still work
             // on block j - 1; dQ += dS K of block j - 1 follows once its dS is in.
             for (int j = 0; ok && j <= nb; ++j) {
                 if (j < nb) {
                     const int s = j & 1;
-                    if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc)) { ok = false; break; }
+                    if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t kb = smem_u32(smem + kDqOffKV + s * 2 * kKVBytes), vb = kb + kKVBytes;
 #pragma unroll
@@ -185,7 +189,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 if (j >= 1) {
                     const int jp = j - 1, sp = jp & 1;
                     // dS of block jp is in TMEM buffer sp once every row has written it
-                    if (!mbar_wait(&ctl.ds_full[sp], (jp >> 1) & 1, wc)) { ok = false; break; }
+                    if (!mbar_wait(&ctl.ds_full[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t kb = smem_u32(smem + kDqOffKV + sp * 2 * kKVBytes);
 #pragma unroll
@@ -196,7 +200,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                     umma_commit(&ctl.dq_done[sp]);
                     umma_commit(&ctl.kv_empty[sp]);
                     if (jp + 2 < nb) {
-                        if (!mbar_wait(&ctl.kv_empty[sp], (jp >> 1) & 1, wc)) { ok = false; break; }
+                        if (!mbar_wait(&ctl.kv_empty[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                         load_kv(jp + 2);
                     }
                 }
@@ -244,9 +248,9 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                     lim = i & (kKeys - 1);
                 }
             }
-            if (!mbar_wait_warp(&ctl.sdp_full[j & 1], (j >> 1) & 1, wc)) { ok = false; break; }
+            if (!mbar_wait_warp(&ctl.sdp_full[j & 1], (j >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
             // the dS buffer j & 1 is free once dQ of block j - 2 has read it
-            if (j >= 2 && !mbar_wait_warp(&ctl.dq_done[j & 1], ((j - 2) >> 1) & 1, wc)) { ok = false; break; }
+            if (j >= 2 && !mbar_wait_warp(&ctl.dq_done[j & 1], ((j - 2) >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
             tc_fence_after();
             float sum = 0.f;
             {
@@ -254,20 +258,33 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 tmem_ld32(lane_addr + kTmemS + (j & 1) * 128 + hk * 32, sv);
                 tmem_ld32(lane_addr + kTmemDP + (j & 1) * 128 + hk * 32, dv);
                 tmem_wait_ld();
+                // P = exp2(S scale + (log g - LSE)) in log2 units; exp2(-inf) = 0 for a
+                // block the row does not attend; the causal limit only on its own block
+                const float boff = lim >= 0 ? bias - lse2 : -CUDART_INF_F;
+                const bool causal = lim >= 0 && lim < kKeys - 1;
+                const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2), bo2 = f32x2(boff, boff);
+                const uint64_t nd2 = f32x2(-delta, -delta);
+                uint64_t acc = 0;
                 uint32_t pk[16];
 #pragma unroll
                 for (int k = 0; k < 32; k += 2) {
-                    float ds2[2];
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const int key = hk * 32 + k + u;
-                        const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
-                        const float pr = key <= lim ? fast_exp2(z - lse2) : 0.f;
-                        ds2[u] = pr * (__uint_as_float(dv[k + u]) - delta);
-                        sum += ds2[u];
+                    float z0, z1;
+                    f32x2_split(fma_f32x2(f32x2(__uint_as_float(sv[k]), __uint_as_float(sv[k + 1])), sc2, bo2), z0, z1);
+                    float p0 = fast_exp2(z0), p1 = fast_exp2(z1);
+                    if (causal) {
+                        p0 = hk * 32 + k <= lim ? p0 : 0.f;
+                        p1 = hk * 32 + k + 1 <= lim ? p1 : 0.f;
                     }
-                    pk[k >> 1] = pack_bf16x2(ds2[0], ds2[1]);
+                    const uint64_t d2 = add_f32x2(f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1])), nd2);
+                    const uint64_t ds2 = fma_f32x2(f32x2(p0, p1), d2, 0ull);
+                    acc = add_f32x2(acc, ds2);
+                    float a0, a1;
+                    f32x2_split(ds2, a0, a1);
+                    pk[k >> 1] = pack_bf16x2(a0, a1);
                 }
+                float s0, s1;
+                f32x2_split(acc, s0, s1);
+                sum = s0 + s1;
                 tmem_st16(lane_addr + kTmemDS + (j & 1) * 32 + hk * 16, pk);
             }
             tmem_wait_st();
@@ -281,7 +298,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             }
         }
         // dQ: columns 64 hk .. 64 hk + 63 of the row
-        if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
+        if (ok && mbar_wait_warp(&ctl.fin, 0, wc, kSleepNs)) {
             tc_fence_after();
 #pragma unroll 1
             for (int cc = 2 * hk; cc < 2 * hk + 2; ++cc) {
@@ -374,7 +391,7 @@ __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* uni
 // ------------------------------------------------------------------ pass 2
 
 struct DkvCtl {
-    uint64_t kv_full, q_full[2], q_empty[2], info_full[2], info_empty[2];
+    uint64_t kv_full, q_full[2], q_empty[2], info_full[4], info_empty[4];
     uint64_t sdp_full, sdp_free, pds_full, half_done, fin;
     uint32_t tmem_base;
     int abort_flag;
@@ -385,8 +402,9 @@ constexpr int kInfoLanes = 64;
 constexpr int kPairBytes = 2 * kKeys * kD * 2;           // 32 KB: K (or V) of the key pair
 constexpr int kDkvOffV = kPairBytes;
 constexpr int kDkvOffQ = 2 * kPairBytes;                 // 2 stages x (Q, dO) tiles
-constexpr int kDkvOffInfo = kDkvOffQ + 2 * 2 * kQBytes;  // 2 stages x [4][128] floats: lse2, delta, bias0, bias1
-constexpr int kDkvOffList = kDkvOffInfo + 2 * 4 * kRows * 4;
+constexpr int kInfoStages = 4;                           // row information computed up to 3 tiles ahead
+constexpr int kDkvOffInfo = kDkvOffQ + 2 * 2 * kQBytes;  // stages x [4][128] floats: lse2, delta, bias0, bias1
+constexpr int kDkvOffList = kDkvOffInfo + kInfoStages * 4 * kRows * 4;
 // query tiles of a key pair (sorted list, then the unsorted copy); the host
 // refuses heads of more than kBwdMaxTiles tiles
 constexpr int kDkvListCap = 2048;
@@ -467,6 +485,8 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         for (int s = 0; s < 2; ++s) {
             mbar_init(&ctl.q_full[s], 1);
             mbar_init(&ctl.q_empty[s], 1);
+        }
+        for (int s = 0; s < kInfoStages; ++s) {
             mbar_init(&ctl.info_full[s], kInfoLanes);
             mbar_init(&ctl.info_empty[s], kWorkers);
         }
@@ -507,8 +527,9 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         // one tile ahead of the key threads; two rows per lane, searched together
         const int il = t - 5 * 32;   // 0 .. 63
         for (int q = 0; q < nq; ++q) {
-            const int s = q & 1;
-            if (q >= 2 && !mbar_wait(&ctl.info_empty[s], ((q - 2) >> 1) & 1, wc)) break;
+            const int s = q % kInfoStages;
+            if (q >= kInfoStages && !mbar_wait(&ctl.info_empty[s], ((q - kInfoStages) / kInfoStages) & 1, wc, kSleepNs))
+                break;
             float* inf = info + s * 4 * kRows;
             const int tq = list[q];
             const int ra = il, rb = il + kInfoLanes;
@@ -520,14 +541,14 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             const float db = ib < p.N ? p.delta[ob] : 0.f;
             float ba[2], bb[2];
             pair_bias2(p, bh, 2 * pr, ia, ib, ba, bb);
-            inf[ra] = la;
-            inf[rb] = lb;
-            inf[kRows + ra] = da;
-            inf[kRows + rb] = db;
-            inf[2 * kRows + ra] = ba[0];
-            inf[2 * kRows + rb] = bb[0];
-            inf[3 * kRows + ra] = ba[1];
-            inf[3 * kRows + rb] = bb[1];
+            // per block: log g - LSE (log2 units), -inf where the row does not attend;
+            // then -Delta
+            inf[ra] = ba[0] - la;
+            inf[rb] = bb[0] - lb;
+            inf[kRows + ra] = ba[1] - la;
+            inf[kRows + rb] = bb[1] - lb;
+            inf[2 * kRows + ra] = -da;
+            inf[2 * kRows + rb] = -db;
             mbar_arrive(&ctl.info_full[s]);
         }
     } else if (warp == 4) {
@@ -554,10 +575,10 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             constexpr uint32_t IDESC_T = idesc_bf16(2 * kKeys, 64, 0, 0);   // M = 128 keys, N = 64 rows
             constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
             const uint32_t kb = smem_u32(smem), vb = smem_u32(smem + kDkvOffV);
-            bool ok = mbar_wait(&ctl.kv_full, 0, wc);
+            bool ok = mbar_wait(&ctl.kv_full, 0, wc, kSleepNs);
             auto issue_sdp = [&](int x) -> bool {
                 const int q = x >> 1, h = x & 1, s = q & 1;
-                if (h == 0 && !mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc)) return false;
+                if (h == 0 && !mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc, kSleepNs)) return false;
                 tc_fence_after();
                 const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
 #pragma unroll
@@ -575,9 +596,9 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             if (ok) ok = issue_sdp(0);
             for (int x = 0; ok && x < nh; ++x) {
                 const int q = x >> 1, h = x & 1, s = q & 1;
-                if (!mbar_wait(&ctl.sdp_free, x & 1, wc)) { ok = false; break; }
+                if (!mbar_wait(&ctl.sdp_free, x & 1, wc, kSleepNs)) { ok = false; break; }
                 if (x + 1 < nh && !issue_sdp(x + 1)) { ok = false; break; }
-                if (!mbar_wait(&ctl.pds_full, x & 1, wc)) { ok = false; break; }
+                if (!mbar_wait(&ctl.pds_full, x & 1, wc, kSleepNs)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
 #pragma unroll
@@ -594,7 +615,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 if (h == 1) {
                     umma_commit(&ctl.q_empty[s]);
                     if (q + 2 < nq) {
-                        if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc)) { ok = false; break; }
+                        if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                         load_q(q + 2);
                     }
                 }
@@ -610,11 +631,11 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
         bool ok = true;
         for (int x = 0; x < nh; ++x) {
-            const int q = x >> 1, h = x & 1, s = q & 1;
+            const int q = x >> 1, h = x & 1, si = q % kInfoStages;
             const int tq = list[q];
-            const float* inf = info + s * 4 * kRows;
-            if (h == 0 && !mbar_wait_warp(&ctl.info_full[s], (q >> 1) & 1, wc)) { ok = false; break; }
-            if (!mbar_wait_warp(&ctl.sdp_full, x & 1, wc)) { ok = false; break; }
+            const float* inf = info + si * 4 * kRows;
+            if (h == 0 && !mbar_wait_warp(&ctl.info_full[si], (q / kInfoStages) & 1, wc, kSleepNs)) { ok = false; break; }
+            if (!mbar_wait_warp(&ctl.sdp_full, x & 1, wc, kSleepNs)) { ok = false; break; }
             tc_fence_after();
             uint32_t sv[64], dv[64];
             tmem_ld32(lane_addr + kTmemST, *reinterpret_cast<uint32_t(*)[32]>(sv));
@@ -625,35 +646,41 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             tc_fence_before();
             mbar_arrive(&ctl.sdp_free);   // S^T, dP^T may be overwritten by the next half
             uint32_t pp[32], dd[32];
+            // In the diagonal tile (the first of the list) the rows of half h have
+            // block 2pr + h as their own block: keys of that block are causal.
+            const bool causal = q == 0 && h == kblk;
+            const float2* off2 = reinterpret_cast<const float2*>(inf + kblk * kRows + h * 64);
+            const float2* nd2p = reinterpret_cast<const float2*>(inf + 2 * kRows + h * 64);
+            const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2);
+            const int kin = key & 63;
 #pragma unroll
             for (int k = 0; k < 64; k += 2) {
-                float pv[2], dsv[2];
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const int rr = h * 64 + k + u;        // row of the query tile
-                    const int i = tq * kRows + rr;
-                    const float bias = inf[(2 + kblk) * kRows + rr];
-                    // the row's own block: causal (key <= row); -inf bias: not attended
-                    const bool vis = bias != -CUDART_INF_F && (kg >> 6 != i >> 6 || kg <= i);
-                    const float z = fmaf(__uint_as_float(sv[k + u]), p.scale_log2, bias);
-                    const float pr_ = vis ? fast_exp2(z - inf[rr]) : 0.f;
-                    pv[u] = pr_;
-                    dsv[u] = pr_ * (__uint_as_float(dv[k + u]) - inf[kRows + rr]);
+                const float2 o = off2[k >> 1], nd = nd2p[k >> 1];
+                float z0, z1;
+                f32x2_split(fma_f32x2(f32x2(__uint_as_float(sv[k]), __uint_as_float(sv[k + 1])), sc2, f32x2(o.x, o.y)),
+                            z0, z1);
+                float p0 = fast_exp2(z0), p1 = fast_exp2(z1);
+                if (causal) {
+                    p0 = kin <= k ? p0 : 0.f;
+                    p1 = kin <= k + 1 ? p1 : 0.f;
                 }
-                pp[k >> 1] = pack_bf16x2(pv[0], pv[1]);
-                dd[k >> 1] = pack_bf16x2(dsv[0], dsv[1]);
+                const uint64_t d2 = add_f32x2(f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1])), f32x2(nd.x, nd.y));
+                float a0, a1;
+                f32x2_split(fma_f32x2(f32x2(p0, p1), d2, 0ull), a0, a1);
+                pp[k >> 1] = pack_bf16x2(p0, p1);
+                dd[k >> 1] = pack_bf16x2(a0, a1);
             }
             // P^T / dS^T columns are free once the previous half's products have read them
-            if (x >= 1 && !mbar_wait_warp(&ctl.half_done, (x - 1) & 1, wc)) { ok = false; break; }
+            if (x >= 1 && !mbar_wait_warp(&ctl.half_done, (x - 1) & 1, wc, kSleepNs)) { ok = false; break; }
             tc_fence_after();
             tmem_st32(lane_addr + kTmemPT, pp);
             tmem_st32(lane_addr + kTmemDST, dd);
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(&ctl.pds_full);
-            if (h == 1) mbar_arrive(&ctl.info_empty[s]);
+            if (h == 1) mbar_arrive(&ctl.info_empty[si]);
         }
-        if (ok && mbar_wait_warp(&ctl.fin, 0, wc)) {
+        if (ok && mbar_wait_warp(&ctl.fin, 0, wc, kSleepNs)) {
             tc_fence_after();
             const bool kv = kg < p.N;
             const long long koff = static_cast<long long>(bh) * p.N + kg;
