@@ -31,7 +31,7 @@ constexpr int kKeys = 64;           // keys per block
 constexpr int kD = 128;             // head dim
 constexpr int kWorkers = 128;       // key threads (pass 2)
 constexpr int kRowThreads = 256;    // pass 1: two threads per row, 32 keys of a block each
-constexpr int kThreadsB = 288;      // + the issuing warp
+constexpr int kThreadsB = 320;      // + two issuing warps (one tcgen05.mma issue takes ~90 cycles)
 constexpr float kLog2eB = 1.4426950408889634f;
 // Waiting threads sleep (woken when the phase completes) instead of spinning:
 // the issuing and row-information warps wait most of the time and would
@@ -70,7 +70,7 @@ __device__ __forceinline__ float row_delta(const bf16* O, const bf16* dO) {
 // ------------------------------------------------------------------ pass 1
 
 struct DqCtl {
-    uint64_t q_full, kv_full[2], kv_empty[2], sdp_full[2], ds_full[2], dq_done[2], fin;
+    uint64_t q_full, kv_full[4], kv_empty[4], sdp_full[2], ds_full[2], dq_done[2], fin;
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -78,8 +78,11 @@ struct DqCtl {
 constexpr int kQBytes = kRows * kD * 2;                 // 32 KB
 constexpr int kKVBytes = kKeys * kD * 2;                // 16 KB
 constexpr int kDqOffDO = kQBytes;
-constexpr int kDqOffKV = 2 * kQBytes;                   // 2 stages x (K, V)
-constexpr int kDqOffCtl = kDqOffKV + 2 * 2 * kKVBytes;
+// K, V ring: the load of block j + 4 goes out once dQ of block j has read K, so
+// three blocks of loads are in flight behind the one being multiplied
+constexpr int kKvStages = 4;
+constexpr int kDqOffKV = 2 * kQBytes;                   // kKvStages x (K, V)
+constexpr int kDqOffCtl = kDqOffKV + kKvStages * 2 * kKVBytes;
 constexpr int kDqSmem = kDqOffCtl + 256 + 1024;         // + alignment slack
 // TMEM: dQ [0,128); S and dP of block j in buffer j & 1: S [128 + 128 b, +64),
 // dP [192 + 128 b, +64); dS buffers [384,416), [416,448)
@@ -120,14 +123,16 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     const int nb = U + ((2 * tile + 1 < p.C) ? 2 : 1);   // visited blocks: union, then the diagonal ones
     if (t == 0) {
         mbar_init(&ctl.q_full, 1);
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < kKvStages; ++s) {
             mbar_init(&ctl.kv_full[s], 1);
-            mbar_init(&ctl.kv_empty[s], 1);
+            mbar_init(&ctl.kv_empty[s], 2);   // dQ (reads K) and dP (reads V)
+        }
+        for (int s = 0; s < 2; ++s) {
             mbar_init(&ctl.ds_full[s], kRowThreads);
             mbar_init(&ctl.dq_done[s], 1);
-            mbar_init(&ctl.sdp_full[s], 1);
+            mbar_init(&ctl.sdp_full[s], 2);   // S from one issuer, dP from the other
         }
-        mbar_init(&ctl.fin, 1);
+        mbar_init(&ctl.fin, 2);
         ctl.abort_flag = 0;
         fence_barrier_init();
     }
@@ -152,7 +157,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 tma_load_3d(smem + kDqOffDO + h * (kRows * 128), &mapDO, &ctl.q_full, h * 64, row0, bh);
             }
             auto load_kv = [&](int j) {
-                const int s = j & 1;
+                const int s = j % kKvStages;
                 const int m = block_at(j);
                 uint8_t* st = smem + kDqOffKV + s * 2 * kKVBytes;
                 mbar_arrive_expect_tx(&ctl.kv_full[s], 2 * kKVBytes);
@@ -161,8 +166,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                     tma_load_3d(st + kKVBytes + h * (kKeys * 128), &mapV, &ctl.kv_full[s], h * 64, m * kKeys, bh);
                 }
             };
-            load_kv(0);
-            if (nb > 1) load_kv(1);
+            for (int j = 0; j < kKvStages && j < nb; ++j) load_kv(j);
             constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
             constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
             const uint32_t qb = smem_u32(smem), gb = smem_u32(smem + kDqOffDO);
@@ -171,39 +175,63 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             // on block j - 1; dQ += dS K of block j - 1 follows once its dS is in.
             for (int j = 0; ok && j <= nb; ++j) {
                 if (j < nb) {
-                    const int s = j & 1;
-                    if (!mbar_wait(&ctl.kv_full[s], (j >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
+                    const int s = j & 1, ks = j % kKvStages;
+                    if (!mbar_wait(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t kb = smem_u32(smem + kDqOffKV + s * 2 * kKVBytes), vb = kb + kKVBytes;
+                    const uint32_t kb = smem_u32(smem + kDqOffKV + ks * 2 * kKVBytes);
 #pragma unroll
                     for (int k = 0; k < kD / 16; ++k) {
                         const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
                         const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
                         umma_bf16(tmem + kTmemS + s * 128, smem_desc_sw128(qb + oq, 16, 1024),
                                   smem_desc_sw128(kb + ok2, 16, 1024), IDESC_S, k > 0);
-                        umma_bf16(tmem + kTmemDP + s * 128, smem_desc_sw128(gb + oq, 16, 1024),
-                                  smem_desc_sw128(vb + ok2, 16, 1024), IDESC_S, k > 0);
                     }
                     umma_commit(&ctl.sdp_full[s]);
                 }
                 if (j >= 1) {
-                    const int jp = j - 1, sp = jp & 1;
+                    const int jp = j - 1, sp = jp & 1, kp = jp % kKvStages;
                     // dS of block jp is in TMEM buffer sp once every row has written it
                     if (!mbar_wait(&ctl.ds_full[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t kb = smem_u32(smem + kDqOffKV + sp * 2 * kKVBytes);
+                    const uint32_t kb = smem_u32(smem + kDqOffKV + kp * 2 * kKVBytes);
 #pragma unroll
                     for (int k = 0; k < kKeys / 16; ++k)
                         umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + sp * 32 + k * 8,
                                      smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ,
                                      (jp > 0 || k > 0) ? 1u : 0u);
                     umma_commit(&ctl.dq_done[sp]);
-                    umma_commit(&ctl.kv_empty[sp]);
-                    if (jp + 2 < nb) {
-                        if (!mbar_wait(&ctl.kv_empty[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
-                        load_kv(jp + 2);
+                    umma_commit(&ctl.kv_empty[kp]);
+                    if (jp + kKvStages < nb) {
+                        if (!mbar_wait(&ctl.kv_empty[kp], (jp / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
+                        load_kv(jp + kKvStages);
                     }
                 }
+            }
+            umma_commit(&ctl.fin);
+            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+        }
+    } else if (warp == 9) {
+        if (lane == 0) {
+            // ---- second issuer: dP = dO V^T of every block into TMEM buffer j & 1,
+            // once the rows are done with block j - 2 (which used that buffer)
+            constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
+            const uint32_t gb = smem_u32(smem + kDqOffDO);
+            bool ok = mbar_wait(&ctl.q_full, 0, wc, kSleepNs);
+            for (int j = 0; ok && j < nb; ++j) {
+                const int s = j & 1, ks = j % kKvStages;
+                if (!mbar_wait(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
+                if (j >= 2 && !mbar_wait(&ctl.ds_full[s], ((j - 2) >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t vb = smem_u32(smem + kDqOffKV + ks * 2 * kKVBytes) + kKVBytes;
+#pragma unroll
+                for (int k = 0; k < kD / 16; ++k) {
+                    const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                    const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+                    umma_bf16(tmem + kTmemDP + s * 128, smem_desc_sw128(gb + oq, 16, 1024),
+                              smem_desc_sw128(vb + ok2, 16, 1024), IDESC_S, k > 0);
+                }
+                umma_commit(&ctl.sdp_full[s]);
+                umma_commit(&ctl.kv_empty[ks]);
             }
             umma_commit(&ctl.fin);
             mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
@@ -230,6 +258,9 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         int e = 0;                             // next kept entry (ascending)
         int km = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
         float kl = nsel > 0 ? __ldg(my_lg) : 0.f;
+        // the entry after it, loaded one step early
+        int km_n = nsel > 1 ? __ldg(my_idx + 1) : 0x7fffffff;
+        float kl_n = nsel > 1 ? __ldg(my_lg + 1) : 0.f;
         const bool train = p.mode == 0;
         bool ok = true;
         for (int j = 0; j < nb; ++j) {
@@ -293,8 +324,10 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             if (kept) {
                 if (train) atomicAdd(my_dlg + e, sum);   // two halves: a + b, order-independent
                 ++e;
-                km = e < nsel ? __ldg(my_idx + e) : 0x7fffffff;
-                kl = e < nsel ? __ldg(my_lg + e) : 0.f;
+                km = km_n;
+                kl = kl_n;
+                km_n = e + 1 < nsel ? __ldg(my_idx + e + 1) : 0x7fffffff;
+                kl_n = e + 1 < nsel ? __ldg(my_lg + e + 1) : 0.f;
             }
         }
         // dQ: columns 64 hk .. 64 hk + 63 of the row
@@ -397,7 +430,7 @@ struct DkvCtl {
     int abort_flag;
 };
 
-constexpr int kThreadsD = 224;                           // keys (4 warps), issuer, two row-info warps
+constexpr int kThreadsD = 256;                           // keys (4 warps), two issuers, two row-info warps
 constexpr int kInfoLanes = 64;
 constexpr int kPairBytes = 2 * kKeys * kD * 2;           // 32 KB: K (or V) of the key pair
 constexpr int kDkvOffV = kPairBytes;
@@ -484,17 +517,17 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         mbar_init(&ctl.kv_full, 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(&ctl.q_full[s], 1);
-            mbar_init(&ctl.q_empty[s], 1);
+            mbar_init(&ctl.q_empty[s], 2);    // both issuers' products of the tile
         }
         for (int s = 0; s < kInfoStages; ++s) {
             mbar_init(&ctl.info_full[s], kInfoLanes);
             mbar_init(&ctl.info_empty[s], kWorkers);
         }
-        mbar_init(&ctl.sdp_full, 1);
+        mbar_init(&ctl.sdp_full, 2);          // S^T from the first issuer, dP^T from the second
         mbar_init(&ctl.sdp_free, kWorkers);
         mbar_init(&ctl.pds_full, kWorkers);
-        mbar_init(&ctl.half_done, 1);
-        mbar_init(&ctl.fin, 1);
+        mbar_init(&ctl.half_done, 2);         // dV and dK
+        mbar_init(&ctl.fin, 2);
         ctl.abort_flag = 0;
         fence_barrier_init();
     }
@@ -522,7 +555,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     float* info = reinterpret_cast<float*>(smem + kDkvOffInfo);
     const int nh = 2 * nq;   // 64-row halves of the query tiles
 
-    if (warp >= 5) {
+    if (warp == 5 || warp == 6) {
         // ---- row information of query tile q (LSE, Delta, bias of both blocks),
         // one tile ahead of the key threads; two rows per lane, searched together
         const int il = t - 5 * 32;   // 0 .. 63
@@ -551,14 +584,20 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             inf[2 * kRows + rb] = -db;
             mbar_arrive(&ctl.info_full[s]);
         }
-    } else if (warp == 4) {
+    } else if (warp == 4 || warp == 7) {
         if (lane == 0) {
-            // ---- issuer: S^T, dP^T of half x+1 go in as soon as the keys have read
-            // those of half x; dV, dK of half x once its P^T, dS^T are written
-            mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
-            for (int h = 0; h < 2; ++h) {
-                tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
-                tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+            // ---- issuers: warp 4 loads the tiles and issues S^T = K Q^T and
+            // dV += P^T dO; warp 7 issues dP^T = V dO^T and dK += dS^T Q.  The
+            // products of half x+1 go in as soon as the keys have read those of
+            // half x; the accumulations of half x once its P^T, dS^T are written.
+            const bool first = warp == 4;
+            if (first) {
+                mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
+                for (int h = 0; h < 2; ++h) {
+                    tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+                    tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys,
+                                bh);
+                }
             }
             auto load_q = [&](int q) {
                 const int s = q & 1;
@@ -570,51 +609,53 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                     tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, tq * kRows, bh);
                 }
             };
-            load_q(0);
-            if (nq > 1) load_q(1);
+            if (first) {
+                load_q(0);
+                if (nq > 1) load_q(1);
+            }
             constexpr uint32_t IDESC_T = idesc_bf16(2 * kKeys, 64, 0, 0);   // M = 128 keys, N = 64 rows
             constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
-            const uint32_t kb = smem_u32(smem), vb = smem_u32(smem + kDkvOffV);
+            // A operand (K or V of the pair) and the TMEM targets of this issuer
+            const uint32_t ab = smem_u32(smem + (first ? 0 : kDkvOffV));
+            const uint32_t t_prod = tmem + (first ? kTmemST : kTmemDPT);
+            const uint32_t t_acc = tmem + (first ? kTmemDV : kTmemDK);
+            const uint32_t t_a2 = tmem + (first ? kTmemPT : kTmemDST);
             bool ok = mbar_wait(&ctl.kv_full, 0, wc, kSleepNs);
-            auto issue_sdp = [&](int x) -> bool {
+            auto issue_prod = [&](int x) -> bool {
                 const int q = x >> 1, h = x & 1, s = q & 1;
                 if (h == 0 && !mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc, kSleepNs)) return false;
                 tc_fence_after();
-                const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
+                // B operand: Q (first issuer) or dO rows of this half, K-major
+                const uint32_t bb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes) + (first ? 0 : kQBytes);
 #pragma unroll
                 for (int k = 0; k < kD / 16; ++k) {
-                    const uint32_t ok2 = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
-                    const uint32_t oq = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
-                    umma_bf16(tmem + kTmemST, smem_desc_sw128(kb + ok2, 16, 1024), smem_desc_sw128(qb + oq, 16, 1024),
-                              IDESC_T, k > 0);
-                    umma_bf16(tmem + kTmemDPT, smem_desc_sw128(vb + ok2, 16, 1024), smem_desc_sw128(gb + oq, 16, 1024),
-                              IDESC_T, k > 0);
+                    const uint32_t oa = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
+                    const uint32_t ob = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
+                    umma_bf16(t_prod, smem_desc_sw128(ab + oa, 16, 1024), smem_desc_sw128(bb + ob, 16, 1024), IDESC_T,
+                              k > 0);
                 }
                 umma_commit(&ctl.sdp_full);
                 return true;
             };
-            if (ok) ok = issue_sdp(0);
+            if (ok) ok = issue_prod(0);
             for (int x = 0; ok && x < nh; ++x) {
                 const int q = x >> 1, h = x & 1, s = q & 1;
                 if (!mbar_wait(&ctl.sdp_free, x & 1, wc, kSleepNs)) { ok = false; break; }
-                if (x + 1 < nh && !issue_sdp(x + 1)) { ok = false; break; }
+                if (x + 1 < nh && !issue_prod(x + 1)) { ok = false; break; }
                 if (!mbar_wait(&ctl.pds_full, x & 1, wc, kSleepNs)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t qb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes), gb = qb + kQBytes;
+                // B operand: dO (first issuer, for dV) or Q (for dK) rows of this half, MN-major
+                const uint32_t bb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes) + (first ? kQBytes : 0);
 #pragma unroll
                 for (int k = 0; k < 64 / 16; ++k) {
-                    // B = dO (or Q) rows of this half, MN-major: 16 rows = two 8-row atoms
-                    const uint32_t ob = h * 64 * 128 + k * 2048;
-                    const uint32_t acc = (x > 0 || k > 0) ? 1u : 0u;
-                    umma_bf16_ta(tmem + kTmemDV, tmem + kTmemPT + k * 8, smem_desc_sw128(gb + ob, kRows * 128, 1024),
-                                 IDESC_ACC, acc);
-                    umma_bf16_ta(tmem + kTmemDK, tmem + kTmemDST + k * 8, smem_desc_sw128(qb + ob, kRows * 128, 1024),
-                                 IDESC_ACC, acc);
+                    const uint32_t ob = h * 64 * 128 + k * 2048;   // 16 rows = two 8-row atoms
+                    umma_bf16_ta(t_acc, t_a2 + k * 8, smem_desc_sw128(bb + ob, kRows * 128, 1024), IDESC_ACC,
+                                 (x > 0 || k > 0) ? 1u : 0u);
                 }
                 umma_commit(&ctl.half_done);
                 if (h == 1) {
                     umma_commit(&ctl.q_empty[s]);
-                    if (q + 2 < nq) {
+                    if (first && q + 2 < nq) {
                         if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                         load_q(q + 2);
                     }
