@@ -157,7 +157,9 @@ sas_status sas_attention_fwd(sas_handle* h,
  *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
  *              row's history; SCORES_GIVEN handles only, else NULL       (out)
  * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
- * allocates the handle's backward workspace (synchronously). */
+ * allocates the handle's backward workspace, and every call reads back how
+ * many blocks the forward's tiles visit to size a buffer: the call
+ * synchronises with its stream once (so it cannot be captured in a graph). */
 sas_status sas_attention_bwd(sas_handle* h,
                              const void* Q, const void* K, const void* V,
                              const float* scores,

@@ -152,10 +152,14 @@ struct AttnBwdArgs {
     int32_t* inv_off;           // [BH*T + 1]
     int32_t* inv_cursor;        // [BH*T]
     int32_t* inv_tiles;         // entries of the inverted lists
+    int32_t* inv_pos;           // their block positions
+    int32_t* slot_off;          // [BH*T + 1] first offset slot of each tile
+    float* offs;                // [slots][128] per-row offsets written by pass 1
     int N, C, T, BH, topk, mode, d;
     float sm_scale;
 };
 extern const int kBwdMaxTiles;   // query tiles per head the backward supports
+cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total);
 cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err);
 
 // ---- failure-path self test (bounded wait on a barrier nothing completes)

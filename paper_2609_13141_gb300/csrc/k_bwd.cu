@@ -103,6 +103,9 @@ struct BwdParams {
     float* delta;
     const int32_t* inv_off;
     const int32_t* inv_tiles;
+    const int32_t* inv_pos;     // per inverted entry: positions of blocks 2p, 2p+1 in the tile's list (+1; 0: absent)
+    const int32_t* slot_off;    // per tile: first slot of its visited blocks in offs
+    float* offs;                // per (tile, visited block) slot: 128 rows of log g - LSE (log2), -inf if not attended
     int N, C, T, BH, topk, mode;
     float sm_scale, scale_log2;
     int* status;
@@ -251,6 +254,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             lse2 = __ldg(p.LSE + roff) * kLog2eB;
             if (hk == 0) p.delta[roff] = delta;
         }
+        const int slot0 = __ldg(p.slot_off + tb);
         const int nsel = valid ? min(p.topk, c) : 0;
         const int32_t* my_idx = p.sel_idx + roff * p.topk;
         const float* my_lg = p.sel_logg + roff * p.topk;
@@ -293,6 +297,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 // block the row does not attend; the causal limit only on its own block
                 const float boff = lim >= 0 ? bias - lse2 : -CUDART_INF_F;
                 const bool causal = lim >= 0 && lim < kKeys - 1;
+                if (hk == 0) p.offs[(static_cast<long long>(slot0) + j) * kRows + r] = boff;   // for pass 2
                 const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2), bo2 = f32x2(boff, boff);
                 const uint64_t nd2 = f32x2(-delta, -delta);
                 uint64_t acc = 0;
@@ -397,14 +402,14 @@ __global__ void __launch_bounds__(1024) bwd_inv_scan_kernel(const int32_t* cnt, 
     int run = part[t] - s;
     for (long long k = lo; k < hi; ++k) {
         off[k] = run;
-        cursor[k] = run;
+        if (cursor) cursor[k] = run;
         run += cnt[k];
     }
     if (t == 1023) off[n] = part[1023];
 }
 
 __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cursor,
-                                    int32_t* tiles, int BH, int T, int C) {
+                                    int32_t* tiles, int32_t* pos, int BH, int T, int C) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * T) return;
     const int bh = static_cast<int>(tb / T);
@@ -413,12 +418,24 @@ __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* uni
     const int U = union_cnt[tb];
     int last = -1;
     for (int k = 0; k < U; ++k) {
-        const int pr = u[k] >> 1;
+        const int m = u[k], pr = m >> 1;
         if (pr == last) continue;
         last = pr;
+        // positions (+1) of blocks 2pr and 2pr+1 in this tile's list (ascending)
+        const int j0 = m == 2 * pr ? k + 1 : 0;
+        const int j1 = m == 2 * pr + 1 ? k + 1 : (k + 1 < U && u[k + 1] == 2 * pr + 1 ? k + 2 : 0);
         const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pr, 1);
         tiles[slot] = tile;
+        pos[slot] = j0 | (j1 << 16);
     }
+}
+
+// visited blocks per tile: its union list plus one or two diagonal blocks
+__global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH, int T, int C) {
+    const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (tb >= static_cast<long long>(BH) * T) return;
+    const int tile = static_cast<int>(tb % T);
+    cnt[tb] = union_cnt[tb] + ((2 * tile + 1 < C) ? 2 : 1);
 }
 
 // ------------------------------------------------------------------ pass 2
@@ -441,64 +458,10 @@ constexpr int kDkvOffList = kDkvOffInfo + kInfoStages * 4 * kRows * 4;
 // query tiles of a key pair (sorted list, then the unsorted copy); the host
 // refuses heads of more than kBwdMaxTiles tiles
 constexpr int kDkvListCap = 2048;
-constexpr int kDkvOffCtl = kDkvOffList + 2 * kDkvListCap * 4;
+constexpr int kDkvOffCtl = kDkvOffList + 3 * kDkvListCap * 4;   // order, tiles, positions
 constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
 // TMEM: dV [0,128), dK [128,256), S^T [256,320), dP^T [320,384), P^T [384,416), dS^T [416,448)
 constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemST = 256, kTmemDPT = 320, kTmemPT = 384, kTmemDST = 416;
-
-// Biases (log2 units, or markers) of blocks m and m+1 (m even) for query
-// rows ia and ib, with the two rows' searches interleaved: kept historical
-// block -> log g (training) or 0; the row's own block -> 0 with the causal
-// limit applied by the caller; otherwise -inf.  One search per row finds the
-// first kept entry >= m, so m+1 is the entry there or the next.
-__device__ __forceinline__ void pair_bias2(const BwdParams& p, int bh, int m, int ia, int ib, float (&ba)[2],
-                                           float (&bb)[2]) {
-    int lo[2] = {0, 0}, hi[2], c[2] = {ia >> 6, ib >> 6};
-    const int32_t* idx[2];
-    long long roff[2];
-    const int rows[2] = {ia, ib};
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const bool v = rows[r] < p.N;
-        roff[r] = static_cast<long long>(bh) * p.N + (v ? rows[r] : 0);
-        idx[r] = p.sel_idx + roff[r] * p.topk;
-        hi[r] = (v && m < c[r]) ? min(p.topk, c[r]) : 0;   // search only where block m is historical
-    }
-    while (lo[0] < hi[0] || lo[1] < hi[1]) {
-        int val[2];
-#pragma unroll
-        for (int r = 0; r < 2; ++r) val[r] = lo[r] < hi[r] ? __ldg(idx[r] + ((lo[r] + hi[r]) >> 1)) : 0;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            if (lo[r] < hi[r]) {
-                const int mid = (lo[r] + hi[r]) >> 1;
-                if (val[r] < m) lo[r] = mid + 1; else hi[r] = mid;
-            }
-        }
-    }
-    float* outs[2] = {ba, bb};
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const int i = rows[r];
-        const int nsel = min(p.topk, c[r]);
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            const int mq = m + q;
-            float b = -CUDART_INF_F;
-            if (i < p.N) {
-                if (mq == c[r]) {
-                    b = 0.f;
-                } else if (mq < c[r]) {
-                    const int e = lo[r] + q;   // m at lo (if kept), m+1 at lo or lo+1
-                    for (int ee = lo[r]; ee <= e && ee < nsel; ++ee)
-                        if (__ldg(idx[r] + ee) == mq)
-                            b = p.mode == 0 ? __ldg(p.sel_logg + roff[r] * p.topk + ee) * kLog2eB : 0.f;
-                }
-            }
-            outs[r][q] = b;
-        }
-    }
-}
 
 __global__ void __launch_bounds__(kThreadsD, 1)
 bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
@@ -537,15 +500,26 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     }
     // the query tiles: diagonal first, then the others in ascending order (a
     // fixed summation order); rank sort of the inverted list in shared memory
+    // list[q]: index into raw / rawpos of the q-th query tile (slot 0: the diagonal
+    // tile, which visits 2pr, 2pr+1 right after its union list)
     int* raw = list + kDkvListCap;
-    if (t == 0) list[0] = pr;
-    for (int k = t; k < cnt; k += kThreadsD) raw[k] = __ldg(p.inv_tiles + off + k);
+    int* rawpos = raw + kDkvListCap;
+    if (t == 0) {
+        list[0] = 0;
+        raw[0] = pr;
+        const int Upr = __ldg(p.union_cnt + pb);
+        rawpos[0] = (Upr + 1) | ((2 * pr + 1 < p.C ? Upr + 2 : 0) << 16);
+    }
+    for (int k = t; k < cnt; k += kThreadsD) {
+        raw[1 + k] = __ldg(p.inv_tiles + off + k);
+        rawpos[1 + k] = __ldg(p.inv_pos + off + k);
+    }
     __syncthreads();
     for (int k = t; k < cnt; k += kThreadsD) {
-        const int v = raw[k];
+        const int v = raw[1 + k];
         int rank = 0;
-        for (int q = 0; q < cnt; ++q) rank += raw[q] < v;
-        list[1 + rank] = v;
+        for (int q = 0; q < cnt; ++q) rank += raw[1 + q] < v;
+        list[1 + rank] = 1 + k;
     }
     tc_fence_before();
     __syncthreads();
@@ -556,32 +530,27 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     const int nh = 2 * nq;   // 64-row halves of the query tiles
 
     if (warp == 5 || warp == 6) {
-        // ---- row information of query tile q (LSE, Delta, bias of both blocks),
-        // one tile ahead of the key threads; two rows per lane, searched together
+        // ---- row information of query tile q, up to three tiles ahead: per row
+        // the offsets (log g - LSE) of blocks 2pr, 2pr+1 that pass 1 wrote, and -Delta
         const int il = t - 5 * 32;   // 0 .. 63
         for (int q = 0; q < nq; ++q) {
             const int s = q % kInfoStages;
             if (q >= kInfoStages && !mbar_wait(&ctl.info_empty[s], ((q - kInfoStages) / kInfoStages) & 1, wc, kSleepNs))
                 break;
             float* inf = info + s * 4 * kRows;
-            const int tq = list[q];
-            const int ra = il, rb = il + kInfoLanes;
-            const int ia = tq * kRows + ra, ib = tq * kRows + rb;
-            const long long oa = static_cast<long long>(bh) * p.N + ia, ob = static_cast<long long>(bh) * p.N + ib;
-            const float la = ia < p.N ? __ldg(p.LSE + oa) * kLog2eB : 0.f;
-            const float lb = ib < p.N ? __ldg(p.LSE + ob) * kLog2eB : 0.f;
-            const float da = ia < p.N ? p.delta[oa] : 0.f;
-            const float db = ib < p.N ? p.delta[ob] : 0.f;
-            float ba[2], bb[2];
-            pair_bias2(p, bh, 2 * pr, ia, ib, ba, bb);
-            // per block: log g - LSE (log2 units), -inf where the row does not attend;
-            // then -Delta
-            inf[ra] = ba[0] - la;
-            inf[rb] = bb[0] - lb;
-            inf[kRows + ra] = ba[1] - la;
-            inf[kRows + rb] = bb[1] - lb;
-            inf[2 * kRows + ra] = -da;
-            inf[2 * kRows + rb] = -db;
+            const int tq = raw[list[q]];
+            const int ps = rawpos[list[q]];
+            const int j0 = (ps & 0xffff) - 1, j1 = (ps >> 16) - 1;
+            const long long tbq = static_cast<long long>(bh) * p.T + tq;
+            const long long so = static_cast<long long>(__ldg(p.slot_off + tbq)) * kRows;
+#pragma unroll
+            for (int rr = 0; rr < 2; ++rr) {
+                const int r = il + rr * kInfoLanes;
+                const int i = tq * kRows + r;
+                inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : -CUDART_INF_F;
+                inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : -CUDART_INF_F;
+                inf[2 * kRows + r] = i < p.N ? -__ldcg(p.delta + static_cast<long long>(bh) * p.N + i) : 0.f;
+            }
             mbar_arrive(&ctl.info_full[s]);
         }
     } else if (warp == 4 || warp == 7) {
@@ -601,7 +570,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             }
             auto load_q = [&](int q) {
                 const int s = q & 1;
-                const int tq = list[q];
+                const int tq = raw[list[q]];
                 uint8_t* st = smem + kDkvOffQ + s * 2 * kQBytes;
                 mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
                 for (int h = 0; h < 2; ++h) {
@@ -673,7 +642,6 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         bool ok = true;
         for (int x = 0; x < nh; ++x) {
             const int q = x >> 1, h = x & 1, si = q % kInfoStages;
-            const int tq = list[q];
             const float* inf = info + si * 4 * kRows;
             if (h == 0 && !mbar_wait_warp(&ctl.info_full[si], (q / kInfoStages) & 1, wc, kSleepNs)) { ok = false; break; }
             if (!mbar_wait_warp(&ctl.sdp_full, x & 1, wc, kSleepNs)) { ok = false; break; }
@@ -791,6 +759,20 @@ __global__ void bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const
 
 const int kBwdMaxTiles = kDkvListCap - 1;
 
+// Slots of the per-tile visited-block offsets pass 1 writes for pass 2: one per
+// visited block of every tile; returns their total in *total (synchronises).
+cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total) {
+    const long long tiles = static_cast<long long>(a.BH) * a.T;
+    const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
+    bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
+    bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.slot_off, nullptr, tiles);
+    int32_t host = 0;
+    cudaError_t e = cudaMemcpyAsync(&host, a.slot_off + tiles, 4, cudaMemcpyDeviceToHost, env.stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(env.stream);
+    *total = host;
+    return e;
+}
+
 cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err) {
     if (a.d != kD) {
         *err = "backward: head dim must be 128";
@@ -829,6 +811,9 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     p.delta = a.delta;
     p.inv_off = a.inv_off;
     p.inv_tiles = a.inv_tiles;
+    p.inv_pos = a.inv_pos;
+    p.slot_off = a.slot_off;
+    p.offs = a.offs;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
     p.sm_scale = a.sm_scale;
     p.scale_log2 = a.sm_scale * kLog2eB;
@@ -849,7 +834,8 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
     bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, tiles);
-    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cursor, a.inv_tiles, a.BH, a.T, a.C);
+    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cursor, a.inv_tiles, a.inv_pos,
+                                                     a.BH, a.T, a.C);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
     // pass 2

@@ -104,9 +104,11 @@ struct sas_handle {
     size_t hidden_bytes = 0;
     // backward workspace (allocated by the first sas_attention_bwd)
     float* bwd_delta = nullptr;
-    int32_t* bwd_inv = nullptr;     // counts, offsets, cursors
-    int32_t* bwd_tiles = nullptr;
+    int32_t* bwd_inv = nullptr;     // counts, cursors, offsets, slot offsets
+    int32_t* bwd_tiles = nullptr;   // inverted lists: tiles, then block positions
     float* bwd_dlogg = nullptr;
+    float* bwd_offs = nullptr;      // per-row offsets of every visited block (pass 1 -> pass 2)
+    size_t bwd_offs_bytes = 0;
     // timing
     bool timing = false;
     std::vector<TimeRec> recs;
@@ -271,6 +273,7 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->bwd_inv);
     cudaFree(h->bwd_tiles);
     cudaFree(h->bwd_dlogg);
+    cudaFree(h->bwd_offs);
     for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
     delete h;
 }
@@ -408,8 +411,8 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         cudaError_t e = cudaStreamSynchronize(s);
         const size_t pairs = static_cast<size_t>(h->T < h->C ? h->T : h->C);
         if (e == cudaSuccess) e = alloc(&h->bwd_delta, rows * 4);
-        if (e == cudaSuccess) e = alloc(&h->bwd_inv, (3 * tiles + 1) * 4);
-        if (e == cudaSuccess) e = alloc(&h->bwd_tiles, tiles * pairs * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_inv, (4 * tiles + 2) * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_tiles, 2 * tiles * pairs * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, rows * (c.topk > 0 ? c.topk : 1) * 4);
         if (e != cudaSuccess) {
             cudaFree(h->bwd_delta); cudaFree(h->bwd_inv); cudaFree(h->bwd_tiles); cudaFree(h->bwd_dlogg);
@@ -430,14 +433,31 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.inv_cnt = h->bwd_inv;
     a.inv_cursor = h->bwd_inv + tiles;
     a.inv_off = h->bwd_inv + 2 * tiles;
+    a.slot_off = h->bwd_inv + 3 * tiles + 1;
     a.inv_tiles = h->bwd_tiles;
+    a.inv_pos = h->bwd_tiles + tiles * static_cast<size_t>(h->T < h->C ? h->T : h->C);
     a.N = c.N; a.C = h->C; a.T = h->T; a.BH = h->BH; a.topk = c.topk; a.mode = c.mode; a.d = c.d;
     a.sm_scale = h->sm_scale;
     const sas::KernelEnv env{s, h->status, h->limit};
     const char* err = "";
-    cudaError_t e = timed_launch(h, 6, s, [&] { return sas::launch_attn_bwd(a, env, &err); });
+    // slots of the per-row offsets pass 1 hands to pass 2 (their number depends
+    // on the forward's tile lists: read back, synchronously, to size the buffer)
+    long long slots = 0;
+    cudaError_t e = sas::launch_bwd_slots(a, env, &slots);
+    if (e != cudaSuccess) return cuda_fail(h, e, "backward slots");
+    const size_t need = static_cast<size_t>(slots) * 128 * 4;
+    if (need > h->bwd_offs_bytes) {
+        cudaFree(h->bwd_offs);
+        h->bwd_offs = nullptr;
+        h->bwd_offs_bytes = 0;
+        e = alloc(&h->bwd_offs, need);
+        if (e != cudaSuccess) return cuda_fail(h, e, "backward offsets");
+        h->bwd_offs_bytes = need;
+    }
+    a.offs = h->bwd_offs;
+    e = timed_launch(h, 6, s, [&] { return sas::launch_attn_bwd(a, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
-    h->launches += (a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 5 : 4;   // six or five kernels in all
+    h->launches += 2 + ((a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 5 : 4);   // all its kernels
     return SAS_OK;
 }
 
