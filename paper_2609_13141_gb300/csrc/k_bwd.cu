@@ -16,8 +16,11 @@
 //                     P^T and dS^T into TMEM, dV += P^T dO and dK += dS^T Q.
 //   bwd_ds_kernel     score gradient of given scores (sparse scope):
 //                     ds_m = dlogg_m [m kept] - g_m sum dlogg.
-// Roles: warps 0-3 are the rows (pass 1) or keys (pass 2) of the tile, one
-// thread per TMEM lane; warp 4 lane 0 issues the TMA loads and the MMAs.
+// Roles, pass 1: warps 0-7 are the rows (two threads per TMEM lane, half a
+// block of keys each), warp 8 issues S and dQ, warp 9 issues dP, warp 10
+// issues the TMA loads.  Pass 2: warps 0-3 are the keys (one thread per TMEM
+// lane), warps 4 and 7 issue the MMAs, warp 5 stages the query tiles' per-row
+// information, warp 6 issues the TMA loads.
 #include <math_constants.h>
 
 #include "internal.h"
@@ -31,7 +34,7 @@ constexpr int kKeys = 64;           // keys per block
 constexpr int kD = 128;             // head dim
 constexpr int kWorkers = 128;       // key threads (pass 2)
 constexpr int kRowThreads = 256;    // pass 1: two threads per row, 32 keys of a block each
-constexpr int kThreadsB = 320;      // + two issuing warps (one tcgen05.mma issue takes ~90 cycles)
+constexpr int kThreadsB = 352;      // + two issuing warps (one tcgen05.mma issue takes ~90 cycles) + a loader
 constexpr float kLog2eB = 1.4426950408889634f;
 // Waiting threads sleep (woken when the phase completes) instead of spinning:
 // the issuing and row-information warps wait most of the time and would
@@ -150,29 +153,33 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
     const int row0 = tile * kRows;
 
-    if (warp == 8) {
+    if (warp == 10) {
         if (lane == 0) {
-            // ---- issuer: TMA loads and MMAs
-            auto block_at = [&](int j) { return j < U ? __ldg(ulist + j) : 2 * tile + (j - U); };
+            // ---- loader: Q and dO once, then K and V of block j into stage
+            // j % kKvStages as soon as dQ and dP of block j - kKvStages are done
             mbar_arrive_expect_tx(&ctl.q_full, 2 * kQBytes);
             for (int h = 0; h < 2; ++h) {
                 tma_load_3d(smem + h * (kRows * 128), &mapQ, &ctl.q_full, h * 64, row0, bh);
                 tma_load_3d(smem + kDqOffDO + h * (kRows * 128), &mapDO, &ctl.q_full, h * 64, row0, bh);
             }
-            auto load_kv = [&](int j) {
+            for (int j = 0; j < nb; ++j) {
                 const int s = j % kKvStages;
-                const int m = block_at(j);
+                if (j >= kKvStages && !mbar_wait(&ctl.kv_empty[s], ((j / kKvStages) - 1) & 1, wc, kSleepNs)) break;
+                const int m = j < U ? __ldg(ulist + j) : 2 * tile + (j - U);
                 uint8_t* st = smem + kDqOffKV + s * 2 * kKVBytes;
                 mbar_arrive_expect_tx(&ctl.kv_full[s], 2 * kKVBytes);
                 for (int h = 0; h < 2; ++h) {
                     tma_load_3d(st + h * (kKeys * 128), &mapK, &ctl.kv_full[s], h * 64, m * kKeys, bh);
                     tma_load_3d(st + kKVBytes + h * (kKeys * 128), &mapV, &ctl.kv_full[s], h * 64, m * kKeys, bh);
                 }
-            };
-            for (int j = 0; j < kKvStages && j < nb; ++j) load_kv(j);
+            }
+        }
+    } else if (warp == 8) {
+        if (lane == 0) {
+            // ---- issuer: S = Q K^T and dQ += dS K
             constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
             constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
-            const uint32_t qb = smem_u32(smem), gb = smem_u32(smem + kDqOffDO);
+            const uint32_t qb = smem_u32(smem);
             bool ok = mbar_wait(&ctl.q_full, 0, wc, kSleepNs);
             // S and dP of block j go to TMEM buffer j & 1 while the rows still work
             // on block j - 1; dQ += dS K of block j - 1 follows once its dS is in.
@@ -204,10 +211,6 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                                      (jp > 0 || k > 0) ? 1u : 0u);
                     umma_commit(&ctl.dq_done[sp]);
                     umma_commit(&ctl.kv_empty[kp]);
-                    if (jp + kKvStages < nb) {
-                        if (!mbar_wait(&ctl.kv_empty[kp], (jp / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
-                        load_kv(jp + kKvStages);
-                    }
                 }
             }
             umma_commit(&ctl.fin);
@@ -447,8 +450,8 @@ struct DkvCtl {
     int abort_flag;
 };
 
-constexpr int kThreadsD = 256;                           // keys (4 warps), two issuers, two row-info warps
-constexpr int kInfoLanes = 64;
+constexpr int kThreadsD = 256;                           // keys (4 warps), two issuers, a row-info warp, a loader
+constexpr int kInfoLanes = 32;
 constexpr int kPairBytes = 2 * kKeys * kD * 2;           // 32 KB: K (or V) of the key pair
 constexpr int kDkvOffV = kPairBytes;
 constexpr int kDkvOffQ = 2 * kPairBytes;                 // 2 stages x (Q, dO) tiles
@@ -529,10 +532,10 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     float* info = reinterpret_cast<float*>(smem + kDkvOffInfo);
     const int nh = 2 * nq;   // 64-row halves of the query tiles
 
-    if (warp == 5 || warp == 6) {
+    if (warp == 5) {
         // ---- row information of query tile q, up to three tiles ahead: per row
         // the offsets (log g - LSE) of blocks 2pr, 2pr+1 that pass 1 wrote, and -Delta
-        const int il = t - 5 * 32;   // 0 .. 63
+        const int il = lane;
         for (int q = 0; q < nq; ++q) {
             const int s = q % kInfoStages;
             if (q >= kInfoStages && !mbar_wait(&ctl.info_empty[s], ((q - kInfoStages) / kInfoStages) & 1, wc, kSleepNs))
@@ -544,7 +547,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             const long long tbq = static_cast<long long>(bh) * p.T + tq;
             const long long so = static_cast<long long>(__ldg(p.slot_off + tbq)) * kRows;
 #pragma unroll
-            for (int rr = 0; rr < 2; ++rr) {
+            for (int rr = 0; rr < kRows / kInfoLanes; ++rr) {
                 const int r = il + rr * kInfoLanes;
                 const int i = tq * kRows + r;
                 inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : -CUDART_INF_F;
@@ -553,23 +556,18 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             }
             mbar_arrive(&ctl.info_full[s]);
         }
-    } else if (warp == 4 || warp == 7) {
+    } else if (warp == 6) {
         if (lane == 0) {
-            // ---- issuers: warp 4 loads the tiles and issues S^T = K Q^T and
-            // dV += P^T dO; warp 7 issues dP^T = V dO^T and dK += dS^T Q.  The
-            // products of half x+1 go in as soon as the keys have read those of
-            // half x; the accumulations of half x once its P^T, dS^T are written.
-            const bool first = warp == 4;
-            if (first) {
-                mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
-                for (int h = 0; h < 2; ++h) {
-                    tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
-                    tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys,
-                                bh);
-                }
+            // ---- loader: K and V of the pair once, then the (Q, dO) rows of
+            // query tile q into stage q & 1 once both products of tile q - 2 are done
+            mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
+            for (int h = 0; h < 2; ++h) {
+                tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+                tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
             }
-            auto load_q = [&](int q) {
+            for (int q = 0; q < nq; ++q) {
                 const int s = q & 1;
+                if (q >= 2 && !mbar_wait(&ctl.q_empty[s], ((q - 2) >> 1) & 1, wc, kSleepNs)) break;
                 const int tq = raw[list[q]];
                 uint8_t* st = smem + kDkvOffQ + s * 2 * kQBytes;
                 mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
@@ -577,11 +575,15 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                     tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, tq * kRows, bh);
                     tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, tq * kRows, bh);
                 }
-            };
-            if (first) {
-                load_q(0);
-                if (nq > 1) load_q(1);
             }
+        }
+    } else if (warp == 4 || warp == 7) {
+        if (lane == 0) {
+            // ---- issuers: warp 4 issues S^T = K Q^T and dV += P^T dO; warp 7
+            // issues dP^T = V dO^T and dK += dS^T Q.  The products of half x+1
+            // go in as soon as the keys have read those of half x; the
+            // accumulations of half x once its P^T, dS^T are written.
+            const bool first = warp == 4;
             constexpr uint32_t IDESC_T = idesc_bf16(2 * kKeys, 64, 0, 0);   // M = 128 keys, N = 64 rows
             constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
             // A operand (K or V of the pair) and the TMEM targets of this issuer
@@ -622,13 +624,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                                  (x > 0 || k > 0) ? 1u : 0u);
                 }
                 umma_commit(&ctl.half_done);
-                if (h == 1) {
-                    umma_commit(&ctl.q_empty[s]);
-                    if (first && q + 2 < nq) {
-                        if (!mbar_wait(&ctl.q_empty[s], (q >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
-                        load_q(q + 2);
-                    }
-                }
+                if (h == 1) umma_commit(&ctl.q_empty[s]);
             }
             umma_commit(&ctl.fin);
             mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
