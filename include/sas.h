@@ -155,7 +155,10 @@ sas_status sas_attention_fwd(sas_handle* h,
  *              mode); may be NULL                                        (out)
  *   dscores    fp32 [B, H, N, C] dL/ds of the given scores, sparse scope:
  *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
- *              row's history; SCORES_GIVEN handles only, else NULL       (out)
+ *              row's history; SCORES_GIVEN handles only, else NULL.
+ *              g_m = exp(s_m - LSE_i) takes the row's log-normaliser
+ *              LSE_i = s_m - log g_m from its first kept entry, so the
+ *              scores must be the ones the forward selected with     (out)
  * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
  * allocates the handle's backward workspace, and every call reads back how
  * many blocks the forward's tiles visit to size a buffer: the call

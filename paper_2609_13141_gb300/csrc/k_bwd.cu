@@ -134,7 +134,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             mbar_init(&ctl.kv_empty[s], 2);   // dQ (reads K) and dP (reads V)
         }
         for (int s = 0; s < 2; ++s) {
-            mbar_init(&ctl.ds_full[s], kRowThreads);
+            mbar_init(&ctl.ds_full[s], kRowThreads / 32);   // one arrive per row warp
             mbar_init(&ctl.dq_done[s], 1);
             mbar_init(&ctl.sdp_full[s], 2);   // S from one issuer, dP from the other
         }
@@ -328,7 +328,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             }
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(&ctl.ds_full[j & 1]);
+            mbar_arrive_warp(&ctl.ds_full[j & 1]);
             if (kept) {
                 if (train) atomicAdd(my_dlg + e, sum);   // two halves: a + b, order-independent
                 ++e;
@@ -486,12 +486,12 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             mbar_init(&ctl.q_empty[s], 2);    // both issuers' products of the tile
         }
         for (int s = 0; s < kInfoStages; ++s) {
-            mbar_init(&ctl.info_full[s], kInfoLanes);
-            mbar_init(&ctl.info_empty[s], kWorkers);
+            mbar_init(&ctl.info_full[s], 1);                // the row-information warp
+            mbar_init(&ctl.info_empty[s], kWorkers / 32);   // one arrive per key warp
         }
         mbar_init(&ctl.sdp_full, 2);          // S^T from the first issuer, dP^T from the second
-        mbar_init(&ctl.sdp_free, kWorkers);
-        mbar_init(&ctl.pds_full, kWorkers);
+        mbar_init(&ctl.sdp_free, kWorkers / 32);
+        mbar_init(&ctl.pds_full, kWorkers / 32);
         mbar_init(&ctl.half_done, 2);         // dV and dK
         mbar_init(&ctl.fin, 2);
         ctl.abort_flag = 0;
@@ -554,7 +554,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : -CUDART_INF_F;
                 inf[2 * kRows + r] = i < p.N ? -__ldcg(p.delta + static_cast<long long>(bh) * p.N + i) : 0.f;
             }
-            mbar_arrive(&ctl.info_full[s]);
+            mbar_arrive_warp(&ctl.info_full[s]);
         }
     } else if (warp == 6) {
         if (lane == 0) {
@@ -649,7 +649,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             tmem_ld32(lane_addr + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
             tmem_wait_ld();
             tc_fence_before();
-            mbar_arrive(&ctl.sdp_free);   // S^T, dP^T may be overwritten by the next half
+            mbar_arrive_warp(&ctl.sdp_free);   // S^T, dP^T may be overwritten by the next half
             uint32_t pp[32], dd[32];
             // In the diagonal tile (the first of the list) the rows of half h have
             // block 2pr + h as their own block: keys of that block are causal.
@@ -682,8 +682,8 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             tmem_st32(lane_addr + kTmemDST, dd);
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(&ctl.pds_full);
-            if (h == 1) mbar_arrive(&ctl.info_empty[si]);
+            mbar_arrive_warp(&ctl.pds_full);
+            if (h == 1) mbar_arrive_warp(&ctl.info_empty[si]);
         }
         if (ok && mbar_wait_warp(&ctl.fin, 0, wc, kSleepNs)) {
             tc_fence_after();
@@ -721,33 +721,54 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
 
 // --------------------------------------------------------- score gradient
 
-// one warp per row: ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of
-// the row's C_i given scores; 0 past the history
-__global__ void bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* dlogg, float* ds, int BH,
-                              int N, int C, int topk) {
-    const long long w = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (w >= static_cast<long long>(BH) * N) return;
-    const int i = static_cast<int>(w % N);
-    const int c = i >> 6;
-    const float* s = scores + w * C;
-    float* out = ds + w * C;
-    float mx = -CUDART_INF_F;
-    for (int m = lane; m < c; m += 32) mx = fmaxf(mx, s[m]);
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float se = 0.f;
-    for (int m = lane; m < c; m += 32) se += __expf(s[m] - mx);
-    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
-    const float lse = mx + __logf(se);
-    const int nsel = min(topk, c);
-    float sum = 0.f;
-    for (int e = lane; e < nsel; e += 32) sum += dlogg[w * topk + e];
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    for (int m = lane; m < C; m += 32) out[m] = m < c ? -__expf(s[m] - lse) * sum : 0.f;
-    __syncwarp();
-    for (int e = lane; e < nsel; e += 32) {
-        const int m = sel_idx[w * topk + e];
-        out[m] += dlogg[w * topk + e];
+// ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of the row's C_i
+// given scores; 0 past the history.  One CTA per run of R consecutive rows
+// (their score rows are contiguous): the row's log-normaliser comes back from
+// its first kept entry (log g_m = s_m - LSE of the scores, Eq.
+// normalized_log_gate), the kept dlogg values are scattered into shared
+// memory, and the R x C outputs go out in one coalesced sweep.
+__global__ void __launch_bounds__(256)
+bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg, const float* dlogg, float* ds,
+              long long rows, int N, int C, int topk, int R, int train) {
+    extern __shared__ float dsh[];   // [R][C] kept dlogg, then R normalisers and R sums
+    float* add = dsh;
+    float* rlse = dsh + static_cast<long long>(R) * C;
+    float* rsum = rlse + R;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const long long w0 = static_cast<long long>(blockIdx.x) * R;
+    const int nr = static_cast<int>(min(static_cast<long long>(R), rows - w0));
+    const int tot = nr * C;
+    for (int k = t; k < tot; k += blockDim.x) add[k] = 0.f;
+    __syncthreads();
+    for (int rr = warp; rr < nr; rr += blockDim.x >> 5) {
+        const long long w = w0 + rr;
+        const int c = static_cast<int>(w % N) >> 6;
+        const int nsel = train ? min(topk, c) : 0;
+        float sum = 0.f;
+        for (int e = lane; e < nsel; e += 32) {
+            const float v = __ldg(dlogg + w * topk + e);
+            sum += v;
+            add[rr * C + __ldg(sel_idx + w * topk + e)] = v;   // kept blocks are distinct
+        }
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if (lane == 0) {
+            rsum[rr] = sum;
+            rlse[rr] = nsel > 0 ? __ldg(scores + w * C + __ldg(sel_idx + w * topk)) - __ldg(sel_logg + w * topk) : 0.f;
+        }
+    }
+    __syncthreads();
+    const float* s = scores + w0 * C;
+    float* out = ds + w0 * C;
+    for (int k = t; k < tot; k += blockDim.x) {
+        const int rr = k / C, m = k - rr * C;
+        const int c = static_cast<int>((w0 + rr) % N) >> 6;
+        float v = 0.f;
+        if (m < c) {
+            v = add[k];
+            const float sm = rsum[rr];
+            if (sm != 0.f) v -= __expf(__ldg(s + k) - rlse[rr]) * sm;
+        }
+        out[k] = v;
     }
 }
 
@@ -840,8 +861,10 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
         const long long rows = static_cast<long long>(a.BH) * a.N;
-        bwd_ds_kernel<<<static_cast<unsigned>((rows * 32 + 255) / 256), 256, 0, env.stream>>>(
-            a.scores, a.sel_idx, a.dlogg, a.ds, a.BH, a.N, a.C, a.topk);
+        const int R = max(1, min(32, 8192 / a.C));   // <= 32 KB of shared memory
+        const size_t sh = (static_cast<size_t>(R) * a.C + 2 * R) * sizeof(float);
+        bwd_ds_kernel<<<static_cast<unsigned>((rows + R - 1) / R), 256, sh, env.stream>>>(
+            a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows, a.N, a.C, a.topk, R, a.mode == 0 ? 1 : 0);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     } else if (a.ds != nullptr) {

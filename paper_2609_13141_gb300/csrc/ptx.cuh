@@ -39,6 +39,16 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
         : "memory");
 }
 
+// One arrive for the whole (converged) warp: the lanes meet at __syncwarp,
+// which orders their earlier writes (and, after tcgen05.fence::before_thread_sync,
+// their tensor-memory stores) before lane 0's release-arrive.  The barrier's
+// count is then per warp; 32 lanes arriving one by one serialise on the
+// barrier's shared-memory word.
+__device__ __forceinline__ void mbar_arrive_warp(uint64_t* bar) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
 // Raises the barrier's expected transaction count without arriving.
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
     asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
