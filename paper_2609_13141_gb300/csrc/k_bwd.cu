@@ -175,72 +175,87 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             }
         }
     } else if (warp == 8) {
-        if (lane == 0) {
-            // ---- issuer: S = Q K^T and dQ += dS K
+        {
+            // ---- issuer of S = Q K^T and dQ += dS K (whole warp; the elected lane issues)
             constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
             constexpr uint32_t IDESC_DQ = idesc_bf16(kRows, kD, 0, 1);
             const uint32_t qb = smem_u32(smem);
-            bool ok = mbar_wait(&ctl.q_full, 0, wc, kSleepNs);
+            bool ok = mbar_wait_warp(&ctl.q_full, 0, wc, kSleepNs);
             // S and dP of block j go to TMEM buffer j & 1 while the rows still work
             // on block j - 1; dQ += dS K of block j - 1 follows once its dS is in.
             for (int j = 0; ok && j <= nb; ++j) {
                 if (j < nb) {
                     const int s = j & 1, ks = j % kKvStages;
-                    if (!mbar_wait(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
+                    if (!mbar_wait_warp(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t kb = smem_u32(smem + kDqOffKV + ks * 2 * kKVBytes);
+                    if (elect_one()) {
 #pragma unroll
-                    for (int k = 0; k < kD / 16; ++k) {
-                        const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
-                        const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
-                        umma_bf16(tmem + kTmemS + s * 128, smem_desc_sw128(qb + oq, 16, 1024),
-                                  smem_desc_sw128(kb + ok2, 16, 1024), IDESC_S, k > 0);
+                        for (int k = 0; k < kD / 16; ++k) {
+                            const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                            const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+                            umma_bf16(tmem + kTmemS + s * 128, smem_desc_sw128(qb + oq, 16, 1024),
+                                      smem_desc_sw128(kb + ok2, 16, 1024), IDESC_S, k > 0);
+                        }
+                        umma_commit(&ctl.sdp_full[s]);
                     }
-                    umma_commit(&ctl.sdp_full[s]);
+                    __syncwarp();
                 }
                 if (j >= 1) {
                     const int jp = j - 1, sp = jp & 1, kp = jp % kKvStages;
                     // dS of block jp is in TMEM buffer sp once every row has written it
-                    if (!mbar_wait(&ctl.ds_full[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
+                    if (!mbar_wait_warp(&ctl.ds_full[sp], (jp >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t kb = smem_u32(smem + kDqOffKV + kp * 2 * kKVBytes);
+                    if (elect_one()) {
 #pragma unroll
-                    for (int k = 0; k < kKeys / 16; ++k)
-                        umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + sp * 32 + k * 8,
-                                     smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ,
-                                     (jp > 0 || k > 0) ? 1u : 0u);
-                    umma_commit(&ctl.dq_done[sp]);
-                    umma_commit(&ctl.kv_empty[kp]);
+                        for (int k = 0; k < kKeys / 16; ++k)
+                            umma_bf16_ta(tmem + kTmemDQ, tmem + kTmemDS + sp * 32 + k * 8,
+                                         smem_desc_sw128(kb + k * 2048, kKeys * 128, 1024), IDESC_DQ,
+                                         (jp > 0 || k > 0) ? 1u : 0u);
+                        umma_commit(&ctl.dq_done[sp]);
+                        umma_commit(&ctl.kv_empty[kp]);
+                    }
+                    __syncwarp();
                 }
             }
-            umma_commit(&ctl.fin);
-            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            if (elect_one()) {
+                umma_commit(&ctl.fin);
+                mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            }
+            __syncwarp();
         }
     } else if (warp == 9) {
-        if (lane == 0) {
+        {
             // ---- second issuer: dP = dO V^T of every block into TMEM buffer j & 1,
             // once the rows are done with block j - 2 (which used that buffer)
             constexpr uint32_t IDESC_S = idesc_bf16(kRows, kKeys, 0, 0);
             const uint32_t gb = smem_u32(smem + kDqOffDO);
-            bool ok = mbar_wait(&ctl.q_full, 0, wc, kSleepNs);
+            bool ok = mbar_wait_warp(&ctl.q_full, 0, wc, kSleepNs);
             for (int j = 0; ok && j < nb; ++j) {
                 const int s = j & 1, ks = j % kKvStages;
-                if (!mbar_wait(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
-                if (j >= 2 && !mbar_wait(&ctl.ds_full[s], ((j - 2) >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
+                if (!mbar_wait_warp(&ctl.kv_full[ks], (j / kKvStages) & 1, wc, kSleepNs)) { ok = false; break; }
+                if (j >= 2 && !mbar_wait_warp(&ctl.ds_full[s], ((j - 2) >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t vb = smem_u32(smem + kDqOffKV + ks * 2 * kKVBytes) + kKVBytes;
+                if (elect_one()) {
 #pragma unroll
-                for (int k = 0; k < kD / 16; ++k) {
-                    const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
-                    const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
-                    umma_bf16(tmem + kTmemDP + s * 128, smem_desc_sw128(gb + oq, 16, 1024),
-                              smem_desc_sw128(vb + ok2, 16, 1024), IDESC_S, k > 0);
+                    for (int k = 0; k < kD / 16; ++k) {
+                        const uint32_t oq = (k >> 2) * (kRows * 128) + (k & 3) * 32;
+                        const uint32_t ok2 = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+                        umma_bf16(tmem + kTmemDP + s * 128, smem_desc_sw128(gb + oq, 16, 1024),
+                                  smem_desc_sw128(vb + ok2, 16, 1024), IDESC_S, k > 0);
+                    }
+                    umma_commit(&ctl.sdp_full[s]);
+                    umma_commit(&ctl.kv_empty[ks]);
                 }
-                umma_commit(&ctl.sdp_full[s]);
-                umma_commit(&ctl.kv_empty[ks]);
+                __syncwarp();
             }
-            umma_commit(&ctl.fin);
-            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            if (elect_one()) {
+                umma_commit(&ctl.fin);
+                mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            }
+            __syncwarp();
         }
     } else {
         // ---- rows: thread t takes row t % 128 (its TMEM lane) and keys
@@ -445,7 +460,7 @@ __global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH,
 
 struct DkvCtl {
     uint64_t kv_full, q_full[2], q_empty[2], info_full[4], info_empty[4];
-    uint64_t sdp_full, sdp_free, pds_full, half_done, fin;
+    uint64_t sdp_full[2], pds_full[2], fin;   // per TMEM buffer
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -463,8 +478,10 @@ constexpr int kDkvOffList = kDkvOffInfo + kInfoStages * 4 * kRows * 4;
 constexpr int kDkvListCap = 2048;
 constexpr int kDkvOffCtl = kDkvOffList + 3 * kDkvListCap * 4;   // order, tiles, positions
 constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
-// TMEM: dV [0,128), dK [128,256), S^T [256,320), dP^T [320,384), P^T [384,416), dS^T [416,448)
-constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemST = 256, kTmemDPT = 320, kTmemPT = 384, kTmemDST = 416;
+// TMEM: dV [0,128), dK [128,256), then two buffers b of 128 columns at 256 + 128 b:
+// S^T in the first 64, dP^T in the last 64.  The keys write P^T (dS^T) in place
+// over the first 32 columns of the S^T (dP^T) they have read.
+constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemBuf = 256, kTmemST = 0, kTmemDPT = 64;
 
 __global__ void __launch_bounds__(kThreadsD, 1)
 bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
@@ -489,10 +506,10 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             mbar_init(&ctl.info_full[s], 1);                // the row-information warp
             mbar_init(&ctl.info_empty[s], kWorkers / 32);   // one arrive per key warp
         }
-        mbar_init(&ctl.sdp_full, 2);          // S^T from the first issuer, dP^T from the second
-        mbar_init(&ctl.sdp_free, kWorkers / 32);
-        mbar_init(&ctl.pds_full, kWorkers / 32);
-        mbar_init(&ctl.half_done, 2);         // dV and dK
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&ctl.sdp_full[b], 2);   // S^T from the first issuer, dP^T from the second
+            mbar_init(&ctl.pds_full[b], kWorkers / 32);
+        }
         mbar_init(&ctl.fin, 2);
         ctl.abort_flag = 0;
         fence_barrier_init();
@@ -578,56 +595,71 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             }
         }
     } else if (warp == 4 || warp == 7) {
-        if (lane == 0) {
-            // ---- issuers: warp 4 issues S^T = K Q^T and dV += P^T dO; warp 7
-            // issues dP^T = V dO^T and dK += dS^T Q.  The products of half x+1
-            // go in as soon as the keys have read those of half x; the
-            // accumulations of half x once its P^T, dS^T are written.
+        {
+            // ---- issuers (whole warp; the elected lane issues): warp 4 issues
+            // S^T = K Q^T and dV += P^T dO; warp 7 issues dP^T = V dO^T and
+            // dK += dS^T Q.  Half x uses TMEM buffer x & 1: its products go in
+            // two halves ahead, right behind the accumulation of half x - 2
+            // (which reads P^T / dS^T from that buffer); its accumulation once
+            // the keys have written P^T, dS^T.
             const bool first = warp == 4;
             constexpr uint32_t IDESC_T = idesc_bf16(2 * kKeys, 64, 0, 0);   // M = 128 keys, N = 64 rows
             constexpr uint32_t IDESC_ACC = idesc_bf16(2 * kKeys, kD, 0, 1);
-            // A operand (K or V of the pair) and the TMEM targets of this issuer
+            // A operand (K or V of the pair) and this issuer's columns of the buffers
             const uint32_t ab = smem_u32(smem + (first ? 0 : kDkvOffV));
-            const uint32_t t_prod = tmem + (first ? kTmemST : kTmemDPT);
+            const uint32_t t_own = tmem + kTmemBuf + (first ? kTmemST : kTmemDPT);
             const uint32_t t_acc = tmem + (first ? kTmemDV : kTmemDK);
-            const uint32_t t_a2 = tmem + (first ? kTmemPT : kTmemDST);
-            bool ok = mbar_wait(&ctl.kv_full, 0, wc, kSleepNs);
+            bool ok = mbar_wait_warp(&ctl.kv_full, 0, wc, kSleepNs);
             auto issue_prod = [&](int x) -> bool {
                 const int q = x >> 1, h = x & 1, s = q & 1;
-                if (h == 0 && !mbar_wait(&ctl.q_full[s], (q >> 1) & 1, wc, kSleepNs)) return false;
+                if (h == 0 && !mbar_wait_warp(&ctl.q_full[s], (q >> 1) & 1, wc, kSleepNs)) return false;
                 tc_fence_after();
                 // B operand: Q (first issuer) or dO rows of this half, K-major
                 const uint32_t bb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes) + (first ? 0 : kQBytes);
+                const uint32_t dst = t_own + (x & 1) * 128;
+                if (elect_one()) {
 #pragma unroll
-                for (int k = 0; k < kD / 16; ++k) {
-                    const uint32_t oa = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
-                    const uint32_t ob = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
-                    umma_bf16(t_prod, smem_desc_sw128(ab + oa, 16, 1024), smem_desc_sw128(bb + ob, 16, 1024), IDESC_T,
-                              k > 0);
+                    for (int k = 0; k < kD / 16; ++k) {
+                        const uint32_t oa = (k >> 2) * (2 * kKeys * 128) + (k & 3) * 32;
+                        const uint32_t ob = (k >> 2) * (kRows * 128) + h * 64 * 128 + (k & 3) * 32;
+                        umma_bf16(dst, smem_desc_sw128(ab + oa, 16, 1024), smem_desc_sw128(bb + ob, 16, 1024),
+                                  IDESC_T, k > 0);
+                    }
+                    umma_commit(&ctl.sdp_full[x & 1]);
                 }
-                umma_commit(&ctl.sdp_full);
+                __syncwarp();
                 return true;
             };
             if (ok) ok = issue_prod(0);
+            if (ok && nh > 1) ok = issue_prod(1);
             for (int x = 0; ok && x < nh; ++x) {
-                const int q = x >> 1, h = x & 1, s = q & 1;
-                if (!mbar_wait(&ctl.sdp_free, x & 1, wc, kSleepNs)) { ok = false; break; }
-                if (x + 1 < nh && !issue_prod(x + 1)) { ok = false; break; }
-                if (!mbar_wait(&ctl.pds_full, x & 1, wc, kSleepNs)) { ok = false; break; }
+                const int q = x >> 1, h = x & 1, s = q & 1, b = x & 1;
+                if (!mbar_wait_warp(&ctl.pds_full[b], (x >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
                 tc_fence_after();
                 // B operand: dO (first issuer, for dV) or Q (for dK) rows of this half, MN-major
                 const uint32_t bb = smem_u32(smem + kDkvOffQ + s * 2 * kQBytes) + (first ? kQBytes : 0);
+                const uint32_t a2 = t_own + b * 128;   // P^T or dS^T, in place
+                if (elect_one()) {
 #pragma unroll
-                for (int k = 0; k < 64 / 16; ++k) {
-                    const uint32_t ob = h * 64 * 128 + k * 2048;   // 16 rows = two 8-row atoms
-                    umma_bf16_ta(t_acc, t_a2 + k * 8, smem_desc_sw128(bb + ob, kRows * 128, 1024), IDESC_ACC,
-                                 (x > 0 || k > 0) ? 1u : 0u);
+                    for (int k = 0; k < 64 / 16; ++k) {
+                        const uint32_t ob = h * 64 * 128 + k * 2048;   // 16 rows = two 8-row atoms
+                        umma_bf16_ta(t_acc, a2 + k * 8, smem_desc_sw128(bb + ob, kRows * 128, 1024), IDESC_ACC,
+                                     (x > 0 || k > 0) ? 1u : 0u);
+                    }
+                    if (h == 1) umma_commit(&ctl.q_empty[s]);
                 }
-                umma_commit(&ctl.half_done);
-                if (h == 1) umma_commit(&ctl.q_empty[s]);
+                __syncwarp();
+                // The products of half x + 2 overwrite the columns this accumulation
+                // reads: MMAs of one thread (elect.sync of a full warp always picks
+                // its lowest lane) run in issue order through the tensor pipe, so
+                // they are issued right behind it without a wait.
+                if (x + 2 < nh && !issue_prod(x + 2)) { ok = false; break; }
             }
-            umma_commit(&ctl.fin);
-            mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            if (elect_one()) {
+                umma_commit(&ctl.fin);
+                mbar_wait_drain(&ctl.fin, 0, p.limit, p.status);
+            }
+            __syncwarp();
         }
     } else {
         // ---- keys: thread = key of the pair (TMEM lane)
@@ -637,19 +669,18 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
         bool ok = true;
         for (int x = 0; x < nh; ++x) {
-            const int q = x >> 1, h = x & 1, si = q % kInfoStages;
+            const int q = x >> 1, h = x & 1, si = q % kInfoStages, b = x & 1;
             const float* inf = info + si * 4 * kRows;
+            const uint32_t buf = lane_addr + kTmemBuf + b * 128;
             if (h == 0 && !mbar_wait_warp(&ctl.info_full[si], (q / kInfoStages) & 1, wc, kSleepNs)) { ok = false; break; }
-            if (!mbar_wait_warp(&ctl.sdp_full, x & 1, wc, kSleepNs)) { ok = false; break; }
+            if (!mbar_wait_warp(&ctl.sdp_full[b], (x >> 1) & 1, wc, kSleepNs)) { ok = false; break; }
             tc_fence_after();
             uint32_t sv[64], dv[64];
-            tmem_ld32(lane_addr + kTmemST, *reinterpret_cast<uint32_t(*)[32]>(sv));
-            tmem_ld32(lane_addr + kTmemST + 32, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
-            tmem_ld32(lane_addr + kTmemDPT, *reinterpret_cast<uint32_t(*)[32]>(dv));
-            tmem_ld32(lane_addr + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
+            tmem_ld32(buf + kTmemST, *reinterpret_cast<uint32_t(*)[32]>(sv));
+            tmem_ld32(buf + kTmemST + 32, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
+            tmem_ld32(buf + kTmemDPT, *reinterpret_cast<uint32_t(*)[32]>(dv));
+            tmem_ld32(buf + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
             tmem_wait_ld();
-            tc_fence_before();
-            mbar_arrive_warp(&ctl.sdp_free);   // S^T, dP^T may be overwritten by the next half
             uint32_t pp[32], dd[32];
             // In the diagonal tile (the first of the list) the rows of half h have
             // block 2pr + h as their own block: keys of that block are causal.
@@ -675,14 +706,12 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 pp[k >> 1] = pack_bf16x2(p0, p1);
                 dd[k >> 1] = pack_bf16x2(a0, a1);
             }
-            // P^T / dS^T columns are free once the previous half's products have read them
-            if (x >= 1 && !mbar_wait_warp(&ctl.half_done, (x - 1) & 1, wc, kSleepNs)) { ok = false; break; }
-            tc_fence_after();
-            tmem_st32(lane_addr + kTmemPT, pp);
-            tmem_st32(lane_addr + kTmemDST, dd);
+            // P^T and dS^T over the S^T and dP^T columns just read
+            tmem_st32(buf + kTmemST, pp);
+            tmem_st32(buf + kTmemDPT, dd);
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive_warp(&ctl.pds_full);
+            mbar_arrive_warp(&ctl.pds_full[b]);
             if (h == 1) mbar_arrive_warp(&ctl.info_empty[si]);
         }
         if (ok && mbar_wait_warp(&ctl.fin, 0, wc, kSleepNs)) {
