@@ -751,53 +751,83 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
 // --------------------------------------------------------- score gradient
 
 // ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of the row's C_i
-// given scores; 0 past the history.  One CTA per run of R consecutive rows
-// (their score rows are contiguous): the row's log-normaliser comes back from
-// its first kept entry (log g_m = s_m - LSE of the scores, Eq.
-// normalized_log_gate), the kept dlogg values are scattered into shared
-// memory, and the R x C outputs go out in one coalesced sweep.
+// given scores; 0 past the history.  One warp per row, every load of the row
+// issued first (the row's scores are held in registers when C <= 32 NCH):
+// the log-normaliser comes back from the first kept entry (log g_m = s_m -
+// LSE of the scores, Eq. normalized_log_gate), the kept dlogg values are
+// scattered into the warp's C floats of shared memory.
+template <int NCH>
 __global__ void __launch_bounds__(256)
 bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg, const float* dlogg, float* ds,
-              long long rows, int N, int C, int topk, int R, int train) {
-    extern __shared__ float dsh[];   // [R][C] kept dlogg, then R normalisers and R sums
-    float* add = dsh;
-    float* rlse = dsh + static_cast<long long>(R) * C;
-    float* rsum = rlse + R;
-    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const long long w0 = static_cast<long long>(blockIdx.x) * R;
-    const int nr = static_cast<int>(min(static_cast<long long>(R), rows - w0));
-    const int tot = nr * C;
-    for (int k = t; k < tot; k += blockDim.x) add[k] = 0.f;
-    __syncthreads();
-    for (int rr = warp; rr < nr; rr += blockDim.x >> 5) {
-        const long long w = w0 + rr;
-        const int c = static_cast<int>(w % N) >> 6;
-        const int nsel = train ? min(topk, c) : 0;
-        float sum = 0.f;
-        for (int e = lane; e < nsel; e += 32) {
-            const float v = __ldg(dlogg + w * topk + e);
-            sum += v;
-            add[rr * C + __ldg(sel_idx + w * topk + e)] = v;   // kept blocks are distinct
-        }
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-        if (lane == 0) {
-            rsum[rr] = sum;
-            rlse[rr] = nsel > 0 ? __ldg(scores + w * C + __ldg(sel_idx + w * topk)) - __ldg(sel_logg + w * topk) : 0.f;
+              long long rows, int N, int C, int topk, int train) {
+    extern __shared__ float dsh[];   // per warp: C floats (the row's kept dlogg, scattered)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long w = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + warp;
+    if (w >= rows) return;           // no block-wide synchronisation below
+    float* add = dsh + warp * C;
+    const int c = static_cast<int>(w % N) >> 6;
+    const int nsel = train ? min(topk, c) : 0;
+    const float* s = scores + w * C;
+    float* out = ds + w * C;
+    float sv[NCH > 0 ? NCH : 1];
+    if (NCH > 0) {
+#pragma unroll
+        for (int q = 0; q < NCH; ++q) {
+            const int m = lane + 32 * q;
+            sv[q] = m < c ? __ldg(s + m) : 0.f;
         }
     }
-    __syncthreads();
-    const float* s = scores + w0 * C;
-    float* out = ds + w0 * C;
-    for (int k = t; k < tot; k += blockDim.x) {
-        const int rr = k / C, m = k - rr * C;
-        const int c = static_cast<int>((w0 + rr) % N) >> 6;
-        float v = 0.f;
-        if (m < c) {
-            v = add[k];
-            const float sm = rsum[rr];
-            if (sm != 0.f) v -= __expf(__ldg(s + k) - rlse[rr]) * sm;
+    const int32_t* ix = sel_idx + w * topk;
+    const float* dl = dlogg + w * topk;
+    const float v0 = lane < nsel ? __ldg(dl + lane) : 0.f;
+    const int i0 = lane < nsel ? __ldg(ix + lane) : 0;
+    const float lg0 = nsel > 0 ? __ldg(sel_logg + w * topk) : 0.f;
+    for (int m = lane; m < C; m += 32) add[m] = 0.f;
+    __syncwarp();
+    float sum = v0;
+    if (lane < nsel) add[i0] = v0;   // kept blocks are distinct
+    for (int e = lane + 32; e < nsel; e += 32) {
+        const float v = __ldg(dl + e);
+        sum += v;
+        add[__ldg(ix + e)] = v;
+    }
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    // LSE = s_m0 - log g_m0 for the first kept block m0 (< c, so in registers)
+    const int m0 = __shfl_sync(0xffffffffu, i0, 0);
+    float s0;
+    if (NCH > 0) {
+        float mine = 0.f;
+#pragma unroll
+        for (int q = 0; q < NCH; ++q)
+            if (q == (m0 >> 5)) mine = sv[q];
+        s0 = __shfl_sync(0xffffffffu, mine, m0 & 31);
+    } else {
+        s0 = nsel > 0 ? __ldg(s + m0) : 0.f;
+    }
+    const float lse = s0 - lg0;
+    __syncwarp();
+    if (NCH > 0) {
+#pragma unroll
+        for (int q = 0; q < NCH; ++q) {
+            const int m = lane + 32 * q;
+            if (m < C) {
+                float v = 0.f;
+                if (m < c) {
+                    v = add[m];
+                    if (sum != 0.f) v -= __expf(sv[q] - lse) * sum;
+                }
+                out[m] = v;
+            }
         }
-        out[k] = v;
+    } else {
+        for (int m = lane; m < C; m += 32) {
+            float v = 0.f;
+            if (m < c) {
+                v = add[m];
+                if (sum != 0.f) v -= __expf(__ldg(s + m) - lse) * sum;
+            }
+            out[m] = v;
+        }
     }
 }
 
@@ -890,10 +920,20 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
         const long long rows = static_cast<long long>(a.BH) * a.N;
-        const int R = max(1, min(32, 8192 / a.C));   // <= 32 KB of shared memory
-        const size_t sh = (static_cast<size_t>(R) * a.C + 2 * R) * sizeof(float);
-        bwd_ds_kernel<<<static_cast<unsigned>((rows + R - 1) / R), 256, sh, env.stream>>>(
-            a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows, a.N, a.C, a.topk, R, a.mode == 0 ? 1 : 0);
+        // one warp per row, at most 32 KB of shared memory per CTA
+        const int wpc = max(1, min(8, 8192 / a.C));
+        const size_t sh = static_cast<size_t>(wpc) * a.C * sizeof(float);
+        const unsigned grid = static_cast<unsigned>((rows + wpc - 1) / wpc);
+        const int train = a.mode == 0 ? 1 : 0;
+        if (a.C <= 128)
+            bwd_ds_kernel<4><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
+                                                                 a.N, a.C, a.topk, train);
+        else if (a.C <= 384)
+            bwd_ds_kernel<12><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
+                                                                  a.N, a.C, a.topk, train);
+        else
+            bwd_ds_kernel<0><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
+                                                                 a.N, a.C, a.topk, train);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     } else if (a.ds != nullptr) {
