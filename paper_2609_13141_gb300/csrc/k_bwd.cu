@@ -759,13 +759,16 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
 template <int NCH>
 __global__ void __launch_bounds__(256)
 bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg, const float* dlogg, float* ds,
-              long long rows, int N, int C, int topk, int train) {
+              int N, int C, int topk, int train, int chunks) {
     extern __shared__ float dsh[];   // per warp: C floats (the row's kept dlogg, scattered)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const long long w = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + warp;
-    if (w >= rows) return;           // no block-wide synchronisation below
+    // CTA = (head, run of blockDim / 32 rows of it): one division per CTA
+    const int bh = static_cast<int>(blockIdx.x / static_cast<unsigned>(chunks));
+    const int i = static_cast<int>(blockIdx.x - static_cast<unsigned>(bh) * chunks) * (blockDim.x >> 5) + warp;
+    if (i >= N) return;              // no block-wide synchronisation below
+    const long long w = static_cast<long long>(bh) * N + i;
     float* add = dsh + warp * C;
-    const int c = static_cast<int>(w % N) >> 6;
+    const int c = i >> 6;
     const int nsel = train ? min(topk, c) : 0;
     const float* s = scores + w * C;
     float* out = ds + w * C;
@@ -919,21 +922,21 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
-        const long long rows = static_cast<long long>(a.BH) * a.N;
         // one warp per row, at most 32 KB of shared memory per CTA
         const int wpc = max(1, min(8, 8192 / a.C));
         const size_t sh = static_cast<size_t>(wpc) * a.C * sizeof(float);
-        const unsigned grid = static_cast<unsigned>((rows + wpc - 1) / wpc);
+        const int chunks = (a.N + wpc - 1) / wpc;
+        const unsigned grid = static_cast<unsigned>(static_cast<long long>(a.BH) * chunks);
         const int train = a.mode == 0 ? 1 : 0;
         if (a.C <= 128)
-            bwd_ds_kernel<4><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
-                                                                 a.N, a.C, a.topk, train);
+            bwd_ds_kernel<4><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
+                                                                 a.C, a.topk, train, chunks);
         else if (a.C <= 384)
-            bwd_ds_kernel<12><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
-                                                                  a.N, a.C, a.topk, train);
+            bwd_ds_kernel<12><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
+                                                                  a.C, a.topk, train, chunks);
         else
-            bwd_ds_kernel<0><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, rows,
-                                                                 a.N, a.C, a.topk, train);
+            bwd_ds_kernel<0><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
+                                                                 a.C, a.topk, train, chunks);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     } else if (a.ds != nullptr) {
