@@ -285,6 +285,29 @@ def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
     return out
 
 
+def sas_attention_gqa(Q, K, V, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                      heads=None, rows=None, act=GATE_SOFTMAX, pos=GATE_INNER):
+    """GQA form with group-shared selection (Sec. 5.3: the query heads of a
+    GQA group share one Top-K; Sec. 5 inference implementation: Top-K per
+    query group).  Q [B, Hq, N, d]; K, V [B, Hkv, N, d]; scores
+    [B, Hkv, N, >=C-1], one table per KV group; Hq = G Hkv, query head h
+    belongs to group h // G.  Every query head attends with its group's K,
+    V, kept blocks and log-gates.  Returns {(bi, h): result-dict}.
+    """
+    Bn, Hq, N, d = Q.shape
+    Hkv = K.shape[1]
+    if Hq % Hkv:
+        raise ValueError("Hq must be a multiple of Hkv")
+    G = Hq // Hkv
+    heads = [(bi, hi) for bi in range(Bn) for hi in range(Hq)] if heads is None else heads
+    out = {}
+    for bi, hi in heads:
+        g = hi // G
+        out[(bi, hi)] = sas_attention_head(Q[bi, hi], K[bi, g], V[bi, g], scores[bi, g], b,
+                                           topk, mode, sm_scale, rows, act, pos)
+    return out
+
+
 # -------------------------------------------------------------------- a6 --
 
 def gelu(x):
