@@ -93,6 +93,12 @@ typedef struct {
     int32_t d_sel;        /* selector dim d_sel in {64, 128}; 0 selects d             */
     int32_t gate_act;     /* sas_gate_act (0 = SOFTMAX, the SAS default)               */
     int32_t gate_pos;     /* sas_gate_pos (0 = INNER, the SAS default)                 */
+    int32_t Hkv;          /* KV heads (GQA); 0 selects H.  H must be a multiple of it:
+                             query head h uses KV head h / (H / Hkv), and the G = H / Hkv
+                             query heads of a group share one selection (Sec. 5.3;
+                             Sec. 5 inference implementation).  Hkv < H needs
+                             SCORES_GIVEN (one score table per group) and has no
+                             backward.                                                */
 } sas_config;
 
 typedef struct sas_handle sas_handle;
@@ -110,8 +116,9 @@ void sas_destroy(sas_handle* h);
  * with the fused-kernel structure of Alg. 3 (skip blocks no query in a tile
  * keeps, online softmax, O and LSE outputs).
  *
- *   Q, K, V   bf16 [B, H, N, d]                                       (in)
- *   scores    fp32 [B, H, N, C], C = ceil(N / 64); row i reads entries
+ *   Q         bf16 [B, H, N, d]                                       (in)
+ *   K, V      bf16 [B, Hkv, N, d] (Hkv = H without GQA)               (in)
+ *   scores    fp32 [B, Hkv, N, C], C = ceil(N / 64); row i reads entries
  *             0 .. floor(i/64)-1 and ignores the rest.  Required for
  *             SCORES_GIVEN, must be NULL for MEANPOOL_PROJ.  Scores must
  *             be finite.                                              (in)
@@ -121,9 +128,10 @@ void sas_destroy(sas_handle* h);
  *   O         bf16 [B, H, N, d]                                       (out)
  *   LSE       fp32 [B, H, N] natural-log log-sum-exp of each row's
  *             gated logits (Alg. 3 output); may be NULL.              (out)
- *   sel_idx   int32 [B, H, N, topk]: each row's kept historical blocks in
- *             ascending order, padded with -1; may be NULL.           (out)
- *   sel_logg  fp32 [B, H, N, topk]: log g of the kept blocks under the
+ *   sel_idx   int32 [B, Hkv, N, topk]: each row's kept historical blocks
+ *             (per group) in ascending order, padded with -1; may be
+ *             NULL.                                                   (out)
+ *   sel_logg  fp32 [B, Hkv, N, topk]: log g of the kept blocks under the
  *             handle's gate activation (same order, 0 where padded);
  *             may be NULL.                                            (out)
  *
@@ -246,7 +254,8 @@ int64_t sas_launch_count(const sas_handle* h);
 /* Copies the per-tile count of historical blocks the attention kernel
  * processes (the union of the kept blocks of the tile's 128 query rows,
  * excluding the tile's own two diagonal blocks) from the last
- * sas_attention_fwd: out[B * H * ceil(N/128)].  Synchronises. */
+ * sas_attention_fwd: out[B * Hkv * ceil(N/128)] (one per KV group and
+ * tile).  Synchronises. */
 sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n);
 
 /* Failure-path self-test: launches one block that waits on an mbarrier that

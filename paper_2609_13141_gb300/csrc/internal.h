@@ -78,7 +78,8 @@ struct AttnArgs {
     const int32_t* union_cnt;
     const int32_t* sel_idx;
     const float* sel_logg;
-    int BH, N, d, C, T, topk, mode;
+    int BH, N, d, C, T, topk, mode;    // BH: query heads x batch
+    int G;                      // query heads per KV group (1 without GQA): K, V, lists of group bh / G
     int gate_pos;               // 0 inner (+ log g in the logits), 1 outer (g scales P after the softmax)
     float sm_scale;
     int* sched;                 // 16 zeroed bytes owned by the caller, left zeroed after each launch

@@ -90,7 +90,8 @@ struct AttnParams {
     const int32_t* sel_idx;
     const float* sel_logg;
     int N, C, T, BH, topk, mode;
-    int group;              // heads per group of the work list
+    int G;                  // query heads per KV group: K, V and the lists of head bh are group bh / G
+    int group;              // heads per group of the work list (a multiple of G)
     int* sched;             // [0] next work item, [1] CTAs finished; both zero between launches
     float scale_log2;
     int* status;
@@ -104,9 +105,11 @@ struct AttnParams {
 // producer takes the next item from a global counter when it starts a tile
 // (tile costs vary with their union lists, so a fixed split would leave SMs
 // idle) and passes it to the CTA's other roles through a small shared ring.
+// With GQA the G query heads of a KV group are adjacent in that order, so they
+// run the same tile at about the same time over the same K, V blocks.
 
 struct TileRef {
-    int t, bh;
+    int t, bh, kv;          // tile, query head, KV group (= bh without GQA)
     const int32_t* ulist;   // the tile's union list (ascending historical blocks)
     int U;                  // its length
 };
@@ -120,7 +123,8 @@ __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w) {
     const int wi = w - g0 * per_group;
     x.t = p.T - 1 - wi / gs;
     x.bh = h0 + wi % gs;
-    const long long tb = static_cast<long long>(x.bh) * p.T + x.t;
+    x.kv = x.bh / p.G;
+    const long long tb = static_cast<long long>(x.kv) * p.T + x.t;
     x.ulist = p.union_idx + tb * p.C;
     x.U = __ldg(p.union_cnt + tb);
     return x;
@@ -234,7 +238,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
 #pragma unroll
                 for (int a = 0; a < D / 64; ++a)
-                    tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, x.bh);
+                    tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, x.kv);
                 ++nk;
             }
             g += n;
@@ -275,7 +279,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
 #pragma unroll
                 for (int a = 0; a < D / 64; ++a)
-                    tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, x.bh);
+                    tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, x.kv);
                 ++nv;
             }
             g += n;
@@ -382,9 +386,10 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             const bool valid = i < p.N;
             const int c = i >> 6;
             const int nsel = valid ? min(p.topk, c) : 0;
-            const long long row_off = static_cast<long long>(x.bh) * p.N + i;
-            const int32_t* my_idx = p.sel_idx + row_off * p.topk;
-            const float* my_lg = p.sel_logg + row_off * p.topk;
+            const long long row_off = static_cast<long long>(x.bh) * p.N + i;   // O, LSE
+            const long long sel_off = static_cast<long long>(x.kv) * p.N + i;   // the group's kept list
+            const int32_t* my_idx = p.sel_idx + sel_off * p.topk;
+            const float* my_lg = p.sel_logg + sel_off * p.topk;
             // The row's kept list is staged kRing entries ahead in a shared ring
             // (entry e in slot e % kRing, one commit group per entry), so the walk
             // below only reads entries that have landed long ago.  Every entry of
@@ -613,8 +618,9 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     if (e != cudaSuccess) { *err = "device attributes"; return e; }
     CUtensorMap mq, mk, mv;
     if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kBM) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
-    if (make_tmap_bf16_3d(&mk, a.K, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
-    if (make_tmap_bf16_3d(&mv, a.V, D, a.N, a.BH, 64, kBN) != 0) { *err = "tensor map V"; return cudaErrorInvalidValue; }
+    const int BHkv = a.BH / a.G;
+    if (make_tmap_bf16_3d(&mk, a.K, D, a.N, BHkv, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mv, a.V, D, a.N, BHkv, 64, kBN) != 0) { *err = "tensor map V"; return cudaErrorInvalidValue; }
     AttnParams p;
     p.O = static_cast<bf16*>(a.O);
     p.LSE = a.LSE;
@@ -623,10 +629,13 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.sel_idx = a.sel_idx;
     p.sel_logg = a.sel_logg;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
-    // heads whose K and V (2 * N * d bf16 each) fit in half of L2 together, at least one
+    p.G = a.G;
+    // KV groups whose K and V (2 * N * d bf16 each) fit in half of L2 together,
+    // at least one; the work list takes their G query heads each
     const long long kv_head = 4LL * a.N * D;
-    const long long fit = kv_head > 0 ? (static_cast<long long>(l2) / 2) / kv_head : a.BH;
-    p.group = static_cast<int>(fit < 1 ? 1 : (fit > a.BH ? a.BH : fit));
+    const long long fit = kv_head > 0 ? (static_cast<long long>(l2) / 2) / kv_head : BHkv;
+    const long long groups = fit < 1 ? 1 : (fit > BHkv ? BHkv : fit);
+    p.group = static_cast<int>(groups * a.G);
     p.scale_log2 = a.sm_scale * kLog2e;
     p.status = env.status;
     p.limit = env.limit;
@@ -643,6 +652,10 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
 }  // namespace
 
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err) {
+    if (a.G < 1 || a.BH % a.G != 0) {
+        *err = "attention: query heads must fill whole KV groups";
+        return cudaErrorInvalidValue;
+    }
     const bool outer = a.gate_pos == 1;
     if (a.d == 128) return outer ? launch_d<128, true>(a, env, err) : launch_d<128, false>(a, env, err);
     if (a.d == 64) return outer ? launch_d<64, true>(a, env, err) : launch_d<64, false>(a, env, err);

@@ -91,6 +91,7 @@ struct sas_handle {
     int d_sel = 0;
     float sm_scale = 0.f;
     int BH = 0, C = 0, T = 0, F = 0;
+    int Hkv = 0, G = 1, BHkv = 0;   // KV heads, query heads per group, KV groups x batch
     // workspace
     void* Kt = nullptr;         // bf16 [BH][max(F,1)][d_sel]
     int32_t* union_idx = nullptr;
@@ -219,7 +220,11 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (!(c.sm_scale >= 0.f) || !std::isfinite(c.sm_scale)) return SAS_ERR_INVALID_ARG;
     const int d_sel = c.d_sel == 0 ? c.d : c.d_sel;
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
+    const int Hkv = c.Hkv == 0 ? c.H : c.Hkv;
+    if (Hkv < 1 || Hkv > c.H || c.H % Hkv != 0) return SAS_ERR_INVALID_ARG;
+    if (Hkv != c.H && c.selector != SAS_SEL_SCORES_GIVEN) return SAS_ERR_UNSUPPORTED;
     const long long BH = static_cast<long long>(c.B) * c.H;
+    const long long BHkv = static_cast<long long>(c.B) * Hkv;
     if (BH > (1LL << 30) || BH * c.N > (1LL << 40)) return SAS_ERR_UNSUPPORTED;
     if (BH * ((c.N + 127) / 128) > 0x7fffffffLL) return SAS_ERR_UNSUPPORTED;   // (head, tile) pairs index a 1-D grid
 
@@ -228,6 +233,9 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     h->d_sel = d_sel;
     h->sm_scale = c.sm_scale > 0.f ? c.sm_scale : 1.0f / std::sqrt(static_cast<float>(c.d));
     h->BH = static_cast<int>(BH);
+    h->Hkv = Hkv;
+    h->G = c.H / Hkv;
+    h->BHkv = static_cast<int>(BHkv);
     h->C = (c.N + 63) / 64;
     h->T = (c.N + 127) / 128;
     h->F = c.N / 64;
@@ -236,12 +244,12 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     cudaGetDevice(&h->device);
 
     cudaError_t e = cudaSuccess;
-    const size_t rows = static_cast<size_t>(BH) * c.N;
+    const size_t rows = static_cast<size_t>(BHkv) * c.N;   // selection rows: one per group and token
     if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
         if (e == cudaSuccess) e = alloc(&h->Kt, static_cast<size_t>(BH) * (h->F > 0 ? h->F : 1) * d_sel * 2);
     }
-    if (e == cudaSuccess) e = alloc(&h->union_idx, static_cast<size_t>(BH) * h->T * h->C * 4);
-    if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BH) * h->T * 4);
+    if (e == cudaSuccess) e = alloc(&h->union_idx, static_cast<size_t>(BHkv) * h->T * h->C * 4);
+    if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BHkv) * h->T * 4);
     if (e == cudaSuccess) e = alloc(&h->sel_idx, rows * (c.topk > 0 ? c.topk : 1) * 4);
     if (e == cudaSuccess) e = alloc(&h->sel_logg, rows * (c.topk > 0 ? c.topk : 1) * 4);
     if (e == cudaSuccess) e = alloc(&h->status, 16);
@@ -313,7 +321,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     }
     // a2-a4: query projection (learned selector), scores, log-gates, Top-K, tile unions
     sas::SelectArgs sa{};
-    sa.BH = h->BH; sa.H = c.H; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.BH = h->BHkv; sa.H = h->Hkv; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
     sa.gate_act = c.gate_act;
     sa.score_scale = c.selector == SAS_SEL_MEANPOOL_PROJ ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
     sa.scores = scores;
@@ -328,6 +336,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
     aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.G = h->G;
     aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
     aa.sched = h->sched;
@@ -398,6 +407,7 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     if (c.d != 128) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports d = 128");
     if (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER)
         return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
+    if (h->G != 1) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports Hkv = H");
     if (h->T > sas::kBwdMaxTiles) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports N <= 262016");
     if (dscores) {
         if (c.selector != SAS_SEL_SCORES_GIVEN || !scores)
@@ -503,7 +513,7 @@ int64_t sas_launch_count(const sas_handle* h) { return h ? h->launches : 0; }
 
 sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n) {
     if (h == nullptr || host_out == nullptr) return SAS_ERR_INVALID_ARG;
-    const int64_t total = static_cast<int64_t>(h->BH) * h->T;
+    const int64_t total = static_cast<int64_t>(h->BHkv) * h->T;   // one union list per KV group and tile
     if (n < total) return fail(h, SAS_ERR_INVALID_ARG, "output too small");
     cudaError_t e = cudaDeviceSynchronize();
     if (e == cudaSuccess) e = cudaMemcpy(host_out, h->union_cnt, total * 4, cudaMemcpyDeviceToHost);

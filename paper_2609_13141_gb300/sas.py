@@ -43,7 +43,7 @@ class SasConfig(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("d", ctypes.c_int32),
                 ("block", ctypes.c_int32), ("topk", ctypes.c_int32), ("sm_scale", ctypes.c_float),
                 ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32),
-                ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32)]
+                ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32), ("Hkv", ctypes.c_int32)]
 
 
 class SasDecodeConfig(ctypes.Structure):
@@ -168,17 +168,17 @@ def sas_status_str(status):
 
 
 def sas_create(B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-               sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos)
+               sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv)
     h = ctypes.c_void_p()
     _check(lib().sas_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_create")
     return h
 
 
 def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64,
-                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
+                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
     """Raw status of sas_create (for argument-check tests); destroys the handle on success."""
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos)
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv)
     h = ctypes.c_void_p()
     st = lib().sas_create(ctypes.byref(cfg), ctypes.byref(h))
     if st == SAS_OK:
@@ -279,10 +279,11 @@ class SasLayer:
     """Owns one handle; allocates outputs and calls the C ABI."""
 
     def __init__(self, B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER):
+                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
         self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
+        self.Hkv = Hkv or H                      # kept lists are per KV group
         self.selector = selector
-        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos)
+        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv)
 
     def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
         dev = Q.device
@@ -291,8 +292,8 @@ class SasLayer:
         sel_idx = sel_logg = None
         if want_sel:
             k = max(self.topk, 1)
-            sel_idx = torch.empty(self.B, self.H, self.N, k, device=dev, dtype=torch.int32)
-            sel_logg = torch.empty(self.B, self.H, self.N, k, device=dev, dtype=torch.float32)
+            sel_idx = torch.empty(self.B, self.Hkv, self.N, k, device=dev, dtype=torch.int32)
+            sel_logg = torch.empty(self.B, self.Hkv, self.N, k, device=dev, dtype=torch.float32)
         sas_attention_fwd(self.h, Q, K, V, O, scores, Wq, Wk, LSE, sel_idx, sel_logg, stream)
         return O, LSE, sel_idx, sel_logg
 

@@ -49,6 +49,10 @@ def test_status_strings(lib):
     (dict(B=1, H=1, N=128, d=64, topk=2, gate_act=3), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=1, N=128, d=64, topk=2, gate_act=-1), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=1, N=128, d=64, topk=2, gate_pos=2), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=6, N=128, d=64, topk=2, Hkv=4), sas.SAS_ERR_INVALID_ARG),      # H not a multiple of Hkv
+    (dict(B=1, H=2, N=128, d=64, topk=2, Hkv=4), sas.SAS_ERR_INVALID_ARG),      # more KV heads than heads
+    (dict(B=1, H=2, N=128, d=64, topk=2, Hkv=-1), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=4, N=128, d=64, topk=2, Hkv=2, selector=1), sas.SAS_ERR_UNSUPPORTED),   # GQA needs given scores
 ])
 def test_create_rejects_bad_configs(lib, kw, expect):
     assert sas.sas_create_status(**kw) == expect

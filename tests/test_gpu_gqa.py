@@ -1,0 +1,102 @@
+"""GPU parity of the GQA forward (group-shared selection: the G query heads of
+a KV group share one score table, one Top-K and one set of tile unions;
+Sec. 5.3, Sec. 5 inference implementation) against the fp64 oracle, and
+bit-identity with the MHA path run on per-head repeated K, V and scores."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import sas_oracle as OR
+from paper_2609_13141_gb300 import sas, synth
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+
+TRAIN, INFER = sas.SAS_MODE_TRAIN_SOFT, sas.SAS_MODE_INFER_HARD
+
+
+def _inputs(B, Hq, Hkv, N, d, seed, regime="R1"):
+    Q = synth.qkv(B, Hq, N, d, seed=seed)[0]
+    _, K, V = synth.qkv(B, Hkv, N, d, seed=seed + 100)
+    S = synth.scores(B, Hkv, N, -(-N // 64), seed=seed, regime=regime)
+    return Q, K, V, S
+
+
+def _run(B, Hq, Hkv, N, d, topk, mode, Q, K, V, S):
+    layer = sas.SasLayer(B, Hq, N, d, topk, mode=mode, Hkv=Hkv)
+    dev = torch.device("cuda:0")
+    O, LSE, si, sl = layer.attention(*(t.to(dev).contiguous() for t in (Q, K, V)), scores=S.to(dev).contiguous())
+    T = -(-N // 128)
+    unions = np.array(sas.sas_get_tile_union_counts(layer.h, B * Hkv * T)).reshape(B, Hkv, T)
+    status = sas.sas_get_device_status(layer.h)
+    layer.close()
+    return {"O": O.cpu(), "LSE": LSE.cpu(), "sel_idx": si.cpu(), "sel_logg": sl.cpu(), "unions": unions,
+            "status": status}
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,N,d,topk,mode", [
+    (1, 8, 2, 700, 128, 4, TRAIN),     # G = 4, ragged tail, several tiles
+    (2, 6, 3, 389, 128, 2, INFER),     # G = 2, inference form
+    (1, 4, 1, 517, 64, 3, TRAIN),      # MQA (one KV head), d = 64
+])
+def test_gqa_matches_oracle(B, Hq, Hkv, N, d, topk, mode):
+    Q, K, V, S = _inputs(B, Hq, Hkv, N, d, seed=Hq + N)
+    g = _run(B, Hq, Hkv, N, d, topk, mode, Q, K, V, S)
+    assert g["status"] == 0
+    ref = OR.sas_attention_gqa(P.f64(Q), P.f64(K), P.f64(V), 64, topk, P.f64(S), mode=mode)
+    G = Hq // Hkv
+    for bi in range(B):
+        for hi in range(Hq):
+            r = ref[(bi, hi)]
+            gk = hi // G
+            if hi % G == 0:   # the group's kept lists, once per group
+                gi = g["sel_idx"][bi, gk].numpy()[:, :topk]
+                P.check_selection_rows(gi, P.f64(S[bi, gk]), np.arange(N), topk)
+                lg = g["sel_logg"][bi, gk].numpy()[:, :topk]
+                assert np.abs(lg - r["sel_logg"]).max(initial=0) <= P.LOGG_MAX_ABS
+                assert np.array_equal(g["unions"][bi, gk], P.oracle_union_counts(gi, N, topk))
+            P.compare_o(P.f64(g["O"][bi, hi]), r["O"], f"O[{bi},{hi}]", max(1.0, np.abs(r["O"]).max()))
+            assert np.abs(g["LSE"][bi, hi].numpy() - r["LSE"]).max() <= P.LSE_MAX_ABS
+
+
+def test_gqa_is_bit_identical_to_mha_on_repeated_inputs():
+    B, Hq, Hkv, N, d, topk = 2, 8, 2, 1100, 128, 5
+    G = Hq // Hkv
+    Q, K, V, S = _inputs(B, Hq, Hkv, N, d, seed=3)
+    g = _run(B, Hq, Hkv, N, d, topk, TRAIN, Q, K, V, S)
+    rep = lambda t: t.repeat_interleave(G, dim=1)
+    m = _run(B, Hq, Hq, N, d, topk, TRAIN, Q, rep(K), rep(V), rep(S))
+    assert g["status"] == 0 and m["status"] == 0
+    assert torch.equal(g["O"], m["O"])
+    assert torch.equal(g["LSE"], m["LSE"])
+    assert torch.equal(rep(g["sel_idx"]), m["sel_idx"])
+    assert torch.equal(rep(g["sel_logg"]), m["sel_logg"])
+
+
+def test_qwen3_4b_shaped_prefill_sampled_rows():
+    # Hq = 32, Hkv = 8 (G = 4), d = 128, K = 32, 8192 tokens: sampled rows of two heads
+    B, Hq, Hkv, N, d, topk = 1, 32, 8, 8192, 128, 32
+    Q, K, V, S = _inputs(B, Hq, Hkv, N, d, seed=5)
+    g = _run(B, Hq, Hkv, N, d, topk, TRAIN, Q, K, V, S)
+    assert g["status"] == 0
+    rows = P.sample_rows(N, 128, seed=1)
+    heads = [(0, 5), (0, 30)]
+    ref = OR.sas_attention_gqa(P.f64(Q), P.f64(K), P.f64(V), 64, topk, P.f64(S), heads=heads, rows=rows)
+    for (bi, hi), r in ref.items():
+        P.compare_o(P.f64(g["O"][bi, hi])[rows], r["O"], f"O[{bi},{hi}]", max(1.0, np.abs(r["O"]).max()))
+        assert np.abs(g["LSE"][bi, hi].numpy()[rows] - r["LSE"]).max() <= P.LSE_MAX_ABS
+        gi = g["sel_idx"][bi, hi // 4].numpy()[rows][:, :topk]
+        P.check_selection_rows(gi, P.f64(S[bi, hi // 4])[rows], rows, topk)
+
+
+def test_gqa_backward_is_refused():
+    layer = sas.SasLayer(1, 4, 256, 128, 2, Hkv=2)
+    dev = torch.device("cuda:0")
+    Q = torch.zeros(1, 4, 256, 128, device=dev, dtype=torch.bfloat16)
+    K = torch.zeros(1, 2, 256, 128, device=dev, dtype=torch.bfloat16)
+    S = torch.zeros(1, 2, 256, 4, device=dev)
+    O, LSE, si, sl = layer.attention(Q, K, K, scores=S)
+    with pytest.raises(sas.SasError) as e:
+        layer.attention_bwd(Q, K, K, O, LSE, O, scores=S, sel_idx=si, sel_logg=sl)
+    assert e.value.status == sas.SAS_ERR_UNSUPPORTED
+    layer.close()
