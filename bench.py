@@ -46,6 +46,11 @@ WORKLOADS = {
                   name="high-resolution causal SAS layer: B=1 H=24 N=16384+512 d=128 K=32, MLP 16896x3072->12288->3072"),
     "video": dict(B=1, H=24, N=75600 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
                   name="video-scale causal SAS layer: B=1 H=24 N=75600+512 d=128 K=32, MLP 76112x3072->12288->3072"),
+    # GQA prefill (group-shared selection from given scores, one table per KV group)
+    "qwen3_4b_prefill": dict(B=1, H=32, Hkv=8, N=32768, d=128, topk=32, d_sel=128, D=2560, F=9728,
+                             name="Qwen3-4B-shaped GQA prefill layer: B=1 Hq=32 Hkv=8 N=32768 d=128 b=64 K=32 "
+                                  "(2048-token budget), given R1 scores per KV group, GELU MLP "
+                                  "32768x2560->9728->2560 (in place of the model's SwiGLU MLP)"),
 }
 
 
@@ -185,16 +190,21 @@ def run_ours(args, w, rank, world):
         dist.init_process_group("nccl", device_id=dev)
 
     B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
+    Hkv = w.get("Hkv", H)
     T = B * N
-    learned = args.regime == "R2"
+    learned = args.regime == "R2" and Hkv == H   # GQA takes given scores (one table per KV group)
     if learned:
         # R2: block-correlated queries through the learned selector
         Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
         S = None
-    else:
+    elif Hkv == H:
         # R1: block-coherent selector scores supplied by the caller
         Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="iid")
         S = synth.scores(B, H, N, (N + 63) // 64, seed=rank, regime="R1")
+    else:
+        Q = synth.qkv(B, H, N, d, seed=rank, regime="iid")[0]
+        _, Kk, V = synth.qkv(B, Hkv, N, d, seed=rank + 100, regime="iid")
+        S = synth.scores(B, Hkv, N, (N + 63) // 64, seed=rank, regime="R1")
     Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
     X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
     Qd, Kd, Vd, Wqd, Wkd = (t.to(dev) for t in (Q, Kk, V, Wq, Wk))
@@ -208,7 +218,7 @@ def run_ours(args, w, rank, world):
     if learned:
         layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
     else:
-        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN)
+        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv)
     h = layer.h
     stream = torch.cuda.current_stream(dev)
 
@@ -281,7 +291,7 @@ def run_ours(args, w, rank, world):
 
     # tile-union statistics of the last forward (executed vs algorithmic work)
     Tt = (N + 127) // 128
-    unions = sas.sas_get_tile_union_counts(h, B * H * Tt)
+    unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
     layer.close()
 
     ms, e2e_ms = reduce_max([ms, e2e_ms], dist, dev)
@@ -314,7 +324,8 @@ def run_ours(args, w, rank, world):
         "data": ("synthetic (seeded; R2 block-correlated queries, N(0,1) K/V/X, weights N(0,0.02))" if learned else
                  "synthetic (seeded; R1 block-coherent selector scores s = u[block] + 0.05 eps given by the caller, "
                  "N(0,1) Q/K/V/X, weights N(0,0.02))"),
-        "config": {"workload": w["name"], "B": B, "H": H, "N": N, "d": d, "block": 64, "topk": K, "d_sel": ds,
+        "config": {"workload": w["name"], "B": B, "H": H, "Hkv": Hkv, "N": N, "d": d, "block": 64, "topk": K,
+                   "d_sel": ds,
                    "mlp": [T, D, F, D], "selector": "meanpool_proj" if learned else "scores_given (R1)",
                    "l2": "flushed between timed steps (256 MiB write)",
                    "parallelism": f"replicas x{world}"},
@@ -421,13 +432,14 @@ def run_reference(args, w, rank, world):
         return None
     rates = []
     desc = ""
+    learned = args.regime == "R2" and w.get("Hkv", w["H"]) == w["H"]   # the same selector as our arm
     for k in range(args.warmup + args.steps):
-        rate, dt, desc = oracle_sample(w, budget_s=args.ref_step_s, seed=k)
+        rate, dt, desc = oracle_sample(w, budget_s=args.ref_step_s, seed=k, learned=learned)
         if k >= args.warmup:
             rates.append(rate)
     # harmonic mean: total FLOPs over total time for equal-work steps
     value = len(rates) / sum(1.0 / r for r in rates) / 1e12
-    full = algorithmic_flops(w)["total"]
+    full = algorithmic_flops(w, learned)["total"]
     ms = full / (value * 1e12) * 1e3
     return {
         "impl": "reference", "metric": METRIC, "value": round(value, 8), "unit": UNIT, "n_gpus": world,
