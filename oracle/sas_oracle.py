@@ -308,6 +308,44 @@ def sas_attention_gqa(Q, K, V, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=N
     return out
 
 
+def sas_attention_varlen(Q, K, V, cu_seqlens, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                         act=GATE_SOFTMAX, pos=GATE_INNER):
+    """Packed variable-length form: sequences s = 0 .. S-1 occupy rows
+    cu_seqlens[s] .. cu_seqlens[s+1]-1 of the token axis; each is its own
+    causal problem whose block partition starts at its first token (token t
+    of sequence s is in its block floor(t / b); nothing crosses sequences).
+    Q [Hq, total, d]; K, V [Hkv, total, d]; scores [Hkv, total, >=C-1], row
+    cu[s] + t reading entries 0 .. floor(t / b) - 1; Hq = G Hkv (GQA, query
+    head h uses group h // G).  Returns dict of [Hq, total, ...] O, LSE and
+    [Hkv, total, topk] sel_idx / sel_logg (rows past cu[S] stay zero / -1).
+    """
+    Hq, total, d = Q.shape
+    Hkv = K.shape[0]
+    if Hq % Hkv:
+        raise ValueError("Hq must be a multiple of Hkv")
+    G = Hq // Hkv
+    cu = [int(x) for x in cu_seqlens]
+    if cu[0] != 0 or any(cu[k + 1] < cu[k] for k in range(len(cu) - 1)) or cu[-1] > total:
+        raise ValueError("cu_seqlens must start at 0, not decrease and stay within the token axis")
+    O = np.zeros((Hq, total, V.shape[2]))
+    LSE = np.zeros((Hq, total))
+    sel_idx = np.full((Hkv, total, topk), -1, dtype=np.int64)
+    sel_logg = np.zeros((Hkv, total, topk))
+    for s0, s1 in zip(cu[:-1], cu[1:]):
+        if s1 == s0:
+            continue
+        for h in range(Hq):
+            g = h // G
+            r = sas_attention_head(Q[h, s0:s1], K[g, s0:s1], V[g, s0:s1], scores[g, s0:s1], b, topk, mode,
+                                   sm_scale, None, act, pos)
+            O[h, s0:s1] = r["O"]
+            LSE[h, s0:s1] = r["LSE"]
+            if h % G == 0:
+                sel_idx[g, s0:s1] = r["sel_idx"]
+                sel_logg[g, s0:s1] = r["sel_logg"]
+    return {"O": O, "LSE": LSE, "sel_idx": sel_idx, "sel_logg": sel_logg}
+
+
 # -------------------------------------------------------------------- a6 --
 
 def gelu(x):
