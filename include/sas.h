@@ -99,6 +99,13 @@ typedef struct {
                              Sec. 5 inference implementation).  Hkv < H needs
                              SCORES_GIVEN (one score table per group) and has no
                              backward.                                                */
+    int32_t max_seqs;     /* 0: [B, H, N, d] batches of N-token sequences.  > 0: packed
+                             variable-length sequences, at most max_seqs of them, in
+                             [H, N, d] tensors whose token axis (N = capacity) holds
+                             them back to back (sas_attention_fwd_varlen); needs B = 1
+                             and SCORES_GIVEN, has no backward.                        */
+    int32_t max_seqlen;   /* packed mode: longest sequence (1 .. N; 0 selects N); the
+                             score table has C = ceil(max_seqlen / 64) columns         */
 } sas_config;
 
 typedef struct sas_handle sas_handle;
@@ -188,6 +195,28 @@ sas_status sas_attention_bwd(sas_handle* h,
  * D and F must be multiples of 64; T >= 1.  The hidden activation
  * GELU(X W1^T + b1) is kept as a bf16 [T, F] tensor in handle-owned
  * memory, allocated (synchronously) the first time a call needs more. */
+/* Packed variable-length form of sas_attention_fwd, on a handle created
+ * with max_seqs > 0.  Sequence s holds rows cu_seqlens[s] .. cu_seqlens[s+1]-1
+ * of the token axis and is its own causal problem: its blocks of 64 tokens
+ * start at its first row, and no row attends outside its sequence.
+ *
+ *   cu_seqlens int32 [num_seqs + 1], DEVICE: cu[0] = 0, non-decreasing,
+ *              every length <= max_seqlen, cu[num_seqs] <= N.  Checked on
+ *              the device: offsets that break this set the device status
+ *              word to SAS_ERR_INVALID_ARG and nothing is computed.     (in)
+ *   num_seqs   1 .. max_seqs
+ *   Q          bf16 [H, N, d]; K, V bf16 [Hkv, N, d]                     (in)
+ *   scores     fp32 [Hkv, N, C], C = ceil(max_seqlen / 64); row cu[s] + t
+ *              reads entries 0 .. floor(t/64)-1 (blocks of its sequence)  (in)
+ *   O          bf16 [H, N, d]; LSE fp32 [H, N] (may be NULL)            (out)
+ *   sel_idx, sel_logg  [Hkv, N, topk] as in sas_attention_fwd, block
+ *              indices counted within the row's sequence (may be NULL) (out)
+ * Rows past cu[num_seqs] are not written.  Graph-capturable (no host
+ * synchronisation). */
+sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, int32_t num_seqs,
+                                    const void* Q, const void* K, const void* V, const float* scores,
+                                    void* O, float* LSE, int32_t* sel_idx, float* sel_logg, void* stream);
+
 sas_status sas_mlp_fwd(sas_handle* h,
                        const void* X, const void* W1, const void* b1,
                        const void* W2, const void* b2, void* Y,

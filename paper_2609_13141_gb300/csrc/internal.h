@@ -64,8 +64,18 @@ struct SelectArgs {
     float* sel_logg;                // [BH][N][topk]
     int32_t* union_idx;             // [BH][T][C]
     int32_t* union_cnt;             // [BH][T]
+    // packed sequences (given scores only): T tile slots, the first *ntiles
+    // used; tiles[g] = {first row, tile index within the sequence, sequence
+    // length, 0}; N is then the token capacity of each head.  Null otherwise.
+    const int4* tiles;
+    const int* ntiles;
 };
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err);
+// Builds the tile table of packed sequences cu[0..S] (device offsets) with
+// sequences of at most max_len tokens within Ncap rows; bad offsets set the
+// status word to SAS_ERR_INVALID_ARG and leave *ntiles = 0.
+cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len, int4* tiles, int* ntiles,
+                                const KernelEnv& env);
 
 // ---- a5: fused gated block-sparse attention forward.
 struct AttnArgs {
@@ -80,6 +90,8 @@ struct AttnArgs {
     const float* sel_logg;
     int BH, N, d, C, T, topk, mode;    // BH: query heads x batch
     int G;                      // query heads per KV group (1 without GQA): K, V, lists of group bh / G
+    const int4* tiles;          // packed sequences: as in SelectArgs (null otherwise)
+    const int* ntiles;
     int gate_pos;               // 0 inner (+ log g in the logits), 1 outer (g scales P after the softmax)
     float sm_scale;
     int* sched;                 // 16 zeroed bytes owned by the caller, left zeroed after each launch

@@ -92,6 +92,8 @@ struct AttnParams {
     int N, C, T, BH, topk, mode;
     int G;                  // query heads per KV group: K, V and the lists of head bh are group bh / G
     int group;              // heads per group of the work list (a multiple of G)
+    const int4* tiles;      // packed sequences: {first row, tile in sequence, length} per slot (else null)
+    const int* ntiles;      // slots in use (device)
     int* sched;             // [0] next work item, [1] CTAs finished; both zero between launches
     float scale_log2;
     int* status;
@@ -109,22 +111,36 @@ struct AttnParams {
 // run the same tile at about the same time over the same K, V blocks.
 
 struct TileRef {
-    int t, bh, kv;          // tile, query head, KV group (= bh without GQA)
+    int t, bh, kv;          // tile (within its sequence), query head, KV group (= bh without GQA)
+    int base, n;            // the sequence's first row in the token axis and its length
     const int32_t* ulist;   // the tile's union list (ascending historical blocks)
     int U;                  // its length
 };
 
-__device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w) {
+// T: tile slots in use (p.T, or the packed sequences' tile count).
+__device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w, int T) {
     TileRef x;
-    const int per_group = p.group * p.T;                  // items of a full group
+    const int per_group = p.group * T;                    // items of a full group
     const int g0 = w / per_group;                         // group index
     const int h0 = g0 * p.group;                          // its first head
     const int gs = min(p.group, p.BH - h0);               // heads in this group
     const int wi = w - g0 * per_group;
-    x.t = p.T - 1 - wi / gs;
+    int slot;
+    if (p.tiles == nullptr) {
+        x.t = T - 1 - wi / gs;
+        x.base = 0;
+        x.n = p.N;
+        slot = x.t;
+    } else {
+        slot = wi / gs;                                   // the table is ordered longest history first
+        const int4 v = __ldg(p.tiles + slot);
+        x.base = v.x;
+        x.t = v.y;
+        x.n = v.z;
+    }
     x.bh = h0 + wi % gs;
     x.kv = x.bh / p.G;
-    const long long tb = static_cast<long long>(x.kv) * p.T + x.t;
+    const long long tb = static_cast<long long>(x.kv) * p.T + slot;
     x.ulist = p.union_idx + tb * p.C;
     x.U = __ldg(p.union_cnt + tb);
     return x;
@@ -141,7 +157,7 @@ __device__ __forceinline__ bool read_item(AttnCtl& ctl, int r, const WaitCtl& wc
 
 // visited blocks of a tile: its union list, then the diagonal block(s)
 __device__ __forceinline__ int tile_blocks(const AttnParams& p, const TileRef& x) {
-    return x.U + ((2 * x.t + 1 < p.C) ? 2 : 1);
+    return x.U + ((2 * x.t + 1) * kBN < x.n ? 2 : 1);
 }
 
 __device__ __forceinline__ int block_at(const TileRef& x, int j) {
@@ -178,7 +194,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     int& abort_flag = ctl.abort_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
-    const int W = p.T * p.BH;
+    const int Tn = p.tiles == nullptr ? p.T : __ldg(p.ntiles);   // tile slots in use
+    const int W = Tn * p.BH;
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
@@ -227,7 +244,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             mbar_arrive(&ctl.item_full[slot]);
             mbar_arrive(&ctl.item_empty[slot]);   // this thread has read it too
             if (w < 0) break;
-            const TileRef x = tile_ref(p, w);
+            const TileRef x = tile_ref(p, w, Tn);
             const int n = tile_blocks(p, x);
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
@@ -238,7 +255,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
 #pragma unroll
                 for (int a = 0; a < D / 64; ++a)
-                    tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, m * kBN, x.kv);
+                    tma_load_3d(dst + a * (kBN * 128), &mapK, &k_full[s], a * 64, x.base + m * kBN, x.kv);
                 ++nk;
             }
             g += n;
@@ -262,13 +279,13 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (!read_item(ctl, r, wc, w)) { ok = false; break; }
             mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
-            const TileRef x = tile_ref(p, w);
+            const TileRef x = tile_ref(p, w, Tn);
             const int n = tile_blocks(p, x);
             if (!mbar_wait(&q_empty, (tc & 1) ^ 1u, wc)) { ok = false; break; }
             mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
 #pragma unroll
             for (int a = 0; a < D / 64; ++a)
-                tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, x.t * kBM, x.bh);
+                tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, x.base + x.t * kBM, x.bh);
             ++nq;
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
@@ -279,7 +296,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
 #pragma unroll
                 for (int a = 0; a < D / 64; ++a)
-                    tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, m * kBN, x.kv);
+                    tma_load_3d(dst + a * (kBN * 128), &mapV, &v_full[s], a * 64, x.base + m * kBN, x.kv);
                 ++nv;
             }
             g += n;
@@ -302,7 +319,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (!read_item(ctl, r, wc, w)) { ok = false; break; }
             mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
-            const int n = tile_blocks(p, tile_ref(p, w));
+            const int n = tile_blocks(p, tile_ref(p, w, Tn));
             if (!mbar_wait(&q_full, tc & 1, wc)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
@@ -338,7 +355,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (!read_item(ctl, r, wc, w)) { ok = false; break; }
             mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
-            const int n = tile_blocks(p, tile_ref(p, w));
+            const int n = tile_blocks(p, tile_ref(p, w, Tn));
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int vs = gb % Cfg::VST;
@@ -379,15 +396,15 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             __syncwarp();
             if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
             if (w < 0) break;
-            const TileRef x = tile_ref(p, w);
+            const TileRef x = tile_ref(p, w, Tn);
             const int n = tile_blocks(p, x);
             const int t = x.t;
-            const int i = t * kBM + r_row;
-            const bool valid = i < p.N;
+            const int i = t * kBM + r_row;   // row within its sequence
+            const bool valid = i < x.n;
             const int c = i >> 6;
             const int nsel = valid ? min(p.topk, c) : 0;
-            const long long row_off = static_cast<long long>(x.bh) * p.N + i;   // O, LSE
-            const long long sel_off = static_cast<long long>(x.kv) * p.N + i;   // the group's kept list
+            const long long row_off = static_cast<long long>(x.bh) * p.N + x.base + i;   // O, LSE
+            const long long sel_off = static_cast<long long>(x.kv) * p.N + x.base + i;   // the group's kept list
             const int32_t* my_idx = p.sel_idx + sel_off * p.topk;
             const float* my_lg = p.sel_logg + sel_off * p.topk;
             // The row's kept list is staged kRing entries ahead in a shared ring
@@ -630,6 +647,8 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.sel_logg = a.sel_logg;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
     p.G = a.G;
+    p.tiles = a.tiles;
+    p.ntiles = a.ntiles;
     // KV groups whose K and V (2 * N * d bf16 each) fit in half of L2 together,
     // at least one; the work list takes their G query heads each
     const long long kv_head = 4LL * a.N * D;

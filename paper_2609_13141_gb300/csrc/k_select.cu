@@ -47,8 +47,17 @@ struct SelParams {
     float* sel_logg;
     int32_t* union_idx;
     int32_t* union_cnt;
+    const int4* tiles;            // packed sequences: {first row, local tile, sequence length} per tile slot
+    const int* ntiles;            // their number (device); both null for [B, H, N] inputs
     int* status;
     long long limit;
+};
+
+// Where a CTA's 128-row tile lies: its union-list slot, its tile index within
+// its sequence, the sequence's first row in the head's token axis and the
+// sequence length.  [B, H, N] inputs: one sequence of N rows per head.
+struct TileGeo {
+    int slot, t, base, n;
 };
 
 // One CTA per (head, 128-row tile) on a 1-D grid: the tile index falls with
@@ -56,6 +65,16 @@ struct SelParams {
 // histories of every head are dispatched first and the light ones fill the tail.
 __device__ __forceinline__ int tile_of_block(int T, int BH) { return T - 1 - static_cast<int>(blockIdx.x / BH); }
 __device__ __forceinline__ int head_of_block(int BH) { return static_cast<int>(blockIdx.x % BH); }
+// Packed sequences: the tile table is already ordered longest history first.
+__device__ __forceinline__ TileGeo tile_geo(const SelParams& p) {
+    if (p.tiles == nullptr) {
+        const int t = tile_of_block(p.T, p.BH);
+        return {t, t, 0, p.N};
+    }
+    const int g = static_cast<int>(blockIdx.x / p.BH);
+    const int4 v = __ldg(p.tiles + g);
+    return {g, v.y, v.x, v.z};
+}
 
 // Online log-sum-exp of a row's scores.
 struct RowLse {
@@ -308,13 +327,14 @@ __device__ __forceinline__ void stage_entry(const Staging& st, int r, int e, int
     st.lg[r * st.stride + e] = lg;
 }
 
-// Copies the staged rows of tile t to sel_idx / sel_logg (rows >= N skipped).
-// Consecutive threads take consecutive entries of a row, so stores coalesce.
-__device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, int bh, int t, int tid, int nthreads) {
+// Copies the staged rows (the tile's first `rows`, from row `row0` of the
+// head's token axis) to sel_idx / sel_logg.  Consecutive threads take
+// consecutive entries of a row, so stores coalesce.
+__device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, int bh, long long row0, int rows,
+                                         int tid, int nthreads) {
     const int K = p.topk;
     if (K == 0) return;
-    const int rows = min(kRows, p.N - t * kRows);
-    const long long base = (static_cast<long long>(bh) * p.N + static_cast<long long>(t) * kRows) * K;
+    const long long base = (static_cast<long long>(bh) * p.N + row0) * K;
     int r = tid / K, e = tid - r * K;
     const int dr = nthreads / K, de = nthreads - dr * K;
     const bool sigm = p.gate_act == 1;
@@ -410,12 +430,14 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ float stage[4][32][33];
 
-    const int t = tile_of_block(p.T, p.BH);
+    if (p.tiles != nullptr && static_cast<int>(blockIdx.x / p.BH) >= __ldg(p.ntiles)) return;   // spare slot
+    const TileGeo geo = tile_geo(p);
+    const int t = geo.t;
     const int bh = head_of_block(p.BH);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int r = threadIdx.x;
-    const int i = t * kRows + r;
-    const bool valid = i < p.N;
+    const int i = t * kRows + r;            // row within its sequence
+    const bool valid = i < geo.n;
     const int Ci = valid ? (i >> 6) : 0;
     const int diag = 2 * t;
     const int K = p.topk;
@@ -441,16 +463,16 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     RowLse lse{-CUDART_INF_F, 0.f};
 
     const int row0 = t * kRows + warp * 32;
-    const int last = min(row0 + 31, p.N - 1);
-    const int Cw = row0 < p.N ? (last >> 6) : 0;   // largest C_i among the warp's rows
-    const float* sbase = p.scores + static_cast<long long>(bh) * p.N * p.C;
+    const int last = min(row0 + 31, geo.n - 1);
+    const int Cw = row0 < geo.n ? (last >> 6) : 0;   // largest C_i among the warp's rows
+    const float* sbase = p.scores + (static_cast<long long>(bh) * p.N + geo.base) * p.C;
     for (int c = 0; 32 * c < Cw; ++c) {
         const int m = 32 * c + lane;
 #pragma unroll 4
         for (int rho = 0; rho < 32; ++rho) {
             const int row = row0 + rho;
             float v = 0.f;
-            if (row < p.N && m < p.C) v = __ldg(sbase + static_cast<long long>(row) * p.C + m);
+            if (row < geo.n && m < p.C) v = __ldg(sbase + static_cast<long long>(row) * p.C + m);
             stage[warp][lane][rho] = v;
         }
         __syncwarp();
@@ -470,10 +492,11 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
         else row_emit(stk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
     }
     __syncthreads();
-    copy_out(st, p, bh, t, threadIdx.x, 128);
+    copy_out(st, p, bh, static_cast<long long>(geo.base) + t * kRows, min(kRows, geo.n - t * kRows), threadIdx.x,
+             128);
     if (warp == 0)
-        compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
-                      p.union_cnt + static_cast<long long>(bh) * p.T + t);
+        compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + geo.slot) * p.C,
+                      p.union_cnt + static_cast<long long>(bh) * p.T + geo.slot);
 }
 
 // --------------------------------------------------------- learned selector
@@ -702,7 +725,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             else row_emit(stk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
         }
         named_bar_sync(1, 128);
-        if (ok) copy_out(st, p, bh, t, static_cast<int>(threadIdx.x) - 64, 128);
+        if (ok)
+            copy_out(st, p, bh, static_cast<long long>(t) * kRows, min(kRows, p.N - t * kRows),
+                     static_cast<int>(threadIdx.x) - 64, 128);
         if (warp == 2)
             compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
                           p.union_cnt + static_cast<long long>(bh) * p.T + t);
@@ -751,7 +776,77 @@ cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelE
     return a.topk <= 32 ? launch_proj<D, DS, true>(a, p, env, err) : launch_proj<D, DS, false>(a, p, env, err);
 }
 
+constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
+
+// Tile table of packed sequences (one CTA).  Sequence s holds rows
+// cu[s] .. cu[s+1]-1 and T_s = ceil(n_s / 128) tiles.  Entries are ordered by
+// the tile's index within its sequence, descending (longest key history
+// first): tile t of every sequence with T_s > t sits at off(t) + rank(s),
+// off(t) = number of tiles with a larger index, rank(s) = the sequence's place
+// when sequences are ordered by T_s descending (ties in arrival order: the
+// order only schedules work).  Bad offsets set the status word and leave no
+// tiles.
+__global__ void __launch_bounds__(1024) varlen_tiles_kernel(const int32_t* cu, int S, int Ncap, int max_len,
+                                                            int tmax, int4* tiles, int* ntiles, int* status) {
+    extern __shared__ int vsh[];   // hist[tmax + 2], cnt_gt[tmax + 2], off[tmax + 2], next[tmax + 2]
+    int* hist = vsh;
+    int* gt = hist + tmax + 2;     // gt[t] = number of sequences with T_s > t
+    int* off = gt + tmax + 2;
+    int* nxt = off + tmax + 2;
+    __shared__ int bad;
+    const int tid = threadIdx.x;
+    for (int k = tid; k < tmax + 2; k += blockDim.x) { hist[k] = 0; nxt[k] = 0; }
+    if (tid == 0) bad = (S < 1 || __ldg(cu) != 0 || __ldg(cu + S) > Ncap) ? 1 : 0;
+    __syncthreads();
+    for (int s = tid; s < S; s += blockDim.x) {
+        const int n = __ldg(cu + s + 1) - __ldg(cu + s);
+        if (n < 0 || n > max_len) { bad = 1; continue; }
+        atomicAdd(&hist[(n + kRows - 1) / kRows], 1);
+    }
+    __syncthreads();
+    if (bad) {
+        if (tid == 0) {
+            *ntiles = 0;
+            atomicExch(status, kStatusBadInput);
+        }
+        return;
+    }
+    if (tid == 0) {
+        // gt[t] = sum_{T > t} hist[T]; off[t] = sum_{t' > t} gt[t']
+        int g = 0, o = 0;
+        for (int t = tmax; t >= 0; --t) {
+            g += hist[t + 1];
+            gt[t] = g;
+            off[t] = o;
+            o += g;
+        }
+        *ntiles = o;
+    }
+    __syncthreads();
+    for (int s = tid; s < S; s += blockDim.x) {
+        const int b0 = __ldg(cu + s), n = __ldg(cu + s + 1) - b0;
+        const int T = (n + kRows - 1) / kRows;
+        if (T == 0) continue;
+        const int rank = gt[T] + atomicAdd(&nxt[T], 1);   // sequences with more tiles come first
+        for (int t = 0; t < T; ++t) tiles[off[t] + rank] = make_int4(b0, t, n, 0);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len, int4* tiles, int* ntiles,
+                                const KernelEnv& env) {
+    const int tmax = (max_len + kRows - 1) / kRows;
+    const size_t smem = static_cast<size_t>(4) * (tmax + 2) * sizeof(int);
+    if (smem > 200 * 1024) return cudaErrorInvalidValue;
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(varlen_tiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+    }
+    varlen_tiles_kernel<<<1, 1024, smem, env.stream>>>(cu, S, Ncap, max_len, tmax, tiles, ntiles, env.status);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
     SelParams p;
@@ -761,7 +856,12 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     p.scores = a.scores;
     p.sel_idx = a.sel_idx; p.sel_logg = a.sel_logg;
     p.union_idx = a.union_idx; p.union_cnt = a.union_cnt;
+    p.tiles = a.tiles; p.ntiles = a.ntiles;
     p.status = env.status; p.limit = env.limit;
+    if (a.tiles != nullptr && a.scores == nullptr) {
+        *err = "selection: packed sequences need given scores";
+        return cudaErrorInvalidValue;
+    }
     const bool reg = a.topk <= 32;
     if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
     if (a.d == 128 && a.d_sel == 128) return launch_proj_k<128, 128>(a, p, env, err);

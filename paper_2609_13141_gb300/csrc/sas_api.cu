@@ -92,6 +92,9 @@ struct sas_handle {
     float sm_scale = 0.f;
     int BH = 0, C = 0, T = 0, F = 0;
     int Hkv = 0, G = 1, BHkv = 0;   // KV heads, query heads per group, KV groups x batch
+    bool varlen = false;            // packed sequences: T = tile slots, C from max_seqlen
+    int4* tiles = nullptr;          // packed sequences' tile table [T] and its count
+    int* ntiles = nullptr;
     // workspace
     void* Kt = nullptr;         // bf16 [BH][max(F,1)][d_sel]
     int32_t* union_idx = nullptr;
@@ -223,6 +226,11 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     const int Hkv = c.Hkv == 0 ? c.H : c.Hkv;
     if (Hkv < 1 || Hkv > c.H || c.H % Hkv != 0) return SAS_ERR_INVALID_ARG;
     if (Hkv != c.H && c.selector != SAS_SEL_SCORES_GIVEN) return SAS_ERR_UNSUPPORTED;
+    if (c.max_seqs < 0 || c.max_seqlen < 0 || c.max_seqlen > c.N) return SAS_ERR_INVALID_ARG;
+    const bool varlen = c.max_seqs > 0;
+    if (varlen && c.B != 1) return SAS_ERR_INVALID_ARG;
+    if (varlen && c.selector != SAS_SEL_SCORES_GIVEN) return SAS_ERR_UNSUPPORTED;
+    if (varlen && c.max_seqs > (1 << 20)) return SAS_ERR_UNSUPPORTED;
     const long long BH = static_cast<long long>(c.B) * c.H;
     const long long BHkv = static_cast<long long>(c.B) * Hkv;
     if (BH > (1LL << 30) || BH * c.N > (1LL << 40)) return SAS_ERR_UNSUPPORTED;
@@ -236,8 +244,11 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     h->Hkv = Hkv;
     h->G = c.H / Hkv;
     h->BHkv = static_cast<int>(BHkv);
-    h->C = (c.N + 63) / 64;
-    h->T = (c.N + 127) / 128;
+    h->varlen = varlen;
+    const int max_len = varlen && c.max_seqlen > 0 ? c.max_seqlen : c.N;
+    h->C = (max_len + 63) / 64;
+    // packed sequences: at most N / 128 + max_seqs tiles (each sequence adds one partial tile)
+    h->T = (c.N + 127) / 128 + (varlen ? c.max_seqs : 0);
     h->F = c.N / 64;
     sas_status st = check_device(h);
     if (st != SAS_OK) { delete h; return st; }
@@ -252,6 +263,11 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BHkv) * h->T * 4);
     if (e == cudaSuccess) e = alloc(&h->sel_idx, rows * (c.topk > 0 ? c.topk : 1) * 4);
     if (e == cudaSuccess) e = alloc(&h->sel_logg, rows * (c.topk > 0 ? c.topk : 1) * 4);
+    if (varlen) {
+        if (e == cudaSuccess) e = alloc(&h->tiles, static_cast<size_t>(h->T) * sizeof(int4));
+        if (e == cudaSuccess) e = alloc(&h->ntiles, 16);
+        if (e == cudaSuccess) e = cudaMemset(h->ntiles, 0, 16);
+    }
     if (e == cudaSuccess) e = alloc(&h->status, 16);
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, 16);
     if (e == cudaSuccess) e = alloc(&h->sched, 16);
@@ -274,6 +290,8 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->union_cnt);
     cudaFree(h->sel_idx);
     cudaFree(h->sel_logg);
+    cudaFree(h->tiles);
+    cudaFree(h->ntiles);
     cudaFree(h->status);
     cudaFree(h->sched);
     cudaFree(h->hidden);
@@ -291,6 +309,7 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
                              float* sel_logg, void* stream) {
     if (h == nullptr) return SAS_ERR_INVALID_ARG;
     const sas_config& c = h->cfg;
+    if (h->varlen) return fail(h, SAS_ERR_INVALID_ARG, "packed-sequence handle: use sas_attention_fwd_varlen");
     if (!Q || !K || !V || !O) return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O are required");
     if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
         return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O must be 16-byte aligned");
@@ -337,6 +356,61 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
     aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
     aa.G = h->G;
+    aa.gate_pos = c.gate_pos;
+    aa.sm_scale = h->sm_scale;
+    aa.sched = h->sched;
+    e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    return SAS_OK;
+}
+
+sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, int32_t num_seqs, const void* Q,
+                                    const void* K, const void* V, const float* scores, void* O, float* LSE,
+                                    int32_t* sel_idx, float* sel_logg, void* stream) {
+    if (h == nullptr) return SAS_ERR_INVALID_ARG;
+    const sas_config& c = h->cfg;
+    if (!h->varlen) return fail(h, SAS_ERR_INVALID_ARG, "handle not created for packed sequences (max_seqs = 0)");
+    if (num_seqs < 1 || num_seqs > c.max_seqs)
+        return fail(h, SAS_ERR_INVALID_ARG, "num_seqs must be in 1 .. max_seqs");
+    if (!cu_seqlens || !aligned4(cu_seqlens)) return fail(h, SAS_ERR_INVALID_ARG, "cu_seqlens required (4-byte aligned)");
+    if (!Q || !K || !V || !O) return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O are required");
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O must be 16-byte aligned");
+    if (!scores || !aligned4(scores)) return fail(h, SAS_ERR_INVALID_ARG, "scores required (4-byte aligned)");
+    if ((LSE && !aligned4(LSE)) || (sel_idx && !aligned4(sel_idx)) || (sel_logg && !aligned4(sel_logg)))
+        return fail(h, SAS_ERR_INVALID_ARG, "LSE / sel_idx / sel_logg must be 4-byte aligned");
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const sas::KernelEnv env{s, h->status, h->limit};
+    const char* err = "";
+    int32_t* out_idx = sel_idx ? sel_idx : h->sel_idx;
+    float* out_lg = sel_logg ? sel_logg : h->sel_logg;
+    const int max_len = c.max_seqlen > 0 ? c.max_seqlen : c.N;
+    // tile table, then a2-a4 over the tiles of every sequence
+    sas::SelectArgs sa{};
+    sa.BH = h->BHkv; sa.H = h->Hkv; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.gate_act = c.gate_act;
+    sa.score_scale = 1.0f;
+    sa.scores = scores;
+    sa.d = c.d;
+    sa.sel_idx = out_idx; sa.sel_logg = out_lg;
+    sa.union_idx = h->union_idx; sa.union_cnt = h->union_cnt;
+    sa.tiles = h->tiles; sa.ntiles = h->ntiles;
+    cudaError_t e = timed_launch(h, 2, s, [&] {
+        cudaError_t r = sas::launch_varlen_tiles(cu_seqlens, num_seqs, c.N, max_len, h->tiles, h->ntiles, env);
+        if (r != cudaSuccess) { err = "packed-sequence tile table"; return r; }
+        return sas::launch_select(sa, env, &err);
+    });
+    if (e != cudaSuccess) return cuda_fail(h, e, err);
+    h->launches += 1;   // the tile table
+    // a5 over the same tiles
+    sas::AttnArgs aa{};
+    aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
+    aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
+    aa.sel_idx = out_idx; aa.sel_logg = out_lg;
+    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.G = h->G;
+    aa.tiles = h->tiles; aa.ntiles = h->ntiles;
     aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
     aa.sched = h->sched;
@@ -408,6 +482,7 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     if (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER)
         return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
     if (h->G != 1) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports Hkv = H");
+    if (h->varlen) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports [B, H, N, d] batches");
     if (h->T > sas::kBwdMaxTiles) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports N <= 262016");
     if (dscores) {
         if (c.selector != SAS_SEL_SCORES_GIVEN || !scores)

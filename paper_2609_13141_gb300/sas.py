@@ -43,7 +43,8 @@ class SasConfig(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("d", ctypes.c_int32),
                 ("block", ctypes.c_int32), ("topk", ctypes.c_int32), ("sm_scale", ctypes.c_float),
                 ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32),
-                ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32), ("Hkv", ctypes.c_int32)]
+                ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32), ("Hkv", ctypes.c_int32),
+                ("max_seqs", ctypes.c_int32), ("max_seqlen", ctypes.c_int32)]
 
 
 class SasDecodeConfig(ctypes.Structure):
@@ -81,6 +82,8 @@ def lib():
     L.sas_destroy.restype = None
     L.sas_attention_fwd.argtypes = [vp] * 12
     L.sas_attention_fwd.restype = i32
+    L.sas_attention_fwd_varlen.argtypes = [vp, vp, i32] + [vp] * 9
+    L.sas_attention_fwd_varlen.restype = i32
     L.sas_attention_bwd.argtypes = [vp] * 16
     L.sas_attention_bwd.restype = i32
     L.sas_mlp_fwd.argtypes = [vp] * 7 + [i64, i64, i64, vp]
@@ -168,17 +171,20 @@ def sas_status_str(status):
 
 
 def sas_create(B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-               sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv)
+               sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0,
+               max_seqlen=0):
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv, max_seqs,
+                    max_seqlen)
     h = ctypes.c_void_p()
     _check(lib().sas_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_create")
     return h
 
 
 def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64,
-                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
+                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0):
     """Raw status of sas_create (for argument-check tests); destroys the handle on success."""
-    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv)
+    cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv, max_seqs,
+                    max_seqlen)
     h = ctypes.c_void_p()
     st = lib().sas_create(ctypes.byref(cfg), ctypes.byref(h))
     if st == SAS_OK:
@@ -188,6 +194,17 @@ def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.
 
 def sas_destroy(h):
     lib().sas_destroy(h)
+
+
+def sas_attention_fwd_varlen(h, cu_seqlens, Q, K, V, scores, O, LSE=None, sel_idx=None, sel_logg=None,
+                             stream=None):
+    bf = torch.bfloat16
+    st = lib().sas_attention_fwd_varlen(
+        h, _ptr(cu_seqlens, torch.int32, "cu_seqlens"), ctypes.c_int32(cu_seqlens.numel() - 1),
+        _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"), _ptr(scores, torch.float32, "scores"),
+        _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False), _ptr(sel_idx, torch.int32, "sel_idx", False),
+        _ptr(sel_logg, torch.float32, "sel_logg", False), _stream(stream))
+    _check(st, h, "sas_attention_fwd_varlen")
 
 
 def sas_attention_fwd(h, Q, K, V, O, scores=None, Wq=None, Wk=None, LSE=None, sel_idx=None, sel_logg=None,
@@ -279,11 +296,27 @@ class SasLayer:
     """Owns one handle; allocates outputs and calls the C ABI."""
 
     def __init__(self, B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0):
+                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0):
         self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
         self.Hkv = Hkv or H                      # kept lists are per KV group
         self.selector = selector
-        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv)
+        self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv,
+                            max_seqs, max_seqlen)
+
+    def attention_varlen(self, cu_seqlens, Q, K, V, scores, want_sel=True, stream=None):
+        """Packed sequences (handle made with max_seqs > 0): Q [H, N, d], K/V [Hkv, N, d],
+        scores [Hkv, N, C], cu_seqlens int32 on the device.  Rows past cu[-1] keep the
+        values the output tensors were created with (zeros here)."""
+        dev = Q.device
+        O = torch.zeros_like(Q)
+        LSE = torch.zeros(self.H, self.N, device=dev, dtype=torch.float32)
+        sel_idx = sel_logg = None
+        if want_sel:
+            k = max(self.topk, 1)
+            sel_idx = torch.full((self.Hkv, self.N, k), -7, device=dev, dtype=torch.int32)
+            sel_logg = torch.zeros(self.Hkv, self.N, k, device=dev, dtype=torch.float32)
+        sas_attention_fwd_varlen(self.h, cu_seqlens, Q, K, V, scores, O, LSE, sel_idx, sel_logg, stream)
+        return O, LSE, sel_idx, sel_logg
 
     def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
         dev = Q.device
