@@ -51,6 +51,12 @@ WORKLOADS = {
                              name="Qwen3-4B-shaped GQA prefill layer: B=1 Hq=32 Hkv=8 N=32768 d=128 b=64 K=32 "
                                   "(2048-token budget), given R1 scores per KV group, GELU MLP "
                                   "32768x2560->9728->2560 (in place of the model's SwiGLU MLP)"),
+    # the same layer on 32768 tokens packed from 12 sequences of geometric lengths
+    "qwen3_4b_packed": dict(B=1, H=32, Hkv=8, N=32768, d=128, topk=32, d_sel=128, D=2560, F=9728,
+                            lens=[16384, 8192, 4096, 2048, 1024, 512, 256, 128, 64, 32, 16, 16],
+                            name="Qwen3-4B-shaped GQA prefill layer on 32768 packed tokens (12 sequences of "
+                                 "16384, 8192, ..., 32, 16, 16 tokens): Hq=32 Hkv=8 d=128 b=64 K=32, given R1 "
+                                 "scores per KV group, GELU MLP 32768x2560->9728->2560"),
 }
 
 
@@ -78,6 +84,18 @@ def algorithmic_flops(w, learned=True):
     mlp = 4 * w["B"] * N * w["D"] * w["F"]
     return {"attention": BH * attn, "selector": BH * sel, "mlp": mlp,
             "total": BH * (attn + sel) + mlp}
+
+
+def packed_flops(w, learned=False):
+    """algorithmic_flops summed over the packed sequences (the MLP runs on all tokens)."""
+    att = sel = 0
+    for n in w["lens"]:
+        if n > 0:
+            f = algorithmic_flops(dict(w, N=n, B=1), learned)
+            att += f["attention"]
+            sel += f["selector"]
+    mlp = 4 * w["N"] * w["D"] * w["F"]
+    return {"attention": att, "selector": sel, "mlp": mlp, "total": att + sel + mlp}
 
 
 def load_peaks():
@@ -191,8 +209,9 @@ def run_ours(args, w, rank, world):
 
     B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
     Hkv = w.get("Hkv", H)
+    lens = w.get("lens")                          # packed sequences (B = 1, token axis of N rows)
     T = B * N
-    learned = args.regime == "R2" and Hkv == H   # GQA takes given scores (one table per KV group)
+    learned = args.regime == "R2" and Hkv == H and not lens   # GQA / packing take given scores
     if learned:
         # R2: block-correlated queries through the learned selector
         Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
@@ -204,7 +223,7 @@ def run_ours(args, w, rank, world):
     else:
         Q = synth.qkv(B, H, N, d, seed=rank, regime="iid")[0]
         _, Kk, V = synth.qkv(B, Hkv, N, d, seed=rank + 100, regime="iid")
-        S = synth.scores(B, Hkv, N, (N + 63) // 64, seed=rank, regime="R1")
+        S = synth.scores(B, Hkv, N, (max(lens) + 63) // 64 if lens else (N + 63) // 64, seed=rank, regime="R1")
     Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
     X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
     Qd, Kd, Vd, Wqd, Wkd = (t.to(dev) for t in (Q, Kk, V, Wq, Wk))
@@ -217,12 +236,23 @@ def run_ours(args, w, rank, world):
 
     if learned:
         layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
+    elif lens:
+        layer = sas.SasLayer(1, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv, max_seqs=len(lens),
+                             max_seqlen=max(lens))
     else:
         layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv)
     h = layer.h
     stream = torch.cuda.current_stream(dev)
+    cud = None
+    if lens:
+        import numpy as np
+        cud = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
 
     def step(Qx, Kx, Vx, Xx, O, Y, Sx=None):
+        if lens:
+            sas.sas_attention_fwd_varlen(h, cud, Qx[0], Kx[0], Vx[0], Sx[0], O[0], LSEd[0], None, None, stream)
+            sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
+            return
         if learned:
             sas.sas_attention_fwd(h, Qx, Kx, Vx, O, None, Wqd, Wkd, LSEd, None, None, stream)
         else:
@@ -291,7 +321,14 @@ def run_ours(args, w, rank, world):
 
     # tile-union statistics of the last forward (executed vs algorithmic work)
     Tt = (N + 127) // 128
-    unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
+    if lens:
+        # packed: the first sum(ceil(n/128)) slots of each group are the tiles in use
+        slots = (N + 127) // 128 + len(lens)
+        used = sum((n + 127) // 128 for n in lens)
+        allc = sas.sas_get_tile_union_counts(h, Hkv * slots)
+        unions = [allc[g * slots + k] for g in range(Hkv) for k in range(used)]
+    else:
+        unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
     layer.close()
 
     ms, e2e_ms = reduce_max([ms, e2e_ms], dist, dev)
@@ -300,7 +337,7 @@ def run_ours(args, w, rank, world):
             dist.destroy_process_group()
         return None
 
-    fl = algorithmic_flops(w, learned)
+    fl = packed_flops(w) if lens else algorithmic_flops(w, learned)
     tflop = fl["total"] / 1e12
     value = job_throughput(tflop, world, ms)
     per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None)} for k, (n, t) in kt.items()}
@@ -325,7 +362,7 @@ def run_ours(args, w, rank, world):
                  "synthetic (seeded; R1 block-coherent selector scores s = u[block] + 0.05 eps given by the caller, "
                  "N(0,1) Q/K/V/X, weights N(0,0.02))"),
         "config": {"workload": w["name"], "B": B, "H": H, "Hkv": Hkv, "N": N, "d": d, "block": 64, "topk": K,
-                   "d_sel": ds,
+                   "d_sel": ds, "packed_lengths": lens,
                    "mlp": [T, D, F, D], "selector": "meanpool_proj" if learned else "scores_given (R1)",
                    "l2": "flushed between timed steps (256 MiB write)",
                    "parallelism": f"replicas x{world}"},
@@ -411,7 +448,7 @@ def oracle_sample(w, budget_s, seed=0, learned=True):
     m_time = time.perf_counter() - t1
     m_rate = m_flops / m_time
 
-    fl = algorithmic_flops(w, learned)
+    fl = packed_flops(w) if w.get("lens") else algorithmic_flops(w, learned)
     full_time = (fl["attention"] + fl["selector"]) / a_rate + fl["mlp"] / m_rate
     rate = fl["total"] / full_time
     how = "with that head's selector" if learned else "with that head's given R1 scores"
@@ -432,14 +469,14 @@ def run_reference(args, w, rank, world):
         return None
     rates = []
     desc = ""
-    learned = args.regime == "R2" and w.get("Hkv", w["H"]) == w["H"]   # the same selector as our arm
+    learned = args.regime == "R2" and w.get("Hkv", w["H"]) == w["H"] and not w.get("lens")   # as our arm
     for k in range(args.warmup + args.steps):
         rate, dt, desc = oracle_sample(w, budget_s=args.ref_step_s, seed=k, learned=learned)
         if k >= args.warmup:
             rates.append(rate)
     # harmonic mean: total FLOPs over total time for equal-work steps
     value = len(rates) / sum(1.0 / r for r in rates) / 1e12
-    full = algorithmic_flops(w, learned)["total"]
+    full = (packed_flops(w) if w.get("lens") else algorithmic_flops(w, learned))["total"]
     ms = full / (value * 1e12) * 1e3
     return {
         "impl": "reference", "metric": METRIC, "value": round(value, 8), "unit": UNIT, "n_gpus": world,
