@@ -307,53 +307,62 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             for (int q = nv - 1; q >= 0 && q >= nv - Cfg::VST; --q)
                 mbar_wait_drain(&v_full[q % Cfg::VST], (q / Cfg::VST) & 1, p.limit, p.status);
         }
-    } else if (warp == 2 && lane == 0) {
-        // ---------------- QK issuer: S = Q K_g^T for every visited block g, once the
-        // softmax warps have loaded S_{g-1}
+    } else if (warp == 2) {
+        // ---------------- QK issuer (whole warp; the elected lane issues): S = Q K_g^T
+        // for every visited block g, once the softmax warps have loaded S_{g-1}
         const uint64_t dq0 = smem_desc_sw128(smem_u32(smem), 16, 1024);
         const uint64_t dk0 = smem_desc_sw128(smem_u32(smem + Cfg::OFF_K), 16, 1024);
         int g = 0, tc = 0;
         bool ok = true;
         for (int r = 0; ok; ++r) {
             int w;
-            if (!read_item(ctl, r, wc, w)) { ok = false; break; }
-            mbar_arrive(&ctl.item_empty[r % kItemSlots]);
+            if (!__all_sync(0xffffffffu, read_item(ctl, r, wc, w))) { ok = false; break; }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
             const int n = tile_blocks(p, tile_ref(p, w, Tn));
-            if (!mbar_wait(&q_full, tc & 1, wc)) { ok = false; break; }
+            if (!mbar_wait_warp(&q_full, tc & 1, wc)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int s = gb % Cfg::KST;
-                if (!mbar_wait(&k_full[s], (gb / Cfg::KST) & 1, wc)) { ok = false; break; }
-                if (gb >= 1 && !mbar_wait(&s_free, (gb - 1) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait_warp(&k_full[s], (gb / Cfg::KST) & 1, wc)) { ok = false; break; }
+                if (gb >= 1 && !mbar_wait_warp(&s_free, (gb - 1) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
                 // descriptors advance by (byte offset >> 4) in their start-address field
                 const uint64_t dk = dk0 + static_cast<uint64_t>((s * Cfg::KV_BYTES) >> 4);
+                if (elect_one()) {
 #pragma unroll
-                for (int k = 0; k < D / 16; ++k) {
-                    const uint32_t off_q = (k >> 2) * (kBM * 128) + (k & 3) * 32;
-                    const uint32_t off_k = (k >> 2) * (kBN * 128) + (k & 3) * 32;
-                    umma_bf16(tmem_base + Cfg::TMEM_S, dq0 + (off_q >> 4), dk + (off_k >> 4), Cfg::IDESC_S, k > 0);
+                    for (int k = 0; k < D / 16; ++k) {
+                        const uint32_t off_q = (k >> 2) * (kBM * 128) + (k & 3) * 32;
+                        const uint32_t off_k = (k >> 2) * (kBN * 128) + (k & 3) * 32;
+                        umma_bf16(tmem_base + Cfg::TMEM_S, dq0 + (off_q >> 4), dk + (off_k >> 4), Cfg::IDESC_S,
+                                  k > 0);
+                    }
+                    umma_commit(&s_full);
+                    umma_commit(&k_empty[s]);
+                    if (j == n - 1) umma_commit(&q_empty);   // Q slot free for the next tile
                 }
-                umma_commit(&s_full);
-                umma_commit(&k_empty[s]);
-                if (j == n - 1) umma_commit(&q_empty);   // Q slot free for the next tile
+                __syncwarp();
             }
             g += n;
             ++tc;
         }
-        umma_commit(&drain_bar);
-        mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
-    } else if (warp == 3 && lane == 0) {
-        // ---------------- PV issuer: O += P_g V_g for every visited block g; the first
-        // block of a tile starts a new accumulator
+        if (elect_one()) {
+            umma_commit(&drain_bar);
+            mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+        }
+        __syncwarp();
+    } else if (warp == 3) {
+        // ---------------- PV issuer (whole warp; the elected lane issues): O += P_g V_g
+        // for every visited block g; the first block of a tile starts a new accumulator
         const uint64_t dv0 = smem_desc_sw128(smem_u32(smem + Cfg::OFF_V), kBN * 128, 1024);
         int g = 0;
         bool ok = true;
         for (int r = 0; ok; ++r) {
             int w;
-            if (!read_item(ctl, r, wc, w)) { ok = false; break; }
-            mbar_arrive(&ctl.item_empty[r % kItemSlots]);
+            if (!__all_sync(0xffffffffu, read_item(ctl, r, wc, w))) { ok = false; break; }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.item_empty[r % kItemSlots]);
             if (w < 0) break;
             const int n = tile_blocks(p, tile_ref(p, w, Tn));
             for (int j = 0; j < n; ++j) {
@@ -361,25 +370,31 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
                 const int vs = gb % Cfg::VST;
                 // p_full[gb&1] cannot run two phases ahead: the softmax writes P_{gb+2}
                 // only after PV_gb (issued after this wait) has read the buffer.
-                if (!mbar_wait(&p_full[gb & 1], (gb >> 1) & 1, wc)) { ok = false; break; }
-                if (!mbar_wait(&v_full[vs], (gb / Cfg::VST) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait_warp(&p_full[gb & 1], (gb >> 1) & 1, wc)) { ok = false; break; }
+                if (!mbar_wait_warp(&v_full[vs], (gb / Cfg::VST) & 1, wc)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t dv = dv0 + static_cast<uint64_t>((vs * Cfg::KV_BYTES) >> 4);
+                if (elect_one()) {
 #pragma unroll
-                for (int k = 0; k < kBN / 16; ++k) {
-                    // P_gb sits in P buffer gb & 1 (16 keys = 8 packed columns per step).
-                    // V is MN-major (d contiguous): 16 keys = two 8-row atoms (2048 bytes);
-                    // the two 64-wide d halves sit kBN*128 bytes apart.
-                    umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + Cfg::TMEM_P + (gb & 1) * 32 + k * 8,
-                                 dv + ((k * 2048) >> 4), Cfg::IDESC_O, (j > 0 || k > 0) ? 1u : 0u);
+                    for (int k = 0; k < kBN / 16; ++k) {
+                        // P_gb sits in P buffer gb & 1 (16 keys = 8 packed columns per step).
+                        // V is MN-major (d contiguous): 16 keys = two 8-row atoms (2048 bytes);
+                        // the two 64-wide d halves sit kBN*128 bytes apart.
+                        umma_bf16_ta(tmem_base + Cfg::TMEM_O, tmem_base + Cfg::TMEM_P + (gb & 1) * 32 + k * 8,
+                                     dv + ((k * 2048) >> 4), Cfg::IDESC_O, (j > 0 || k > 0) ? 1u : 0u);
+                    }
+                    umma_commit(&pv_done[gb & 1]);
+                    umma_commit(&v_empty[vs]);
                 }
-                umma_commit(&pv_done[gb & 1]);
-                umma_commit(&v_empty[vs]);
+                __syncwarp();
             }
             g += n;
         }
-        umma_commit(&drain_bar);
-        mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+        if (elect_one()) {
+            umma_commit(&drain_bar);
+            mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+        }
+        __syncwarp();
     } else if (warp >= 4) {
         // ---------------- softmax / correction / epilogue: one thread per row
         const int q = warp - 4;
