@@ -128,6 +128,23 @@ def selector_scores(Q, K, Wq, Wk, b):
     return (qt @ kt.T) / math.sqrt(d_s)
 
 
+def selector_scores_group(Qg, K, Wq_g, Wk, b):
+    """a2 for a GQA group (MEANPOOL_PROJ reading, group gate query): one score
+    table for the G query heads of a KV group, so that they share one Top-K
+    (Sec. 5.3).  The paper does not say how the G heads form one gate query;
+    the reading is q~_i = bf16(Wq_g [q_{0,i}; ...; q_{G-1,i}]) with
+    Wq_g [d_s, G d] (G = 1 is selector_scores; averaging the heads is the
+    special case Wq_g = [W ... W] / G), and K~_m = bf16(Wk Kbar_m) of the
+    group's keys.  Qg: [G, N, d]; K: [N, d]; Wk: [d_s, d].
+    """
+    G, N, d = Qg.shape
+    d_s = Wq_g.shape[0]
+    qcat = np.concatenate([Qg[h] for h in range(G)], axis=1)   # [N, G d], head-major
+    qt = round_to_bf16(qcat @ Wq_g.T)
+    kt = round_to_bf16(block_summaries(K, b) @ Wk.T)
+    return (qt @ kt.T) / math.sqrt(d_s)
+
+
 # --------------------------------------------------------------- a3 / a4 --
 
 def log_gates(s_hist, act=GATE_SOFTMAX):
@@ -285,14 +302,16 @@ def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,
     return out
 
 
-def sas_attention_gqa(Q, K, V, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=None,
-                      heads=None, rows=None, act=GATE_SOFTMAX, pos=GATE_INNER):
+def sas_attention_gqa(Q, K, V, b, topk, scores=None, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                      heads=None, rows=None, act=GATE_SOFTMAX, pos=GATE_INNER, Wq=None, Wk=None):
     """GQA form with group-shared selection (Sec. 5.3: the query heads of a
     GQA group share one Top-K; Sec. 5 inference implementation: Top-K per
     query group).  Q [B, Hq, N, d]; K, V [B, Hkv, N, d]; scores
     [B, Hkv, N, >=C-1], one table per KV group; Hq = G Hkv, query head h
     belongs to group h // G.  Every query head attends with its group's K,
-    V, kept blocks and log-gates.  Returns {(bi, h): result-dict}.
+    V, kept blocks and log-gates.  Without scores, the learned selector with
+    the group gate query (selector_scores_group; Wq [Hkv, d_s, G d], Wk
+    [Hkv, d_s, d]) gives each group's table.  Returns {(bi, h): result-dict}.
     """
     Bn, Hq, N, d = Q.shape
     Hkv = K.shape[1]
@@ -301,9 +320,16 @@ def sas_attention_gqa(Q, K, V, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=N
     G = Hq // Hkv
     heads = [(bi, hi) for bi in range(Bn) for hi in range(Hq)] if heads is None else heads
     out = {}
+    tables = {}
     for bi, hi in heads:
         g = hi // G
-        out[(bi, hi)] = sas_attention_head(Q[bi, hi], K[bi, g], V[bi, g], scores[bi, g], b,
+        if scores is not None:
+            sg = scores[bi, g]
+        else:
+            if (bi, g) not in tables:
+                tables[(bi, g)] = selector_scores_group(Q[bi, g * G:(g + 1) * G], K[bi, g], Wq[g], Wk[g], b)
+            sg = tables[(bi, g)]
+        out[(bi, hi)] = sas_attention_head(Q[bi, hi], K[bi, g], V[bi, g], sg, b,
                                            topk, mode, sm_scale, rows, act, pos)
     return out
 

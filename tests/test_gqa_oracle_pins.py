@@ -68,3 +68,57 @@ def test_query_heads_must_fill_whole_groups():
     Q, K, V, s = _inputs(1, 3, 2, 16, 2, 1)
     with pytest.raises(ValueError):
         O.sas_attention_gqa(Q, K, V, 8, 1, s)
+
+
+def test_group_gate_query_reduces_to_the_head_selector():
+    # G = 1: the group gate query is the per-head selector
+    rng = np.random.default_rng(3)
+    N, d, ds = 70, 6, 4
+    Q, K = rng.standard_normal((1, N, d)), rng.standard_normal((N, d))
+    Wq, Wk = rng.standard_normal((ds, d)), rng.standard_normal((ds, d))
+    assert np.array_equal(O.selector_scores_group(Q, K, Wq, Wk, 8), O.selector_scores(Q[0], K, Wq, Wk, 8))
+    # G = 3 with weight only on head 1's slice: head 1's per-head selector, exactly
+    Qg = rng.standard_normal((3, N, d))
+    Wg = np.zeros((ds, 3 * d))
+    Wg[:, d:2 * d] = Wq
+    assert np.array_equal(O.selector_scores_group(Qg, K, Wg, Wk, 8), O.selector_scores(Qg[1], K, Wq, Wk, 8))
+
+
+def test_group_gate_query_with_equal_slices_is_the_sum_of_the_heads():
+    # Wq_g = [W W] makes q~ = bf16(W (q_0 + q_1)): the selector of the summed queries
+    rng = np.random.default_rng(4)
+    N, d, ds = 64, 4, 4
+    Qg, K = rng.standard_normal((2, N, d)), rng.standard_normal((N, d))
+    W, Wk = rng.standard_normal((ds, d)), rng.standard_normal((ds, d))
+    a = O.selector_scores_group(Qg, K, np.concatenate([W, W], axis=1), Wk, 8)
+    b = O.selector_scores(Qg[0] + Qg[1], K, W, Wk, 8)
+    assert np.allclose(a, b, rtol=0, atol=1e-12)
+
+
+def test_learned_gqa_uses_one_table_per_group():
+    rng = np.random.default_rng(5)
+    B, Hkv, G, N, d, ds = 1, 2, 2, 48, 4, 4
+    Q = rng.standard_normal((B, Hkv * G, N, d))
+    K, V = rng.standard_normal((B, Hkv, N, d)), rng.standard_normal((B, Hkv, N, d))
+    Wq, Wk = rng.standard_normal((Hkv, ds, G * d)), rng.standard_normal((Hkv, ds, d))
+    a = O.sas_attention_gqa(Q, K, V, 8, 2, Wq=Wq, Wk=Wk)
+    for g in range(Hkv):
+        s = O.selector_scores_group(Q[0, g * G:(g + 1) * G], K[0, g], Wq[g], Wk[g], 8)
+        ref = O.sas_attention_gqa(Q, K, V, 8, 2, scores=np.broadcast_to(s, (B, Hkv) + s.shape).copy())
+        for h in range(g * G, (g + 1) * G):
+            assert np.array_equal(a[(0, h)]["O"], ref[(0, h)]["O"])
+            assert np.array_equal(a[(0, h)]["sel_idx"], ref[(0, h)]["sel_idx"])
+
+
+def test_group_gate_query_agrees_with_the_decode_oracle():
+    # the decode step (its own oracle module) reads the group gate query the same
+    # way: its scores for the newest token are the last prefill row's
+    from oracle import decode_oracle as D
+    rng = np.random.default_rng(6)
+    G, n, d, ds, b = 4, 200, 8, 4, 16
+    Qg, K, V = rng.standard_normal((G, n, d)), rng.standard_normal((n, d)), rng.standard_normal((n, d))
+    Wq, Wk = rng.standard_normal((ds, G * d)), rng.standard_normal((ds, d))
+    pre = O.selector_scores_group(Qg, K, Wq, Wk, b)
+    dec = D.decode_group(Qg[:, n - 1, :], K, V, Wq, Wk, b, 3)
+    C = (n - 1) // b
+    assert np.allclose(pre[n - 1, :C], dec["scores"], rtol=0, atol=1e-12)
