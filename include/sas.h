@@ -96,9 +96,9 @@ typedef struct {
     int32_t Hkv;          /* KV heads (GQA); 0 selects H.  H must be a multiple of it:
                              query head h uses KV head h / (H / Hkv), and the G = H / Hkv
                              query heads of a group share one selection (Sec. 5.3;
-                             Sec. 5 inference implementation).  Hkv < H needs
-                             SCORES_GIVEN (one score table per group) and has no
-                             backward.                                                */
+                             Sec. 5 inference implementation): one score table
+                             per group, given or from the learned selector's group
+                             gate query.  Hkv < H has no backward.                    */
     int32_t max_seqs;     /* 0: [B, H, N, d] batches of N-token sequences.  > 0: packed
                              variable-length sequences, at most max_seqs of them, in
                              [H, N, d] tensors whose token axis (N = capacity) holds
@@ -129,9 +129,13 @@ void sas_destroy(sas_handle* h);
  *             0 .. floor(i/64)-1 and ignores the rest.  Required for
  *             SCORES_GIVEN, must be NULL for MEANPOOL_PROJ.  Scores must
  *             be finite.                                              (in)
- *   Wq, Wk    bf16 [H, d_sel, d] selector projections (linear-layer
- *             layout [out, in]); required for MEANPOOL_PROJ, NULL
- *             otherwise.                                              (in)
+ *   Wq        bf16 [Hkv, d_sel, G d], G = H / Hkv: the gate-query
+ *             projection of each KV group, applied to its G query heads'
+ *             rows concatenated head by head, q~ = bf16(Wq [q_0; ...;
+ *             q_{G-1}]) ([H, d_sel, d] without GQA);
+ *   Wk        bf16 [Hkv, d_sel, d] key projection of the block summaries.
+ *             Linear-layer layout [out, in]; required for MEANPOOL_PROJ,
+ *             NULL otherwise.                                         (in)
  *   O         bf16 [B, H, N, d]                                       (out)
  *   LSE       fp32 [B, H, N] natural-log log-sum-exp of each row's
  *             gated logits (Alg. 3 output); may be NULL.              (out)

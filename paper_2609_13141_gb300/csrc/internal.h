@@ -51,12 +51,13 @@ cudaError_t launch_pool(const void* K, const void* Wk, void* Kt, int BH, int H, 
 // scores, the Top-K blocks (ascending, -1 padded) with their log-gates, and
 // per 128-row tile the sorted union of kept blocks below the tile's diagonal.
 struct SelectArgs {
-    int BH, H, N, C, T, topk, d_sel;
+    int BH, H, N, C, T, topk, d_sel;   // BH, H: selection groups (KV heads) x batch, KV heads
+    int G;                          // query heads per group (MEANPOOL_PROJ: the gate query reads all G)
     int gate_act;                   // 0 softmax (log g = s - LSE), 1 sigmoid, 2 logit (log g = s)
     float score_scale;              // 1/sqrt(d_sel) for projected scores, 1 for given scores
     const float* scores;            // SCORES_GIVEN: [BH][N][C]
     const void* Q;                  // MEANPOOL_PROJ: queries bf16 [BH][N][d]
-    const void* Wq;                 // MEANPOOL_PROJ: query projection bf16 [H][d_sel][d]
+    const void* Wq;                 // MEANPOOL_PROJ: gate-query projection bf16 [H][d_sel][G d]
     const void* Kt;                 // MEANPOOL_PROJ: projected block summaries bf16 [BH][F][d_sel]
     int d;
     int F;

@@ -530,10 +530,14 @@ __host__ __device__ constexpr size_t proj_region0(int K) {
 template <int D, int DS, bool REG>
 __global__ void __launch_bounds__(192, 2)
 select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapWq,
-                   const __grid_constant__ CUtensorMap mapKt, SelParams p, int H) {
+                   const __grid_constant__ CUtensorMap mapKt, SelParams p, int H, int G) {
+    // H: KV heads (selection groups), G: query heads per group.  The gate query of
+    // group bh is q~ = Wq[bh % H] [q_{bh G}; ...; q_{bh G + G - 1}]: G rounds that
+    // each stage one head's Q tile and its d columns of Wq and accumulate.
     using Cfg = SelProjCfg<D, DS>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    __shared__ uint64_t in_full, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2], drain_bar;
+    __shared__ uint64_t in_full, in_empty, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2],
+        drain_bar;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
 
@@ -557,6 +561,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
     if (threadIdx.x == 0) {
         mbar_init(&in_full, 1);
+        mbar_init(&in_empty, 1);
         mbar_init(&proj_done, 1);
         mbar_init(&qt_ready, 4);
         for (int b = 0; b < 2; ++b) {
@@ -584,14 +589,21 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             tma_prefetch_desc(&mapQ);
             tma_prefetch_desc(&mapWq);
             tma_prefetch_desc(&mapKt);
-            mbar_arrive_expect_tx(&in_full, Cfg::Q_BYTES + Cfg::WQ_BYTES);
+            bool ok = true;
+            int rounds = 0;
+            for (int hq = 0; hq < G; ++hq) {
+                // round hq: query head bh G + hq and its columns hq D .. hq D + D - 1 of Wq
+                if (hq > 0 && !mbar_wait(&in_empty, (hq - 1) & 1, wc)) { ok = false; break; }
+                mbar_arrive_expect_tx(&in_full, Cfg::Q_BYTES + Cfg::WQ_BYTES);
 #pragma unroll
-            for (int a = 0; a < D / 64; ++a) {
-                tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, t * kRows, bh);
-                tma_load_3d(b_s + a * (DS * 128), &mapWq, &in_full, a * 64, 0, bh % H);
+                for (int a = 0; a < D / 64; ++a) {
+                    tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, t * kRows, bh * G + hq);
+                    tma_load_3d(b_s + a * (DS * 128), &mapWq, &in_full, hq * D + a * 64, 0, bh % H);
+                }
+                ++rounds;
             }
             int issued = 0;
-            bool ok = mbar_wait(&proj_done, 0, wc);   // region B is free once the projection ran
+            if (ok) ok = mbar_wait(&proj_done, 0, wc);   // region B is free once the projection ran
             for (int c = 0; ok && c < nchunks; ++c) {
                 const int b = c & 1;
                 if (!mbar_wait(&kc_empty[b], ((c >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
@@ -602,25 +614,29 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 ++issued;
             }
             if (!ok) {
-                mbar_wait_drain(&in_full, 0, p.limit, p.status);
+                if (rounds > 0) mbar_wait_drain(&in_full, (rounds - 1) & 1, p.limit, p.status);
                 for (int q = issued - 1; q >= 0 && q >= issued - 2; --q)
                     mbar_wait_drain(&kc_full[q & 1], (q >> 1) & 1, p.limit, p.status);
             }
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
-        if (nchunks > 0 && mbar_wait(&in_full, 0, wc)) {
+        bool in_ok = nchunks > 0;
+        const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);
+        for (int hq = 0; in_ok && hq < G; ++hq) {
+            if (!mbar_wait(&in_full, hq & 1, wc)) { in_ok = false; break; }
             tc_fence_after();
-            // q~ (fp32, TMEM columns 0 .. DS-1) = Q (128 x D) * Wq[h] (DS x D)^T
-            const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);
+            // q~ (fp32, TMEM columns 0 .. DS-1) += Q_hq (128 x D) * Wq[h][:, hq D : hq D + D] (DS x D)^T
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
                 const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
                 const uint32_t off_w = (k >> 2) * (DS * 128) + (k & 3) * 32;
                 umma_bf16(tmem_base, smem_desc_sw128(q_addr + off_q, 16, 1024),
-                          smem_desc_sw128(w_addr + off_w, 16, 1024), Cfg::IDESC_PROJ, k > 0);
+                          smem_desc_sw128(w_addr + off_w, 16, 1024), Cfg::IDESC_PROJ, (hq > 0 || k > 0) ? 1u : 0u);
             }
-            umma_commit(&proj_done);
+            umma_commit(hq + 1 < G ? &in_empty : &proj_done);   // regions A, B free for the next round
+        }
+        if (in_ok) {
             // S[c&1] = q~ (128 x DS, bf16 in region A) * Kt_chunk (64 x DS)^T
             if (mbar_wait(&qt_ready, 0, wc)) {
                 for (int c = 0; c < nchunks; ++c) {
@@ -747,11 +763,12 @@ cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv
                                          static_cast<int>(smem));
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mw, mk;
-    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kRows) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
-    if (make_tmap_bf16_3d(&mw, a.Wq, D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
+    // Q of all query heads; Wq [H][DS][G D] (a group's gate-query projection)
+    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH * a.G, 64, kRows) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mw, a.Wq, static_cast<uint64_t>(a.G) * D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
     const dim3 grid(a.BH * a.T);
-    select_proj_kernel<D, DS, REG><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H);
+    select_proj_kernel<D, DS, REG><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H, a.G);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;

@@ -225,7 +225,6 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
     const int Hkv = c.Hkv == 0 ? c.H : c.Hkv;
     if (Hkv < 1 || Hkv > c.H || c.H % Hkv != 0) return SAS_ERR_INVALID_ARG;
-    if (Hkv != c.H && c.selector != SAS_SEL_SCORES_GIVEN) return SAS_ERR_UNSUPPORTED;
     if (c.max_seqs < 0 || c.max_seqlen < 0 || c.max_seqlen > c.N) return SAS_ERR_INVALID_ARG;
     const bool varlen = c.max_seqs > 0;
     if (varlen && c.B != 1) return SAS_ERR_INVALID_ARG;
@@ -257,7 +256,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     cudaError_t e = cudaSuccess;
     const size_t rows = static_cast<size_t>(BHkv) * c.N;   // selection rows: one per group and token
     if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
-        if (e == cudaSuccess) e = alloc(&h->Kt, static_cast<size_t>(BH) * (h->F > 0 ? h->F : 1) * d_sel * 2);
+        if (e == cudaSuccess) e = alloc(&h->Kt, static_cast<size_t>(BHkv) * (h->F > 0 ? h->F : 1) * d_sel * 2);
     }
     if (e == cudaSuccess) e = alloc(&h->union_idx, static_cast<size_t>(BHkv) * h->T * h->C * 4);
     if (e == cudaSuccess) e = alloc(&h->union_cnt, static_cast<size_t>(BHkv) * h->T * 4);
@@ -334,13 +333,16 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     if (c.selector == SAS_SEL_MEANPOOL_PROJ) {
         // a1: block summaries -> projected summaries
         if (h->F > 0) {
-            e = timed_launch(h, 0, s, [&] { return sas::launch_pool(K, Wk, h->Kt, h->BH, c.H, c.N, c.d, h->d_sel, env); });
+            e = timed_launch(h, 0, s, [&] {
+                return sas::launch_pool(K, Wk, h->Kt, h->BHkv, h->Hkv, c.N, c.d, h->d_sel, env);   // per KV group
+            });
             if (e != cudaSuccess) return cuda_fail(h, e, "block summaries");
         }
     }
     // a2-a4: query projection (learned selector), scores, log-gates, Top-K, tile unions
     sas::SelectArgs sa{};
     sa.BH = h->BHkv; sa.H = h->Hkv; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.G = h->G;
     sa.gate_act = c.gate_act;
     sa.score_scale = c.selector == SAS_SEL_MEANPOOL_PROJ ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
     sa.scores = scores;
@@ -389,6 +391,7 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     // tile table, then a2-a4 over the tiles of every sequence
     sas::SelectArgs sa{};
     sa.BH = h->BHkv; sa.H = h->Hkv; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
+    sa.G = h->G;
     sa.gate_act = c.gate_act;
     sa.score_scale = 1.0f;
     sa.scores = scores;

@@ -52,7 +52,6 @@ def test_status_strings(lib):
     (dict(B=1, H=6, N=128, d=64, topk=2, Hkv=4), sas.SAS_ERR_INVALID_ARG),      # H not a multiple of Hkv
     (dict(B=1, H=2, N=128, d=64, topk=2, Hkv=4), sas.SAS_ERR_INVALID_ARG),      # more KV heads than heads
     (dict(B=1, H=2, N=128, d=64, topk=2, Hkv=-1), sas.SAS_ERR_INVALID_ARG),
-    (dict(B=1, H=4, N=128, d=64, topk=2, Hkv=2, selector=1), sas.SAS_ERR_UNSUPPORTED),   # GQA needs given scores
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=-1), sas.SAS_ERR_INVALID_ARG),
     (dict(B=2, H=2, N=128, d=64, topk=2, max_seqs=4), sas.SAS_ERR_INVALID_ARG),          # packed needs B = 1
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=4, selector=1), sas.SAS_ERR_UNSUPPORTED),

@@ -100,3 +100,37 @@ def test_gqa_backward_is_refused():
         layer.attention_bwd(Q, K, K, O, LSE, O, scores=S, sel_idx=si, sel_logg=sl)
     assert e.value.status == sas.SAS_ERR_UNSUPPORTED
     layer.close()
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,N,d,d_sel,topk", [
+    (1, 8, 2, 1000, 128, 128, 4),     # G = 4
+    (2, 4, 2, 700, 64, 64, 3),        # G = 2, d = 64
+])
+def test_gqa_learned_selector_exact_inputs(B, Hq, Hkv, N, d, d_sel, topk):
+    # integer Q, K and {-1, 0, 1} projections: every selector sum is exact in fp32,
+    # so the group gate query's kept sets must equal the oracle's on every row
+    G = Hq // Hkv
+    Q = synth.integer_selector_inputs(B, Hq, N, d, d_sel, seed=Hq)[0]
+    _, K, V, _, _ = synth.integer_selector_inputs(B, Hkv, N, d, d_sel, seed=Hq + 1)
+    Wq, Wk = synth.decode_selector_weights(Hkv, G, d, d_sel, seed=Hq, exact=True)
+    dev = torch.device("cuda:0")
+    layer = sas.SasLayer(B, Hq, N, d, topk, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=d_sel, Hkv=Hkv)
+    O, LSE, si, sl = layer.attention(*(t.to(dev).contiguous() for t in (Q, K, V)), Wq=Wq.to(dev), Wk=Wk.to(dev))
+    T = -(-N // 128)
+    unions = np.array(sas.sas_get_tile_union_counts(layer.h, B * Hkv * T)).reshape(B, Hkv, T)
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    ref = OR.sas_attention_gqa(P.f64(Q), P.f64(K), P.f64(V), 64, topk, Wq=P.f64(Wq), Wk=P.f64(Wk))
+    for bi in range(B):
+        for g in range(Hkv):
+            s = OR.selector_scores_group(P.f64(Q[bi, g * G:(g + 1) * G]), P.f64(K[bi, g]), P.f64(Wq[g]),
+                                         P.f64(Wk[g]), 64)
+            gi = si[bi, g].cpu().numpy()[:, :topk]
+            P.check_selection_rows(gi, s, np.arange(N), topk)
+            assert np.array_equal(unions[bi, g], P.oracle_union_counts(gi, N, topk))
+            lg = sl[bi, g].cpu().numpy()[:, :topk]
+            assert np.abs(lg - ref[(bi, g * G)]["sel_logg"]).max(initial=0) <= P.LOGG_MAX_ABS
+        for hi in range(Hq):
+            r = ref[(bi, hi)]
+            P.compare_o(P.f64(O[bi, hi].cpu()), r["O"], f"O[{bi},{hi}]", max(1.0, np.abs(r["O"]).max()))
+            assert np.abs(LSE[bi, hi].cpu().numpy() - r["LSE"]).max() <= P.LSE_MAX_ABS
