@@ -43,6 +43,11 @@ reasoning in the design notes of the repository):
     exists to check it against; only its arithmetic is pinned.
   * MLP: the hidden activation GELU(X W1^T + b1) is a bf16 tensor between the
     two products (the precision of a stored bf16 activation).
+  * GQA: the G query heads of a KV group share one selection (Sec. 5.3); with
+    the learned selector the group's gate query is q~ = bf16(Wq_g [q_0; ...;
+    q_{G-1}]), Wq_g [d_s, G d] (the paper does not say how the heads combine).
+  * Packed sequences: each is its own causal problem; its blocks start at its
+    first token.
 
 Arrays are float64 numpy arrays holding the bf16-rounded inputs the GPU sees.
 One "head" means one (batch, head) pair; Q, K, V of a head are [N, d].
