@@ -179,9 +179,11 @@ sas_status sas_attention_fwd(sas_handle* h,
  *              LSE_i = s_m - log g_m from its first kept entry, so the
  *              scores must be the ones the forward selected with     (out)
  * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
- * allocates the handle's backward workspace, and every call reads back how
- * many blocks the forward's tiles visit to size a buffer: the call
- * synchronises with its stream once (so it cannot be captured in a graph). */
+ * allocates the handle's backward workspace (synchronously); later calls are
+ * asynchronous and can be captured in a CUDA graph when B * H * T * (T + 1)
+ * * 512 bytes <= 8 GiB (T = ceil(N / 128)).  Above that size every call reads
+ * back how many blocks the forward's tiles visit, to size a buffer, and so
+ * synchronises with its stream once. */
 sas_status sas_attention_bwd(sas_handle* h,
                              const void* Q, const void* K, const void* V,
                              const float* scores,

@@ -845,6 +845,7 @@ cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long lo
     const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
     bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.slot_off, nullptr, tiles);
+    if (total == nullptr) return cudaGetLastError();   // the caller's buffer holds the upper bound
     int32_t host = 0;
     cudaError_t e = cudaMemcpyAsync(&host, a.slot_off + tiles, 4, cudaMemcpyDeviceToHost, env.stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(env.stream);

@@ -113,6 +113,7 @@ struct sas_handle {
     float* bwd_dlogg = nullptr;
     float* bwd_offs = nullptr;      // per-row offsets of every visited block (pass 1 -> pass 2)
     size_t bwd_offs_bytes = 0;
+    bool bwd_offs_bound = false;    // sized for the upper bound: no per-call read-back
     // timing
     bool timing = false;
     std::vector<TimeRec> recs;
@@ -502,6 +503,16 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         if (e == cudaSuccess) e = alloc(&h->bwd_inv, (4 * tiles + 2) * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_tiles, 2 * tiles * pairs * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, rows * (c.topk > 0 ? c.topk : 1) * 4);
+        // offsets of pass 1 for pass 2: a tile visits at most 2t + 2 blocks, so a head
+        // needs at most T (T + 1) slots of 128 rows; held whole when that fits in 8 GiB
+        const size_t bound = tiles * static_cast<size_t>(h->T + 1) * 128 * 4;
+        if (e == cudaSuccess && bound <= (static_cast<size_t>(8) << 30)) {
+            e = alloc(&h->bwd_offs, bound);
+            if (e == cudaSuccess) {
+                h->bwd_offs_bytes = bound;
+                h->bwd_offs_bound = true;
+            }
+        }
         if (e != cudaSuccess) {
             cudaFree(h->bwd_delta); cudaFree(h->bwd_inv); cudaFree(h->bwd_tiles); cudaFree(h->bwd_dlogg);
             h->bwd_delta = nullptr; h->bwd_inv = nullptr; h->bwd_tiles = nullptr; h->bwd_dlogg = nullptr;
@@ -528,13 +539,14 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.sm_scale = h->sm_scale;
     const sas::KernelEnv env{s, h->status, h->limit};
     const char* err = "";
-    // slots of the per-row offsets pass 1 hands to pass 2 (their number depends
-    // on the forward's tile lists: read back, synchronously, to size the buffer)
+    // slots of the per-row offsets pass 1 hands to pass 2: their number depends on
+    // the forward's tile lists; a buffer of the upper bound needs no read-back,
+    // otherwise it is read back (synchronously) to size the buffer
     long long slots = 0;
-    cudaError_t e = sas::launch_bwd_slots(a, env, &slots);
+    cudaError_t e = sas::launch_bwd_slots(a, env, h->bwd_offs_bound ? nullptr : &slots);
     if (e != cudaSuccess) return cuda_fail(h, e, "backward slots");
     const size_t need = static_cast<size_t>(slots) * 128 * 4;
-    if (need > h->bwd_offs_bytes) {
+    if (!h->bwd_offs_bound && need > h->bwd_offs_bytes) {
         cudaFree(h->bwd_offs);
         h->bwd_offs = nullptr;
         h->bwd_offs_bytes = 0;

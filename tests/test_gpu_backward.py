@@ -102,3 +102,32 @@ def test_backward_repeated_calls_identical():
     b = run_bwd(1, 4, 800, 4, TRAIN, seed=7, heads=[(0, 0)])
     for x, y in zip(a, b):
         assert torch.equal(x, y)
+
+
+def test_backward_captured_in_a_cuda_graph_matches_eager():
+    # after the first call has sized the workspace, a backward call is
+    # asynchronous: captured in a CUDA graph, each replay equals the eager result
+    B, H, N, d, K = 1, 4, 1000, 128, 4
+    C = -(-N // 64)
+    Q, Kk, V = (t.to(DEV) for t in synth.qkv(B, H, N, d, seed=8))
+    S = synth.scores(B, H, N, C, seed=8, regime="R1").to(DEV)
+    dO = synth.normal((B, H, N, d), 9).to(torch.bfloat16).to(DEV)
+    layer = sas.SasLayer(B, H, N, d, K)
+    O, LSE, si, sl = layer.attention(Q, Kk, V, scores=S)
+    eager = layer.attention_bwd(Q, Kk, V, O, LSE, dO, scores=S, sel_idx=si, sel_logg=sl, want_ds=True)
+    torch.cuda.synchronize()
+    outs = [torch.empty_like(t) for t in eager]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        st = torch.cuda.current_stream()
+        sas.sas_attention_bwd(layer.h, Q, Kk, V, O, LSE, dO, outs[0], outs[1], outs[2], S, si, sl, outs[3], outs[4],
+                              st)
+    for _ in range(2):
+        for t in outs:
+            t.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        for x, y in zip(eager, outs):
+            assert torch.equal(x, y)
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
