@@ -288,9 +288,11 @@ int64_t sas_launch_count(const sas_handle* h);
 
 /* Copies the per-tile count of historical blocks the attention kernel
  * processes (the union of the kept blocks of the tile's 128 query rows,
- * excluding the tile's own two diagonal blocks) from the last
- * sas_attention_fwd: out[B * Hkv * ceil(N/128)] (one per KV group and
- * tile).  Synchronises. */
+ * excluding the tile's own two diagonal blocks) from the last forward:
+ * out[B * Hkv * T], one per KV group and tile slot, T = ceil(N/128).  A
+ * packed-sequence handle has T = ceil(N/128) + max_seqs slots per group, of
+ * which the first sum_s ceil(n_s/128) hold the sequences' tiles (longest key
+ * history first).  Synchronises. */
 sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n);
 
 /* Failure-path self-test: launches one block that waits on an mbarrier that
