@@ -303,17 +303,18 @@ class SasLayer:
         self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv,
                             max_seqs, max_seqlen)
 
-    def attention_varlen(self, cu_seqlens, Q, K, V, scores, want_sel=True, stream=None):
+    def attention_varlen(self, cu_seqlens, Q, K, V, scores, want_sel=True, stream=None, sel_fill=-1):
         """Packed sequences (handle made with max_seqs > 0): Q [H, N, d], K/V [Hkv, N, d],
-        scores [Hkv, N, C], cu_seqlens int32 on the device.  Rows past cu[-1] keep the
-        values the output tensors were created with (zeros here)."""
+        scores [Hkv, N, C], cu_seqlens int32 on the device.  The library does not write
+        rows past cu[-1]: they keep the fill of the tensors made here (0, and sel_fill
+        in sel_idx)."""
         dev = Q.device
         O = torch.zeros_like(Q)
         LSE = torch.zeros(self.H, self.N, device=dev, dtype=torch.float32)
         sel_idx = sel_logg = None
         if want_sel:
             k = max(self.topk, 1)
-            sel_idx = torch.full((self.Hkv, self.N, k), -7, device=dev, dtype=torch.int32)
+            sel_idx = torch.full((self.Hkv, self.N, k), sel_fill, device=dev, dtype=torch.int32)
             sel_logg = torch.zeros(self.Hkv, self.N, k, device=dev, dtype=torch.float32)
         sas_attention_fwd_varlen(self.h, cu_seqlens, Q, K, V, scores, O, LSE, sel_idx, sel_logg, stream)
         return O, LSE, sel_idx, sel_logg

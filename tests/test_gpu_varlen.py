@@ -26,7 +26,8 @@ def _packed(lens, cap, Hq, Hkv, d, max_len, seed):
 
 def _run(lens, cap, Hq, Hkv, d, topk, mode, max_len, Q, K, V, S, cu):
     layer = sas.SasLayer(1, Hq, cap, d, topk, mode=mode, Hkv=Hkv, max_seqs=max(len(lens), 1), max_seqlen=max_len)
-    O, LSE, si, sl = layer.attention_varlen(cu.to(DEV), *(t.to(DEV).contiguous() for t in (Q, K, V, S)))
+    O, LSE, si, sl = layer.attention_varlen(cu.to(DEV), *(t.to(DEV).contiguous() for t in (Q, K, V, S)),
+                                            sel_fill=-7)   # a value the library never writes
     status = sas.sas_get_device_status(layer.h)
     layer.close()
     return {"O": O.cpu(), "LSE": LSE.cpu(), "sel_idx": si.cpu(), "sel_logg": sl.cpu(), "status": status}
