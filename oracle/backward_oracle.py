@@ -90,3 +90,47 @@ def backward_flops_head(N, b, topk, d, sel_counts=None):
         kept = min(topk, c)
         pairs += kept * b + (i - c * b + 1)
     return 10 * d * pairs
+
+
+def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
+    """Gradients of the GQA forward (group-shared selection, Sec. 5.3) of one
+    batch element.  Q, dO: [Hq, N, d]; K, V: [Hkv, N, d]; s: [Hkv, N, >=C-1];
+    Hq = G Hkv, query head h uses group h // G.  A group's K, V and log-gates
+    enter the logits of all its G heads, so their gradients are the sums of
+    the heads' contributions: dK_g, dV_g, dlogg_g = sum over the group of the
+    per-head terms, and the score gradient applies the gate softmax's
+    Jacobian (App. D) to the summed dlogg: ds_m = dl_m [m kept] - g_m sum dl.
+    Returns dict with dQ [Hq, N, d], dK, dV [Hkv, N, d], dlogg [Hkv, N, topk],
+    ds [Hkv, N, C].
+    """
+    Hq, N, d = Q.shape
+    Hkv = K.shape[0]
+    if Hq % Hkv:
+        raise ValueError("Hq must be a multiple of Hkv")
+    G = Hq // Hkv
+    C = -(-N // b)
+    dQ = np.zeros_like(Q, dtype=np.float64)
+    dK = np.zeros((Hkv, N, d))
+    dV = np.zeros((Hkv, N, V.shape[2]))
+    dlogg = np.zeros((Hkv, N, max(topk, 1)))[:, :, :topk]
+    ds = np.zeros((Hkv, N, C))
+    for h in range(Hq):
+        g = h // G
+        r = sas_attention_bwd_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, mode, sm_scale)
+        dQ[h] = r["dQ"]
+        dK[g] += r["dK"]
+        dV[g] += r["dV"]
+        dlogg[g] += r["dlogg"]
+    if mode == MODE_TRAIN_SOFT:
+        for g in range(Hkv):
+            for i in range(N):
+                c = historical_count(i, b)
+                if c == 0:
+                    continue
+                _, _, _, sel, _ = _row_keys_and_bias(i, s[g, i], b, topk, mode)
+                dl = np.zeros(c)
+                for e, m in enumerate(sel):
+                    dl[m] = dlogg[g, i, e]
+                gates = np.exp(log_gates(np.asarray(s[g, i][:c], dtype=np.float64)))
+                ds[g, i, :c] = dl - gates * dl.sum()
+    return {"dQ": dQ, "dK": dK, "dV": dV, "dlogg": dlogg, "ds": ds}

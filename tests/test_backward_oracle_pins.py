@@ -121,3 +121,52 @@ def test_delta_is_rowsum_of_o_times_do():
     r = BO.sas_attention_bwd_head(Q, K, V, s, dO, b, topk)
     fwd = O.sas_attention_head(Q, K, V, s, b, topk)
     assert np.allclose(r["Delta"], (fwd["O"] * dO).sum(axis=1), atol=1e-13)
+
+
+def test_gqa_backward_equals_autograd_with_shared_keys_values_and_gates():
+    # one group of G = 2 heads over shared K, V and scores: torch autograd through the
+    # dense masked form of both heads (the same shared tensors feed both) gives the
+    # sums the GQA oracle must produce
+    b, d, N, topk, G = 8, 4, 30, 2, 2
+    rng = np.random.default_rng(21)
+    Q = rng.standard_normal((G, N, d))
+    K, V = rng.standard_normal((1, N, d)), rng.standard_normal((1, N, d))
+    s = rng.standard_normal((1, N, -(-N // b)))
+    dO = rng.standard_normal((G, N, d))
+    sm = 1 / math.sqrt(d)
+    t = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
+    kk, vv, st = t(K[0]), t(V[0]), t(s[0])
+    qs = [t(Q[h]) for h in range(G)]
+    loss = 0
+    for h in range(G):
+        rows = []
+        for i in range(N):
+            c = i // b
+            bias = torch.full((N,), -math.inf, dtype=torch.float64)
+            if c:
+                lg = torch.log_softmax(st[i, :c], dim=0)
+                for m in O.topk_blocks(s[0, i, :c], topk):
+                    bias = torch.cat([bias[:m * b], lg[m].expand(b), bias[(m + 1) * b:]])
+            bias = torch.cat([bias[:c * b], torch.zeros(i + 1 - c * b, dtype=torch.float64), bias[i + 1:]])
+            rows.append(bias)
+        P = torch.softmax(sm * qs[h] @ kk.T + torch.stack(rows), dim=1)
+        loss = loss + ((P @ vv) * torch.tensor(dO[h])).sum()
+    loss.backward()
+    r = BO.sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk)
+    for h in range(G):
+        assert np.allclose(r["dQ"][h], qs[h].grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dK"][0], kk.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dV"][0], vv.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["ds"][0], st.grad.numpy()[:, :r["ds"].shape[2]], atol=1e-12)
+
+
+def test_gqa_backward_with_one_head_per_group_is_the_head_backward():
+    b, d, N, topk = 8, 3, 26, 2
+    rng = np.random.default_rng(22)
+    Q, K, V, dO = (rng.standard_normal((2, N, d)) for _ in range(4))
+    s = rng.standard_normal((2, N, 4))
+    r = BO.sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk)
+    for h in range(2):
+        m = BO.sas_attention_bwd_head(Q[h], K[h], V[h], s[h], dO[h], b, topk)
+        for f in ("dQ", "dK", "dV", "dlogg", "ds"):
+            assert np.allclose(r[f][h], m[f], atol=1e-13), f
