@@ -24,6 +24,11 @@ gate gradient and the sparse-scope score gradient):
 
 Selection (which blocks are kept) is taken from the forward: the gradient
 treats it as fixed, as the kernels do.
+
+GQA (sas_attention_bwd_gqa): a group's K, V and log-gates feed its G query
+heads, so dK, dV and d(log g) are sums over the heads, and the score
+gradient applies the gate softmax's Jacobian to the summed d(log g).  The
+library has no kernel for it yet.
 """
 from __future__ import annotations
 
