@@ -7,13 +7,16 @@
 //                     on the tensor cores, P = exp(S + log g - LSE) and
 //                     dS = P (dP - Delta) per row, dS into TMEM as the A
 //                     operand of dQ += dS K; the row sum of dS over a kept
-//                     block is that row's log-gate gradient.
+//                     block is that row's log-gate gradient.  Also writes
+//                     Delta and, per (visited block, row), log g - LSE for
+//                     pass 2 (slots from bwd_slots + a scan).
 //   bwd_inv_*         the forward's per-tile block lists inverted into, per
 //                     key pair (blocks 2p, 2p+1), the query tiles that visit
 //                     them (count, scan, fill).
 //   bwd_dkv_kernel    pass 2, one CTA per (head, key pair) over those query
-//                     tiles, 64 rows at a time: S^T = K Q^T, dP^T = V dO^T,
-//                     P^T and dS^T into TMEM, dV += P^T dO and dK += dS^T Q.
+//                     tiles, 64 rows at a time: S^T = K Q^T, dP^T = V dO^T
+//                     into two TMEM buffers, P^T and dS^T written in place
+//                     over them, dV += P^T dO and dK += dS^T Q.
 //   bwd_ds_kernel     score gradient of given scores (sparse scope):
 //                     ds_m = dlogg_m [m kept] - g_m sum dlogg.
 // Roles, pass 1: warps 0-7 are the rows (two threads per TMEM lane, half a
@@ -34,7 +37,7 @@ constexpr int kKeys = 64;           // keys per block
 constexpr int kD = 128;             // head dim
 constexpr int kWorkers = 128;       // key threads (pass 2)
 constexpr int kRowThreads = 256;    // pass 1: two threads per row, 32 keys of a block each
-constexpr int kThreadsB = 352;      // + two issuing warps (one tcgen05.mma issue takes ~90 cycles) + a loader
+constexpr int kThreadsB = 352;      // + two MMA-issuing warps (one thread cannot feed N = 64 MMAs fast enough) + a loader
 constexpr float kLog2eB = 1.4426950408889634f;
 // Waiting threads sleep (woken when the phase completes) instead of spinning:
 // the issuing and row-information warps wait most of the time and would
