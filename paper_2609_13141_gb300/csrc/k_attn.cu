@@ -12,12 +12,13 @@
 // the tile's union list from the selection pass (blocks < 2t, ascending),
 // then the diagonal blocks 2t and 2t+1.  Per visited 64-key block:
 //   * warp 0 TMA-loads K (two-stage ring), warp 1 TMA-loads V (own ring);
-//   * warp 2 (one lane) issues S = Q K^T into the TMEM score buffer
-//     (tcgen05.mma M=128 N=64 K=16 steps); warp 3 (one lane) issues
-//     O += P V into the TMEM output accumulator (M=128 N=d, P read from TMEM,
-//     V as an MN-major operand).  The two streams use different accumulators
-//     and are issued independently: one thread cannot issue the small score
-//     MMAs as fast as the tensor pipe runs them;
+//   * warp 2 issues S = Q K^T into the TMEM score buffer (tcgen05.mma M=128
+//     N=64 K=16 steps); warp 3 issues O += P V into the TMEM output
+//     accumulator (M=128 N=d, P read from TMEM, V as an MN-major operand).
+//     Each walks its loop as a whole warp and issues from the elect.sync
+//     lane; the two streams use different accumulators and are issued
+//     independently: one thread cannot issue the small score MMAs as fast
+//     as the tensor pipe runs them;
 //   * warps 4-7, one thread per query row (TMEM lane), read the score row,
 //     add the row's gate or mask (each thread walks its own ascending list of
 //     kept blocks), run the online softmax in the log2 domain, write P as
@@ -27,6 +28,9 @@
 // so the next block's QK runs during this block's softmax; a P buffer is
 // reused once the PV two blocks back has read it.
 // The epilogue divides by the row sum and writes bf16 O and fp32 LSE.
+// GQA: K, V and the kept lists of query head bh are those of KV group bh / G.
+// Packed sequences: each tile's first row, tile index within its sequence and
+// sequence length come from the selection pass's tile table.
 #include <math_constants.h>
 
 #include "internal.h"

@@ -16,13 +16,18 @@
 //
 // One CTA owns one (batch*head, 128-row tile); one thread owns one row and
 // keeps its running max/sum and its Top-K candidates (registers for K <= 32,
-// a shared-memory column otherwise) with replace-the-worst updates.
+// a shared-memory column otherwise) with replace-the-worst updates.  Under
+// GQA the "head" is a KV group: its G query heads share the selection
+// (Sec. 5.3).  Packed sequences: a tile table (varlen_tiles_kernel) gives each
+// CTA its tile's first row, tile index within its sequence and sequence
+// length, so blocks and causality restart at every sequence.
 //
 // Two score sources:
 //   * scores given: 32x32 score sub-tiles are staged through shared memory
 //     with coalesced 128-byte row loads;
 //   * learned selector: on the tensor cores, one thread first projects the
-//     tile's 128 queries (q~ = Q Wq^T into TMEM); the row threads round q~
+//     tile's 128 queries (q~ = Q Wq^T into TMEM; under GQA q~ = Wq_g [q_0; ...;
+//     q_{G-1}], accumulated over G rounds of one head each); the row threads round q~
 //     to bf16 into shared memory as the A operand of the score product; then
 //     s = q~ Kt^T / sqrt(d_sel) runs chunk by chunk (M=128, N=64) over
 //     64-block chunks of projected summaries in a double-buffered TMA ring,
