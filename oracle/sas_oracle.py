@@ -339,16 +339,19 @@ def sas_attention_gqa(Q, K, V, b, topk, scores=None, mode=MODE_TRAIN_SOFT, sm_sc
     return out
 
 
-def sas_attention_varlen(Q, K, V, cu_seqlens, b, topk, scores, mode=MODE_TRAIN_SOFT, sm_scale=None,
-                         act=GATE_SOFTMAX, pos=GATE_INNER):
+def sas_attention_varlen(Q, K, V, cu_seqlens, b, topk, scores=None, mode=MODE_TRAIN_SOFT, sm_scale=None,
+                         act=GATE_SOFTMAX, pos=GATE_INNER, Wq=None, Wk=None):
     """Packed variable-length form: sequences s = 0 .. S-1 occupy rows
     cu_seqlens[s] .. cu_seqlens[s+1]-1 of the token axis; each is its own
     causal problem whose block partition starts at its first token (token t
     of sequence s is in its block floor(t / b); nothing crosses sequences).
     Q [Hq, total, d]; K, V [Hkv, total, d]; scores [Hkv, total, >=C-1], row
     cu[s] + t reading entries 0 .. floor(t / b) - 1; Hq = G Hkv (GQA, query
-    head h uses group h // G).  Returns dict of [Hq, total, ...] O, LSE and
-    [Hkv, total, topk] sel_idx / sel_logg (rows past cu[S] stay zero / -1).
+    head h uses group h // G).  Without scores, the learned selector with the
+    group gate query (selector_scores_group; Wq [Hkv, d_s, G d], Wk
+    [Hkv, d_s, d]) scores each sequence against the summaries of its own
+    blocks.  Returns dict of [Hq, total, ...] O, LSE and [Hkv, total, topk]
+    sel_idx / sel_logg (rows past cu[S] stay zero / -1).
     """
     Hq, total, d = Q.shape
     Hkv = K.shape[0]
@@ -365,9 +368,16 @@ def sas_attention_varlen(Q, K, V, cu_seqlens, b, topk, scores, mode=MODE_TRAIN_S
     for s0, s1 in zip(cu[:-1], cu[1:]):
         if s1 == s0:
             continue
+        tables = {}
         for h in range(Hq):
             g = h // G
-            r = sas_attention_head(Q[h, s0:s1], K[g, s0:s1], V[g, s0:s1], scores[g, s0:s1], b, topk, mode,
+            if scores is not None:
+                sg = scores[g, s0:s1]
+            else:
+                if g not in tables:
+                    tables[g] = selector_scores_group(Q[g * G:(g + 1) * G, s0:s1], K[g, s0:s1], Wq[g], Wk[g], b)
+                sg = tables[g]
+            r = sas_attention_head(Q[h, s0:s1], K[g, s0:s1], V[g, s0:s1], sg, b, topk, mode,
                                    sm_scale, None, act, pos)
             O[h, s0:s1] = r["O"]
             LSE[h, s0:s1] = r["LSE"]

@@ -85,3 +85,37 @@ def test_gqa_packing_and_empty_sequences_and_bad_offsets():
         O.sas_attention_varlen(Q, K, V, [0, 40, 30, 51], 8, 2, s)
     with pytest.raises(ValueError):
         O.sas_attention_varlen(Q, K, V, [1, 30, 51], 8, 2, s)
+
+
+def test_learned_selector_pack_equals_the_batched_learned_oracle():
+    # equal lengths, the learned selector (group gate query, G = 2): the pack equals
+    # the batched GQA oracle, whose block summaries are per batch element
+    S, Hkv, G, n, d, ds = 2, 1, 2, 70, 4, 4
+    rng = np.random.default_rng(31)
+    Q = rng.standard_normal((Hkv * G, S * n, d))
+    K, V = rng.standard_normal((Hkv, S * n, d)), rng.standard_normal((Hkv, S * n, d))
+    Wq, Wk = rng.standard_normal((Hkv, ds, G * d)), rng.standard_normal((Hkv, ds, d))
+    cu = np.array([0, n, 2 * n])
+    v = O.sas_attention_varlen(Q, K, V, cu, 8, 2, Wq=Wq, Wk=Wk)
+    bat = lambda x: x.reshape(x.shape[0], S, n, -1).transpose(1, 0, 2, 3)
+    m = O.sas_attention_gqa(bat(Q), bat(K), bat(V), 8, 2, Wq=Wq, Wk=Wk)
+    for bi in range(S):
+        for h in range(Hkv * G):
+            assert np.array_equal(v["O"][h, bi * n:(bi + 1) * n], m[(bi, h)]["O"])
+            assert np.array_equal(v["sel_idx"][h // G, bi * n:(bi + 1) * n], m[(bi, h)]["sel_idx"])
+
+
+def test_learned_selector_summaries_stay_within_the_sequence():
+    # changing the keys of the first sequence leaves the second one's selection alone
+    rng = np.random.default_rng(32)
+    Q = rng.standard_normal((1, 150, 4))
+    K, V = rng.standard_normal((1, 150, 4)), rng.standard_normal((1, 150, 4))
+    Wq, Wk = rng.standard_normal((1, 4, 4)), rng.standard_normal((1, 4, 4))
+    cu = [0, 61, 150]
+    a = O.sas_attention_varlen(Q, K, V, cu, 8, 2, Wq=Wq, Wk=Wk)
+    K2 = K.copy()
+    K2[:, :61] *= -2.0
+    b = O.sas_attention_varlen(Q, K2, V, cu, 8, 2, Wq=Wq, Wk=Wk)
+    assert np.array_equal(a["sel_idx"][:, 61:], b["sel_idx"][:, 61:])
+    assert np.array_equal(a["O"][:, 61:], b["O"][:, 61:])
+    assert not np.array_equal(a["O"][:, :61], b["O"][:, :61])
