@@ -139,3 +139,28 @@ def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scal
                 gates = np.exp(log_gates(np.asarray(s[g, i][:c], dtype=np.float64)))
                 ds[g, i, :c] = dl - gates * dl.sum()
     return {"dQ": dQ, "dK": dK, "dV": dV, "dlogg": dlogg, "ds": ds}
+
+
+def sas_attention_bwd_varlen(Q, K, V, s, dO, cu_seqlens, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
+    """Gradients of the packed variable-length forward: every sequence
+    (rows cu[k] .. cu[k+1]-1) is its own problem, so its gradients are those
+    of the GQA backward on its slice, and nothing crosses sequences.
+    Q, dO: [Hq, total, d]; K, V: [Hkv, total, d]; s: [Hkv, total, >=C-1]
+    (C from the longest sequence).  Returns the fields of
+    sas_attention_bwd_gqa on the whole token axis (ds has the columns of s
+    that a sequence's rows can read; rows past cu[S] stay zero)."""
+    Hq, total, d = Q.shape
+    Hkv = K.shape[0]
+    cu = [int(x) for x in cu_seqlens]
+    Cs = s.shape[2]
+    out = {"dQ": np.zeros((Hq, total, d)), "dK": np.zeros((Hkv, total, d)), "dV": np.zeros((Hkv, total, V.shape[2])),
+           "dlogg": np.zeros((Hkv, total, topk)), "ds": np.zeros((Hkv, total, Cs))}
+    for s0, s1 in zip(cu[:-1], cu[1:]):
+        if s1 == s0:
+            continue
+        r = sas_attention_bwd_gqa(Q[:, s0:s1], K[:, s0:s1], V[:, s0:s1], s[:, s0:s1], dO[:, s0:s1], b, topk,
+                                  mode, sm_scale)
+        for f in ("dQ", "dK", "dV", "dlogg"):
+            out[f][:, s0:s1] = r[f]
+        out["ds"][:, s0:s1, :r["ds"].shape[2]] = r["ds"]
+    return out

@@ -170,3 +170,32 @@ def test_gqa_backward_with_one_head_per_group_is_the_head_backward():
         m = BO.sas_attention_bwd_head(Q[h], K[h], V[h], s[h], dO[h], b, topk)
         for f in ("dQ", "dK", "dV", "dlogg", "ds"):
             assert np.allclose(r[f][h], m[f], atol=1e-13), f
+
+
+def test_packed_backward_equals_autograd_of_the_packed_forward_oracle():
+    # central finite differences of the packed forward oracle (through K of both
+    # sequences and the scores) against the packed backward: the sequences' block
+    # partitions start at their own first rows, and no gradient crosses them
+    b, d, topk = 4, 3, 1
+    rng = np.random.default_rng(23)
+    lens = [9, 11]
+    T = sum(lens)
+    cu = [0, 9, 20]
+    Q, K, V, dO = (rng.standard_normal((1, T, d)) for _ in range(4))
+    s = rng.standard_normal((1, T, 3))
+    r = BO.sas_attention_bwd_varlen(Q, K, V, s, dO, cu, b, topk)
+
+    def loss(Kx, sx):
+        return float((O.sas_attention_varlen(Q, Kx, V, cu, b, topk, sx)["O"] * dO).sum())
+
+    h = 1e-6
+    for name, X, ref in (("K", K, r["dK"]), ("s", s, r["ds"])):
+        G = np.zeros_like(X)
+        for idx in np.ndindex(X.shape):
+            Xp, Xm = X.copy(), X.copy()
+            Xp[idx] += h
+            Xm[idx] -= h
+            args_p = (Xp, s) if name == "K" else (K, Xp)
+            args_m = (Xm, s) if name == "K" else (K, Xm)
+            G[idx] = (loss(*args_p) - loss(*args_m)) / (2 * h)
+        assert np.allclose(G, ref, atol=1e-6), name
