@@ -63,6 +63,28 @@ def test_selector_worked_example():
     assert np.allclose(s[3], g["expect_s_row3"], rtol=0, atol=1e-15)
 
 
+def test_selector_hand_example_projected():
+    # Non-identity projections with d_s = 2 != d = 3 and Wq != Wk, values whose
+    # projections fall between bf16 neighbours (one exactly on a midpoint):
+    # the expected numbers are worked out by hand in the fixture.  A transposed
+    # weight, a dropped bf16 rounding of q~ or K~, or sqrt(d) for sqrt(d_s)
+    # each changes at least one of them.
+    g = json.load(open(GOLDEN))["selector_example_projected"]
+    K, Q = np.array(g["K"], float), np.array(g["Q"], float)
+    Wq, Wk = np.array(g["Wq"], float), np.array(g["Wk"], float)
+    assert np.array_equal(O.round_to_bf16(np.concatenate([K.ravel(), Q.ravel(), Wq.ravel(), Wk.ravel()])),
+                          np.concatenate([K.ravel(), Q.ravel(), Wq.ravel(), Wk.ravel()]))
+    assert np.array_equal(O.block_summaries(K, g["b"]), np.array(g["expect_Kbar"]))
+    assert np.array_equal(O.round_to_bf16(Q[5] @ Wq.T), np.array(g["expect_qt_row5"]))
+    assert np.array_equal(O.round_to_bf16(O.block_summaries(K, g["b"]) @ Wk.T), np.array(g["expect_Kt"]))
+    s = O.selector_scores(Q, K, Wq, Wk, g["b"])
+    assert s.shape == (6, 3)
+    assert np.allclose(s[5, :2] * math.sqrt(2.0), g["expect_s_row5_times_sqrt2"], rtol=0, atol=1e-14)
+    # the group form with G = 1 is the same selector
+    sg = O.selector_scores_group(Q[None], K, Wq, Wk, g["b"])
+    assert np.array_equal(sg, s)
+
+
 def test_selector_scores_scaling_and_permutation():
     # doubling Wq (exact in bf16) doubles every score; permuting key blocks
     # permutes the score columns.
