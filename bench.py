@@ -1,21 +1,24 @@
-"""Benchmark: one SAS transformer layer on GB300 through the C ABI.
+"""Benchmark: the SAS attention layer on GB300 through the C ABI.
 
 A step is one pass of the whole hot path over one batch of synthetic input:
 the SAS attention forward (block summaries, query projection, selector scores,
-log-gates, Top-K, gated block-sparse attention) followed by the dense GELU MLP
-on the same tokens.  Workload (the DiT-scale layer): B=2, H=24, N=4096+512,
-d=128, b=64, K=32, learned selector with d_sel=128, MLP 9216 x 3072 -> 12288
--> 3072.  Inputs are seeded synthetic data resident in HBM; L2 is flushed
-(256 MiB write) between timed steps, outside the timed events.
+log-gates, Top-K, gated block-sparse attention), followed by the dense GELU
+MLP on the same tokens where the workload has one.  Default workload
+(video-scale long-sequence attention): B=1, H=24, N=75600+512, d=128, b=64,
+K=32, learned selector with d_sel=128 on block-correlated queries (R2),
+attention only.  Inputs are seeded synthetic data resident in HBM; L2 is
+flushed (256 MiB write) between timed steps, outside the timed events.
 
 Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
 bounded sample of the same workload instead.
 
---workload decode times the SAS decode step instead (Alg. 2 with per-group
-block selection over a paged KV cache): a Qwen3-4B-shaped attention layer
+Other workloads (--workload): tiny, dit and hires (SAS layer + MLP),
+mlp_stress (the MLP sublayer alone), qwen3_4b_prefill / qwen3_4b_packed (GQA
+prefill, given scores), and decode: the SAS decode step (Alg. 2 with
+per-group block selection over a paged KV cache) of a Qwen3-4B-shaped layer
 (32 query heads, 8 KV heads, d=128, b=64, K=32 = a 2048-token budget) at
---context tokens for --batch sequences, captured in a CUDA graph, next to the
-dense decode of the same cache.
+--context tokens for --batch sequences, captured in a CUDA graph, next to
+the dense decode of the same cache.
 """
 from __future__ import annotations
 
@@ -37,6 +40,10 @@ METRIC = "ms/layer and effective TFLOP/s on 1xGB300; % of bf16 tensor-core roofl
 UNIT = "TFLOP/s"
 
 WORKLOADS = {
+    # D = F = 0: no MLP in the step; attn False: the MLP alone
+    "video": dict(B=1, H=24, N=75600 + 512, d=128, topk=32, d_sel=128, D=0, F=0,
+                  name="video-scale long-sequence SAS attention: B=1 H=24 N=75600+512 (21x45x80 patches + 512 text "
+                       "tokens; last block 16 tokens) d=128 b=64 K=32, learned selector d_sel=128, attention only"),
     "dit": dict(B=2, H=24, N=4096 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
                 name="DiT-scale causal SAS layer: B=2 H=24 N=4096+512 d=128 b=64 K=32, learned selector d_sel=128, "
                      "GELU MLP 9216x3072->12288->3072"),
@@ -44,8 +51,8 @@ WORKLOADS = {
                  name="tiny SAS layer: B=1 H=4 N=256 d=64 K=32, MLP 256->1024->256"),
     "hires": dict(B=1, H=24, N=16384 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
                   name="high-resolution causal SAS layer: B=1 H=24 N=16384+512 d=128 K=32, MLP 16896x3072->12288->3072"),
-    "video": dict(B=1, H=24, N=75600 + 512, d=128, topk=32, d_sel=128, D=3072, F=12288,
-                  name="video-scale causal SAS layer: B=1 H=24 N=75600+512 d=128 K=32, MLP 76112x3072->12288->3072"),
+    "mlp_stress": dict(B=1, H=0, N=16384, d=128, topk=0, d_sel=128, D=3072, F=12288, attn=False,
+                       name="MLP-sublayer stress: 16384 tokens x 3072 -> 12288 -> 3072 bf16, exact-erf GELU"),
     # GQA prefill (group-shared selection from given scores, one table per KV group)
     "qwen3_4b_prefill": dict(B=1, H=32, Hkv=8, N=32768, d=128, topk=32, d_sel=128, D=2560, F=9728,
                              name="Qwen3-4B-shaped GQA prefill layer: B=1 Hq=32 Hkv=8 N=32768 d=128 b=64 K=32 "
@@ -81,9 +88,29 @@ def algorithmic_flops(w, learned=True):
     sel += (N // 64) * 2 * d * ds
     if not learned:
         sel = 0
+    if not w.get("attn", True):
+        attn = sel = 0
     mlp = 4 * w["B"] * N * w["D"] * w["F"]
     return {"attention": BH * attn, "selector": BH * sel, "mlp": mlp,
             "total": BH * (attn + sel) + mlp}
+
+
+def executed_attention_flops(unions, N, d, G, lens=None):
+    """FLOPs the attention kernel executes: every 128-row tile runs QK^T and PV
+    (4 * 128 * 64 * d) for each block of its union list plus its one or two
+    diagonal blocks, for each of the G query heads that share the list.
+    unions: per (KV group, tile) union counts of the last forward."""
+    per_block = 4 * 128 * 64 * d
+    if lens is None:
+        T = (N + 127) // 128
+        ndiag = [2 if (2 * t + 1) * 64 < N else 1 for t in range(T)]
+        total = sum(u + ndiag[k % T] for k, u in enumerate(unions))
+    else:
+        diag = []
+        for n in lens:
+            diag += [2 if (2 * t + 1) * 64 < n else 1 for t in range((n + 127) // 128)]
+        total = sum(unions) + sum(diag) * (len(unions) // max(len(diag), 1))
+    return G * total * per_block
 
 
 def packed_flops(w, learned=False):
@@ -208,14 +235,18 @@ def run_ours(args, w, rank, world):
         dist.init_process_group("nccl", device_id=dev)
 
     B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
+    attn = w.get("attn", True)
+    mlp = D > 0 and F > 0
     Hkv = w.get("Hkv", H)
     lens = w.get("lens")                          # packed sequences (B = 1, token axis of N rows)
     T = B * N
-    learned = args.regime == "R2" and Hkv == H and not lens   # GQA / packing take given scores
-    if learned:
+    learned = attn and args.regime == "R2" and Hkv == H and not lens   # GQA / packing take given scores
+    Q = Kk = V = S = None
+    if not attn:
+        pass
+    elif learned:
         # R2: block-correlated queries through the learned selector
         Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="R2")
-        S = None
     elif Hkv == H:
         # R1: block-coherent selector scores supplied by the caller
         Q, Kk, V = synth.qkv(B, H, N, d, seed=rank, regime="iid")
@@ -224,17 +255,24 @@ def run_ours(args, w, rank, world):
         Q = synth.qkv(B, H, N, d, seed=rank, regime="iid")[0]
         _, Kk, V = synth.qkv(B, Hkv, N, d, seed=rank + 100, regime="iid")
         S = synth.scores(B, Hkv, N, (max(lens) + 63) // 64 if lens else (N + 63) // 64, seed=rank, regime="R1")
-    Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
-    X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
-    Qd, Kd, Vd, Wqd, Wkd = (t.to(dev) for t in (Q, Kk, V, Wq, Wk))
-    Sd = None if S is None else S.to(dev)
-    Xd, W1d, W2d = X.to(dev), W1.to(dev), W2.to(dev)
-    Od = torch.empty_like(Qd)
-    LSEd = torch.empty(B, H, N, device=dev, dtype=torch.float32)
-    Yd = torch.empty(T, D, device=dev, dtype=torch.bfloat16)
+    to = lambda t: None if t is None else t.to(dev)
+    Qd, Kd, Vd, Sd = to(Q), to(Kk), to(V), to(S)
+    Wqd = Wkd = None
+    if learned:
+        Wq, Wk = synth.selector_weights(H, d, ds, seed=rank)
+        Wqd, Wkd = Wq.to(dev), Wk.to(dev)
+    X = W1d = W2d = Xd = Yd = None
+    if mlp:
+        X, W1, W2, _, _ = synth.mlp(T, D, F, seed=rank)
+        Xd, W1d, W2d = X.to(dev), W1.to(dev), W2.to(dev)
+        Yd = torch.empty(T, D, device=dev, dtype=torch.bfloat16)
+    Od = torch.empty_like(Qd) if attn else None
+    LSEd = torch.empty(B, H, N, device=dev, dtype=torch.float32) if attn else None
     flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
 
-    if learned:
+    if not attn:
+        layer = sas.SasLayer(1, 1, 64, 64, 0)     # a handle for the MLP entry point
+    elif learned:
         layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=ds)
     elif lens:
         layer = sas.SasLayer(1, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv, max_seqs=len(lens),
@@ -249,15 +287,14 @@ def run_ours(args, w, rank, world):
         cud = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
 
     def step(Qx, Kx, Vx, Xx, O, Y, Sx=None):
-        if lens:
+        if attn and lens:
             sas.sas_attention_fwd_varlen(h, cud, Qx[0], Kx[0], Vx[0], Sx[0], O[0], LSEd[0], None, None, stream)
-            sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
-            return
-        if learned:
+        elif attn and learned:
             sas.sas_attention_fwd(h, Qx, Kx, Vx, O, None, Wqd, Wkd, LSEd, None, None, stream)
-        else:
+        elif attn:
             sas.sas_attention_fwd(h, Qx, Kx, Vx, O, Sx, None, None, LSEd, None, None, stream)
-        sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
+        if mlp:
+            sas.sas_mlp_fwd(h, Xx, W1d, W2d, Y, None, None, stream)
 
     for _ in range(max(args.warmup, 3)):
         step(Qd, Kd, Vd, Xd, Od, Yd, Sd)
@@ -294,13 +331,20 @@ def run_ours(args, w, rank, world):
     assert sas.sas_get_device_status(h) == 0, "device status word reports a timed-out wait"
 
     # end to end: pinned host inputs -> device -> layer -> host outputs, every step
-    hQ, hK, hV, hX = (t.pin_memory() for t in (Q, Kk, V, X))
-    hO = torch.empty(Q.shape, dtype=torch.bfloat16).pin_memory()
-    hY = torch.empty(T, D, dtype=torch.bfloat16).pin_memory()
-    dQ, dK, dV, dX = (torch.empty_like(t) for t in (Qd, Kd, Vd, Xd))
-    hS = None if S is None else S.pin_memory()
-    dS = None if S is None else torch.empty_like(Sd)
-    copies = [(dQ, hQ), (dK, hK), (dV, hV), (dX, hX)] + ([] if S is None else [(dS, hS)])
+    copies, outs = [], []
+    dQ = dK = dV = dX = dS = None
+    if attn:
+        hQ, hK, hV = (t.pin_memory() for t in (Q, Kk, V))
+        dQ, dK, dV = (torch.empty_like(t) for t in (Qd, Kd, Vd))
+        copies += [(dQ, hQ), (dK, hK), (dV, hV)]
+        outs.append((torch.empty(Q.shape, dtype=torch.bfloat16).pin_memory(), Od))
+        if S is not None:
+            dS = torch.empty_like(Sd)
+            copies.append((dS, S.pin_memory()))
+    if mlp:
+        dX = torch.empty_like(Xd)
+        copies.append((dX, X.pin_memory()))
+        outs.append((torch.empty(T, D, dtype=torch.bfloat16).pin_memory(), Yd))
     e_st = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     e_en = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     for k in range(-2, args.steps):
@@ -310,25 +354,27 @@ def run_ours(args, w, rank, world):
         for dst, src in copies:
             dst.copy_(src, non_blocking=True)
         step(dQ, dK, dV, dX, Od, Yd, dS)
-        hO.copy_(Od, non_blocking=True)
-        hY.copy_(Yd, non_blocking=True)
+        for host, devt in outs:
+            host.copy_(devt, non_blocking=True)
         if k >= 0:
             e_en[k].record(stream)
     torch.cuda.synchronize()
     e2e_ms = sum(s.elapsed_time(e) for s, e in zip(e_st, e_en)) / args.steps
     h2d = sum(src.numel() * src.element_size() for _, src in copies)
-    d2h = hO.numel() * 2 + hY.numel() * 2
+    d2h = sum(host.numel() * host.element_size() for host, _ in outs)
 
     # tile-union statistics of the last forward (executed vs algorithmic work)
-    Tt = (N + 127) // 128
-    if lens:
-        # packed: the first sum(ceil(n/128)) slots of each group are the tiles in use
-        slots = (N + 127) // 128 + len(lens)
-        used = sum((n + 127) // 128 for n in lens)
-        allc = sas.sas_get_tile_union_counts(h, Hkv * slots)
-        unions = [allc[g * slots + k] for g in range(Hkv) for k in range(used)]
-    else:
-        unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
+    unions = []
+    if attn:
+        Tt = (N + 127) // 128
+        if lens:
+            # packed: the first sum(ceil(n/128)) slots of each group are the tiles in use
+            slots = (N + 127) // 128 + len(lens)
+            used = sum((n + 127) // 128 for n in lens)
+            allc = sas.sas_get_tile_union_counts(h, Hkv * slots)
+            unions = [allc[g * slots + k] for g in range(Hkv) for k in range(used)]
+        else:
+            unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
     layer.close()
 
     ms, e2e_ms = reduce_max([ms, e2e_ms], dist, dev)
@@ -351,25 +397,22 @@ def run_ours(args, w, rank, world):
         roof = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1), "peak": peaks["bf16"],
                 "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16"], 4), "traffic": kernel_traffic(dom),
                 "peak_source": f"{peaks['source']} bf16 dense burst"}
-    # attention-kernel view (the SAS kernel proper)
-    a_avg = kt["attention"][1] / max(kt["attention"][0], 1)
-    hist_blocks = sum(unions) / max(len(unions), 1)
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
-        "data": ("synthetic (seeded; R2 block-correlated queries, N(0,1) K/V/X, weights N(0,0.02))" if learned else
+        "data": ("synthetic (seeded; N(0,1) X, weights N(0,0.02))" if not attn else
+                 "synthetic (seeded; R2 block-correlated queries q_i = (mu[block] + 0.3 eps_i)/sqrt(1.09), "
+                 "N(0,1) K/V" + ("/X" if mlp else "") + ", weights N(0,0.02))" if learned else
                  "synthetic (seeded; R1 block-coherent selector scores s = u[block] + 0.05 eps given by the caller, "
-                 "N(0,1) Q/K/V/X, weights N(0,0.02))"),
+                 "N(0,1) Q/K/V" + ("/X" if mlp else "") + ", weights N(0,0.02))"),
         "config": {"workload": w["name"], "B": B, "H": H, "Hkv": Hkv, "N": N, "d": d, "block": 64, "topk": K,
                    "d_sel": ds, "packed_lengths": lens,
-                   "mlp": [T, D, F, D], "selector": "meanpool_proj" if learned else "scores_given (R1)",
+                   "mlp": [T, D, F, D] if mlp else None,
+                   "selector": None if not attn else ("meanpool_proj (R2)" if learned else "scores_given (R1)"),
                    "l2": "flushed between timed steps (256 MiB write)",
                    "parallelism": f"replicas x{world}"},
         "roofline": roof,
-        "attention_kernel": {"ms": round(a_avg, 4), "algorithmic_tflops": round(fl["attention"] / (a_avg / 1e3) / 1e12, 1),
-                             "frac_of_bf16_peak": round(fl["attention"] / (a_avg / 1e3) / 1e12 / peaks["bf16"], 4),
-                             "mean_union_blocks_per_tile": round(hist_blocks, 2)},
         "kernels": per_kind,
         "algorithmic_tflop_per_step": round(tflop, 4),
         "e2e": {"value": round(job_throughput(tflop, world, e2e_ms), 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
@@ -377,8 +420,27 @@ def run_ours(args, w, rank, world):
         "gpu_launches": launches,
         "clocks": clocks,
     }
+    if attn:
+        # the SAS attention kernel proper: algorithmic work (each row's kept keys)
+        # and executed work (every 128-row tile over its union of kept blocks)
+        a_avg = kt["attention"][1] / max(kt["attention"][0], 1)
+        exe = executed_attention_flops(unions, N, d, H // Hkv, lens)
+        a_alg = fl["attention"] / (a_avg / 1e3) / 1e12
+        a_exe = exe / (a_avg / 1e3) / 1e12
+        sas_ms = sum(kt[k][1] / max(kt[k][0], 1) for k in ("block_summaries", "selection", "attention"))
+        out["attention_kernel"] = {
+            "ms": round(a_avg, 4), "algorithmic_tflops": round(a_alg, 1),
+            "frac_of_bf16_peak": round(a_alg / peaks["bf16"], 4),
+            "executed_tflop": round(exe / 1e12, 4), "executed_tflops": round(a_exe, 1),
+            "executed_frac_of_bf16_peak": round(a_exe / peaks["bf16"], 4),
+            "mean_union_blocks_per_tile": round(sum(unions) / max(len(unions), 1), 2)}
+        out["sas_layer"] = {"ms": round(sas_ms, 4),
+                            "algorithmic_tflops": round((fl["attention"] + fl["selector"]) / (sas_ms / 1e3) / 1e12, 1),
+                            "selection_ms": round(kt["selection"][1] / max(kt["selection"][0], 1), 4),
+                            "block_summaries_ms": round(kt["block_summaries"][1] / max(kt["block_summaries"][0], 1), 4)}
     if not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget, learned=learned)
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget, learned=learned, workload=args.workload,
+                                           topk=args.topk)
     if dist is not None:
         dist.destroy_process_group()
     return out
@@ -386,24 +448,38 @@ def run_ours(args, w, rank, world):
 
 # ----------------------------------------------------------- CPU oracle
 
+def _nproc():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
 def _oracle_threads():
+    """Threads the oracle's matrix products may use (its BLAS pool; the
+    per-row loops are single-threaded Python)."""
     try:
         from threadpoolctl import threadpool_info
         n = [i.get("num_threads", 1) for i in threadpool_info()]
         return max(n) if n else 1
     except Exception:
-        return os.cpu_count() or 1
+        for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+            if os.environ.get(var, "").isdigit():
+                return int(os.environ[var])
+        return _nproc()
 
 
 def oracle_sample(w, budget_s, seed=0, learned=True):
     """Runs the oracle on a bounded sample of the workload and returns its
     throughput on the workload's FLOP mix.
 
-    Half the budget goes to query rows of one head (selector scores for the
+    The attention part runs query rows of one head (selector scores for the
     whole head, or the head's given R1 scores, then the gated attention of
-    random rows), half to random MLP token rows.  Each part's rate (algorithmic FLOPs per second) is measured
-    on its own; the full layer's time is attention FLOPs / attention rate +
-    MLP FLOPs / MLP rate.  Returns (rate_flops_per_s, seconds, desc)."""
+    random rows); the MLP part runs random token rows.  With both, each gets
+    half the budget and its rate (algorithmic FLOPs per second) is measured on
+    its own; the full step's time is extrapolated as attention FLOPs /
+    attention rate + MLP FLOPs / MLP rate.  Returns (rate_flops_per_s,
+    seconds, desc)."""
     import numpy as np
     import torch
 
@@ -411,57 +487,90 @@ def oracle_sample(w, budget_s, seed=0, learned=True):
     from paper_2609_13141_gb300 import synth
 
     B, H, N, d, K, ds, D, F = (w[k] for k in ("B", "H", "N", "d", "topk", "d_sel", "D", "F"))
-    Q, Kk, V = synth.qkv(1, 1, N, d, seed=seed, regime="R2")
-    Wq, Wk = synth.selector_weights(1, d, ds, seed=seed)
-    X, W1, W2, _, _ = synth.mlp(256, D, F, seed=seed)
+    attn, mlp = w.get("attn", True), D > 0 and F > 0
+    share = budget_s / 2 if (attn and mlp) else budget_s
     f = lambda t: t.to(torch.float64).numpy()
-    q, k, v, wq, wk = f(Q[0, 0]), f(Kk[0, 0]), f(V[0, 0]), f(Wq[0]), f(Wk[0])
-    x, w1, w2 = f(X), f(W1), f(W2)
     rng = np.random.default_rng(seed)
-
-    if learned:
-        t0 = time.perf_counter()
-        s = OR.selector_scores(q, k, wq, wk, 64)
-        a_flops = N * 2 * d * ds + (N // 64) * 2 * d * ds
-    else:
-        s = f(synth.scores(1, 1, N, (N + 63) // 64, seed=seed, regime="R1")[0, 0])
-        t0 = time.perf_counter()
-        a_flops = 0
-    rows_done = 0
-    while time.perf_counter() - t0 < budget_s / 2:
-        rows = rng.integers(0, N, size=32)
-        OR.sas_attention_head(q, k, v, s, 64, K, rows=rows)
-        a_flops += sum(OR.attention_flops_row(int(i), 64, K, d, ds if learned else 0) for i in rows)
-        rows_done += len(rows)
-    a_time = time.perf_counter() - t0
-    # the whole head's selector is amortised over the rows actually run
-    a_rate = a_flops / a_time
-
-    t1 = time.perf_counter()
-    m_flops = 0
-    tok_done = 0
-    while time.perf_counter() - t1 < budget_s / 2:
-        toks = rng.integers(0, 256, size=2)
-        OR.gelu_mlp(x, w1, w2, rows=toks)
-        m_flops += 4 * len(toks) * D * F
-        tok_done += len(toks)
-    m_time = time.perf_counter() - t1
-    m_rate = m_flops / m_time
+    parts = []
+    a_time = m_time = 0.0
+    a_rate = m_rate = None
+    if attn:
+        Q, Kk, V = synth.qkv(1, 1, N, d, seed=seed, regime="R2")
+        Wq, Wk = synth.selector_weights(1, d, ds, seed=seed)
+        q, k, v, wq, wk = f(Q[0, 0]), f(Kk[0, 0]), f(V[0, 0]), f(Wq[0]), f(Wk[0])
+        if learned:
+            t0 = time.perf_counter()
+            s = OR.selector_scores(q, k, wq, wk, 64)
+            a_flops = N * 2 * d * ds + (N // 64) * 2 * d * ds
+        else:
+            s = f(synth.scores(1, 1, N, (N + 63) // 64, seed=seed, regime="R1")[0, 0])
+            t0 = time.perf_counter()
+            a_flops = 0
+        rows_done = 0
+        while time.perf_counter() - t0 < share:
+            rows = rng.integers(0, N, size=32)
+            OR.sas_attention_head(q, k, v, s, 64, K, rows=rows)
+            a_flops += sum(OR.attention_flops_row(int(i), 64, K, d, ds if learned else 0) for i in rows)
+            rows_done += len(rows)
+        a_time = time.perf_counter() - t0
+        # the whole head's selector is amortised over the rows actually run
+        a_rate = a_flops / a_time
+        how = "with that head's selector" if learned else "with that head's given R1 scores"
+        parts.append(f"{rows_done} random query rows of one head ({how}) in {a_time:.1f} s")
+    if mlp:
+        X, W1, W2, _, _ = synth.mlp(256, D, F, seed=seed)
+        x, w1, w2 = f(X), f(W1), f(W2)
+        t1 = time.perf_counter()
+        m_flops = 0
+        tok_done = 0
+        while time.perf_counter() - t1 < share:
+            toks = rng.integers(0, 256, size=2)
+            OR.gelu_mlp(x, w1, w2, rows=toks)
+            m_flops += 4 * len(toks) * D * F
+            tok_done += len(toks)
+        m_time = time.perf_counter() - t1
+        m_rate = m_flops / m_time
+        parts.append(f"{tok_done} MLP token rows in {m_time:.1f} s")
 
     fl = packed_flops(w) if w.get("lens") else algorithmic_flops(w, learned)
-    full_time = (fl["attention"] + fl["selector"]) / a_rate + fl["mlp"] / m_rate
+    full_time = ((fl["attention"] + fl["selector"]) / a_rate if attn else 0.0) + (fl["mlp"] / m_rate if mlp else 0.0)
     rate = fl["total"] / full_time
-    how = "with that head's selector" if learned else "with that head's given R1 scores"
-    desc = (f"oracle (numpy fp64): {rows_done} random query rows of one head ({how}) "
-            f"in {a_time:.1f} s and {tok_done} MLP token rows in {m_time:.1f} s; the two measured rates are "
-            f"combined by the layer's FLOP mix")
+    desc = "oracle (numpy fp64): " + " and ".join(parts)
+    if attn and mlp:
+        desc += "; the two measured rates are combined by the layer's FLOP mix"
+    desc += "; the full step's time is extrapolated from the sampled rate"
     return rate, a_time + m_time, desc
 
 
-def cpu_baseline(w, budget_s=12.0, learned=True):
-    rate, dt, desc = oracle_sample(w, budget_s, learned=learned)
-    return {"value": round(rate / 1e12, 8), "unit": UNIT, "cores": _oracle_threads(), "kind": "oracle",
-            "sample": desc, "seconds": round(dt, 2)}
+def _oracle_sample_one_thread(workload, budget_s, learned, topk):
+    """oracle_sample in a fresh process whose BLAS pools are pinned to one
+    thread (the variables are read when numpy loads, so it needs its own
+    process).  Returns the rate in FLOP/s, or None if the run fails."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    cmd = [sys.executable, os.path.abspath(__file__), "--oracle-sample-only", "--workload", workload,
+           "--cpu-budget", str(budget_s), "--regime", "R2" if learned else "R1"]
+    if topk is not None:
+        cmd += ["--topk", str(topk)]
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=budget_s * 4 + 120)
+        return json.loads(r.stdout.strip().splitlines()[-1])["rate"]
+    except Exception:
+        return None
+
+
+def cpu_baseline(w, budget_s=12.0, learned=True, workload=None, topk=None):
+    """The oracle timed on this host: once with its BLAS pool on every core
+    (`value`), once pinned to one thread (`value_1_thread`), half the budget
+    each."""
+    rate, dt, desc = oracle_sample(w, budget_s / 2, learned=learned)
+    one = _oracle_sample_one_thread(workload, budget_s / 2, learned, topk) if workload else None
+    return {"value": round(rate / 1e12, 8), "unit": UNIT, "cores": _nproc(),
+            "threads": _oracle_threads(), "kind": "oracle",
+            "value_1_thread": None if one is None else round(one / 1e12, 8),
+            "sample": desc + f"; matrix products on a BLAS pool of {_oracle_threads()} threads, per-row loops "
+                             "single-threaded; value_1_thread: the same sample with the pool pinned to one thread",
+            "seconds": round(dt, 2)}
 
 
 def run_reference(args, w, rank, world):
@@ -480,11 +589,14 @@ def run_reference(args, w, rank, world):
     ms = full / (value * 1e12) * 1e3
     return {
         "impl": "reference", "metric": METRIC, "value": round(value, 8), "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2), "higher_is_better": True,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 2),
+        "ms_per_step_extrapolated": True, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
         "config": {"workload": w["name"], "B": w["B"], "H": w["H"], "N": w["N"], "d": w["d"], "topk": w["topk"]},
-        "cpu_baseline": {"value": round(value, 8), "unit": UNIT, "cores": _oracle_threads(), "kind": "oracle",
-                         "sample": desc + f"; each step a {args.ref_step_s:.0f}-second sample"},
+        "cpu_baseline": {"value": round(value, 8), "unit": UNIT, "cores": _nproc(), "threads": _oracle_threads(),
+                         "kind": "oracle",
+                         "sample": desc + f"; each step a {args.ref_step_s:.0f}-second sample; ms_per_step is the "
+                                          "whole step's FLOPs at the sampled rate (extrapolated, not run in full)"},
         "e2e": {"value": round(value, 8), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
@@ -788,7 +900,7 @@ def run_decode(args, rank, world):
     }
     if not args.no_cpu_baseline:
         v, secs, desc = decode_oracle_us(B, Hq, Hkv, d, ds, K, n, args.cpu_budget / 2)
-        out["cpu_baseline"] = {"value": round(v, 1), "unit": "us", "cores": _oracle_threads(), "kind": "oracle",
+        out["cpu_baseline"] = {"value": round(v, 1), "unit": "us", "cores": _nproc(), "threads": _oracle_threads(), "kind": "oracle",
                                "sample": desc, "seconds": round(secs, 2)}
     if dist is not None:
         dist.destroy_process_group()
@@ -812,7 +924,7 @@ def run_decode_reference(args, rank, world):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
         "config": {"workload": f"Qwen3-4B-shaped decode attention layer, context {args.context}, batch {args.batch}",
                    "B": args.batch, "context": args.context, "topk": K},
-        "cpu_baseline": {"value": round(value, 1), "unit": "us", "cores": _oracle_threads(), "kind": "oracle",
+        "cpu_baseline": {"value": round(value, 1), "unit": "us", "cores": _nproc(), "threads": _oracle_threads(), "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": round(value, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -824,7 +936,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["decode"], default="dit")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["decode"], default="video")
     ap.add_argument("--context", type=int, default=65536, help="decode: cached tokens per sequence")
     ap.add_argument("--batch", type=int, default=1, help="decode: sequences per step")
     ap.add_argument("--decode-only", choices=["sparse", "dense"], default=None,
@@ -837,6 +949,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=4.0)
+    ap.add_argument("--oracle-sample-only", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -849,6 +962,11 @@ def main():
     if args.topk is not None:
         w["topk"] = args.topk
         w["name"] = w["name"].replace("K=32", f"K={args.topk}")
+    if args.oracle_sample_only:
+        rate, dt, _ = oracle_sample(w, args.cpu_budget, learned=args.regime == "R2" and w.get("Hkv", w["H"]) == w["H"]
+                                    and not w.get("lens"))
+        print(json.dumps({"rate": rate, "seconds": dt}))
+        return
     if args.train:
         out = run_train(args, w, rank, world) if args.impl == "ours" else None
         if out is not None and rank == 0:

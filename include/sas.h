@@ -181,9 +181,9 @@ sas_status sas_attention_fwd(sas_handle* h,
  * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
  * allocates the handle's backward workspace (synchronously); later calls are
  * asynchronous and can be captured in a CUDA graph when B * H * T * (T + 1)
- * * 512 bytes <= 8 GiB (T = ceil(N / 128)).  Above that size every call reads
- * back how many blocks the forward's tiles visit, to size a buffer, and so
- * synchronises with its stream once. */
+ * * 512 bytes <= 8 GiB (T = ceil(N / 128)) and that much memory is free at the
+ * first call.  Otherwise every call reads back how many blocks the forward's
+ * tiles visit, to size a buffer, and so synchronises with its stream once. */
 sas_status sas_attention_bwd(sas_handle* h,
                              const void* Q, const void* K, const void* V,
                              const float* scores,
@@ -193,14 +193,6 @@ sas_status sas_attention_bwd(sas_handle* h,
                              float* dlogg, float* dscores,
                              void* stream);
 
-/* Dense MLP sublayer Y = GELU(X W1^T + b1) W2^T + b2 with the exact (erf)
- * GELU.  SAS itself does not define or change the MLP; this is the plain
- * transformer MLP that completes a layer.
- *   X  bf16 [T, D]; W1 bf16 [F, D]; b1 bf16 [F] or NULL;
- *   W2 bf16 [D, F]; b2 bf16 [D] or NULL; Y bf16 [T, D].
- * D and F must be multiples of 64; T >= 1.  The hidden activation
- * GELU(X W1^T + b1) is kept as a bf16 [T, F] tensor in handle-owned
- * memory, allocated (synchronously) the first time a call needs more. */
 /* Packed variable-length form of sas_attention_fwd, on a handle created
  * with max_seqs > 0.  Sequence s holds rows cu_seqlens[s] .. cu_seqlens[s+1]-1
  * of the token axis and is its own causal problem: its blocks of 64 tokens
@@ -223,6 +215,14 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
                                     const void* Q, const void* K, const void* V, const float* scores,
                                     void* O, float* LSE, int32_t* sel_idx, float* sel_logg, void* stream);
 
+/* Dense MLP sublayer Y = GELU(X W1^T + b1) W2^T + b2 with the exact (erf)
+ * GELU.  SAS itself does not define or change the MLP; this is the plain
+ * transformer MLP that completes a layer.
+ *   X  bf16 [T, D]; W1 bf16 [F, D]; b1 bf16 [F] or NULL;
+ *   W2 bf16 [D, F]; b2 bf16 [D] or NULL; Y bf16 [T, D].
+ * D and F must be multiples of 64; T >= 1.  The hidden activation
+ * GELU(X W1^T + b1) is kept as a bf16 [T, F] tensor in handle-owned
+ * memory, allocated (synchronously) the first time a call needs more. */
 sas_status sas_mlp_fwd(sas_handle* h,
                        const void* X, const void* W1, const void* b1,
                        const void* W2, const void* b2, void* Y,
@@ -252,12 +252,25 @@ sas_status sas_mlp_fwd(sas_handle* h,
  * array, and it keeps whatever the last call left in it: two calls whose
  * work overlaps on the GPU (different streams without ordering between
  * them) race on it and may corrupt each other's results.  Calls ordered on
- * one stream are safe. */
+ * one stream are safe.
+ *
+ * The return value covers what the host can check before launching.  What
+ * the kernels find while they run (a bounded wait that ran out, misaligned
+ * shared memory: Y is then incomplete) is latched in a per-device status
+ * word, read with sas_mlp_noalloc_get_device_status. */
 #define SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES (32u * 1024u * 1024u)
 sas_status sas_mlp_fwd_noalloc(const void* X, const void* W1, const void* b1,
                                const void* W2, const void* b2, void* Y,
                                int64_t T, int64_t D, int64_t F,
                                void* stream);
+
+/* Status word of sas_mlp_fwd_noalloc on the current device (there is no
+ * handle to hold one).  Synchronises the device, then writes to *out_status
+ * what the kernels of every earlier call recorded -- SAS_OK, SAS_ERR_TIMEOUT
+ * (a bounded wait ran out) or SAS_ERR_CUDA (a kernel found its shared memory
+ * not 1024-byte aligned) -- and clears it.  Allocates nothing.  Returns
+ * SAS_ERR_CUDA if the synchronisation or the read fails. */
+sas_status sas_mlp_noalloc_get_device_status(int32_t* out_status);
 
 /* Static text for a status code. */
 const char* sas_status_str(sas_status s);

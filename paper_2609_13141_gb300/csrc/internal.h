@@ -18,6 +18,15 @@ using bf16 = __nv_bfloat16;
 int make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t outer,
                       uint32_t box_inner, uint32_t box_rows);
 
+// Raises `func`'s dynamic shared-memory limit to at least `bytes` on the
+// current device.  The attribute belongs to the device, so it is recorded per
+// (kernel, device): the first launch on each device sets it, later ones find
+// the record and call nothing (so a launch inside a stream capture that was
+// preceded by one outside it sets nothing).  Thread-safe.
+cudaError_t ensure_smem_attr(const void* func, size_t bytes);
+// Multiprocessor count of the current device (cached per device, thread-safe).
+int device_sm_count();
+
 struct KernelEnv {
     cudaStream_t stream;
     int* status;        // device status word

@@ -641,11 +641,9 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
 template <int D, bool OUTER>
 cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) {
     using Cfg = AttnCfg<D>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, OUTER>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    {
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(attn_kernel<D, OUTER>), Cfg::SMEM);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
-        attr_set = true;
     }
     int dev = 0, sms = 0, l2 = 0;
     cudaError_t e = cudaGetDevice(&dev);

@@ -861,13 +861,10 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         *err = "backward: head dim must be 128";
         return cudaErrorInvalidValue;
     }
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(bwd_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bwd_dkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDkvSmem);
+    {
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel), kDqSmem);
+        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel), kDkvSmem);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(bwd)"; return e; }
-        attr = true;
     }
     CUtensorMap mq, mdo, mk, mv, mk2, mv2;
     if (make_tmap_bf16_3d(&mq, a.Q, kD, a.N, a.BH, 64, kRows) != 0 ||

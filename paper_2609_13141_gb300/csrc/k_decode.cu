@@ -1226,14 +1226,7 @@ cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, si
 template <int D, int G>
 cudaError_t prepare_attn_dg(const DecodeArgs& a) {
     const size_t smem = attn_layout(D, G, a.nst, a.bpc).total;
-    static size_t set = 0;
-    if (smem > set) {
-        cudaError_t e = cudaFuncSetAttribute(dec_attn_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        set = smem;
-    }
-    return cudaSuccess;
+    return ensure_smem_attr(reinterpret_cast<const void*>(dec_attn_kernel<D, G>), smem);
 }
 
 template <int D, int G>
@@ -1249,14 +1242,7 @@ cudaError_t launch_attn_dg(const DecodeArgs& a, const KernelEnv& env) {
 template <int G>
 cudaError_t prepare_attn_tc(const DecodeArgs& a) {
     const size_t smem = tc_layout(a.nst, a.bpc).total;
-    static size_t set = 0;
-    if (smem > set) {
-        cudaError_t e = cudaFuncSetAttribute(dec_attn_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        set = smem;
-    }
-    return cudaSuccess;
+    return ensure_smem_attr(reinterpret_cast<const void*>(dec_attn_tc_kernel<G>), smem);
 }
 
 template <int G>
@@ -1315,14 +1301,7 @@ cudaError_t prepare_attn_d(const DecodeArgs& a) {
 template <int DSEL>
 cudaError_t prepare_score_d(const DecodeArgs& a) {
     const size_t smem = score_smem_layout(a.nsplit_s, a.topk, DSEL).total;
-    static size_t set = 0;
-    if (smem > set) {
-        cudaError_t e = cudaFuncSetAttribute(dec_score_kernel<DSEL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        set = smem;
-    }
-    return cudaSuccess;
+    return ensure_smem_attr(reinterpret_cast<const void*>(dec_score_kernel<DSEL>), smem);
 }
 
 template <int DSEL>

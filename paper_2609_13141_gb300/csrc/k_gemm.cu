@@ -246,25 +246,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
 }
 
-int sm_count() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (n <= 0) n = 1;
-    }
-    return n;
-}
-
 template <int BN>
 cudaError_t launch_bn(const GemmProblem& p, const KernelEnv& env, const char** err) {
     using Cfg = GemmCfg<BN>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    {
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(gemm_kernel<BN>), Cfg::SMEM);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(gemm)"; return e; }
-        attr_set = true;
     }
     if (p.ldc != p.N || (p.batches > 1 && p.c_batch_stride != static_cast<long long>(p.M) * p.N)) {
         *err = "gemm: C must be a dense [batches][M][N] tensor";
@@ -283,7 +270,7 @@ cudaError_t launch_bn(const GemmProblem& p, const KernelEnv& env, const char** e
     gp.c_batch_stride = p.c_batch_stride; gp.ldc = p.ldc; gp.gelu = p.gelu;
     gp.status = env.status; gp.limit = env.limit;
     const long long tiles = static_cast<long long>(p.batches) * ((p.M + kBM - 1) / kBM) * (p.N / BN);
-    int grid = p.max_ctas > 0 ? p.max_ctas : sm_count();
+    int grid = p.max_ctas > 0 ? p.max_ctas : device_sm_count();
     if (tiles < grid) grid = static_cast<int>(tiles);
     gemm_kernel<BN><<<grid, kThreads, Cfg::SMEM, env.stream>>>(ma, mb, mc, gp);
     cudaError_t e = cudaGetLastError();

@@ -764,8 +764,7 @@ template <int D, int DS, bool REG>
 cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
     const size_t smem = 1024 + proj_region0<D, DS>(a.topk) + smem_topk_bytes(a.topk) + kValuesBytes + bitmap_bytes(a.C);
     if (smem > 227 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = cudaFuncSetAttribute(select_proj_kernel<D, DS, REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS, REG>), smem);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mw, mk;
     // Q of all query heads; Wq [H][DS][G D] (a group's gate-query projection)
@@ -783,8 +782,7 @@ template <bool REG>
 cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
     const size_t smem = smem_topk_bytes(a.topk) + staging_bytes(a.topk) + bitmap_bytes(a.C);
     if (smem > 200 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = cudaFuncSetAttribute(select_given_kernel<REG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_given_kernel<REG>), smem);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select_given)"; return e; }
     const dim3 grid(a.BH * a.T);
     select_given_kernel<REG><<<grid, 128, smem, env.stream>>>(p);
@@ -862,8 +860,7 @@ cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len,
     const size_t smem = static_cast<size_t>(4) * (tmax + 2) * sizeof(int);
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(varlen_tiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(varlen_tiles_kernel), smem);
         if (e != cudaSuccess) return e;
     }
     varlen_tiles_kernel<<<1, 1024, smem, env.stream>>>(cu, S, Ncap, max_len, tmax, tiles, ntiles, env.status);

@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -44,6 +45,38 @@ int make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64
                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return static_cast<int>(r);
+}
+
+// --------------------------------------------- per-device launch attributes
+
+namespace {
+std::mutex g_attr_mutex;
+std::map<std::pair<const void*, int>, size_t> g_smem_attr;   // (kernel, device) -> limit set
+std::map<int, int> g_sms;                                     // device -> SM count
+}  // namespace
+
+cudaError_t ensure_smem_attr(const void* func, size_t bytes) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_attr_mutex);
+    size_t& set = g_smem_attr[{func, dev}];
+    if (bytes <= set) return cudaSuccess;
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+    if (e == cudaSuccess) set = bytes;
+    return e;
+}
+
+int device_sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    std::lock_guard<std::mutex> lock(g_attr_mutex);
+    int& n = g_sms[dev];
+    if (n <= 0) {
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (n <= 0) n = 1;
+    }
+    return n;
 }
 
 // ------------------------------------------------------- failure self test
@@ -507,10 +540,17 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         // needs at most T (T + 1) slots of 128 rows; held whole when that fits in 8 GiB
         const size_t bound = tiles * static_cast<size_t>(h->T + 1) * 128 * 4;
         if (e == cudaSuccess && bound <= (static_cast<size_t>(8) << 30)) {
-            e = alloc(&h->bwd_offs, bound);
-            if (e == cudaSuccess) {
+            cudaError_t eb = alloc(&h->bwd_offs, bound);
+            if (eb == cudaSuccess) {
                 h->bwd_offs_bytes = bound;
                 h->bwd_offs_bound = true;
+            } else if (eb == cudaErrorMemoryAllocation) {
+                // no room for the bound: clear the error and size the buffer from the
+                // slot count each call reads back (the path used above 8 GiB)
+                cudaGetLastError();
+                h->bwd_offs = nullptr;
+            } else {
+                e = eb;
             }
         }
         if (e != cudaSuccess) {

@@ -21,7 +21,9 @@ static_assert(kScratchBytes == SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES, "header and arr
 
 // Hidden activation of the handle-free MLP, bf16 [T][F] with T*F*2 <= 32 MiB.
 static __device__ __align__(256) unsigned char g_mlp_hidden[kScratchBytes];
-// Status word for the GEMM kernels' bounded waits (written only when a wait runs out).
+// Status word of the GEMM kernels (written only when a bounded wait runs out,
+// or when a CTA finds its shared memory misaligned); read and cleared by
+// sas_mlp_noalloc_get_device_status.
 static __device__ __align__(256) int g_mlp_wait_status[64];
 
 constexpr int kMaxDevices = 128;
@@ -96,5 +98,20 @@ extern "C" sas_status sas_mlp_fwd_noalloc(const void* X, const void* W1, const v
     g2.batches = 1; g2.b_mod = 1; g2.c_batch_stride = 0; g2.ldc = static_cast<int>(D);
     g2.gelu = 0; g2.bn = pick_bn(D); g2.max_ctas = 0;
     if (sas::launch_gemm(g2, env, &err) != cudaSuccess) return SAS_ERR_CUDA;
+    return SAS_OK;
+}
+
+extern "C" sas_status sas_mlp_noalloc_get_device_status(int32_t* out_status) {
+    if (out_status == nullptr) return SAS_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return SAS_ERR_CUDA;
+    // every call's kernels have finished once the device is idle
+    if (cudaDeviceSynchronize() != cudaSuccess) return SAS_ERR_CUDA;
+    int v = 0;
+    // reads and clears the current device's copy of the word; neither copy allocates
+    if (cudaMemcpyFromSymbol(&v, g_mlp_wait_status, sizeof(int)) != cudaSuccess) return SAS_ERR_CUDA;
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_mlp_wait_status, &zero, sizeof(int)) != cudaSuccess) return SAS_ERR_CUDA;
+    *out_status = v;
     return SAS_OK;
 }

@@ -104,6 +104,8 @@ def lib():
     L.sas_get_tile_union_counts.restype = i32
     L.sas_mlp_fwd_noalloc.argtypes = [vp] * 6 + [i64, i64, i64, vp]
     L.sas_mlp_fwd_noalloc.restype = i32
+    L.sas_mlp_noalloc_get_device_status.argtypes = [ctypes.POINTER(i32)]
+    L.sas_mlp_noalloc_get_device_status.restype = i32
     L.sas_selftest_wait_timeout.argtypes = [i64, ctypes.POINTER(i32)]
     L.sas_selftest_wait_timeout.restype = i32
     L.sas_decode_create.argtypes = [ctypes.POINTER(SasDecodeConfig), ctypes.POINTER(vp)]
@@ -255,6 +257,14 @@ def sas_mlp_fwd_noalloc(X, W1, W2, Y, b1=None, b2=None, stream=None):
         raise SasError(st, f"sas_mlp_fwd_noalloc: hidden activation of {T}x{F} bf16 ({T * F * 2} bytes) exceeds "
                            f"the fixed {SAS_MLP_NOALLOC_MAX_HIDDEN_BYTES}-byte array")
     _check(st, None, "sas_mlp_fwd_noalloc")
+
+
+def sas_mlp_noalloc_get_device_status():
+    """Reads and clears the status word of sas_mlp_fwd_noalloc on the current
+    device (synchronises the device)."""
+    v = ctypes.c_int32(-1)
+    _check(lib().sas_mlp_noalloc_get_device_status(ctypes.byref(v)), None, "sas_mlp_noalloc_get_device_status")
+    return v.value
 
 
 def sas_get_device_status(h):

@@ -24,3 +24,16 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Worst max / mean abs error of every bf16 output each parity test compared."""
+    try:
+        from tests import parity
+    except Exception:  # pragma: no cover
+        return
+    if not parity.WORST:
+        return
+    terminalreporter.section("worst parity errors (bf16 outputs vs the fp64 oracle)")
+    for (test, what), (mx, mean) in sorted(parity.WORST.items()):
+        terminalreporter.write_line(f"{test}  {what}: max {mx:.3e}  mean {mean:.3e}")

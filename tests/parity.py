@@ -7,13 +7,20 @@ Tolerances (written here once, used by every parity test):
     margin exceeds the bound on how far the GPU's fp32 score may sit from
     the oracle's (selector_score_bound), and a valid Top-K set on the rest.
   * O (bf16): max |err| <= 2e-2 and mean |err| <= 2e-3 against the fp64
-    oracle.
+    oracle, absolute, wherever O is a convex combination of value rows (every
+    gate g <= 1: softmax and sigmoid activations, the inner position, the
+    inference form, GQA, packed sequences, decode).  Two outputs are sums
+    whose terms are not bounded by |v|, and get a derived extra term on top
+    (outer_logit_extra, grad_extra): the outer position with the raw-logit
+    activation (g = e^s > 1 scales probabilities after the softmax) and the
+    backward's dQ, dK, dV (sums over many rows or keys).
   * LSE (fp32): max |err| <= 1e-2.
   * sel_logg (fp32, log g = s - LSE over up to ~1200 blocks): max |err| <= 1e-4.
 """
 from __future__ import annotations
 
 import math
+import os
 
 import numpy as np
 import torch
@@ -62,15 +69,87 @@ def oracle_scores(Q, K, Wq, Wk, bi, hi):
     return OR.selector_scores(f64(Q[bi, hi]), f64(K[bi, hi]), f64(Wq[hi]), f64(Wk[hi]), 64)
 
 
-def compare_o(gpu_O, ref_O, what="O", scale=1.0):
-    """Max and mean abs error of O against the oracle; scale > 1 widens both
-    bounds in proportion, for outputs whose magnitude grows past that of V
-    (bf16 rounding error is relative)."""
-    err = np.abs(gpu_O - ref_O) / scale
-    mx, mean = float(err.max()), float(err.mean())
-    assert mx <= O_MAX_ABS, f"{what}: max abs err {mx:.3e} > {O_MAX_ABS}"
-    assert mean <= O_MEAN_ABS, f"{what}: mean abs err {mean:.3e} > {O_MEAN_ABS}"
+# worst errors seen by compare_o, per test (printed in the terminal summary)
+WORST = {}
+
+
+def _record(what, mx, mean, derived):
+    test = os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0]
+    key = (test, what.split("[")[0] + (" (derived bound)" if derived else ""))
+    old = WORST.get(key, (0.0, 0.0))
+    WORST[key] = (max(old[0], mx), max(old[1], mean))
+
+
+def compare_o(gpu_O, ref_O, what="O", extra=None):
+    """Max and mean abs error of a bf16 output against the oracle.
+
+    extra=None: the stated absolute bounds, max <= 2e-2, mean <= 2e-3.
+    extra (same shape as ref_O): a derived per-element error bound of the
+    output's own arithmetic, added to the stated bound element by element
+    (max) and on average (mean); see outer_logit_extra and grad_extra."""
+    err = np.abs(gpu_O - ref_O)
+    if extra is None:
+        mx, mean = float(err.max(initial=0.0)), float(err.mean()) if err.size else 0.0
+        _record(what, mx, mean, False)
+        assert mx <= O_MAX_ABS, f"{what}: max abs err {mx:.3e} > {O_MAX_ABS}"
+        assert mean <= O_MEAN_ABS, f"{what}: mean abs err {mean:.3e} > {O_MEAN_ABS}"
+        return mx, mean
+    extra = np.broadcast_to(extra, err.shape)
+    over = err - (O_MAX_ABS + extra)
+    mx, mean = float(err.max(initial=0.0)), float(err.mean()) if err.size else 0.0
+    _record(what, mx, mean, True)
+    assert float(over.max(initial=-1.0)) <= 0, (
+        f"{what}: max abs err {mx:.3e}, worst excess over 2e-2 + derived bound {float(over.max()):.3e}")
+    mean_bound = O_MEAN_ABS + (float(extra.mean()) if extra.size else 0.0)
+    assert mean <= mean_bound, f"{what}: mean abs err {mean:.3e} > {mean_bound:.3e}"
     return mx, mean
+
+
+def outer_logit_extra(Q, K, V, s, b, topk, mode, rows, act, pos):
+    """Derived extra bound for the outer position with the raw-logit gate.
+
+    There O_i = sum_j p_j g_j v_j with g_j = e^{s} unbounded, so O is not a
+    convex combination of value rows.  Each term p_j g_j is rounded to bf16
+    before the PV product (relative error <= 2^-9) and O is rounded to bf16
+    on output (<= 2^-9 |O_i| <= 2^-9 A_i), where A_i = sum_j p_j g_j |v_j| is
+    the same sum over absolute values -- the oracle's output on |V|.  The
+    extra term is 2^-8 A_i (first order; fp32 accumulation is far below)."""
+    if not (act == OR.GATE_LOGIT and pos == OR.GATE_OUTER):
+        return None
+    A = OR.sas_attention_head(Q, K, np.abs(V), s, b, topk, mode, rows=rows, act=act, pos=pos)["O"]
+    return 2.0 ** -8 * A
+
+
+def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None):
+    """Derived extra bounds for the backward's dQ, dK, dV of one head.
+
+    dV_j = sum_i P_ij dO_i, dK_j = scale sum_i dS_ij q_i and dQ_i = scale sum_j
+    dS_ij k_j are sums over up to thousands of terms, so their rounding error
+    scales with the sums of absolute terms, not with |v|.  Per term the kernel
+    rounds P and dS = P (dP - Delta) to bf16 (relative 2^-9), and Delta =
+    dO.O uses the forward's bf16 O, which may sit dDelta_i = 2^-8 sum_c
+    |dO_ic O_ic| from the exact value (moving dS_ij by P_ij dDelta_i); the
+    output is rounded to bf16 (2^-9 of its value).  First order:
+      E_S    = 2^-9 |dS| + P dDelta
+      dQ: scale E_S |K| + 2^-9 |dQ|,   dK: scale E_S^T |Q| + 2^-9 |dK|,
+      dV: 2^-9 P^T |dO| + 2^-9 |dV|,
+    each doubled to cover the second-order and fp32 terms.  P comes from the
+    oracle's materialised forward (Q, K, V [N, d]; s the head's scores)."""
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    P = OR.sas_attention_materialized(Q, K, V, s, b, topk, mode, sm_scale)["P"]
+    dP = dO @ V.T
+    Delta = (P * dP).sum(axis=1)
+    dS = P * (dP - Delta[:, None])
+    dDelta = 2.0 ** -8 * np.abs(dO * O_gpu).sum(axis=1)
+    ES = 2.0 ** -9 * np.abs(dS) + P * dDelta[:, None]
+    dQ = sm_scale * dS @ K
+    dK = sm_scale * dS.T @ Q
+    dV = P.T @ dO
+    return {"dQ": 2 * (sm_scale * ES @ np.abs(K) + 2.0 ** -9 * np.abs(dQ)),
+            "dK": 2 * (sm_scale * ES.T @ np.abs(Q) + 2.0 ** -9 * np.abs(dK)),
+            "dV": 2 * (2.0 ** -9 * P.T @ np.abs(dO) + 2.0 ** -9 * np.abs(dV))}
 
 
 def _flip_size(x, delta):

@@ -32,7 +32,9 @@ def _given_case(B, H, N, d, topk, mode, regime="R1", seed=0, rows=None, act=OR.G
             P.check_selection_rows(gi, P.f64(S[bi, hi])[rr], rr, topk)
             lg = g["sel_logg"][bi, hi].numpy()[rr][:, :topk]
             assert np.abs(lg - ref["sel_logg"]).max(initial=0) <= P.LOGG_MAX_ABS
-            P.compare_o(P.f64(g["O"][bi, hi])[rr], ref["O"], f"O[{bi},{hi}]", max(1.0, np.abs(ref["O"]).max()))
+            extra = P.outer_logit_extra(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), P.f64(S[bi, hi]), 64,
+                                        topk, mode, rr, act, pos)
+            P.compare_o(P.f64(g["O"][bi, hi])[rr], ref["O"], f"O[{bi},{hi}]", extra)
             assert np.abs(g["LSE"][bi, hi].numpy()[rr] - ref["LSE"]).max() <= P.LSE_MAX_ABS
             if rows is None and topk > 0:
                 full = g["sel_idx"][bi, hi].numpy()[:, :topk]
@@ -129,7 +131,10 @@ def _learned_case(B, H, N, d, topk, mode=TRAIN, d_sel=0, seed=0, heads=None, row
         total_mismatch += int(mism.sum())
         total += len(rr)
         keep = ~mism
-        P.compare_o(P.f64(g["O"][bi, hi])[rr][keep], ref["O"][keep], f"O[{bi},{hi}]")
+        extra = P.outer_logit_extra(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s, 64, topk, mode, rr,
+                                    act, pos)
+        P.compare_o(P.f64(g["O"][bi, hi])[rr][keep], ref["O"][keep], f"O[{bi},{hi}]",
+                    None if extra is None else extra[keep])
         assert np.abs(g["LSE"][bi, hi].numpy()[rr][keep] - ref["LSE"][keep]).max() <= P.LSE_MAX_ABS
         lg = g["sel_logg"][bi, hi].numpy()[rr][:, :topk][keep]
         assert np.abs(lg - ref["sel_logg"][keep]).max(initial=0) <= P.LOGG_MAX_ABS

@@ -54,9 +54,11 @@ def run_bwd(B, H, N, topk, mode, seed, learned=False, heads=None, rows=None):
         ref = BO.sas_attention_bwd_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s,
                                         P.f64(dO[bi, hi]), 64, topk, mode)
         rr = np.arange(N) if rows is None else rows
+        extra = P.grad_extra(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s, P.f64(dO[bi, hi]),
+                             P.f64(O[bi, hi].cpu()), 64, topk, mode)
         for name, g in (("dQ", dQ), ("dK", dK), ("dV", dV)):
             r = ref[name][rr]
-            P.compare_o(P.f64(g[bi, hi].cpu())[rr], r, f"{name}[{bi},{hi}]", max(1.0, np.abs(r).max()))
+            P.compare_o(P.f64(g[bi, hi].cpu())[rr], r, f"{name}[{bi},{hi}]", extra[name][rr])
         tol = _delta_bound(O[bi, hi].cpu(), dO[bi, hi])[rr][:, None]
         if topk > 0:
             gl = dlogg[bi, hi].cpu().numpy()[rr][:, :topk]

@@ -126,8 +126,7 @@ def run_case(B, Hq, Hkv, d, d_sel, topk, lens, seed=0, exact=False, dense=False,
             elif C and not _check_sets(gs, r, topk, tol):
                 mism += 1
                 continue
-        scale = max(1.0, np.abs(r["O"]).max())
-        P.compare_o(Og[bi, hs], r["O"], f"O[{bi},{g}]", scale)
+        P.compare_o(Og[bi, hs], r["O"], f"O[{bi},{g}]")
         assert np.abs(Lg[bi, hs] - r["LSE"]).max() <= P.LSE_MAX_ABS
     return {"mismatched_groups": mism, "groups": len(ref["groups"]), "launches": launches}
 
@@ -228,8 +227,7 @@ def test_consecutive_steps_in_a_cuda_graph():
                                 P.f64(Wk.cpu()), 64, topk)
             assert np.array_equal(out[2].cpu().numpy(), ref["sel_idx"]), f"step {s}"
             for bi in range(B):
-                P.compare_o(P.f64(out[0][bi].cpu()), ref["O"][bi], f"step {s} O[{bi}]",
-                            max(1.0, np.abs(ref["O"][bi]).max()))
+                P.compare_o(P.f64(out[0][bi].cpu()), ref["O"][bi], f"step {s} O[{bi}]")
                 for g in range(Hkv):
                     summ = ref["groups"][(bi, g)]["summaries"]
                     assert np.array_equal(P.f64(Ksum[bi, g, :summ.shape[0]].cpu()), summ)

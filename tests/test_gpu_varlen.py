@@ -46,7 +46,7 @@ def test_varlen_matches_oracle(lens, cap, Hq, Hkv, d, topk, mode):
     end = int(cu[-1])
     rows = np.arange(end)
     for hi in range(Hq):
-        P.compare_o(P.f64(g["O"][hi])[:end], ref["O"][hi, :end], f"O[{hi}]", max(1.0, np.abs(ref["O"]).max()))
+        P.compare_o(P.f64(g["O"][hi])[:end], ref["O"][hi, :end], f"O[{hi}]")
         assert np.abs(g["LSE"][hi].numpy()[:end] - ref["LSE"][hi, :end]).max() <= P.LSE_MAX_ABS
     for gk in range(Hkv):
         assert np.array_equal(g["sel_idx"][gk].numpy()[:end, :topk], ref["sel_idx"][gk, :end])
@@ -85,7 +85,7 @@ def test_long_gqa_pack_sampled_rows():
         gk = hi // (Hq // Hkv)
         r = OR.sas_attention_head(P.f64(Q[hi, b0:b0 + n]), P.f64(K[gk, b0:b0 + n]), P.f64(V[gk, b0:b0 + n]),
                                   P.f64(S[gk, b0:b0 + n]), 64, topk, rows=rows)
-        P.compare_o(P.f64(g["O"][hi, b0 + rows]), r["O"], f"O[{hi}]", max(1.0, np.abs(r["O"]).max()))
+        P.compare_o(P.f64(g["O"][hi, b0 + rows]), r["O"], f"O[{hi}]")
         assert np.abs(g["LSE"][hi, b0 + rows].numpy() - r["LSE"]).max() <= P.LSE_MAX_ABS
         assert np.array_equal(g["sel_idx"][gk, b0 + rows].numpy()[:, :topk], r["sel_idx"])
 
