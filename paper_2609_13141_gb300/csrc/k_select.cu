@@ -510,8 +510,29 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 //   region A: the 128-row Q tile, overwritten by the bf16 projected queries q~;
 //   region B: the tile's Wq[h], then (once the projection has run) the
 //             double-buffered 64-block chunks of projected block summaries;
-//   after the last chunk, regions A and B hold the output staging;
-//   then the Top-K columns, the current 32 scores of each row, the union bitmap.
+//   then the per-row score histograms, the output staging and the union bitmap.
+//
+// Top-K without per-row replacement.  Replacing the worst kept entry whenever a
+// better score arrives diverges across the 32 rows of a warp (each row
+// replaces at different times, so the warp pays for every row's replacements),
+// so the score chunks are streamed several times instead, with uniform work
+// per score (the score products are cheap to re-issue):
+//   pass A: the row's log-sum-exp, maximum, minimum and the first two moments
+//           of its scores;
+//   pass B: a histogram of the scores above a low threshold lo, in kBins - 1
+//           equal bins up to a high threshold hi and one bin above hi (lo and
+//           hi placed from the moments where about K + 5 sqrt(K) and K -
+//           5 sqrt(K) scores of a normal sample lie above them); it locates
+//           the bin holding the K-th largest score;
+//   pass C: scores in bins above that bin are kept and staged in block order;
+//           the boundary bin's few scores are held in the row's histogram
+//           words (no longer needed) and the best R = K - (number above) of
+//           them, by (score descending, block ascending), join the list;
+//   pass D: only if some row of the tile could not use A-C (its scores are
+//           too concentrated for the bins: equal scores, a crowded boundary bin):
+//           that row runs replace-the-worst over all its scores.
+// Every pass compares the same fp32 scores with the same bin arithmetic
+// (rounded steps, no contraction), so the passes agree on every score.
 template <int D, int DS>
 struct SelProjCfg {
     static constexpr int Q_BYTES = kRows * D * 2;
@@ -524,15 +545,305 @@ struct SelProjCfg {
     static constexpr uint32_t IDESC_S = idesc_bf16(kRows, 64, 0, 0);
     static constexpr int TMEM_S = 128;            // score buffers at columns 128 and 192
 };
-constexpr size_t kValuesBytes = size_t(32) * kRows * 4;
+
+constexpr int kBins = 48;                           // histogram bins per row (pass B)
+constexpr int kBinWords = kBins / 2;                // two 16-bit counters per word
+constexpr int kBoundaryMax = kBinWords / 2;         // boundary-bin scores a row holds (in its dead histogram words)
+constexpr size_t kHistBytes = size_t(kBinWords) * kRows * 4;
+constexpr int kPassA = 0, kPassB = 1, kPassC = 2, kPassD = 3;
+constexpr int kRowAll = 0, kRowNormal = 1, kRowFail = 2;   // C_i <= K: keep all; thresholds; fallback
+
 template <int D, int DS>
-__host__ __device__ constexpr size_t proj_region0(int K) {
-    return size_t(SelProjCfg<D, DS>::A_BYTES + SelProjCfg<D, DS>::B_BYTES) > staging_bytes(K)
-               ? size_t(SelProjCfg<D, DS>::A_BYTES + SelProjCfg<D, DS>::B_BYTES)
-               : staging_bytes(K);
+__host__ __device__ constexpr size_t proj_smem_bytes(int K, int C) {
+    return size_t(SelProjCfg<D, DS>::A_BYTES) + SelProjCfg<D, DS>::B_BYTES + kHistBytes + staging_bytes(K) +
+           bitmap_bytes(C);
 }
 
-template <int D, int DS, bool REG>
+// Selection works on the raw products u = q~ . K~ (the scores are s = u / sqrt(d_sel),
+// an order-preserving scale): thresholds, bins and ties are all on u, and s is
+// formed only for the log-sum-exp and the emitted log-gates.
+//
+// Bin of a product at or above lo: floor((u - lo) / w) with w = (hi - lo) / (kBins - 1),
+// clamped to the top bin (everything from hi up).  Rounded steps without
+// contraction (the packed and the scalar forms round identically), so passes B
+// and C place every product in the same bin.
+__device__ __forceinline__ int bin_clamp(float x) { return min(kBins - 1, __float2int_rz(x)); }
+__device__ __forceinline__ float bin_x(float u, float neg_lo, float inv_w) {
+    return __fmul_rn(__fadd_rn(u, neg_lo), inv_w);
+}
+
+// The per-row state carried across the passes.
+struct RowSel {
+    RowLse l;                   // pass A: running max of u, sum of exp(s - s_max)
+    float v0;                   // pass A: shift (the row's first product)
+    uint64_t s1, s2;            // pass A: packed sums of (u - v0) and (u - v0)^2
+    float mn;                   // pass A: minimum
+    float lo, inv_w;            // histogram origin and inverse bin width (lo = -inf: keep all, +inf: fallback)
+    int mode;                   // kRowAll / kRowNormal / kRowFail
+    int bstar, hi_bin, nabove;  // after B: boundary bin, first bin kept whole, products above it
+    int pos;                    // pass C / D: entries staged so far
+    int nbc;                    // boundary products held (product, block) in the row's histogram words
+    float ws;                   // pass D: worst kept product, its slot
+    int wpos;
+};
+
+// Shared-memory addresses of one row's staging entries and histogram words.
+struct RowAddr {
+    uint32_t idx, lg;           // staging entry 0 of the row (int32 block, fp32 product)
+    uint32_t hist;              // histogram word 0 of the row (word w at hist + w * kRows * 4)
+};
+
+__device__ __forceinline__ void stage_score(const Staging& st, int r, int e, int m, float u) {
+    st.idx[r * st.stride + e] = m;
+    st.lg[r * st.stride + e] = u;
+}
+
+// Pass D state of a row: entries staged, worst kept product and its slot.
+struct FallbackState {
+    int pos;
+    float ws;
+    int wpos;
+};
+
+// Pass D, one product: the row's first K' products fill its staging row, a later
+// one replaces the worst kept entry (lowest product; among equal ones the highest
+// block, which ranks last because ties go to the lower block) when strictly
+// larger.  Kept out of line: the fallback is rare, and its loops inlined at every
+// one of the 32 unrolled positions would crowd the hot passes out of the
+// instruction cache.
+__device__ __noinline__ FallbackState fallback_offer(FallbackState f, float u, int m, int32_t* idx, float* sc,
+                                                     int Kp) {
+    if (f.pos < Kp) {
+        idx[f.pos] = m;
+        sc[f.pos] = u;
+        ++f.pos;
+        if (f.pos < Kp) return f;
+    } else if (u > f.ws) {
+        idx[f.wpos] = m;
+        sc[f.wpos] = u;
+    } else {
+        return f;
+    }
+    float ws = CUDART_INF_F;
+    int wm = -1, wp = 0;
+    for (int e = 0; e < Kp; ++e) {
+        const float se = sc[e];
+        const int me = idx[e];
+        if (se < ws || (se == ws && me > wm)) {
+            ws = se;
+            wm = me;
+            wp = e;
+        }
+    }
+    f.ws = ws;
+    f.wpos = wp;
+    return f;
+}
+
+// Sorts a staged row's first n entries by block index (insertion sort: the rows
+// reaching it are sorted but for a short tail, or rare fallback rows).
+__device__ __forceinline__ void staged_sort_by_block(const Staging& st, int r, int n) {
+    int32_t* idx = st.idx + r * st.stride;
+    float* sc = st.lg + r * st.stride;
+    for (int a = 1; a < n; ++a) {
+        const int km = idx[a];
+        const float ks = sc[a];
+        int b = a - 1;
+        while (b >= 0 && idx[b] > km) {
+            idx[b + 1] = idx[b];
+            sc[b + 1] = sc[b];
+            --b;
+        }
+        idx[b + 1] = km;
+        sc[b + 1] = ks;
+    }
+}
+
+// One half-chunk (32 products of blocks m0 .. m0 + 31) of pass `kind` for one
+// row.  FULL: all 32 are within the row's history (the common case, no
+// per-entry range test); otherwise entries j >= lim = C_i - m0 are ignored.
+// c2 = scale * log2(e) packed twice (exp of s - s_max as exp2 of u c - u_max c).
+template <bool FULL>
+__device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, int m0, int lim, int Kp,
+                                         const RowAddr& ra, const Staging& st, int r, float c) {
+    if (kind == kPassA) {
+        if (m0 == 0) rs.v0 = u[0];
+        float cm = -CUDART_INF_F, mn = rs.mn;
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            const bool in0 = FULL || j < lim, in1 = FULL || j + 1 < lim;
+            cm = max3f(cm, in0 ? u[j] : -CUDART_INF_F, in1 ? u[j + 1] : -CUDART_INF_F);
+            mn = min3f(mn, in0 ? u[j] : CUDART_INF_F, in1 ? u[j + 1] : CUDART_INF_F);
+        }
+        const float nm = fmaxf(rs.l.mx, cm);
+        const float noff = -nm * c;
+        const uint64_t c2 = f32x2(c, c), off2 = f32x2(noff, noff);
+        const uint64_t nv0 = f32x2(-rs.v0, -rs.v0);
+        uint64_t acc[2] = {0, 0};
+        uint64_t s1 = rs.s1, s2 = rs.s2;
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            const bool in0 = FULL || j < lim, in1 = FULL || j + 1 < lim;
+            float a0, a1;
+            f32x2_split(fma_f32x2(f32x2(u[j], u[j + 1]), c2, off2), a0, a1);
+            const float e0 = in0 ? fast_exp2(a0) : 0.f, e1 = in1 ? fast_exp2(a1) : 0.f;
+            acc[(j >> 1) & 1] = add_f32x2(acc[(j >> 1) & 1], f32x2(e0, e1));
+            uint64_t x = add_f32x2(f32x2(u[j], u[j + 1]), nv0);
+            if (!FULL) {
+                float x0, x1;
+                f32x2_split(x, x0, x1);
+                x = f32x2(in0 ? x0 : 0.f, in1 ? x1 : 0.f);
+            }
+            s1 = add_f32x2(s1, x);
+            s2 = fma_f32x2(x, x, s2);
+        }
+        float q0, q1, q2, q3;
+        f32x2_split(acc[0], q0, q1);
+        f32x2_split(acc[1], q2, q3);
+        const float scale_old = rs.l.mx == -CUDART_INF_F ? 0.f : fast_exp2((rs.l.mx - nm) * c);
+        rs.l.sum = rs.l.sum * scale_old + ((q0 + q1) + (q2 + q3));
+        rs.l.mx = nm;
+        rs.s1 = s1;
+        rs.s2 = s2;
+        rs.mn = mn;
+    } else if (kind == kPassB) {
+        const float nlo = -rs.lo, iw = rs.inv_w;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const bool p = (FULL || j < lim) && u[j] >= rs.lo;
+            const int b = bin_clamp(bin_x(u[j], nlo, iw));
+            const bool hi = b >= kBinWords;
+            red_shared_add_if(p, ra.hist + static_cast<uint32_t>((hi ? b - kBinWords : b) * (kRows * 4)),
+                              hi ? 0x10000u : 1u);
+        }
+    } else if (kind == kPassC) {
+        const float nlo = -rs.lo, iw = rs.inv_w;
+        int pos = rs.pos, nbc = rs.nbc;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const bool in = (FULL || j < lim) && u[j] >= rs.lo;
+            const int b = bin_clamp(bin_x(u[j], nlo, iw));
+            const bool keep = in && b >= rs.hi_bin;
+            const bool bnd = in && b == rs.bstar && b < rs.hi_bin;
+            st_shared_if(keep, ra.idx + pos * 4, static_cast<uint32_t>(m0 + j));
+            st_shared_if(keep, ra.lg + pos * 4, __float_as_uint(u[j]));
+            pos += keep ? 1 : 0;
+            st_shared_if(bnd, ra.hist + (2 * nbc) * (kRows * 4), __float_as_uint(u[j]));
+            st_shared_if(bnd, ra.hist + (2 * nbc + 1) * (kRows * 4), static_cast<uint32_t>(m0 + j));
+            nbc += bnd ? 1 : 0;
+        }
+        rs.pos = pos;
+        rs.nbc = nbc;
+    } else {   // kPassD: replace-the-worst for the rows the bins could not resolve
+        if (rs.mode != kRowFail) return;
+        FallbackState f{rs.pos, rs.ws, rs.wpos};
+        int32_t* idx = st.idx + r * st.stride;
+        float* sc = st.lg + r * st.stride;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (FULL || j < lim) f = fallback_offer(f, u[j], m0 + j, idx, sc, Kp);
+        rs.pos = f.pos;
+        rs.ws = f.ws;
+        rs.wpos = f.wpos;
+    }
+}
+
+__device__ __forceinline__ void row_set_all(RowSel& rs) {
+    rs.mode = kRowAll;
+    rs.lo = -CUDART_INF_F;
+    rs.inv_w = 1.f;
+    rs.hi_bin = 0;
+    rs.bstar = -1;
+}
+__device__ __forceinline__ void row_set_fail(RowSel& rs) {
+    rs.mode = kRowFail;
+    rs.lo = CUDART_INF_F;   // passes B and C take nothing from this row
+    rs.hi_bin = kBins;
+    rs.bstar = -1;
+}
+
+// After pass A: the histogram range of a row with more than K blocks.
+__device__ __forceinline__ void row_after_a(RowSel& rs, int Ci, int K) {
+    if (Ci <= K) {
+        row_set_all(rs);
+        return;
+    }
+    const float n = static_cast<float>(Ci);
+    float a0, a1, b0, b1;
+    f32x2_split(rs.s1, a0, a1);
+    f32x2_split(rs.s2, b0, b1);
+    const float mean = (a0 + a1) / n;
+    const float var = fmaxf(fmaf(-mean, mean, (b0 + b1) / n), 0.f);
+    const float sd = sqrtf(var);
+    // a normal sample has a fraction P(Z > z) above mean + sd z; lo leaves about
+    // K + 5 sqrt(K) products above it, hi about K - 5 sqrt(K) (at least half a one)
+    const float kf = static_cast<float>(K), dk = 5.f * sqrtf(kf);
+    const float p_lo = (kf + dk) / n, p_hi = fmaxf(kf - dk, 0.5f) / n;
+    float lo = rs.mn, hi = rs.l.mx;
+    if (p_lo < 1.f) lo = fmaxf(rs.mn, rs.v0 + mean + sd * 1.41421356f * erfinvf(1.f - 2.f * p_lo));
+    if (p_hi < 1.f) hi = fminf(rs.l.mx, rs.v0 + mean + sd * 1.41421356f * erfinvf(1.f - 2.f * p_hi));
+    const float span = hi - lo;
+    const float inv_w = static_cast<float>(kBins - 1) / span;
+    if (span > 0.f && isfinite(inv_w) && Ci <= 65535) {
+        rs.mode = kRowNormal;
+        rs.lo = lo;
+        rs.inv_w = inv_w;
+        rs.hi_bin = kBins;   // nothing is kept before pass B has placed the K-th product
+        rs.bstar = -1;
+    } else {
+        row_set_fail(rs);
+    }
+}
+
+// After pass B: the bin holding the K-th largest product (scanning from the top).
+// Word w of the row holds bin w in its low half and bin w + kBinWords in its high half.
+__device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, int r, int Kp) {
+    if (rs.mode != kRowNormal) return;
+    int cum = 0, bstar = -1, nabove = 0, nb = 0;
+#pragma unroll
+    for (int b = kBins - 1; b >= 0; --b) {
+        const uint32_t word = hist[(b % kBinWords) * kRows + r];
+        const int cb = static_cast<int>(b >= kBinWords ? (word >> 16) : (word & 0xffffu));
+        if (bstar < 0 && cum + cb >= Kp) {
+            bstar = b;
+            nabove = cum;
+            nb = cb;
+        }
+        cum += cb;
+    }
+    if (bstar < 0) {   // fewer than K' products above lo: the estimate was too high
+        row_set_fail(rs);
+        return;
+    }
+    const bool take_all = nabove + nb == Kp;
+    if (!take_all && nb > kBoundaryMax) {
+        row_set_fail(rs);
+        return;
+    }
+    rs.bstar = bstar;
+    rs.hi_bin = take_all ? bstar : bstar + 1;
+    rs.nabove = nabove;
+}
+
+// After pass C: the best R = K' - nabove boundary products join the list (rank by
+// product descending, then block ascending; they are held in block order).
+__device__ __forceinline__ void row_after_c(RowSel& rs, const uint32_t* hist, const Staging& st, int r, int Kp) {
+    if (rs.mode != kRowNormal || rs.pos >= Kp) return;
+    const int R = Kp - rs.nabove;
+    for (int a = 0; a < rs.nbc; ++a) {
+        const float sa = __uint_as_float(hist[(2 * a) * kRows + r]);
+        const int ma = static_cast<int>(hist[(2 * a + 1) * kRows + r]);
+        int rank = 0;
+        for (int b = 0; b < rs.nbc; ++b) {
+            const float sb = __uint_as_float(hist[(2 * b) * kRows + r]);
+            rank += (sb > sa || (sb == sa && b < a)) ? 1 : 0;   // b < a: lower block
+        }
+        if (rank < R) stage_score(st, r, rs.pos++, ma, sa);
+    }
+    if (rs.nabove > 0) staged_sort_by_block(st, r, rs.pos);
+}
+
+template <int D, int DS>
 __global__ void __launch_bounds__(192, 2)
 select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapWq,
                    const __grid_constant__ CUtensorMap mapKt, SelParams p, int H, int G) {
@@ -542,9 +853,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     using Cfg = SelProjCfg<D, DS>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ uint64_t in_full, in_empty, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2],
-        drain_bar;
+        drain_bar, plan_bar;
     __shared__ uint32_t tmem_base_sh;
-    __shared__ int abort_flag;
+    __shared__ int abort_flag, fail_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
     const uint32_t raw = smem_u32(smem_raw);
@@ -552,15 +863,26 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     const int K = p.topk;
     uint8_t* a_s = smem;                        // Q tile, then q~
     uint8_t* b_s = smem + Cfg::A_BYTES;         // Wq, then summary chunks
-    uint8_t* topk_s = smem + proj_region0<D, DS>(K);
-    float* values_s = reinterpret_cast<float*>(topk_s + smem_topk_bytes(K));
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(topk_s + smem_topk_bytes(K) + kValuesBytes);
+    uint32_t* hist = reinterpret_cast<uint32_t*>(smem + Cfg::A_BYTES + Cfg::B_BYTES);
+    uint8_t* stage_base = smem + Cfg::A_BYTES + Cfg::B_BYTES + kHistBytes;
+    const Staging st{reinterpret_cast<int32_t*>(stage_base),
+                     reinterpret_cast<float*>(stage_base + size_t(kRows) * (K + 1) * 4), K + 1};
+    uint32_t* bitmap = reinterpret_cast<uint32_t*>(stage_base + staging_bytes(K));
 
     const int t = tile_of_block(p.T, p.BH);
     const int bh = head_of_block(p.BH);
     const int diag = 2 * t;
     const int nb = min(2 * t + 1, p.F);          // blocks scored for this tile
-    const int nchunks = (nb + 63) >> 6;
+    const int nchunks = K > 0 ? (nb + 63) >> 6 : 0;
+    // the most blocks any row of the tile has: a histogram pass only when it exceeds K
+    const int last_row = min(p.N, (t + 1) * kRows) - 1;
+    const int tile_ci = last_row >= t * kRows ? (last_row >> 6) : 0;
+    const bool pass_b = tile_ci > K;
+    // passes over the chunks, in order; D runs only if a row fails (decided after B)
+    const int npre = nchunks > 0 ? (pass_b ? 3 : 2) : 0;   // A, [B], C
+    // a history of at most two chunks stays in the two TMEM score buffers: its
+    // products are computed once and every pass reads them again
+    const bool resident = nchunks <= 2;
 
     const int nwords = (p.C + 31) >> 5;
     for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
@@ -576,7 +898,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             mbar_init(&s_free[b], 128);
         }
         mbar_init(&drain_bar, 1);
+        mbar_init(&plan_bar, 4);   // one arrive per row warp once its rows know their mode (after pass B)
         abort_flag = 0;
+        fail_flag = 0;
         fence_barrier_init();
     }
     if (warp == 1) {
@@ -609,14 +933,25 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             }
             int issued = 0;
             if (ok) ok = mbar_wait(&proj_done, 0, wc);   // region B is free once the projection ran
-            for (int c = 0; ok && c < nchunks; ++c) {
-                const int b = c & 1;
-                if (!mbar_wait(&kc_empty[b], ((c >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
-                mbar_arrive_expect_tx(&kc_full[b], Cfg::KC_BYTES);
+            const int npass = resident ? 1 : npre;
+            for (int ps = 0; ok && ps < npass + 1; ++ps) {
+                if (resident && ps == npass) break;
+                if (ps == npass) {
+                    // after the pre-planned passes: pass D if a row failed
+                    if (!pass_b) break;
+                    if (!mbar_wait(&plan_bar, 0, wc)) { ok = false; break; }
+                    if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
+                }
+                for (int c = 0; ok && c < nchunks; ++c) {
+                    const int gc = issued;
+                    const int b = gc & 1;
+                    if (!mbar_wait(&kc_empty[b], ((gc >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
+                    mbar_arrive_expect_tx(&kc_full[b], Cfg::KC_BYTES);
 #pragma unroll
-                for (int a = 0; a < DS / 64; ++a)
-                    tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, c * 64, bh);
-                ++issued;
+                    for (int a = 0; a < DS / 64; ++a)
+                        tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, c * 64, bh);
+                    ++issued;
+                }
             }
             if (!ok) {
                 if (rounds > 0) mbar_wait_drain(&in_full, (rounds - 1) & 1, p.limit, p.status);
@@ -641,14 +976,24 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             }
             umma_commit(hq + 1 < G ? &in_empty : &proj_done);   // regions A, B free for the next round
         }
-        if (in_ok) {
-            // S[c&1] = q~ (128 x DS, bf16 in region A) * Kt_chunk (64 x DS)^T
-            if (mbar_wait(&qt_ready, 0, wc)) {
-                for (int c = 0; c < nchunks; ++c) {
-                    const int b = c & 1;
-                    const uint32_t ph = (c >> 1) & 1;
-                    if (!mbar_wait(&kc_full[b], ph, wc)) break;
-                    if (!mbar_wait(&s_free[b], ph ^ 1u, wc)) break;
+        if (in_ok && mbar_wait(&qt_ready, 0, wc)) {
+            // S[gc&1] = q~ (128 x DS, bf16 in region A) * Kt_chunk (64 x DS)^T, for every
+            // chunk of every pass
+            int gc = 0;
+            bool ok = true;
+            const int npass = resident ? 1 : npre;
+            for (int ps = 0; ok && ps < npass + 1; ++ps) {
+                if (resident && ps == npass) break;
+                if (ps == npass) {
+                    if (!pass_b) break;
+                    if (!mbar_wait(&plan_bar, 0, wc)) break;
+                    if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
+                }
+                for (int c = 0; c < nchunks; ++c, ++gc) {
+                    const int b = gc & 1;
+                    const uint32_t ph = (gc >> 1) & 1;
+                    if (!mbar_wait(&kc_full[b], ph, wc)) { ok = false; break; }
+                    if (!mbar_wait(&s_free[b], ph ^ 1u, wc)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t k_addr = smem_u32(b_s + b * Cfg::KC_BYTES);
 #pragma unroll
@@ -672,7 +1017,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         const int i = t * kRows + r;
         const bool valid = i < p.N;
         const int Ci = valid ? (i >> 6) : 0;
+        const int Kp = min(K, Ci);
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+        for (int w = 0; w < kBinWords; ++w) hist[w * kRows + r] = 0u;   // this row's counters
         bool ok = true;
         if (nchunks > 0) {
             // q~ row: fp32 from TMEM -> bf16 -> region A in the 128-byte-swizzled
@@ -703,47 +1050,86 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&qt_ready);
         }
-        RegTopK rtk;
-        reg_init(rtk);
-        SmemTopK stk{};
-        if constexpr (!REG) {
-            stk.s = reinterpret_cast<float*>(topk_s) + r;
-            stk.m = reinterpret_cast<int*>(topk_s + size_t(K) * kRows * 4) + r;
-            stk.ws = -CUDART_INF_F;
-        }
-        RowLse lse{-CUDART_INF_F, 0.f};
-        float* vcol = values_s + r;   // this row's current 32 scores, element j at j * kRows
-        for (int c = 0; ok && c < nchunks; ++c) {
-            const int b = c & 1;
-            if (!mbar_wait_warp(&s_full[b], (c >> 1) & 1, wc)) break;
-            tc_fence_after();
+        RowSel rs;
+        rs.l = RowLse{-CUDART_INF_F, 0.f};
+        rs.v0 = 0.f; rs.s1 = 0; rs.s2 = 0; rs.mn = CUDART_INF_F;
+        row_set_all(rs);
+        rs.nabove = 0; rs.pos = 0; rs.nbc = 0;
+        rs.ws = -CUDART_INF_F; rs.wpos = 0;
+        const float c_exp = p.score_scale * kLog2e;
+        const uint32_t hist_r = smem_u32(hist + r);
+        const RowAddr ra{smem_u32(st.idx + r * st.stride), smem_u32(st.lg + r * st.stride), hist_r};
+        int gc = 0;
+        for (int ps = 0; ok && ps < npre + 1; ++ps) {
+            int kind;
+            if (ps == npre) {
+                if (!pass_b) break;
+                if (!mbar_wait_warp(&plan_bar, 0, wc)) { ok = false; break; }
+                if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
+                kind = kPassD;
+            } else {
+                kind = ps == 0 ? kPassA : (ps == npre - 1 ? kPassC : kPassB);
+            }
+            for (int c = 0; c < nchunks; ++c, ++gc) {
+                const int b = resident ? c : (gc & 1);
+                if ((!resident || ps == 0) && !mbar_wait_warp(&s_full[b], resident ? 0 : ((gc >> 1) & 1), wc)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
 #pragma unroll 1
-            for (int half = 0; half < 2; ++half) {
-                uint32_t u[32];
-                tmem_ld32(lane_addr + Cfg::TMEM_S + b * 64 + half * 32, u);
-                tmem_wait_ld();
-                if (half == 1) {
-                    tc_fence_before();
-                    mbar_arrive(&s_free[b]);
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t uu[32];
+                    tmem_ld32(lane_addr + Cfg::TMEM_S + b * 64 + half * 32, uu);
+                    tmem_wait_ld();
+                    if (half == 1 && !resident) {
+                        tc_fence_before();
+                        mbar_arrive(&s_free[b]);
+                    }
+                    const int m0 = 64 * c + 32 * half;
+                    const int lim = Ci - m0;
+                    // the vote comes before any lane leaves; the lanes meet again
+                    // before the next warp-collective TMEM load
+                    const bool full = __all_sync(0xffffffffu, lim >= 32);
+                    const float* u = reinterpret_cast<const float*>(uu);
+                    if (full)
+                        row_pass<true>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    else if (lim > 0)
+                        row_pass<false>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    __syncwarp();
                 }
-                float v[32];
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    v[j] = __uint_as_float(u[j]) * p.score_scale;
-                    vcol[j * kRows] = v[j];
-                }
-                if constexpr (REG) reg_consume(rtk, lse, v, vcol, kRows, 2 * c + half, Ci, K);
-                else smem_consume(stk, lse, v, vcol, kRows, 2 * c + half, Ci, K);
+            }
+            if (!ok) break;
+            if (kind == kPassA) {
+                row_after_a(rs, Ci, K);
+            } else if (kind == kPassB) {
+                row_after_b(rs, hist, r, Kp);
+                // whether pass D runs (some row failed), for the producer, the MMA
+                // issuer and the row warps: flag first, then one arrive per warp
+                if (rs.mode == kRowFail) atomicOr(&fail_flag, 1);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&plan_bar);
+            } else if (kind == kPassC) {
+                row_after_c(rs, hist, st, r, Kp);
+            } else {
+                staged_sort_by_block(st, r, rs.pos);
             }
         }
-        // Every MMA has completed once the last chunk was read, so regions A
-        // and B are free and become the output staging area.
-        const Staging st{reinterpret_cast<int32_t*>(smem),
-                         reinterpret_cast<float*>(smem + size_t(kRows) * (K + 1) * 4), K + 1};
-        ok = !abort_flag;
+        ok = ok && !abort_flag;
         if (valid && ok) {
-            if constexpr (REG) row_emit(rtk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
-            else row_emit(stk, lse, st, r, Ci, K, diag, bitmap, p.gate_act);
+            // log-gates from s = u / sqrt(d_sel), -1 padding, tile-union bits
+            const float lse = Ci > 0 ? __fmul_rn(rs.l.mx, p.score_scale) + logf(rs.l.sum) : 0.f;
+            for (int e = 0; e < K; ++e) {
+                if (e < Kp) {
+                    const int m = st.idx[r * st.stride + e];
+                    const float sc = __fmul_rn(st.lg[r * st.stride + e], p.score_scale);
+                    st.lg[r * st.stride + e] = staged_gate(sc, lse, p.gate_act);
+                    if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
+                } else {
+                    st.idx[r * st.stride + e] = -1;
+                    st.lg[r * st.stride + e] = 0.f;
+                }
+            }
         }
         named_bar_sync(1, 128);
         if (ok)
@@ -760,11 +1146,11 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     }
 }
 
-template <int D, int DS, bool REG>
+template <int D, int DS>
 cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
-    const size_t smem = 1024 + proj_region0<D, DS>(a.topk) + smem_topk_bytes(a.topk) + kValuesBytes + bitmap_bytes(a.C);
+    const size_t smem = 1024 + proj_smem_bytes<D, DS>(a.topk, a.C);
     if (smem > 227 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS, REG>), smem);
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS>), smem);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mw, mk;
     // Q of all query heads; Wq [H][DS][G D] (a group's gate-query projection)
@@ -772,7 +1158,7 @@ cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv
     if (make_tmap_bf16_3d(&mw, a.Wq, static_cast<uint64_t>(a.G) * D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
     const dim3 grid(a.BH * a.T);
-    select_proj_kernel<D, DS, REG><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H, a.G);
+    select_proj_kernel<D, DS><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H, a.G);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;
@@ -791,10 +1177,6 @@ cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEn
     return e;
 }
 
-template <int D, int DS>
-cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
-    return a.topk <= 32 ? launch_proj<D, DS, true>(a, p, env, err) : launch_proj<D, DS, false>(a, p, env, err);
-}
 
 constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
 
@@ -883,10 +1265,10 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     }
     const bool reg = a.topk <= 32;
     if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
-    if (a.d == 128 && a.d_sel == 128) return launch_proj_k<128, 128>(a, p, env, err);
-    if (a.d == 128 && a.d_sel == 64) return launch_proj_k<128, 64>(a, p, env, err);
-    if (a.d == 64 && a.d_sel == 64) return launch_proj_k<64, 64>(a, p, env, err);
-    if (a.d == 64 && a.d_sel == 128) return launch_proj_k<64, 128>(a, p, env, err);
+    if (a.d == 128 && a.d_sel == 128) return launch_proj<128, 128>(a, p, env, err);
+    if (a.d == 128 && a.d_sel == 64) return launch_proj<128, 64>(a, p, env, err);
+    if (a.d == 64 && a.d_sel == 64) return launch_proj<64, 64>(a, p, env, err);
+    if (a.d == 64 && a.d_sel == 128) return launch_proj<64, 128>(a, p, env, err);
     *err = "selection: unsupported head / selector dims";
     return cudaErrorInvalidValue;
 }

@@ -339,6 +339,22 @@ __device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
     asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
     return d;
 }
+// Shared-memory reduction and stores under a predicate, without a branch around
+// them (per-lane work that is rare for each lane but frequent for the warp).
+__device__ __forceinline__ void red_shared_add_if(bool p, uint32_t saddr, uint32_t v) {
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t@q red.shared.add.u32 [%1], %2;\n\t}" ::"r"(
+            static_cast<int>(p)),
+        "r"(saddr), "r"(v)
+        : "memory");
+}
+__device__ __forceinline__ void st_shared_if(bool p, uint32_t saddr, uint32_t v) {
+    asm volatile("{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t@q st.shared.u32 [%1], %2;\n\t}" ::"r"(
+                     static_cast<int>(p)),
+                 "r"(saddr), "r"(v)
+                 : "memory");
+}
+
 __device__ __forceinline__ float max3f(float a, float b, float c) {
     float d;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));

@@ -153,6 +153,31 @@ def test_learned_selector_exact_inputs_bit_exact():
     _learned_case(1, 2, 700, 64, 3, exact_inputs=True, seed=12, mode=INFER)
 
 
+def test_learned_selector_tiles_mixing_tied_and_spread_rows():
+    # Integer inputs (every selector sum exact) where rows 32q .. 32q+15 of each
+    # group of 48 have zero queries: their scores all tie at 0, so the kept set
+    # is the lowest K blocks (ties go to the lower block) and the selection
+    # kernel's histogram cannot separate them; those rows take its
+    # replace-the-worst pass while the other rows of the same tiles take the
+    # threshold path.  Kept sets, unions and outputs must match the oracle.
+    B, H, N, d, topk = 1, 2, 2000, 128, 5
+    Q, K, V, Wq, Wk = synth.integer_selector_inputs(B, H, N, d, d, seed=17)
+    zero = (torch.arange(N) % 48) < 16
+    Q[:, :, zero, :] = 0
+    g = P.run_gpu(B, H, N, d, topk, TRAIN, Q, K, V, Wq=Wq, Wk=Wk, d_sel=d)
+    assert g["status"] == 0
+    for hi in range(H):
+        s = P.oracle_scores(Q, K, Wq, Wk, 0, hi)
+        rr = np.arange(N)
+        ref = OR.sas_attention_head(P.f64(Q[0, hi]), P.f64(K[0, hi]), P.f64(V[0, hi]), s, 64, topk, TRAIN)
+        P.check_selection_rows(g["sel_idx"][0, hi].numpy()[:, :topk], s, rr, topk)
+        tied = rr[zero.numpy() & (rr >= 64 * (topk + 1))]
+        assert np.array_equal(g["sel_idx"][0, hi].numpy()[tied, :topk], np.tile(np.arange(topk), (len(tied), 1)))
+        P.compare_o(P.f64(g["O"][0, hi]), ref["O"], f"O[0,{hi}]")
+        assert np.abs(g["sel_logg"][0, hi].numpy()[:, :topk] - ref["sel_logg"]).max() <= P.LOGG_MAX_ABS
+        assert np.array_equal(g["unions"][0, hi], P.oracle_union_counts(g["sel_idx"][0, hi].numpy()[:, :topk], N, topk))
+
+
 def test_learned_selector_ragged():
     _learned_case(2, 2, 1000, 128, 4)
 
