@@ -15,6 +15,8 @@ What it computes (SAS, "Simple Attention Sparsification", arXiv 2609.13141):
   a5  gated attention      o = softmax(q K_S^T + log g_S) V_S                (Eq. ours_train; Alg. 2 for the ungated form)
       ablation forms       gate activation softmax / sigmoid / logit and gate position inner / outer
                            (Sec. 4.2, Components of learnable ranking; Eq. general_gate)
+      training scopes      full scope: every historical block gated, no Top-K (Table 1 setting 9);
+                           full*: noise added to s before activation and Top-K (Table 1 setting 11)
   a6  dense MLP (not SAS)  Y = GELU(X W1^T + b1) W2^T + b2, exact-erf GELU
 
 Readings of points the paper leaves open (each one is also listed with its
@@ -385,6 +387,47 @@ def sas_attention_varlen(Q, K, V, cu_seqlens, b, topk, scores=None, mode=MODE_TR
                 sel_idx[g, s0:s1] = r["sel_idx"]
                 sel_logg[g, s0:s1] = r["sel_logg"]
     return {"O": O, "LSE": LSE, "sel_idx": sel_idx, "sel_logg": sel_logg}
+
+
+# ------------------------------------------------------ training scopes --
+
+def sas_attention_full_scope(Q, K, V, s, b, sm_scale=None, rows=None):
+    """Full training scope (Table 1 setting 9: Eq. fula with the log-gates of
+    Eq. ours_train; Sec. 4.2 "training scope"): no Top-K.  Row i attends to
+    every key of its history; a key of historical block m < C_i gets the bias
+    log g_m = s_m - LSE(s_0 .. s_{C_i - 1}) (Eq. normalized_log_gate), a key of
+    the current block (j <= i) gets 0 (unit gate).
+    Q, K, V [N, d]; s [N, >=C-1].  Returns dict with O [R, d] and LSE [R].
+    """
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    rows = np.arange(N) if rows is None else np.asarray(rows)
+    O = np.zeros((len(rows), V.shape[1]))
+    LSE = np.zeros(len(rows))
+    for r, i in enumerate(rows):
+        i = int(i)
+        c = historical_count(i, b)
+        bias = np.zeros(i + 1)
+        if c:
+            hist = np.asarray(s[i][:c], dtype=np.float64)
+            top = hist.max()
+            lse = top + math.log(np.exp(hist - top).sum())
+            bias[:c * b] = np.repeat(hist - lse, b)
+        z = sm_scale * (K[:i + 1] @ Q[i]) + bias
+        zmax = z.max()
+        w = np.exp(z - zmax)
+        O[r] = (w @ V[:i + 1]) / w.sum()
+        LSE[r] = zmax + math.log(w.sum())
+    return {"O": O, "LSE": LSE}
+
+
+def noisy_scores(s, noise):
+    """full* (Table 1 setting 11): noise is added to the selector scores before
+    the gate activation, so both the Top-K choice and the gates use
+    s~ = s + eps (Sec. 4.2: a stochastic approximation of the full scope).
+    Reading: scores and noise are fp32 tensors and their sum is formed in fp32."""
+    return (np.asarray(s, dtype=np.float32) + np.asarray(noise, dtype=np.float32)).astype(np.float64)
 
 
 # -------------------------------------------------------------------- a6 --

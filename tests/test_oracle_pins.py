@@ -361,3 +361,66 @@ def test_ablation_forms_match_materialized_matrix():
             mat = O.sas_attention_materialized(Q, K, V, s, 64, 2, act=act, pos=pos)
             assert np.allclose(row["O"], mat["O"], atol=1e-12)
             assert np.allclose(row["LSE"], mat["LSE"], atol=1e-12)
+
+
+# ---------------------------------------------- training scopes (Sec. 4.2, Table 1)
+
+@pytest.mark.parametrize("N,b", [(200, 16), (130, 64)])
+def test_full_scope_equals_keep_all_sparse_and_materialised(N, b):
+    # Full scope is the sparse oracle with every historical block kept (K >= C_i)
+    # and the brute-force matrix with K = C: three separate code paths.
+    rng = np.random.default_rng(7)
+    d = 16
+    Q, K, V = (O.round_to_bf16(rng.standard_normal((N, d))) for _ in range(3))
+    s = rng.standard_normal((N, -(-N // b)))
+    full = O.sas_attention_full_scope(Q, K, V, s, b)
+    C = -(-N // b)
+    keep_all = O.sas_attention_head(Q, K, V, s, b, C)
+    mat = O.sas_attention_materialized(Q, K, V, s, b, C)
+    assert np.allclose(full["O"], keep_all["O"], atol=1e-12)
+    assert np.allclose(full["LSE"], keep_all["LSE"], atol=1e-12)
+    assert np.allclose(full["O"], mat["O"], atol=1e-12)
+
+
+def test_full_scope_constant_scores_is_biased_dense_sdpa():
+    # constant scores: log g = -log C_i on every historical key, 0 on the causal
+    # current block -> torch SDPA with that additive mask
+    N, b, d = 192, 32, 16
+    rng = np.random.default_rng(8)
+    Q, K, V = (O.round_to_bf16(rng.standard_normal((N, d))) for _ in range(3))
+    s = np.full((N, N // b), 0.7)
+    full = O.sas_attention_full_scope(Q, K, V, s, b)
+    mask = np.full((N, N), -np.inf)
+    for i in range(N):
+        c = i // b
+        if c:
+            mask[i, :c * b] = -math.log(c)
+        mask[i, c * b:i + 1] = 0.0
+    ref = F.scaled_dot_product_attention(torch.tensor(Q)[None], torch.tensor(K)[None], torch.tensor(V)[None],
+                                         attn_mask=torch.tensor(mask)[None])[0].numpy()
+    assert np.allclose(full["O"], ref, atol=1e-10)
+
+
+def test_noisy_scores_zero_noise_and_shift():
+    # full* with zero noise is the sparse form; a constant noise only shifts s,
+    # which changes neither the kept set nor log g (Eq. normalized_log_gate)
+    rng = np.random.default_rng(9)
+    N, b, d, K = 150, 16, 8, 3
+    Q, Kk, V = (O.round_to_bf16(rng.standard_normal((N, d))) for _ in range(3))
+    s = rng.standard_normal((N, -(-N // b))).astype(np.float32).astype(np.float64)
+    base = O.sas_attention_head(Q, Kk, V, s, b, K)
+    zero = O.sas_attention_head(Q, Kk, V, O.noisy_scores(s, np.zeros_like(s)), b, K)
+    assert np.array_equal(base["sel_idx"], zero["sel_idx"]) and np.allclose(base["O"], zero["O"], atol=0)
+    shifted = O.sas_attention_head(Q, Kk, V, O.noisy_scores(s, np.full_like(s, 0.25)), b, K)
+    assert np.array_equal(base["sel_idx"], shifted["sel_idx"])
+    assert np.allclose(base["O"], shifted["O"], atol=1e-6)
+
+
+def test_noisy_scores_flip_the_selection():
+    # hand example, K = 1: s = (1.0, 1.5) keeps block 1; noise (+1, 0) makes
+    # s~ = (2.0, 1.5), which keeps block 0 with log g = 2 - log(e^2 + e^1.5)
+    s = np.array([[1.0, 1.5]])
+    sn = O.noisy_scores(s, np.array([[1.0, 0.0]]))
+    assert O.topk_blocks(s[0], 1).tolist() == [1] and O.topk_blocks(sn[0], 1).tolist() == [0]
+    lg = O.log_gates(sn[0])
+    assert abs(lg[0] - (2.0 - math.log(math.exp(2.0) + math.exp(1.5)))) < 1e-12
