@@ -83,6 +83,21 @@ typedef enum { SAS_GATE_SOFTMAX = 0, SAS_GATE_SIGMOID = 1, SAS_GATE_LOGIT = 2 } 
  *           LSE is then that of the plain logits. */
 typedef enum { SAS_GATE_INNER = 0, SAS_GATE_OUTER = 1 } sas_gate_pos;
 
+/* Training scope (Sec. 4.2 "training scope"; Table 1 settings 9-11):
+ *   SPARSE : only the Top-K historical blocks enter the attention (the SAS
+ *            form, Eq. spa with the gates of Eq. ours_train).
+ *   FULL   : no Top-K: every historical block of a row enters with its
+ *            log-gate, softmax(q K^T + log g) V over the row's whole history
+ *            (Eq. fula with the gates, setting 9).  Needs the softmax gate in
+ *            the inner position and [B, H, N, d] inputs (max_seqs = 0); topk
+ *            is not used; sel_idx / sel_logg must be NULL; no backward.
+ *            With the learned selector the handle keeps a [B, Hkv, N, C]
+ *            fp32 score table (the dense gate table the paper's kernel
+ *            reads, App. E); with given scores the caller's table is read.
+ * The stochastic approximation of the full scope (full*, setting 11) is the
+ * sparse scope with noise added to the scores: sas_attention_fwd_noisy. */
+typedef enum { SAS_SCOPE_SPARSE = 0, SAS_SCOPE_FULL = 1 } sas_scope;
+
 typedef struct {
     int32_t B, H, N, d;   /* batch, heads, tokens (N <= 2^30), head dim (d in {64, 128}) */
     int32_t block;        /* block size b; must be 64 (Sec. 4.2.1 setup)             */
@@ -106,6 +121,7 @@ typedef struct {
                              and SCORES_GIVEN, has no backward.                        */
     int32_t max_seqlen;   /* packed mode: longest sequence (1 .. N; 0 selects N); the
                              score table has C = ceil(max_seqlen / 64) columns         */
+    int32_t scope;        /* sas_scope (0 = SPARSE, the SAS default)                   */
 } sas_config;
 
 typedef struct sas_handle sas_handle;
@@ -155,6 +171,25 @@ sas_status sas_attention_fwd(sas_handle* h,
                              void* O, float* LSE,
                              int32_t* sel_idx, float* sel_logg,
                              void* stream);
+
+/* full* training scope (Table 1 setting 11; Sec. 4.2: "a stochastic
+ * approximation to full scope by adding noise to the scores before
+ * activation"): sas_attention_fwd with s~ = s + noise in place of the scores
+ * s, for the gate activation and for the Top-K alike.  The sum is formed in
+ * fp32: s~ = fp32(s + noise) with s the given score or, for the learned
+ * selector, fp32(q~ . K~ / sqrt(d_sel)).
+ *   noise  fp32 [B, Hkv, N, C], C = ceil(N / 64), the same layout as given
+ *          scores (entries m >= floor(i/64) are not read); finite.  DEVICE.
+ * Sparse-scope handles of [B, H, N, d] inputs only; other arguments as in
+ * sas_attention_fwd.  sel_logg reports log g of the noisy scores. */
+sas_status sas_attention_fwd_noisy(sas_handle* h,
+                                   const void* Q, const void* K, const void* V,
+                                   const float* scores,
+                                   const void* Wq, const void* Wk,
+                                   const float* noise,
+                                   void* O, float* LSE,
+                                   int32_t* sel_idx, float* sel_logg,
+                                   void* stream);
 
 /* Backward of sas_attention_fwd (Alg. 4 of App. E; gate and score gradients
  * of App. D), for d = 128, softmax gates in the inner position, either mode.

@@ -79,6 +79,14 @@ struct SelectArgs {
     // length, 0}; N is then the token capacity of each head.  Null otherwise.
     const int4* tiles;
     const int* ntiles;
+    // full training scope: no Top-K; each row's log-sum-exp of its scores into
+    // full_lse [BH][N] and, with the learned selector, its scores into
+    // full_table [BH][N][C] (entries m < C_i).  Null in the sparse scope.
+    float* full_lse;
+    float* full_table;
+    // full*: a noise table [BH][N][C] added to the scores before the gate and
+    // the Top-K (null otherwise)
+    const float* noise;
 };
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err);
 // Builds the tile table of packed sequences cu[0..S] (device offsets) with
@@ -105,6 +113,10 @@ struct AttnArgs {
     int gate_pos;               // 0 inner (+ log g in the logits), 1 outer (g scales P after the softmax)
     float sm_scale;
     int* sched;                 // 16 zeroed bytes owned by the caller, left zeroed after each launch
+    // full training scope: every historical block of a row kept with
+    // log g_m = full_table[row][m] - full_lse[row] (tables per KV group); null otherwise
+    const float* full_table;
+    const float* full_lse;
 };
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err);
 

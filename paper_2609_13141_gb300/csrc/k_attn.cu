@@ -99,6 +99,8 @@ struct AttnParams {
     const int4* tiles;      // packed sequences: {first row, tile in sequence, length} per slot (else null)
     const int* ntiles;      // slots in use (device)
     int* sched;             // [0] next work item, [1] CTAs finished; both zero between launches
+    const float* full_table;   // full training scope: scores [BHkv][N][C] and normalisers [BHkv][N]
+    const float* full_lse;
     float scale_log2;
     int* status;
     long long limit;
@@ -146,7 +148,8 @@ __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w, int T) {
     x.kv = x.bh / p.G;
     const long long tb = static_cast<long long>(x.kv) * p.T + slot;
     x.ulist = p.union_idx + tb * p.C;
-    x.U = __ldg(p.union_cnt + tb);
+    // full scope: every historical block of the tile (blocks 0 .. 2t-1, all full)
+    x.U = p.full_table != nullptr ? 2 * x.t : __ldg(p.union_cnt + tb);
     return x;
 }
 
@@ -164,14 +167,18 @@ __device__ __forceinline__ int tile_blocks(const AttnParams& p, const TileRef& x
     return x.U + ((2 * x.t + 1) * kBN < x.n ? 2 : 1);
 }
 
+template <bool FULL>
 __device__ __forceinline__ int block_at(const TileRef& x, int j) {
-    return j < x.U ? __ldg(x.ulist + j) : 2 * x.t + (j - x.U);
+    return j < x.U ? (FULL ? j : __ldg(x.ulist + j)) : 2 * x.t + (j - x.U);
 }
 
 // OUTER: the gate of a kept block multiplies its probabilities after the
 // softmax (gate position "outer" of Sec. 4.2) instead of adding log g to its
 // logits; the row sum and LSE then stay those of the ungated logits.
-template <int D, bool OUTER>
+// FULL: the full training scope (Table 1 setting 9): no kept lists, every
+// historical block m of a row enters with log g_m = s_m - LSE of the row's
+// scores, read from a [N][C] score table and a per-row normaliser.
+template <int D, bool OUTER, bool FULL>
 __global__ void __launch_bounds__(kThreads, 2)
 attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
             const __grid_constant__ CUtensorMap mapV, AttnParams p) {
@@ -253,7 +260,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int s = gb % Cfg::KST;
-                const int m = block_at(x, j);
+                const int m = block_at<FULL>(x, j);
                 if (!mbar_wait(&k_empty[s], ((gb / Cfg::KST) & 1) ^ 1u, wc)) { ok = false; break; }
                 uint8_t* dst = smem + Cfg::OFF_K + s * Cfg::KV_BYTES;
                 mbar_arrive_expect_tx(&k_full[s], Cfg::KV_BYTES);
@@ -294,7 +301,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int s = gb % Cfg::VST;
-                const int m = block_at(x, j);
+                const int m = block_at<FULL>(x, j);
                 if (!mbar_wait(&v_empty[s], ((gb / Cfg::VST) & 1) ^ 1u, wc)) { ok = false; break; }
                 uint8_t* dst = smem + Cfg::OFF_V + s * Cfg::KV_BYTES;
                 mbar_arrive_expect_tx(&v_full[s], Cfg::KV_BYTES);
@@ -421,7 +428,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             const int i = t * kBM + r_row;   // row within its sequence
             const bool valid = i < x.n;
             const int c = i >> 6;
-            const int nsel = valid ? min(p.topk, c) : 0;
+            const int nsel = (valid && !FULL) ? min(p.topk, c) : 0;
             const long long row_off = static_cast<long long>(x.bh) * p.N + x.base + i;   // O, LSE
             const long long sel_off = static_cast<long long>(x.kv) * p.N + x.base + i;   // the group's kept list
             const int32_t* my_idx = p.sel_idx + sel_off * p.topk;
@@ -453,17 +460,39 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             float l = 0.f;
             // raw list entry for the next iteration (entries past the union are the diagonal blocks)
             int raw_next = 0;
-            if (x.U > 0) raw_next = __ldg(x.ulist);
+            if (!FULL && x.U > 0) raw_next = __ldg(x.ulist);
+            // full scope: the row's score of the next historical block, loaded one block ahead
+            const float* tbl = nullptr;
+            float lse_row = 0.f, t_next = 0.f;
+            if constexpr (FULL) {
+                tbl = p.full_table + sel_off * p.C;
+                if (valid) lse_row = __ldg(p.full_lse + sel_off);
+                if (valid && c > 0 && n > 0) t_next = __ldg(tbl);   // the first visited block is 0
+            }
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int pb = gb & 1;
-                const int m = j < x.U ? raw_next : 2 * t + (j - x.U);
-                if (j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
+                const int m = FULL ? block_at<true>(x, j) : (j < x.U ? raw_next : 2 * t + (j - x.U));
+                if (!FULL && j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
                 // gate (log2 units) and the last visible key column of block m for this row
                 float bias = 0.f;
                 float gsc = 1.f;   // outer position: gate applied to the probabilities
                 int lim;
-                if (m < c) {
+                if constexpr (FULL) {
+                    const float t_cur = t_next;
+                    if (j + 1 < n) {
+                        const int m1 = block_at<true>(x, j + 1);
+                        t_next = (valid && m1 < c) ? __ldg(tbl + m1) : 0.f;
+                    }
+                    if (m < c) {
+                        bias = train ? (t_cur - lse_row) * kLog2e : 0.f;
+                        lim = kBN - 1;
+                    } else if (m == c) {
+                        lim = i & (kBN - 1);
+                    } else {
+                        lim = -1;
+                    }
+                } else if (m < c) {
                     if (m == km0) {
                         if constexpr (OUTER) gsc = train ? fast_exp2(kl0 * kLog2e) : 1.f;
                         else bias = train ? kl0 * kLog2e : 0.f;
@@ -638,11 +667,11 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     }
 }
 
-template <int D, bool OUTER>
+template <int D, bool OUTER, bool FULL>
 cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) {
     using Cfg = AttnCfg<D>;
     {
-        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(attn_kernel<D, OUTER>), Cfg::SMEM);
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(attn_kernel<D, OUTER, FULL>), Cfg::SMEM);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(attn)"; return e; }
     }
     int dev = 0, sms = 0, l2 = 0;
@@ -676,10 +705,12 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.status = env.status;
     p.limit = env.limit;
     p.sched = a.sched;
+    p.full_table = a.full_table;
+    p.full_lse = a.full_lse;
     // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
     const long long items = static_cast<long long>(a.T) * a.BH;
     const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);
-    attn_kernel<D, OUTER><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
+    attn_kernel<D, OUTER, FULL><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "attention launch";
     return e;
@@ -693,8 +724,16 @@ cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** er
         return cudaErrorInvalidValue;
     }
     const bool outer = a.gate_pos == 1;
-    if (a.d == 128) return outer ? launch_d<128, true>(a, env, err) : launch_d<128, false>(a, env, err);
-    if (a.d == 64) return outer ? launch_d<64, true>(a, env, err) : launch_d<64, false>(a, env, err);
+    if (a.full_table != nullptr) {
+        if (outer || a.tiles != nullptr || a.full_lse == nullptr) {
+            *err = "attention: the full scope takes the inner gate position and [B, H, N] inputs";
+            return cudaErrorInvalidValue;
+        }
+        if (a.d == 128) return launch_d<128, false, true>(a, env, err);
+        if (a.d == 64) return launch_d<64, false, true>(a, env, err);
+    }
+    if (a.d == 128) return outer ? launch_d<128, true, false>(a, env, err) : launch_d<128, false, false>(a, env, err);
+    if (a.d == 64) return outer ? launch_d<64, true, false>(a, env, err) : launch_d<64, false, false>(a, env, err);
     *err = "attention: unsupported head dim";
     return cudaErrorInvalidValue;
 }

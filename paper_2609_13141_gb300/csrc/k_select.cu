@@ -56,6 +56,9 @@ struct SelParams {
     const int* ntiles;            // their number (device); both null for [B, H, N] inputs
     int* status;
     long long limit;
+    float* full_lse;              // full training scope (see SelectArgs)
+    float* full_table;
+    const float* noise;           // full*: added to every score before gate and Top-K
 };
 
 // Where a CTA's 128-row tile lies: its union-list slot, its tile index within
@@ -471,13 +474,18 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     const int last = min(row0 + 31, geo.n - 1);
     const int Cw = row0 < geo.n ? (last >> 6) : 0;   // largest C_i among the warp's rows
     const float* sbase = p.scores + (static_cast<long long>(bh) * p.N + geo.base) * p.C;
+    const float* nbase = p.noise == nullptr ? nullptr : p.noise + (static_cast<long long>(bh) * p.N + geo.base) * p.C;
     for (int c = 0; 32 * c < Cw; ++c) {
         const int m = 32 * c + lane;
 #pragma unroll 4
         for (int rho = 0; rho < 32; ++rho) {
             const int row = row0 + rho;
             float v = 0.f;
-            if (row < geo.n && m < p.C) v = __ldg(sbase + static_cast<long long>(row) * p.C + m);
+            if (row < geo.n && m < p.C) {
+                const long long o = static_cast<long long>(row) * p.C + m;
+                v = __ldg(sbase + o);
+                if (nbase != nullptr) v = __fadd_rn(v, __ldg(nbase + o));   // full*: s~ = s + eps in fp32
+            }
             stage[warp][lane][rho] = v;
         }
         __syncwarp();
@@ -551,6 +559,7 @@ constexpr int kBinWords = kBins / 2;                // two 16-bit counters per w
 constexpr int kBoundaryMax = kBinWords / 2;         // boundary-bin scores a row holds (in its dead histogram words)
 constexpr size_t kHistBytes = size_t(kBinWords) * kRows * 4;
 constexpr int kPassA = 0, kPassB = 1, kPassC = 2, kPassD = 3;
+constexpr int kPassW = 4;   // full training scope: write every score to the table
 constexpr int kRowAll = 0, kRowNormal = 1, kRowFail = 2;   // C_i <= K: keep all; thresholds; fallback
 
 template <int D, int DS>
@@ -872,14 +881,18 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     const int t = tile_of_block(p.T, p.BH);
     const int bh = head_of_block(p.BH);
     const int diag = 2 * t;
+    // full training scope: no Top-K, the scores and their log-sum-exp are written out
+    const bool full = p.full_lse != nullptr;
+    // full*: noise added to the scores before the gate and the Top-K
+    const bool noisy = p.noise != nullptr;
     const int nb = min(2 * t + 1, p.F);          // blocks scored for this tile
-    const int nchunks = K > 0 ? (nb + 63) >> 6 : 0;
+    const int nchunks = (K > 0 || full) ? (nb + 63) >> 6 : 0;
     // the most blocks any row of the tile has: a histogram pass only when it exceeds K
     const int last_row = min(p.N, (t + 1) * kRows) - 1;
     const int tile_ci = last_row >= t * kRows ? (last_row >> 6) : 0;
-    const bool pass_b = tile_ci > K;
+    const bool pass_b = !full && tile_ci > K;
     // passes over the chunks, in order; D runs only if a row fails (decided after B)
-    const int npre = nchunks > 0 ? (pass_b ? 3 : 2) : 0;   // A, [B], C
+    const int npre = nchunks > 0 ? (full || !pass_b ? 2 : 3) : 0;   // A, [B], C  or  A, W
     // a history of at most two chunks stays in the two TMEM score buffers: its
     // products are computed once and every pass reads them again
     const bool resident = nchunks <= 2;
@@ -1056,7 +1069,11 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         row_set_all(rs);
         rs.nabove = 0; rs.pos = 0; rs.nbc = 0;
         rs.ws = -CUDART_INF_F; rs.wpos = 0;
-        const float c_exp = p.score_scale * kLog2e;
+        // the products u are selected on directly (s = u scale); with noise the
+        // pass works on s~ = s + eps itself
+        const float c_exp = noisy ? kLog2e : p.score_scale * kLog2e;
+        const float emit_scale = noisy ? 1.f : p.score_scale;
+        const long long row_off = static_cast<long long>(bh) * p.N + i;
         const uint32_t hist_r = smem_u32(hist + r);
         const RowAddr ra{smem_u32(st.idx + r * st.stride), smem_u32(st.lg + r * st.stride), hist_r};
         int gc = 0;
@@ -1067,6 +1084,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 if (!mbar_wait_warp(&plan_bar, 0, wc)) { ok = false; break; }
                 if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
                 kind = kPassD;
+            } else if (full) {
+                kind = ps == 0 ? kPassA : kPassW;
             } else {
                 kind = ps == 0 ? kPassA : (ps == npre - 1 ? kPassC : kPassB);
             }
@@ -1088,14 +1107,29 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     }
                     const int m0 = 64 * c + 32 * half;
                     const int lim = Ci - m0;
-                    // the vote comes before any lane leaves; the lanes meet again
-                    // before the next warp-collective TMEM load
-                    const bool full = __all_sync(0xffffffffu, lim >= 32);
+                    if (noisy) {
+                        const float* nrow = p.noise + row_off * p.C + m0;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (j < lim)
+                                uu[j] = __float_as_uint(
+                                    __fadd_rn(__fmul_rn(__uint_as_float(uu[j]), p.score_scale), __ldg(nrow + j)));
+                    }
                     const float* u = reinterpret_cast<const float*>(uu);
-                    if (full)
-                        row_pass<true>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
-                    else if (lim > 0)
-                        row_pass<false>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    if (kind == kPassW) {
+                        float* dst = p.full_table + row_off * p.C + m0;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (j < lim) dst[j] = __fmul_rn(u[j], p.score_scale);
+                    } else {
+                        // the vote comes before any lane leaves; the lanes meet again
+                        // before the next warp-collective TMEM load
+                        const bool whole = __all_sync(0xffffffffu, lim >= 32);
+                        if (whole)
+                            row_pass<true>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                        else if (lim > 0)
+                            row_pass<false>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    }
                     __syncwarp();
                 }
             }
@@ -1116,13 +1150,16 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             }
         }
         ok = ok && !abort_flag;
-        if (valid && ok) {
+        if (full) {
+            // full scope: the row's log-sum-exp of its scores (the table is written)
+            if (valid && ok) p.full_lse[row_off] = Ci > 0 ? __fmul_rn(rs.l.mx, p.score_scale) + logf(rs.l.sum) : 0.f;
+        } else if (valid && ok) {
             // log-gates from s = u / sqrt(d_sel), -1 padding, tile-union bits
-            const float lse = Ci > 0 ? __fmul_rn(rs.l.mx, p.score_scale) + logf(rs.l.sum) : 0.f;
+            const float lse = Ci > 0 ? __fmul_rn(rs.l.mx, emit_scale) + logf(rs.l.sum) : 0.f;
             for (int e = 0; e < K; ++e) {
                 if (e < Kp) {
                     const int m = st.idx[r * st.stride + e];
-                    const float sc = __fmul_rn(st.lg[r * st.stride + e], p.score_scale);
+                    const float sc = __fmul_rn(st.lg[r * st.stride + e], emit_scale);
                     st.lg[r * st.stride + e] = staged_gate(sc, lse, p.gate_act);
                     if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
                 } else {
@@ -1131,13 +1168,15 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 }
             }
         }
-        named_bar_sync(1, 128);
-        if (ok)
-            copy_out(st, p, bh, static_cast<long long>(t) * kRows, min(kRows, p.N - t * kRows),
-                     static_cast<int>(threadIdx.x) - 64, 128);
-        if (warp == 2)
-            compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
-                          p.union_cnt + static_cast<long long>(bh) * p.T + t);
+        if (!full) {
+            named_bar_sync(1, 128);
+            if (ok)
+                copy_out(st, p, bh, static_cast<long long>(t) * kRows, min(kRows, p.N - t * kRows),
+                         static_cast<int>(threadIdx.x) - 64, 128);
+            if (warp == 2)
+                compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
+                              p.union_cnt + static_cast<long long>(bh) * p.T + t);
+        }
     }
     __syncthreads();
     if (warp == 1) {
@@ -1177,6 +1216,28 @@ cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEn
     return e;
 }
 
+
+// Full training scope with given scores: each row's log-sum-exp over its C_i
+// scores (Eq. normalized_log_gate's normaliser), one warp per row, reading the
+// row twice (maximum, then the sum; the second read hits the cache).
+__global__ void __launch_bounds__(256) row_lse_kernel(const float* scores, int N, int C, long long rows,
+                                                      float* out) {
+    const long long w = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= rows) return;
+    const int i = static_cast<int>(w % N);
+    const int Ci = i >> 6;
+    const float* s = scores + w * C;
+    float mx = -CUDART_INF_F;
+    for (int m = lane; m < Ci; m += 32) mx = fmaxf(mx, __ldg(s + m));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float sum = 0.f;
+    for (int m = lane; m < Ci; m += 32) sum += fast_exp2((__ldg(s + m) - mx) * kLog2e);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) out[w] = Ci > 0 ? mx + logf(sum) : 0.f;
+}
 
 constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
 
@@ -1259,6 +1320,20 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     p.union_idx = a.union_idx; p.union_cnt = a.union_cnt;
     p.tiles = a.tiles; p.ntiles = a.ntiles;
     p.status = env.status; p.limit = env.limit;
+    p.full_lse = a.full_lse; p.full_table = a.full_table; p.noise = a.noise;
+    if (a.full_lse != nullptr && (a.tiles != nullptr || a.noise != nullptr)) {
+        *err = "selection: the full scope takes neither packed sequences nor noise";
+        return cudaErrorInvalidValue;
+    }
+    if (a.full_lse != nullptr && a.scores != nullptr) {
+        // given scores: the attention kernel reads them directly; only the normalisers
+        const long long rows = static_cast<long long>(a.BH) * a.N;
+        const long long blocks = (rows * 32 + 255) / 256;
+        row_lse_kernel<<<static_cast<unsigned>(blocks), 256, 0, env.stream>>>(a.scores, a.N, a.C, rows, a.full_lse);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) *err = "row log-sum-exp launch";
+        return e;
+    }
     if (a.tiles != nullptr && a.scores == nullptr) {
         *err = "selection: packed sequences need given scores";
         return cudaErrorInvalidValue;

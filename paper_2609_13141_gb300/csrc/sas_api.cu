@@ -136,6 +136,9 @@ struct sas_handle {
     float* sel_logg = nullptr;
     int* status = nullptr;
     int* sched = nullptr;       // attention work counters (zero between launches)
+    bool full = false;          // full training scope
+    float* full_lse = nullptr;  // [BHkv][N] row normalisers of the scores
+    float* full_table = nullptr;   // learned selector, full scope: scores [BHkv][N][C]
     // MLP hidden activation
     void* hidden = nullptr;
     size_t hidden_bytes = 0;
@@ -255,6 +258,10 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
         return SAS_ERR_INVALID_ARG;
     if (c.gate_pos != SAS_GATE_INNER && c.gate_pos != SAS_GATE_OUTER) return SAS_ERR_INVALID_ARG;
     if (!(c.sm_scale >= 0.f) || !std::isfinite(c.sm_scale)) return SAS_ERR_INVALID_ARG;
+    if (c.scope != SAS_SCOPE_SPARSE && c.scope != SAS_SCOPE_FULL) return SAS_ERR_INVALID_ARG;
+    if (c.scope == SAS_SCOPE_FULL &&
+        (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER || c.max_seqs > 0))
+        return SAS_ERR_UNSUPPORTED;
     const int d_sel = c.d_sel == 0 ? c.d : c.d_sel;
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
     const int Hkv = c.Hkv == 0 ? c.H : c.Hkv;
@@ -278,6 +285,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     h->G = c.H / Hkv;
     h->BHkv = static_cast<int>(BHkv);
     h->varlen = varlen;
+    h->full = c.scope == SAS_SCOPE_FULL;
     const int max_len = varlen && c.max_seqlen > 0 ? c.max_seqlen : c.N;
     h->C = (max_len + 63) / 64;
     // packed sequences: at most N / 128 + max_seqs tiles (each sequence adds one partial tile)
@@ -300,6 +308,11 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
         if (e == cudaSuccess) e = alloc(&h->tiles, static_cast<size_t>(h->T) * sizeof(int4));
         if (e == cudaSuccess) e = alloc(&h->ntiles, 16);
         if (e == cudaSuccess) e = cudaMemset(h->ntiles, 0, 16);
+    }
+    if (h->full) {
+        if (e == cudaSuccess) e = alloc(&h->full_lse, rows * 4);
+        if (e == cudaSuccess && c.selector == SAS_SEL_MEANPOOL_PROJ)
+            e = alloc(&h->full_table, rows * static_cast<size_t>(h->C) * 4);
     }
     if (e == cudaSuccess) e = alloc(&h->status, 16);
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, 16);
@@ -327,6 +340,8 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->ntiles);
     cudaFree(h->status);
     cudaFree(h->sched);
+    cudaFree(h->full_lse);
+    cudaFree(h->full_table);
     cudaFree(h->hidden);
     cudaFree(h->bwd_delta);
     cudaFree(h->bwd_inv);
@@ -337,12 +352,20 @@ void sas_destroy(sas_handle* h) {
     delete h;
 }
 
-sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
-                             const void* Wq, const void* Wk, void* O, float* LSE, int32_t* sel_idx,
-                             float* sel_logg, void* stream) {
+}  // extern "C"
+
+namespace {
+
+sas_status attention_fwd(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
+                         const void* Wq, const void* Wk, const float* noise, void* O, float* LSE, int32_t* sel_idx,
+                         float* sel_logg, void* stream) {
     if (h == nullptr) return SAS_ERR_INVALID_ARG;
     const sas_config& c = h->cfg;
     if (h->varlen) return fail(h, SAS_ERR_INVALID_ARG, "packed-sequence handle: use sas_attention_fwd_varlen");
+    if (noise != nullptr && h->full) return fail(h, SAS_ERR_INVALID_ARG, "noise belongs to the sparse scope (full*)");
+    if (noise != nullptr && !aligned4(noise)) return fail(h, SAS_ERR_INVALID_ARG, "noise must be 4-byte aligned");
+    if (h->full && (sel_idx != nullptr || sel_logg != nullptr))
+        return fail(h, SAS_ERR_INVALID_ARG, "the full scope keeps no Top-K: sel_idx and sel_logg must be NULL");
     if (!Q || !K || !V || !O) return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O are required");
     if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
         return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O must be 16-byte aligned");
@@ -383,6 +406,11 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     sa.Q = Q; sa.Wq = Wq; sa.d = c.d; sa.Kt = h->Kt; sa.F = h->F;
     sa.sel_idx = out_idx; sa.sel_logg = out_lg;
     sa.union_idx = h->union_idx; sa.union_cnt = h->union_cnt;
+    sa.noise = noise;
+    if (h->full) {
+        sa.full_lse = h->full_lse;
+        sa.full_table = h->full_table;
+    }
     e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     // a5: gated sparse attention
@@ -395,9 +423,30 @@ sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const 
     aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
     aa.sched = h->sched;
+    if (h->full) {
+        aa.full_table = c.selector == SAS_SEL_SCORES_GIVEN ? scores : h->full_table;
+        aa.full_lse = h->full_lse;
+    }
     e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     return SAS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+sas_status sas_attention_fwd(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
+                             const void* Wq, const void* Wk, void* O, float* LSE, int32_t* sel_idx,
+                             float* sel_logg, void* stream) {
+    return attention_fwd(h, Q, K, V, scores, Wq, Wk, nullptr, O, LSE, sel_idx, sel_logg, stream);
+}
+
+sas_status sas_attention_fwd_noisy(sas_handle* h, const void* Q, const void* K, const void* V, const float* scores,
+                                   const void* Wq, const void* Wk, const float* noise, void* O, float* LSE,
+                                   int32_t* sel_idx, float* sel_logg, void* stream) {
+    if (h != nullptr && noise == nullptr) return fail(h, SAS_ERR_INVALID_ARG, "noise is required");
+    return attention_fwd(h, Q, K, V, scores, Wq, Wk, noise, O, LSE, sel_idx, sel_logg, stream);
 }
 
 sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, int32_t num_seqs, const void* Q,
@@ -520,6 +569,7 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
     if (h->G != 1) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports Hkv = H");
     if (h->varlen) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports [B, H, N, d] batches");
+    if (h->full) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports the sparse scope");
     if (h->T > sas::kBwdMaxTiles) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports N <= 262016");
     if (dscores) {
         if (c.selector != SAS_SEL_SCORES_GIVEN || !scores)

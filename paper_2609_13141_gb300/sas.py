@@ -32,6 +32,8 @@ SAS_GATE_SIGMOID = 1
 SAS_GATE_LOGIT = 2
 SAS_GATE_INNER = 0
 SAS_GATE_OUTER = 1
+SAS_SCOPE_SPARSE = 0
+SAS_SCOPE_FULL = 1
 SAS_NUM_KERNEL_KINDS = 7
 KERNEL_KINDS = ["block_summaries", "query_projection", "selection", "attention", "mlp_up_gelu", "mlp_down",
                 "attention_bwd"]
@@ -44,7 +46,7 @@ class SasConfig(ctypes.Structure):
                 ("block", ctypes.c_int32), ("topk", ctypes.c_int32), ("sm_scale", ctypes.c_float),
                 ("mode", ctypes.c_int32), ("selector", ctypes.c_int32), ("d_sel", ctypes.c_int32),
                 ("gate_act", ctypes.c_int32), ("gate_pos", ctypes.c_int32), ("Hkv", ctypes.c_int32),
-                ("max_seqs", ctypes.c_int32), ("max_seqlen", ctypes.c_int32)]
+                ("max_seqs", ctypes.c_int32), ("max_seqlen", ctypes.c_int32), ("scope", ctypes.c_int32)]
 
 
 class SasDecodeConfig(ctypes.Structure):
@@ -82,6 +84,8 @@ def lib():
     L.sas_destroy.restype = None
     L.sas_attention_fwd.argtypes = [vp] * 12
     L.sas_attention_fwd.restype = i32
+    L.sas_attention_fwd_noisy.argtypes = [vp] * 13
+    L.sas_attention_fwd_noisy.restype = i32
     L.sas_attention_fwd_varlen.argtypes = [vp, vp, i32] + [vp] * 9
     L.sas_attention_fwd_varlen.restype = i32
     L.sas_attention_bwd.argtypes = [vp] * 16
@@ -174,19 +178,20 @@ def sas_status_str(status):
 
 def sas_create(B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
                sm_scale=0.0, block=64, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0,
-               max_seqlen=0):
+               max_seqlen=0, scope=SAS_SCOPE_SPARSE):
     cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv, max_seqs,
-                    max_seqlen)
+                    max_seqlen, scope)
     h = ctypes.c_void_p()
     _check(lib().sas_create(ctypes.byref(cfg), ctypes.byref(h)), None, "sas_create")
     return h
 
 
 def sas_create_status(B, H, N, d, topk, mode=0, selector=0, d_sel=0, sm_scale=0.0, block=64,
-                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0):
+                      gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0,
+                      scope=SAS_SCOPE_SPARSE):
     """Raw status of sas_create (for argument-check tests); destroys the handle on success."""
     cfg = SasConfig(B, H, N, d, block, topk, sm_scale, mode, selector, d_sel, gate_act, gate_pos, Hkv, max_seqs,
-                    max_seqlen)
+                    max_seqlen, scope)
     h = ctypes.c_void_p()
     st = lib().sas_create(ctypes.byref(cfg), ctypes.byref(h))
     if st == SAS_OK:
@@ -218,6 +223,18 @@ def sas_attention_fwd(h, Q, K, V, O, scores=None, Wq=None, Wk=None, LSE=None, se
         _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False), _ptr(sel_idx, torch.int32, "sel_idx", False),
         _ptr(sel_logg, torch.float32, "sel_logg", False), _stream(stream))
     _check(st, h, "sas_attention_fwd")
+
+
+def sas_attention_fwd_noisy(h, Q, K, V, O, noise, scores=None, Wq=None, Wk=None, LSE=None, sel_idx=None,
+                            sel_logg=None, stream=None):
+    bf = torch.bfloat16
+    st = lib().sas_attention_fwd_noisy(
+        h, _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"),
+        _ptr(scores, torch.float32, "scores", False), _ptr(Wq, bf, "Wq", False), _ptr(Wk, bf, "Wk", False),
+        _ptr(noise, torch.float32, "noise"), _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False),
+        _ptr(sel_idx, torch.int32, "sel_idx", False), _ptr(sel_logg, torch.float32, "sel_logg", False),
+        _stream(stream))
+    _check(st, h, "sas_attention_fwd_noisy")
 
 
 def sas_attention_bwd(h, Q, K, V, O, LSE, dO, dQ, dK, dV, scores=None, sel_idx=None, sel_logg=None, dlogg=None,
@@ -306,12 +323,14 @@ class SasLayer:
     """Owns one handle; allocates outputs and calls the C ABI."""
 
     def __init__(self, B, H, N, d, topk, mode=SAS_MODE_TRAIN_SOFT, selector=SAS_SEL_SCORES_GIVEN, d_sel=0,
-                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0):
+                 sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0,
+                 scope=SAS_SCOPE_SPARSE):
         self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
         self.Hkv = Hkv or H                      # kept lists are per KV group
         self.selector = selector
+        self.scope = scope
         self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv,
-                            max_seqs, max_seqlen)
+                            max_seqs, max_seqlen, scope)
 
     def attention_varlen(self, cu_seqlens, Q, K, V, scores, want_sel=True, stream=None, sel_fill=-1):
         """Packed sequences (handle made with max_seqs > 0): Q [H, N, d], K/V [Hkv, N, d],
@@ -329,16 +348,27 @@ class SasLayer:
         sas_attention_fwd_varlen(self.h, cu_seqlens, Q, K, V, scores, O, LSE, sel_idx, sel_logg, stream)
         return O, LSE, sel_idx, sel_logg
 
-    def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
+    def _outputs(self, Q, want_sel):
         dev = Q.device
         O = torch.empty_like(Q)
         LSE = torch.empty(self.B, self.H, self.N, device=dev, dtype=torch.float32)
         sel_idx = sel_logg = None
-        if want_sel:
+        if want_sel and self.scope == SAS_SCOPE_SPARSE:
             k = max(self.topk, 1)
             sel_idx = torch.empty(self.B, self.Hkv, self.N, k, device=dev, dtype=torch.int32)
             sel_logg = torch.empty(self.B, self.Hkv, self.N, k, device=dev, dtype=torch.float32)
+        return O, LSE, sel_idx, sel_logg
+
+    def attention(self, Q, K, V, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
+        """Returns (O, LSE, sel_idx, sel_logg); the full scope keeps no Top-K (sel_* None)."""
+        O, LSE, sel_idx, sel_logg = self._outputs(Q, want_sel)
         sas_attention_fwd(self.h, Q, K, V, O, scores, Wq, Wk, LSE, sel_idx, sel_logg, stream)
+        return O, LSE, sel_idx, sel_logg
+
+    def attention_noisy(self, Q, K, V, noise, scores=None, Wq=None, Wk=None, want_sel=True, stream=None):
+        """full*: the scores plus `noise` (fp32, the layout of given scores) choose and gate the blocks."""
+        O, LSE, sel_idx, sel_logg = self._outputs(Q, want_sel)
+        sas_attention_fwd_noisy(self.h, Q, K, V, O, noise, scores, Wq, Wk, LSE, sel_idx, sel_logg, stream)
         return O, LSE, sel_idx, sel_logg
 
     def attention_bwd(self, Q, K, V, O, LSE, dO, scores=None, sel_idx=None, sel_logg=None, want_ds=False,

@@ -56,6 +56,10 @@ def test_status_strings(lib):
     (dict(B=2, H=2, N=128, d=64, topk=2, max_seqs=4), sas.SAS_ERR_INVALID_ARG),          # packed needs B = 1
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=4, selector=1), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=4, max_seqlen=129), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=2, N=128, d=64, topk=2, scope=2), sas.SAS_ERR_INVALID_ARG),
+    (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, gate_pos=1), sas.SAS_ERR_UNSUPPORTED),   # full scope: inner only
+    (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, gate_act=1), sas.SAS_ERR_UNSUPPORTED),   # full scope: softmax only
+    (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, max_seqs=2), sas.SAS_ERR_UNSUPPORTED),   # full scope: no packing
 ])
 def test_create_rejects_bad_configs(lib, kw, expect):
     assert sas.sas_create_status(**kw) == expect
@@ -70,6 +74,7 @@ def test_create_without_gpu_fails_cleanly(lib):
 def test_null_handle_and_null_arguments(lib):
     null = ctypes.c_void_p()
     assert lib.sas_attention_fwd(null, *([None] * 10), None) == sas.SAS_ERR_INVALID_ARG
+    assert lib.sas_attention_fwd_noisy(null, *([None] * 11), None) == sas.SAS_ERR_INVALID_ARG
     assert lib.sas_mlp_fwd(null, None, None, None, None, None, None, 1, 64, 64, None) == sas.SAS_ERR_INVALID_ARG
     v = ctypes.c_int32()
     assert lib.sas_get_device_status(null, ctypes.byref(v)) == sas.SAS_ERR_INVALID_ARG
