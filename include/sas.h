@@ -334,6 +334,16 @@ sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, i
 /* Total number of kernels this handle has launched since creation. */
 int64_t sas_launch_count(const sas_handle* h);
 
+/* Failure-path diagnostics: the budget, in SM clock cycles, of every bounded
+ * wait in the main loops of the kernels this handle launches from now on
+ * (0 restores the default of about 2 s).  A budget too short for the work
+ * makes those waits give up: the kernels then record SAS_ERR_TIMEOUT in the
+ * device status word and return early, leaving their outputs incomplete.
+ * The waits that drain a kernel's own copies and tensor-core work before it
+ * exits keep at least the default budget, so nothing is left in flight and
+ * the context stays usable.  Not for production use. */
+sas_status sas_set_wait_limit(sas_handle* h, int64_t cycles);
+
 /* Copies the per-tile count of historical blocks the attention kernel
  * processes (the union of the kept blocks of the tile's 128 query rows,
  * excluding the tile's own two diagonal blocks) from the last forward:

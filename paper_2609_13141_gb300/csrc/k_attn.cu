@@ -650,6 +650,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             tc_fence_before();
             g += n;
         }
+        // a row that stopped early may still have kept-list copies in flight
+        cp_async_wait<0>();
     }
     __syncthreads();
     if (threadIdx.x == 0) {

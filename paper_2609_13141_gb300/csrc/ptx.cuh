@@ -12,6 +12,10 @@
 namespace sas {
 
 constexpr int kStatusTimeout = 4;   // == SAS_ERR_TIMEOUT
+// Budget of the waits that drain a CTA's own copies and tensor-core work before
+// it exits (~2 s of SM clock): never shorter than this, whatever budget the
+// main-loop waits run under, so a CTA that gives up leaves nothing in flight.
+constexpr long long kDrainLimit = 4000000000LL;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -121,9 +125,11 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, c
     return __all_sync(0xffffffffu, ok);
 }
 
-// Wait used only while draining at exit: ignores the abort flag.
+// Wait used only while draining at exit: ignores the abort flag, and waits at
+// least kDrainLimit cycles.
 __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity, long long limit, int* status,
                                                 uint32_t suspend_ns = 0) {
+    if (limit < kDrainLimit) limit = kDrainLimit;
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity, suspend_ns)) {
         if (clock64() - t0 > limit) {

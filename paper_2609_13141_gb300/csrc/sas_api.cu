@@ -691,6 +691,12 @@ sas_status sas_get_timings(sas_handle* h, int64_t* launches, double* total_ms, i
 
 int64_t sas_launch_count(const sas_handle* h) { return h ? h->launches : 0; }
 
+sas_status sas_set_wait_limit(sas_handle* h, int64_t cycles) {
+    if (h == nullptr || cycles < 0) return SAS_ERR_INVALID_ARG;
+    h->limit = cycles == 0 ? kDefaultWaitLimit : cycles;
+    return SAS_OK;
+}
+
 sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n) {
     if (h == nullptr || host_out == nullptr) return SAS_ERR_INVALID_ARG;
     const int64_t total = static_cast<int64_t>(h->BHkv) * h->T;   // one union list per KV group and tile

@@ -104,6 +104,8 @@ def lib():
     L.sas_get_timings.restype = i32
     L.sas_launch_count.argtypes = [vp]
     L.sas_launch_count.restype = i64
+    L.sas_set_wait_limit.argtypes = [vp, i64]
+    L.sas_set_wait_limit.restype = i32
     L.sas_get_tile_union_counts.argtypes = [vp, ctypes.POINTER(i32), i64]
     L.sas_get_tile_union_counts.restype = i32
     L.sas_mlp_fwd_noalloc.argtypes = [vp] * 6 + [i64, i64, i64, vp]
@@ -305,6 +307,11 @@ def sas_get_timings(h):
 
 def sas_launch_count(h):
     return lib().sas_launch_count(h)
+
+
+def sas_set_wait_limit(h, cycles):
+    """Failure-path diagnostics: main-loop wait budget in SM cycles (0: default)."""
+    _check(lib().sas_set_wait_limit(h, int(cycles)), h, "sas_set_wait_limit")
 
 
 def sas_get_tile_union_counts(h, n):

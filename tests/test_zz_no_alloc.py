@@ -44,10 +44,13 @@ def test_noalloc_mlp_matches_regular_entry_point_and_oracle_twice(T, D, F, bias)
     yref = OR.gelu_mlp(f(host[0]), f(host[1]), f(host[2]), f(host[3]), f(host[4]), rows=rows)
     assert sas.sas_mlp_noalloc_get_device_status() == sas.SAS_OK   # clears anything left before
     for _ in range(2):
-        Y = torch.full((T, D), float("nan"), device=dev, dtype=torch.bfloat16)
+        # Y is followed in memory by a NaN guard that the call must leave alone
+        buf = torch.full((T * D + 4096,), float("nan"), device=dev, dtype=torch.bfloat16)
+        Y = buf[:T * D].view(T, D)
         sas.sas_mlp_fwd_noalloc(X, W1, W2, Y, b1, b2)
         assert sas.sas_mlp_noalloc_get_device_status() == sas.SAS_OK
         assert not torch.isnan(Y).any()
+        assert bool(torch.isnan(buf[T * D:]).all())
         _within_mlp_tolerance(Y.cpu(), P.f64(ref.cpu()))
         _within_mlp_tolerance(Y.cpu()[rows], yref)
 
