@@ -117,8 +117,8 @@ typedef struct {
     int32_t max_seqs;     /* 0: [B, H, N, d] batches of N-token sequences.  > 0: packed
                              variable-length sequences, at most max_seqs of them, in
                              [H, N, d] tensors whose token axis (N = capacity) holds
-                             them back to back (sas_attention_fwd_varlen); needs B = 1
-                             and SCORES_GIVEN, has no backward.                        */
+                             them back to back (sas_attention_fwd_varlen); needs B = 1,
+                             has no backward.                                          */
     int32_t max_seqlen;   /* packed mode: longest sequence (1 .. N; 0 selects N); the
                              score table has C = ceil(max_seqlen / 64) columns         */
     int32_t scope;        /* sas_scope (0 = SPARSE, the SAS default)                   */
@@ -231,7 +231,9 @@ sas_status sas_attention_bwd(sas_handle* h,
 /* Packed variable-length form of sas_attention_fwd, on a handle created
  * with max_seqs > 0.  Sequence s holds rows cu_seqlens[s] .. cu_seqlens[s+1]-1
  * of the token axis and is its own causal problem: its blocks of 64 tokens
- * start at its first row, and no row attends outside its sequence.
+ * start at its first row, and no row attends outside its sequence (with the
+ * learned selector each sequence is scored against the summaries of its own
+ * blocks).
  *
  *   cu_seqlens int32 [num_seqs + 1], DEVICE: cu[0] = 0, non-decreasing,
  *              every length <= max_seqlen, cu[num_seqs] <= N.  Checked on
@@ -240,7 +242,10 @@ sas_status sas_attention_bwd(sas_handle* h,
  *   num_seqs   1 .. max_seqs
  *   Q          bf16 [H, N, d]; K, V bf16 [Hkv, N, d]                     (in)
  *   scores     fp32 [Hkv, N, C], C = ceil(max_seqlen / 64); row cu[s] + t
- *              reads entries 0 .. floor(t/64)-1 (blocks of its sequence)  (in)
+ *              reads entries 0 .. floor(t/64)-1 (blocks of its sequence).
+ *              SCORES_GIVEN; NULL for MEANPOOL_PROJ                        (in)
+ *   Wq, Wk     the learned selector's projections as in sas_attention_fwd
+ *              (MEANPOOL_PROJ); NULL with given scores                     (in)
  *   O          bf16 [H, N, d]; LSE fp32 [H, N] (may be NULL)            (out)
  *   sel_idx, sel_logg  [Hkv, N, topk] as in sas_attention_fwd, block
  *              indices counted within the row's sequence (may be NULL) (out)
@@ -248,6 +253,7 @@ sas_status sas_attention_bwd(sas_handle* h,
  * synchronisation). */
 sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, int32_t num_seqs,
                                     const void* Q, const void* K, const void* V, const float* scores,
+                                    const void* Wq, const void* Wk,
                                     void* O, float* LSE, int32_t* sel_idx, float* sel_logg, void* stream);
 
 /* Dense MLP sublayer Y = GELU(X W1^T + b1) W2^T + b2 with the exact (erf)

@@ -53,8 +53,12 @@ cudaError_t launch_gemm(const GemmProblem& p, const KernelEnv& env, const char**
 
 // ---- a1: block summaries and key projection
 // Kt[bh][m][:] = bf16(Wk[h] @ mean(K[bh][64m : 64m+64][:])) for m < F = N / 64.
+// Packed sequences (tiles non-null, F = N / 64 + max_seqs slots): block m of
+// sequence s goes to slot floor(cu[s] / 64) + s + m (the tile table's entries
+// carry the sequence index s).
 cudaError_t launch_pool(const void* K, const void* Wk, void* Kt, int BH, int H, int N, int d, int d_sel,
-                        const KernelEnv& env);
+                        const KernelEnv& env, int F = -1, const int4* tiles = nullptr, const int* ntiles = nullptr,
+                        int T = 0);
 
 // ---- a2-a4: selection.  Per query row: the log-sum-exp of its C_i causal
 // scores, the Top-K blocks (ascending, -1 padded) with their log-gates, and

@@ -11,6 +11,13 @@
 // with Wk[h] staged row-major in shared memory (rows padded by one word so
 // that the 32 threads of a warp, one output each, hit distinct banks).  The pass is HBM-bound: it
 // reads every full-block key once and writes 2*d_sel bytes per block.
+//
+// Packed sequences: blocks restart at every sequence's first token.  Block m
+// of sequence s (tokens cu[s] + 64 m .. + 63) goes to summary slot
+// floor(cu[s] / 64) + s + m: the slots of different sequences never overlap
+// (floor((a + b) / 64) >= floor(a / 64) + floor(b / 64)), and a head needs at
+// most N / 64 + max_seqs of them.  The CTAs walk the selection pass's tile
+// table: tile t of a sequence covers its blocks 2t and 2t + 1.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -21,14 +28,29 @@ constexpr int kGroup = 8;   // blocks per CTA == warps per CTA
 
 template <int D, int DS>
 __global__ void __launch_bounds__(256) pool_kernel(const bf16* __restrict__ K, const bf16* __restrict__ Wk,
-                                                    bf16* __restrict__ Kt, int H, int N, int F) {
+                                                    bf16* __restrict__ Kt, int H, int N, int F,
+                                                    const int4* __restrict__ tiles, const int* __restrict__ ntiles) {
     __shared__ float kbar[kGroup][D];
     __shared__ __align__(16) bf16 ws[DS][D + 2];   // ws[j][k] = Wk[h][j][k]; rows 4-byte aligned
+    __shared__ int slot_of[kGroup];                // summary slot of each warp's block, -1 if none
 
     const int bh = blockIdx.y;
     const int h = bh % H;
-    const int m0 = blockIdx.x * kGroup;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // this warp's block: its first key row in the head's token axis and its slot
+    int first = -1, slot = -1;
+    if (tiles == nullptr) {
+        const int m = blockIdx.x * kGroup + warp;
+        if (m < F) { first = 64 * m; slot = m; }
+    } else {
+        const int g = blockIdx.x * (kGroup / 2) + warp / 2;   // tile slot: its blocks 2t, 2t + 1
+        if (g < __ldg(ntiles)) {
+            const int4 v = __ldg(tiles + g);                    // {first row, tile, length, sequence}
+            const int lb = 2 * v.y + (warp & 1);
+            if (64 * (lb + 1) <= v.z) { first = v.x + 64 * lb; slot = v.x / 64 + v.w + lb; }
+        }
+    }
+    if (lane == 0) slot_of[warp] = slot;
 
     // Wk[h] rows (D bf16 = D/8 16-byte pieces each) into the padded shared copy
     const bf16* w = Wk + static_cast<long long>(h) * DS * D;
@@ -43,16 +65,15 @@ __global__ void __launch_bounds__(256) pool_kernel(const bf16* __restrict__ K, c
     // Warp w sums block m0 + w.  A key row is D * 2 bytes: D / 8 lanes cover it
     // with 16-byte loads, so one warp instruction reads LPR = 256 / D rows and
     // each lane keeps fp32 sums of 8 dims over its rows.
-    const int m = m0 + warp;
     constexpr int LANES_PER_ROW = D / 8;
     constexpr int ROWS_PER_STEP = 32 / LANES_PER_ROW;
-    if (m < F) {
+    if (slot >= 0) {
         const int sub = lane / LANES_PER_ROW;            // which of the step's rows
         const int dl = (lane % LANES_PER_ROW) * 8;       // first of this lane's 8 dims
         float acc[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-        const bf16* base = K + (static_cast<long long>(bh) * N + static_cast<long long>(m) * 64 + sub) * D + dl;
+        const bf16* base = K + (static_cast<long long>(bh) * N + first + sub) * D + dl;
         // issue all of the lane's row loads before summing (16 in flight)
         constexpr int STEPS = 64 / ROWS_PER_STEP;
 #pragma unroll
@@ -86,33 +107,38 @@ __global__ void __launch_bounds__(256) pool_kernel(const bf16* __restrict__ K, c
 
     for (int o = threadIdx.x; o < kGroup * DS; o += blockDim.x) {
         const int g = o / DS, j = o - g * DS;
-        const int mm = m0 + g;
-        if (mm >= F) continue;
+        const int sl = slot_of[g];
+        if (sl < 0) continue;
         float s = 0.f;
 #pragma unroll 8
         for (int k = 0; k < D; ++k) s = fmaf(kbar[g][k], __bfloat162float(ws[j][k]), s);
-        Kt[(static_cast<long long>(bh) * F + mm) * DS + j] = __float2bfloat16_rn(s);
+        Kt[(static_cast<long long>(bh) * F + sl) * DS + j] = __float2bfloat16_rn(s);
     }
 }
 
+// F: summary slots per head (N / 64, or N / 64 + max_seqs for packed sequences);
+// tiles / ntiles / T: the packed sequences' tile table and its slot count (null otherwise).
 template <int D, int DS>
-cudaError_t launch_dd(const void* K, const void* Wk, void* Kt, int BH, int H, int N, const KernelEnv& env) {
-    const int F = N / 64;
+cudaError_t launch_dd(const void* K, const void* Wk, void* Kt, int BH, int H, int N, int F, const int4* tiles,
+                      const int* ntiles, int T, const KernelEnv& env) {
     if (F == 0) return cudaSuccess;
-    dim3 grid((F + kGroup - 1) / kGroup, BH);
+    const int gx = tiles == nullptr ? (F + kGroup - 1) / kGroup : (T + kGroup / 2 - 1) / (kGroup / 2);
+    if (gx == 0) return cudaSuccess;
+    dim3 grid(gx, BH);
     pool_kernel<D, DS><<<grid, 256, 0, env.stream>>>(static_cast<const bf16*>(K), static_cast<const bf16*>(Wk),
-                                                     static_cast<bf16*>(Kt), H, N, F);
+                                                     static_cast<bf16*>(Kt), H, N, F, tiles, ntiles);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_pool(const void* K, const void* Wk, void* Kt, int BH, int H, int N, int d, int d_sel,
-                        const KernelEnv& env) {
-    if (d == 128 && d_sel == 128) return launch_dd<128, 128>(K, Wk, Kt, BH, H, N, env);
-    if (d == 128 && d_sel == 64) return launch_dd<128, 64>(K, Wk, Kt, BH, H, N, env);
-    if (d == 64 && d_sel == 64) return launch_dd<64, 64>(K, Wk, Kt, BH, H, N, env);
-    if (d == 64 && d_sel == 128) return launch_dd<64, 128>(K, Wk, Kt, BH, H, N, env);
+                        const KernelEnv& env, int F, const int4* tiles, const int* ntiles, int T) {
+    if (F < 0) F = N / 64;
+    if (d == 128 && d_sel == 128) return launch_dd<128, 128>(K, Wk, Kt, BH, H, N, F, tiles, ntiles, T, env);
+    if (d == 128 && d_sel == 64) return launch_dd<128, 64>(K, Wk, Kt, BH, H, N, F, tiles, ntiles, T, env);
+    if (d == 64 && d_sel == 64) return launch_dd<64, 64>(K, Wk, Kt, BH, H, N, F, tiles, ntiles, T, env);
+    if (d == 64 && d_sel == 128) return launch_dd<64, 128>(K, Wk, Kt, BH, H, N, F, tiles, ntiles, T, env);
     return cudaErrorInvalidValue;
 }
 

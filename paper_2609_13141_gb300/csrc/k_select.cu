@@ -66,6 +66,7 @@ struct SelParams {
 // sequence length.  [B, H, N] inputs: one sequence of N rows per head.
 struct TileGeo {
     int slot, t, base, n;
+    int seq;   // the sequence's index (packed sequences; 0 otherwise)
 };
 
 // One CTA per (head, 128-row tile) on a 1-D grid: the tile index falls with
@@ -77,11 +78,11 @@ __device__ __forceinline__ int head_of_block(int BH) { return static_cast<int>(b
 __device__ __forceinline__ TileGeo tile_geo(const SelParams& p) {
     if (p.tiles == nullptr) {
         const int t = tile_of_block(p.T, p.BH);
-        return {t, t, 0, p.N};
+        return {t, t, 0, p.N, 0};
     }
     const int g = static_cast<int>(blockIdx.x / p.BH);
     const int4 v = __ldg(p.tiles + g);
-    return {g, v.y, v.x, v.z};
+    return {g, v.y, v.x, v.z, v.w};
 }
 
 // Online log-sum-exp of a row's scores.
@@ -861,6 +862,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     // each stage one head's Q tile and its d columns of Wq and accumulate.
     using Cfg = SelProjCfg<D, DS>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
+    if (p.tiles != nullptr && static_cast<int>(blockIdx.x / p.BH) >= __ldg(p.ntiles)) return;   // spare slot
     __shared__ uint64_t in_full, in_empty, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2],
         drain_bar, plan_bar;
     __shared__ uint32_t tmem_base_sh;
@@ -878,17 +880,23 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                      reinterpret_cast<float*>(stage_base + size_t(kRows) * (K + 1) * 4), K + 1};
     uint32_t* bitmap = reinterpret_cast<uint32_t*>(stage_base + staging_bytes(K));
 
-    const int t = tile_of_block(p.T, p.BH);
+    // the tile: its index within its sequence, the sequence's first row and
+    // length, and the summary slot of the sequence's block 0 (packed sequences:
+    // floor(cu[s] / 64) + s, see the block-summary pass)
+    const TileGeo geo = tile_geo(p);
+    const int t = geo.t;
+    const int seq_n = geo.n;
+    const int kt0 = p.tiles == nullptr ? 0 : geo.base / 64 + geo.seq;
     const int bh = head_of_block(p.BH);
     const int diag = 2 * t;
     // full training scope: no Top-K, the scores and their log-sum-exp are written out
     const bool full = p.full_lse != nullptr;
     // full*: noise added to the scores before the gate and the Top-K
     const bool noisy = p.noise != nullptr;
-    const int nb = min(2 * t + 1, p.F);          // blocks scored for this tile
+    const int nb = min(2 * t + 1, seq_n / 64);  // blocks scored for this tile (full blocks of its sequence)
     const int nchunks = (K > 0 || full) ? (nb + 63) >> 6 : 0;
     // the most blocks any row of the tile has: a histogram pass only when it exceeds K
-    const int last_row = min(p.N, (t + 1) * kRows) - 1;
+    const int last_row = min(seq_n, (t + 1) * kRows) - 1;
     const int tile_ci = last_row >= t * kRows ? (last_row >> 6) : 0;
     const bool pass_b = !full && tile_ci > K;
     // passes over the chunks, in order; D runs only if a row fails (decided after B)
@@ -939,7 +947,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 mbar_arrive_expect_tx(&in_full, Cfg::Q_BYTES + Cfg::WQ_BYTES);
 #pragma unroll
                 for (int a = 0; a < D / 64; ++a) {
-                    tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, t * kRows, bh * G + hq);
+                    tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, geo.base + t * kRows, bh * G + hq);
                     tma_load_3d(b_s + a * (DS * 128), &mapWq, &in_full, hq * D + a * 64, 0, bh % H);
                 }
                 ++rounds;
@@ -962,7 +970,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     mbar_arrive_expect_tx(&kc_full[b], Cfg::KC_BYTES);
 #pragma unroll
                     for (int a = 0; a < DS / 64; ++a)
-                        tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, c * 64, bh);
+                        tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, kt0 + c * 64,
+                                    bh);
                     ++issued;
                 }
             }
@@ -1027,8 +1036,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         // ---------------- row threads
         const int q = warp & 3;
         const int r = q * 32 + lane;
-        const int i = t * kRows + r;
-        const bool valid = i < p.N;
+        const int i = t * kRows + r;   // row within its sequence
+        const bool valid = i < seq_n;
         const int Ci = valid ? (i >> 6) : 0;
         const int Kp = min(K, Ci);
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
@@ -1073,7 +1082,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         // pass works on s~ = s + eps itself
         const float c_exp = noisy ? kLog2e : p.score_scale * kLog2e;
         const float emit_scale = noisy ? 1.f : p.score_scale;
-        const long long row_off = static_cast<long long>(bh) * p.N + i;
+        const long long row_off = static_cast<long long>(bh) * p.N + geo.base + i;
         const uint32_t hist_r = smem_u32(hist + r);
         const RowAddr ra{smem_u32(st.idx + r * st.stride), smem_u32(st.lg + r * st.stride), hist_r};
         int gc = 0;
@@ -1171,11 +1180,11 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         if (!full) {
             named_bar_sync(1, 128);
             if (ok)
-                copy_out(st, p, bh, static_cast<long long>(t) * kRows, min(kRows, p.N - t * kRows),
+                copy_out(st, p, bh, static_cast<long long>(geo.base) + t * kRows, min(kRows, seq_n - t * kRows),
                          static_cast<int>(threadIdx.x) - 64, 128);
             if (warp == 2)
-                compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + t) * p.C,
-                              p.union_cnt + static_cast<long long>(bh) * p.T + t);
+                compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + geo.slot) * p.C,
+                              p.union_cnt + static_cast<long long>(bh) * p.T + geo.slot);
         }
     }
     __syncthreads();
@@ -1242,7 +1251,8 @@ __global__ void __launch_bounds__(256) row_lse_kernel(const float* scores, int N
 constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
 
 // Tile table of packed sequences (one CTA).  Sequence s holds rows
-// cu[s] .. cu[s+1]-1 and T_s = ceil(n_s / 128) tiles.  Entries are ordered by
+// cu[s] .. cu[s+1]-1 and T_s = ceil(n_s / 128) tiles; an entry is
+// {first row cu[s], tile index within the sequence, n_s, s}.  Entries are ordered by
 // the tile's index within its sequence, descending (longest key history
 // first): tile t of every sequence with T_s > t sits at off(t) + rank(s),
 // off(t) = number of tiles with a larger index, rank(s) = the sequence's place
@@ -1291,7 +1301,7 @@ __global__ void __launch_bounds__(1024) varlen_tiles_kernel(const int32_t* cu, i
         const int T = (n + kRows - 1) / kRows;
         if (T == 0) continue;
         const int rank = gt[T] + atomicAdd(&nxt[T], 1);   // sequences with more tiles come first
-        for (int t = 0; t < T; ++t) tiles[off[t] + rank] = make_int4(b0, t, n, 0);
+        for (int t = 0; t < T; ++t) tiles[off[t] + rank] = make_int4(b0, t, n, s);
     }
 }
 
@@ -1334,10 +1344,7 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
         if (e != cudaSuccess) *err = "row log-sum-exp launch";
         return e;
     }
-    if (a.tiles != nullptr && a.scores == nullptr) {
-        *err = "selection: packed sequences need given scores";
-        return cudaErrorInvalidValue;
-    }
+
     const bool reg = a.topk <= 32;
     if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
     if (a.d == 128 && a.d_sel == 128) return launch_proj<128, 128>(a, p, env, err);

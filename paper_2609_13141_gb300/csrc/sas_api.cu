@@ -269,7 +269,6 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (c.max_seqs < 0 || c.max_seqlen < 0 || c.max_seqlen > c.N) return SAS_ERR_INVALID_ARG;
     const bool varlen = c.max_seqs > 0;
     if (varlen && c.B != 1) return SAS_ERR_INVALID_ARG;
-    if (varlen && c.selector != SAS_SEL_SCORES_GIVEN) return SAS_ERR_UNSUPPORTED;
     if (varlen && c.max_seqs > (1 << 20)) return SAS_ERR_UNSUPPORTED;
     const long long BH = static_cast<long long>(c.B) * c.H;
     const long long BHkv = static_cast<long long>(c.B) * Hkv;
@@ -290,7 +289,9 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     h->C = (max_len + 63) / 64;
     // packed sequences: at most N / 128 + max_seqs tiles (each sequence adds one partial tile)
     h->T = (c.N + 127) / 128 + (varlen ? c.max_seqs : 0);
-    h->F = c.N / 64;
+    // summary slots per KV group: N / 64 blocks, and with packed sequences one
+    // more per sequence (block m of sequence s sits at floor(cu[s] / 64) + s + m)
+    h->F = c.N / 64 + (varlen ? c.max_seqs : 0);
     sas_status st = check_device(h);
     if (st != SAS_OK) { delete h; return st; }
     cudaGetDevice(&h->device);
@@ -391,7 +392,7 @@ sas_status attention_fwd(sas_handle* h, const void* Q, const void* K, const void
         // a1: block summaries -> projected summaries
         if (h->F > 0) {
             e = timed_launch(h, 0, s, [&] {
-                return sas::launch_pool(K, Wk, h->Kt, h->BHkv, h->Hkv, c.N, c.d, h->d_sel, env);   // per KV group
+                return sas::launch_pool(K, Wk, h->Kt, h->BHkv, h->Hkv, c.N, c.d, h->d_sel, env, h->F);   // per KV group
             });
             if (e != cudaSuccess) return cuda_fail(h, e, "block summaries");
         }
@@ -450,8 +451,8 @@ sas_status sas_attention_fwd_noisy(sas_handle* h, const void* Q, const void* K, 
 }
 
 sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, int32_t num_seqs, const void* Q,
-                                    const void* K, const void* V, const float* scores, void* O, float* LSE,
-                                    int32_t* sel_idx, float* sel_logg, void* stream) {
+                                    const void* K, const void* V, const float* scores, const void* Wq, const void* Wk,
+                                    void* O, float* LSE, int32_t* sel_idx, float* sel_logg, void* stream) {
     if (h == nullptr) return SAS_ERR_INVALID_ARG;
     const sas_config& c = h->cfg;
     if (!h->varlen) return fail(h, SAS_ERR_INVALID_ARG, "handle not created for packed sequences (max_seqs = 0)");
@@ -461,7 +462,15 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     if (!Q || !K || !V || !O) return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O are required");
     if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
         return fail(h, SAS_ERR_INVALID_ARG, "Q, K, V and O must be 16-byte aligned");
-    if (!scores || !aligned4(scores)) return fail(h, SAS_ERR_INVALID_ARG, "scores required (4-byte aligned)");
+    const bool learned = c.selector == SAS_SEL_MEANPOOL_PROJ;
+    if (!learned) {
+        if (!scores || !aligned4(scores)) return fail(h, SAS_ERR_INVALID_ARG, "scores required (4-byte aligned)");
+        if (Wq || Wk) return fail(h, SAS_ERR_INVALID_ARG, "Wq/Wk must be NULL with given scores");
+    } else {
+        if (scores) return fail(h, SAS_ERR_INVALID_ARG, "scores must be NULL with the learned selector");
+        if (!Wq || !Wk || !aligned16(Wq) || !aligned16(Wk))
+            return fail(h, SAS_ERR_INVALID_ARG, "Wq and Wk required (16-byte aligned)");
+    }
     if ((LSE && !aligned4(LSE)) || (sel_idx && !aligned4(sel_idx)) || (sel_logg && !aligned4(sel_logg)))
         return fail(h, SAS_ERR_INVALID_ARG, "LSE / sel_idx / sel_logg must be 4-byte aligned");
 
@@ -471,24 +480,32 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     int32_t* out_idx = sel_idx ? sel_idx : h->sel_idx;
     float* out_lg = sel_logg ? sel_logg : h->sel_logg;
     const int max_len = c.max_seqlen > 0 ? c.max_seqlen : c.N;
-    // tile table, then a2-a4 over the tiles of every sequence
+    // the tile table of the packed sequences (device offsets, checked on the device)
+    cudaError_t e = sas::launch_varlen_tiles(cu_seqlens, num_seqs, c.N, max_len, h->tiles, h->ntiles, env);
+    if (e != cudaSuccess) return cuda_fail(h, e, "packed-sequence tile table");
+    h->launches += 1;
+    if (learned) {
+        // a1: each sequence's block summaries (blocks restart at its first token)
+        e = timed_launch(h, 0, s, [&] {
+            return sas::launch_pool(K, Wk, h->Kt, h->BHkv, h->Hkv, c.N, c.d, h->d_sel, env, h->F, h->tiles,
+                                    h->ntiles, h->T);
+        });
+        if (e != cudaSuccess) return cuda_fail(h, e, "block summaries");
+    }
+    // a2-a4 over the tiles of every sequence
     sas::SelectArgs sa{};
     sa.BH = h->BHkv; sa.H = h->Hkv; sa.N = c.N; sa.C = h->C; sa.T = h->T; sa.topk = c.topk; sa.d_sel = h->d_sel;
     sa.G = h->G;
     sa.gate_act = c.gate_act;
-    sa.score_scale = 1.0f;
+    sa.score_scale = learned ? 1.0f / std::sqrt(static_cast<float>(h->d_sel)) : 1.0f;
     sa.scores = scores;
+    sa.Q = Q; sa.Wq = Wq; sa.Kt = h->Kt; sa.F = h->F;
     sa.d = c.d;
     sa.sel_idx = out_idx; sa.sel_logg = out_lg;
     sa.union_idx = h->union_idx; sa.union_cnt = h->union_cnt;
     sa.tiles = h->tiles; sa.ntiles = h->ntiles;
-    cudaError_t e = timed_launch(h, 2, s, [&] {
-        cudaError_t r = sas::launch_varlen_tiles(cu_seqlens, num_seqs, c.N, max_len, h->tiles, h->ntiles, env);
-        if (r != cudaSuccess) { err = "packed-sequence tile table"; return r; }
-        return sas::launch_select(sa, env, &err);
-    });
+    e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
-    h->launches += 1;   // the tile table
     // a5 over the same tiles
     sas::AttnArgs aa{};
     aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;

@@ -86,7 +86,7 @@ def lib():
     L.sas_attention_fwd.restype = i32
     L.sas_attention_fwd_noisy.argtypes = [vp] * 13
     L.sas_attention_fwd_noisy.restype = i32
-    L.sas_attention_fwd_varlen.argtypes = [vp, vp, i32] + [vp] * 9
+    L.sas_attention_fwd_varlen.argtypes = [vp, vp, i32] + [vp] * 11
     L.sas_attention_fwd_varlen.restype = i32
     L.sas_attention_bwd.argtypes = [vp] * 16
     L.sas_attention_bwd.restype = i32
@@ -206,12 +206,12 @@ def sas_destroy(h):
 
 
 def sas_attention_fwd_varlen(h, cu_seqlens, Q, K, V, scores, O, LSE=None, sel_idx=None, sel_logg=None,
-                             stream=None):
+                             stream=None, Wq=None, Wk=None):
     bf = torch.bfloat16
     st = lib().sas_attention_fwd_varlen(
         h, _ptr(cu_seqlens, torch.int32, "cu_seqlens"), ctypes.c_int32(cu_seqlens.numel() - 1),
-        _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"), _ptr(scores, torch.float32, "scores"),
-        _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False), _ptr(sel_idx, torch.int32, "sel_idx", False),
+        _ptr(Q, bf, "Q"), _ptr(K, bf, "K"), _ptr(V, bf, "V"), _ptr(scores, torch.float32, "scores", False),
+        _ptr(Wq, bf, "Wq", False), _ptr(Wk, bf, "Wk", False), _ptr(O, bf, "O"), _ptr(LSE, torch.float32, "LSE", False), _ptr(sel_idx, torch.int32, "sel_idx", False),
         _ptr(sel_logg, torch.float32, "sel_logg", False), _stream(stream))
     _check(st, h, "sas_attention_fwd_varlen")
 
@@ -339,11 +339,12 @@ class SasLayer:
         self.h = sas_create(B, H, N, d, topk, mode, selector, d_sel, sm_scale, 64, gate_act, gate_pos, Hkv,
                             max_seqs, max_seqlen, scope)
 
-    def attention_varlen(self, cu_seqlens, Q, K, V, scores, want_sel=True, stream=None, sel_fill=-1):
+    def attention_varlen(self, cu_seqlens, Q, K, V, scores=None, want_sel=True, stream=None, sel_fill=-1, Wq=None,
+                         Wk=None):
         """Packed sequences (handle made with max_seqs > 0): Q [H, N, d], K/V [Hkv, N, d],
-        scores [Hkv, N, C], cu_seqlens int32 on the device.  The library does not write
-        rows past cu[-1]: they keep the fill of the tensors made here (0, and sel_fill
-        in sel_idx)."""
+        scores [Hkv, N, C] (or the learned selector's Wq, Wk), cu_seqlens int32 on the
+        device.  The library does not write rows past cu[-1]: they keep the fill of
+        the tensors made here (0, and sel_fill in sel_idx)."""
         dev = Q.device
         O = torch.zeros_like(Q)
         LSE = torch.zeros(self.H, self.N, device=dev, dtype=torch.float32)
@@ -352,7 +353,7 @@ class SasLayer:
             k = max(self.topk, 1)
             sel_idx = torch.full((self.Hkv, self.N, k), sel_fill, device=dev, dtype=torch.int32)
             sel_logg = torch.zeros(self.Hkv, self.N, k, device=dev, dtype=torch.float32)
-        sas_attention_fwd_varlen(self.h, cu_seqlens, Q, K, V, scores, O, LSE, sel_idx, sel_logg, stream)
+        sas_attention_fwd_varlen(self.h, cu_seqlens, Q, K, V, scores, O, LSE, sel_idx, sel_logg, stream, Wq, Wk)
         return O, LSE, sel_idx, sel_logg
 
     def _outputs(self, Q, want_sel):

@@ -54,7 +54,6 @@ def test_status_strings(lib):
     (dict(B=1, H=2, N=128, d=64, topk=2, Hkv=-1), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=-1), sas.SAS_ERR_INVALID_ARG),
     (dict(B=2, H=2, N=128, d=64, topk=2, max_seqs=4), sas.SAS_ERR_INVALID_ARG),          # packed needs B = 1
-    (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=4, selector=1), sas.SAS_ERR_UNSUPPORTED),
     (dict(B=1, H=2, N=128, d=64, topk=2, max_seqs=4, max_seqlen=129), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=2, N=128, d=64, topk=2, scope=2), sas.SAS_ERR_INVALID_ARG),
     (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, gate_pos=1), sas.SAS_ERR_UNSUPPORTED),   # full scope: inner only

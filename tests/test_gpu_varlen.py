@@ -114,3 +114,66 @@ def test_wrong_entry_points_are_refused():
         layer.attention_varlen(torch.tensor([0, 256], dtype=torch.int32, device=DEV), z[0], z[0], z[0],
                                torch.zeros(2, 256, 4, device=DEV))
     layer.close()
+
+
+@pytest.mark.parametrize("lens,cap,Hq,Hkv,d,topk,mode", [
+    ([700, 1, 64, 129, 0, 300, 255], 1500, 4, 2, 128, 3, TRAIN),   # ragged, empty, one-token, GQA, spare rows
+    ([513, 130, 77], 720, 2, 2, 64, 2, INFER),                     # d = 64, offsets off the block grid
+])
+def test_varlen_learned_selector_exact_inputs(lens, cap, Hq, Hkv, d, topk, mode):
+    # integer Q, K and {-1, 0, 1} projections: every selector sum is exact in
+    # fp32, so each sequence's kept sets -- scored against the summaries of its
+    # own blocks with its group gate query -- equal the oracle's on every row
+    G = Hq // Hkv
+    Q = synth.integer_selector_inputs(1, Hq, cap, d, d, seed=len(lens))[0][0]
+    _, K, V, _, _ = synth.integer_selector_inputs(1, Hkv, cap, d, d, seed=len(lens) + 1)
+    K, V = K[0], V[0]
+    Wq, Wk = synth.decode_selector_weights(Hkv, G, d, d, seed=len(lens), exact=True)
+    cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32)
+    max_len = max(lens)
+    layer = sas.SasLayer(1, Hq, cap, d, topk, mode=mode, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=d, Hkv=Hkv,
+                         max_seqs=len(lens), max_seqlen=max_len)
+    O, LSE, si, sl = layer.attention_varlen(cu.to(DEV), *(t.to(DEV).contiguous() for t in (Q, K, V)), None,
+                                            sel_fill=-7, Wq=Wq.to(DEV), Wk=Wk.to(DEV))
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    ref = OR.sas_attention_varlen(P.f64(Q), P.f64(K), P.f64(V), cu.numpy(), 64, topk, mode=mode, Wq=P.f64(Wq),
+                                  Wk=P.f64(Wk))
+    end = int(cu[-1])
+    for gk in range(Hkv):
+        for s0, s1 in zip(cu[:-1].tolist(), cu[1:].tolist()):
+            if s1 == s0:
+                continue
+            s = OR.selector_scores_group(P.f64(Q[gk * G:(gk + 1) * G, s0:s1]), P.f64(K[gk, s0:s1]), P.f64(Wq[gk]),
+                                         P.f64(Wk[gk]), 64)
+            P.check_selection_rows(si[gk, s0:s1].cpu().numpy()[:, :topk], s, np.arange(s1 - s0), topk)
+        assert np.abs(sl[gk].cpu().numpy()[:end, :topk] - ref["sel_logg"][gk, :end]).max() <= P.LOGG_MAX_ABS
+    for hi in range(Hq):
+        P.compare_o(P.f64(O[hi].cpu())[:end], ref["O"][hi, :end], f"O[{hi}]")
+        assert np.abs(LSE[hi].cpu().numpy()[:end] - ref["LSE"][hi, :end]).max() <= P.LSE_MAX_ABS
+    assert torch.count_nonzero(O[:, end:]) == 0
+    assert bool((si[:, end:] == -7).all())
+
+
+def test_varlen_learned_equal_lengths_match_the_batched_path():
+    # three sequences of 640 tokens packed = a batch of three 640-token sequences
+    S_, n, H, d, topk = 3, 640, 2, 128, 4
+    Q, K, V = synth.qkv(S_, H, n, d, seed=12, regime="R2")
+    Wq, Wk = synth.selector_weights(H, d, d, seed=12)
+    dev = DEV
+    batched = sas.SasLayer(S_, H, n, d, topk, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=d)
+    Ob, Lb, sib, slb = batched.attention(*(t.to(dev) for t in (Q, K, V)), Wq=Wq.to(dev), Wk=Wk.to(dev))
+    batched.close()
+    packed = sas.SasLayer(1, H, S_ * n, d, topk, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=d, max_seqs=S_,
+                          max_seqlen=n)
+    pack = lambda t: t.permute(1, 0, 2, 3).reshape(t.shape[1], S_ * n, d).contiguous().to(dev)
+    cu = torch.arange(0, S_ * n + 1, n, dtype=torch.int32, device=dev)
+    Op, Lp, sip, slp = packed.attention_varlen(cu, pack(Q), pack(K), pack(V), None, Wq=Wq.to(dev), Wk=Wk.to(dev))
+    assert sas.sas_get_device_status(packed.h) == 0
+    packed.close()
+    for b in range(S_):
+        rows = slice(b * n, (b + 1) * n)
+        assert torch.equal(Op[:, rows], Ob[b])
+        assert torch.equal(Lp[:, rows], Lb[b])
+        assert torch.equal(sip[:, rows], sib[b])
+        assert torch.equal(slp[:, rows], slb[b])
