@@ -206,14 +206,14 @@ def job_throughput(tflop_per_step, world, ms_per_step):
 
 # --------------------------------------------------------------- our arm
 
-def kernel_traffic(kind):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's
-    sources are unchanged since the capture (else None)."""
+def kernel_traffic(kind, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    this workload and the kernel's sources are unchanged since (else None)."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
         return None
     rec = json.load(open(p)).get(kind)
-    if not rec:
+    if not rec or rec.get("workload") != workload:
         return None
     m = hashlib.sha256()
     for f in rec["sources"]:
@@ -395,7 +395,7 @@ def run_ours(args, w, rank, world):
         avg = kt[dom][1] / kt[dom][0]
         achieved = flops_per_launch[dom] / (avg / 1e3) / 1e12
         roof = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1), "peak": peaks["bf16"],
-                "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16"], 4), "traffic": kernel_traffic(dom),
+                "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16"], 4), "traffic": kernel_traffic(dom, w["name"]),
                 "peak_source": f"{peaks['source']} bf16 dense burst"}
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -946,6 +946,8 @@ def main():
     ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
                     help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
     ap.add_argument("--topk", type=int, default=None, help="override the workload's K")
+    ap.add_argument("--heads", type=int, default=None,
+                    help="override the workload's head count (smaller cases of the same shape, for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=4.0)
@@ -962,6 +964,11 @@ def main():
     if args.topk is not None:
         w["topk"] = args.topk
         w["name"] = w["name"].replace("K=32", f"K={args.topk}")
+    if args.heads is not None:
+        if w.get("Hkv", w["H"]) != w["H"]:
+            ap.error("--heads applies to workloads without GQA")
+        w["name"] = w["name"].replace(f"H={w['H']}", f"H={args.heads}")
+        w["H"] = args.heads
     if args.oracle_sample_only:
         rate, dt, _ = oracle_sample(w, args.cpu_budget, learned=args.regime == "R2" and w.get("Hkv", w["H"]) == w["H"]
                                     and not w.get("lens"))
