@@ -609,9 +609,11 @@ TRAIN_METRIC = "SAS attention training step (forward + backward) of one layer: m
 def run_train(args, w, rank, world):
     """Forward + backward of the SAS attention (Alg. 1 steps 1-4 and Alg. 4) on
     the workload's attention shape, given block-coherent scores (R1) so that
-    the score gradient is produced too.  Algorithmic FLOPs: the forward's
-    4 d per attended (row, key) pair plus the backward's 10 d (QK^T, dO V^T,
-    dS K, dS^T Q, P^T dO)."""
+    the score gradient is produced too; GQA workloads share K, V, the kept
+    sets and the gates per KV group, packed ones run every sequence as its own
+    problem.  Algorithmic FLOPs: the forward's 4 d per attended (row, key)
+    pair plus the backward's 10 d (QK^T, dO V^T, dS K, dS^T Q, P^T dO)."""
+    import numpy as np
     import torch
 
     from paper_2609_13141_gb300 import sas, synth
@@ -620,25 +622,36 @@ def run_train(args, w, rank, world):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     B, H, N, d, K = (w[k] for k in ("B", "H", "N", "d", "topk"))
-    C = (N + 63) // 64
-    Q, Kk, V = synth.qkv(B, H, N, d, seed=rank)
-    S = synth.scores(B, H, N, C, seed=rank, regime="R1")
+    Hkv = w.get("Hkv", H)
+    lens = w.get("lens")
+    C = ((max(lens) if lens else N) + 63) // 64
+    Q = synth.qkv(B, H, N, d, seed=rank)[0]
+    _, Kk, V = synth.qkv(B, Hkv, N, d, seed=rank + 100)
+    S = synth.scores(B, Hkv, N, C, seed=rank, regime="R1")
     dO = synth.normal((B, H, N, d), rank + 5).to(torch.bfloat16)
     Qd, Kd, Vd, Sd, dOd = (t.to(dev) for t in (Q, Kk, V, S, dO))
-    layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN)
+    if lens:
+        layer = sas.SasLayer(1, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv, max_seqs=len(lens),
+                             max_seqlen=max(lens))
+        cud = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
+    else:
+        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv)
     h = layer.h
     stream = torch.cuda.current_stream(dev)
     O = torch.empty_like(Qd)
     LSE = torch.empty(B, H, N, device=dev, dtype=torch.float32)
-    si = torch.empty(B, H, N, max(K, 1), device=dev, dtype=torch.int32)
-    sl = torch.empty(B, H, N, max(K, 1), device=dev, dtype=torch.float32)
+    si = torch.empty(B, Hkv, N, max(K, 1), device=dev, dtype=torch.int32)
+    sl = torch.empty(B, Hkv, N, max(K, 1), device=dev, dtype=torch.float32)
     dQ, dK, dV = torch.empty_like(Qd), torch.empty_like(Kd), torch.empty_like(Vd)
     dl = torch.empty_like(sl)
     ds = torch.empty_like(Sd)
     flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
 
     def step():
-        sas.sas_attention_fwd(h, Qd, Kd, Vd, O, Sd, None, None, LSE, si, sl, stream)
+        if lens:
+            sas.sas_attention_fwd_varlen(h, cud, Qd[0], Kd[0], Vd[0], Sd[0], O[0], LSE[0], si[0], sl[0], stream)
+        else:
+            sas.sas_attention_fwd(h, Qd, Kd, Vd, O, Sd, None, None, LSE, si, sl, stream)
         sas.sas_attention_bwd(h, Qd, Kd, Vd, O, LSE, dOd, dQ, dK, dV, Sd, si, sl, dl, ds, stream)
 
     for _ in range(max(args.warmup, 3)):
@@ -662,10 +675,14 @@ def run_train(args, w, rank, world):
     clocks = sampler.stop()
     assert sas.sas_get_device_status(h) == 0
     ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
-    Tt = (N + 127) // 128
-    unions = sas.sas_get_tile_union_counts(h, B * H * Tt)
+    Tt = (N + 127) // 128 + (len(lens) if lens else 0)
+    unions = sas.sas_get_tile_union_counts(h, B * Hkv * Tt)
+    if lens:
+        # packed: the first sum(ceil(n/128)) slots of each group are the tiles in use
+        used = sum((n + 127) // 128 for n in lens)
+        unions = [unions[g * Tt + k] for g in range(Hkv) for k in range(used)]
     layer.close()
-    fl = algorithmic_flops(w, learned=False)
+    fl = packed_flops(w) if lens else algorithmic_flops(w, learned=False)
     f_fwd = fl["attention"]
     f_bwd = f_fwd * 10 // 4
     tflop = (f_fwd + f_bwd) / 1e12
@@ -679,8 +696,9 @@ def run_train(args, w, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 softmax and gradients of log g, s)",
         "data": "synthetic (seeded; R1 block-coherent scores given, N(0,1) Q/K/V/dO)",
-        "config": {"workload": w["name"] + " (attention only, forward + backward)", "B": B, "H": H, "N": N, "d": d,
-                   "topk": K, "l2": "flushed between timed steps (256 MiB write)", "parallelism": f"replicas x{world}"},
+        "config": {"workload": w["name"] + " (attention only, forward + backward)", "B": B, "H": H, "Hkv": Hkv,
+                   "N": N, "d": d, "topk": K, "packed_lengths": lens,
+                   "l2": "flushed between timed steps (256 MiB write)", "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "tensor", "kernel": "attention_bwd", "achieved": round(ach, 1), "peak": peaks["bf16"],
                      "unit": "TFLOP/s", "frac": round(ach / peaks["bf16"], 4), "traffic": None,
                      "peak_source": f"{peaks['source']} bf16 dense burst"},

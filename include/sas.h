@@ -196,24 +196,33 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
  * The kept sets are those of the forward (the Top-K choice is a constant of
  * the backward), and the per-tile block lists are read from the handle: call
  * it after the sas_attention_fwd of the same inputs on this handle, with no
- * other forward in between.
+ * other forward in between.  With grouped-query attention (Hkv < H) a
+ * group's K, V, kept sets and gates serve its H / Hkv query heads, so dK, dV
+ * and the gate gradients are sums over those heads (Sec. 3.3).
  *
- *   Q, K, V, O bf16 [B, H, N, d]; LSE fp32 [B, H, N]: the forward's     (in)
+ * Packed sequences (a handle created with max_seqs > 0): the backward of the
+ * last sas_attention_fwd_varlen on the handle, whose tile table it reads;
+ * the layouts drop B ([H, N, d], [Hkv, N, C], ...), every sequence is its
+ * own problem (no gradient crosses sequences), and rows past cu[num_seqs]
+ * of dQ, dK, dV, dlogg and dscores are not written.
+ *
+ *   Q, O       bf16 [B, H, N, d]; LSE fp32 [B, H, N]: the forward's      (in)
+ *   K, V       bf16 [B, Hkv, N, d]                                       (in)
  *   dO         bf16 [B, H, N, d] gradient of the loss w.r.t. O          (in)
  *   sel_idx, sel_logg: the forward's outputs, or NULL if the forward
  *              was given NULL for them                                   (in)
- *   scores     fp32 [B, H, N, C] given scores; needed only for dscores   (in)
- *   dQ, dK, dV bf16 [B, H, N, d]                                         (out)
- *   dlogg      fp32 [B, H, N, topk] dL/d(log g) of each kept block, in
- *              the order of sel_idx (0 where padded; all 0 in INFER_HARD
- *              mode); may be NULL                                        (out)
- *   dscores    fp32 [B, H, N, C] dL/ds of the given scores, sparse scope:
+ *   scores     fp32 [B, Hkv, N, C] given scores; needed only for dscores (in)
+ *   dQ         bf16 [B, H, N, d]; dK, dV bf16 [B, Hkv, N, d]             (out)
+ *   dlogg      fp32 [B, Hkv, N, topk] dL/d(log g) of each kept block, in
+ *              the order of sel_idx, summed over the group's query heads
+ *              (0 where padded; all 0 in INFER_HARD mode); may be NULL   (out)
+ *   dscores    fp32 [B, Hkv, N, C] dL/ds of the given scores, sparse scope:
  *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
  *              row's history; SCORES_GIVEN handles only, else NULL.
  *              g_m = exp(s_m - LSE_i) takes the row's log-normaliser
  *              LSE_i = s_m - log g_m from its first kept entry, so the
  *              scores must be the ones the forward selected with     (out)
- * N must not exceed 262016 (2047 tiles of 128 rows).  The first call
+ * N (packed: max_seqlen) must not exceed 262016 (2047 tiles of 128 rows).  The first call
  * allocates the handle's backward workspace (synchronously); later calls are
  * asynchronous and can be captured in a CUDA graph when B * H * T * (T + 1)
  * * 512 bytes <= 8 GiB (T = ceil(N / 128)) and that much memory is free at the

@@ -95,9 +95,12 @@ struct SelectArgs {
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err);
 // Builds the tile table of packed sequences cu[0..S] (device offsets) with
 // sequences of at most max_len tokens within Ncap rows; bad offsets set the
-// status word to SAS_ERR_INVALID_ARG and leave *ntiles = 0.
+// status word to SAS_ERR_INVALID_ARG and leave *ntiles = 0.  Slots are
+// ordered by local tile index, longest sequences first: local tile t of the
+// sequence of rank r sits at slot tile_off[t] + r (tile_off: ceil(max_len /
+// 128) + 1 ints).
 cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len, int4* tiles, int* ntiles,
-                                const KernelEnv& env);
+                                int* tile_off, const KernelEnv& env);
 
 // ---- a5: fused gated block-sparse attention forward.
 struct AttnArgs {
@@ -183,8 +186,9 @@ struct AttnBwdArgs {
     void* dQ;
     void* dK;
     void* dV;
-    float* dlogg;               // [BH][N][topk]
-    float* ds;                  // [BH][N][C] or null
+    float* dlogg;               // [BH / G][N][topk] (per KV group: the G heads' sum)
+    float* ds;                  // [BH / G][N][C] or null
+    float* dlogg_heads;         // G > 1: [BH][N][topk] per query head, summed into dlogg
     // workspace
     float* delta;               // [BH][N]
     int32_t* inv_cnt;           // [BH*T]
@@ -194,7 +198,13 @@ struct AttnBwdArgs {
     int32_t* inv_pos;           // their block positions
     int32_t* slot_off;          // [BH*T + 1] first offset slot of each tile
     float* offs;                // [slots][128] per-row offsets written by pass 1
+    // packed sequences: the forward's tile table (as in SelectArgs) and its
+    // per-local-tile first slots; null for [B, H, N, d] batches
+    const int4* tiles;
+    const int* ntiles;
+    const int* tile_off;
     int N, C, T, BH, topk, mode, d;
+    int G;                      // query heads per KV group: K, V, the lists and the gate gradients are per group
     float sm_scale;
 };
 extern const int kBwdMaxTiles;   // query tiles per head the backward supports

@@ -19,6 +19,12 @@
 //                     over them, dV += P^T dO and dK += dS^T Q.
 //   bwd_ds_kernel     score gradient of given scores (sparse scope):
 //                     ds_m = dlogg_m [m kept] - g_m sum dlogg.
+// GQA: a KV group's K, V, kept lists and log-gates feed its G query heads, so
+// pass 1 runs per query head on its group's K, V and lists and writes the
+// head's log-gate gradient, bwd_dlogg_sum adds the G heads (in head order:
+// deterministic), pass 2 runs per (group, key pair) over every visiting query
+// tile of each of the G heads, accumulating dK, dV of the group, and the score
+// gradient applies the gate softmax's Jacobian to the summed d(log g).
 // Roles, pass 1: warps 0-7 are the rows (two threads per TMEM lane, half a
 // block of keys each), warp 8 issues S and dQ, warp 9 issues dP, warp 10
 // issues the TMA loads.  Pass 2: warps 0-3 are the keys (one thread per TMEM
@@ -112,11 +118,31 @@ struct BwdParams {
     const int32_t* inv_pos;     // per inverted entry: positions of blocks 2p, 2p+1 in the tile's list (+1; 0: absent)
     const int32_t* slot_off;    // per tile: first slot of its visited blocks in offs
     float* offs;                // per (tile, visited block) slot: 128 rows of log g - LSE (log2), -inf if not attended
+    const int4* tiles;          // packed sequences: {first row of the sequence, local tile, length, sequence} per slot
+    const int* ntiles;          // slots in use (device)
+    const int* tile_off;        // first slot of each local tile index
     int N, C, T, BH, topk, mode;
+    int G;                      // query heads per KV group (BH counts query heads)
     float sm_scale, scale_log2;
     int* status;
     long long limit;
 };
+
+// A tile slot's place in its sequence: the local tile index t (rows 128 t ..
+// 128 t + 127 of the sequence, key blocks 2t, 2t + 1), the sequence's first
+// row in the head's token axis and its length.  [B, H, N, d] batches: one
+// sequence of N rows, slot = tile.
+struct BwdTile {
+    int t, base, n;
+};
+__device__ __forceinline__ BwdTile bwd_tile(const BwdParams& p, int slot) {
+    if (p.tiles == nullptr) return {slot, 0, p.N};
+    const int4 v = __ldg(p.tiles + slot);
+    return {v.y, v.x, v.z};
+}
+__device__ __forceinline__ int bwd_slots_in_use(const int4* tiles, const int* ntiles, int T) {
+    return tiles == nullptr ? T : __ldg(ntiles);
+}
 
 __global__ void __launch_bounds__(kThreadsB, 1)
 bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
@@ -125,11 +151,17 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     uint8_t* smem = dsm + ((1024u - (smem_u32(dsm) & 1023u)) & 1023u);
     DqCtl& ctl = *reinterpret_cast<DqCtl*>(smem + kDqOffCtl);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int tile = blockIdx.x % p.T, bh = blockIdx.x / p.T;
-    const long long tb = static_cast<long long>(bh) * p.T + tile;
-    const int32_t* ulist = p.union_idx + tb * p.C;
-    const int U = __ldg(p.union_cnt + tb);
-    const int nb = U + ((2 * tile + 1 < p.C) ? 2 : 1);   // visited blocks: union, then the diagonal ones
+    const int slot = blockIdx.x % p.T, bh = blockIdx.x / p.T;   // (query head, tile slot)
+    if (slot >= bwd_slots_in_use(p.tiles, p.ntiles, p.T)) return;   // an unused slot (packed sequences)
+    const BwdTile tg = bwd_tile(p, slot);
+    const int tile = tg.t;                                       // local tile index
+    const int kv = bh / p.G;                                     // its KV group
+    const long long tb = static_cast<long long>(bh) * p.T + slot;
+    const long long tbk = static_cast<long long>(kv) * p.T + slot;
+    const int32_t* ulist = p.union_idx + tbk * p.C;
+    const int U = __ldg(p.union_cnt + tbk);
+    const int cseq = (tg.n + kKeys - 1) / kKeys;                 // blocks of the sequence
+    const int nb = U + ((2 * tile + 1 < cseq) ? 2 : 1);   // visited blocks: union, then the diagonal ones
     if (t == 0) {
         mbar_init(&ctl.q_full, 1);
         for (int s = 0; s < kKvStages; ++s) {
@@ -154,7 +186,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     tc_fence_after();
     const uint32_t tmem = ctl.tmem_base;
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
-    const int row0 = tile * kRows;
+    const int row0 = tg.base + tile * kRows;   // the tile's first row in the token axis
 
     if (warp == 10) {
         if (lane == 0) {
@@ -172,8 +204,9 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 uint8_t* st = smem + kDqOffKV + s * 2 * kKVBytes;
                 mbar_arrive_expect_tx(&ctl.kv_full[s], 2 * kKVBytes);
                 for (int h = 0; h < 2; ++h) {
-                    tma_load_3d(st + h * (kKeys * 128), &mapK, &ctl.kv_full[s], h * 64, m * kKeys, bh);
-                    tma_load_3d(st + kKVBytes + h * (kKeys * 128), &mapV, &ctl.kv_full[s], h * 64, m * kKeys, bh);
+                    tma_load_3d(st + h * (kKeys * 128), &mapK, &ctl.kv_full[s], h * 64, tg.base + m * kKeys, kv);
+                    tma_load_3d(st + kKVBytes + h * (kKeys * 128), &mapV, &ctl.kv_full[s], h * 64,
+                                tg.base + m * kKeys, kv);
                 }
             }
         }
@@ -264,11 +297,12 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         // ---- rows: thread t takes row t % 128 (its TMEM lane) and keys
         // 32 hk .. 32 hk + 31 of every block, hk = t / 128
         const int r = t & (kRows - 1), hk = t >> 7;
-        const int i = row0 + r;
-        const bool valid = i < p.N;
+        const int i = tile * kRows + r;        // row index within the sequence
+        const bool valid = i < tg.n;
         const int c = i >> 6;                  // the row's current block
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-        const long long roff = static_cast<long long>(bh) * p.N + i;
+        const long long roff = static_cast<long long>(bh) * p.N + row0 + r;
+        const long long kvoff = static_cast<long long>(kv) * p.N + row0 + r;   // the group's kept list
         float delta = 0.f, lse2 = 0.f;
         if (valid) {
             delta = row_delta(p.O + roff * kD, p.dO + roff * kD);
@@ -277,9 +311,9 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         }
         const int slot0 = __ldg(p.slot_off + tb);
         const int nsel = valid ? min(p.topk, c) : 0;
-        const int32_t* my_idx = p.sel_idx + roff * p.topk;
-        const float* my_lg = p.sel_logg + roff * p.topk;
-        float* my_dlg = p.dlogg + roff * p.topk;   // zeroed before this kernel; both halves add
+        const int32_t* my_idx = p.sel_idx + kvoff * p.topk;
+        const float* my_lg = p.sel_logg + kvoff * p.topk;
+        float* my_dlg = p.dlogg + roff * p.topk;   // this head's (zeroed before this kernel; both halves add)
         int e = 0;                             // next kept entry (ascending)
         int km = nsel > 0 ? __ldg(my_idx) : 0x7fffffff;
         float kl = nsel > 0 ? __ldg(my_lg) : 0.f;
@@ -386,12 +420,23 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
 
 // ------------------------------------------------------- inverted block lists
 
+// Slot of the key pair (blocks 2 pr, 2 pr + 1) of the sequence whose local
+// tile tq sits at slot g: the pair's keys are the rows of local tile pr, and a
+// sequence of rank r keeps its tile t at tile_off[t] + r.  [B, H, N, d]: pr.
+__device__ __forceinline__ int pair_slot(const int4* tiles, const int* tile_off, int g, int pr) {
+    if (tiles == nullptr) return pr;
+    const int tq = __ldg(tiles + g).y;
+    return g - __ldg(tile_off + tq) + __ldg(tile_off + pr);
+}
+
 // count: for every tile, the key pairs (2p, 2p+1) its union list touches
 __global__ void bwd_inv_count_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cnt, int BH,
-                                     int T, int C) {
+                                     int T, int C, const int4* tiles, const int* ntiles, const int* tile_off) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * T) return;
     const int bh = static_cast<int>(tb / T);
+    const int g = static_cast<int>(tb - static_cast<long long>(bh) * T);
+    if (g >= bwd_slots_in_use(tiles, ntiles, T)) return;
     const int32_t* u = union_idx + tb * C;
     const int U = union_cnt[tb];
     int last = -1;
@@ -399,7 +444,7 @@ __global__ void bwd_inv_count_kernel(const int32_t* union_idx, const int32_t* un
         const int pr = u[k] >> 1;
         if (pr == last) continue;
         last = pr;
-        atomicAdd(cnt + static_cast<long long>(bh) * T + pr, 1);
+        atomicAdd(cnt + static_cast<long long>(bh) * T + pair_slot(tiles, tile_off, g, pr), 1);
     }
 }
 
@@ -429,12 +474,16 @@ __global__ void __launch_bounds__(1024) bwd_inv_scan_kernel(const int32_t* cnt, 
     if (t == 1023) off[n] = part[1023];
 }
 
+// fill: entry = the visiting tile's index within its sequence and the positions
+// of the pair's blocks in its list
 __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cursor,
-                                    int32_t* tiles, int32_t* pos, int BH, int T, int C) {
+                                    int32_t* tiles, int32_t* pos, int BH, int T, int C, const int4* ttab,
+                                    const int* ntiles, const int* tile_off) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * T) return;
     const int bh = static_cast<int>(tb / T);
     const int tile = static_cast<int>(tb - static_cast<long long>(bh) * T);
+    if (tile >= bwd_slots_in_use(ttab, ntiles, T)) return;
     const int32_t* u = union_idx + tb * C;
     const int U = union_cnt[tb];
     int last = -1;
@@ -445,18 +494,43 @@ __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* uni
         // positions (+1) of blocks 2pr and 2pr+1 in this tile's list (ascending)
         const int j0 = m == 2 * pr ? k + 1 : 0;
         const int j1 = m == 2 * pr + 1 ? k + 1 : (k + 1 < U && u[k + 1] == 2 * pr + 1 ? k + 2 : 0);
-        const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pr, 1);
-        tiles[slot] = tile;
+        const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pair_slot(ttab, tile_off, tile, pr), 1);
+        tiles[slot] = ttab == nullptr ? tile : __ldg(ttab + tile).y;
         pos[slot] = j0 | (j1 << 16);
     }
 }
 
-// visited blocks per tile: its union list plus one or two diagonal blocks
-__global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH, int T, int C) {
+// visited blocks per (query head, tile): its group's union list plus one or two diagonal blocks
+__global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH, int T, int N, int G,
+                                 const int4* tiles, const int* ntiles) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * T) return;
-    const int tile = static_cast<int>(tb % T);
-    cnt[tb] = union_cnt[tb] + ((2 * tile + 1 < C) ? 2 : 1);
+    const int g = static_cast<int>(tb % T);
+    if (g >= bwd_slots_in_use(tiles, ntiles, T)) {
+        cnt[tb] = 0;
+        return;
+    }
+    int t = g, n = N;
+    if (tiles != nullptr) {
+        const int4 v = __ldg(tiles + g);
+        t = v.y;
+        n = v.z;
+    }
+    const long long tbk = (tb / T) / G * T + g;
+    cnt[tb] = union_cnt[tbk] + ((2 * t + 1 < (n + kKeys - 1) / kKeys) ? 2 : 1);
+}
+
+// GQA: the log-gate gradient of a KV group is the sum of its G query heads'
+// (Eq. ours_train: the group's log-gates enter the logits of all G heads),
+// added in head order so the result does not depend on scheduling.
+__global__ void bwd_dlogg_sum_kernel(const float* heads, float* out, long long per_group, long long total, int G) {
+    const long long x = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (x >= total) return;
+    const long long g = x / per_group, k = x - g * per_group;
+    const float* src = heads + g * G * per_group + k;
+    float s = 0.f;
+    for (int h = 0; h < G; ++h) s += __ldg(src + h * per_group);
+    out[x] = s;
 }
 
 // ------------------------------------------------------------------ pass 2
@@ -494,11 +568,21 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     DkvCtl& ctl = *reinterpret_cast<DkvCtl*>(smem + kDkvOffCtl);
     int* list = reinterpret_cast<int*>(smem + kDkvOffList);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int pr = blockIdx.x % p.T, bh = blockIdx.x / p.T;   // key pair = blocks 2pr, 2pr+1 (keys 128 pr ..)
-    const long long pb = static_cast<long long>(bh) * p.T + pr;
+    // key pair = blocks 2pr, 2pr+1 (keys 128 pr .. of the sequence) of group kv; its
+    // slot is that of the sequence's local tile pr
+    const int pslot = blockIdx.x % p.T, kv = blockIdx.x / p.T;
+    if (pslot >= bwd_slots_in_use(p.tiles, p.ntiles, p.T)) return;   // an unused slot (packed sequences)
+    const BwdTile ptg = bwd_tile(p, pslot);
+    const int pr = ptg.t;
+    const int cseq = (ptg.n + kKeys - 1) / kKeys;
+    const long long pb = static_cast<long long>(kv) * p.T + pslot;
     const int off = __ldg(p.inv_off + pb);
     const int cnt = min(__ldg(p.inv_off + pb + 1) - off, kDkvListCap - 1);
     const int nq = cnt + 1;                                    // the diagonal tile pr first
+    // work items: every visiting query tile once for each of the group's G query
+    // heads (item k: tile list[k / G] of head kv G + k % G)
+    const int G = p.G;
+    const int nitems = nq * G;
     if (t == 0) {
         mbar_init(&ctl.kv_full, 1);
         for (int s = 0; s < 2; ++s) {
@@ -524,14 +608,16 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     // the query tiles: diagonal first, then the others in ascending order (a
     // fixed summation order); rank sort of the inverted list in shared memory
     // list[q]: index into raw / rawpos of the q-th query tile (slot 0: the diagonal
-    // tile, which visits 2pr, 2pr+1 right after its union list)
+    // tile, which visits 2pr, 2pr+1 right after its union list); raw holds the
+    // tiles' indices within the sequence (so packed sequences sum in the order of
+    // a batch of the same data)
     int* raw = list + kDkvListCap;
     int* rawpos = raw + kDkvListCap;
     if (t == 0) {
         list[0] = 0;
         raw[0] = pr;
         const int Upr = __ldg(p.union_cnt + pb);
-        rawpos[0] = (Upr + 1) | ((2 * pr + 1 < p.C ? Upr + 2 : 0) << 16);
+        rawpos[0] = (Upr + 1) | ((2 * pr + 1 < cseq ? Upr + 2 : 0) << 16);
     }
     for (int k = t; k < cnt; k += kThreadsD) {
         raw[1 + k] = __ldg(p.inv_tiles + off + k);
@@ -550,29 +636,34 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     const uint32_t tmem = ctl.tmem_base;
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
     float* info = reinterpret_cast<float*>(smem + kDkvOffInfo);
-    const int nh = 2 * nq;   // 64-row halves of the query tiles
+    const int nh = 2 * nitems;   // 64-row halves of the items
 
     if (warp == 5) {
         // ---- row information of query tile q, up to three tiles ahead: per row
         // the offsets (log g - LSE) of blocks 2pr, 2pr+1 that pass 1 wrote, and -Delta
         const int il = lane;
-        for (int q = 0; q < nq; ++q) {
-            const int s = q % kInfoStages;
-            if (q >= kInfoStages && !mbar_wait(&ctl.info_empty[s], ((q - kInfoStages) / kInfoStages) & 1, wc, kSleepNs))
+        for (int it = 0; it < nitems; ++it) {
+            const int s = it % kInfoStages;
+            if (it >= kInfoStages &&
+                !mbar_wait(&ctl.info_empty[s], ((it - kInfoStages) / kInfoStages) & 1, wc, kSleepNs))
                 break;
             float* inf = info + s * 4 * kRows;
-            const int tq = raw[list[q]];
+            const int q = it / G;
+            const int bhq = kv * G + it % G;   // the item's query head
+            const int tq = raw[list[q]];       // the query tile within the sequence, and its slot
+            const int gq = p.tiles == nullptr ? tq : pslot - __ldg(p.tile_off + pr) + __ldg(p.tile_off + tq);
             const int ps = rawpos[list[q]];
             const int j0 = (ps & 0xffff) - 1, j1 = (ps >> 16) - 1;
-            const long long tbq = static_cast<long long>(bh) * p.T + tq;
+            const long long tbq = static_cast<long long>(bhq) * p.T + gq;
             const long long so = static_cast<long long>(__ldg(p.slot_off + tbq)) * kRows;
+            const long long drow = static_cast<long long>(bhq) * p.N + ptg.base + tq * kRows;
 #pragma unroll
             for (int rr = 0; rr < kRows / kInfoLanes; ++rr) {
                 const int r = il + rr * kInfoLanes;
-                const int i = tq * kRows + r;
+                const int i = tq * kRows + r;   // row index within the sequence
                 inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : -CUDART_INF_F;
                 inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : -CUDART_INF_F;
-                inf[2 * kRows + r] = i < p.N ? -__ldcg(p.delta + static_cast<long long>(bh) * p.N + i) : 0.f;
+                inf[2 * kRows + r] = i < ptg.n ? -__ldcg(p.delta + drow + r) : 0.f;
             }
             mbar_arrive_warp(&ctl.info_full[s]);
         }
@@ -582,18 +673,21 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             // query tile q into stage q & 1 once both products of tile q - 2 are done
             mbar_arrive_expect_tx(&ctl.kv_full, 2 * kPairBytes);
             for (int h = 0; h < 2; ++h) {
-                tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
-                tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64, pr * 2 * kKeys, bh);
+                tma_load_3d(smem + h * (2 * kKeys * 128), &mapK2, &ctl.kv_full, h * 64, ptg.base + pr * 2 * kKeys, kv);
+                tma_load_3d(smem + kDkvOffV + h * (2 * kKeys * 128), &mapV2, &ctl.kv_full, h * 64,
+                            ptg.base + pr * 2 * kKeys, kv);
             }
-            for (int q = 0; q < nq; ++q) {
-                const int s = q & 1;
-                if (q >= 2 && !mbar_wait(&ctl.q_empty[s], ((q - 2) >> 1) & 1, wc, kSleepNs)) break;
-                const int tq = raw[list[q]];
+            for (int it = 0; it < nitems; ++it) {
+                const int s = it & 1;
+                if (it >= 2 && !mbar_wait(&ctl.q_empty[s], ((it - 2) >> 1) & 1, wc, kSleepNs)) break;
+                const int tq = raw[list[it / G]];
+                const int row = ptg.base + tq * kRows;
+                const int bhq = kv * G + it % G;
                 uint8_t* st = smem + kDkvOffQ + s * 2 * kQBytes;
                 mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
                 for (int h = 0; h < 2; ++h) {
-                    tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, tq * kRows, bh);
-                    tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, tq * kRows, bh);
+                    tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, row, bhq);
+                    tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, row, bhq);
                 }
             }
         }
@@ -667,7 +761,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     } else {
         // ---- keys: thread = key of the pair (TMEM lane)
         const int key = t;
-        const int kg = pr * 2 * kKeys + key;      // global key index
+        const int kl = pr * 2 * kKeys + key;      // key index within the sequence
         const int kblk = key >> 6;                // 0: block 2pr, 1: block 2pr + 1
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
         bool ok = true;
@@ -685,9 +779,9 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             tmem_ld32(buf + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
             tmem_wait_ld();
             uint32_t pp[32], dd[32];
-            // In the diagonal tile (the first of the list) the rows of half h have
-            // block 2pr + h as their own block: keys of that block are causal.
-            const bool causal = q == 0 && h == kblk;
+            // In the diagonal tile (the first of the list, items 0 .. G-1) the rows of
+            // half h have block 2pr + h as their own block: keys of that block are causal.
+            const bool causal = q < G && h == kblk;
             const float2* off2 = reinterpret_cast<const float2*>(inf + kblk * kRows + h * 64);
             const float2* nd2p = reinterpret_cast<const float2*>(inf + 2 * kRows + h * 64);
             const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2);
@@ -719,8 +813,8 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
         }
         if (ok && mbar_wait_warp(&ctl.fin, 0, wc, kSleepNs)) {
             tc_fence_after();
-            const bool kv = kg < p.N;
-            const long long koff = static_cast<long long>(bh) * p.N + kg;
+            const bool kv_in = kl < ptg.n;
+            const long long koff = static_cast<long long>(kv) * p.N + ptg.base + kl;
 #pragma unroll 1
             for (int which = 0; which < 2; ++which) {
                 bf16* dst_row = (which == 0 ? p.dV : p.dK) + koff * kD;
@@ -730,7 +824,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                     uint32_t o[32];
                     tmem_ld32(lane_addr + (which == 0 ? kTmemDV : kTmemDK) + cc * 32, o);
                     tmem_wait_ld();
-                    if (kv) {
+                    if (kv_in) {
                         uint4* dst = reinterpret_cast<uint4*>(dst_row + cc * 32);
 #pragma unroll
                         for (int q2 = 0; q2 < 4; ++q2)
@@ -762,14 +856,30 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
 template <int NCH>
 __global__ void __launch_bounds__(256)
 bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg, const float* dlogg, float* ds,
-              int N, int C, int topk, int train, int chunks) {
+              int N, int C, int topk, int train, int chunks, const int4* tiles, const int* ntiles) {
     extern __shared__ float dsh[];   // per warp: C floats (the row's kept dlogg, scattered)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // CTA = (head, run of blockDim / 32 rows of it): one division per CTA
+    // CTA = (head, run of blockDim / 32 rows of it): one division per CTA.
+    // Packed sequences: chunks = tile slots x runs per 128-row tile, and i is
+    // the row's index within its sequence (its blocks count from there).
     const int bh = static_cast<int>(blockIdx.x / static_cast<unsigned>(chunks));
-    const int i = static_cast<int>(blockIdx.x - static_cast<unsigned>(bh) * chunks) * (blockDim.x >> 5) + warp;
-    if (i >= N) return;              // no block-wide synchronisation below
-    const long long w = static_cast<long long>(bh) * N + i;
+    const int run = static_cast<int>(blockIdx.x - static_cast<unsigned>(bh) * chunks);
+    int i, row;
+    if (tiles == nullptr) {
+        i = run * (blockDim.x >> 5) + warp;
+        row = i;
+        if (i >= N) return;          // no block-wide synchronisation below
+    } else {
+        const int per_tile = kRows / (blockDim.x >> 5);
+        const int g = run / per_tile;
+        if (g >= __ldg(ntiles)) return;
+        const int4 v = __ldg(tiles + g);
+        const int r = (run - g * per_tile) * (blockDim.x >> 5) + warp;
+        i = v.y * kRows + r;
+        row = v.x + i;
+        if (i >= v.z) return;
+    }
+    const long long w = static_cast<long long>(bh) * N + row;
     float* add = dsh + warp * C;
     const int c = i >> 6;
     const int nsel = train ? min(topk, c) : 0;
@@ -846,7 +956,7 @@ const int kBwdMaxTiles = kDkvListCap - 1;
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total) {
     const long long tiles = static_cast<long long>(a.BH) * a.T;
     const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
-    bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
+    bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.N, a.G, a.tiles, a.ntiles);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.slot_off, nullptr, tiles);
     if (total == nullptr) return cudaGetLastError();   // the caller's buffer holds the upper bound
     int32_t host = 0;
@@ -861,6 +971,12 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         *err = "backward: head dim must be 128";
         return cudaErrorInvalidValue;
     }
+    const int G = a.G > 0 ? a.G : 1;
+    if (a.BH % G != 0 || (G > 1 && a.dlogg_heads == nullptr)) {
+        *err = "backward: query heads must fill whole KV groups";
+        return cudaErrorInvalidValue;
+    }
+    const int BHkv = a.BH / G;   // KV groups x batch
     {
         cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel), kDqSmem);
         if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel), kDkvSmem);
@@ -869,10 +985,10 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     CUtensorMap mq, mdo, mk, mv, mk2, mv2;
     if (make_tmap_bf16_3d(&mq, a.Q, kD, a.N, a.BH, 64, kRows) != 0 ||
         make_tmap_bf16_3d(&mdo, a.dO, kD, a.N, a.BH, 64, kRows) != 0 ||
-        make_tmap_bf16_3d(&mk, a.K, kD, a.N, a.BH, 64, kKeys) != 0 ||
-        make_tmap_bf16_3d(&mv, a.V, kD, a.N, a.BH, 64, kKeys) != 0 ||
-        make_tmap_bf16_3d(&mk2, a.K, kD, a.N, a.BH, 64, 2 * kKeys) != 0 ||
-        make_tmap_bf16_3d(&mv2, a.V, kD, a.N, a.BH, 64, 2 * kKeys) != 0) {
+        make_tmap_bf16_3d(&mk, a.K, kD, a.N, BHkv, 64, kKeys) != 0 ||
+        make_tmap_bf16_3d(&mv, a.V, kD, a.N, BHkv, 64, kKeys) != 0 ||
+        make_tmap_bf16_3d(&mk2, a.K, kD, a.N, BHkv, 64, 2 * kKeys) != 0 ||
+        make_tmap_bf16_3d(&mv2, a.V, kD, a.N, BHkv, 64, 2 * kKeys) != 0) {
         *err = "backward tensor maps";
         return cudaErrorInvalidValue;
     }
@@ -887,61 +1003,79 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     p.dQ = static_cast<bf16*>(a.dQ);
     p.dK = static_cast<bf16*>(a.dK);
     p.dV = static_cast<bf16*>(a.dV);
-    p.dlogg = a.dlogg;
+    p.dlogg = G > 1 ? a.dlogg_heads : a.dlogg;   // pass 1 writes per query head
     p.delta = a.delta;
     p.inv_off = a.inv_off;
     p.inv_tiles = a.inv_tiles;
     p.inv_pos = a.inv_pos;
     p.slot_off = a.slot_off;
     p.offs = a.offs;
+    p.tiles = a.tiles;
+    p.ntiles = a.ntiles;
+    p.tile_off = a.tile_off;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
+    p.G = G;
     p.sm_scale = a.sm_scale;
     p.scale_log2 = a.sm_scale * kLog2eB;
     p.status = env.status;
     p.limit = env.limit;
-    const long long tiles = static_cast<long long>(a.BH) * a.T;
+    const long long tiles = static_cast<long long>(a.BH) * a.T;        // (query head, tile)
+    const long long gtiles = static_cast<long long>(BHkv) * a.T;       // (KV group, tile or key pair)
     if (tiles > 0x7fffffffLL) { *err = "backward: too many tiles"; return cudaErrorInvalidValue; }
     // pass 1 (also writes Delta for pass 2); both halves of a row add into dlogg
-    cudaError_t e0 = cudaMemsetAsync(a.dlogg, 0, static_cast<size_t>(a.BH) * a.N * (a.topk > 0 ? a.topk : 1) * 4,
-                                     env.stream);
+    const long long per_head = static_cast<long long>(a.N) * (a.topk > 0 ? a.topk : 1);
+    cudaError_t e0 = cudaMemsetAsync(p.dlogg, 0, static_cast<size_t>(a.BH) * per_head * 4, env.stream);
     if (e0 != cudaSuccess) { *err = "backward dlogg"; return e0; }
     bwd_dq_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
-    // inverted lists
-    e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(tiles) * 4, env.stream);
+    // inverted lists of the KV groups' union lists
+    e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(gtiles) * 4, env.stream);
     if (e != cudaSuccess) { *err = "backward list counts"; return e; }
-    const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
-    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cnt, a.BH, a.T, a.C);
-    bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, tiles);
+    const unsigned gb = static_cast<unsigned>((gtiles + 255) / 256);
+    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cnt, BHkv, a.T, a.C, a.tiles,
+                                                      a.ntiles, a.tile_off);
+    bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, gtiles);
     bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cursor, a.inv_tiles, a.inv_pos,
-                                                     a.BH, a.T, a.C);
+                                                     BHkv, a.T, a.C, a.tiles, a.ntiles, a.tile_off);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
-    // pass 2
-    bwd_dkv_kernel<<<static_cast<unsigned>(tiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+    // pass 2: one CTA per (KV group, key pair)
+    bwd_dkv_kernel<<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
+    if (G > 1 && a.topk > 0) {
+        const long long total = static_cast<long long>(BHkv) * per_head;
+        bwd_dlogg_sum_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, env.stream>>>(
+            a.dlogg_heads, a.dlogg, per_head, total, G);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) { *err = "backward gate-gradient sum"; return e; }
+    } else if (G > 1) {
+        e = cudaMemsetAsync(a.dlogg, 0, static_cast<size_t>(BHkv) * per_head * 4, env.stream);
+        if (e != cudaSuccess) { *err = "backward dlogg"; return e; }
+    }
     if (a.scores != nullptr && a.ds != nullptr && a.topk > 0) {
-        // one warp per row, at most 32 KB of shared memory per CTA
-        const int wpc = max(1, min(8, 8192 / a.C));
+        // one warp per row, at most 32 KB of shared memory per CTA; packed
+        // sequences: a power of two of warps, so that runs tile 128 rows
+        int wpc = max(1, min(8, 8192 / a.C));
+        if (a.tiles != nullptr) wpc = 1 << (31 - __builtin_clz(static_cast<unsigned>(wpc)));
         const size_t sh = static_cast<size_t>(wpc) * a.C * sizeof(float);
-        const int chunks = (a.N + wpc - 1) / wpc;
-        const unsigned grid = static_cast<unsigned>(static_cast<long long>(a.BH) * chunks);
+        const int chunks = a.tiles != nullptr ? a.T * (kRows / wpc) : (a.N + wpc - 1) / wpc;
+        const unsigned grid = static_cast<unsigned>(static_cast<long long>(BHkv) * chunks);
         const int train = a.mode == 0 ? 1 : 0;
         if (a.C <= 128)
             bwd_ds_kernel<4><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                 a.C, a.topk, train, chunks);
+                                                                 a.C, a.topk, train, chunks, a.tiles, a.ntiles);
         else if (a.C <= 384)
             bwd_ds_kernel<12><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                  a.C, a.topk, train, chunks);
+                                                                  a.C, a.topk, train, chunks, a.tiles, a.ntiles);
         else
             bwd_ds_kernel<0><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                 a.C, a.topk, train, chunks);
+                                                                 a.C, a.topk, train, chunks, a.tiles, a.ntiles);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     } else if (a.ds != nullptr) {
-        e = cudaMemsetAsync(a.ds, 0, static_cast<size_t>(a.BH) * a.N * a.C * 4, env.stream);
+        e = cudaMemsetAsync(a.ds, 0, static_cast<size_t>(BHkv) * a.N * a.C * 4, env.stream);
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     }
     return cudaSuccess;

@@ -1260,7 +1260,8 @@ constexpr int kStatusBadInput = 1;   // == SAS_ERR_INVALID_ARG
 // order only schedules work).  Bad offsets set the status word and leave no
 // tiles.
 __global__ void __launch_bounds__(1024) varlen_tiles_kernel(const int32_t* cu, int S, int Ncap, int max_len,
-                                                            int tmax, int4* tiles, int* ntiles, int* status) {
+                                                            int tmax, int4* tiles, int* ntiles, int* tile_off,
+                                                            int* status) {
     extern __shared__ int vsh[];   // hist[tmax + 2], cnt_gt[tmax + 2], off[tmax + 2], next[tmax + 2]
     int* hist = vsh;
     int* gt = hist + tmax + 2;     // gt[t] = number of sequences with T_s > t
@@ -1296,6 +1297,10 @@ __global__ void __launch_bounds__(1024) varlen_tiles_kernel(const int32_t* cu, i
         *ntiles = o;
     }
     __syncthreads();
+    // first slot of every local tile index: sequence s of rank r keeps its
+    // tile t at slot tile_off[t] + r (the backward maps tiles of a sequence
+    // to one another through it)
+    for (int t = tid; t <= tmax; t += blockDim.x) tile_off[t] = off[t];
     for (int s = tid; s < S; s += blockDim.x) {
         const int b0 = __ldg(cu + s), n = __ldg(cu + s + 1) - b0;
         const int T = (n + kRows - 1) / kRows;
@@ -1308,7 +1313,7 @@ __global__ void __launch_bounds__(1024) varlen_tiles_kernel(const int32_t* cu, i
 }  // namespace
 
 cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len, int4* tiles, int* ntiles,
-                                const KernelEnv& env) {
+                                int* tile_off, const KernelEnv& env) {
     const int tmax = (max_len + kRows - 1) / kRows;
     const size_t smem = static_cast<size_t>(4) * (tmax + 2) * sizeof(int);
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
@@ -1316,7 +1321,8 @@ cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len,
         cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(varlen_tiles_kernel), smem);
         if (e != cudaSuccess) return e;
     }
-    varlen_tiles_kernel<<<1, 1024, smem, env.stream>>>(cu, S, Ncap, max_len, tmax, tiles, ntiles, env.status);
+    varlen_tiles_kernel<<<1, 1024, smem, env.stream>>>(cu, S, Ncap, max_len, tmax, tiles, ntiles, tile_off,
+                                                       env.status);
     return cudaGetLastError();
 }
 

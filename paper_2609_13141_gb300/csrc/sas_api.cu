@@ -128,6 +128,7 @@ struct sas_handle {
     bool varlen = false;            // packed sequences: T = tile slots, C from max_seqlen
     int4* tiles = nullptr;          // packed sequences' tile table [T] and its count
     int* ntiles = nullptr;
+    int* tile_off = nullptr;    // first slot of every local tile index (see launch_varlen_tiles)
     // workspace
     void* Kt = nullptr;         // bf16 [BH][max(F,1)][d_sel]
     int32_t* union_idx = nullptr;
@@ -146,7 +147,7 @@ struct sas_handle {
     float* bwd_delta = nullptr;
     int32_t* bwd_inv = nullptr;     // counts, cursors, offsets, slot offsets
     int32_t* bwd_tiles = nullptr;   // inverted lists: tiles, then block positions
-    float* bwd_dlogg = nullptr;
+    float* bwd_dlogg = nullptr;     // GQA: per query head [BH][N][topk], then per group [BHkv][N][topk]
     float* bwd_offs = nullptr;      // per-row offsets of every visited block (pass 1 -> pass 2)
     size_t bwd_offs_bytes = 0;
     bool bwd_offs_bound = false;    // sized for the upper bound: no per-call read-back
@@ -309,6 +310,7 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
         if (e == cudaSuccess) e = alloc(&h->tiles, static_cast<size_t>(h->T) * sizeof(int4));
         if (e == cudaSuccess) e = alloc(&h->ntiles, 16);
         if (e == cudaSuccess) e = cudaMemset(h->ntiles, 0, 16);
+        if (e == cudaSuccess) e = alloc(&h->tile_off, static_cast<size_t>((max_len + 127) / 128 + 2) * 4);
     }
     if (h->full) {
         if (e == cudaSuccess) e = alloc(&h->full_lse, rows * 4);
@@ -339,6 +341,7 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->sel_logg);
     cudaFree(h->tiles);
     cudaFree(h->ntiles);
+    cudaFree(h->tile_off);
     cudaFree(h->status);
     cudaFree(h->sched);
     cudaFree(h->full_lse);
@@ -481,7 +484,8 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     float* out_lg = sel_logg ? sel_logg : h->sel_logg;
     const int max_len = c.max_seqlen > 0 ? c.max_seqlen : c.N;
     // the tile table of the packed sequences (device offsets, checked on the device)
-    cudaError_t e = sas::launch_varlen_tiles(cu_seqlens, num_seqs, c.N, max_len, h->tiles, h->ntiles, env);
+    cudaError_t e =
+        sas::launch_varlen_tiles(cu_seqlens, num_seqs, c.N, max_len, h->tiles, h->ntiles, h->tile_off, env);
     if (e != cudaSuccess) return cuda_fail(h, e, "packed-sequence tile table");
     h->launches += 1;
     if (learned) {
@@ -584,10 +588,11 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     if (c.d != 128) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports d = 128");
     if (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER)
         return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
-    if (h->G != 1) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports Hkv = H");
-    if (h->varlen) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports [B, H, N, d] batches");
     if (h->full) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports the sparse scope");
-    if (h->T > sas::kBwdMaxTiles) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports N <= 262016");
+    // query tiles of one sequence (a key pair's inverted list holds at most that many)
+    const int tseq = h->varlen ? (h->C + 1) / 2 : h->T;
+    if (tseq > sas::kBwdMaxTiles)
+        return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports sequences of at most 262016 tokens");
     if (dscores) {
         if (c.selector != SAS_SEL_SCORES_GIVEN || !scores)
             return fail(h, SAS_ERR_INVALID_ARG, "dscores needs given scores (SCORES_GIVEN)");
@@ -602,10 +607,13 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         if (e == cudaSuccess) e = alloc(&h->bwd_delta, rows * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_inv, (4 * tiles + 2) * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_tiles, 2 * tiles * pairs * 4);
-        if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, rows * (c.topk > 0 ? c.topk : 1) * 4);
-        // offsets of pass 1 for pass 2: a tile visits at most 2t + 2 blocks, so a head
-        // needs at most T (T + 1) slots of 128 rows; held whole when that fits in 8 GiB
-        const size_t bound = tiles * static_cast<size_t>(h->T + 1) * 128 * 4;
+        const size_t dl_rows = rows + (h->G > 1 ? static_cast<size_t>(h->BHkv) * c.N : 0);
+        if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, dl_rows * (c.topk > 0 ? c.topk : 1) * 4);
+        // offsets of pass 1 for pass 2: local tile t visits at most 2t + 2 blocks, so a
+        // head needs at most T (T + 1) slots of 128 rows (packed sequences: 2 tseq per
+        // tile slot); held whole when that fits in 8 GiB
+        const size_t per_tile = h->varlen ? 2 * static_cast<size_t>(tseq) : static_cast<size_t>(h->T + 1);
+        const size_t bound = tiles * per_tile * 128 * 4;
         if (e == cudaSuccess && bound <= (static_cast<size_t>(8) << 30)) {
             cudaError_t eb = alloc(&h->bwd_offs, bound);
             if (eb == cudaSuccess) {
@@ -633,7 +641,9 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.sel_logg = sel_logg ? sel_logg : h->sel_logg;
     a.scores = dscores ? scores : nullptr;
     a.dQ = dQ; a.dK = dK; a.dV = dV;
-    a.dlogg = dlogg ? dlogg : h->bwd_dlogg;
+    // GQA: pass 1 writes each query head's d(log g); the group's is their sum
+    a.dlogg_heads = h->G > 1 ? h->bwd_dlogg : nullptr;
+    a.dlogg = dlogg ? dlogg : h->bwd_dlogg + (h->G > 1 ? rows * (c.topk > 0 ? c.topk : 1) : 0);
     a.ds = dscores;
     a.delta = h->bwd_delta;
     a.inv_cnt = h->bwd_inv;
@@ -643,7 +653,14 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.inv_tiles = h->bwd_tiles;
     a.inv_pos = h->bwd_tiles + tiles * static_cast<size_t>(h->T < h->C ? h->T : h->C);
     a.N = c.N; a.C = h->C; a.T = h->T; a.BH = h->BH; a.topk = c.topk; a.mode = c.mode; a.d = c.d;
+    a.G = h->G;
     a.sm_scale = h->sm_scale;
+    if (h->varlen) {
+        // the tile table of the last sas_attention_fwd_varlen (its union lists are per slot)
+        a.tiles = h->tiles;
+        a.ntiles = h->ntiles;
+        a.tile_off = h->tile_off;
+    }
     const sas::KernelEnv env{s, h->status, h->limit};
     const char* err = "";
     // slots of the per-row offsets pass 1 hands to pass 2: their number depends on
@@ -664,7 +681,10 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.offs = h->bwd_offs;
     e = timed_launch(h, 6, s, [&] { return sas::launch_attn_bwd(a, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
-    h->launches += 2 + ((a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 5 : 4);   // all its kernels
+    // all its kernels: slot count and scan, pass 1, the inverted lists (count, scan,
+    // fill), pass 2, the group sum of d(log g) and the score gradient
+    h->launches += 7 + ((h->G > 1 && c.topk > 0) ? 1 : 0) +
+                   ((a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 1 : 0);
     return SAS_OK;
 }
 

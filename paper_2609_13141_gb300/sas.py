@@ -381,12 +381,27 @@ class SasLayer:
 
     def attention_bwd(self, Q, K, V, O, LSE, dO, scores=None, sel_idx=None, sel_logg=None, want_ds=False,
                       stream=None):
-        """Returns (dQ, dK, dV, dlogg, dscores); dscores only with want_ds (given scores)."""
+        """Returns (dQ, dK, dV, dlogg, dscores); dscores only with want_ds (given scores).
+        With Hkv < H, dK, dV, dlogg and dscores are per KV group (sums over its heads)."""
         dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
-        dlogg = torch.empty(self.B, self.H, self.N, max(self.topk, 1), device=Q.device, dtype=torch.float32)
+        dlogg = torch.empty(self.B, self.Hkv, self.N, max(self.topk, 1), device=Q.device, dtype=torch.float32)
         ds = None
         if want_ds:
-            ds = torch.empty(self.B, self.H, self.N, -(-self.N // 64), device=Q.device, dtype=torch.float32)
+            ds = torch.empty(self.B, self.Hkv, self.N, -(-self.N // 64), device=Q.device, dtype=torch.float32)
+        sas_attention_bwd(self.h, Q, K, V, O, LSE, dO, dQ, dK, dV, scores, sel_idx, sel_logg, dlogg, ds, stream)
+        return dQ, dK, dV, dlogg, ds
+
+    def attention_bwd_varlen(self, Q, K, V, O, LSE, dO, scores=None, sel_idx=None, sel_logg=None, want_ds=False,
+                             stream=None):
+        """Backward of the last attention_varlen on this handle: Q, O, dO [H, N, d],
+        K, V [Hkv, N, d].  Returns (dQ, dK, dV, dlogg [Hkv, N, topk], dscores [Hkv, N, C]
+        or None); rows past cu[-1] keep the zero fill of the tensors made here."""
+        dev = Q.device
+        dQ, dK, dV = torch.zeros_like(Q), torch.zeros_like(K), torch.zeros_like(V)
+        dlogg = torch.zeros(self.Hkv, self.N, max(self.topk, 1), device=dev, dtype=torch.float32)
+        ds = None
+        if want_ds:
+            ds = torch.zeros(self.Hkv, self.N, scores.shape[-1], device=dev, dtype=torch.float32)
         sas_attention_bwd(self.h, Q, K, V, O, LSE, dO, dQ, dK, dV, scores, sel_idx, sel_logg, dlogg, ds, stream)
         return dQ, dK, dV, dlogg, ds
 

@@ -78,6 +78,16 @@ def test_gqa_and_full_scope_outputs():
     sl, gl = guarded((B, Hkv, N, K), torch.float32)
     sas.sas_attention_fwd(layer.h, Q, Kk, V, O, S, LSE=L, sel_idx=si, sel_logg=sl)
     _check(gO, gL, gi, gl)
+    # the GQA backward: dQ per query head, the rest per KV group
+    dO = synth.normal((B, H, N, d), 6).to(torch.bfloat16).to(DEV)
+    dQ, gq = guarded((B, H, N, d), torch.bfloat16)
+    dK, gk = guarded((B, Hkv, N, d), torch.bfloat16)
+    dV, gv = guarded((B, Hkv, N, d), torch.bfloat16)
+    dl, gdl = guarded((B, Hkv, N, K), torch.float32)
+    ds, gds = guarded((B, Hkv, N, -(-N // 64)), torch.float32)
+    sas.sas_attention_bwd(layer.h, Q, Kk, V, O, L, dO, dQ, dK, dV, S, si, sl, dl, ds)
+    _check(gq, gk, gv, gdl, gds)
+    assert sas.sas_get_device_status(layer.h) == 0
     layer.close()
     full = sas.SasLayer(B, H, N, d, K, Hkv=Hkv, scope=sas.SAS_SCOPE_FULL)
     O, gO = guarded((B, H, N, d), torch.bfloat16)
@@ -101,6 +111,16 @@ def test_varlen_outputs():
     sl, gl = guarded((Hkv, cap, K), torch.float32)
     sas.sas_attention_fwd_varlen(layer.h, cu, Q, Kk, V, S, O, L, si, sl)
     _check(gO, gL, gi, gl)
+    # the packed backward
+    dO = synth.normal((H, cap, d), 7).to(torch.bfloat16).to(DEV)
+    dQ, gq = guarded((H, cap, d), torch.bfloat16)
+    dK, gk = guarded((Hkv, cap, d), torch.bfloat16)
+    dV, gv = guarded((Hkv, cap, d), torch.bfloat16)
+    dl, gdl = guarded((Hkv, cap, K), torch.float32)
+    ds, gds = guarded((Hkv, cap, S.shape[-1]), torch.float32)
+    sas.sas_attention_bwd(layer.h, Q, Kk, V, O, L, dO, dQ, dK, dV, S, si, sl, dl, ds)
+    _check(gq, gk, gv, gdl, gds)
+    assert sas.sas_get_device_status(layer.h) == 0
     layer.close()
 
 

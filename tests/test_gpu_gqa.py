@@ -89,19 +89,6 @@ def test_qwen3_4b_shaped_prefill_sampled_rows():
         P.check_selection_rows(gi, P.f64(S[bi, hi // 4])[rows], rows, topk)
 
 
-def test_gqa_backward_is_refused():
-    layer = sas.SasLayer(1, 4, 256, 128, 2, Hkv=2)
-    dev = torch.device("cuda:0")
-    Q = torch.zeros(1, 4, 256, 128, device=dev, dtype=torch.bfloat16)
-    K = torch.zeros(1, 2, 256, 128, device=dev, dtype=torch.bfloat16)
-    S = torch.zeros(1, 2, 256, 4, device=dev)
-    O, LSE, si, sl = layer.attention(Q, K, K, scores=S)
-    with pytest.raises(sas.SasError) as e:
-        layer.attention_bwd(Q, K, K, O, LSE, O, scores=S, sel_idx=si, sel_logg=sl)
-    assert e.value.status == sas.SAS_ERR_UNSUPPORTED
-    layer.close()
-
-
 @pytest.mark.parametrize("B,Hq,Hkv,N,d,d_sel,topk", [
     (1, 8, 2, 1000, 128, 128, 4),     # G = 4
     (2, 4, 2, 700, 64, 64, 3),        # G = 2, d = 64
