@@ -28,7 +28,7 @@
 //   * learned selector: on the tensor cores, one thread first projects the
 //     tile's 128 queries (q~ = Q Wq^T into TMEM; under GQA q~ = Wq_g [q_0; ...;
 //     q_{G-1}], accumulated over G rounds of one head each); the row threads round q~
-//     to bf16 into shared memory as the A operand of the score product; then
+//     to bf16 in TMEM, where it is the A operand of the score product; then
 //     s = q~ Kt^T / sqrt(d_sel) runs chunk by chunk (M=128, N=64) over
 //     64-block chunks of projected summaries in a double-buffered TMA ring,
 //     and the row threads read their scores back with tcgen05.ld.
@@ -322,18 +322,21 @@ __device__ __forceinline__ float log_sigmoid(float s) {
     return -(fmaxf(-s, 0.f) + log1pf(expf(-fabsf(s))));
 }
 
-// Output staging: each row's K entries are written to shared memory (row
-// stride K + 1 words, so a warp's rows hit distinct banks) and then copied to
-// global memory with coalesced stores.
+// Output staging: each row's K entries are written to shared memory and then
+// copied to global memory with coalesced stores.  Entry e of row r sits at
+// r * stride + e * es: row-major with a row stride of K + 1 words (scores
+// given) or entry-major (learned selector); either way a warp's rows hit
+// distinct banks.
 struct Staging {
     int32_t* idx;
     float* lg;
     int stride;
+    int es;
 };
 
 __device__ __forceinline__ void stage_entry(const Staging& st, int r, int e, int m, float lg) {
-    st.idx[r * st.stride + e] = m;
-    st.lg[r * st.stride + e] = lg;
+    st.idx[r * st.stride + e * st.es] = m;
+    st.lg[r * st.stride + e * st.es] = lg;
 }
 
 // Copies the staged rows (the tile's first `rows`, from row `row0` of the
@@ -348,8 +351,8 @@ __device__ __forceinline__ void copy_out(const Staging& st, const SelParams& p, 
     const int dr = nthreads / K, de = nthreads - dr * K;
     const bool sigm = p.gate_act == 1;
     for (int q = tid; q < rows * K; q += nthreads) {
-        const int m = st.idx[r * st.stride + e];
-        const float lg = st.lg[r * st.stride + e];
+        const int m = st.idx[r * st.stride + e * st.es];
+        const float lg = st.lg[r * st.stride + e * st.es];
         p.sel_idx[base + q] = m;
         p.sel_logg[base + q] = (sigm && m >= 0) ? log_sigmoid(lg) : lg;
         r += dr;
@@ -460,7 +463,7 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
         ptr += smem_topk_bytes(K);
     }
     const Staging st{reinterpret_cast<int32_t*>(ptr), reinterpret_cast<float*>(ptr + size_t(kRows) * (K + 1) * 4),
-                     K + 1};
+                     K + 1, 1};
     ptr += staging_bytes(K);
     uint32_t* bitmap = reinterpret_cast<uint32_t*>(ptr);
     const int nwords = (p.C + 31) >> 5;
@@ -516,10 +519,15 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 // --------------------------------------------------------- learned selector
 
 // Shared memory of the learned-selector kernel (offsets from a 1024-aligned base):
-//   region A: the 128-row Q tile, overwritten by the bf16 projected queries q~;
+//   region A: the 128-row Q tile of each projection round; once the projection
+//             has run, the per-row score histograms (and, after pass B, a
+//             row's boundary-bin scores while pass C's list is resolved);
 //   region B: the tile's Wq[h], then (once the projection has run) the
 //             double-buffered 64-block chunks of projected block summaries;
-//   then the per-row score histograms, the output staging and the union bitmap.
+//   then the per-row lists of selected scores (entry-major: entry e of row r
+//   at e * 128 + r, so a warp's 32 rows hit 32 banks) and the union bitmap.
+// The projected queries q~ stay in TMEM, rounded to bf16, as the A operand of
+// the score products.
 //
 // Top-K without per-row replacement.  Replacing the worst kept entry whenever a
 // better score arrives diverges across the 32 rows of a warp (each row
@@ -528,58 +536,63 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 // per score (the score products are cheap to re-issue):
 //   pass A: the row's log-sum-exp, maximum, minimum and the first two moments
 //           of its scores;
-//   pass B: a histogram of the scores above a low threshold lo, in kBins - 1
-//           equal bins up to a high threshold hi and one bin above hi (lo and
+//   pass B: a histogram of the scores above a low threshold lo in kBins bins
+//           of width (hi - lo) / (kBins - 1), the last one open above (lo and
 //           hi placed from the moments where about K + 5 sqrt(K) and K -
 //           5 sqrt(K) scores of a normal sample lie above them); it locates
 //           the bin holding the K-th largest score;
-//   pass C: scores in bins above that bin are kept and staged in block order;
-//           the boundary bin's few scores are held in the row's histogram
-//           words (no longer needed) and the best R = K - (number above) of
-//           them, by (score descending, block ascending), join the list;
+//   pass C: every score in that bin or above is appended to the row's list in
+//           block order; afterwards the best R = K - (number above the bin)
+//           of the boundary bin's scores, by (score descending, block
+//           ascending), stay and the list is compacted in place;
 //   pass D: only if some row of the tile could not use A-C (its scores are
 //           too concentrated for the bins: equal scores, a crowded boundary bin):
 //           that row runs replace-the-worst over all its scores.
-// Every pass compares the same fp32 scores with the same bin arithmetic
-// (rounded steps, no contraction), so the passes agree on every score.
+// Every pass places a score in its bin with the same rounded operations (no
+// contraction), so the passes agree on every score.
+constexpr int kBins = 48;                           // histogram bins per row (pass B)
+constexpr int kBoundaryMax = 12;                    // boundary-bin scores a row's list holds beyond K
+constexpr size_t kHistBytes = size_t(kBins) * kRows * 4;
+// Bin arithmetic: v = 2^23 + (u - lo) / w, rounded to an integer by the add
+// itself (the float spacing at 2^23 is 1), holds the bin in the low bits of
+// its representation, so the bin's shared-memory word follows from the bits
+// of v with one integer multiply-add.
+constexpr float kBinMagic = 8388608.f;
+constexpr uint32_t kBinMagicBits = 0x4B000000u;
+constexpr float kBinTop = kBinMagic + float(kBins - 1);
+
 template <int D, int DS>
 struct SelProjCfg {
     static constexpr int Q_BYTES = kRows * D * 2;
-    static constexpr int QT_BYTES = kRows * DS * 2;
-    static constexpr int A_BYTES = Q_BYTES > QT_BYTES ? Q_BYTES : QT_BYTES;
+    static constexpr int A_BYTES = Q_BYTES > int(kHistBytes) ? Q_BYTES : int(kHistBytes);
     static constexpr int WQ_BYTES = DS * D * 2;
     static constexpr int KC_BYTES = 64 * DS * 2;   // 64 blocks per chunk
     static constexpr int B_BYTES = WQ_BYTES > 2 * KC_BYTES ? WQ_BYTES : 2 * KC_BYTES;
     static constexpr uint32_t IDESC_PROJ = idesc_bf16(kRows, DS, 0, 0);
     static constexpr uint32_t IDESC_S = idesc_bf16(kRows, 64, 0, 0);
-    static constexpr int TMEM_S = 128;            // score buffers at columns 128 and 192
+    static constexpr int TMEM_S = 128;            // score buffers at columns 128 and 192; q~ (bf16) at 0 .. DS/2
 };
 
-constexpr int kBins = 48;                           // histogram bins per row (pass B)
-constexpr int kBinWords = kBins / 2;                // two 16-bit counters per word
-constexpr int kBoundaryMax = kBinWords / 2;         // boundary-bin scores a row holds (in its dead histogram words)
-constexpr size_t kHistBytes = size_t(kBinWords) * kRows * 4;
 constexpr int kPassA = 0, kPassB = 1, kPassC = 2, kPassD = 3;
 constexpr int kPassW = 4;   // full training scope: write every score to the table
 constexpr int kRowAll = 0, kRowNormal = 1, kRowFail = 2;   // C_i <= K: keep all; thresholds; fallback
 
+__host__ __device__ constexpr size_t list_bytes(int K) { return size_t(K + kBoundaryMax) * kRows * 8; }
+
 template <int D, int DS>
 __host__ __device__ constexpr size_t proj_smem_bytes(int K, int C) {
-    return size_t(SelProjCfg<D, DS>::A_BYTES) + SelProjCfg<D, DS>::B_BYTES + kHistBytes + staging_bytes(K) +
-           bitmap_bytes(C);
+    return size_t(SelProjCfg<D, DS>::A_BYTES) + SelProjCfg<D, DS>::B_BYTES + list_bytes(K) + bitmap_bytes(C);
 }
 
 // Selection works on the raw products u = q~ . K~ (the scores are s = u / sqrt(d_sel),
 // an order-preserving scale): thresholds, bins and ties are all on u, and s is
 // formed only for the log-sum-exp and the emitted log-gates.
 //
-// Bin of a product at or above lo: floor((u - lo) / w) with w = (hi - lo) / (kBins - 1),
-// clamped to the top bin (everything from hi up).  Rounded steps without
-// contraction (the packed and the scalar forms round identically), so passes B
-// and C place every product in the same bin.
-__device__ __forceinline__ int bin_clamp(float x) { return min(kBins - 1, __float2int_rz(x)); }
-__device__ __forceinline__ float bin_x(float u, float neg_lo, float inv_w) {
-    return __fmul_rn(__fadd_rn(u, neg_lo), inv_w);
+// The bin value of a product at or above lo (monotone in u; the top bin takes
+// everything from about hi up).  Passes B and C form it with the packed
+// operations, which round exactly like these scalar ones.
+__device__ __forceinline__ float bin_v(float u, float neg_lo, float inv_w) {
+    return fminf(__fmaf_rn(__fadd_rn(u, neg_lo), inv_w, kBinMagic), kBinTop);
 }
 
 // The per-row state carried across the passes.
@@ -590,23 +603,18 @@ struct RowSel {
     float mn;                   // pass A: minimum
     float lo, inv_w;            // histogram origin and inverse bin width (lo = -inf: keep all, +inf: fallback)
     int mode;                   // kRowAll / kRowNormal / kRowFail
-    int bstar, hi_bin, nabove;  // after B: boundary bin, first bin kept whole, products above it
-    int pos;                    // pass C / D: entries staged so far
-    int nbc;                    // boundary products held (product, block) in the row's histogram words
+    float tb;                   // after B: bin value of the boundary bin (pass C takes v >= tb)
+    int hi_bin, nabove;         // after B: first bin kept whole, products above the boundary bin
+    int pos;                    // pass C / D: entries in the row's list
     float ws;                   // pass D: worst kept product, its slot
     int wpos;
 };
 
-// Shared-memory addresses of one row's staging entries and histogram words.
+// Shared-memory addresses of one row's list and histogram.
 struct RowAddr {
-    uint32_t idx, lg;           // staging entry 0 of the row (int32 block, fp32 product)
-    uint32_t hist;              // histogram word 0 of the row (word w at hist + w * kRows * 4)
+    uint32_t idx, lg;           // list entry 0 of the row (int32 block, fp32 product); entry e at + e * kRows * 4
+    uint32_t hist_off;          // the row's histogram word of bin b at hist_off + bits(v) * kRows * 4 (mod 2^32)
 };
-
-__device__ __forceinline__ void stage_score(const Staging& st, int r, int e, int m, float u) {
-    st.idx[r * st.stride + e] = m;
-    st.lg[r * st.stride + e] = u;
-}
 
 // Pass D state of a row: entries staged, worst kept product and its slot.
 struct FallbackState {
@@ -615,30 +623,30 @@ struct FallbackState {
     int wpos;
 };
 
-// Pass D, one product: the row's first K' products fill its staging row, a later
-// one replaces the worst kept entry (lowest product; among equal ones the highest
+// Pass D, one product: the row's first K' products fill its list, a later one
+// replaces the worst kept entry (lowest product; among equal ones the highest
 // block, which ranks last because ties go to the lower block) when strictly
 // larger.  Kept out of line: the fallback is rare, and its loops inlined at every
 // one of the 32 unrolled positions would crowd the hot passes out of the
-// instruction cache.
+// instruction cache.  Entry e of the row at idx[e * es], sc[e * es].
 __device__ __noinline__ FallbackState fallback_offer(FallbackState f, float u, int m, int32_t* idx, float* sc,
-                                                     int Kp) {
+                                                     int Kp, int es) {
     if (f.pos < Kp) {
-        idx[f.pos] = m;
-        sc[f.pos] = u;
+        idx[f.pos * es] = m;
+        sc[f.pos * es] = u;
         ++f.pos;
         if (f.pos < Kp) return f;
     } else if (u > f.ws) {
-        idx[f.wpos] = m;
-        sc[f.wpos] = u;
+        idx[f.wpos * es] = m;
+        sc[f.wpos * es] = u;
     } else {
         return f;
     }
     float ws = CUDART_INF_F;
     int wm = -1, wp = 0;
     for (int e = 0; e < Kp; ++e) {
-        const float se = sc[e];
-        const int me = idx[e];
+        const float se = sc[e * es];
+        const int me = idx[e * es];
         if (se < ws || (se == ws && me > wm)) {
             ws = se;
             wm = me;
@@ -650,29 +658,30 @@ __device__ __noinline__ FallbackState fallback_offer(FallbackState f, float u, i
     return f;
 }
 
-// Sorts a staged row's first n entries by block index (insertion sort: the rows
-// reaching it are sorted but for a short tail, or rare fallback rows).
+// Sorts a row's first n list entries by block index (insertion sort: rare
+// fallback rows).
 __device__ __forceinline__ void staged_sort_by_block(const Staging& st, int r, int n) {
     int32_t* idx = st.idx + r * st.stride;
     float* sc = st.lg + r * st.stride;
+    const int es = st.es;
     for (int a = 1; a < n; ++a) {
-        const int km = idx[a];
-        const float ks = sc[a];
+        const int km = idx[a * es];
+        const float ks = sc[a * es];
         int b = a - 1;
-        while (b >= 0 && idx[b] > km) {
-            idx[b + 1] = idx[b];
-            sc[b + 1] = sc[b];
+        while (b >= 0 && idx[b * es] > km) {
+            idx[(b + 1) * es] = idx[b * es];
+            sc[(b + 1) * es] = sc[b * es];
             --b;
         }
-        idx[b + 1] = km;
-        sc[b + 1] = ks;
+        idx[(b + 1) * es] = km;
+        sc[(b + 1) * es] = ks;
     }
 }
 
 // One half-chunk (32 products of blocks m0 .. m0 + 31) of pass `kind` for one
 // row.  FULL: all 32 are within the row's history (the common case, no
 // per-entry range test); otherwise entries j >= lim = C_i - m0 are ignored.
-// c2 = scale * log2(e) packed twice (exp of s - s_max as exp2 of u c - u_max c).
+// c = scale * log2(e) (exp of s - s_max as exp2 of u c - u_max c).
 template <bool FULL>
 __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, int m0, int lim, int Kp,
                                          const RowAddr& ra, const Staging& st, int r, float c) {
@@ -717,33 +726,38 @@ __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, i
         rs.s2 = s2;
         rs.mn = mn;
     } else if (kind == kPassB) {
-        const float nlo = -rs.lo, iw = rs.inv_w;
+        const uint64_t nlo2 = f32x2(-rs.lo, -rs.lo), iw2 = f32x2(rs.inv_w, rs.inv_w);
+        const uint64_t mg2 = f32x2(kBinMagic, kBinMagic);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const bool p = (FULL || j < lim) && u[j] >= rs.lo;
-            const int b = bin_clamp(bin_x(u[j], nlo, iw));
-            const bool hi = b >= kBinWords;
-            red_shared_add_if(p, ra.hist + static_cast<uint32_t>((hi ? b - kBinWords : b) * (kRows * 4)),
-                              hi ? 0x10000u : 1u);
+        for (int j = 0; j < 32; j += 2) {
+            float v0, v1;
+            f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
+            v0 = fminf(v0, kBinTop);
+            v1 = fminf(v1, kBinTop);
+            const bool p0 = (FULL || j < lim) && u[j] >= rs.lo;
+            const bool p1 = (FULL || j + 1 < lim) && u[j + 1] >= rs.lo;
+            red_shared_add_if(p0, ra.hist_off + __float_as_uint(v0) * static_cast<uint32_t>(kRows * 4), 1u);
+            red_shared_add_if(p1, ra.hist_off + __float_as_uint(v1) * static_cast<uint32_t>(kRows * 4), 1u);
         }
     } else if (kind == kPassC) {
-        const float nlo = -rs.lo, iw = rs.inv_w;
-        int pos = rs.pos, nbc = rs.nbc;
+        // v >= tb needs no clamp (tb <= kBinTop)
+        const uint64_t nlo2 = f32x2(-rs.lo, -rs.lo), iw2 = f32x2(rs.inv_w, rs.inv_w);
+        const uint64_t mg2 = f32x2(kBinMagic, kBinMagic);
+        int pos = rs.pos;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const bool in = (FULL || j < lim) && u[j] >= rs.lo;
-            const int b = bin_clamp(bin_x(u[j], nlo, iw));
-            const bool keep = in && b >= rs.hi_bin;
-            const bool bnd = in && b == rs.bstar && b < rs.hi_bin;
-            st_shared_if(keep, ra.idx + pos * 4, static_cast<uint32_t>(m0 + j));
-            st_shared_if(keep, ra.lg + pos * 4, __float_as_uint(u[j]));
-            pos += keep ? 1 : 0;
-            st_shared_if(bnd, ra.hist + (2 * nbc) * (kRows * 4), __float_as_uint(u[j]));
-            st_shared_if(bnd, ra.hist + (2 * nbc + 1) * (kRows * 4), static_cast<uint32_t>(m0 + j));
-            nbc += bnd ? 1 : 0;
+        for (int j = 0; j < 32; j += 2) {
+            float v0, v1;
+            f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
+            const bool p0 = (FULL || j < lim) && u[j] >= rs.lo && v0 >= rs.tb;
+            const bool p1 = (FULL || j + 1 < lim) && u[j + 1] >= rs.lo && v1 >= rs.tb;
+            st_shared_if(p0, ra.idx + pos * (kRows * 4), static_cast<uint32_t>(m0 + j));
+            st_shared_if(p0, ra.lg + pos * (kRows * 4), __float_as_uint(u[j]));
+            pos += p0 ? 1 : 0;
+            st_shared_if(p1, ra.idx + pos * (kRows * 4), static_cast<uint32_t>(m0 + j + 1));
+            st_shared_if(p1, ra.lg + pos * (kRows * 4), __float_as_uint(u[j + 1]));
+            pos += p1 ? 1 : 0;
         }
         rs.pos = pos;
-        rs.nbc = nbc;
     } else {   // kPassD: replace-the-worst for the rows the bins could not resolve
         if (rs.mode != kRowFail) return;
         FallbackState f{rs.pos, rs.ws, rs.wpos};
@@ -751,7 +765,7 @@ __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, i
         float* sc = st.lg + r * st.stride;
 #pragma unroll
         for (int j = 0; j < 32; ++j)
-            if (FULL || j < lim) f = fallback_offer(f, u[j], m0 + j, idx, sc, Kp);
+            if (FULL || j < lim) f = fallback_offer(f, u[j], m0 + j, idx, sc, Kp, st.es);
         rs.pos = f.pos;
         rs.ws = f.ws;
         rs.wpos = f.wpos;
@@ -762,14 +776,14 @@ __device__ __forceinline__ void row_set_all(RowSel& rs) {
     rs.mode = kRowAll;
     rs.lo = -CUDART_INF_F;
     rs.inv_w = 1.f;
+    rs.tb = -CUDART_INF_F;   // pass C takes every score of the history
     rs.hi_bin = 0;
-    rs.bstar = -1;
 }
 __device__ __forceinline__ void row_set_fail(RowSel& rs) {
     rs.mode = kRowFail;
     rs.lo = CUDART_INF_F;   // passes B and C take nothing from this row
+    rs.tb = CUDART_INF_F;
     rs.hi_bin = kBins;
-    rs.bstar = -1;
 }
 
 // After pass A: the histogram range of a row with more than K blocks.
@@ -794,26 +808,24 @@ __device__ __forceinline__ void row_after_a(RowSel& rs, int Ci, int K) {
     if (p_hi < 1.f) hi = fminf(rs.l.mx, rs.v0 + mean + sd * 1.41421356f * erfinvf(1.f - 2.f * p_hi));
     const float span = hi - lo;
     const float inv_w = static_cast<float>(kBins - 1) / span;
-    if (span > 0.f && isfinite(inv_w) && Ci <= 65535) {
+    if (span > 0.f && isfinite(inv_w)) {
         rs.mode = kRowNormal;
         rs.lo = lo;
         rs.inv_w = inv_w;
-        rs.hi_bin = kBins;   // nothing is kept before pass B has placed the K-th product
-        rs.bstar = -1;
+        rs.tb = CUDART_INF_F;   // nothing is listed before pass B has placed the K-th product
+        rs.hi_bin = kBins;
     } else {
         row_set_fail(rs);
     }
 }
 
 // After pass B: the bin holding the K-th largest product (scanning from the top).
-// Word w of the row holds bin w in its low half and bin w + kBinWords in its high half.
 __device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, int r, int Kp) {
     if (rs.mode != kRowNormal) return;
     int cum = 0, bstar = -1, nabove = 0, nb = 0;
 #pragma unroll
     for (int b = kBins - 1; b >= 0; --b) {
-        const uint32_t word = hist[(b % kBinWords) * kRows + r];
-        const int cb = static_cast<int>(b >= kBinWords ? (word >> 16) : (word & 0xffffu));
+        const int cb = static_cast<int>(hist[b * kRows + r]);
         if (bstar < 0 && cum + cb >= Kp) {
             bstar = b;
             nabove = cum;
@@ -830,27 +842,57 @@ __device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, in
         row_set_fail(rs);
         return;
     }
-    rs.bstar = bstar;
+    rs.tb = kBinMagic + static_cast<float>(bstar);
     rs.hi_bin = take_all ? bstar : bstar + 1;
     rs.nabove = nabove;
 }
 
-// After pass C: the best R = K' - nabove boundary products join the list (rank by
-// product descending, then block ascending; they are held in block order).
-__device__ __forceinline__ void row_after_c(RowSel& rs, const uint32_t* hist, const Staging& st, int r, int Kp) {
-    if (rs.mode != kRowNormal || rs.pos >= Kp) return;
+// After pass C: the list holds, in block order, the nabove products above the
+// boundary bin and (unless the bin is taken whole) the boundary bin's products.
+// The best R = K' - nabove of the latter, by (product descending, block
+// ascending), stay; the list is compacted in place.  The boundary products are
+// ranked from a copy in the row's (no longer used) histogram words.
+__device__ __forceinline__ void row_after_c(RowSel& rs, uint32_t* hist, const Staging& st, int r, int Kp) {
+    if (rs.mode != kRowNormal || rs.pos <= Kp) return;
+    int32_t* idx = st.idx + r * st.stride;
+    float* sc = st.lg + r * st.stride;
+    const int es = st.es;
+    const int n = rs.pos;
     const int R = Kp - rs.nabove;
-    for (int a = 0; a < rs.nbc; ++a) {
-        const float sa = __uint_as_float(hist[(2 * a) * kRows + r]);
-        const int ma = static_cast<int>(hist[(2 * a + 1) * kRows + r]);
-        int rank = 0;
-        for (int b = 0; b < rs.nbc; ++b) {
-            const float sb = __uint_as_float(hist[(2 * b) * kRows + r]);
-            rank += (sb > sa || (sb == sa && b < a)) ? 1 : 0;   // b < a: lower block
+    const float nlo = -rs.lo, iw = rs.inv_w;
+    const float tk = kBinMagic + static_cast<float>(rs.hi_bin);   // bins kept whole
+    int nbd = 0;
+    for (int a = 0; a < n; ++a) {
+        const float ua = sc[a * es];
+        if (bin_v(ua, nlo, iw) < tk) {
+            hist[(2 * nbd) * kRows + r] = __float_as_uint(ua);
+            hist[(2 * nbd + 1) * kRows + r] = static_cast<uint32_t>(idx[a * es]);
+            ++nbd;
         }
-        if (rank < R) stage_score(st, r, rs.pos++, ma, sa);
     }
-    if (rs.nabove > 0) staged_sort_by_block(st, r, rs.pos);
+    uint32_t keep = 0;   // bit x: the x-th boundary product (in block order) stays
+    for (int x = 0; x < nbd; ++x) {
+        const float ux = __uint_as_float(hist[(2 * x) * kRows + r]);
+        int rank = 0;
+        for (int y = 0; y < nbd; ++y) {
+            const float uy = __uint_as_float(hist[(2 * y) * kRows + r]);
+            rank += (uy > ux || (uy == ux && y < x)) ? 1 : 0;   // y < x: lower block
+        }
+        if (rank < R) keep |= 1u << x;
+    }
+    int out = 0, bi = 0;
+    for (int a = 0; a < n; ++a) {
+        const float ua = sc[a * es];
+        const int ma = idx[a * es];
+        bool k = true;
+        if (bin_v(ua, nlo, iw) < tk) k = (keep >> bi++) & 1u;
+        if (k) {
+            idx[out * es] = ma;
+            sc[out * es] = ua;
+            ++out;
+        }
+    }
+    rs.pos = out;
 }
 
 template <int D, int DS>
@@ -872,13 +914,14 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
     const int K = p.topk;
-    uint8_t* a_s = smem;                        // Q tile, then q~
+    uint8_t* a_s = smem;                        // Q tile, then the histograms
     uint8_t* b_s = smem + Cfg::A_BYTES;         // Wq, then summary chunks
-    uint32_t* hist = reinterpret_cast<uint32_t*>(smem + Cfg::A_BYTES + Cfg::B_BYTES);
-    uint8_t* stage_base = smem + Cfg::A_BYTES + Cfg::B_BYTES + kHistBytes;
-    const Staging st{reinterpret_cast<int32_t*>(stage_base),
-                     reinterpret_cast<float*>(stage_base + size_t(kRows) * (K + 1) * 4), K + 1};
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(stage_base + staging_bytes(K));
+    uint32_t* hist = reinterpret_cast<uint32_t*>(a_s);
+    uint8_t* list_base = smem + Cfg::A_BYTES + Cfg::B_BYTES;
+    const int cap = K + kBoundaryMax;           // list entries per row
+    const Staging st{reinterpret_cast<int32_t*>(list_base),
+                     reinterpret_cast<float*>(list_base + size_t(kRows) * cap * 4), 1, kRows};
+    uint32_t* bitmap = reinterpret_cast<uint32_t*>(list_base + list_bytes(K));
 
     // the tile: its index within its sequence, the sequence's first row and
     // length, and the summary slot of the sequence's block 0 (packed sequences:
@@ -984,7 +1027,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
         bool in_ok = nchunks > 0;
-        const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);
+        const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);   // projection operands
         for (int hq = 0; in_ok && hq < G; ++hq) {
             if (!mbar_wait(&in_full, hq & 1, wc)) { in_ok = false; break; }
             tc_fence_after();
@@ -999,8 +1042,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             umma_commit(hq + 1 < G ? &in_empty : &proj_done);   // regions A, B free for the next round
         }
         if (in_ok && mbar_wait(&qt_ready, 0, wc)) {
-            // S[gc&1] = q~ (128 x DS, bf16 in region A) * Kt_chunk (64 x DS)^T, for every
-            // chunk of every pass
+            // S[gc&1] = q~ (128 x DS, bf16 in TMEM columns 0 .. DS/2) * Kt_chunk (64 x DS)^T,
+            // for every chunk of every pass
             int gc = 0;
             bool ok = true;
             const int npass = resident ? 1 : npre;
@@ -1020,10 +1063,9 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     const uint32_t k_addr = smem_u32(b_s + b * Cfg::KC_BYTES);
 #pragma unroll
                     for (int k = 0; k < DS / 16; ++k) {
-                        const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
                         const uint32_t off_k = (k >> 2) * (64 * 128) + (k & 3) * 32;
-                        umma_bf16(tmem_base + Cfg::TMEM_S + b * 64, smem_desc_sw128(q_addr + off_q, 16, 1024),
-                                  smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                        umma_bf16_ta(tmem_base + Cfg::TMEM_S + b * 64, tmem_base + k * 8,
+                                     smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
                     }
                     umma_commit(&s_full[b]);
                     umma_commit(&kc_empty[b]);
@@ -1041,50 +1083,51 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         const int Ci = valid ? (i >> 6) : 0;
         const int Kp = min(K, Ci);
         const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-        for (int w = 0; w < kBinWords; ++w) hist[w * kRows + r] = 0u;   // this row's counters
         bool ok = true;
         if (nchunks > 0) {
-            // q~ row: fp32 from TMEM -> bf16 -> region A in the 128-byte-swizzled
-            // K-major layout of an MMA operand (16-byte chunk k of the row at k ^ (r & 7))
+            // q~ row: fp32 from TMEM columns 0 .. DS-1 -> bf16 pairs into columns
+            // 0 .. DS/2-1 (element 2k in the low half of column k), the A operand
+            // of the score products; each 64-column step reads its columns before
+            // writing the 32 below them
             ok = mbar_wait_warp(&proj_done, 0, wc);
             if (ok) {
                 tc_fence_after();
 #pragma unroll 1
-                for (int cc = 0; cc < DS / 32; ++cc) {
-                    uint32_t u[32];
-                    tmem_ld32(lane_addr + cc * 32, u);
+                for (int cc = 0; cc < DS / 64; ++cc) {
+                    uint32_t u[32], o[32];
+                    tmem_ld32(lane_addr + cc * 64, u);
                     tmem_wait_ld();
-                    uint8_t* row = a_s + (cc >> 1) * (kRows * 128) + r * 128;
 #pragma unroll
-                    for (int k4 = 0; k4 < 4; ++k4) {
-                        const int k = (cc & 1) * 4 + k4;
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(u[8 * k4 + 0]), __uint_as_float(u[8 * k4 + 1]));
-                        w.y = pack_bf16x2(__uint_as_float(u[8 * k4 + 2]), __uint_as_float(u[8 * k4 + 3]));
-                        w.z = pack_bf16x2(__uint_as_float(u[8 * k4 + 4]), __uint_as_float(u[8 * k4 + 5]));
-                        w.w = pack_bf16x2(__uint_as_float(u[8 * k4 + 6]), __uint_as_float(u[8 * k4 + 7]));
-                        *reinterpret_cast<uint4*>(row + ((k ^ (r & 7)) << 4)) = w;
-                    }
+                    for (int k = 0; k < 16; ++k)
+                        o[k] = pack_bf16x2(__uint_as_float(u[2 * k]), __uint_as_float(u[2 * k + 1]));
+                    tmem_ld32(lane_addr + cc * 64 + 32, u);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int k = 0; k < 16; ++k)
+                        o[16 + k] = pack_bf16x2(__uint_as_float(u[2 * k]), __uint_as_float(u[2 * k + 1]));
+                    tmem_st32(lane_addr + cc * 32, o);
                 }
-                fence_proxy_async_smem();
+                tmem_wait_st();
                 tc_fence_before();
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&qt_ready);
         }
+        // this row's counters, in region A once the projection has read its Q tiles
+        for (int w = 0; w < kBins; ++w) hist[w * kRows + r] = 0u;
         RowSel rs;
         rs.l = RowLse{-CUDART_INF_F, 0.f};
         rs.v0 = 0.f; rs.s1 = 0; rs.s2 = 0; rs.mn = CUDART_INF_F;
         row_set_all(rs);
-        rs.nabove = 0; rs.pos = 0; rs.nbc = 0;
+        rs.nabove = 0; rs.pos = 0;
         rs.ws = -CUDART_INF_F; rs.wpos = 0;
         // the products u are selected on directly (s = u scale); with noise the
         // pass works on s~ = s + eps itself
         const float c_exp = noisy ? kLog2e : p.score_scale * kLog2e;
         const float emit_scale = noisy ? 1.f : p.score_scale;
         const long long row_off = static_cast<long long>(bh) * p.N + geo.base + i;
-        const uint32_t hist_r = smem_u32(hist + r);
-        const RowAddr ra{smem_u32(st.idx + r * st.stride), smem_u32(st.lg + r * st.stride), hist_r};
+        const RowAddr ra{smem_u32(st.idx + r), smem_u32(st.lg + r),
+                         smem_u32(hist + r) - kBinMagicBits * static_cast<uint32_t>(kRows * 4)};
         int gc = 0;
         for (int ps = 0; ok && ps < npre + 1; ++ps) {
             int kind;
@@ -1167,13 +1210,13 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             const float lse = Ci > 0 ? __fmul_rn(rs.l.mx, emit_scale) + logf(rs.l.sum) : 0.f;
             for (int e = 0; e < K; ++e) {
                 if (e < Kp) {
-                    const int m = st.idx[r * st.stride + e];
-                    const float sc = __fmul_rn(st.lg[r * st.stride + e], emit_scale);
-                    st.lg[r * st.stride + e] = staged_gate(sc, lse, p.gate_act);
+                    const int m = st.idx[r + e * kRows];
+                    const float sc = __fmul_rn(st.lg[r + e * kRows], emit_scale);
+                    st.lg[r + e * kRows] = staged_gate(sc, lse, p.gate_act);
                     if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
                 } else {
-                    st.idx[r * st.stride + e] = -1;
-                    st.lg[r * st.stride + e] = 0.f;
+                    st.idx[r + e * kRows] = -1;
+                    st.lg[r + e * kRows] = 0.f;
                 }
             }
         }
