@@ -19,7 +19,7 @@ int make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64
                       uint32_t box_inner, uint32_t box_rows);
 
 // Raises `func`'s dynamic shared-memory limit to at least `bytes` on the
-// current device.  The attribute belongs to the device, so it is recorded per
+// current device, with the largest shared-memory carveout.  The attribute belongs to the device, so it is recorded per
 // (kernel, device): the first launch on each device sets it, later ones find
 // the record and call nothing (so a launch inside a stream capture that was
 // preceded by one outside it sets nothing).  Thread-safe.

@@ -518,16 +518,10 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 
 // --------------------------------------------------------- learned selector
 
-// Shared memory of the learned-selector kernel (offsets from a 1024-aligned base):
-//   region A: the 128-row Q tile of each projection round; once the projection
-//             has run, the per-row score histograms (and, after pass B, a
-//             row's boundary-bin scores while pass C's list is resolved);
-//   region B: the tile's Wq[h], then (once the projection has run) the
-//             double-buffered 64-block chunks of projected block summaries;
-//   then the per-row lists of selected scores (entry-major: entry e of row r
-//   at e * 128 + r, so a warp's 32 rows hit 32 banks) and the union bitmap.
-// The projected queries q~ stay in TMEM, rounded to bf16, as the A operand of
-// the score products.
+// The learned-selector kernel keeps the projected queries q~ in TMEM, rounded
+// to bf16, as the A operand of the score products; its shared-memory plan is
+// under SelProjCfg.  A CTA needs 128 TMEM columns and (K <= 36) about 72 KB of
+// shared memory, so three CTAs (twelve row warps) share an SM.
 //
 // Top-K without per-row replacement.  Replacing the worst kept entry whenever a
 // better score arrives diverges across the 32 rows of a warp (each row
@@ -561,27 +555,44 @@ constexpr float kBinMagic = 8388608.f;
 constexpr uint32_t kBinMagicBits = 0x4B000000u;
 constexpr float kBinTop = kBinMagic + float(kBins - 1);
 
-template <int D, int DS>
+constexpr int kChunk = 32;                          // blocks per score chunk (one TMEM buffer, one MMA)
+constexpr int kRing = 3;                            // summary-chunk stages in shared memory
+constexpr int kListSmall = kBins;                   // list capacity when K + kBoundaryMax fits the histogram words
+constexpr int kListBig = 64 + kBoundaryMax;         // list capacity for larger K
+
+// Shared-memory plan (bytes from the 1024-aligned base):
+//   [0, LIST): the rows' list blocks; before that the histograms (pass B),
+//              and during the projection a 64-column half of the Q tile;
+//   [LIST, 2 LIST): the rows' list products;
+//   ring: the summary-chunk stages, during the projection a 64-column slice of Wq;
+//   then the union bitmap.
+template <int D, int DS, bool BIGK>
 struct SelProjCfg {
-    static constexpr int Q_BYTES = kRows * D * 2;
-    static constexpr int A_BYTES = Q_BYTES > int(kHistBytes) ? Q_BYTES : int(kHistBytes);
-    static constexpr int WQ_BYTES = DS * D * 2;
-    static constexpr int KC_BYTES = 64 * DS * 2;   // 64 blocks per chunk
-    static constexpr int B_BYTES = WQ_BYTES > 2 * KC_BYTES ? WQ_BYTES : 2 * KC_BYTES;
+    static constexpr int CAP = BIGK ? kListBig : kListSmall;   // list entries per row
+    static constexpr int LIST_BYTES = CAP * kRows * 4;         // one of the two list arrays
+    static constexpr int QH_BYTES = kRows * 64 * 2;            // a 64-column half of the Q tile
+    static constexpr int WQH_BYTES = DS * 64 * 2;              // a 64-column slice of Wq
+    static constexpr int KC_BYTES = kChunk * DS * 2;           // one chunk of projected summaries
+    static constexpr int RING_BYTES = kRing * KC_BYTES > WQH_BYTES ? kRing * KC_BYTES : WQH_BYTES;
+    static constexpr int OFF_LG = LIST_BYTES;
+    static constexpr int OFF_RING = 2 * LIST_BYTES;
+    static constexpr int OFF_BITMAP = OFF_RING + RING_BYTES;
     static constexpr uint32_t IDESC_PROJ = idesc_bf16(kRows, DS, 0, 0);
-    static constexpr uint32_t IDESC_S = idesc_bf16(kRows, 64, 0, 0);
-    static constexpr int TMEM_S = 128;            // score buffers at columns 128 and 192; q~ (bf16) at 0 .. DS/2
+    static constexpr uint32_t IDESC_S = idesc_bf16(kRows, kChunk, 0, 0);
+    // TMEM (128 columns): q~ in fp32 at 0 .. DS-1 during the projection, then in
+    // bf16 at 0 .. DS/2-1; the two score buffers at 64 and 96
+    static constexpr int TMEM_S = 64;
+    static_assert(LIST_BYTES >= int(kHistBytes) && LIST_BYTES >= QH_BYTES, "histogram / Q half exceed the list");
+    static_assert(DS <= 128 && D % 64 == 0 && DS % 64 == 0, "projection shape");
 };
 
 constexpr int kPassA = 0, kPassB = 1, kPassC = 2, kPassD = 3;
 constexpr int kPassW = 4;   // full training scope: write every score to the table
 constexpr int kRowAll = 0, kRowNormal = 1, kRowFail = 2;   // C_i <= K: keep all; thresholds; fallback
 
-__host__ __device__ constexpr size_t list_bytes(int K) { return size_t(K + kBoundaryMax) * kRows * 8; }
-
-template <int D, int DS>
-__host__ __device__ constexpr size_t proj_smem_bytes(int K, int C) {
-    return size_t(SelProjCfg<D, DS>::A_BYTES) + SelProjCfg<D, DS>::B_BYTES + list_bytes(K) + bitmap_bytes(C);
+template <int D, int DS, bool BIGK>
+__host__ __device__ constexpr size_t proj_smem_bytes(int C) {
+    return size_t(SelProjCfg<D, DS, BIGK>::OFF_BITMAP) + bitmap_bytes(C);
 }
 
 // Selection works on the raw products u = q~ . K~ (the scores are s = u / sqrt(d_sel),
@@ -611,8 +622,9 @@ struct RowSel {
 };
 
 // Shared-memory addresses of one row's list and histogram.
+constexpr uint32_t kListStep = kRows * 4;   // bytes between a row's list entries
 struct RowAddr {
-    uint32_t idx, lg;           // list entry 0 of the row (int32 block, fp32 product); entry e at + e * kRows * 4
+    uint32_t list;              // the row's list entry 0 (int32 block; its fp32 product OFF_LG bytes on); entry e at + e * kListStep
     uint32_t hist_off;          // the row's histogram word of bin b at hist_off + bits(v) * kRows * 4 (mod 2^32)
 };
 
@@ -681,8 +693,10 @@ __device__ __forceinline__ void staged_sort_by_block(const Staging& st, int r, i
 // One half-chunk (32 products of blocks m0 .. m0 + 31) of pass `kind` for one
 // row.  FULL: all 32 are within the row's history (the common case, no
 // per-entry range test); otherwise entries j >= lim = C_i - m0 are ignored.
+// Passes B and C always run FULL: the caller turns the products past the
+// history into NaN, which no comparison takes.
 // c = scale * log2(e) (exp of s - s_max as exp2 of u c - u_max c).
-template <bool FULL>
+template <bool FULL, uint32_t OFF_LG>
 __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, int m0, int lim, int Kp,
                                          const RowAddr& ra, const Staging& st, int r, float c) {
     if (kind == kPassA) {
@@ -728,36 +742,28 @@ __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, i
     } else if (kind == kPassB) {
         const uint64_t nlo2 = f32x2(-rs.lo, -rs.lo), iw2 = f32x2(rs.inv_w, rs.inv_w);
         const uint64_t mg2 = f32x2(kBinMagic, kBinMagic);
+        const float lo = rs.lo;
 #pragma unroll
         for (int j = 0; j < 32; j += 2) {
             float v0, v1;
             f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
-            v0 = fminf(v0, kBinTop);
-            v1 = fminf(v1, kBinTop);
-            const bool p0 = (FULL || j < lim) && u[j] >= rs.lo;
-            const bool p1 = (FULL || j + 1 < lim) && u[j + 1] >= rs.lo;
-            red_shared_add_if(p0, ra.hist_off + __float_as_uint(v0) * static_cast<uint32_t>(kRows * 4), 1u);
-            red_shared_add_if(p1, ra.hist_off + __float_as_uint(v1) * static_cast<uint32_t>(kRows * 4), 1u);
+            red_shared_inc_if_ge(u[j], lo, ra.hist_off + __float_as_uint(fminf(v0, kBinTop)) * (kRows * 4u));
+            red_shared_inc_if_ge(u[j + 1], lo, ra.hist_off + __float_as_uint(fminf(v1, kBinTop)) * (kRows * 4u));
         }
     } else if (kind == kPassC) {
         // v >= tb needs no clamp (tb <= kBinTop)
         const uint64_t nlo2 = f32x2(-rs.lo, -rs.lo), iw2 = f32x2(rs.inv_w, rs.inv_w);
         const uint64_t mg2 = f32x2(kBinMagic, kBinMagic);
-        int pos = rs.pos;
+        const float lo = rs.lo, tb = rs.tb;
+        uint32_t addr = ra.list + static_cast<uint32_t>(rs.pos) * kListStep;
 #pragma unroll
         for (int j = 0; j < 32; j += 2) {
             float v0, v1;
             f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
-            const bool p0 = (FULL || j < lim) && u[j] >= rs.lo && v0 >= rs.tb;
-            const bool p1 = (FULL || j + 1 < lim) && u[j + 1] >= rs.lo && v1 >= rs.tb;
-            st_shared_if(p0, ra.idx + pos * (kRows * 4), static_cast<uint32_t>(m0 + j));
-            st_shared_if(p0, ra.lg + pos * (kRows * 4), __float_as_uint(u[j]));
-            pos += p0 ? 1 : 0;
-            st_shared_if(p1, ra.idx + pos * (kRows * 4), static_cast<uint32_t>(m0 + j + 1));
-            st_shared_if(p1, ra.lg + pos * (kRows * 4), __float_as_uint(u[j + 1]));
-            pos += p1 ? 1 : 0;
+            st_shared_split_if_ge2<OFF_LG>(u[j], lo, v0, tb, addr, static_cast<uint32_t>(m0 + j), kListStep);
+            st_shared_split_if_ge2<OFF_LG>(u[j + 1], lo, v1, tb, addr, static_cast<uint32_t>(m0 + j + 1), kListStep);
         }
-        rs.pos = pos;
+        rs.pos = static_cast<int>((addr - ra.list) / kListStep);
     } else {   // kPassD: replace-the-worst for the rows the bins could not resolve
         if (rs.mode != kRowFail) return;
         FallbackState f{rs.pos, rs.ws, rs.wpos};
@@ -850,62 +856,70 @@ __device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, in
 // After pass C: the list holds, in block order, the nabove products above the
 // boundary bin and (unless the bin is taken whole) the boundary bin's products.
 // The best R = K' - nabove of the latter, by (product descending, block
-// ascending), stay; the list is compacted in place.  The boundary products are
-// ranked from a copy in the row's (no longer used) histogram words.
-__device__ __forceinline__ void row_after_c(RowSel& rs, uint32_t* hist, const Staging& st, int r, int Kp) {
+// ascending), stay; the list is compacted in place.
+__device__ __forceinline__ void row_after_c(RowSel& rs, const Staging& st, int r, int Kp) {
     if (rs.mode != kRowNormal || rs.pos <= Kp) return;
     int32_t* idx = st.idx + r * st.stride;
     float* sc = st.lg + r * st.stride;
     const int es = st.es;
-    const int n = rs.pos;
+    const int n = rs.pos;   // <= K' - 1 + kBoundaryMax < 128
     const int R = Kp - rs.nabove;
     const float nlo = -rs.lo, iw = rs.inv_w;
     const float tk = kBinMagic + static_cast<float>(rs.hi_bin);   // bins kept whole
-    int nbd = 0;
+    // bit a of (bl, bh): entry a is in the boundary bin; likewise the kept ones
+    uint64_t bl = 0, bh = 0;
     for (int a = 0; a < n; ++a) {
-        const float ua = sc[a * es];
-        if (bin_v(ua, nlo, iw) < tk) {
-            hist[(2 * nbd) * kRows + r] = __float_as_uint(ua);
-            hist[(2 * nbd + 1) * kRows + r] = static_cast<uint32_t>(idx[a * es]);
-            ++nbd;
+        if (bin_v(sc[a * es], nlo, iw) < tk) {
+            if (a < 64) bl |= 1ull << a;
+            else bh |= 1ull << (a - 64);
         }
     }
-    uint32_t keep = 0;   // bit x: the x-th boundary product (in block order) stays
-    for (int x = 0; x < nbd; ++x) {
-        const float ux = __uint_as_float(hist[(2 * x) * kRows + r]);
-        int rank = 0;
-        for (int y = 0; y < nbd; ++y) {
-            const float uy = __uint_as_float(hist[(2 * y) * kRows + r]);
-            rank += (uy > ux || (uy == ux && y < x)) ? 1 : 0;   // y < x: lower block
+    uint64_t kl = 0, kh = 0;
+    for (int hx = 0; hx < 2; ++hx) {
+        for (uint64_t mx = hx ? bh : bl; mx != 0; mx &= mx - 1) {
+            const int x = hx * 64 + __ffsll(static_cast<long long>(mx)) - 1;
+            const float ux = sc[x * es];
+            int rank = 0;
+            for (int hy = 0; hy < 2; ++hy)
+                for (uint64_t my = hy ? bh : bl; my != 0; my &= my - 1) {
+                    const int y = hy * 64 + __ffsll(static_cast<long long>(my)) - 1;
+                    const float uy = sc[y * es];
+                    rank += (uy > ux || (uy == ux && y < x)) ? 1 : 0;   // y < x: lower block
+                }
+            if (rank < R) {
+                if (hx) kh |= 1ull << (x - 64);
+                else kl |= 1ull << x;
+            }
         }
-        if (rank < R) keep |= 1u << x;
     }
-    int out = 0, bi = 0;
+    int out = 0;
     for (int a = 0; a < n; ++a) {
-        const float ua = sc[a * es];
-        const int ma = idx[a * es];
-        bool k = true;
-        if (bin_v(ua, nlo, iw) < tk) k = (keep >> bi++) & 1u;
-        if (k) {
-            idx[out * es] = ma;
-            sc[out * es] = ua;
+        const uint64_t bw = a < 64 ? bl : bh, kw = a < 64 ? kl : kh;
+        const int sh = a & 63;
+        if (!((bw >> sh) & 1ull) || ((kw >> sh) & 1ull)) {
+            idx[out * es] = idx[a * es];
+            sc[out * es] = sc[a * es];
             ++out;
         }
     }
     rs.pos = out;
 }
 
-template <int D, int DS>
-__global__ void __launch_bounds__(192, 2)
+// Registers: three CTAs of 192 threads share an SM for K <= 36 (two above).  An
+// SM sub-partition holds 16K registers and takes up to five of those 18 warps,
+// so a thread may have 96.
+template <int D, int DS, bool BIGK>
+__global__ void __maxnreg__(BIGK ? 168 : 96)
 select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapWq,
                    const __grid_constant__ CUtensorMap mapKt, SelParams p, int H, int G) {
     // H: KV heads (selection groups), G: query heads per group.  The gate query of
-    // group bh is q~ = Wq[bh % H] [q_{bh G}; ...; q_{bh G + G - 1}]: G rounds that
-    // each stage one head's Q tile and its d columns of Wq and accumulate.
-    using Cfg = SelProjCfg<D, DS>;
+    // group bh is q~ = Wq[bh % H] [q_{bh G}; ...; q_{bh G + G - 1}]: rounds that
+    // each stage a 64-column half of one head's Q tile and the matching columns
+    // of Wq and accumulate.
+    using Cfg = SelProjCfg<D, DS, BIGK>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     if (p.tiles != nullptr && static_cast<int>(blockIdx.x / p.BH) >= __ldg(p.ntiles)) return;   // spare slot
-    __shared__ uint64_t in_full, in_empty, proj_done, qt_ready, kc_full[2], kc_empty[2], s_full[2], s_free[2],
+    __shared__ uint64_t in_full, in_empty, proj_done, qt_ready, kc_full[kRing], kc_empty[kRing], s_full[2], s_free[2],
         drain_bar, plan_bar;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag, fail_flag;
@@ -914,14 +928,12 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
     const int K = p.topk;
-    uint8_t* a_s = smem;                        // Q tile, then the histograms
-    uint8_t* b_s = smem + Cfg::A_BYTES;         // Wq, then summary chunks
-    uint32_t* hist = reinterpret_cast<uint32_t*>(a_s);
-    uint8_t* list_base = smem + Cfg::A_BYTES + Cfg::B_BYTES;
-    const int cap = K + kBoundaryMax;           // list entries per row
-    const Staging st{reinterpret_cast<int32_t*>(list_base),
-                     reinterpret_cast<float*>(list_base + size_t(kRows) * cap * 4), 1, kRows};
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(list_base + list_bytes(K));
+    uint8_t* qh_s = smem;                                  // Q half (projection), then histograms / list blocks
+    uint8_t* ring = smem + Cfg::OFF_RING;                  // Wq slice (projection), then summary chunks
+    uint32_t* hist = reinterpret_cast<uint32_t*>(smem);
+    // list entry e of row r: block at word e * kRows + r, product OFF_LG bytes on
+    const Staging st{reinterpret_cast<int32_t*>(smem), reinterpret_cast<float*>(smem + Cfg::OFF_LG), 1, kRows};
+    uint32_t* bitmap = reinterpret_cast<uint32_t*>(smem + Cfg::OFF_BITMAP);
 
     // the tile: its index within its sequence, the sequence's first row and
     // length, and the summary slot of the sequence's block 0 (packed sequences:
@@ -937,7 +949,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     // full*: noise added to the scores before the gate and the Top-K
     const bool noisy = p.noise != nullptr;
     const int nb = min(2 * t + 1, seq_n / 64);  // blocks scored for this tile (full blocks of its sequence)
-    const int nchunks = (K > 0 || full) ? (nb + 63) >> 6 : 0;
+    const int nchunks = (K > 0 || full) ? (nb + kChunk - 1) / kChunk : 0;
     // the most blocks any row of the tile has: a histogram pass only when it exceeds K
     const int last_row = min(seq_n, (t + 1) * kRows) - 1;
     const int tile_ci = last_row >= t * kRows ? (last_row >> 6) : 0;
@@ -947,6 +959,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     // a history of at most two chunks stays in the two TMEM score buffers: its
     // products are computed once and every pass reads them again
     const bool resident = nchunks <= 2;
+    const int rounds_total = G * (D / 64);   // projection rounds
 
     const int nwords = (p.C + 31) >> 5;
     for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
@@ -955,9 +968,11 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         mbar_init(&in_empty, 1);
         mbar_init(&proj_done, 1);
         mbar_init(&qt_ready, 4);
+        for (int s = 0; s < kRing; ++s) {
+            mbar_init(&kc_full[s], 1);
+            mbar_init(&kc_empty[s], 1);
+        }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(&kc_full[b], 1);
-            mbar_init(&kc_empty[b], 1);
             mbar_init(&s_full[b], 1);
             mbar_init(&s_free[b], 128);
         }
@@ -968,7 +983,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         fence_barrier_init();
     }
     if (warp == 1) {
-        tmem_alloc(&tmem_base_sh, 256);
+        tmem_alloc(&tmem_base_sh, 128);
         tmem_relinquish();
     }
     __syncthreads();
@@ -984,19 +999,18 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             tma_prefetch_desc(&mapKt);
             bool ok = true;
             int rounds = 0;
-            for (int hq = 0; hq < G; ++hq) {
-                // round hq: query head bh G + hq and its columns hq D .. hq D + D - 1 of Wq
-                if (hq > 0 && !mbar_wait(&in_empty, (hq - 1) & 1, wc)) { ok = false; break; }
-                mbar_arrive_expect_tx(&in_full, Cfg::Q_BYTES + Cfg::WQ_BYTES);
-#pragma unroll
-                for (int a = 0; a < D / 64; ++a) {
-                    tma_load_3d(a_s + a * (kRows * 128), &mapQ, &in_full, a * 64, geo.base + t * kRows, bh * G + hq);
-                    tma_load_3d(b_s + a * (DS * 128), &mapWq, &in_full, hq * D + a * 64, 0, bh % H);
-                }
+            for (int rd = 0; rd < rounds_total; ++rd) {
+                // round rd: columns 64 a .. 64 a + 63 of query head bh G + hq and the
+                // matching columns hq D + 64 a .. of Wq
+                const int hq = rd / (D / 64), a = rd % (D / 64);
+                if (rd > 0 && !mbar_wait(&in_empty, (rd - 1) & 1, wc)) { ok = false; break; }
+                mbar_arrive_expect_tx(&in_full, Cfg::QH_BYTES + Cfg::WQH_BYTES);
+                tma_load_3d(qh_s, &mapQ, &in_full, a * 64, geo.base + t * kRows, bh * G + hq);
+                tma_load_3d(ring, &mapWq, &in_full, hq * D + a * 64, 0, bh % H);
                 ++rounds;
             }
             int issued = 0;
-            if (ok) ok = mbar_wait(&proj_done, 0, wc);   // region B is free once the projection ran
+            if (ok) ok = mbar_wait(&proj_done, 0, wc);   // the ring is free once the projection ran
             const int npass = resident ? 1 : npre;
             for (int ps = 0; ok && ps < npass + 1; ++ps) {
                 if (resident && ps == npass) break;
@@ -1008,41 +1022,38 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 }
                 for (int c = 0; ok && c < nchunks; ++c) {
                     const int gc = issued;
-                    const int b = gc & 1;
-                    if (!mbar_wait(&kc_empty[b], ((gc >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
-                    mbar_arrive_expect_tx(&kc_full[b], Cfg::KC_BYTES);
+                    const int s = gc % kRing;
+                    if (!mbar_wait(&kc_empty[s], ((gc / kRing) & 1) ^ 1u, wc)) { ok = false; break; }
+                    mbar_arrive_expect_tx(&kc_full[s], Cfg::KC_BYTES);
 #pragma unroll
                     for (int a = 0; a < DS / 64; ++a)
-                        tma_load_3d(b_s + b * Cfg::KC_BYTES + a * (64 * 128), &mapKt, &kc_full[b], a * 64, kt0 + c * 64,
-                                    bh);
+                        tma_load_3d(ring + s * Cfg::KC_BYTES + a * (kChunk * 128), &mapKt, &kc_full[s], a * 64,
+                                    kt0 + c * kChunk, bh);
                     ++issued;
                 }
             }
             if (!ok) {
                 if (rounds > 0) mbar_wait_drain(&in_full, (rounds - 1) & 1, p.limit, p.status);
-                for (int q = issued - 1; q >= 0 && q >= issued - 2; --q)
-                    mbar_wait_drain(&kc_full[q & 1], (q >> 1) & 1, p.limit, p.status);
+                for (int q = issued - 1; q >= 0 && q >= issued - kRing; --q)
+                    mbar_wait_drain(&kc_full[q % kRing], (q / kRing) & 1, p.limit, p.status);
             }
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
         bool in_ok = nchunks > 0;
-        const uint32_t q_addr = smem_u32(a_s), w_addr = smem_u32(b_s);   // projection operands
-        for (int hq = 0; in_ok && hq < G; ++hq) {
-            if (!mbar_wait(&in_full, hq & 1, wc)) { in_ok = false; break; }
+        const uint32_t q_addr = smem_u32(qh_s), w_addr = smem_u32(ring);   // projection operands
+        for (int rd = 0; in_ok && rd < rounds_total; ++rd) {
+            if (!mbar_wait(&in_full, rd & 1, wc)) { in_ok = false; break; }
             tc_fence_after();
-            // q~ (fp32, TMEM columns 0 .. DS-1) += Q_hq (128 x D) * Wq[h][:, hq D : hq D + D] (DS x D)^T
+            // q~ (fp32, TMEM columns 0 .. DS-1) += Q half (128 x 64) * Wq slice (DS x 64)^T
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-                const uint32_t off_q = (k >> 2) * (kRows * 128) + (k & 3) * 32;
-                const uint32_t off_w = (k >> 2) * (DS * 128) + (k & 3) * 32;
-                umma_bf16(tmem_base, smem_desc_sw128(q_addr + off_q, 16, 1024),
-                          smem_desc_sw128(w_addr + off_w, 16, 1024), Cfg::IDESC_PROJ, (hq > 0 || k > 0) ? 1u : 0u);
-            }
-            umma_commit(hq + 1 < G ? &in_empty : &proj_done);   // regions A, B free for the next round
+            for (int k = 0; k < 4; ++k)
+                umma_bf16(tmem_base, smem_desc_sw128(q_addr + k * 32, 16, 1024),
+                          smem_desc_sw128(w_addr + k * 32, 16, 1024), Cfg::IDESC_PROJ, (rd > 0 || k > 0) ? 1u : 0u);
+            umma_commit(rd + 1 < rounds_total ? &in_empty : &proj_done);   // Q half and Wq slice free
         }
         if (in_ok && mbar_wait(&qt_ready, 0, wc)) {
-            // S[gc&1] = q~ (128 x DS, bf16 in TMEM columns 0 .. DS/2) * Kt_chunk (64 x DS)^T,
+            // S[gc&1] = q~ (128 x DS, bf16 in TMEM columns 0 .. DS/2) * Kt_chunk (32 x DS)^T,
             // for every chunk of every pass
             int gc = 0;
             bool ok = true;
@@ -1055,20 +1066,19 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
                 }
                 for (int c = 0; c < nchunks; ++c, ++gc) {
-                    const int b = gc & 1;
-                    const uint32_t ph = (gc >> 1) & 1;
-                    if (!mbar_wait(&kc_full[b], ph, wc)) { ok = false; break; }
-                    if (!mbar_wait(&s_free[b], ph ^ 1u, wc)) { ok = false; break; }
+                    const int s = gc % kRing, b = gc & 1;
+                    if (!mbar_wait(&kc_full[s], (gc / kRing) & 1, wc)) { ok = false; break; }
+                    if (!mbar_wait(&s_free[b], ((gc >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t k_addr = smem_u32(b_s + b * Cfg::KC_BYTES);
+                    const uint32_t k_addr = smem_u32(ring + s * Cfg::KC_BYTES);
 #pragma unroll
                     for (int k = 0; k < DS / 16; ++k) {
-                        const uint32_t off_k = (k >> 2) * (64 * 128) + (k & 3) * 32;
-                        umma_bf16_ta(tmem_base + Cfg::TMEM_S + b * 64, tmem_base + k * 8,
+                        const uint32_t off_k = (k >> 2) * (kChunk * 128) + (k & 3) * 32;
+                        umma_bf16_ta(tmem_base + Cfg::TMEM_S + b * kChunk, tmem_base + k * 8,
                                      smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
                     }
                     umma_commit(&s_full[b]);
-                    umma_commit(&kc_empty[b]);
+                    umma_commit(&kc_empty[s]);
                 }
             }
         }
@@ -1113,7 +1123,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&qt_ready);
         }
-        // this row's counters, in region A once the projection has read its Q tiles
+        // this row's counters, over the Q half once the projection has read it
         for (int w = 0; w < kBins; ++w) hist[w * kRows + r] = 0u;
         RowSel rs;
         rs.l = RowLse{-CUDART_INF_F, 0.f};
@@ -1126,7 +1136,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         const float c_exp = noisy ? kLog2e : p.score_scale * kLog2e;
         const float emit_scale = noisy ? 1.f : p.score_scale;
         const long long row_off = static_cast<long long>(bh) * p.N + geo.base + i;
-        const RowAddr ra{smem_u32(st.idx + r), smem_u32(st.lg + r),
+        const RowAddr ra{smem_u32(st.idx + r * st.stride),
                          smem_u32(hist + r) - kBinMagicBits * static_cast<uint32_t>(kRows * 4)};
         int gc = 0;
         for (int ps = 0; ok && ps < npre + 1; ++ps) {
@@ -1148,42 +1158,47 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     break;
                 }
                 tc_fence_after();
-#pragma unroll 1
-                for (int half = 0; half < 2; ++half) {
-                    uint32_t uu[32];
-                    tmem_ld32(lane_addr + Cfg::TMEM_S + b * 64 + half * 32, uu);
-                    tmem_wait_ld();
-                    if (half == 1 && !resident) {
-                        tc_fence_before();
-                        mbar_arrive(&s_free[b]);
-                    }
-                    const int m0 = 64 * c + 32 * half;
-                    const int lim = Ci - m0;
-                    if (noisy) {
-                        const float* nrow = p.noise + row_off * p.C + m0;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j < lim)
-                                uu[j] = __float_as_uint(
-                                    __fadd_rn(__fmul_rn(__uint_as_float(uu[j]), p.score_scale), __ldg(nrow + j)));
-                    }
-                    const float* u = reinterpret_cast<const float*>(uu);
-                    if (kind == kPassW) {
-                        float* dst = p.full_table + row_off * p.C + m0;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (j < lim) dst[j] = __fmul_rn(u[j], p.score_scale);
-                    } else {
-                        // the vote comes before any lane leaves; the lanes meet again
-                        // before the next warp-collective TMEM load
-                        const bool whole = __all_sync(0xffffffffu, lim >= 32);
-                        if (whole)
-                            row_pass<true>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
-                        else if (lim > 0)
-                            row_pass<false>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
-                    }
-                    __syncwarp();
+                uint32_t uu[32];
+                tmem_ld32(lane_addr + Cfg::TMEM_S + b * kChunk, uu);
+                tmem_wait_ld();
+                if (!resident) {
+                    tc_fence_before();
+                    mbar_arrive(&s_free[b]);
                 }
+                const int m0 = kChunk * c;
+                const int lim = Ci - m0;
+                if (noisy) {
+                    const float* nrow = p.noise + row_off * p.C + m0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < lim)
+                            uu[j] = __float_as_uint(
+                                __fadd_rn(__fmul_rn(__uint_as_float(uu[j]), p.score_scale), __ldg(nrow + j)));
+                }
+                const float* u = reinterpret_cast<const float*>(uu);
+                if (kind == kPassW) {
+                    float* dst = p.full_table + row_off * p.C + m0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < lim) dst[j] = __fmul_rn(u[j], p.score_scale);
+                } else {
+                    // the vote comes before any lane leaves; the lanes meet again
+                    // before the next warp-collective TMEM load
+                    const bool whole = __all_sync(0xffffffffu, lim >= 32);
+                    if (kind == kPassB || kind == kPassC) {
+                        if (!whole) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (j >= lim) uu[j] = 0x7fc00000u;   // NaN: past the history
+                        }
+                        row_pass<true, Cfg::OFF_LG>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    } else if (whole) {
+                        row_pass<true, Cfg::OFF_LG>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    } else if (lim > 0) {
+                        row_pass<false, Cfg::OFF_LG>(rs, kind, u, m0, lim, Kp, ra, st, r, c_exp);
+                    }
+                }
+                __syncwarp();
             }
             if (!ok) break;
             if (kind == kPassA) {
@@ -1196,7 +1211,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&plan_bar);
             } else if (kind == kPassC) {
-                row_after_c(rs, hist, st, r, Kp);
+                row_after_c(rs, st, r, Kp);
             } else {
                 staged_sort_by_block(st, r, rs.pos);
             }
@@ -1210,13 +1225,13 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             const float lse = Ci > 0 ? __fmul_rn(rs.l.mx, emit_scale) + logf(rs.l.sum) : 0.f;
             for (int e = 0; e < K; ++e) {
                 if (e < Kp) {
-                    const int m = st.idx[r + e * kRows];
-                    const float sc = __fmul_rn(st.lg[r + e * kRows], emit_scale);
-                    st.lg[r + e * kRows] = staged_gate(sc, lse, p.gate_act);
+                    const int m = st.idx[r * st.stride + e * st.es];
+                    const float sc = __fmul_rn(st.lg[r * st.stride + e * st.es], emit_scale);
+                    st.lg[r * st.stride + e * st.es] = staged_gate(sc, lse, p.gate_act);
                     if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
                 } else {
-                    st.idx[r + e * kRows] = -1;
-                    st.lg[r + e * kRows] = 0.f;
+                    st.idx[r * st.stride + e * st.es] = -1;
+                    st.lg[r * st.stride + e * st.es] = 0.f;
                 }
             }
         }
@@ -1233,26 +1248,35 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, 256);
+        tmem_dealloc(tmem_base, 128);
     }
 }
 
-template <int D, int DS>
-cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
-    const size_t smem = 1024 + proj_smem_bytes<D, DS>(a.topk, a.C);
-    if (smem > 227 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS>), smem);
+template <int D, int DS, bool BIGK>
+cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
+    const size_t smem = 1024 + proj_smem_bytes<D, DS, BIGK>(a.C);
+    if (smem > 227 * 1024) { *err = "selection: too many blocks for shared memory"; return cudaErrorInvalidValue; }
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS, BIGK>), smem);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mw, mk;
     // Q of all query heads; Wq [H][DS][G D] (a group's gate-query projection)
     if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH * a.G, 64, kRows) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mw, a.Wq, static_cast<uint64_t>(a.G) * D, DS, a.H, 64, DS) != 0) { *err = "tensor map Wq"; return cudaErrorInvalidValue; }
-    if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, 64) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
+    if (make_tmap_bf16_3d(&mk, a.Kt, DS, a.F > 0 ? a.F : 1, a.BH, 64, kChunk) != 0) { *err = "tensor map Kt"; return cudaErrorInvalidValue; }
     const dim3 grid(a.BH * a.T);
-    select_proj_kernel<D, DS><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H, a.G);
+    select_proj_kernel<D, DS, BIGK><<<grid, 192, smem, env.stream>>>(mq, mw, mk, p, a.H, a.G);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;
+}
+
+// K + kBoundaryMax list entries per row: within the histogram words up to K = 36
+template <int D, int DS>
+cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
+    if (a.topk + kBoundaryMax <= kListSmall) return launch_proj_k<D, DS, false>(a, p, env, err);
+    if (a.topk + kBoundaryMax <= kListBig) return launch_proj_k<D, DS, true>(a, p, env, err);
+    *err = "selection: top-K too large";
+    return cudaErrorInvalidValue;
 }
 
 template <bool REG>

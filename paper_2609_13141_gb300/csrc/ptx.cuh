@@ -345,20 +345,24 @@ __device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
     asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
     return d;
 }
-// Shared-memory reduction and stores under a predicate, without a branch around
-// them (per-lane work that is rare for each lane but frequent for the warp).
-__device__ __forceinline__ void red_shared_add_if(bool p, uint32_t saddr, uint32_t v) {
-    asm volatile(
-        "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t@q red.shared.add.u32 [%1], %2;\n\t}" ::"r"(
-            static_cast<int>(p)),
-        "r"(saddr), "r"(v)
-        : "memory");
-}
-__device__ __forceinline__ void st_shared_if(bool p, uint32_t saddr, uint32_t v) {
-    asm volatile("{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t@q st.shared.u32 [%1], %2;\n\t}" ::"r"(
-                     static_cast<int>(p)),
-                 "r"(saddr), "r"(v)
+// One to the shared word at saddr when u >= lo (false for a NaN u), the
+// comparison inside the predicated block.
+__device__ __forceinline__ void red_shared_inc_if_ge(float u, float lo, uint32_t saddr) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ge.f32 p, %0, %1;\n\t@p red.shared.add.u32 [%2], 1;\n\t}" ::"f"(u),
+                 "f"(lo), "r"(saddr)
                  : "memory");
+}
+// Stores m at addr and u at addr + OFF and advances addr by step when u >= lo
+// and v >= tb (false for NaN operands).
+template <uint32_t OFF>
+__device__ __forceinline__ void st_shared_split_if_ge2(float u, float lo, float v, float tb, uint32_t& addr,
+                                                       uint32_t m, uint32_t step) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ge.f32 p, %1, %2;\n\tsetp.ge.and.f32 p, %3, %4, p;\n\t"
+        "@p st.shared.b32 [%0], %5;\n\t@p st.shared.b32 [%0+%7], %6;\n\t@p add.u32 %0, %0, %8;\n\t}"
+        : "+r"(addr)
+        : "f"(u), "f"(lo), "f"(v), "f"(tb), "r"(m), "f"(u), "n"(OFF), "r"(step)
+        : "memory");
 }
 
 __device__ __forceinline__ float max3f(float a, float b, float c) {

@@ -63,6 +63,9 @@ cudaError_t ensure_smem_attr(const void* func, size_t bytes) {
     size_t& set = g_smem_attr[{func, dev}];
     if (bytes <= set) return cudaSuccess;
     e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+    // the largest shared-memory carveout, so that several CTAs of such a kernel fit an SM
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e == cudaSuccess) set = bytes;
     return e;
 }
