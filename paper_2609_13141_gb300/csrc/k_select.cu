@@ -430,6 +430,20 @@ __device__ __forceinline__ void compact_union(const uint32_t* bitmap, int diag, 
     if (lane == 0) *out_cnt = base;
 }
 
+// One warp turns a byte map of the tile's kept blocks (< diag) into a sorted list.
+__device__ __forceinline__ void compact_union_bytes(const uint8_t* map, int diag, int32_t* out, int32_t* out_cnt) {
+    const int lane = threadIdx.x & 31;
+    int base = 0;
+    for (int m0 = 0; m0 < diag; m0 += 32) {
+        const int m = m0 + lane;
+        const bool set = m < diag && map[m] != 0;
+        const uint32_t bal = __ballot_sync(0xffffffffu, set);
+        if (set) out[base + __popc(bal & ((1u << lane) - 1u))] = m;
+        base += __popc(bal);
+    }
+    if (lane == 0) *out_cnt = base;
+}
+
 // Shared-memory plan of the per-row state and outputs (bytes).
 __host__ __device__ constexpr size_t smem_topk_bytes(int K) { return K > 32 ? size_t(K) * kRows * 8 : 0; }
 __host__ __device__ constexpr size_t staging_bytes(int K) { return size_t(kRows) * (K + 1) * 8; }
@@ -544,7 +558,7 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
 //           that row runs replace-the-worst over all its scores.
 // Every pass places a score in its bin with the same rounded operations (no
 // contraction), so the passes agree on every score.
-constexpr int kBins = 48;                           // histogram bins per row (pass B)
+constexpr int kBins = 44;                           // histogram bins per row (pass B)
 constexpr int kBoundaryMax = 12;                    // boundary-bin scores a row's list holds beyond K
 constexpr size_t kHistBytes = size_t(kBins) * kRows * 4;
 // Bin arithmetic: v = 2^23 + (u - lo) / w, rounded to an integer by the add
@@ -559,17 +573,23 @@ constexpr int kChunk = 32;                          // blocks per score chunk (o
 constexpr int kRing = 3;                            // summary-chunk stages in shared memory
 constexpr int kListSmall = kBins;                   // list capacity when K + kBoundaryMax fits the histogram words
 constexpr int kListBig = 64 + kBoundaryMax;         // list capacity for larger K
+// Row stride (words) of the lists and histograms: row-major with an odd stride,
+// so that a warp's 32 rows fall in 32 different banks and a row's entries are
+// consecutive words (the copy-out reads them in order).
+__host__ __device__ constexpr int list_stride(int cap) { return (cap + 1) | 1; }
 
 // Shared-memory plan (bytes from the 1024-aligned base):
-//   [0, LIST): the rows' list blocks; before that the histograms (pass B),
-//              and during the projection a 64-column half of the Q tile;
+//   [0, LIST): the rows' list blocks (row r at word r * STRIDE); before that
+//              the histograms (bin b of row r at word r * STRIDE + b), and
+//              during the projection a 64-column half of the Q tile;
 //   [LIST, 2 LIST): the rows' list products;
 //   ring: the summary-chunk stages, during the projection a 64-column slice of Wq;
-//   then the union bitmap.
+//   then the tile's union map (one byte per block).
 template <int D, int DS, bool BIGK>
 struct SelProjCfg {
     static constexpr int CAP = BIGK ? kListBig : kListSmall;   // list entries per row
-    static constexpr int LIST_BYTES = CAP * kRows * 4;         // one of the two list arrays
+    static constexpr int STRIDE = list_stride(CAP);            // words between rows (odd)
+    static constexpr int LIST_BYTES = STRIDE * kRows * 4;      // one of the two list arrays
     static constexpr int QH_BYTES = kRows * 64 * 2;            // a 64-column half of the Q tile
     static constexpr int WQH_BYTES = DS * 64 * 2;              // a 64-column slice of Wq
     static constexpr int KC_BYTES = kChunk * DS * 2;           // one chunk of projected summaries
@@ -582,7 +602,7 @@ struct SelProjCfg {
     // TMEM (128 columns): q~ in fp32 at 0 .. DS-1 during the projection, then in
     // bf16 at 0 .. DS/2-1; the two score buffers at 64 and 96
     static constexpr int TMEM_S = 64;
-    static_assert(LIST_BYTES >= int(kHistBytes) && LIST_BYTES >= QH_BYTES, "histogram / Q half exceed the list");
+    static_assert(STRIDE >= kBins && LIST_BYTES >= QH_BYTES, "histogram / Q half exceed the list");
     static_assert(DS <= 128 && D % 64 == 0 && DS % 64 == 0, "projection shape");
 };
 
@@ -592,7 +612,7 @@ constexpr int kRowAll = 0, kRowNormal = 1, kRowFail = 2;   // C_i <= K: keep all
 
 template <int D, int DS, bool BIGK>
 __host__ __device__ constexpr size_t proj_smem_bytes(int C) {
-    return size_t(SelProjCfg<D, DS, BIGK>::OFF_BITMAP) + bitmap_bytes(C);
+    return size_t(SelProjCfg<D, DS, BIGK>::OFF_BITMAP) + ((C + 15) & ~15);
 }
 
 // Selection works on the raw products u = q~ . K~ (the scores are s = u / sqrt(d_sel),
@@ -622,10 +642,10 @@ struct RowSel {
 };
 
 // Shared-memory addresses of one row's list and histogram.
-constexpr uint32_t kListStep = kRows * 4;   // bytes between a row's list entries
+constexpr uint32_t kListStep = 4;   // bytes between a row's list entries
 struct RowAddr {
     uint32_t list;              // the row's list entry 0 (int32 block; its fp32 product OFF_LG bytes on); entry e at + e * kListStep
-    uint32_t hist_off;          // the row's histogram word of bin b at hist_off + bits(v) * kRows * 4 (mod 2^32)
+    uint32_t hist_off;          // the row's histogram word of bin b at hist_off + bits(v) * 4 (mod 2^32)
 };
 
 // Pass D state of a row: entries staged, worst kept product and its slot.
@@ -747,8 +767,8 @@ __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, i
         for (int j = 0; j < 32; j += 2) {
             float v0, v1;
             f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
-            red_shared_inc_if_ge(u[j], lo, ra.hist_off + __float_as_uint(fminf(v0, kBinTop)) * (kRows * 4u));
-            red_shared_inc_if_ge(u[j + 1], lo, ra.hist_off + __float_as_uint(fminf(v1, kBinTop)) * (kRows * 4u));
+            red_shared_inc_if_ge(u[j], lo, ra.hist_off + __float_as_uint(fminf(v0, kBinTop)) * 4u);
+            red_shared_inc_if_ge(u[j + 1], lo, ra.hist_off + __float_as_uint(fminf(v1, kBinTop)) * 4u);
         }
     } else if (kind == kPassC) {
         // v >= tb needs no clamp (tb <= kBinTop)
@@ -826,12 +846,13 @@ __device__ __forceinline__ void row_after_a(RowSel& rs, int Ci, int K) {
 }
 
 // After pass B: the bin holding the K-th largest product (scanning from the top).
-__device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, int r, int Kp) {
+// hist: the row's counters (bin b at hist[b]).
+__device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, int Kp) {
     if (rs.mode != kRowNormal) return;
     int cum = 0, bstar = -1, nabove = 0, nb = 0;
 #pragma unroll
     for (int b = kBins - 1; b >= 0; --b) {
-        const int cb = static_cast<int>(hist[b * kRows + r]);
+        const int cb = static_cast<int>(hist[b]);
         if (bstar < 0 && cum + cb >= Kp) {
             bstar = b;
             nabove = cum;
@@ -932,8 +953,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     uint8_t* ring = smem + Cfg::OFF_RING;                  // Wq slice (projection), then summary chunks
     uint32_t* hist = reinterpret_cast<uint32_t*>(smem);
     // list entry e of row r: block at word e * kRows + r, product OFF_LG bytes on
-    const Staging st{reinterpret_cast<int32_t*>(smem), reinterpret_cast<float*>(smem + Cfg::OFF_LG), 1, kRows};
-    uint32_t* bitmap = reinterpret_cast<uint32_t*>(smem + Cfg::OFF_BITMAP);
+    const Staging st{reinterpret_cast<int32_t*>(smem), reinterpret_cast<float*>(smem + Cfg::OFF_LG), Cfg::STRIDE, 1};
+    uint8_t* umap = smem + Cfg::OFF_BITMAP;   // union map: byte m set when some row keeps block m
 
     // the tile: its index within its sequence, the sequence's first row and
     // length, and the summary slot of the sequence's block 0 (packed sequences:
@@ -961,8 +982,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
     const bool resident = nchunks <= 2;
     const int rounds_total = G * (D / 64);   // projection rounds
 
-    const int nwords = (p.C + 31) >> 5;
-    for (int w = threadIdx.x; w < nwords; w += blockDim.x) bitmap[w] = 0u;
+    for (int w = threadIdx.x; w < ((p.C + 15) >> 2); w += blockDim.x) reinterpret_cast<uint32_t*>(umap)[w] = 0u;
     if (threadIdx.x == 0) {
         mbar_init(&in_full, 1);
         mbar_init(&in_empty, 1);
@@ -1124,7 +1144,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             if (lane == 0) mbar_arrive(&qt_ready);
         }
         // this row's counters, over the Q half once the projection has read it
-        for (int w = 0; w < kBins; ++w) hist[w * kRows + r] = 0u;
+        uint32_t* my_hist = hist + r * Cfg::STRIDE;
+        for (int w = 0; w < kBins; ++w) my_hist[w] = 0u;
         RowSel rs;
         rs.l = RowLse{-CUDART_INF_F, 0.f};
         rs.v0 = 0.f; rs.s1 = 0; rs.s2 = 0; rs.mn = CUDART_INF_F;
@@ -1136,8 +1157,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         const float c_exp = noisy ? kLog2e : p.score_scale * kLog2e;
         const float emit_scale = noisy ? 1.f : p.score_scale;
         const long long row_off = static_cast<long long>(bh) * p.N + geo.base + i;
-        const RowAddr ra{smem_u32(st.idx + r * st.stride),
-                         smem_u32(hist + r) - kBinMagicBits * static_cast<uint32_t>(kRows * 4)};
+        const RowAddr ra{smem_u32(st.idx + r * st.stride), smem_u32(my_hist) - kBinMagicBits * 4u};
         int gc = 0;
         for (int ps = 0; ok && ps < npre + 1; ++ps) {
             int kind;
@@ -1204,7 +1224,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
             if (kind == kPassA) {
                 row_after_a(rs, Ci, K);
             } else if (kind == kPassB) {
-                row_after_b(rs, hist, r, Kp);
+                row_after_b(rs, my_hist, Kp);
                 // whether pass D runs (some row failed), for the producer, the MMA
                 // issuer and the row warps: flag first, then one arrive per warp
                 if (rs.mode == kRowFail) atomicOr(&fail_flag, 1);
@@ -1228,7 +1248,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     const int m = st.idx[r * st.stride + e * st.es];
                     const float sc = __fmul_rn(st.lg[r * st.stride + e * st.es], emit_scale);
                     st.lg[r * st.stride + e * st.es] = staged_gate(sc, lse, p.gate_act);
-                    if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) atomicOr(&bitmap[m >> 5], 1u << (m & 31));
+                    if (static_cast<unsigned>(m) < static_cast<unsigned>(diag)) umap[m] = 1;   // same value from any row
                 } else {
                     st.idx[r * st.stride + e * st.es] = -1;
                     st.lg[r * st.stride + e * st.es] = 0.f;
@@ -1241,8 +1261,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 copy_out(st, p, bh, static_cast<long long>(geo.base) + t * kRows, min(kRows, seq_n - t * kRows),
                          static_cast<int>(threadIdx.x) - 64, 128);
             if (warp == 2)
-                compact_union(bitmap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + geo.slot) * p.C,
-                              p.union_cnt + static_cast<long long>(bh) * p.T + geo.slot);
+                compact_union_bytes(umap, diag, p.union_idx + (static_cast<long long>(bh) * p.T + geo.slot) * p.C,
+                                    p.union_cnt + static_cast<long long>(bh) * p.T + geo.slot);
         }
     }
     __syncthreads();
