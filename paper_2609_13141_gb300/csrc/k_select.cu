@@ -994,7 +994,7 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&s_free[b], 128);
+            mbar_init(&s_free[b], 4);   // one arrive per row warp
         }
         mbar_init(&drain_bar, 1);
         mbar_init(&plan_bar, 4);   // one arrive per row warp once its rows know their mode (after pass B)
@@ -1058,21 +1058,26 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                     mbar_wait_drain(&kc_full[q % kRing], (q / kRing) & 1, p.limit, p.status);
             }
         }
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer
+    } else if (warp == 1) {
+        // ---------------- MMA issuer (whole warp; the elected lane issues: one thread
+        // alone needs more cycles per tcgen05.mma issue)
         bool in_ok = nchunks > 0;
         const uint32_t q_addr = smem_u32(qh_s), w_addr = smem_u32(ring);   // projection operands
         for (int rd = 0; in_ok && rd < rounds_total; ++rd) {
-            if (!mbar_wait(&in_full, rd & 1, wc)) { in_ok = false; break; }
+            if (!mbar_wait_warp(&in_full, rd & 1, wc)) { in_ok = false; break; }
             tc_fence_after();
             // q~ (fp32, TMEM columns 0 .. DS-1) += Q half (128 x 64) * Wq slice (DS x 64)^T
+            if (elect_one()) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-                umma_bf16(tmem_base, smem_desc_sw128(q_addr + k * 32, 16, 1024),
-                          smem_desc_sw128(w_addr + k * 32, 16, 1024), Cfg::IDESC_PROJ, (rd > 0 || k > 0) ? 1u : 0u);
-            umma_commit(rd + 1 < rounds_total ? &in_empty : &proj_done);   // Q half and Wq slice free
+                for (int k = 0; k < 4; ++k)
+                    umma_bf16(tmem_base, smem_desc_sw128(q_addr + k * 32, 16, 1024),
+                              smem_desc_sw128(w_addr + k * 32, 16, 1024), Cfg::IDESC_PROJ,
+                              (rd > 0 || k > 0) ? 1u : 0u);
+                umma_commit(rd + 1 < rounds_total ? &in_empty : &proj_done);   // Q half and Wq slice free
+            }
+            __syncwarp();
         }
-        if (in_ok && mbar_wait(&qt_ready, 0, wc)) {
+        if (in_ok && mbar_wait_warp(&qt_ready, 0, wc)) {
             // S[gc&1] = q~ (128 x DS, bf16 in TMEM columns 0 .. DS/2) * Kt_chunk (32 x DS)^T,
             // for every chunk of every pass
             int gc = 0;
@@ -1082,28 +1087,34 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 if (resident && ps == npass) break;
                 if (ps == npass) {
                     if (!pass_b) break;
-                    if (!mbar_wait(&plan_bar, 0, wc)) break;
-                    if (!*reinterpret_cast<volatile int*>(&fail_flag)) break;
+                    if (!mbar_wait_warp(&plan_bar, 0, wc)) break;
+                    if (!__all_sync(0xffffffffu, *reinterpret_cast<volatile int*>(&fail_flag) != 0)) break;
                 }
                 for (int c = 0; c < nchunks; ++c, ++gc) {
                     const int s = gc % kRing, b = gc & 1;
-                    if (!mbar_wait(&kc_full[s], (gc / kRing) & 1, wc)) { ok = false; break; }
-                    if (!mbar_wait(&s_free[b], ((gc >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
+                    if (!mbar_wait_warp(&kc_full[s], (gc / kRing) & 1, wc)) { ok = false; break; }
+                    if (!mbar_wait_warp(&s_free[b], ((gc >> 1) & 1) ^ 1u, wc)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t k_addr = smem_u32(ring + s * Cfg::KC_BYTES);
+                    if (elect_one()) {
 #pragma unroll
-                    for (int k = 0; k < DS / 16; ++k) {
-                        const uint32_t off_k = (k >> 2) * (kChunk * 128) + (k & 3) * 32;
-                        umma_bf16_ta(tmem_base + Cfg::TMEM_S + b * kChunk, tmem_base + k * 8,
-                                     smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                        for (int k = 0; k < DS / 16; ++k) {
+                            const uint32_t off_k = (k >> 2) * (kChunk * 128) + (k & 3) * 32;
+                            umma_bf16_ta(tmem_base + Cfg::TMEM_S + b * kChunk, tmem_base + k * 8,
+                                         smem_desc_sw128(k_addr + off_k, 16, 1024), Cfg::IDESC_S, k > 0);
+                        }
+                        umma_commit(&s_full[b]);
+                        umma_commit(&kc_empty[s]);
                     }
-                    umma_commit(&s_full[b]);
-                    umma_commit(&kc_empty[s]);
+                    __syncwarp();
                 }
             }
         }
-        umma_commit(&drain_bar);
-        mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+        if (elect_one()) {
+            umma_commit(&drain_bar);
+            mbar_wait_drain(&drain_bar, 0, p.limit, p.status);
+        }
+        __syncwarp();
     } else if (warp >= 2) {
         // ---------------- row threads
         const int q = warp & 3;
@@ -1183,7 +1194,8 @@ select_proj_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_consta
                 tmem_wait_ld();
                 if (!resident) {
                     tc_fence_before();
-                    mbar_arrive(&s_free[b]);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&s_free[b]);
                 }
                 const int m0 = kChunk * c;
                 const int lim = Ci - m0;
