@@ -771,17 +771,20 @@ __device__ __forceinline__ void row_pass(RowSel& rs, int kind, const float* u, i
             red_shared_inc_if_ge(u[j + 1], lo, ra.hist_off + __float_as_uint(fminf(v1, kBinTop)) * 4u);
         }
     } else if (kind == kPassC) {
-        // v >= tb needs no clamp (tb <= kBinTop)
+        // v >= tb needs no clamp (tb <= kBinTop) and no test of u >= lo: a product
+        // below lo has v <= 2^23 < tb, as the boundary bin is at least bin 1
+        // (bin 0 sends the row to the fallback), and for rows that keep every
+        // score tb = -inf and v = +inf
         const uint64_t nlo2 = f32x2(-rs.lo, -rs.lo), iw2 = f32x2(rs.inv_w, rs.inv_w);
         const uint64_t mg2 = f32x2(kBinMagic, kBinMagic);
-        const float lo = rs.lo, tb = rs.tb;
+        const float tb = rs.tb;
         uint32_t addr = ra.list + static_cast<uint32_t>(rs.pos) * kListStep;
 #pragma unroll
         for (int j = 0; j < 32; j += 2) {
             float v0, v1;
             f32x2_split(fma_f32x2(add_f32x2(f32x2(u[j], u[j + 1]), nlo2), iw2, mg2), v0, v1);
-            st_shared_split_if_ge2<OFF_LG>(u[j], lo, v0, tb, addr, static_cast<uint32_t>(m0 + j), kListStep);
-            st_shared_split_if_ge2<OFF_LG>(u[j + 1], lo, v1, tb, addr, static_cast<uint32_t>(m0 + j + 1), kListStep);
+            st_shared_split_if_ge<OFF_LG>(u[j], v0, tb, addr, static_cast<uint32_t>(m0 + j), kListStep);
+            st_shared_split_if_ge<OFF_LG>(u[j + 1], v1, tb, addr, static_cast<uint32_t>(m0 + j + 1), kListStep);
         }
         rs.pos = static_cast<int>((addr - ra.list) / kListStep);
     } else {   // kPassD: replace-the-worst for the rows the bins could not resolve
@@ -860,7 +863,9 @@ __device__ __forceinline__ void row_after_b(RowSel& rs, const uint32_t* hist, in
         }
         cum += cb;
     }
-    if (bstar < 0) {   // fewer than K' products above lo: the estimate was too high
+    if (bstar <= 0) {
+        // fewer than K' products above lo (the estimate was too high), or the
+        // K-th in the lowest bin, which pass C cannot tell from just below lo
         row_set_fail(rs);
         return;
     }

@@ -352,16 +352,16 @@ __device__ __forceinline__ void red_shared_inc_if_ge(float u, float lo, uint32_t
                  "f"(lo), "r"(saddr)
                  : "memory");
 }
-// Stores m at addr and u at addr + OFF and advances addr by step when u >= lo
-// and v >= tb (false for NaN operands).
+// Stores m at addr and u at addr + OFF and advances addr by step when v >= tb
+// (false for a NaN v).
 template <uint32_t OFF>
-__device__ __forceinline__ void st_shared_split_if_ge2(float u, float lo, float v, float tb, uint32_t& addr,
-                                                       uint32_t m, uint32_t step) {
+__device__ __forceinline__ void st_shared_split_if_ge(float u, float v, float tb, uint32_t& addr, uint32_t m,
+                                                      uint32_t step) {
     asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ge.f32 p, %1, %2;\n\tsetp.ge.and.f32 p, %3, %4, p;\n\t"
-        "@p st.shared.b32 [%0], %5;\n\t@p st.shared.b32 [%0+%7], %6;\n\t@p add.u32 %0, %0, %8;\n\t}"
+        "{\n\t.reg .pred p;\n\tsetp.ge.f32 p, %1, %2;\n\t"
+        "@p st.shared.b32 [%0], %3;\n\t@p st.shared.b32 [%0+%5], %4;\n\t@p add.u32 %0, %0, %6;\n\t}"
         : "+r"(addr)
-        : "f"(u), "f"(lo), "f"(v), "f"(tb), "r"(m), "f"(u), "n"(OFF), "r"(step)
+        : "f"(v), "f"(tb), "r"(m), "f"(u), "n"(OFF), "r"(step)
         : "memory");
 }
 
