@@ -95,24 +95,6 @@ def algorithmic_flops(w, learned=True):
             "total": BH * (attn + sel) + mlp}
 
 
-def executed_attention_flops(unions, N, d, G, lens=None):
-    """FLOPs the attention kernel executes: every 128-row tile runs QK^T and PV
-    (4 * 128 * 64 * d) for each block of its union list plus its one or two
-    diagonal blocks, for each of the G query heads that share the list.
-    unions: per (KV group, tile) union counts of the last forward."""
-    per_block = 4 * 128 * 64 * d
-    if lens is None:
-        T = (N + 127) // 128
-        ndiag = [2 if (2 * t + 1) * 64 < N else 1 for t in range(T)]
-        total = sum(u + ndiag[k % T] for k, u in enumerate(unions))
-    else:
-        diag = []
-        for n in lens:
-            diag += [2 if (2 * t + 1) * 64 < n else 1 for t in range((n + 127) // 128)]
-        total = sum(unions) + sum(diag) * (len(unions) // max(len(diag), 1))
-    return G * total * per_block
-
-
 def packed_flops(w, learned=False):
     """algorithmic_flops summed over the packed sequences (the MLP runs on all tokens)."""
     att = sel = 0
@@ -325,6 +307,8 @@ def run_ours(args, w, rank, world):
         dist.barrier()
     launches = sas.sas_launch_count(h) - launches0
     kt = sas.sas_get_timings(h)
+    # the attention kernel's executed work in the last forward: (128-row tile, 64-key block) products
+    work_tiles, work_blocks = sas.sas_get_attention_work(h) if attn else (0, 0)
     sas.sas_set_timing(h, False)
     clocks = sampler.stop()
     ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
@@ -477,9 +461,9 @@ def run_ours(args, w, rank, world):
     }
     if attn:
         # the SAS attention kernel proper: algorithmic work (each row's kept keys)
-        # and executed work (every 128-row tile over its union of kept blocks)
+        # and executed work (every 128-row tile over the blocks it visits)
         a_avg = kt["attention"][1] / max(kt["attention"][0], 1)
-        exe = executed_attention_flops(unions, N, d, H // Hkv, lens)
+        exe = work_blocks * 4 * 128 * 64 * d
         a_alg = fl["attention"] / (a_avg / 1e3) / 1e12
         a_exe = exe / (a_avg / 1e3) / 1e12
         sas_ms = sum(kt[k][1] / max(kt[k][0], 1) for k in ("block_summaries", "selection", "attention"))
@@ -488,6 +472,8 @@ def run_ours(args, w, rank, world):
             "frac_of_bf16_peak": round(a_alg / peaks["bf16"], 4),
             "executed_tflop": round(exe / 1e12, 4), "executed_tflops": round(a_exe, 1),
             "executed_frac_of_bf16_peak": round(a_exe / peaks["bf16"], 4),
+            "tiles": work_tiles,
+            "mean_visited_blocks_per_tile": round(work_blocks / max(work_tiles, 1), 2),
             "mean_union_blocks_per_tile": round(sum(unions) / max(len(unions), 1), 2)}
         out["sas_layer"] = {"ms": round(sas_ms, 4),
                             "algorithmic_tflops": round((fl["attention"] + fl["selector"]) / (sas_ms / 1e3) / 1e12, 1),

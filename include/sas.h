@@ -368,6 +368,16 @@ sas_status sas_set_wait_limit(sas_handle* h, int64_t cycles);
  * history first).  Synchronises. */
 sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n);
 
+/* The work of the last attention forward: *tiles 128-row tiles computed and
+ * *tile_blocks (tile, 64-key block) products, each 4 * 128 * 64 * d FLOPs
+ * over QK^T and PV whether or not every row of the tile keeps the block.
+ * Tiles hold 128 rows of one query head, or with GQA (G >= 2, 128 a multiple
+ * of 8 G, [B, H, N, d] inputs, sparse scope) 128 / G tokens of each of the G
+ * query heads of a KV group: those share one kept list per token, so a tile
+ * visits the union of 128 / G tokens' kept blocks and its one diagonal block
+ * (head-packed tiles).  Synchronises. */
+sas_status sas_get_attention_work(sas_handle* h, int64_t* tiles, int64_t* tile_blocks);
+
 /* Failure-path self-test: launches one block that waits on an mbarrier that
  * nothing completes, with the library's bounded wait and a limit of
  * `limit_cycles` SM clock cycles, and returns in *host_status what the

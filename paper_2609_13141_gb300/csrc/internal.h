@@ -124,8 +124,19 @@ struct AttnArgs {
     // log g_m = full_table[row][m] - full_lse[row] (tables per KV group); null otherwise
     const float* full_table;
     const float* full_lse;
+    // head-packed GQA tiles (seg_rows = 128 / G tokens of each of the G heads;
+    // 0: tiles of 128 rows of one head): segment unions [BH/G][nseg][C] and
+    // their counts, nseg = ceil(N / seg_rows); [B, H, N, d] inputs only
+    int seg_rows;
+    int nseg;
+    const int32_t* seg_union_idx;
+    const int32_t* seg_union_cnt;
 };
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err);
+// Segment unions for head-packed tiles: per (KV group, segment of seg_rows
+// tokens) the sorted union of the tokens' kept blocks (from the kept lists).
+cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, int topk, int seg_rows, int nseg,
+                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env);
 
 // ---- decode step (Alg. 2, per-group selection over a paged cache).
 struct DecodeArgs {

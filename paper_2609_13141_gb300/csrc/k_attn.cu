@@ -29,6 +29,11 @@
 // reused once the PV two blocks back has read it.
 // The epilogue divides by the row sum and writes bf16 O and fp32 LSE.
 // GQA: K, V and the kept lists of query head bh are those of KV group bh / G.
+// Head-packed GQA tiles (G >= 2, 128 = G R): a tile takes R consecutive
+// tokens of all G query heads of a KV group (rows h R .. h R + R - 1 are head
+// h), which share one kept list per token, so the tile visits the union of R
+// tokens' kept blocks (one query block's worth at most) instead of two query
+// blocks' for each head; the segment unions come from seg_union_kernel.
 // Packed sequences: each tile's first row, tile index within its sequence and
 // sequence length come from the selection pass's tile table.
 #include <math_constants.h>
@@ -101,6 +106,9 @@ struct AttnParams {
     int* sched;             // [0] next work item, [1] CTAs finished; both zero between launches
     const float* full_table;   // full training scope: scores [BHkv][N][C] and normalisers [BHkv][N]
     const float* full_lse;
+    int seg_rows;              // head-packed tiles: tokens per head R (0: tiles of 128 rows of one head)
+    const int32_t* seg_union_idx;   // head-packed: [BHkv][T][C] segment unions (T = segments)
+    const int32_t* seg_union_cnt;
     float scale_log2;
     int* status;
     long long limit;
@@ -117,15 +125,41 @@ struct AttnParams {
 // run the same tile at about the same time over the same K, V blocks.
 
 struct TileRef {
-    int t, bh, kv;          // tile (within its sequence), query head, KV group (= bh without GQA)
+    int t, bh, kv;          // tile (within its sequence), query head (head-packed: the first), KV group
     int base, n;            // the sequence's first row in the token axis and its length
+    int row0;               // the tile's first token row within the sequence
+    int diag0, ndiag;       // its diagonal blocks: diag0 .. diag0 + ndiag - 1
     const int32_t* ulist;   // the tile's union list (ascending historical blocks)
     int U;                  // its length
 };
 
-// T: tile slots in use (p.T, or the packed sequences' tile count).
+// T: tile slots in use (p.T, or the packed sequences' tile count; head-packed: segments).
 __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w, int T) {
     TileRef x;
+    if (p.seg_rows > 0) {
+        // head-packed: items over (KV group, segment), the group varying fastest
+        // within L2-sized groups of KV groups, longest history first
+        const int BHkv = p.BH / p.G;
+        const int gkv = max(1, p.group / p.G);
+        const int per_group = gkv * T;
+        const int g0 = w / per_group;
+        const int k0 = g0 * gkv;
+        const int gs = min(gkv, BHkv - k0);
+        const int wi = w - g0 * per_group;
+        const int sg = T - 1 - wi / gs;
+        x.kv = k0 + wi % gs;
+        x.bh = x.kv * p.G;
+        x.t = sg;
+        x.base = 0;
+        x.n = p.N;
+        x.row0 = sg * p.seg_rows;
+        x.diag0 = x.row0 >> 6;   // all R <= 64 tokens share one block
+        x.ndiag = 1;
+        const long long tb = static_cast<long long>(x.kv) * T + sg;
+        x.ulist = p.seg_union_idx + tb * min(p.C, p.seg_rows * max(p.topk, 1));   // rows of min(C, R K) entries
+        x.U = p.full_table != nullptr ? x.diag0 : __ldg(p.seg_union_cnt + tb);
+        return x;
+    }
     const int per_group = p.group * T;                    // items of a full group
     const int g0 = w / per_group;                         // group index
     const int h0 = g0 * p.group;                          // its first head
@@ -146,6 +180,9 @@ __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w, int T) {
     }
     x.bh = h0 + wi % gs;
     x.kv = x.bh / p.G;
+    x.row0 = x.t * kBM;
+    x.diag0 = 2 * x.t;
+    x.ndiag = (2 * x.t + 1) * kBN < x.n ? 2 : 1;
     const long long tb = static_cast<long long>(x.kv) * p.T + slot;
     x.ulist = p.union_idx + tb * p.C;
     // full scope: every historical block of the tile (blocks 0 .. 2t-1, all full)
@@ -164,12 +201,12 @@ __device__ __forceinline__ bool read_item(AttnCtl& ctl, int r, const WaitCtl& wc
 
 // visited blocks of a tile: its union list, then the diagonal block(s)
 __device__ __forceinline__ int tile_blocks(const AttnParams& p, const TileRef& x) {
-    return x.U + ((2 * x.t + 1) * kBN < x.n ? 2 : 1);
+    return x.U + x.ndiag;
 }
 
 template <bool FULL>
 __device__ __forceinline__ int block_at(const TileRef& x, int j) {
-    return j < x.U ? (FULL ? j : __ldg(x.ulist + j)) : 2 * x.t + (j - x.U);
+    return j < x.U ? (FULL ? j : __ldg(x.ulist + j)) : x.diag0 + (j - x.U);
 }
 
 // OUTER: the gate of a kept block multiplies its probabilities after the
@@ -205,8 +242,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
     int& abort_flag = ctl.abort_flag;
 
     const uint32_t warp = warp_id(), lane = lane_id();
-    const int Tn = p.tiles == nullptr ? p.T : __ldg(p.ntiles);   // tile slots in use
-    const int W = Tn * p.BH;
+    const int Tn = p.tiles == nullptr ? p.T : __ldg(p.ntiles);   // tile slots in use (head-packed: segments)
+    const int W = Tn * (p.seg_rows > 0 ? p.BH / p.G : p.BH);
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
@@ -294,9 +331,18 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             const int n = tile_blocks(p, x);
             if (!mbar_wait(&q_empty, (tc & 1) ^ 1u, wc)) { ok = false; break; }
             mbar_arrive_expect_tx(&q_full, Cfg::Q_BYTES);
+            if (p.seg_rows > 0) {
+                // R rows of each of the G heads (the Q map's box is R rows high)
+                for (int hq = 0; hq < p.G; ++hq)
 #pragma unroll
-            for (int a = 0; a < D / 64; ++a)
-                tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, x.base + x.t * kBM, x.bh);
+                    for (int a = 0; a < D / 64; ++a)
+                        tma_load_3d(smem + a * (kBM * 128) + hq * p.seg_rows * 128, &mapQ, &q_full, a * 64,
+                                    x.base + x.row0, x.bh + hq);
+            } else {
+#pragma unroll
+                for (int a = 0; a < D / 64; ++a)
+                    tma_load_3d(smem + a * (kBM * 128), &mapQ, &q_full, a * 64, x.base + x.row0, x.bh);
+            }
             ++nq;
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
@@ -424,12 +470,13 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             if (w < 0) break;
             const TileRef x = tile_ref(p, w, Tn);
             const int n = tile_blocks(p, x);
-            const int t = x.t;
-            const int i = t * kBM + r_row;   // row within its sequence
+            // the row's query head and token (within its sequence)
+            const int hq = p.seg_rows > 0 ? r_row / p.seg_rows : 0;
+            const int i = x.row0 + (p.seg_rows > 0 ? r_row - hq * p.seg_rows : r_row);
             const bool valid = i < x.n;
             const int c = i >> 6;
             const int nsel = (valid && !FULL) ? min(p.topk, c) : 0;
-            const long long row_off = static_cast<long long>(x.bh) * p.N + x.base + i;   // O, LSE
+            const long long row_off = static_cast<long long>(x.bh + hq) * p.N + x.base + i;   // O, LSE
             const long long sel_off = static_cast<long long>(x.kv) * p.N + x.base + i;   // the group's kept list
             const int32_t* my_idx = p.sel_idx + sel_off * p.topk;
             const float* my_lg = p.sel_logg + sel_off * p.topk;
@@ -472,7 +519,7 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
             for (int j = 0; j < n; ++j) {
                 const int gb = g + j;
                 const int pb = gb & 1;
-                const int m = FULL ? block_at<true>(x, j) : (j < x.U ? raw_next : 2 * t + (j - x.U));
+                const int m = FULL ? block_at<true>(x, j) : (j < x.U ? raw_next : x.diag0 + (j - x.U));
                 if (!FULL && j + 1 < x.U) raw_next = __ldg(x.ulist + j + 1);
                 // gate (log2 units) and the last visible key column of block m for this row
                 float bias = 0.f;
@@ -682,7 +729,11 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev);
     if (e != cudaSuccess) { *err = "device attributes"; return e; }
     CUtensorMap mq, mk, mv;
-    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, kBM) != 0) { *err = "tensor map Q"; return cudaErrorInvalidValue; }
+    const bool hp = a.seg_rows > 0;   // head-packed tiles: the Q box is one head's seg_rows rows
+    if (make_tmap_bf16_3d(&mq, a.Q, D, a.N, a.BH, 64, hp ? a.seg_rows : kBM) != 0) {
+        *err = "tensor map Q";
+        return cudaErrorInvalidValue;
+    }
     const int BHkv = a.BH / a.G;
     if (make_tmap_bf16_3d(&mk, a.K, D, a.N, BHkv, 64, kBN) != 0) { *err = "tensor map K"; return cudaErrorInvalidValue; }
     if (make_tmap_bf16_3d(&mv, a.V, D, a.N, BHkv, 64, kBN) != 0) { *err = "tensor map V"; return cudaErrorInvalidValue; }
@@ -693,7 +744,10 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.union_cnt = a.union_cnt;
     p.sel_idx = a.sel_idx;
     p.sel_logg = a.sel_logg;
-    p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
+    p.N = a.N; p.C = a.C; p.T = hp ? a.nseg : a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
+    p.seg_rows = hp ? a.seg_rows : 0;
+    p.seg_union_idx = a.seg_union_idx;
+    p.seg_union_cnt = a.seg_union_cnt;
     p.G = a.G;
     p.tiles = a.tiles;
     p.ntiles = a.ntiles;
@@ -710,7 +764,7 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.full_table = a.full_table;
     p.full_lse = a.full_lse;
     // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
-    const long long items = static_cast<long long>(a.T) * a.BH;
+    const long long items = hp ? static_cast<long long>(a.nseg) * BHkv : static_cast<long long>(a.T) * a.BH;
     const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);
     attn_kernel<D, OUTER, FULL><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
     e = cudaGetLastError();
@@ -723,6 +777,12 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
 cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** err) {
     if (a.G < 1 || a.BH % a.G != 0) {
         *err = "attention: query heads must fill whole KV groups";
+        return cudaErrorInvalidValue;
+    }
+    if (a.seg_rows > 0 && (a.G < 2 || a.seg_rows * a.G != kBM || a.seg_rows % 8 != 0 || a.tiles != nullptr ||
+                           a.full_table != nullptr || a.seg_union_idx == nullptr || a.seg_union_cnt == nullptr)) {
+        *err = "attention: head-packed tiles need G >= 2 with 128 = G x seg_rows (a multiple of 8), [B, H, N, d] "
+               "inputs and the sparse scope";
         return cudaErrorInvalidValue;
     }
     const bool outer = a.gate_pos == 1;

@@ -1430,6 +1430,56 @@ cudaError_t launch_varlen_tiles(const int32_t* cu, int S, int Ncap, int max_len,
     return cudaGetLastError();
 }
 
+namespace {
+
+// Head-packed GQA tiles: per (KV group, segment of R tokens) the sorted union
+// of the tokens' kept blocks, from the kept lists.  One warp per segment; its
+// tokens share one current block c (R <= 64, segments aligned), and kept
+// blocks are < c.  cap: row stride of the output lists (>= min(C, R topk)).
+__global__ void __launch_bounds__(256) seg_union_kernel(const int32_t* sel_idx, int BHkv, int N, int C, int topk,
+                                                        int R, int nseg, int cap, int32_t* out_idx,
+                                                        int32_t* out_cnt) {
+    extern __shared__ uint32_t segbits[];   // per warp: ceil(C / 32) words
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long item = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + warp;
+    if (item >= static_cast<long long>(BHkv) * nseg) return;   // no block-wide synchronisation below
+    const int kv = static_cast<int>(item / nseg), sg = static_cast<int>(item - static_cast<long long>(kv) * nseg);
+    const int nw = (C + 31) >> 5;
+    uint32_t* bits = segbits + warp * nw;
+    for (int w = lane; w < nw; w += 32) bits[w] = 0u;
+    __syncwarp();
+    const int i0 = sg * R;
+    for (int rr = lane; rr < R; rr += 32) {
+        const int i = i0 + rr;
+        if (i >= N) break;
+        const int c = i >> 6;
+        const int ne = min(topk, c);
+        const int32_t* idx = sel_idx + (static_cast<long long>(kv) * N + i) * topk;
+        for (int e = 0; e < ne; ++e) {
+            const int m = __ldg(idx + e);
+            if (static_cast<unsigned>(m) < static_cast<unsigned>(c)) atomicOr(&bits[m >> 5], 1u << (m & 31));
+        }
+    }
+    __syncwarp();
+    compact_union(bits, i0 >> 6, out_idx + item * cap, out_cnt + item);
+}
+
+}  // namespace
+
+cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, int topk, int seg_rows, int nseg,
+                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env) {
+    const long long items = static_cast<long long>(BHkv) * nseg;
+    const size_t smem = static_cast<size_t>(8) * ((C + 31) / 32) * 4;
+    if (smem > 48 * 1024) {
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(seg_union_kernel), smem);
+        if (e != cudaSuccess) return e;
+    }
+    const int cap = min(C, seg_rows * max(topk, 1));
+    seg_union_kernel<<<static_cast<unsigned>((items + 7) / 8), 256, smem, env.stream>>>(
+        sel_idx, BHkv, N, C, topk, seg_rows, nseg, cap, seg_union_idx, seg_union_cnt);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
     SelParams p;
     p.BH = a.BH; p.N = a.N; p.C = a.C; p.T = a.T; p.F = a.F; p.topk = a.topk;

@@ -7,6 +7,7 @@
 #include <map>
 #include <mutex>
 #include <string>
+#include <algorithm>
 #include <vector>
 
 #include <cudaTypedefs.h>
@@ -129,6 +130,11 @@ struct sas_handle {
     int BH = 0, C = 0, T = 0, F = 0;
     int Hkv = 0, G = 1, BHkv = 0;   // KV heads, query heads per group, KV groups x batch
     bool varlen = false;            // packed sequences: T = tile slots, C from max_seqlen
+    // head-packed GQA attention tiles (G >= 2, 128 = G seg_rows): segment unions
+    int seg_rows = 0, nseg = 0, seg_cap = 0;
+    int32_t* seg_union_idx = nullptr;   // [BHkv][nseg][seg_cap]
+    int32_t* seg_union_cnt = nullptr;   // [BHkv][nseg]
+    int last_fwd = 0;                   // tiles of the last forward: 0 per head, 1 head-packed, 2 packed sequences
     int4* tiles = nullptr;          // packed sequences' tile table [T] and its count
     int* ntiles = nullptr;
     int* tile_off = nullptr;    // first slot of every local tile index (see launch_varlen_tiles)
@@ -315,6 +321,16 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
         if (e == cudaSuccess) e = cudaMemset(h->ntiles, 0, 16);
         if (e == cudaSuccess) e = alloc(&h->tile_off, static_cast<size_t>((max_len + 127) / 128 + 2) * 4);
     }
+    // head-packed attention tiles: G query heads x 128 / G tokens share one kept
+    // list per token (sparse scope, [B, H, N, d] inputs)
+    if (!varlen && !h->full && h->G >= 2 && 128 % h->G == 0 && (128 / h->G) % 8 == 0 && c.topk > 0) {
+        h->seg_rows = 128 / h->G;
+        h->nseg = (c.N + h->seg_rows - 1) / h->seg_rows;
+        h->seg_cap = std::min(h->C, h->seg_rows * c.topk);
+        if (e == cudaSuccess)
+            e = alloc(&h->seg_union_idx, static_cast<size_t>(BHkv) * h->nseg * std::max(h->seg_cap, 1) * 4);
+        if (e == cudaSuccess) e = alloc(&h->seg_union_cnt, static_cast<size_t>(BHkv) * h->nseg * 4);
+    }
     if (h->full) {
         if (e == cudaSuccess) e = alloc(&h->full_lse, rows * 4);
         if (e == cudaSuccess && c.selector == SAS_SEL_MEANPOOL_PROJ)
@@ -349,6 +365,8 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->sched);
     cudaFree(h->full_lse);
     cudaFree(h->full_table);
+    cudaFree(h->seg_union_idx);
+    cudaFree(h->seg_union_cnt);
     cudaFree(h->hidden);
     cudaFree(h->bwd_delta);
     cudaFree(h->bwd_inv);
@@ -420,6 +438,14 @@ sas_status attention_fwd(sas_handle* h, const void* Q, const void* K, const void
     }
     e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
+    if (h->seg_rows > 0) {
+        // the segment unions of the head-packed attention tiles (timed with the selection)
+        e = timed_launch(h, 2, s, [&] {
+            return sas::launch_seg_unions(out_idx, h->BHkv, c.N, h->C, c.topk, h->seg_rows, h->nseg, h->seg_union_idx,
+                                          h->seg_union_cnt, env);
+        });
+        if (e != cudaSuccess) return cuda_fail(h, e, "segment unions");
+    }
     // a5: gated sparse attention
     sas::AttnArgs aa{};
     aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
@@ -434,6 +460,13 @@ sas_status attention_fwd(sas_handle* h, const void* Q, const void* K, const void
         aa.full_table = c.selector == SAS_SEL_SCORES_GIVEN ? scores : h->full_table;
         aa.full_lse = h->full_lse;
     }
+    if (h->seg_rows > 0) {
+        aa.seg_rows = h->seg_rows;
+        aa.nseg = h->nseg;
+        aa.seg_union_idx = h->seg_union_idx;
+        aa.seg_union_cnt = h->seg_union_cnt;
+    }
+    h->last_fwd = h->seg_rows > 0 ? 1 : 0;
     e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     return SAS_OK;
@@ -744,6 +777,48 @@ sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n
     cudaError_t e = cudaDeviceSynchronize();
     if (e == cudaSuccess) e = cudaMemcpy(host_out, h->union_cnt, total * 4, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(h, e, "union counts");
+    return SAS_OK;
+}
+
+sas_status sas_get_attention_work(sas_handle* h, int64_t* tiles, int64_t* tile_blocks) {
+    if (h == nullptr || tiles == nullptr || tile_blocks == nullptr) return SAS_ERR_INVALID_ARG;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(h, e, "synchronize");
+    const int N = h->cfg.N;
+    int64_t nt = 0, nb = 0;
+    auto ndiag = [](int t, int n) { return (2 * t + 1) * 64 < n ? 2 : 1; };
+    if (h->last_fwd == 1) {
+        // head-packed: one tile per (KV group, segment), its union and one diagonal block
+        std::vector<int32_t> cnt(static_cast<size_t>(h->BHkv) * h->nseg);
+        e = cudaMemcpy(cnt.data(), h->seg_union_cnt, cnt.size() * 4, cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return cuda_fail(h, e, "segment union counts");
+        for (int32_t u : cnt) nb += u + 1;
+        nt = static_cast<int64_t>(cnt.size());
+    } else {
+        // one tile per (query head, tile slot): its group's union and one or two diagonal blocks
+        std::vector<int32_t> cnt(static_cast<size_t>(h->BHkv) * h->T);
+        e = cudaMemcpy(cnt.data(), h->union_cnt, cnt.size() * 4, cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return cuda_fail(h, e, "union counts");
+        std::vector<int4> tl;
+        int used = h->T;
+        if (h->varlen) {
+            e = cudaMemcpy(&used, h->ntiles, 4, cudaMemcpyDeviceToHost);
+            tl.resize(static_cast<size_t>(std::max(used, 0)));
+            if (e == cudaSuccess && used > 0)
+                e = cudaMemcpy(tl.data(), h->tiles, tl.size() * sizeof(int4), cudaMemcpyDeviceToHost);
+            if (e != cudaSuccess) return cuda_fail(h, e, "tile table");
+        }
+        for (int kv = 0; kv < h->BHkv; ++kv)
+            for (int g = 0; g < used; ++g) {
+                const int t = h->varlen ? tl[g].y : g;
+                const int n = h->varlen ? tl[g].z : N;
+                const int u = h->full ? 2 * t : cnt[static_cast<size_t>(kv) * h->T + g];
+                nb += static_cast<int64_t>(h->G) * (u + ndiag(t, n));
+                nt += h->G;
+            }
+    }
+    *tiles = nt;
+    *tile_blocks = nb;
     return SAS_OK;
 }
 

@@ -108,6 +108,8 @@ def lib():
     L.sas_set_wait_limit.restype = i32
     L.sas_get_tile_union_counts.argtypes = [vp, ctypes.POINTER(i32), i64]
     L.sas_get_tile_union_counts.restype = i32
+    L.sas_get_attention_work.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(i64)]
+    L.sas_get_attention_work.restype = i32
     L.sas_mlp_fwd_noalloc.argtypes = [vp] * 6 + [i64, i64, i64, vp]
     L.sas_mlp_fwd_noalloc.restype = i32
     L.sas_mlp_noalloc_get_device_status.argtypes = [ctypes.POINTER(i32)]
@@ -318,6 +320,13 @@ def sas_get_tile_union_counts(h, n):
     out = (ctypes.c_int32 * n)()
     _check(lib().sas_get_tile_union_counts(h, out, n), h, "sas_get_tile_union_counts")
     return list(out)
+
+
+def sas_get_attention_work(h):
+    """(tiles, tile_blocks) of the last attention forward (see sas.h)."""
+    t, b = ctypes.c_int64(0), ctypes.c_int64(0)
+    _check(lib().sas_get_attention_work(h, ctypes.byref(t), ctypes.byref(b)), h, "sas_get_attention_work")
+    return t.value, b.value
 
 
 def sas_selftest_wait_timeout(limit_cycles):

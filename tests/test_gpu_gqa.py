@@ -89,6 +89,32 @@ def test_qwen3_4b_shaped_prefill_sampled_rows():
         P.check_selection_rows(gi, P.f64(S[bi, hi // 4])[rows], rows, topk)
 
 
+@pytest.mark.parametrize("G,Hkv,N,topk", [
+    (2, 2, 700, 4),     # 64 tokens of 2 heads per tile
+    (8, 1, 517, 3),     # 16 tokens of 8 heads
+    (16, 1, 389, 2),    # 8 tokens of 16 heads
+])
+def test_head_packed_tiles_match_oracle(G, Hkv, N, topk):
+    # tiles of 128 / G tokens x the G heads of a KV group (one kept list per token):
+    # every row against the oracle, and the tile count of the work the kernel did
+    Hq = G * Hkv
+    Q, K, V, S = _inputs(1, Hq, Hkv, N, 128, seed=G + N)
+    layer = sas.SasLayer(1, Hq, N, 128, topk, Hkv=Hkv)
+    dev = torch.device("cuda:0")
+    O, LSE, si, sl = layer.attention(*(t.to(dev).contiguous() for t in (Q, K, V)), scores=S.to(dev).contiguous())
+    tiles, blocks = sas.sas_get_attention_work(layer.h)
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    R = 128 // G
+    assert tiles == Hkv * -(-N // R)
+    assert blocks >= tiles   # every tile visits at least its diagonal block
+    ref = OR.sas_attention_gqa(P.f64(Q), P.f64(K), P.f64(V), 64, topk, P.f64(S))
+    for hi in range(Hq):
+        r = ref[(0, hi)]
+        P.compare_o(P.f64(O[0, hi].cpu()), r["O"], f"O[0,{hi}]")
+        assert np.abs(LSE[0, hi].cpu().numpy() - r["LSE"]).max() <= P.LSE_MAX_ABS
+
+
 @pytest.mark.parametrize("B,Hq,Hkv,N,d,d_sel,topk", [
     (1, 8, 2, 1000, 128, 128, 4),     # G = 4
     (2, 4, 2, 700, 64, 64, 3),        # G = 2, d = 64
