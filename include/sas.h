@@ -372,10 +372,11 @@ sas_status sas_get_tile_union_counts(sas_handle* h, int32_t* host_out, int64_t n
  * *tile_blocks (tile, 64-key block) products, each 4 * 128 * 64 * d FLOPs
  * over QK^T and PV whether or not every row of the tile keeps the block.
  * Tiles hold 128 rows of one query head, or with GQA (G >= 2, 128 a multiple
- * of 8 G, [B, H, N, d] inputs, sparse scope) 128 / G tokens of each of the G
- * query heads of a KV group: those share one kept list per token, so a tile
- * visits the union of 128 / G tokens' kept blocks and its one diagonal block
- * (head-packed tiles).  Synchronises. */
+ * of 8 G, sparse scope) 128 / G tokens of each of the G query heads of a KV
+ * group: those share one kept list per token, so a tile visits the union of
+ * 128 / G tokens' kept blocks and its one diagonal block (head-packed tiles;
+ * packed sequences: G such tiles per 128-row tile of a sequence, the last
+ * ones possibly past its end and empty).  Synchronises. */
 sas_status sas_get_attention_work(sas_handle* h, int64_t* tiles, int64_t* tile_blocks);
 
 /* Failure-path self-test: launches one block that waits on an mbarrier that

@@ -125,8 +125,9 @@ struct AttnArgs {
     const float* full_table;
     const float* full_lse;
     // head-packed GQA tiles (seg_rows = 128 / G tokens of each of the G heads;
-    // 0: tiles of 128 rows of one head): segment unions [BH/G][nseg][C] and
-    // their counts, nseg = ceil(N / seg_rows); [B, H, N, d] inputs only
+    // 0: tiles of 128 rows of one head): segment unions [BH/G][nseg][cap]
+    // (cap = min(C, seg_rows topk)) and their counts; nseg = ceil(N / seg_rows),
+    // or with packed sequences G per tile slot (nseg = T G, part k of slot g at g G + k)
     int seg_rows;
     int nseg;
     const int32_t* seg_union_idx;
@@ -136,7 +137,8 @@ cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** er
 // Segment unions for head-packed tiles: per (KV group, segment of seg_rows
 // tokens) the sorted union of the tokens' kept blocks (from the kept lists).
 cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, int topk, int seg_rows, int nseg,
-                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env);
+                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env,
+                              const int4* tiles = nullptr, const int* ntiles = nullptr);
 
 // ---- decode step (Alg. 2, per-group selection over a paged cache).
 struct DecodeArgs {

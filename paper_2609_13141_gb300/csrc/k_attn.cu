@@ -138,24 +138,33 @@ __device__ __forceinline__ TileRef tile_ref(const AttnParams& p, int w, int T) {
     TileRef x;
     if (p.seg_rows > 0) {
         // head-packed: items over (KV group, segment), the group varying fastest
-        // within L2-sized groups of KV groups, longest history first
+        // within L2-sized groups of KV groups, longest history first.  Packed
+        // sequences: segment sg is part sg % G of the table's tile slot sg / G.
         const int BHkv = p.BH / p.G;
+        const int Ts = p.tiles == nullptr ? T : T * p.G;   // segments in use
         const int gkv = max(1, p.group / p.G);
-        const int per_group = gkv * T;
+        const int per_group = gkv * Ts;
         const int g0 = w / per_group;
         const int k0 = g0 * gkv;
         const int gs = min(gkv, BHkv - k0);
         const int wi = w - g0 * per_group;
-        const int sg = T - 1 - wi / gs;
+        const int sg = p.tiles == nullptr ? Ts - 1 - wi / gs : wi / gs;
         x.kv = k0 + wi % gs;
         x.bh = x.kv * p.G;
         x.t = sg;
-        x.base = 0;
-        x.n = p.N;
-        x.row0 = sg * p.seg_rows;
+        if (p.tiles == nullptr) {
+            x.base = 0;
+            x.n = p.N;
+            x.row0 = sg * p.seg_rows;
+        } else {
+            const int4 v = __ldg(p.tiles + sg / p.G);
+            x.base = v.x;
+            x.n = v.z;
+            x.row0 = v.y * kBM + (sg % p.G) * p.seg_rows;
+        }
         x.diag0 = x.row0 >> 6;   // all R <= 64 tokens share one block
         x.ndiag = 1;
-        const long long tb = static_cast<long long>(x.kv) * T + sg;
+        const long long tb = static_cast<long long>(x.kv) * p.T + sg;   // p.T: segment slots per KV group
         x.ulist = p.seg_union_idx + tb * min(p.C, p.seg_rows * max(p.topk, 1));   // rows of min(C, R K) entries
         x.U = p.full_table != nullptr ? x.diag0 : __ldg(p.seg_union_cnt + tb);
         return x;
@@ -243,7 +252,8 @@ attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CU
 
     const uint32_t warp = warp_id(), lane = lane_id();
     const int Tn = p.tiles == nullptr ? p.T : __ldg(p.ntiles);   // tile slots in use (head-packed: segments)
-    const int W = Tn * (p.seg_rows > 0 ? p.BH / p.G : p.BH);
+    // head-packed: G segments per tile slot of packed sequences
+    const int W = p.seg_rows > 0 ? (p.tiles == nullptr ? Tn : Tn * p.G) * (p.BH / p.G) : Tn * p.BH;
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
@@ -764,6 +774,7 @@ cudaError_t launch_d(const AttnArgs& a, const KernelEnv& env, const char** err) 
     p.full_table = a.full_table;
     p.full_lse = a.full_lse;
     // persistent grid: two CTAs per SM (their shared memory and TMEM both fit twice)
+    // head-packed: segments (packed sequences: G per tile slot; the slot count caps the grid)
     const long long items = hp ? static_cast<long long>(a.nseg) * BHkv : static_cast<long long>(a.T) * a.BH;
     const int G = static_cast<int>(items < 2LL * sms ? items : 2LL * sms);
     attn_kernel<D, OUTER, FULL><<<G, kThreads, Cfg::SMEM, env.stream>>>(mq, mk, mv, p);
@@ -779,10 +790,9 @@ cudaError_t launch_attn(const AttnArgs& a, const KernelEnv& env, const char** er
         *err = "attention: query heads must fill whole KV groups";
         return cudaErrorInvalidValue;
     }
-    if (a.seg_rows > 0 && (a.G < 2 || a.seg_rows * a.G != kBM || a.seg_rows % 8 != 0 || a.tiles != nullptr ||
-                           a.full_table != nullptr || a.seg_union_idx == nullptr || a.seg_union_cnt == nullptr)) {
-        *err = "attention: head-packed tiles need G >= 2 with 128 = G x seg_rows (a multiple of 8), [B, H, N, d] "
-               "inputs and the sparse scope";
+    if (a.seg_rows > 0 && (a.G < 2 || a.seg_rows * a.G != kBM || a.seg_rows % 8 != 0 || a.full_table != nullptr ||
+                           a.seg_union_idx == nullptr || a.seg_union_cnt == nullptr)) {
+        *err = "attention: head-packed tiles need G >= 2 with 128 = G x seg_rows (a multiple of 8) and the sparse scope";
         return cudaErrorInvalidValue;
     }
     const bool outer = a.gate_pos == 1;

@@ -1436,9 +1436,10 @@ namespace {
 // of the tokens' kept blocks, from the kept lists.  One warp per segment; its
 // tokens share one current block c (R <= 64, segments aligned), and kept
 // blocks are < c.  cap: row stride of the output lists (>= min(C, R topk)).
+// Packed sequences: segment sg is part sg % G of tile slot sg / G (G = 128 / R).
 __global__ void __launch_bounds__(256) seg_union_kernel(const int32_t* sel_idx, int BHkv, int N, int C, int topk,
                                                         int R, int nseg, int cap, int32_t* out_idx,
-                                                        int32_t* out_cnt) {
+                                                        int32_t* out_cnt, const int4* tiles, const int* ntiles) {
     extern __shared__ uint32_t segbits[];   // per warp: ceil(C / 32) words
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long item = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + warp;
@@ -1448,13 +1449,22 @@ __global__ void __launch_bounds__(256) seg_union_kernel(const int32_t* sel_idx, 
     uint32_t* bits = segbits + warp * nw;
     for (int w = lane; w < nw; w += 32) bits[w] = 0u;
     __syncwarp();
-    const int i0 = sg * R;
+    // the segment's first token within its sequence, the sequence's first row and length
+    int i0 = sg * R, base = 0, n = N;
+    if (tiles != nullptr) {
+        const int G = kRows / R;
+        if (sg / G >= __ldg(ntiles)) return;   // an unused slot: the attention does not read it
+        const int4 v = __ldg(tiles + sg / G);
+        i0 = v.y * kRows + (sg % G) * R;
+        base = v.x;
+        n = v.z;
+    }
     for (int rr = lane; rr < R; rr += 32) {
         const int i = i0 + rr;
-        if (i >= N) break;
+        if (i >= n) break;
         const int c = i >> 6;
         const int ne = min(topk, c);
-        const int32_t* idx = sel_idx + (static_cast<long long>(kv) * N + i) * topk;
+        const int32_t* idx = sel_idx + (static_cast<long long>(kv) * N + base + i) * topk;
         for (int e = 0; e < ne; ++e) {
             const int m = __ldg(idx + e);
             if (static_cast<unsigned>(m) < static_cast<unsigned>(c)) atomicOr(&bits[m >> 5], 1u << (m & 31));
@@ -1467,7 +1477,8 @@ __global__ void __launch_bounds__(256) seg_union_kernel(const int32_t* sel_idx, 
 }  // namespace
 
 cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, int topk, int seg_rows, int nseg,
-                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env) {
+                              int32_t* seg_union_idx, int32_t* seg_union_cnt, const KernelEnv& env, const int4* tiles,
+                              const int* ntiles) {
     const long long items = static_cast<long long>(BHkv) * nseg;
     const size_t smem = static_cast<size_t>(8) * ((C + 31) / 32) * 4;
     if (smem > 48 * 1024) {
@@ -1476,7 +1487,7 @@ cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, in
     }
     const int cap = min(C, seg_rows * max(topk, 1));
     seg_union_kernel<<<static_cast<unsigned>((items + 7) / 8), 256, smem, env.stream>>>(
-        sel_idx, BHkv, N, C, topk, seg_rows, nseg, cap, seg_union_idx, seg_union_cnt);
+        sel_idx, BHkv, N, C, topk, seg_rows, nseg, cap, seg_union_idx, seg_union_cnt, tiles, ntiles);
     return cudaGetLastError();
 }
 

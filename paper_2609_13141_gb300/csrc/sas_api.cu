@@ -322,10 +322,10 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
         if (e == cudaSuccess) e = alloc(&h->tile_off, static_cast<size_t>((max_len + 127) / 128 + 2) * 4);
     }
     // head-packed attention tiles: G query heads x 128 / G tokens share one kept
-    // list per token (sparse scope, [B, H, N, d] inputs)
-    if (!varlen && !h->full && h->G >= 2 && 128 % h->G == 0 && (128 / h->G) % 8 == 0 && c.topk > 0) {
+    // list per token (sparse scope; packed sequences: G segments per tile slot)
+    if (!h->full && h->G >= 2 && 128 % h->G == 0 && (128 / h->G) % 8 == 0 && c.topk > 0) {
         h->seg_rows = 128 / h->G;
-        h->nseg = (c.N + h->seg_rows - 1) / h->seg_rows;
+        h->nseg = varlen ? h->T * h->G : (c.N + h->seg_rows - 1) / h->seg_rows;
         h->seg_cap = std::min(h->C, h->seg_rows * c.topk);
         if (e == cudaSuccess)
             e = alloc(&h->seg_union_idx, static_cast<size_t>(BHkv) * h->nseg * std::max(h->seg_cap, 1) * 4);
@@ -546,6 +546,14 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     sa.tiles = h->tiles; sa.ntiles = h->ntiles;
     e = timed_launch(h, 2, s, [&] { return sas::launch_select(sa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
+    if (h->seg_rows > 0) {
+        // the segment unions of the head-packed attention tiles (timed with the selection)
+        e = timed_launch(h, 2, s, [&] {
+            return sas::launch_seg_unions(out_idx, h->BHkv, c.N, h->C, c.topk, h->seg_rows, h->nseg, h->seg_union_idx,
+                                          h->seg_union_cnt, env, h->tiles, h->ntiles);
+        });
+        if (e != cudaSuccess) return cuda_fail(h, e, "segment unions");
+    }
     // a5 over the same tiles
     sas::AttnArgs aa{};
     aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
@@ -557,6 +565,13 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
     aa.sched = h->sched;
+    if (h->seg_rows > 0) {
+        aa.seg_rows = h->seg_rows;
+        aa.nseg = h->nseg;
+        aa.seg_union_idx = h->seg_union_idx;
+        aa.seg_union_cnt = h->seg_union_cnt;
+    }
+    h->last_fwd = h->seg_rows > 0 ? 1 : 0;
     e = timed_launch(h, 3, s, [&] { return sas::launch_attn(aa, env, &err); });
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     return SAS_OK;
@@ -788,12 +803,18 @@ sas_status sas_get_attention_work(sas_handle* h, int64_t* tiles, int64_t* tile_b
     int64_t nt = 0, nb = 0;
     auto ndiag = [](int t, int n) { return (2 * t + 1) * 64 < n ? 2 : 1; };
     if (h->last_fwd == 1) {
-        // head-packed: one tile per (KV group, segment), its union and one diagonal block
+        // head-packed: one tile per (KV group, segment in use), its union and one diagonal block
         std::vector<int32_t> cnt(static_cast<size_t>(h->BHkv) * h->nseg);
         e = cudaMemcpy(cnt.data(), h->seg_union_cnt, cnt.size() * 4, cudaMemcpyDeviceToHost);
+        int used = h->nseg;
+        if (e == cudaSuccess && h->varlen) {
+            e = cudaMemcpy(&used, h->ntiles, 4, cudaMemcpyDeviceToHost);
+            used *= h->G;
+        }
         if (e != cudaSuccess) return cuda_fail(h, e, "segment union counts");
-        for (int32_t u : cnt) nb += u + 1;
-        nt = static_cast<int64_t>(cnt.size());
+        for (int kv = 0; kv < h->BHkv; ++kv)
+            for (int sg = 0; sg < used; ++sg) nb += cnt[static_cast<size_t>(kv) * h->nseg + sg] + 1;
+        nt = static_cast<int64_t>(h->BHkv) * used;
     } else {
         // one tile per (query head, tile slot): its group's union and one or two diagonal blocks
         std::vector<int32_t> cnt(static_cast<size_t>(h->BHkv) * h->T);

@@ -36,6 +36,7 @@ def _run(lens, cap, Hq, Hkv, d, topk, mode, max_len, Q, K, V, S, cu):
 @pytest.mark.parametrize("lens,cap,Hq,Hkv,d,topk,mode", [
     ([700, 1, 64, 129, 0, 300, 255], 1500, 4, 2, 128, 3, TRAIN),   # ragged, empty, one-token, GQA, spare rows
     ([513, 130, 77], 720, 2, 2, 64, 2, INFER),                     # d = 64, inference form, offsets off the block grid
+    ([300, 17, 140, 1], 500, 8, 1, 128, 3, TRAIN),                 # G = 8: head-packed tiles of 16 tokens
 ])
 def test_varlen_matches_oracle(lens, cap, Hq, Hkv, d, topk, mode):
     max_len = max(lens)
