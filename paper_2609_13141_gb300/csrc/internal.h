@@ -19,11 +19,13 @@ int make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64
                       uint32_t box_inner, uint32_t box_rows);
 
 // Raises `func`'s dynamic shared-memory limit to at least `bytes` on the
-// current device, with the largest shared-memory carveout.  The attribute belongs to the device, so it is recorded per
+// current device.  The attribute belongs to the device, so it is recorded per
 // (kernel, device): the first launch on each device sets it, later ones find
 // the record and call nothing (so a launch inside a stream capture that was
 // preceded by one outside it sets nothing).  Thread-safe.
-cudaError_t ensure_smem_attr(const void* func, size_t bytes);
+// max_carveout also asks for the largest shared-memory carveout (L1 shrinks to
+// what is left), for kernels that need it to fit several CTAs on an SM.
+cudaError_t ensure_smem_attr(const void* func, size_t bytes, bool max_carveout = false);
 // Multiprocessor count of the current device (cached per device, thread-safe).
 int device_sm_count();
 
@@ -216,11 +218,16 @@ struct AttnBwdArgs {
     const int4* tiles;
     const int* ntiles;
     const int* tile_off;
+    // head-packed tiles (as in AttnArgs; seg_rows = 0: tiles of one head):
+    // segments of seg_rows tokens x G heads, their unions with row stride seg_cap
+    int seg_rows, nseg, seg_cap;
+    const int32_t* seg_union_idx;
+    const int32_t* seg_union_cnt;
     int N, C, T, BH, topk, mode, d;
     int G;                      // query heads per KV group: K, V, the lists and the gate gradients are per group
     float sm_scale;
 };
-extern const int kBwdMaxTiles;   // query tiles per head the backward supports
+extern const int kBwdMaxTiles;   // query tiles per head the backward supports (head-packed: segments + G)
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total);
 cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err);
 

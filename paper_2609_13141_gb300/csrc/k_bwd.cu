@@ -121,6 +121,12 @@ struct BwdParams {
     const int4* tiles;          // packed sequences: {first row of the sequence, local tile, length, sequence} per slot
     const int* ntiles;          // slots in use (device)
     const int* tile_off;        // first slot of each local tile index
+    // head-packed tiles (the forward's): R tokens x G heads of a KV group per
+    // tile, segments sg = 0 .. nseg - 1 of R tokens per group, their unions
+    // (row stride seg_cap); 0 = tiles of 128 rows of one head
+    int seg_rows, nseg, seg_cap;
+    const int32_t* seg_union_idx;
+    const int32_t* seg_union_cnt;
     int N, C, T, BH, topk, mode;
     int G;                      // query heads per KV group (BH counts query heads)
     float sm_scale, scale_log2;
@@ -144,6 +150,7 @@ __device__ __forceinline__ int bwd_slots_in_use(const int4* tiles, const int* nt
     return tiles == nullptr ? T : __ldg(ntiles);
 }
 
+template <bool HP>
 __global__ void __launch_bounds__(kThreadsB, 1)
 bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
               const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapV, BwdParams p) {
@@ -151,17 +158,23 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     uint8_t* smem = dsm + ((1024u - (smem_u32(dsm) & 1023u)) & 1023u);
     DqCtl& ctl = *reinterpret_cast<DqCtl*>(smem + kDqOffCtl);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int slot = blockIdx.x % p.T, bh = blockIdx.x / p.T;   // (query head, tile slot)
-    if (slot >= bwd_slots_in_use(p.tiles, p.ntiles, p.T)) return;   // an unused slot (packed sequences)
-    const BwdTile tg = bwd_tile(p, slot);
-    const int tile = tg.t;                                       // local tile index
-    const int kv = bh / p.G;                                     // its KV group
-    const long long tb = static_cast<long long>(bh) * p.T + slot;
-    const long long tbk = static_cast<long long>(kv) * p.T + slot;
-    const int32_t* ulist = p.union_idx + tbk * p.C;
-    const int U = __ldg(p.union_cnt + tbk);
+    // per-head tiles: CTA (query head bh, tile slot); head-packed (HP): (KV group, segment)
+    constexpr bool hp = HP;
+    const int nsl = hp ? p.nseg : p.T;
+    const int slot = blockIdx.x % nsl, bh = blockIdx.x / nsl;
+    if (!hp && slot >= bwd_slots_in_use(p.tiles, p.ntiles, p.T)) return;   // an unused slot (packed sequences)
+    const BwdTile tg = hp ? BwdTile{slot, 0, p.N} : bwd_tile(p, slot);
+    const int tile = tg.t;                                       // local tile index (head-packed: segment)
+    const int kv = hp ? bh : bh / p.G;                           // the KV group
+    const int row0 = tg.base + (hp ? slot * p.seg_rows : tile * kRows);   // first token row in the token axis
+    const long long tb = static_cast<long long>(bh) * nsl + slot;   // this tile's offset slots
+    const long long tbk = static_cast<long long>(kv) * nsl + slot;  // its union
+    const int32_t* ulist = hp ? p.seg_union_idx + tbk * p.seg_cap : p.union_idx + tbk * p.C;
+    const int U = __ldg((hp ? p.seg_union_cnt : p.union_cnt) + tbk);
     const int cseq = (tg.n + kKeys - 1) / kKeys;                 // blocks of the sequence
-    const int nb = U + ((2 * tile + 1 < cseq) ? 2 : 1);   // visited blocks: union, then the diagonal ones
+    // visited blocks: the union, then the diagonal one(s)
+    const int diag0 = hp ? (row0 >> 6) : 2 * tile;
+    const int nb = U + (hp ? 1 : ((2 * tile + 1 < cseq) ? 2 : 1));
     if (t == 0) {
         mbar_init(&ctl.q_full, 1);
         for (int s = 0; s < kKvStages; ++s) {
@@ -186,21 +199,30 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     tc_fence_after();
     const uint32_t tmem = ctl.tmem_base;
     const WaitCtl wc{&ctl.abort_flag, p.status, p.limit};
-    const int row0 = tg.base + tile * kRows;   // the tile's first row in the token axis
 
     if (warp == 10) {
         if (lane == 0) {
             // ---- loader: Q and dO once, then K and V of block j into stage
             // j % kKvStages as soon as dQ and dP of block j - kKvStages are done
             mbar_arrive_expect_tx(&ctl.q_full, 2 * kQBytes);
-            for (int h = 0; h < 2; ++h) {
-                tma_load_3d(smem + h * (kRows * 128), &mapQ, &ctl.q_full, h * 64, row0, bh);
-                tma_load_3d(smem + kDqOffDO + h * (kRows * 128), &mapDO, &ctl.q_full, h * 64, row0, bh);
+            if (hp) {
+                // R rows of each of the G heads (the Q / dO maps' box is R rows high)
+                for (int hq = 0; hq < p.G; ++hq)
+                    for (int h = 0; h < 2; ++h) {
+                        const int so = h * (kRows * 128) + hq * p.seg_rows * 128;
+                        tma_load_3d(smem + so, &mapQ, &ctl.q_full, h * 64, row0, bh * p.G + hq);
+                        tma_load_3d(smem + kDqOffDO + so, &mapDO, &ctl.q_full, h * 64, row0, bh * p.G + hq);
+                    }
+            } else {
+                for (int h = 0; h < 2; ++h) {
+                    tma_load_3d(smem + h * (kRows * 128), &mapQ, &ctl.q_full, h * 64, row0, bh);
+                    tma_load_3d(smem + kDqOffDO + h * (kRows * 128), &mapDO, &ctl.q_full, h * 64, row0, bh);
+                }
             }
             for (int j = 0; j < nb; ++j) {
                 const int s = j % kKvStages;
                 if (j >= kKvStages && !mbar_wait(&ctl.kv_empty[s], ((j / kKvStages) - 1) & 1, wc, kSleepNs)) break;
-                const int m = j < U ? __ldg(ulist + j) : 2 * tile + (j - U);
+                const int m = j < U ? __ldg(ulist + j) : diag0 + (j - U);
                 uint8_t* st = smem + kDqOffKV + s * 2 * kKVBytes;
                 mbar_arrive_expect_tx(&ctl.kv_full[s], 2 * kKVBytes);
                 for (int h = 0; h < 2; ++h) {
@@ -297,12 +319,15 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         // ---- rows: thread t takes row t % 128 (its TMEM lane) and keys
         // 32 hk .. 32 hk + 31 of every block, hk = t / 128
         const int r = t & (kRows - 1), hk = t >> 7;
-        const int i = tile * kRows + r;        // row index within the sequence
+        // the row's query head and token (head-packed: row r is head r / R, token r % R of the segment)
+        const int hq = hp ? r / p.seg_rows : 0;
+        const int rt = hp ? r - hq * p.seg_rows : r;
+        const int i = row0 - tg.base + rt;     // row index within the sequence
         const bool valid = i < tg.n;
         const int c = i >> 6;                  // the row's current block
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-        const long long roff = static_cast<long long>(bh) * p.N + row0 + r;
-        const long long kvoff = static_cast<long long>(kv) * p.N + row0 + r;   // the group's kept list
+        const long long roff = static_cast<long long>(hp ? bh * p.G + hq : bh) * p.N + row0 + rt;
+        const long long kvoff = static_cast<long long>(kv) * p.N + row0 + rt;   // the group's kept list
         float delta = 0.f, lse2 = 0.f;
         if (valid) {
             delta = row_delta(p.O + roff * kD, p.dO + roff * kD);
@@ -323,7 +348,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
         const bool train = p.mode == 0;
         bool ok = true;
         for (int j = 0; j < nb; ++j) {
-            const int m = j < U ? __ldg(ulist + j) : 2 * tile + (j - U);
+            const int m = j < U ? __ldg(ulist + j) : diag0 + (j - U);
             float bias = 0.f;
             int lim = -1;
             bool kept = false;
@@ -429,20 +454,26 @@ __device__ __forceinline__ int pair_slot(const int4* tiles, const int* tile_off,
     return g - __ldg(tile_off + tq) + __ldg(tile_off + pr);
 }
 
-// count: for every tile, the key pairs (2p, 2p+1) its union list touches
+// count: for every tile (head-packed: segment), the key pairs (2p, 2p+1) its
+// union list touches; nsrc tiles or segments per group, union rows of ustride
+// A segment's own key pair (the pair of its diagonal block, which it visits as
+// a diagonal item of pass 2) is left out: head-packed segments of block 2p + 1
+// may keep block 2p.  seg_rows = 0: tiles, whose unions stay below their pair.
 __global__ void bwd_inv_count_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cnt, int BH,
-                                     int T, int C, const int4* tiles, const int* ntiles, const int* tile_off) {
+                                     int T, int nsrc, int ustride, const int4* tiles, const int* ntiles,
+                                     const int* tile_off, int seg_rows) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (tb >= static_cast<long long>(BH) * T) return;
-    const int bh = static_cast<int>(tb / T);
-    const int g = static_cast<int>(tb - static_cast<long long>(bh) * T);
-    if (g >= bwd_slots_in_use(tiles, ntiles, T)) return;
-    const int32_t* u = union_idx + tb * C;
+    if (tb >= static_cast<long long>(BH) * nsrc) return;
+    const int bh = static_cast<int>(tb / nsrc);
+    const int g = static_cast<int>(tb - static_cast<long long>(bh) * nsrc);
+    if (g >= bwd_slots_in_use(tiles, ntiles, nsrc)) return;
+    const int32_t* u = union_idx + tb * ustride;
     const int U = union_cnt[tb];
+    const int own = seg_rows > 0 ? ((g * seg_rows) >> 6) >> 1 : -1;
     int last = -1;
     for (int k = 0; k < U; ++k) {
         const int pr = u[k] >> 1;
-        if (pr == last) continue;
+        if (pr == last || pr == own) continue;
         last = pr;
         atomicAdd(cnt + static_cast<long long>(bh) * T + pair_slot(tiles, tile_off, g, pr), 1);
     }
@@ -474,22 +505,23 @@ __global__ void __launch_bounds__(1024) bwd_inv_scan_kernel(const int32_t* cnt, 
     if (t == 1023) off[n] = part[1023];
 }
 
-// fill: entry = the visiting tile's index within its sequence and the positions
-// of the pair's blocks in its list
+// fill: entry = the visiting tile's index within its sequence (head-packed: the
+// segment) and the positions of the pair's blocks in its list
 __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cursor,
-                                    int32_t* tiles, int32_t* pos, int BH, int T, int C, const int4* ttab,
-                                    const int* ntiles, const int* tile_off) {
+                                    int32_t* tiles, int32_t* pos, int BH, int T, int nsrc, int ustride,
+                                    const int4* ttab, const int* ntiles, const int* tile_off, int seg_rows) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (tb >= static_cast<long long>(BH) * T) return;
-    const int bh = static_cast<int>(tb / T);
-    const int tile = static_cast<int>(tb - static_cast<long long>(bh) * T);
-    if (tile >= bwd_slots_in_use(ttab, ntiles, T)) return;
-    const int32_t* u = union_idx + tb * C;
+    if (tb >= static_cast<long long>(BH) * nsrc) return;
+    const int bh = static_cast<int>(tb / nsrc);
+    const int tile = static_cast<int>(tb - static_cast<long long>(bh) * nsrc);
+    if (tile >= bwd_slots_in_use(ttab, ntiles, nsrc)) return;
+    const int32_t* u = union_idx + tb * ustride;
     const int U = union_cnt[tb];
+    const int own = seg_rows > 0 ? ((tile * seg_rows) >> 6) >> 1 : -1;   // as in the count
     int last = -1;
     for (int k = 0; k < U; ++k) {
         const int m = u[k], pr = m >> 1;
-        if (pr == last) continue;
+        if (pr == last || pr == own) continue;
         last = pr;
         // positions (+1) of blocks 2pr and 2pr+1 in this tile's list (ascending)
         const int j0 = m == 2 * pr ? k + 1 : 0;
@@ -500,10 +532,16 @@ __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* uni
     }
 }
 
-// visited blocks per (query head, tile): its group's union list plus one or two diagonal blocks
+// visited blocks per (query head, tile): its group's union list plus one or two
+// diagonal blocks; head-packed (seg_cnt non-null): per (KV group, segment), its
+// union plus its one diagonal block
 __global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH, int T, int N, int G,
-                                 const int4* tiles, const int* ntiles) {
+                                 const int4* tiles, const int* ntiles, const int32_t* seg_cnt, long long nseg_total) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (seg_cnt != nullptr) {
+        if (tb < nseg_total) cnt[tb] = seg_cnt[tb] + 1;
+        return;
+    }
     if (tb >= static_cast<long long>(BH) * T) return;
     const int g = static_cast<int>(tb % T);
     if (g >= bwd_slots_in_use(tiles, ntiles, T)) {
@@ -560,6 +598,7 @@ constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
 // over the first 32 columns of the S^T (dP^T) they have read.
 constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemBuf = 256, kTmemST = 0, kTmemDPT = 64;
 
+template <bool HP>
 __global__ void __launch_bounds__(kThreadsD, 1)
 bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
                const __grid_constant__ CUtensorMap mapK2, const __grid_constant__ CUtensorMap mapV2, BwdParams p) {
@@ -576,12 +615,17 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     const int pr = ptg.t;
     const int cseq = (ptg.n + kKeys - 1) / kKeys;
     const long long pb = static_cast<long long>(kv) * p.T + pslot;
+    constexpr bool hp = HP;   // head-packed tiles
+    // diagonal query tiles first: per-head tiles, tile pr; head-packed, the
+    // segments of tokens 128 pr .. 128 pr + 127 that exist
+    const int ndg = hp ? min(p.G, p.nseg - pr * (kRows / p.seg_rows)) : 1;
     const int off = __ldg(p.inv_off + pb);
-    const int cnt = min(__ldg(p.inv_off + pb + 1) - off, kDkvListCap - 1);
-    const int nq = cnt + 1;                                    // the diagonal tile pr first
-    // work items: every visiting query tile once for each of the group's G query
-    // heads (item k: tile list[k / G] of head kv G + k % G)
-    const int G = p.G;
+    const int cnt = min(__ldg(p.inv_off + pb + 1) - off, kDkvListCap - 1 - ndg);
+    const int nq = cnt + ndg;
+    // work items: per-head tiles, every visiting query tile once for each of the
+    // group's G query heads (item k: tile list[k / G] of head kv G + k % G);
+    // head-packed, every visiting segment once (its 128 rows hold all G heads)
+    const int G = hp ? 1 : p.G;
     const int nitems = nq * G;
     if (t == 0) {
         mbar_init(&ctl.kv_full, 1);
@@ -614,21 +658,42 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     int* raw = list + kDkvListCap;
     int* rawpos = raw + kDkvListCap;
     if (t == 0) {
-        list[0] = 0;
-        raw[0] = pr;
-        const int Upr = __ldg(p.union_cnt + pb);
-        rawpos[0] = (Upr + 1) | ((2 * pr + 1 < cseq ? Upr + 2 : 0) << 16);
+        if (!hp) {
+            list[0] = 0;
+            raw[0] = pr;
+            const int Upr = __ldg(p.union_cnt + pb);
+            rawpos[0] = (Upr + 1) | ((2 * pr + 1 < cseq ? Upr + 2 : 0) << 16);
+        } else {
+            // segment sg of block c visits c right after its union (position U); a
+            // segment of block 2 pr + 1 may also keep block 2 pr (its union's last entry)
+            for (int k = 0; k < ndg; ++k) {
+                const int sg = pr * (kRows / p.seg_rows) + k;
+                const long long sb = static_cast<long long>(kv) * p.nseg + sg;
+                const int Us = __ldg(p.seg_union_cnt + sb);
+                const int cb = (sg * p.seg_rows) >> 6;
+                int pos;
+                if (cb == 2 * pr) {
+                    pos = Us + 1;
+                } else {
+                    const bool has0 = Us > 0 && __ldg(p.seg_union_idx + sb * p.seg_cap + Us - 1) == 2 * pr;
+                    pos = (has0 ? Us : 0) | ((Us + 1) << 16);
+                }
+                list[k] = k;
+                raw[k] = sg;
+                rawpos[k] = pos;
+            }
+        }
     }
     for (int k = t; k < cnt; k += kThreadsD) {
-        raw[1 + k] = __ldg(p.inv_tiles + off + k);
-        rawpos[1 + k] = __ldg(p.inv_pos + off + k);
+        raw[ndg + k] = __ldg(p.inv_tiles + off + k);
+        rawpos[ndg + k] = __ldg(p.inv_pos + off + k);
     }
     __syncthreads();
     for (int k = t; k < cnt; k += kThreadsD) {
-        const int v = raw[1 + k];
+        const int v = raw[ndg + k];
         int rank = 0;
-        for (int q = 0; q < cnt; ++q) rank += raw[1 + q] < v;
-        list[1 + rank] = 1 + k;
+        for (int q = 0; q < cnt; ++q) rank += raw[ndg + q] < v;
+        list[ndg + rank] = ndg + k;
     }
     tc_fence_before();
     __syncthreads();
@@ -649,21 +714,23 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 break;
             float* inf = info + s * 4 * kRows;
             const int q = it / G;
-            const int bhq = kv * G + it % G;   // the item's query head
-            const int tq = raw[list[q]];       // the query tile within the sequence, and its slot
+            const int bhq = kv * G + it % G;   // the item's query head (per-head tiles)
+            const int tq = raw[list[q]];       // the query tile within the sequence (head-packed: segment), and its slot
             const int gq = p.tiles == nullptr ? tq : pslot - __ldg(p.tile_off + pr) + __ldg(p.tile_off + tq);
             const int ps = rawpos[list[q]];
             const int j0 = (ps & 0xffff) - 1, j1 = (ps >> 16) - 1;
-            const long long tbq = static_cast<long long>(bhq) * p.T + gq;
+            const long long tbq = hp ? static_cast<long long>(kv) * p.nseg + tq : static_cast<long long>(bhq) * p.T + gq;
             const long long so = static_cast<long long>(__ldg(p.slot_off + tbq)) * kRows;
-            const long long drow = static_cast<long long>(bhq) * p.N + ptg.base + tq * kRows;
 #pragma unroll
             for (int rr = 0; rr < kRows / kInfoLanes; ++rr) {
                 const int r = il + rr * kInfoLanes;
-                const int i = tq * kRows + r;   // row index within the sequence
+                // the row's head and token within the sequence
+                const int hr = hp ? r / p.seg_rows : 0;
+                const int i = hp ? tq * p.seg_rows + (r - hr * p.seg_rows) : tq * kRows + r;
+                const long long drow = static_cast<long long>(hp ? kv * p.G + hr : bhq) * p.N + ptg.base + i;
                 inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : -CUDART_INF_F;
                 inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : -CUDART_INF_F;
-                inf[2 * kRows + r] = i < ptg.n ? -__ldcg(p.delta + drow + r) : 0.f;
+                inf[2 * kRows + r] = i < ptg.n ? -__ldcg(p.delta + drow) : 0.f;
             }
             mbar_arrive_warp(&ctl.info_full[s]);
         }
@@ -681,13 +748,24 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 const int s = it & 1;
                 if (it >= 2 && !mbar_wait(&ctl.q_empty[s], ((it - 2) >> 1) & 1, wc, kSleepNs)) break;
                 const int tq = raw[list[it / G]];
-                const int row = ptg.base + tq * kRows;
-                const int bhq = kv * G + it % G;
                 uint8_t* st = smem + kDkvOffQ + s * 2 * kQBytes;
                 mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
-                for (int h = 0; h < 2; ++h) {
-                    tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, row, bhq);
-                    tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, row, bhq);
+                if (hp) {
+                    // the segment's R rows of each of the G heads
+                    const int row = tq * p.seg_rows;
+                    for (int hq = 0; hq < p.G; ++hq)
+                        for (int h = 0; h < 2; ++h) {
+                            const int so = h * (kRows * 128) + hq * p.seg_rows * 128;
+                            tma_load_3d(st + so, &mapQ, &ctl.q_full[s], h * 64, row, kv * p.G + hq);
+                            tma_load_3d(st + kQBytes + so, &mapDO, &ctl.q_full[s], h * 64, row, kv * p.G + hq);
+                        }
+                } else {
+                    const int row = ptg.base + tq * kRows;
+                    const int bhq = kv * G + it % G;
+                    for (int h = 0; h < 2; ++h) {
+                        tma_load_3d(st + h * (kRows * 128), &mapQ, &ctl.q_full[s], h * 64, row, bhq);
+                        tma_load_3d(st + kQBytes + h * (kRows * 128), &mapDO, &ctl.q_full[s], h * 64, row, bhq);
+                    }
                 }
             }
         }
@@ -779,9 +857,22 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             tmem_ld32(buf + kTmemDPT + 32, *reinterpret_cast<uint32_t(*)[32]>(dv + 32));
             tmem_wait_ld();
             uint32_t pp[32], dd[32];
-            // In the diagonal tile (the first of the list, items 0 .. G-1) the rows of
-            // half h have block 2pr + h as their own block: keys of that block are causal.
-            const bool causal = q < G && h == kblk;
+            // In a diagonal tile the rows whose own block is this key's block see
+            // only the keys up to themselves.  Per-head tiles (the first item of
+            // the list, items 0 .. G-1): the rows of half h have block 2pr + h, and
+            // column k is token k of it.  Head-packed: all rows of diagonal segment
+            // sg are in block (sg R) / 64, column k is token (sg R) % 64 + k % R.
+            const int qi = q / G;
+            bool causal;
+            int toff0 = 0, rmask = 63;
+            if constexpr (HP) {
+                const int sg = raw[list[qi]];
+                causal = qi < ndg && ((sg * p.seg_rows) >> 6) == 2 * pr + kblk;
+                toff0 = (sg * p.seg_rows) & 63;
+                rmask = p.seg_rows - 1;
+            } else {
+                causal = qi == 0 && h == kblk;
+            }
             const float2* off2 = reinterpret_cast<const float2*>(inf + kblk * kRows + h * 64);
             const float2* nd2p = reinterpret_cast<const float2*>(inf + 2 * kRows + h * 64);
             const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2);
@@ -794,8 +885,8 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                             z0, z1);
                 float p0 = fast_exp2(z0), p1 = fast_exp2(z1);
                 if (causal) {
-                    p0 = kin <= k ? p0 : 0.f;
-                    p1 = kin <= k + 1 ? p1 : 0.f;
+                    p0 = kin <= toff0 + (k & rmask) ? p0 : 0.f;
+                    p1 = kin <= toff0 + ((k + 1) & rmask) ? p1 : 0.f;
                 }
                 const uint64_t d2 = add_f32x2(f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1])), f32x2(nd.x, nd.y));
                 float a0, a1;
@@ -954,9 +1045,11 @@ const int kBwdMaxTiles = kDkvListCap - 1;
 // Slots of the per-tile visited-block offsets pass 1 writes for pass 2: one per
 // visited block of every tile; returns their total in *total (synchronises).
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total) {
-    const long long tiles = static_cast<long long>(a.BH) * a.T;
+    // offset slots per (query head, tile), head-packed per (KV group, segment)
+    const long long tiles = a.seg_rows > 0 ? static_cast<long long>(a.BH / a.G) * a.nseg : static_cast<long long>(a.BH) * a.T;
     const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
-    bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.N, a.G, a.tiles, a.ntiles);
+    bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.N, a.G, a.tiles, a.ntiles,
+                                                 a.seg_rows > 0 ? a.seg_union_cnt : nullptr, tiles);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.slot_off, nullptr, tiles);
     if (total == nullptr) return cudaGetLastError();   // the caller's buffer holds the upper bound
     int32_t host = 0;
@@ -976,15 +1069,24 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         *err = "backward: query heads must fill whole KV groups";
         return cudaErrorInvalidValue;
     }
+    if (a.seg_rows > 0 && (G < 2 || a.seg_rows * G != kRows || a.seg_rows % 8 != 0 || a.tiles != nullptr ||
+                           a.seg_union_idx == nullptr || a.seg_union_cnt == nullptr ||
+                           a.nseg + G > kDkvListCap - 1)) {
+        *err = "backward: head-packed tiles need 128 = G x seg_rows, [B, H, N, d] inputs and segment unions";
+        return cudaErrorInvalidValue;
+    }
     const int BHkv = a.BH / G;   // KV groups x batch
     {
-        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel), kDqSmem);
-        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel), kDkvSmem);
+        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel<false>), kDqSmem);
+        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel<false>), kDkvSmem);
+        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel<true>), kDqSmem);
+        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel<true>), kDkvSmem);
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(bwd)"; return e; }
     }
     CUtensorMap mq, mdo, mk, mv, mk2, mv2;
-    if (make_tmap_bf16_3d(&mq, a.Q, kD, a.N, a.BH, 64, kRows) != 0 ||
-        make_tmap_bf16_3d(&mdo, a.dO, kD, a.N, a.BH, 64, kRows) != 0 ||
+    const bool hp = a.seg_rows > 0;   // head-packed tiles: the Q / dO boxes are one head's seg_rows rows
+    if (make_tmap_bf16_3d(&mq, a.Q, kD, a.N, a.BH, 64, hp ? a.seg_rows : kRows) != 0 ||
+        make_tmap_bf16_3d(&mdo, a.dO, kD, a.N, a.BH, 64, hp ? a.seg_rows : kRows) != 0 ||
         make_tmap_bf16_3d(&mk, a.K, kD, a.N, BHkv, 64, kKeys) != 0 ||
         make_tmap_bf16_3d(&mv, a.V, kD, a.N, BHkv, 64, kKeys) != 0 ||
         make_tmap_bf16_3d(&mk2, a.K, kD, a.N, BHkv, 64, 2 * kKeys) != 0 ||
@@ -1013,35 +1115,48 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     p.tiles = a.tiles;
     p.ntiles = a.ntiles;
     p.tile_off = a.tile_off;
+    p.seg_rows = a.seg_rows;
+    p.nseg = a.nseg;
+    p.seg_cap = a.seg_cap;
+    p.seg_union_idx = a.seg_union_idx;
+    p.seg_union_cnt = a.seg_union_cnt;
     p.N = a.N; p.C = a.C; p.T = a.T; p.BH = a.BH; p.topk = a.topk; p.mode = a.mode;
     p.G = G;
     p.sm_scale = a.sm_scale;
     p.scale_log2 = a.sm_scale * kLog2eB;
     p.status = env.status;
     p.limit = env.limit;
-    const long long tiles = static_cast<long long>(a.BH) * a.T;        // (query head, tile)
-    const long long gtiles = static_cast<long long>(BHkv) * a.T;       // (KV group, tile or key pair)
+    // pass 1 tiles: (query head, tile), head-packed (KV group, segment)
+    const long long tiles = hp ? static_cast<long long>(BHkv) * a.nseg : static_cast<long long>(a.BH) * a.T;
+    const long long gtiles = static_cast<long long>(BHkv) * a.T;       // (KV group, key pair)
+    const int nsrc = hp ? a.nseg : a.T;                                 // union lists per group
+    const long long srcs = static_cast<long long>(BHkv) * nsrc;
     if (tiles > 0x7fffffffLL) { *err = "backward: too many tiles"; return cudaErrorInvalidValue; }
     // pass 1 (also writes Delta for pass 2); both halves of a row add into dlogg
     const long long per_head = static_cast<long long>(a.N) * (a.topk > 0 ? a.topk : 1);
     cudaError_t e0 = cudaMemsetAsync(p.dlogg, 0, static_cast<size_t>(a.BH) * per_head * 4, env.stream);
     if (e0 != cudaSuccess) { *err = "backward dlogg"; return e0; }
-    bwd_dq_kernel<<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+    if (hp) bwd_dq_kernel<true><<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+    else bwd_dq_kernel<false><<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
     // inverted lists of the KV groups' union lists
     e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(gtiles) * 4, env.stream);
     if (e != cudaSuccess) { *err = "backward list counts"; return e; }
-    const unsigned gb = static_cast<unsigned>((gtiles + 255) / 256);
-    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cnt, BHkv, a.T, a.C, a.tiles,
-                                                      a.ntiles, a.tile_off);
+    const unsigned gb = static_cast<unsigned>((srcs + 255) / 256);
+    const int32_t* uidx = hp ? a.seg_union_idx : a.union_idx;
+    const int32_t* ucnt = hp ? a.seg_union_cnt : a.union_cnt;
+    const int ustride = hp ? a.seg_cap : a.C;
+    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cnt, BHkv, a.T, nsrc, ustride, a.tiles,
+                                                      a.ntiles, a.tile_off, hp ? a.seg_rows : 0);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, gtiles);
-    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(a.union_idx, a.union_cnt, a.inv_cursor, a.inv_tiles, a.inv_pos,
-                                                     BHkv, a.T, a.C, a.tiles, a.ntiles, a.tile_off);
+    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cursor, a.inv_tiles, a.inv_pos, BHkv, a.T,
+                                                     nsrc, ustride, a.tiles, a.ntiles, a.tile_off, hp ? a.seg_rows : 0);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
     // pass 2: one CTA per (KV group, key pair)
-    bwd_dkv_kernel<<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+    if (hp) bwd_dkv_kernel<true><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+    else bwd_dkv_kernel<false><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     if (G > 1 && a.topk > 0) {

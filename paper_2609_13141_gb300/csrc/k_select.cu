@@ -451,7 +451,7 @@ __host__ __device__ constexpr size_t bitmap_bytes(int C) { return size_t((C + 31
 
 // ------------------------------------------------------------ scores given
 
-template <bool REG>
+template <bool REG, bool NOISE>
 __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ float stage[4][32][33];
@@ -492,20 +492,26 @@ __global__ void __launch_bounds__(128, 3) select_given_kernel(SelParams p) {
     const int last = min(row0 + 31, geo.n - 1);
     const int Cw = row0 < geo.n ? (last >> 6) : 0;   // largest C_i among the warp's rows
     const float* sbase = p.scores + (static_cast<long long>(bh) * p.N + geo.base) * p.C;
-    const float* nbase = p.noise == nullptr ? nullptr : p.noise + (static_cast<long long>(bh) * p.N + geo.base) * p.C;
+    const float* nbase = NOISE ? p.noise + (static_cast<long long>(bh) * p.N + geo.base) * p.C : nullptr;
     for (int c = 0; 32 * c < Cw; ++c) {
         const int m = 32 * c + lane;
-#pragma unroll 4
+        // block m of the warp's 32 rows: all loads issued before the first is used
+        float w[32];
+#pragma unroll
         for (int rho = 0; rho < 32; ++rho) {
             const int row = row0 + rho;
-            float v = 0.f;
-            if (row < geo.n && m < p.C) {
-                const long long o = static_cast<long long>(row) * p.C + m;
-                v = __ldg(sbase + o);
-                if (nbase != nullptr) v = __fadd_rn(v, __ldg(nbase + o));   // full*: s~ = s + eps in fp32
-            }
-            stage[warp][lane][rho] = v;
+            w[rho] = (row < geo.n && m < p.C) ? __ldg(sbase + static_cast<long long>(row) * p.C + m) : 0.f;
         }
+        if constexpr (NOISE) {
+#pragma unroll
+            for (int rho = 0; rho < 32; ++rho) {
+                const int row = row0 + rho;
+                if (row < geo.n && m < p.C)   // full*: s~ = s + eps in fp32
+                    w[rho] = __fadd_rn(w[rho], __ldg(nbase + static_cast<long long>(row) * p.C + m));
+            }
+        }
+#pragma unroll
+        for (int rho = 0; rho < 32; ++rho) stage[warp][lane][rho] = w[rho];
         __syncwarp();
         float v[32];
 #pragma unroll
@@ -1293,7 +1299,7 @@ template <int D, int DS, bool BIGK>
 cudaError_t launch_proj_k(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
     const size_t smem = 1024 + proj_smem_bytes<D, DS, BIGK>(a.C);
     if (smem > 227 * 1024) { *err = "selection: too many blocks for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS, BIGK>), smem);
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_proj_kernel<D, DS, BIGK>), smem, true);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select)"; return e; }
     CUtensorMap mq, mw, mk;
     // Q of all query heads; Wq [H][DS][G D] (a group's gate-query projection)
@@ -1316,14 +1322,14 @@ cudaError_t launch_proj(const SelectArgs& a, const SelParams& p, const KernelEnv
     return cudaErrorInvalidValue;
 }
 
-template <bool REG>
+template <bool REG, bool NOISE>
 cudaError_t launch_given(const SelectArgs& a, const SelParams& p, const KernelEnv& env, const char** err) {
     const size_t smem = smem_topk_bytes(a.topk) + staging_bytes(a.topk) + bitmap_bytes(a.C);
     if (smem > 200 * 1024) { *err = "selection: top-K too large for shared memory"; return cudaErrorInvalidValue; }
-    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_given_kernel<REG>), smem);
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_given_kernel<REG, NOISE>), smem);
     if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(select_given)"; return e; }
     const dim3 grid(a.BH * a.T);
-    select_given_kernel<REG><<<grid, 128, smem, env.stream>>>(p);
+    select_given_kernel<REG, NOISE><<<grid, 128, smem, env.stream>>>(p);
     e = cudaGetLastError();
     if (e != cudaSuccess) *err = "select launch";
     return e;
@@ -1517,7 +1523,11 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     }
 
     const bool reg = a.topk <= 32;
-    if (a.scores != nullptr) return reg ? launch_given<true>(a, p, env, err) : launch_given<false>(a, p, env, err);
+    if (a.scores != nullptr) {
+        if (a.noise != nullptr)
+            return reg ? launch_given<true, true>(a, p, env, err) : launch_given<false, true>(a, p, env, err);
+        return reg ? launch_given<true, false>(a, p, env, err) : launch_given<false, false>(a, p, env, err);
+    }
     if (a.d == 128 && a.d_sel == 128) return launch_proj<128, 128>(a, p, env, err);
     if (a.d == 128 && a.d_sel == 64) return launch_proj<128, 64>(a, p, env, err);
     if (a.d == 64 && a.d_sel == 64) return launch_proj<64, 64>(a, p, env, err);

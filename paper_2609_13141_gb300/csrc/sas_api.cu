@@ -56,7 +56,7 @@ std::map<std::pair<const void*, int>, size_t> g_smem_attr;   // (kernel, device)
 std::map<int, int> g_sms;                                     // device -> SM count
 }  // namespace
 
-cudaError_t ensure_smem_attr(const void* func, size_t bytes) {
+cudaError_t ensure_smem_attr(const void* func, size_t bytes, bool max_carveout) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -64,8 +64,7 @@ cudaError_t ensure_smem_attr(const void* func, size_t bytes) {
     size_t& set = g_smem_attr[{func, dev}];
     if (bytes <= set) return cudaSuccess;
     e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
-    // the largest shared-memory carveout, so that several CTAs of such a kernel fit an SM
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && max_carveout)
         e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e == cudaSuccess) set = bytes;
     return e;
@@ -711,6 +710,13 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         a.tiles = h->tiles;
         a.ntiles = h->ntiles;
         a.tile_off = h->tile_off;
+    } else if (h->seg_rows > 0 && h->last_fwd == 1 && h->nseg + h->G <= sas::kBwdMaxTiles) {
+        // head-packed tiles over the forward's segment unions
+        a.seg_rows = h->seg_rows;
+        a.nseg = h->nseg;
+        a.seg_cap = h->seg_cap;
+        a.seg_union_idx = h->seg_union_idx;
+        a.seg_union_cnt = h->seg_union_cnt;
     }
     const sas::KernelEnv env{s, h->status, h->limit};
     const char* err = "";
