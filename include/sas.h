@@ -198,7 +198,12 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
  * it after the sas_attention_fwd of the same inputs on this handle, with no
  * other forward in between.  With grouped-query attention (Hkv < H) a
  * group's K, V, kept sets and gates serve its H / Hkv query heads, so dK, dV
- * and the gate gradients are sums over those heads (Sec. 3.3).
+ * and the gate gradients are sums over those heads (Sec. 3.3).  After a
+ * forward on head-packed tiles (see sas_get_attention_work) the backward runs
+ * on the same tiles, batched or packed, when a sequence holds at most
+ * 2047 - G of them (G (N + 127) / 128 with N the longest sequence); else on
+ * tiles of one query head.  The gradients are the same either way, up to the
+ * order of floating-point sums.
  *
  * Packed sequences (a handle created with max_seqs > 0): the backward of the
  * last sas_attention_fwd_varlen on the handle, whose tile table it reads;

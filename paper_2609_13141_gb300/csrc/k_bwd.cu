@@ -123,7 +123,10 @@ struct BwdParams {
     const int* tile_off;        // first slot of each local tile index
     // head-packed tiles (the forward's): R tokens x G heads of a KV group per
     // tile, segments sg = 0 .. nseg - 1 of R tokens per group, their unions
-    // (row stride seg_cap); 0 = tiles of 128 rows of one head
+    // (row stride seg_cap); 0 = tiles of 128 rows of one head.  Packed
+    // sequences: segment slot sg is sub-segment sg % G of tile slot sg / G
+    // (nseg = G T); a segment's index within its sequence is G t + sg % G for
+    // the slot's local tile t
     int seg_rows, nseg, seg_cap;
     const int32_t* seg_union_idx;
     const int32_t* seg_union_cnt;
@@ -149,6 +152,17 @@ __device__ __forceinline__ BwdTile bwd_tile(const BwdParams& p, int slot) {
 __device__ __forceinline__ int bwd_slots_in_use(const int4* tiles, const int* ntiles, int T) {
     return tiles == nullptr ? T : __ldg(ntiles);
 }
+// Head-packed segment slot sg: t = the segment's index within its sequence
+// (rows R t .. R t + R - 1 of it), the sequence's first row and length; t = -1
+// for a slot past the tiles in use or a segment past its sequence's end.
+__device__ __forceinline__ BwdTile bwd_seg(const BwdParams& p, int sg) {
+    if (p.tiles == nullptr) return {sg, 0, p.N};
+    const int ts = sg / p.G;
+    if (ts >= __ldg(p.ntiles)) return {-1, 0, 0};
+    const int4 v = __ldg(p.tiles + ts);
+    const int t = v.y * p.G + (sg - ts * p.G);
+    return {t * p.seg_rows < v.z ? t : -1, v.x, v.z};
+}
 
 template <bool HP>
 __global__ void __launch_bounds__(kThreadsB, 1)
@@ -163,17 +177,18 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
     const int nsl = hp ? p.nseg : p.T;
     const int slot = blockIdx.x % nsl, bh = blockIdx.x / nsl;
     if (!hp && slot >= bwd_slots_in_use(p.tiles, p.ntiles, p.T)) return;   // an unused slot (packed sequences)
-    const BwdTile tg = hp ? BwdTile{slot, 0, p.N} : bwd_tile(p, slot);
+    const BwdTile tg = hp ? bwd_seg(p, slot) : bwd_tile(p, slot);
+    if (hp && tg.t < 0) return;                                  // no rows (packed sequences)
     const int tile = tg.t;                                       // local tile index (head-packed: segment)
     const int kv = hp ? bh : bh / p.G;                           // the KV group
-    const int row0 = tg.base + (hp ? slot * p.seg_rows : tile * kRows);   // first token row in the token axis
+    const int row0 = tg.base + tile * (hp ? p.seg_rows : kRows);   // first token row in the token axis
     const long long tb = static_cast<long long>(bh) * nsl + slot;   // this tile's offset slots
     const long long tbk = static_cast<long long>(kv) * nsl + slot;  // its union
     const int32_t* ulist = hp ? p.seg_union_idx + tbk * p.seg_cap : p.union_idx + tbk * p.C;
     const int U = __ldg((hp ? p.seg_union_cnt : p.union_cnt) + tbk);
     const int cseq = (tg.n + kKeys - 1) / kKeys;                 // blocks of the sequence
     // visited blocks: the union, then the diagonal one(s)
-    const int diag0 = hp ? (row0 >> 6) : 2 * tile;
+    const int diag0 = hp ? (tile * p.seg_rows) >> 6 : 2 * tile;
     const int nb = U + (hp ? 1 : ((2 * tile + 1 < cseq) ? 2 : 1));
     if (t == 0) {
         mbar_init(&ctl.q_full, 1);
@@ -454,28 +469,43 @@ __device__ __forceinline__ int pair_slot(const int4* tiles, const int* tile_off,
     return g - __ldg(tile_off + tq) + __ldg(tile_off + pr);
 }
 
+// A source of the inverted lists: a tile slot g, or (head-packed, hg = G) a
+// segment slot g.  ts = its tile slot, entry = its index within the sequence
+// (tile or segment), own = the key pair of its diagonal block when that pair
+// visits it as a diagonal item (head-packed: segments of block 2p + 1 may keep
+// block 2p), else -1; ts = -1 for an unused slot.
+struct InvSrc {
+    int ts, entry, own;
+};
+__device__ __forceinline__ InvSrc inv_src(int g, int hg, const int4* tiles, const int* ntiles) {
+    const int ts = hg > 0 ? g / hg : g;
+    // every source of a [B, H, N, d] batch is live (its last tile may hold fewer than G segments)
+    if (tiles != nullptr && ts >= __ldg(ntiles)) return {-1, 0, -1};
+    const int tq = tiles == nullptr ? ts : __ldg(tiles + ts).y;   // local tile
+    if (hg == 0) return {ts, tq, -1};
+    return {ts, tq * hg + (g - ts * hg), tq};
+}
+
 // count: for every tile (head-packed: segment), the key pairs (2p, 2p+1) its
-// union list touches; nsrc tiles or segments per group, union rows of ustride
-// A segment's own key pair (the pair of its diagonal block, which it visits as
-// a diagonal item of pass 2) is left out: head-packed segments of block 2p + 1
-// may keep block 2p.  seg_rows = 0: tiles, whose unions stay below their pair.
+// union list touches, but its own pair; nsrc tiles or segments per group,
+// union rows of ustride; hg = G for head-packed segments, else 0
 __global__ void bwd_inv_count_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cnt, int BH,
                                      int T, int nsrc, int ustride, const int4* tiles, const int* ntiles,
-                                     const int* tile_off, int seg_rows) {
+                                     const int* tile_off, int hg) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * nsrc) return;
     const int bh = static_cast<int>(tb / nsrc);
     const int g = static_cast<int>(tb - static_cast<long long>(bh) * nsrc);
-    if (g >= bwd_slots_in_use(tiles, ntiles, nsrc)) return;
+    const InvSrc src = inv_src(g, hg, tiles, ntiles);
+    if (src.ts < 0) return;
     const int32_t* u = union_idx + tb * ustride;
     const int U = union_cnt[tb];
-    const int own = seg_rows > 0 ? ((g * seg_rows) >> 6) >> 1 : -1;
     int last = -1;
     for (int k = 0; k < U; ++k) {
         const int pr = u[k] >> 1;
-        if (pr == last || pr == own) continue;
+        if (pr == last || pr == src.own) continue;
         last = pr;
-        atomicAdd(cnt + static_cast<long long>(bh) * T + pair_slot(tiles, tile_off, g, pr), 1);
+        atomicAdd(cnt + static_cast<long long>(bh) * T + pair_slot(tiles, tile_off, src.ts, pr), 1);
     }
 }
 
@@ -506,40 +536,52 @@ __global__ void __launch_bounds__(1024) bwd_inv_scan_kernel(const int32_t* cnt, 
 }
 
 // fill: entry = the visiting tile's index within its sequence (head-packed: the
-// segment) and the positions of the pair's blocks in its list
+// segment's) and the positions of the pair's blocks in its list
 __global__ void bwd_inv_fill_kernel(const int32_t* union_idx, const int32_t* union_cnt, int32_t* cursor,
                                     int32_t* tiles, int32_t* pos, int BH, int T, int nsrc, int ustride,
-                                    const int4* ttab, const int* ntiles, const int* tile_off, int seg_rows) {
+                                    const int4* ttab, const int* ntiles, const int* tile_off, int hg) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (tb >= static_cast<long long>(BH) * nsrc) return;
     const int bh = static_cast<int>(tb / nsrc);
-    const int tile = static_cast<int>(tb - static_cast<long long>(bh) * nsrc);
-    if (tile >= bwd_slots_in_use(ttab, ntiles, nsrc)) return;
+    const int g = static_cast<int>(tb - static_cast<long long>(bh) * nsrc);
+    const InvSrc src = inv_src(g, hg, ttab, ntiles);
+    if (src.ts < 0) return;
     const int32_t* u = union_idx + tb * ustride;
     const int U = union_cnt[tb];
-    const int own = seg_rows > 0 ? ((tile * seg_rows) >> 6) >> 1 : -1;   // as in the count
     int last = -1;
     for (int k = 0; k < U; ++k) {
         const int m = u[k], pr = m >> 1;
-        if (pr == last || pr == own) continue;
+        if (pr == last || pr == src.own) continue;
         last = pr;
         // positions (+1) of blocks 2pr and 2pr+1 in this tile's list (ascending)
         const int j0 = m == 2 * pr ? k + 1 : 0;
         const int j1 = m == 2 * pr + 1 ? k + 1 : (k + 1 < U && u[k + 1] == 2 * pr + 1 ? k + 2 : 0);
-        const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pair_slot(ttab, tile_off, tile, pr), 1);
-        tiles[slot] = ttab == nullptr ? tile : __ldg(ttab + tile).y;
+        const int slot = atomicAdd(cursor + static_cast<long long>(bh) * T + pair_slot(ttab, tile_off, src.ts, pr), 1);
+        tiles[slot] = src.entry;
         pos[slot] = j0 | (j1 << 16);
     }
 }
 
 // visited blocks per (query head, tile): its group's union list plus one or two
-// diagonal blocks; head-packed (seg_cnt non-null): per (KV group, segment), its
-// union plus its one diagonal block
+// diagonal blocks; head-packed (seg_cnt non-null): per (KV group, segment slot),
+// its union plus its one diagonal block (none for an unused slot or a segment
+// past its sequence's end: seg_R rows per segment)
 __global__ void bwd_slots_kernel(const int32_t* union_cnt, int32_t* cnt, int BH, int T, int N, int G,
-                                 const int4* tiles, const int* ntiles, const int32_t* seg_cnt, long long nseg_total) {
+                                 const int4* tiles, const int* ntiles, const int32_t* seg_cnt, long long nseg_total,
+                                 int nseg, int seg_R) {
     const long long tb = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (seg_cnt != nullptr) {
-        if (tb < nseg_total) cnt[tb] = seg_cnt[tb] + 1;
+        if (tb >= nseg_total) return;
+        bool live = true;
+        if (tiles != nullptr) {
+            const int sg = static_cast<int>(tb % nseg), ts = sg / G;
+            live = ts < __ldg(ntiles);
+            if (live) {
+                const int4 v = __ldg(tiles + ts);
+                live = (v.y * G + (sg - ts * G)) * seg_R < v.z;
+            }
+        }
+        cnt[tb] = live ? seg_cnt[tb] + 1 : 0;
         return;
     }
     if (tb >= static_cast<long long>(BH) * T) return;
@@ -618,7 +660,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     constexpr bool hp = HP;   // head-packed tiles
     // diagonal query tiles first: per-head tiles, tile pr; head-packed, the
     // segments of tokens 128 pr .. 128 pr + 127 that exist
-    const int ndg = hp ? min(p.G, p.nseg - pr * (kRows / p.seg_rows)) : 1;
+    const int ndg = hp ? min(p.G, (ptg.n - pr * kRows + p.seg_rows - 1) / p.seg_rows) : 1;
     const int off = __ldg(p.inv_off + pb);
     const int cnt = min(__ldg(p.inv_off + pb + 1) - off, kDkvListCap - 1 - ndg);
     const int nq = cnt + ndg;
@@ -667,8 +709,8 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             // segment sg of block c visits c right after its union (position U); a
             // segment of block 2 pr + 1 may also keep block 2 pr (its union's last entry)
             for (int k = 0; k < ndg; ++k) {
-                const int sg = pr * (kRows / p.seg_rows) + k;
-                const long long sb = static_cast<long long>(kv) * p.nseg + sg;
+                const int sg = pr * p.G + k;   // within the sequence; its slot: pslot G + k (packed)
+                const long long sb = static_cast<long long>(kv) * p.nseg + (p.tiles == nullptr ? sg : pslot * p.G + k);
                 const int Us = __ldg(p.seg_union_cnt + sb);
                 const int cb = (sg * p.seg_rows) >> 6;
                 int pos;
@@ -716,10 +758,15 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             const int q = it / G;
             const int bhq = kv * G + it % G;   // the item's query head (per-head tiles)
             const int tq = raw[list[q]];       // the query tile within the sequence (head-packed: segment), and its slot
-            const int gq = p.tiles == nullptr ? tq : pslot - __ldg(p.tile_off + pr) + __ldg(p.tile_off + tq);
+            int gq = tq;
+            if (p.tiles != nullptr) {
+                const int tt = hp ? tq / p.G : tq;   // the local tile
+                gq = pslot - __ldg(p.tile_off + pr) + __ldg(p.tile_off + tt);
+                if (hp) gq = gq * p.G + (tq - tt * p.G);
+            }
             const int ps = rawpos[list[q]];
             const int j0 = (ps & 0xffff) - 1, j1 = (ps >> 16) - 1;
-            const long long tbq = hp ? static_cast<long long>(kv) * p.nseg + tq : static_cast<long long>(bhq) * p.T + gq;
+            const long long tbq = hp ? static_cast<long long>(kv) * p.nseg + gq : static_cast<long long>(bhq) * p.T + gq;
             const long long so = static_cast<long long>(__ldg(p.slot_off + tbq)) * kRows;
 #pragma unroll
             for (int rr = 0; rr < kRows / kInfoLanes; ++rr) {
@@ -752,7 +799,7 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 mbar_arrive_expect_tx(&ctl.q_full[s], 2 * kQBytes);
                 if (hp) {
                     // the segment's R rows of each of the G heads
-                    const int row = tq * p.seg_rows;
+                    const int row = ptg.base + tq * p.seg_rows;
                     for (int hq = 0; hq < p.G; ++hq)
                         for (int h = 0; h < 2; ++h) {
                             const int so = h * (kRows * 128) + hq * p.seg_rows * 128;
@@ -1049,7 +1096,7 @@ cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long lo
     const long long tiles = a.seg_rows > 0 ? static_cast<long long>(a.BH / a.G) * a.nseg : static_cast<long long>(a.BH) * a.T;
     const unsigned gb = static_cast<unsigned>((tiles + 255) / 256);
     bwd_slots_kernel<<<gb, 256, 0, env.stream>>>(a.union_cnt, a.inv_cnt, a.BH, a.T, a.N, a.G, a.tiles, a.ntiles,
-                                                 a.seg_rows > 0 ? a.seg_union_cnt : nullptr, tiles);
+                                                 a.seg_rows > 0 ? a.seg_union_cnt : nullptr, tiles, a.nseg, a.seg_rows);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.slot_off, nullptr, tiles);
     if (total == nullptr) return cudaGetLastError();   // the caller's buffer holds the upper bound
     int32_t host = 0;
@@ -1069,10 +1116,12 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         *err = "backward: query heads must fill whole KV groups";
         return cudaErrorInvalidValue;
     }
-    if (a.seg_rows > 0 && (G < 2 || a.seg_rows * G != kRows || a.seg_rows % 8 != 0 || a.tiles != nullptr ||
+    // segments of one sequence: a key pair's inverted list holds at most that many, plus its diagonal ones
+    const long long seq_segs = a.tiles != nullptr ? static_cast<long long>(G) * ((a.C + 1) / 2) : a.nseg;
+    if (a.seg_rows > 0 && (G < 2 || a.seg_rows * G != kRows || a.seg_rows % 8 != 0 ||
                            a.seg_union_idx == nullptr || a.seg_union_cnt == nullptr ||
-                           a.nseg + G > kDkvListCap - 1)) {
-        *err = "backward: head-packed tiles need 128 = G x seg_rows, [B, H, N, d] inputs and segment unions";
+                           (a.tiles != nullptr && a.nseg != G * a.T) || seq_segs + G > kDkvListCap - 1)) {
+        *err = "backward: head-packed tiles need 128 = G x seg_rows, segment unions and short enough sequences";
         return cudaErrorInvalidValue;
     }
     const int BHkv = a.BH / G;   // KV groups x batch
@@ -1148,10 +1197,10 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     const int32_t* ucnt = hp ? a.seg_union_cnt : a.union_cnt;
     const int ustride = hp ? a.seg_cap : a.C;
     bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cnt, BHkv, a.T, nsrc, ustride, a.tiles,
-                                                      a.ntiles, a.tile_off, hp ? a.seg_rows : 0);
+                                                      a.ntiles, a.tile_off, hp ? G : 0);
     bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, gtiles);
     bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cursor, a.inv_tiles, a.inv_pos, BHkv, a.T,
-                                                     nsrc, ustride, a.tiles, a.ntiles, a.tile_off, hp ? a.seg_rows : 0);
+                                                     nsrc, ustride, a.tiles, a.ntiles, a.tile_off, hp ? G : 0);
     e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
     // pass 2: one CTA per (KV group, key pair)

@@ -710,7 +710,10 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         a.tiles = h->tiles;
         a.ntiles = h->ntiles;
         a.tile_off = h->tile_off;
-    } else if (h->seg_rows > 0 && h->last_fwd == 1 && h->nseg + h->G <= sas::kBwdMaxTiles) {
+    }
+    // segments of one sequence, each a possible entry of a key pair's inverted list
+    const long long seq_segs = h->varlen ? static_cast<long long>(h->G) * tseq : h->nseg;
+    if (h->seg_rows > 0 && h->last_fwd == 1 && seq_segs + h->G <= sas::kBwdMaxTiles) {
         // head-packed tiles over the forward's segment unions
         a.seg_rows = h->seg_rows;
         a.nseg = h->nseg;

@@ -89,6 +89,7 @@ def _untouched_past_end(g, end):
     ([700, 1, 64, 129, 0, 300, 255], 1500, 4, 2, 3, TRAIN),   # ragged, empty, one-token, GQA, spare rows
     ([513, 130, 77], 720, 2, 2, 2, TRAIN),                     # offsets off the block grid
     ([400, 250], 700, 2, 1, 2, INFER),                         # MQA, inference form: no gate gradient
+    ([300, 129, 64, 1, 190], 700, 8, 1, 3, TRAIN),             # G = 8: head-packed tiles of 16 tokens, empty ones
 ])
 def test_packed_backward_matches_oracle(lens, cap, Hq, Hkv, topk, mode):
     max_len = max(lens)
@@ -102,16 +103,17 @@ def test_packed_backward_matches_oracle(lens, cap, Hq, Hkv, topk, mode):
         assert float(g["ds"].abs().max()) == 0.0
 
 
-def test_packed_backward_equal_lengths_bit_identical_to_batched():
+@pytest.mark.parametrize("H,Hkv", [(4, 4), (8, 2)])   # per-head tiles; head-packed tiles of 32 tokens x 4 heads
+def test_packed_backward_equal_lengths_bit_identical_to_batched(H, Hkv):
     # Same data as a [B = 3, H, n, d] batch: pass 1 runs the same tiles, and pass
     # 2 sums a key pair's query tiles in the same order (by index within the
     # sequence), so every gradient is bit-identical.
-    S_, n, H, topk = 3, 700, 4, 4
-    Q, K, V, S, dO, cu = _packed([n] * S_, S_ * n, H, H, n, seed=9)
-    g = _run([n] * S_, S_ * n, H, H, topk, TRAIN, n, Q, K, V, S, dO, cu)
+    S_, n, topk = 3, 700, 4
+    Q, K, V, S, dO, cu = _packed([n] * S_, S_ * n, H, Hkv, n, seed=9)
+    g = _run([n] * S_, S_ * n, H, Hkv, topk, TRAIN, n, Q, K, V, S, dO, cu)
     assert g["status"] == 0
     bat = lambda x: x.reshape(x.shape[0], S_, n, -1).transpose(0, 1).contiguous().to(DEV)
-    layer = sas.SasLayer(S_, H, n, 128, topk)
+    layer = sas.SasLayer(S_, H, n, 128, topk, Hkv=Hkv)
     Qb, Kb, Vb, Sb, dOb = bat(Q), bat(K), bat(V), bat(S), bat(dO)
     O, LSE, si, sl = layer.attention(Qb, Kb, Vb, scores=Sb)
     out = layer.attention_bwd(Qb, Kb, Vb, O, LSE, dOb, scores=Sb, sel_idx=si, sel_logg=sl, want_ds=True)
