@@ -27,8 +27,24 @@ treats it as fixed, as the kernels do.
 
 GQA (sas_attention_bwd_gqa): a group's K, V and log-gates feed its G query
 heads, so dK, dV and d(log g) are sums over the heads, and the score
-gradient applies the gate softmax's Jacobian to the summed d(log g).  The
-library has no kernel for it yet.
+gradient applies the gate softmax's Jacobian to the summed d(log g).
+
+Full training scope (Sec. 4.2 "training scope", Eq. scope_grad): every
+historical block is gated and nothing is dropped, which is the sparse form
+with K >= C_i; its gradients are sas_attention_bwd_head with topk >= C
+(sas_attention_bwd_full_head).
+
+Hard Top-K gate with the straight-through estimator (Sec. 4.2 "ranking
+preservation", App. D "hard gating with STE", Eq. rank_unbounded;
+sas_attention_bwd_ste_head): the forward gate is g^hard (1 on the kept
+blocks, 0 on the dropped ones: the inference form, logits unbiased, the
+normaliser LSE_S over the attended keys S only); the backward takes
+g^hat = stopgrad(g^hard - g) + g with the soft g = softmax(s), so
+  dQ, dK, dV  are those of the hard forward (constant gates),
+  dg_m        = sum_{j in B_m} p~_j (dp_j - Delta),  p~_j = exp(z_j - LSE_S),
+                for EVERY historical block m (z_j = sm_scale q.k_j; for a
+                dropped block p~ is the unbounded weight of Eq. rank_unbounded),
+  ds_l        = g_l (dg_l - sum_m g_m dg_m)   (the softmax Jacobian).
 """
 from __future__ import annotations
 
@@ -36,7 +52,7 @@ import math
 
 import numpy as np
 
-from oracle.sas_oracle import _row_keys_and_bias, historical_count, log_gates, MODE_TRAIN_SOFT
+from oracle.sas_oracle import _row_keys_and_bias, historical_count, log_gates, MODE_INFER_HARD, MODE_TRAIN_SOFT
 
 
 def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
@@ -163,4 +179,80 @@ def sas_attention_bwd_varlen(Q, K, V, s, dO, cu_seqlens, b, topk, mode=MODE_TRAI
         for f in ("dQ", "dK", "dV", "dlogg"):
             out[f][:, s0:s1] = r[f]
         out["ds"][:, s0:s1, :r["ds"].shape[2]] = r["ds"]
+    return out
+
+
+def sas_attention_bwd_full_head(Q, K, V, s, dO, b, sm_scale=None):
+    """Gradients of the full training scope of one head (every historical
+    block gated with log g = log_softmax(s) over the row's history): the
+    sparse backward keeping every block.  dlogg is [N, C] indexed by block."""
+    N = Q.shape[0]
+    C = -(-N // b)
+    return sas_attention_bwd_head(Q, K, V, s, dO, b, C, MODE_TRAIN_SOFT, sm_scale)
+
+
+def sas_attention_bwd_ste_head(Q, K, V, s, dO, b, topk, sm_scale=None):
+    """Gradients of the hard Top-K gate under the straight-through estimator,
+    one head (see the module docstring).  Q, K, V, dO: [N, d]; s: [N, >=C-1].
+    Returns dQ, dK, dV [N, d] (the hard forward's), dg [N, C] (dL/dg^hat of
+    every historical block, 0 past the history), x = g dg [N, C] (the
+    gradient with respect to log g^hat through the estimator) and ds [N, C]."""
+    N, d = Q.shape
+    if sm_scale is None:
+        sm_scale = 1.0 / math.sqrt(d)
+    C = -(-N // b)
+    hard = sas_attention_bwd_head(Q, K, V, s, dO, b, topk, MODE_INFER_HARD, sm_scale)
+    dg = np.zeros((N, C))
+    x = np.zeros((N, C))
+    ds = np.zeros((N, C))
+    for i in range(N):
+        c = historical_count(i, b)
+        if c == 0:
+            continue
+        # the hard forward of row i: its attended keys, logits and normaliser
+        keys, bias, _, _, _ = _row_keys_and_bias(i, s[i], b, topk, MODE_INFER_HARD)
+        zs = sm_scale * (K[keys] @ Q[i]) + bias
+        zmax = zs.max()
+        lse_s = zmax + math.log(np.exp(zs - zmax).sum())
+        o = np.exp(zs - lse_s) @ V[keys]
+        delta = dO[i] @ o
+        # every historical block, attended or not, under the same normaliser
+        for m in range(c):
+            toks = np.arange(m * b, (m + 1) * b)
+            pt = np.exp(sm_scale * (K[toks] @ Q[i]) - lse_s)
+            dg[i, m] = (pt * (V[toks] @ dO[i] - delta)).sum()
+        g = np.exp(log_gates(np.asarray(s[i][:c], dtype=np.float64)))
+        x[i, :c] = g * dg[i, :c]
+        ds[i, :c] = g * (dg[i, :c] - (g * dg[i, :c]).sum())
+    return {"dQ": hard["dQ"], "dK": hard["dK"], "dV": hard["dV"], "dg": dg, "x": x, "ds": ds}
+
+
+def sas_attention_bwd_ste_gqa(Q, K, V, s, dO, b, topk, sm_scale=None):
+    """The hard-STE gradients under GQA: Q, dO [Hq, N, d]; K, V, s per KV
+    group.  dK, dV and the group's dg (hence x and ds) are sums over its G
+    query heads; ds applies the Jacobian to the summed dg."""
+    Hq, N, d = Q.shape
+    Hkv = K.shape[0]
+    if Hq % Hkv:
+        raise ValueError("Hq must be a multiple of Hkv")
+    G = Hq // Hkv
+    C = -(-N // b)
+    out = {"dQ": np.zeros((Hq, N, d)), "dK": np.zeros((Hkv, N, d)), "dV": np.zeros((Hkv, N, V.shape[2])),
+           "dg": np.zeros((Hkv, N, C)), "x": np.zeros((Hkv, N, C)), "ds": np.zeros((Hkv, N, C))}
+    for h in range(Hq):
+        g = h // G
+        r = sas_attention_bwd_ste_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, sm_scale)
+        out["dQ"][h] = r["dQ"]
+        out["dK"][g] += r["dK"]
+        out["dV"][g] += r["dV"]
+        out["dg"][g] += r["dg"]
+    for g in range(Hkv):
+        for i in range(N):
+            c = historical_count(i, b)
+            if c == 0:
+                continue
+            gates = np.exp(log_gates(np.asarray(s[g, i][:c], dtype=np.float64)))
+            dgi = out["dg"][g, i, :c]
+            out["x"][g, i, :c] = gates * dgi
+            out["ds"][g, i, :c] = gates * (dgi - (gates * dgi).sum())
     return out

@@ -199,3 +199,136 @@ def test_packed_backward_equals_autograd_of_the_packed_forward_oracle():
             args_m = (Xm, s) if name == "K" else (K, Xm)
             G[idx] = (loss(*args_p) - loss(*args_m)) / (2 * h)
         assert np.allclose(G, ref, atol=1e-6), name
+
+
+# ---------------------------------------------------------------- full scope
+
+@pytest.mark.parametrize("N,seed", [(41, 31), (64, 32)])
+def test_full_scope_backward_equals_autograd_with_every_block_gated(N, seed):
+    # Sec. 4.2 full scope: no Top-K, every historical block enters with log g =
+    # log_softmax(s); the dense masked form keeping all blocks gives its gradients
+    b, d = 8, 5
+    Q, K, V, dO, s = _inputs(N, d, seed)
+    sm = 1 / math.sqrt(d)
+    C = -(-N // b)
+    q, k, v, st, Ot = _torch_dense(Q, K, V, s, b, C, sm)
+    (Ot * torch.tensor(dO)).sum().backward()
+    r = BO.sas_attention_bwd_full_head(Q, K, V, s, dO, b)
+    assert np.allclose(r["dQ"], q.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dK"], k.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dV"], v.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["ds"], st.grad.numpy()[:, :C], atol=1e-12)
+    # dlogg is indexed by block (every block is kept): the paper's closed form
+    # dlogg_m = g_m dg_m, dg_m = sum_{j in B_m} (p_j / g_m) dO.(v_j - o) (App. D)
+    assert r["dlogg"].shape == (N, C)
+    fwd = O.sas_attention_full_scope(Q, K, V, s, b)
+    for i in range(b, N):
+        c = i // b
+        lg = O.log_gates(s[i, :c])
+        keys = np.arange(i + 1)
+        z = sm * (K[keys] @ Q[i]) + np.concatenate([np.repeat(lg, b), np.zeros(i + 1 - c * b)])
+        p = np.exp(z - z.max())
+        p /= p.sum()
+        for m in range(c):
+            blk = slice(m * b, (m + 1) * b)
+            g = math.exp(lg[m])
+            dg = ((p[blk] / g) * (V[blk] @ dO[i] - fwd["O"][i] @ dO[i])).sum()
+            assert math.isclose(r["dlogg"][i, m], g * dg, rel_tol=1e-9, abs_tol=1e-12)
+
+
+# -------------------------------------------------------- hard gate with STE
+
+def _torch_ste(Q, K, V, s, b, topk, sm_scale):
+    """Dense form of the hard Top-K gate under the straight-through estimator:
+    row i weighs token j of historical block m by g^hat_m exp(z_j), the current
+    block by exp(z_j), with g^hat = stopgrad(g^hard - g) + g, g = softmax(s_i)
+    over the row's history.  Returns the leaves, O and each row's g^hat (its
+    gradient retained)."""
+    N, d = Q.shape
+    t = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
+    q, k, v, st = t(Q), t(K), t(V), t(s)
+    Z = sm_scale * q @ k.T
+    outs, ghats = [], []
+    for i in range(N):
+        c = i // b
+        w_hist = []
+        if c:
+            g = torch.softmax(st[i, :c], dim=0)
+            hard = torch.zeros(c, dtype=torch.float64)
+            hard[O.topk_blocks(s[i, :c], topk)] = 1.0
+            gh = (hard - g).detach() + g
+            gh.retain_grad()
+            ghats.append(gh)
+            w_hist = [gh.repeat_interleave(b)]
+        else:
+            ghats.append(None)
+        zi = Z[i, :i + 1]
+        w = torch.exp(zi - zi.max().detach())
+        wt = torch.cat(w_hist + [torch.ones(i + 1 - c * b, dtype=torch.float64)]) * w
+        outs.append((wt @ v[:i + 1]) / wt.sum())
+    return q, k, v, st, torch.stack(outs), ghats
+
+
+@pytest.mark.parametrize("N,topk,seed", [(37, 2, 41), (50, 1, 42), (33, 0, 43)])
+def test_ste_backward_equals_autograd_through_the_estimator(N, topk, seed):
+    b, d = 8, 5
+    Q, K, V, dO, s = _inputs(N, d, seed)
+    sm = 1 / math.sqrt(d)
+    q, k, v, st, Ot, ghats = _torch_ste(Q, K, V, s, b, topk, sm)
+    (Ot * torch.tensor(dO)).sum().backward()
+    r = BO.sas_attention_bwd_ste_head(Q, K, V, s, dO, b, topk)
+    # the forward is the hard one
+    assert np.allclose(Ot.detach().numpy(), O.sas_attention_head(Q, K, V, s, b, topk, O.MODE_INFER_HARD)["O"],
+                       atol=1e-12)
+    assert np.allclose(r["dQ"], q.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dK"], k.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dV"], v.grad.numpy(), atol=1e-12)
+    C = r["ds"].shape[1]
+    assert np.allclose(r["ds"], st.grad.numpy()[:, :C], atol=1e-12)
+    for i, gh in enumerate(ghats):
+        if gh is not None:
+            assert np.allclose(r["dg"][i, :gh.shape[0]], gh.grad.numpy(), atol=1e-12)
+    # x = g dg, and ds = x - g sum(x) (the sparse score-gradient formula applied to x)
+    for i in range(N):
+        c = i // b
+        if c:
+            g = np.exp(O.log_gates(s[i, :c]))
+            assert np.allclose(r["x"][i, :c], g * r["dg"][i, :c], atol=1e-14)
+            assert np.allclose(r["ds"][i, :c], r["x"][i, :c] - g * r["x"][i, :c].sum(), atol=1e-12)
+
+
+def test_ste_gate_weight_of_a_dropped_block_is_unbounded():
+    # Eq. rank_unbounded: a dropped block whose logits outscore the attended set
+    # gets p~ = exp(z - LSE_S) > 1, so its dg grows with exp(z - max_S z)
+    b, d, N, topk = 4, 2, 12, 1
+    Q = np.zeros((N, d)); Q[:, 0] = 1.0
+    K = np.zeros((N, d)); K[0:4, 0] = 6.0          # block 0: large logits for every query
+    V = np.zeros((N, d)); V[0:4, 1] = 1.0
+    dO = np.zeros((N, d)); dO[:, 1] = 1.0
+    s = np.zeros((N, 3)); s[:, 1] = 5.0            # the selector keeps block 1, drops block 0
+    r = BO.sas_attention_bwd_ste_head(Q, K, V, s, dO, b, topk, sm_scale=1.0)
+    i = N - 1                                      # row 11: blocks 0, 1 historical, block 1 kept
+    assert O.topk_blocks(s[i, :2], topk).tolist() == [1]
+    # the attended set holds block 1 (z = 0) and row i's own block (z = 0): LSE_S = log 8
+    pt = math.exp(6.0 - math.log(8.0))
+    assert pt > 1
+    assert math.isclose(r["dg"][i, 0], 4 * pt * (1.0 - 0.0), rel_tol=1e-12)
+
+
+def test_ste_gqa_is_the_sum_over_heads():
+    b, d, N, topk = 8, 3, 30, 2
+    rng = np.random.default_rng(44)
+    Q, dO = rng.standard_normal((4, N, d)), rng.standard_normal((4, N, d))
+    K, V = rng.standard_normal((2, N, d)), rng.standard_normal((2, N, d))
+    s = rng.standard_normal((2, N, 4))
+    r = BO.sas_attention_bwd_ste_gqa(Q, K, V, s, dO, b, topk)
+    for g in range(2):
+        parts = [BO.sas_attention_bwd_ste_head(Q[h], K[g], V[g], s[g], dO[h], b, topk) for h in (2 * g, 2 * g + 1)]
+        assert np.allclose(r["dK"][g], parts[0]["dK"] + parts[1]["dK"], atol=1e-13)
+        assert np.allclose(r["dg"][g], parts[0]["dg"] + parts[1]["dg"], atol=1e-13)
+        for i in range(N):
+            c = i // b
+            if c:
+                gt = np.exp(O.log_gates(s[g, i, :c]))
+                dgi = r["dg"][g, i, :c]
+                assert np.allclose(r["ds"][g, i, :c], gt * (dgi - (gt * dgi).sum()), atol=1e-13)
