@@ -57,7 +57,14 @@ typedef enum {
  *   TRAIN_SOFT : Eq. ours_train, logits of a kept block get + log g_m.
  *   INFER_HARD : Alg. 2, kept blocks enter unbiased (the forward of the hard
  *                Top-K gate, Sec. 4.2 "ranking preservation"). */
-typedef enum { SAS_MODE_TRAIN_SOFT = 0, SAS_MODE_INFER_HARD = 1 } sas_mode;
+/*   TRAIN_HARD_STE : the hard Top-K gate trained through the straight-through
+ *                estimator (Sec. 4.2 "ranking preservation", App. D, Eq.
+ *                rank_unbounded): the forward is that of INFER_HARD; the
+ *                backward adds the gate gradient of every historical block,
+ *                kept or dropped, with the soft gates g = softmax(s) standing in
+ *                for the hard ones (see sas_attention_bwd).  Sparse scope,
+ *                softmax gates in the inner position. */
+typedef enum { SAS_MODE_TRAIN_SOFT = 0, SAS_MODE_INFER_HARD = 1, SAS_MODE_TRAIN_HARD_STE = 2 } sas_mode;
 
 /* Where the selector scores s come from (Alg. 1 step 1).
  *   SCORES_GIVEN  : the caller passes s as a [B, H, N, C] fp32 table.
@@ -90,7 +97,7 @@ typedef enum { SAS_GATE_INNER = 0, SAS_GATE_OUTER = 1 } sas_gate_pos;
  *            log-gate, softmax(q K^T + log g) V over the row's whole history
  *            (Eq. fula with the gates, setting 9).  Needs the softmax gate in
  *            the inner position and [B, H, N, d] inputs (max_seqs = 0); topk
- *            is not used; sel_idx / sel_logg must be NULL; no backward.
+ *            is not used; sel_idx / sel_logg must be NULL.
  *            With the learned selector the handle keeps a [B, Hkv, N, C]
  *            fp32 score table (the dense gate table the paper's kernel
  *            reads, App. E); with given scores the caller's table is read.
@@ -113,12 +120,11 @@ typedef struct {
                              query heads of a group share one selection (Sec. 5.3;
                              Sec. 5 inference implementation): one score table
                              per group, given or from the learned selector's group
-                             gate query.  Hkv < H has no backward.                    */
+                             gate query.                                               */
     int32_t max_seqs;     /* 0: [B, H, N, d] batches of N-token sequences.  > 0: packed
                              variable-length sequences, at most max_seqs of them, in
                              [H, N, d] tensors whose token axis (N = capacity) holds
-                             them back to back (sas_attention_fwd_varlen); needs B = 1,
-                             has no backward.                                          */
+                             them back to back (sas_attention_fwd_varlen); needs B = 1. */
     int32_t max_seqlen;   /* packed mode: longest sequence (1 .. N; 0 selects N); the
                              score table has C = ceil(max_seqlen / 64) columns         */
     int32_t scope;        /* sas_scope (0 = SPARSE, the SAS default)                   */
@@ -172,9 +178,9 @@ sas_status sas_attention_fwd(sas_handle* h,
                              int32_t* sel_idx, float* sel_logg,
                              void* stream);
 
-/* full* training scope (Table 1 setting 11; Sec. 4.2: "a stochastic
- * approximation to full scope by adding noise to the scores before
- * activation"): sas_attention_fwd with s~ = s + noise in place of the scores
+/* full* training scope (Table 1 setting 11, Sec. 4.2: the full scope
+ * approximated stochastically, the scores perturbed by noise before the gate
+ * activation and the Top-K): sas_attention_fwd with s~ = s + noise in place of the scores
  * s, for the gate activation and for the Top-K alike.  The sum is formed in
  * fp32: s~ = fp32(s + noise) with s the given score or, for the learned
  * selector, fp32(q~ . K~ / sqrt(d_sel)).
@@ -192,7 +198,7 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
                                    void* stream);
 
 /* Backward of sas_attention_fwd (Alg. 4 of App. E; gate and score gradients
- * of App. D), for d = 128, softmax gates in the inner position, either mode.
+ * of App. D), for d = 128, softmax gates in the inner position, any mode.
  * The kept sets are those of the forward (the Top-K choice is a constant of
  * the backward), and the per-tile block lists are read from the handle: call
  * it after the sas_attention_fwd of the same inputs on this handle, with no
@@ -205,6 +211,24 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
  * tiles of one query head.  The gradients are the same either way, up to the
  * order of floating-point sums.
  *
+ * Full training scope (a SAS_SCOPE_FULL handle; Sec. 4.2, Eq. scope_grad):
+ * every historical block of a row is kept and gated, so dlogg holds one
+ * entry per historical block ([B, Hkv, N, C], entry m for block m) and the
+ * score gradient is ds = dlogg - g sum(dlogg) over the whole history.  With
+ * given scores, `scores` is required (the log-gates s - LSE are rebuilt from
+ * it); with the learned selector the handle's score table is used.
+ *
+ * Hard Top-K gate under the straight-through estimator (a
+ * SAS_MODE_TRAIN_HARD_STE handle, given scores, [B, H, N, d] inputs): dQ, dK
+ * and dV are those of the hard forward (kept blocks unbiased, the rest
+ * dropped); the gate gradient covers every historical block, dropped ones
+ * included, each weighted by exp(z - LSE) under the hard forward's LSE (Eq.
+ * rank_unbounded).  dlogg [B, Hkv, N, C] holds x_m = g_m dL/dg^_m for block m
+ * (g = softmax(s) over the row's history, g^ the estimator's gate), and
+ * dscores = x - g sum(x) = g (dg^ - sum g dg^).  `scores` is required.
+ * Both forms build per-row lists of every historical block ([B, Hkv, N, C]
+ * int32 + fp32 of handle workspace, allocated by the first such call).
+ *
  * Packed sequences (a handle created with max_seqs > 0): the backward of the
  * last sas_attention_fwd_varlen on the handle, whose tile table it reads;
  * the layouts drop B ([H, N, d], [Hkv, N, C], ...), every sequence is its
@@ -216,11 +240,13 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
  *   dO         bf16 [B, H, N, d] gradient of the loss w.r.t. O          (in)
  *   sel_idx, sel_logg: the forward's outputs, or NULL if the forward
  *              was given NULL for them                                   (in)
- *   scores     fp32 [B, Hkv, N, C] given scores; needed only for dscores (in)
+ *   scores     fp32 [B, Hkv, N, C] given scores; needed for dscores and by
+ *              the full scope and hard-STE forms                         (in)
  *   dQ         bf16 [B, H, N, d]; dK, dV bf16 [B, Hkv, N, d]             (out)
  *   dlogg      fp32 [B, Hkv, N, topk] dL/d(log g) of each kept block, in
  *              the order of sel_idx, summed over the group's query heads
- *              (0 where padded; all 0 in INFER_HARD mode); may be NULL   (out)
+ *              (0 where padded; all 0 in INFER_HARD mode); [B, Hkv, N, C]
+ *              by block for the full scope and hard-STE; may be NULL     (out)
  *   dscores    fp32 [B, Hkv, N, C] dL/ds of the given scores, sparse scope:
  *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
  *              row's history; SCORES_GIVEN handles only, else NULL.

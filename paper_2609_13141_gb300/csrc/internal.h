@@ -226,10 +226,21 @@ struct AttnBwdArgs {
     int N, C, T, BH, topk, mode, d;
     int G;                      // query heads per KV group: K, V, the lists and the gate gradients are per group
     float sm_scale;
+    // pass 1 and the gate gradients only (no pass 2; dQ and offs may be null): the
+    // gate pass of the hard Top-K gate under the straight-through estimator
+    bool gate_only;
 };
 extern const int kBwdMaxTiles;   // query tiles per head the backward supports (head-packed: segments + G)
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total);
 cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err);
+// Kept lists that hold every historical block of each row (idx[m] = m, lg[m] =
+// s_m - lse of the row, [BHkv][N][C]) and tile unions of every block below the
+// tile's diagonal ([BHkv][T][C], counts [BHkv][T]); s and lse per KV group.
+cudaError_t launch_bwd_dense_lists(const float* s, const float* lse, int BHkv, int N, int C, int T, int32_t* idx,
+                                   float* lg, int32_t* uidx, int32_t* ucnt, const KernelEnv& env);
+// Each row's log-sum-exp over its C_i = floor(i / 64) scores ([rows][C] fp32,
+// rows = heads x N), 0 for C_i = 0.
+cudaError_t launch_row_lse(const float* scores, int N, int C, long long rows, float* out, const KernelEnv& env);
 
 // ---- failure-path self test (bounded wait on a barrier nothing completes)
 cudaError_t launch_wait_selftest(int* status, long long limit, cudaStream_t stream);

@@ -19,6 +19,13 @@
 //                     over them, dV += P^T dO and dK += dS^T Q.
 //   bwd_ds_kernel     score gradient of given scores (sparse scope):
 //                     ds_m = dlogg_m [m kept] - g_m sum dlogg.
+//   bwd_dense_*       kept lists and tile unions of every historical block:
+//                     with them the same passes give the backward of the
+//                     full training scope (every block kept and gated) and,
+//                     pass 1 alone with the soft log-gates and the hard
+//                     forward's LSE, the gate gradient of the hard Top-K gate
+//                     under the straight-through estimator (x_m = g_m dg_m,
+//                     whose score gradient x - g sum x is g (dg - sum g dg)).
 // GQA: a KV group's K, V, kept lists and log-gates feed its G query heads, so
 // pass 1 runs per query head on its group's K, V and lists and writes the
 // head's log-gate gradient, bwd_dlogg_sum adds the G heads (in head order:
@@ -349,7 +356,8 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
             lse2 = __ldg(p.LSE + roff) * kLog2eB;
             if (hk == 0) p.delta[roff] = delta;
         }
-        const int slot0 = __ldg(p.slot_off + tb);
+        // the per-block offsets for pass 2 (a gate-only pass has no pass 2: offs null)
+        const int slot0 = p.offs != nullptr ? __ldg(p.slot_off + tb) : 0;
         const int nsel = valid ? min(p.topk, c) : 0;
         const int32_t* my_idx = p.sel_idx + kvoff * p.topk;
         const float* my_lg = p.sel_logg + kvoff * p.topk;
@@ -392,7 +400,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 // block the row does not attend; the causal limit only on its own block
                 const float boff = lim >= 0 ? bias - lse2 : -CUDART_INF_F;
                 const bool causal = lim >= 0 && lim < kKeys - 1;
-                if (hk == 0) p.offs[(static_cast<long long>(slot0) + j) * kRows + r] = boff;   // for pass 2
+                if (hk == 0 && p.offs != nullptr) p.offs[(static_cast<long long>(slot0) + j) * kRows + r] = boff;
                 const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2), bo2 = f32x2(boff, boff);
                 const uint64_t nd2 = f32x2(-delta, -delta);
                 uint64_t acc = 0;
@@ -438,7 +446,7 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 uint32_t o[32];
                 tmem_ld32(lane_addr + kTmemDQ + cc * 32, o);
                 tmem_wait_ld();
-                if (valid) {
+                if (valid && p.dQ != nullptr) {   // null: a gate-only pass
                     uint4* dst = reinterpret_cast<uint4*>(p.dQ + roff * kD + cc * 32);
 #pragma unroll
                     for (int q = 0; q < 4; ++q)
@@ -983,6 +991,40 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
     }
 }
 
+// ----------------------------------------------------- dense block lists
+
+// Kept lists and tile unions holding every historical block, for the
+// backwards that gate all of them: the full training scope (Sec. 4.2; log g =
+// s - LSE of the row's scores) and the gate pass of the hard Top-K gate under
+// the straight-through estimator (the soft log g of every block).  Row i keeps
+// blocks 0 .. C_i - 1 in order with log g_m = s_m - lse_i (0 past its
+// history); one warp per row.
+__global__ void __launch_bounds__(256) bwd_dense_rows_kernel(const float* s, const float* lse, int N, int C,
+                                                             long long rows, int32_t* idx, float* lg) {
+    const long long w = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= rows) return;
+    const int c = min(static_cast<int>(w % N) >> 6, C);
+    const float l = c > 0 ? __ldg(lse + w) : 0.f;
+    const float* sr = s + w * C;
+    for (int m = lane; m < C; m += 32) {
+        idx[w * C + m] = m;
+        lg[w * C + m] = m < c ? __ldg(sr + m) - l : 0.f;
+    }
+}
+
+// Tile t's union: blocks 0 .. 2t - 1 (its diagonal blocks are visited apart).
+// One warp per (group, tile).
+__global__ void __launch_bounds__(256) bwd_dense_unions_kernel(int32_t* uidx, int32_t* ucnt, int T, int C,
+                                                               long long tiles) {
+    const long long w = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= tiles) return;
+    const int n = min(2 * static_cast<int>(w % T), C);
+    for (int k = lane; k < n; k += 32) uidx[w * C + k] = k;
+    if (lane == 0) ucnt[w] = n;
+}
+
 // --------------------------------------------------------- score gradient
 
 // ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of the row's C_i
@@ -1106,6 +1148,17 @@ cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long lo
     return e;
 }
 
+cudaError_t launch_bwd_dense_lists(const float* s, const float* lse, int BHkv, int N, int C, int T, int32_t* idx,
+                                   float* lg, int32_t* uidx, int32_t* ucnt, const KernelEnv& env) {
+    const long long rows = static_cast<long long>(BHkv) * N;
+    const long long tiles = static_cast<long long>(BHkv) * T;
+    bwd_dense_rows_kernel<<<static_cast<unsigned>((rows * 32 + 255) / 256), 256, 0, env.stream>>>(s, lse, N, C, rows,
+                                                                                                  idx, lg);
+    bwd_dense_unions_kernel<<<static_cast<unsigned>((tiles * 32 + 255) / 256), 256, 0, env.stream>>>(uidx, ucnt, T, C,
+                                                                                                    tiles);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const char** err) {
     if (a.d != kD) {
         *err = "backward: head dim must be 128";
@@ -1189,25 +1242,27 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     else bwd_dq_kernel<false><<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
-    // inverted lists of the KV groups' union lists
-    e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(gtiles) * 4, env.stream);
-    if (e != cudaSuccess) { *err = "backward list counts"; return e; }
-    const unsigned gb = static_cast<unsigned>((srcs + 255) / 256);
-    const int32_t* uidx = hp ? a.seg_union_idx : a.union_idx;
-    const int32_t* ucnt = hp ? a.seg_union_cnt : a.union_cnt;
-    const int ustride = hp ? a.seg_cap : a.C;
-    bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cnt, BHkv, a.T, nsrc, ustride, a.tiles,
-                                                      a.ntiles, a.tile_off, hp ? G : 0);
-    bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, gtiles);
-    bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cursor, a.inv_tiles, a.inv_pos, BHkv, a.T,
-                                                     nsrc, ustride, a.tiles, a.ntiles, a.tile_off, hp ? G : 0);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
-    // pass 2: one CTA per (KV group, key pair)
-    if (hp) bwd_dkv_kernel<true><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
-    else bwd_dkv_kernel<false><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
+    if (!a.gate_only) {   // a gate-only pass (the STE gate gradient) has no pass 2
+        // inverted lists of the KV groups' union lists
+        e = cudaMemsetAsync(a.inv_cnt, 0, static_cast<size_t>(gtiles) * 4, env.stream);
+        if (e != cudaSuccess) { *err = "backward list counts"; return e; }
+        const unsigned gb = static_cast<unsigned>((srcs + 255) / 256);
+        const int32_t* uidx = hp ? a.seg_union_idx : a.union_idx;
+        const int32_t* ucnt = hp ? a.seg_union_cnt : a.union_cnt;
+        const int ustride = hp ? a.seg_cap : a.C;
+        bwd_inv_count_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cnt, BHkv, a.T, nsrc, ustride, a.tiles,
+                                                          a.ntiles, a.tile_off, hp ? G : 0);
+        bwd_inv_scan_kernel<<<1, 1024, 0, env.stream>>>(a.inv_cnt, a.inv_off, a.inv_cursor, gtiles);
+        bwd_inv_fill_kernel<<<gb, 256, 0, env.stream>>>(uidx, ucnt, a.inv_cursor, a.inv_tiles, a.inv_pos, BHkv, a.T,
+                                                         nsrc, ustride, a.tiles, a.ntiles, a.tile_off, hp ? G : 0);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
+        // pass 2: one CTA per (KV group, key pair)
+        if (hp) bwd_dkv_kernel<true><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        else bwd_dkv_kernel<false><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
+    }
     if (G > 1 && a.topk > 0) {
         const long long total = static_cast<long long>(BHkv) * per_head;
         bwd_dlogg_sum_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, env.stream>>>(

@@ -1497,6 +1497,12 @@ cudaError_t launch_seg_unions(const int32_t* sel_idx, int BHkv, int N, int C, in
     return cudaGetLastError();
 }
 
+cudaError_t launch_row_lse(const float* scores, int N, int C, long long rows, float* out, const KernelEnv& env) {
+    const long long blocks = (rows * 32 + 255) / 256;
+    row_lse_kernel<<<static_cast<unsigned>(blocks), 256, 0, env.stream>>>(scores, N, C, rows, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char** err) {
     SelParams p;
     p.BH = a.BH; p.N = a.N; p.C = a.C; p.T = a.T; p.F = a.F; p.topk = a.topk;
@@ -1514,10 +1520,7 @@ cudaError_t launch_select(const SelectArgs& a, const KernelEnv& env, const char*
     }
     if (a.full_lse != nullptr && a.scores != nullptr) {
         // given scores: the attention kernel reads them directly; only the normalisers
-        const long long rows = static_cast<long long>(a.BH) * a.N;
-        const long long blocks = (rows * 32 + 255) / 256;
-        row_lse_kernel<<<static_cast<unsigned>(blocks), 256, 0, env.stream>>>(a.scores, a.N, a.C, rows, a.full_lse);
-        cudaError_t e = cudaGetLastError();
+        cudaError_t e = launch_row_lse(a.scores, a.N, a.C, static_cast<long long>(a.BH) * a.N, a.full_lse, env);
         if (e != cudaSuccess) *err = "row log-sum-exp launch";
         return e;
     }

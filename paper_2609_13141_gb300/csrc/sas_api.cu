@@ -157,6 +157,12 @@ struct sas_handle {
     int32_t* bwd_tiles = nullptr;   // inverted lists: tiles, then block positions
     float* bwd_dlogg = nullptr;     // GQA: per query head [BH][N][topk], then per group [BHkv][N][topk]
     float* bwd_offs = nullptr;      // per-row offsets of every visited block (pass 1 -> pass 2)
+    // full scope and hard-STE backwards: lists of every historical block
+    int32_t* dense_idx = nullptr;   // [BHkv][N][C] block indices 0 .. C_i - 1
+    float* dense_lg = nullptr;      // [BHkv][N][C] their log-gates s - LSE
+    int32_t* dense_uidx = nullptr;  // [BHkv][T][C] tile unions (every block below the diagonal)
+    int32_t* dense_ucnt = nullptr;  // [BHkv][T]
+    float* dense_lse = nullptr;     // [BHkv][N] soft normalisers of the given scores (hard-STE)
     size_t bwd_offs_bytes = 0;
     bool bwd_offs_bound = false;    // sized for the upper bound: no per-call read-back
     // timing
@@ -182,6 +188,9 @@ sas_status cuda_fail(sas_handle* h, cudaError_t e, const char* what) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Gate form the forward kernels run: the hard-STE mode's forward is the hard one.
+int kernel_mode(const sas_config& c) { return c.mode == SAS_MODE_TRAIN_HARD_STE ? SAS_MODE_INFER_HARD : c.mode; }
 bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
 cudaEvent_t next_event(sas_handle* h) {
@@ -261,7 +270,8 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (c.d != 64 && c.d != 128) return SAS_ERR_UNSUPPORTED;
     if (c.topk < 0) return SAS_ERR_INVALID_ARG;
     if (c.topk > 64) return SAS_ERR_UNSUPPORTED;
-    if (c.mode != SAS_MODE_TRAIN_SOFT && c.mode != SAS_MODE_INFER_HARD) return SAS_ERR_INVALID_ARG;
+    if (c.mode != SAS_MODE_TRAIN_SOFT && c.mode != SAS_MODE_INFER_HARD && c.mode != SAS_MODE_TRAIN_HARD_STE)
+        return SAS_ERR_INVALID_ARG;
     if (c.selector != SAS_SEL_SCORES_GIVEN && c.selector != SAS_SEL_MEANPOOL_PROJ) return SAS_ERR_INVALID_ARG;
     if (c.gate_act != SAS_GATE_SOFTMAX && c.gate_act != SAS_GATE_SIGMOID && c.gate_act != SAS_GATE_LOGIT)
         return SAS_ERR_INVALID_ARG;
@@ -270,6 +280,10 @@ sas_status sas_create(const sas_config* cfg, sas_handle** out) {
     if (c.scope != SAS_SCOPE_SPARSE && c.scope != SAS_SCOPE_FULL) return SAS_ERR_INVALID_ARG;
     if (c.scope == SAS_SCOPE_FULL &&
         (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER || c.max_seqs > 0))
+        return SAS_ERR_UNSUPPORTED;
+    // the straight-through estimator of the hard gate stands the softmax gates in
+    if (c.mode == SAS_MODE_TRAIN_HARD_STE &&
+        (c.scope != SAS_SCOPE_SPARSE || c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER))
         return SAS_ERR_UNSUPPORTED;
     const int d_sel = c.d_sel == 0 ? c.d : c.d_sel;
     if (d_sel != 64 && d_sel != 128) return SAS_ERR_UNSUPPORTED;
@@ -372,6 +386,11 @@ void sas_destroy(sas_handle* h) {
     cudaFree(h->bwd_tiles);
     cudaFree(h->bwd_dlogg);
     cudaFree(h->bwd_offs);
+    cudaFree(h->dense_idx);
+    cudaFree(h->dense_lg);
+    cudaFree(h->dense_uidx);
+    cudaFree(h->dense_ucnt);
+    cudaFree(h->dense_lse);
     for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
     delete h;
 }
@@ -450,7 +469,7 @@ sas_status attention_fwd(sas_handle* h, const void* Q, const void* K, const void
     aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
     aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
-    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = kernel_mode(c);
     aa.G = h->G;
     aa.gate_pos = c.gate_pos;
     aa.sm_scale = h->sm_scale;
@@ -558,7 +577,7 @@ sas_status sas_attention_fwd_varlen(sas_handle* h, const int32_t* cu_seqlens, in
     aa.Q = Q; aa.K = K; aa.V = V; aa.O = O; aa.LSE = LSE;
     aa.union_idx = h->union_idx; aa.union_cnt = h->union_cnt;
     aa.sel_idx = out_idx; aa.sel_logg = out_lg;
-    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = c.mode;
+    aa.BH = h->BH; aa.N = c.N; aa.d = c.d; aa.C = h->C; aa.T = h->T; aa.topk = c.topk; aa.mode = kernel_mode(c);
     aa.G = h->G;
     aa.tiles = h->tiles; aa.ntiles = h->ntiles;
     aa.gate_pos = c.gate_pos;
@@ -638,7 +657,16 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     if (c.d != 128) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports d = 128");
     if (c.gate_act != SAS_GATE_SOFTMAX || c.gate_pos != SAS_GATE_INNER)
         return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports softmax gates in the inner position");
-    if (h->full) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports the sparse scope");
+    // the full scope and the hard gate's estimator gate every historical block
+    const bool ste = c.mode == SAS_MODE_TRAIN_HARD_STE;
+    const bool dense = h->full || ste;
+    if (dense) {
+        if (h->varlen) return fail(h, SAS_ERR_UNSUPPORTED, "the full-scope and hard-STE backwards take [B, H, N, d] inputs");
+        if (ste && c.selector != SAS_SEL_SCORES_GIVEN)
+            return fail(h, SAS_ERR_UNSUPPORTED, "the hard-STE backward needs given scores (SCORES_GIVEN)");
+        if (c.selector == SAS_SEL_SCORES_GIVEN && !scores)
+            return fail(h, SAS_ERR_INVALID_ARG, "the full-scope and hard-STE backwards need the given scores");
+    }
     // query tiles of one sequence (a key pair's inverted list holds at most that many)
     const int tseq = h->varlen ? (h->C + 1) / 2 : h->T;
     if (tseq > sas::kBwdMaxTiles)
@@ -650,6 +678,8 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const size_t rows = static_cast<size_t>(h->BH) * c.N;
     const size_t tiles = static_cast<size_t>(h->BH) * h->T;
+    // gate-gradient entries per row: the kept blocks, or every block (dense)
+    const size_t dl_w = std::max<size_t>(1, std::max(c.topk, dense ? h->C : 0));
     if (h->bwd_delta == nullptr) {
         // first backward on this handle: workspace (synchronous)
         cudaError_t e = cudaStreamSynchronize(s);
@@ -658,7 +688,7 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         if (e == cudaSuccess) e = alloc(&h->bwd_inv, (4 * tiles + 2) * 4);
         if (e == cudaSuccess) e = alloc(&h->bwd_tiles, 2 * tiles * pairs * 4);
         const size_t dl_rows = rows + (h->G > 1 ? static_cast<size_t>(h->BHkv) * c.N : 0);
-        if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, dl_rows * (c.topk > 0 ? c.topk : 1) * 4);
+        if (e == cudaSuccess) e = alloc(&h->bwd_dlogg, dl_rows * dl_w * 4);
         // offsets of pass 1 for pass 2: local tile t visits at most 2t + 2 blocks, so a
         // head needs at most T (T + 1) slots of 128 rows (packed sequences: 2 tseq per
         // tile slot); held whole when that fits in 8 GiB
@@ -684,6 +714,24 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
             return cuda_fail(h, e, "backward workspace");
         }
     }
+    if (dense && h->dense_idx == nullptr) {
+        // lists of every historical block (first dense backward on this handle; synchronous)
+        cudaError_t e = cudaStreamSynchronize(s);
+        const size_t cells = static_cast<size_t>(h->BHkv) * c.N * h->C;
+        const size_t utiles = static_cast<size_t>(h->BHkv) * h->T;
+        if (e == cudaSuccess) e = alloc(&h->dense_idx, cells * 4);
+        if (e == cudaSuccess) e = alloc(&h->dense_lg, cells * 4);
+        if (e == cudaSuccess) e = alloc(&h->dense_uidx, utiles * h->C * 4);
+        if (e == cudaSuccess) e = alloc(&h->dense_ucnt, utiles * 4);
+        if (e == cudaSuccess) e = alloc(&h->dense_lse, static_cast<size_t>(h->BHkv) * c.N * 4);
+        if (e != cudaSuccess) {
+            cudaFree(h->dense_idx); cudaFree(h->dense_lg); cudaFree(h->dense_uidx); cudaFree(h->dense_ucnt);
+            cudaFree(h->dense_lse);
+            h->dense_idx = nullptr; h->dense_lg = nullptr; h->dense_uidx = nullptr; h->dense_ucnt = nullptr;
+            h->dense_lse = nullptr;
+            return cuda_fail(h, e, "backward block lists");
+        }
+    }
     sas::AttnBwdArgs a{};
     a.Q = Q; a.K = K; a.V = V; a.O = O; a.dO = dO; a.LSE = LSE;
     a.union_idx = h->union_idx; a.union_cnt = h->union_cnt;
@@ -693,7 +741,8 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.dQ = dQ; a.dK = dK; a.dV = dV;
     // GQA: pass 1 writes each query head's d(log g); the group's is their sum
     a.dlogg_heads = h->G > 1 ? h->bwd_dlogg : nullptr;
-    a.dlogg = dlogg ? dlogg : h->bwd_dlogg + (h->G > 1 ? rows * (c.topk > 0 ? c.topk : 1) : 0);
+    float* dlogg_scratch = h->bwd_dlogg + (h->G > 1 ? rows * dl_w : 0);   // the group sums when dlogg is NULL
+    a.dlogg = dlogg ? dlogg : dlogg_scratch;
     a.ds = dscores;
     a.delta = h->bwd_delta;
     a.inv_cnt = h->bwd_inv;
@@ -723,6 +772,45 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     }
     const sas::KernelEnv env{s, h->status, h->limit};
     const char* err = "";
+    sas::AttnBwdArgs ag{};   // hard-STE: the gate pass over every historical block
+    if (dense) {
+        // log g = s - LSE of every historical block: the full scope's own
+        // normalisers, or (hard-STE) the soft ones of the given scores
+        const float* sv = c.selector == SAS_SEL_SCORES_GIVEN ? scores : h->full_table;
+        const float* lse = h->full_lse;
+        cudaError_t e = cudaSuccess;
+        if (ste) {
+            e = sas::launch_row_lse(scores, c.N, h->C, static_cast<long long>(h->BHkv) * c.N, h->dense_lse, env);
+            lse = h->dense_lse;
+        }
+        if (e == cudaSuccess)
+            e = sas::launch_bwd_dense_lists(sv, lse, h->BHkv, c.N, h->C, h->T, h->dense_idx, h->dense_lg,
+                                            h->dense_uidx, h->dense_ucnt, env);
+        if (e != cudaSuccess) return cuda_fail(h, e, "backward block lists");
+        h->launches += 2 + (ste ? 1 : 0);
+        if (ste) {
+            // the gate pass: pass 1 alone over every block, the soft log-gates as
+            // biases under the hard forward's LSE; its row sums are x = g dg
+            ag = a;
+            ag.mode = SAS_MODE_TRAIN_SOFT;
+            ag.sel_idx = h->dense_idx; ag.sel_logg = h->dense_lg;
+            ag.union_idx = h->dense_uidx; ag.union_cnt = h->dense_ucnt;
+            ag.topk = h->C;
+            ag.seg_rows = 0; ag.nseg = 0; ag.seg_cap = 0; ag.seg_union_idx = nullptr; ag.seg_union_cnt = nullptr;
+            ag.gate_only = true;
+            ag.dQ = nullptr;
+            ag.offs = nullptr;
+            // the hard pass: no gate gradient (its zeros go to the scratch), no score gradient
+            a.mode = SAS_MODE_INFER_HARD;
+            a.dlogg = dlogg_scratch;
+            a.ds = nullptr;
+            a.scores = nullptr;
+        } else {
+            a.sel_idx = h->dense_idx; a.sel_logg = h->dense_lg;
+            a.union_idx = h->dense_uidx; a.union_cnt = h->dense_ucnt;
+            a.topk = h->C;
+        }
+    }
     // slots of the per-row offsets pass 1 hands to pass 2: their number depends on
     // the forward's tile lists; a buffer of the upper bound needs no read-back,
     // otherwise it is read back (synchronously) to size the buffer
@@ -743,8 +831,14 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     if (e != cudaSuccess) return cuda_fail(h, e, err);
     // all its kernels: slot count and scan, pass 1, the inverted lists (count, scan,
     // fill), pass 2, the group sum of d(log g) and the score gradient
-    h->launches += 7 + ((h->G > 1 && c.topk > 0) ? 1 : 0) +
-                   ((a.ds != nullptr && a.scores != nullptr && c.topk > 0) ? 1 : 0);
+    h->launches += 7 + ((h->G > 1 && a.topk > 0) ? 1 : 0) +
+                   ((a.ds != nullptr && a.scores != nullptr && a.topk > 0) ? 1 : 0);
+    if (ste) {
+        e = timed_launch(h, 6, s, [&] { return sas::launch_attn_bwd(ag, env, &err); });
+        if (e != cudaSuccess) return cuda_fail(h, e, err);
+        h->launches += 1 + ((h->G > 1 && ag.topk > 0) ? 1 : 0) +
+                       ((ag.ds != nullptr && ag.scores != nullptr && ag.topk > 0) ? 1 : 0);
+    }
     return SAS_OK;
 }
 

@@ -25,6 +25,7 @@ SAS_ERR_OOM = 5
 
 SAS_MODE_TRAIN_SOFT = 0
 SAS_MODE_INFER_HARD = 1
+SAS_MODE_TRAIN_HARD_STE = 2
 SAS_SEL_SCORES_GIVEN = 0
 SAS_SEL_MEANPOOL_PROJ = 1
 SAS_GATE_SOFTMAX = 0
@@ -342,6 +343,7 @@ class SasLayer:
                  sm_scale=0.0, gate_act=SAS_GATE_SOFTMAX, gate_pos=SAS_GATE_INNER, Hkv=0, max_seqs=0, max_seqlen=0,
                  scope=SAS_SCOPE_SPARSE):
         self.B, self.H, self.N, self.d, self.topk = B, H, N, d, topk
+        self.mode = mode
         self.Hkv = Hkv or H                      # kept lists are per KV group
         self.selector = selector
         self.scope = scope
@@ -391,9 +393,12 @@ class SasLayer:
     def attention_bwd(self, Q, K, V, O, LSE, dO, scores=None, sel_idx=None, sel_logg=None, want_ds=False,
                       stream=None):
         """Returns (dQ, dK, dV, dlogg, dscores); dscores only with want_ds (given scores).
-        With Hkv < H, dK, dV, dlogg and dscores are per KV group (sums over its heads)."""
+        With Hkv < H, dK, dV, dlogg and dscores are per KV group (sums over its heads).
+        The full scope and the hard-STE mode report dlogg for every block: [B, Hkv, N, C]."""
         dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
-        dlogg = torch.empty(self.B, self.Hkv, self.N, max(self.topk, 1), device=Q.device, dtype=torch.float32)
+        C = -(-self.N // 64)
+        width = C if (self.scope == SAS_SCOPE_FULL or self.mode == SAS_MODE_TRAIN_HARD_STE) else max(self.topk, 1)
+        dlogg = torch.empty(self.B, self.Hkv, self.N, width, device=Q.device, dtype=torch.float32)
         ds = None
         if want_ds:
             ds = torch.empty(self.B, self.Hkv, self.N, -(-self.N // 64), device=Q.device, dtype=torch.float32)

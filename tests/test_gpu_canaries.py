@@ -94,7 +94,34 @@ def test_gqa_and_full_scope_outputs():
     L, gL = guarded((B, H, N), torch.float32)
     sas.sas_attention_fwd(full.h, Q, Kk, V, O, S, LSE=L)
     _check(gO, gL)
+    # the full scope's backward: a gate gradient for every block, [B, Hkv, N, C]
+    C = -(-N // 64)
+    dQ, gq = guarded((B, H, N, d), torch.bfloat16)
+    dK, gk = guarded((B, Hkv, N, d), torch.bfloat16)
+    dV, gv = guarded((B, Hkv, N, d), torch.bfloat16)
+    dl, gdl = guarded((B, Hkv, N, C), torch.float32)
+    ds, gds = guarded((B, Hkv, N, C), torch.float32)
+    sas.sas_attention_bwd(full.h, Q, Kk, V, O, L, dO, dQ, dK, dV, S, None, None, dl, ds)
+    _check(gq, gk, gv, gdl, gds)
+    assert sas.sas_get_device_status(full.h) == 0
     full.close()
+    # the hard gate under the straight-through estimator: hard forward, dense gate gradient
+    ste = sas.SasLayer(B, H, N, d, K, Hkv=Hkv, mode=sas.SAS_MODE_TRAIN_HARD_STE)
+    O, gO = guarded((B, H, N, d), torch.bfloat16)
+    L, gL = guarded((B, H, N), torch.float32)
+    si, gi = guarded((B, Hkv, N, K), torch.int32)
+    sl, gl = guarded((B, Hkv, N, K), torch.float32)
+    sas.sas_attention_fwd(ste.h, Q, Kk, V, O, S, LSE=L, sel_idx=si, sel_logg=sl)
+    _check(gO, gL, gi, gl)
+    dQ, gq = guarded((B, H, N, d), torch.bfloat16)
+    dK, gk = guarded((B, Hkv, N, d), torch.bfloat16)
+    dV, gv = guarded((B, Hkv, N, d), torch.bfloat16)
+    dl, gdl = guarded((B, Hkv, N, C), torch.float32)
+    ds, gds = guarded((B, Hkv, N, C), torch.float32)
+    sas.sas_attention_bwd(ste.h, Q, Kk, V, O, L, dO, dQ, dK, dV, S, si, sl, dl, ds)
+    _check(gq, gk, gv, gdl, gds)
+    assert sas.sas_get_device_status(ste.h) == 0
+    ste.close()
 
 
 def test_varlen_outputs():
