@@ -21,6 +21,10 @@ gate gradient and the sparse-scope score gradient):
   constant of the forward):
     ds_m = dlogg_m [m kept] - g_m sum_{l kept} dlogg_l,   m < C_i
   (from ds_m = g_m (dg_m - sum_l g_l dg_l) with dg_l = 0 for dropped blocks).
+  Other gate activations of Sec. 4.2 (inner position): the gates are
+  independent of one another, so only kept blocks get a score gradient,
+  ds_m = dlogg_m d(log g_m)/ds_m: sigmoid, dlogg_m (1 - g_m); raw logit
+  (log g = s), dlogg_m.
 
 Selection (which blocks are kept) is taken from the forward: the gradient
 treats it as fixed, as the kernels do.
@@ -52,11 +56,13 @@ import math
 
 import numpy as np
 
-from oracle.sas_oracle import _row_keys_and_bias, historical_count, log_gates, MODE_INFER_HARD, MODE_TRAIN_SOFT
+from oracle.sas_oracle import (GATE_LOGIT, GATE_SIGMOID, GATE_SOFTMAX, MODE_INFER_HARD, MODE_TRAIN_SOFT,
+                               _row_keys_and_bias, historical_count, log_gates)
 
 
-def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
-    """Gradients of one head's SAS forward (inner softmax gates).
+def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX):
+    """Gradients of one head's SAS forward (gates in the inner position, gate
+    activation `act`).
 
     Q, K, V, dO: [N, d]; s: [N, >=C-1] selector scores (row i reads s[i, :C_i]).
     Returns dict with dQ, dK, dV [N, d], dlogg [N, topk] (aligned with the
@@ -74,7 +80,7 @@ def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_sca
     ds = np.zeros((N, C))
     Delta = np.zeros(N)
     for i in range(N):
-        keys, bias, weight, sel, _ = _row_keys_and_bias(i, s[i], b, topk, mode)
+        keys, bias, weight, sel, _ = _row_keys_and_bias(i, s[i], b, topk, mode, act)
         z = sm_scale * (K[keys] @ Q[i]) + bias
         w = np.exp(z - z.max())
         p = w / w.sum()
@@ -89,15 +95,24 @@ def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_sca
             continue
         # kept blocks come first in `keys`, b tokens each, in ascending order
         c = historical_count(i, b)
-        lg_all = log_gates(np.asarray(s[i][:c], dtype=np.float64))
+        lg_all = log_gates(np.asarray(s[i][:c], dtype=np.float64), act)
         dl = np.zeros(c)
         for e, m in enumerate(sel):
             dl[m] = dz[e * b:(e + 1) * b].sum()
             dlogg[i, e] = dl[m]
         if c:
-            g = np.exp(lg_all)
-            ds[i, :c] = dl - g * dl.sum()
+            ds[i, :c] = _score_grad(dl, lg_all, act)
     return {"dQ": dQ, "dK": dK, "dV": dV, "dlogg": dlogg[:, :topk], "ds": ds, "Delta": Delta}
+
+
+def _score_grad(dl, lg, act):
+    """ds over a row's history from dlogg (0 on dropped blocks) and log g."""
+    g = np.exp(lg)
+    if act == GATE_SIGMOID:
+        return dl * (1.0 - g)
+    if act == GATE_LOGIT:
+        return dl.copy()
+    return dl - g * dl.sum()
 
 
 def backward_flops_head(N, b, topk, d, sel_counts=None):
@@ -113,7 +128,7 @@ def backward_flops_head(N, b, topk, d, sel_counts=None):
     return 10 * d * pairs
 
 
-def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None):
+def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX):
     """Gradients of the GQA forward (group-shared selection, Sec. 5.3) of one
     batch element.  Q, dO: [Hq, N, d]; K, V: [Hkv, N, d]; s: [Hkv, N, >=C-1];
     Hq = G Hkv, query head h uses group h // G.  A group's K, V and log-gates
@@ -137,7 +152,7 @@ def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scal
     ds = np.zeros((Hkv, N, C))
     for h in range(Hq):
         g = h // G
-        r = sas_attention_bwd_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, mode, sm_scale)
+        r = sas_attention_bwd_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, mode, sm_scale, act)
         dQ[h] = r["dQ"]
         dK[g] += r["dK"]
         dV[g] += r["dV"]
@@ -148,12 +163,11 @@ def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scal
                 c = historical_count(i, b)
                 if c == 0:
                     continue
-                _, _, _, sel, _ = _row_keys_and_bias(i, s[g, i], b, topk, mode)
+                _, _, _, sel, _ = _row_keys_and_bias(i, s[g, i], b, topk, mode, act)
                 dl = np.zeros(c)
                 for e, m in enumerate(sel):
                     dl[m] = dlogg[g, i, e]
-                gates = np.exp(log_gates(np.asarray(s[g, i][:c], dtype=np.float64)))
-                ds[g, i, :c] = dl - gates * dl.sum()
+                ds[g, i, :c] = _score_grad(dl, log_gates(np.asarray(s[g, i][:c], dtype=np.float64), act), act)
     return {"dQ": dQ, "dK": dK, "dV": dV, "dlogg": dlogg, "ds": ds}
 
 

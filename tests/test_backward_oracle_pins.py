@@ -20,9 +20,10 @@ def _inputs(N, d, seed, C=None):
     return Q, K, V, dO, s
 
 
-def _torch_dense(Q, K, V, s, b, topk, sm_scale):
-    """Dense masked attention whose bias on kept blocks is log_softmax(s) over
-    the row's history; autograd gives dQ, dK, dV and ds."""
+def _torch_dense(Q, K, V, s, b, topk, sm_scale, act=O.GATE_SOFTMAX):
+    """Dense masked attention whose bias on kept blocks is log g of the gate
+    activation (softmax: log_softmax(s) over the row's history; sigmoid:
+    logsigmoid(s); raw logit: s); autograd gives dQ, dK, dV and ds."""
     N, d = Q.shape
     t = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
     q, k, v, st = t(Q), t(K), t(V), t(s)
@@ -31,7 +32,12 @@ def _torch_dense(Q, K, V, s, b, topk, sm_scale):
         c = i // b
         bias = torch.full((N,), -math.inf, dtype=torch.float64)
         if c:
-            lg = torch.log_softmax(st[i, :c], dim=0)
+            if act == O.GATE_SIGMOID:
+                lg = torch.nn.functional.logsigmoid(st[i, :c])
+            elif act == O.GATE_LOGIT:
+                lg = st[i, :c]
+            else:
+                lg = torch.log_softmax(st[i, :c], dim=0)
             sel = O.topk_blocks(s[i, :c], topk)
             bias = bias.clone()
             for m in sel:
@@ -332,3 +338,29 @@ def test_ste_gqa_is_the_sum_over_heads():
                 gt = np.exp(O.log_gates(s[g, i, :c]))
                 dgi = r["dg"][g, i, :c]
                 assert np.allclose(r["ds"][g, i, :c], gt * (dgi - (gt * dgi).sum()), atol=1e-13)
+
+
+# ------------------------------------------- other gate activations (inner)
+
+@pytest.mark.parametrize("act", [O.GATE_SIGMOID, O.GATE_LOGIT])
+@pytest.mark.parametrize("N,topk,seed", [(37, 2, 51), (50, 3, 52)])
+def test_other_activations_backward_equals_autograd(act, N, topk, seed):
+    # Sec. 4.2 gate activation: independent gates, so only kept blocks get a
+    # score gradient, through d log g / ds (sigmoid: 1 - g; raw logit: 1)
+    b, d = 8, 5
+    Q, K, V, dO, s = _inputs(N, d, seed)
+    sm = 1 / math.sqrt(d)
+    q, k, v, st, Ot = _torch_dense(Q, K, V, s, b, topk, sm, act)
+    assert np.allclose(Ot.detach().numpy(), O.sas_attention_head(Q, K, V, s, b, topk, act=act)["O"], atol=1e-12)
+    (Ot * torch.tensor(dO)).sum().backward()
+    r = BO.sas_attention_bwd_head(Q, K, V, s, dO, b, topk, act=act)
+    assert np.allclose(r["dQ"], q.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dK"], k.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dV"], v.grad.numpy(), atol=1e-12)
+    C = r["ds"].shape[1]
+    assert np.allclose(r["ds"], st.grad.numpy()[:, :C], atol=1e-12)
+    # dropped blocks get none, unlike the softmax gates
+    for i in range(N):
+        c = i // b
+        dropped = np.setdiff1d(np.arange(c), O.topk_blocks(s[i, :c], topk))
+        assert np.all(r["ds"][i, dropped] == 0)
