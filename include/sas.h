@@ -198,7 +198,8 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
                                    void* stream);
 
 /* Backward of sas_attention_fwd (Alg. 4 of App. E; gate and score gradients
- * of App. D), for d = 128, softmax gates in the inner position, any mode.
+ * of App. D), for d = 128, gates in the inner position (any activation), any
+ * mode.
  * The kept sets are those of the forward (the Top-K choice is a constant of
  * the backward), and the per-tile block lists are read from the handle: call
  * it after the sas_attention_fwd of the same inputs on this handle, with no
@@ -249,7 +250,9 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
  *              by block for the full scope and hard-STE; may be NULL     (out)
  *   dscores    fp32 [B, Hkv, N, C] dL/ds of the given scores, sparse scope:
  *              ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, 0 past each
- *              row's history; SCORES_GIVEN handles only, else NULL.
+ *              row's history (sigmoid gates: dlogg_m (1 - g_m) [m kept];
+ *              raw logits: dlogg_m [m kept]); SCORES_GIVEN handles only,
+ *              else NULL.
  *              g_m = exp(s_m - LSE_i) takes the row's log-normaliser
  *              LSE_i = s_m - log g_m from its first kept entry, so the
  *              scores must be the ones the forward selected with     (out)

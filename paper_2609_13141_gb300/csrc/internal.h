@@ -229,6 +229,7 @@ struct AttnBwdArgs {
     // pass 1 and the gate gradients only (no pass 2; dQ and offs may be null): the
     // gate pass of the hard Top-K gate under the straight-through estimator
     bool gate_only;
+    int act;                    // gate activation (sas_gate_act) of the score gradient
 };
 extern const int kBwdMaxTiles;   // query tiles per head the backward supports (head-packed: segments + G)
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total);

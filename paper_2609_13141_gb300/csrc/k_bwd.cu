@@ -1028,7 +1028,10 @@ __global__ void __launch_bounds__(256) bwd_dense_unions_kernel(int32_t* uidx, in
 // --------------------------------------------------------- score gradient
 
 // ds_m = dlogg_m [m kept] - g_m sum_kept dlogg, g = softmax of the row's C_i
-// given scores; 0 past the history.  One warp per row, every load of the row
+// given scores; 0 past the history.  The other gate activations have
+// independent gates: ds_m = dlogg_m d(log g_m)/ds_m on kept blocks only
+// (act 1, sigmoid: dlogg_m (1 - g_m) = -dlogg_m expm1(log g_m); act 2, raw
+// logit: dlogg_m).  One warp per row, every load of the row
 // issued first (the row's scores are held in registers when C <= 32 NCH):
 // the log-normaliser comes back from the first kept entry (log g_m = s_m -
 // LSE of the scores, Eq. normalized_log_gate), the kept dlogg values are
@@ -1036,7 +1039,7 @@ __global__ void __launch_bounds__(256) bwd_dense_unions_kernel(int32_t* uidx, in
 template <int NCH>
 __global__ void __launch_bounds__(256)
 bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg, const float* dlogg, float* ds,
-              int N, int C, int topk, int train, int chunks, const int4* tiles, const int* ntiles) {
+              int N, int C, int topk, int train, int act, int chunks, const int4* tiles, const int* ntiles) {
     extern __shared__ float dsh[];   // per warp: C floats (the row's kept dlogg, scattered)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // CTA = (head, run of blockDim / 32 rows of it): one division per CTA.
@@ -1075,19 +1078,23 @@ bwd_ds_kernel(const float* scores, const int32_t* sel_idx, const float* sel_logg
     }
     const int32_t* ix = sel_idx + w * topk;
     const float* dl = dlogg + w * topk;
-    const float v0 = lane < nsel ? __ldg(dl + lane) : 0.f;
+    // a kept entry's d(log g)/ds: sigmoid 1 - g, else 1 (softmax couples through the sum below)
+    const float* lgr = sel_logg + w * topk;
+    auto dlds = [&](int e) { return act == 1 ? -expm1f(__ldg(lgr + e)) : 1.f; };
+    const float v0 = lane < nsel ? __ldg(dl + lane) * dlds(lane) : 0.f;
     const int i0 = lane < nsel ? __ldg(ix + lane) : 0;
-    const float lg0 = nsel > 0 ? __ldg(sel_logg + w * topk) : 0.f;
+    const float lg0 = nsel > 0 ? __ldg(lgr) : 0.f;
     for (int m = lane; m < C; m += 32) add[m] = 0.f;
     __syncwarp();
     float sum = v0;
     if (lane < nsel) add[i0] = v0;   // kept blocks are distinct
     for (int e = lane + 32; e < nsel; e += 32) {
-        const float v = __ldg(dl + e);
+        const float v = __ldg(dl + e) * dlds(e);
         sum += v;
         add[__ldg(ix + e)] = v;
     }
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (act != 0) sum = 0.f;   // independent gates: no coupling term
     // LSE = s_m0 - log g_m0 for the first kept block m0 (< c, so in registers)
     const int m0 = __shfl_sync(0xffffffffu, i0, 0);
     float s0;
@@ -1284,13 +1291,13 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         const int train = a.mode == 0 ? 1 : 0;
         if (a.C <= 128)
             bwd_ds_kernel<4><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                 a.C, a.topk, train, chunks, a.tiles, a.ntiles);
+                                                                 a.C, a.topk, train, a.act, chunks, a.tiles, a.ntiles);
         else if (a.C <= 384)
             bwd_ds_kernel<12><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                  a.C, a.topk, train, chunks, a.tiles, a.ntiles);
+                                                                  a.C, a.topk, train, a.act, chunks, a.tiles, a.ntiles);
         else
             bwd_ds_kernel<0><<<grid, 32 * wpc, sh, env.stream>>>(a.scores, a.sel_idx, a.sel_logg, a.dlogg, a.ds, a.N,
-                                                                 a.C, a.topk, train, chunks, a.tiles, a.ntiles);
+                                                                 a.C, a.topk, train, a.act, chunks, a.tiles, a.ntiles);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward score gradient"; return e; }
     } else if (a.ds != nullptr) {

@@ -120,7 +120,7 @@ def outer_logit_extra(Q, K, V, s, b, topk, mode, rows, act, pos):
     return 2.0 ** -8 * A
 
 
-def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None):
+def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None, act=OR.GATE_SOFTMAX):
     """Derived extra bounds for the backward's dQ, dK, dV of one head.
 
     dV_j = sum_i P_ij dO_i, dK_j = scale sum_i dS_ij q_i and dQ_i = scale sum_j
@@ -138,7 +138,7 @@ def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None):
     N, d = Q.shape
     if sm_scale is None:
         sm_scale = 1.0 / math.sqrt(d)
-    P = OR.sas_attention_materialized(Q, K, V, s, b, topk, mode, sm_scale)["P"]
+    P = OR.sas_attention_materialized(Q, K, V, s, b, topk, mode, sm_scale, act=act)["P"]
     dP = dO @ V.T
     Delta = (P * dP).sum(axis=1)
     dS = P * (dP - Delta[:, None])
