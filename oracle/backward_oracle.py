@@ -21,6 +21,10 @@ gate gradient and the sparse-scope score gradient):
   constant of the forward):
     ds_m = dlogg_m [m kept] - g_m sum_{l kept} dlogg_l,   m < C_i
   (from ds_m = g_m (dg_m - sum_l g_l dg_l) with dg_l = 0 for dropped blocks).
+  Outer gate position (Sec. 4.2 gate position, o = softmax(z) (g . V) with
+  z unbiased and w_j = g of key j's block, 1 on the current block):
+    dV_j += p_j w_j dO_i,  dz_j = p_j (w_j dp_j - Delta_i)  (Delta_i = dO_i . o_i),
+    dlogg_m = sum_{j in B_m} p_j w_j dp_j   (= g_m dL/dg_m).
   Other gate activations of Sec. 4.2 (inner position): the gates are
   independent of one another, so only kept blocks get a score gradient,
   ds_m = dlogg_m d(log g_m)/ds_m: sigmoid, dlogg_m (1 - g_m); raw logit
@@ -56,13 +60,14 @@ import math
 
 import numpy as np
 
-from oracle.sas_oracle import (GATE_LOGIT, GATE_SIGMOID, GATE_SOFTMAX, MODE_INFER_HARD, MODE_TRAIN_SOFT,
-                               _row_keys_and_bias, historical_count, log_gates)
+from oracle.sas_oracle import (GATE_INNER, GATE_LOGIT, GATE_SIGMOID, GATE_SOFTMAX, MODE_INFER_HARD,
+                               MODE_TRAIN_SOFT, _row_keys_and_bias, historical_count, log_gates)
 
 
-def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX):
-    """Gradients of one head's SAS forward (gates in the inner position, gate
-    activation `act`).
+def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX,
+                           pos=GATE_INNER):
+    """Gradients of one head's SAS forward (gate activation `act`, gate
+    position `pos`).
 
     Q, K, V, dO: [N, d]; s: [N, >=C-1] selector scores (row i reads s[i, :C_i]).
     Returns dict with dQ, dK, dV [N, d], dlogg [N, topk] (aligned with the
@@ -80,17 +85,19 @@ def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_sca
     ds = np.zeros((N, C))
     Delta = np.zeros(N)
     for i in range(N):
-        keys, bias, weight, sel, _ = _row_keys_and_bias(i, s[i], b, topk, mode, act)
+        keys, bias, weight, sel, _ = _row_keys_and_bias(i, s[i], b, topk, mode, act, pos)
         z = sm_scale * (K[keys] @ Q[i]) + bias
-        w = np.exp(z - z.max())
-        p = w / w.sum()
-        o = p @ V[keys]
+        ez = np.exp(z - z.max())
+        p = ez / ez.sum()
+        o = (p * weight) @ V[keys]
         dp = V[keys] @ dO[i]
         Delta[i] = dO[i] @ o
-        dz = p * (dp - Delta[i])
+        dz = p * (weight * dp - Delta[i])
         dQ[i] = sm_scale * (dz @ K[keys])
         np.add.at(dK, keys, sm_scale * np.outer(dz, Q[i]))
-        np.add.at(dV, keys, np.outer(p, dO[i]))
+        np.add.at(dV, keys, np.outer(p * weight, dO[i]))
+        # d(log g) of a block: the row sum of dz (inner), of p w dp (outer)
+        gsum = dz if pos == GATE_INNER else p * weight * dp
         if mode != MODE_TRAIN_SOFT:
             continue
         # kept blocks come first in `keys`, b tokens each, in ascending order
@@ -98,7 +105,7 @@ def sas_attention_bwd_head(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_sca
         lg_all = log_gates(np.asarray(s[i][:c], dtype=np.float64), act)
         dl = np.zeros(c)
         for e, m in enumerate(sel):
-            dl[m] = dz[e * b:(e + 1) * b].sum()
+            dl[m] = gsum[e * b:(e + 1) * b].sum()
             dlogg[i, e] = dl[m]
         if c:
             ds[i, :c] = _score_grad(dl, lg_all, act)
@@ -128,7 +135,8 @@ def backward_flops_head(N, b, topk, d, sel_counts=None):
     return 10 * d * pairs
 
 
-def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX):
+def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None, act=GATE_SOFTMAX,
+                          pos=GATE_INNER):
     """Gradients of the GQA forward (group-shared selection, Sec. 5.3) of one
     batch element.  Q, dO: [Hq, N, d]; K, V: [Hkv, N, d]; s: [Hkv, N, >=C-1];
     Hq = G Hkv, query head h uses group h // G.  A group's K, V and log-gates
@@ -152,7 +160,7 @@ def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scal
     ds = np.zeros((Hkv, N, C))
     for h in range(Hq):
         g = h // G
-        r = sas_attention_bwd_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, mode, sm_scale, act)
+        r = sas_attention_bwd_head(Q[h], K[g], V[g], s[g], dO[h], b, topk, mode, sm_scale, act, pos)
         dQ[h] = r["dQ"]
         dK[g] += r["dK"]
         dV[g] += r["dV"]
@@ -163,7 +171,7 @@ def sas_attention_bwd_gqa(Q, K, V, s, dO, b, topk, mode=MODE_TRAIN_SOFT, sm_scal
                 c = historical_count(i, b)
                 if c == 0:
                     continue
-                _, _, _, sel, _ = _row_keys_and_bias(i, s[g, i], b, topk, mode, act)
+                _, _, _, sel, _ = _row_keys_and_bias(i, s[g, i], b, topk, mode, act, pos)
                 dl = np.zeros(c)
                 for e, m in enumerate(sel):
                     dl[m] = dlogg[g, i, e]

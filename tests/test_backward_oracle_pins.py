@@ -364,3 +364,42 @@ def test_other_activations_backward_equals_autograd(act, N, topk, seed):
         c = i // b
         dropped = np.setdiff1d(np.arange(c), O.topk_blocks(s[i, :c], topk))
         assert np.all(r["ds"][i, dropped] == 0)
+
+
+# ------------------------------------------------------- outer gate position
+
+@pytest.mark.parametrize("act", [O.GATE_SOFTMAX, O.GATE_SIGMOID])
+@pytest.mark.parametrize("N,topk,seed", [(37, 2, 61), (45, 3, 62)])
+def test_outer_position_backward_equals_autograd(act, N, topk, seed):
+    # Sec. 4.2 gate position: o = softmax(z) (g . V), z unbiased, each kept
+    # block's value rows scaled by its gate (the current block by 1)
+    b, d = 8, 5
+    Q, K, V, dO, s = _inputs(N, d, seed)
+    sm = 1 / math.sqrt(d)
+    t = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
+    q, k, v, st = t(Q), t(K), t(V), t(s)
+    outs = []
+    for i in range(N):
+        c = i // b
+        mask = torch.full((N,), -math.inf, dtype=torch.float64)
+        wts = torch.zeros(N, dtype=torch.float64)
+        if c:
+            lg = torch.nn.functional.logsigmoid(st[i, :c]) if act == O.GATE_SIGMOID else torch.log_softmax(st[i, :c], 0)
+            for m in O.topk_blocks(s[i, :c], topk):
+                mask = torch.cat([mask[:m * b], torch.zeros(b, dtype=torch.float64), mask[(m + 1) * b:]])
+                wts = torch.cat([wts[:m * b], torch.exp(lg[m]).expand(b), wts[(m + 1) * b:]])
+        mask = torch.cat([mask[:c * b], torch.zeros(i + 1 - c * b, dtype=torch.float64), mask[i + 1:]])
+        wts = torch.cat([wts[:c * b], torch.ones(i + 1 - c * b, dtype=torch.float64), wts[i + 1:]])
+        p = torch.softmax(sm * k @ q[i] + mask, dim=0)
+        outs.append((p * wts) @ v)
+    Ot = torch.stack(outs)
+    fwd = O.sas_attention_head(Q, K, V, s, b, topk, act=act, pos=O.GATE_OUTER)
+    assert np.allclose(Ot.detach().numpy(), fwd["O"], atol=1e-12)
+    (Ot * torch.tensor(dO)).sum().backward()
+    r = BO.sas_attention_bwd_head(Q, K, V, s, dO, b, topk, act=act, pos=O.GATE_OUTER)
+    assert np.allclose(r["dQ"], q.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dK"], k.grad.numpy(), atol=1e-12)
+    assert np.allclose(r["dV"], v.grad.numpy(), atol=1e-12)
+    C = r["ds"].shape[1]
+    assert np.allclose(r["ds"], st.grad.numpy()[:, :C], atol=1e-12)
+    assert np.allclose(r["Delta"], (fwd["O"] * dO).sum(axis=1), atol=1e-13)
