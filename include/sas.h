@@ -198,8 +198,9 @@ sas_status sas_attention_fwd_noisy(sas_handle* h,
                                    void* stream);
 
 /* Backward of sas_attention_fwd (Alg. 4 of App. E; gate and score gradients
- * of App. D), for d = 128, gates in the inner position (any activation), any
- * mode.
+ * of App. D), for d = 128, any gate activation and position, any mode.  In
+ * the outer position (o = softmax(z) (g . V)) dV takes P g dO, dS = P (g dP -
+ * Delta), and a block's dlogg is the row sum of P g dP.
  * The kept sets are those of the forward (the Top-K choice is a constant of
  * the backward), and the per-tile block lists are read from the handle: call
  * it after the sas_attention_fwd of the same inputs on this handle, with no

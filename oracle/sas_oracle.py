@@ -283,7 +283,7 @@ def sas_attention_materialized(Q, K, V, s, b, topk, mode=MODE_TRAIN_SOFT,
     zmax = Z.max(axis=1, keepdims=True)
     W = np.exp(Z - zmax)
     l = W.sum(axis=1, keepdims=True)
-    return {"O": (W * gate @ V) / l, "LSE": (zmax + np.log(l))[:, 0], "P": W / l}
+    return {"O": (W * gate @ V) / l, "LSE": (zmax + np.log(l))[:, 0], "P": W / l, "gate": gate}
 
 
 def sas_attention(Q, K, V, b, topk, mode=MODE_TRAIN_SOFT, sm_scale=None,

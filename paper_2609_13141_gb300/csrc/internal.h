@@ -230,6 +230,7 @@ struct AttnBwdArgs {
     // gate pass of the hard Top-K gate under the straight-through estimator
     bool gate_only;
     int act;                    // gate activation (sas_gate_act) of the score gradient
+    int pos;                    // gate position (sas_gate_pos): 1 = outer, o = softmax(z) (g . V)
 };
 extern const int kBwdMaxTiles;   // query tiles per head the backward supports (head-packed: segments + G)
 cudaError_t launch_bwd_slots(const AttnBwdArgs& a, const KernelEnv& env, long long* total);

@@ -171,7 +171,7 @@ __device__ __forceinline__ BwdTile bwd_seg(const BwdParams& p, int sg) {
     return {t * p.seg_rows < v.z ? t : -1, v.x, v.z};
 }
 
-template <bool HP>
+template <bool HP, bool OUTER>
 __global__ void __launch_bounds__(kThreadsB, 1)
 bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
               const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapV, BwdParams p) {
@@ -397,12 +397,17 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                 tmem_ld32(lane_addr + kTmemDP + (j & 1) * 128 + hk * 32, dv);
                 tmem_wait_ld();
                 // P = exp2(S scale + (log g - LSE)) in log2 units; exp2(-inf) = 0 for a
-                // block the row does not attend; the causal limit only on its own block
-                const float boff = lim >= 0 ? bias - lse2 : -CUDART_INF_F;
+                // block the row does not attend; the causal limit only on its own block.
+                // Outer gate position: P is the plain softmax (no bias) and the block's
+                // gate w multiplies dP: dS = P (w dP - Delta); pass 2 gets w (-1: not
+                // attended) in place of the offset
+                const float boff = lim >= 0 ? (OUTER ? -lse2 : bias - lse2) : -CUDART_INF_F;
+                const float wg = OUTER ? fast_exp2(bias) : 1.f;
                 const bool causal = lim >= 0 && lim < kKeys - 1;
-                if (hk == 0 && p.offs != nullptr) p.offs[(static_cast<long long>(slot0) + j) * kRows + r] = boff;
+                if (hk == 0 && p.offs != nullptr)
+                    p.offs[(static_cast<long long>(slot0) + j) * kRows + r] = OUTER ? (lim >= 0 ? wg : -1.f) : boff;
                 const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2), bo2 = f32x2(boff, boff);
-                const uint64_t nd2 = f32x2(-delta, -delta);
+                const uint64_t nd2 = f32x2(-delta, -delta), w2 = f32x2(wg, wg);
                 uint64_t acc = 0;
                 uint32_t pk[16];
 #pragma unroll
@@ -414,16 +419,18 @@ bwd_dq_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ 
                         p0 = hk * 32 + k <= lim ? p0 : 0.f;
                         p1 = hk * 32 + k + 1 <= lim ? p1 : 0.f;
                     }
-                    const uint64_t d2 = add_f32x2(f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1])), nd2);
+                    const uint64_t dv2 = f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1]));
+                    const uint64_t d2 = OUTER ? fma_f32x2(dv2, w2, nd2) : add_f32x2(dv2, nd2);
                     const uint64_t ds2 = fma_f32x2(f32x2(p0, p1), d2, 0ull);
-                    acc = add_f32x2(acc, ds2);
+                    // the block's d(log g): row sum of dS (inner), w times that of P dP (outer)
+                    acc = OUTER ? fma_f32x2(f32x2(p0, p1), dv2, acc) : add_f32x2(acc, ds2);
                     float a0, a1;
                     f32x2_split(ds2, a0, a1);
                     pk[k >> 1] = pack_bf16x2(a0, a1);
                 }
                 float s0, s1;
                 f32x2_split(acc, s0, s1);
-                sum = s0 + s1;
+                sum = OUTER ? wg * (s0 + s1) : s0 + s1;
                 tmem_st16(lane_addr + kTmemDS + (j & 1) * 32 + hk * 16, pk);
             }
             tmem_wait_st();
@@ -648,7 +655,7 @@ constexpr int kDkvSmem = kDkvOffCtl + 256 + 1024;
 // over the first 32 columns of the S^T (dP^T) they have read.
 constexpr uint32_t kTmemDV = 0, kTmemDK = 128, kTmemBuf = 256, kTmemST = 0, kTmemDPT = 64;
 
-template <bool HP>
+template <bool HP, bool OUTER>
 __global__ void __launch_bounds__(kThreadsD, 1)
 bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapDO,
                const __grid_constant__ CUtensorMap mapK2, const __grid_constant__ CUtensorMap mapV2, BwdParams p) {
@@ -783,9 +790,12 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
                 const int hr = hp ? r / p.seg_rows : 0;
                 const int i = hp ? tq * p.seg_rows + (r - hr * p.seg_rows) : tq * kRows + r;
                 const long long drow = static_cast<long long>(hp ? kv * p.G + hr : bhq) * p.N + ptg.base + i;
-                inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : -CUDART_INF_F;
-                inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : -CUDART_INF_F;
+                // outer gate position: the blocks' gates w (-1: not attended) and -LSE
+                const float kAbsent = OUTER ? -1.f : -CUDART_INF_F;
+                inf[r] = j0 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j0) * kRows + r) : kAbsent;
+                inf[kRows + r] = j1 >= 0 ? __ldcg(p.offs + so + static_cast<long long>(j1) * kRows + r) : kAbsent;
                 inf[2 * kRows + r] = i < ptg.n ? -__ldcg(p.delta + drow) : 0.f;
+                if (OUTER) inf[3 * kRows + r] = i < ptg.n ? -__ldg(p.LSE + drow) * kLog2eB : -CUDART_INF_F;
             }
             mbar_arrive_warp(&ctl.info_full[s]);
         }
@@ -930,23 +940,33 @@ bwd_dkv_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__
             }
             const float2* off2 = reinterpret_cast<const float2*>(inf + kblk * kRows + h * 64);
             const float2* nd2p = reinterpret_cast<const float2*>(inf + 2 * kRows + h * 64);
+            const float2* ul2p = reinterpret_cast<const float2*>(inf + 3 * kRows + h * 64);   // outer: -LSE
             const uint64_t sc2 = f32x2(p.scale_log2, p.scale_log2);
             const int kin = key & 63;
 #pragma unroll
             for (int k = 0; k < 64; k += 2) {
+                // inner: o = the offset (log g - LSE); outer: o = the gate w (-1: not
+                // attended), P unweighted from -LSE, P^T = P w, dS^T = P (w dP - Delta)
                 const float2 o = off2[k >> 1], nd = nd2p[k >> 1];
+                const float2 zo = OUTER ? ul2p[k >> 1] : o;
                 float z0, z1;
-                f32x2_split(fma_f32x2(f32x2(__uint_as_float(sv[k]), __uint_as_float(sv[k + 1])), sc2, f32x2(o.x, o.y)),
+                f32x2_split(fma_f32x2(f32x2(__uint_as_float(sv[k]), __uint_as_float(sv[k + 1])), sc2, f32x2(zo.x, zo.y)),
                             z0, z1);
                 float p0 = fast_exp2(z0), p1 = fast_exp2(z1);
+                if (OUTER) {
+                    p0 = o.x >= 0.f ? p0 : 0.f;
+                    p1 = o.y >= 0.f ? p1 : 0.f;
+                }
                 if (causal) {
                     p0 = kin <= toff0 + (k & rmask) ? p0 : 0.f;
                     p1 = kin <= toff0 + ((k + 1) & rmask) ? p1 : 0.f;
                 }
-                const uint64_t d2 = add_f32x2(f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1])), f32x2(nd.x, nd.y));
+                const uint64_t dv2 = f32x2(__uint_as_float(dv[k]), __uint_as_float(dv[k + 1]));
+                const uint64_t d2 = OUTER ? fma_f32x2(dv2, f32x2(o.x, o.y), f32x2(nd.x, nd.y))
+                                          : add_f32x2(dv2, f32x2(nd.x, nd.y));
                 float a0, a1;
                 f32x2_split(fma_f32x2(f32x2(p0, p1), d2, 0ull), a0, a1);
-                pp[k >> 1] = pack_bf16x2(p0, p1);
+                pp[k >> 1] = OUTER ? pack_bf16x2(p0 * o.x, p1 * o.y) : pack_bf16x2(p0, p1);
                 dd[k >> 1] = pack_bf16x2(a0, a1);
             }
             // P^T and dS^T over the S^T and dP^T columns just read
@@ -1186,10 +1206,19 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     }
     const int BHkv = a.BH / G;   // KV groups x batch
     {
-        cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel<false>), kDqSmem);
-        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel<false>), kDkvSmem);
-        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dq_kernel<true>), kDqSmem);
-        if (e == cudaSuccess) e = ensure_smem_attr(reinterpret_cast<const void*>(bwd_dkv_kernel<true>), kDkvSmem);
+        const void* dq[4] = {reinterpret_cast<const void*>(bwd_dq_kernel<false, false>),
+                             reinterpret_cast<const void*>(bwd_dq_kernel<true, false>),
+                             reinterpret_cast<const void*>(bwd_dq_kernel<false, true>),
+                             reinterpret_cast<const void*>(bwd_dq_kernel<true, true>)};
+        const void* dkv[4] = {reinterpret_cast<const void*>(bwd_dkv_kernel<false, false>),
+                              reinterpret_cast<const void*>(bwd_dkv_kernel<true, false>),
+                              reinterpret_cast<const void*>(bwd_dkv_kernel<false, true>),
+                              reinterpret_cast<const void*>(bwd_dkv_kernel<true, true>)};
+        cudaError_t e = cudaSuccess;
+        for (int v = 0; v < 4 && e == cudaSuccess; ++v) {
+            e = ensure_smem_attr(dq[v], kDqSmem);
+            if (e == cudaSuccess) e = ensure_smem_attr(dkv[v], kDkvSmem);
+        }
         if (e != cudaSuccess) { *err = "cudaFuncSetAttribute(bwd)"; return e; }
     }
     CUtensorMap mq, mdo, mk, mv, mk2, mv2;
@@ -1245,8 +1274,15 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
     const long long per_head = static_cast<long long>(a.N) * (a.topk > 0 ? a.topk : 1);
     cudaError_t e0 = cudaMemsetAsync(p.dlogg, 0, static_cast<size_t>(a.BH) * per_head * 4, env.stream);
     if (e0 != cudaSuccess) { *err = "backward dlogg"; return e0; }
-    if (hp) bwd_dq_kernel<true><<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
-    else bwd_dq_kernel<false><<<static_cast<unsigned>(tiles), kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+    // outer gate position with gates (training mode); without gates it is the inner form
+    const bool outer = a.pos == 1 && a.mode == 0;
+    {
+        const dim3 g1(static_cast<unsigned>(tiles));
+        if (hp && outer) bwd_dq_kernel<true, true><<<g1, kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+        else if (hp) bwd_dq_kernel<true, false><<<g1, kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+        else if (outer) bwd_dq_kernel<false, true><<<g1, kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+        else bwd_dq_kernel<false, false><<<g1, kThreadsB, kDqSmem, env.stream>>>(mq, mdo, mk, mv, p);
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) { *err = "backward pass 1"; return e; }
     if (!a.gate_only) {   // a gate-only pass (the STE gate gradient) has no pass 2
@@ -1265,8 +1301,11 @@ cudaError_t launch_attn_bwd(const AttnBwdArgs& a, const KernelEnv& env, const ch
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward inverted lists"; return e; }
         // pass 2: one CTA per (KV group, key pair)
-        if (hp) bwd_dkv_kernel<true><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
-        else bwd_dkv_kernel<false><<<static_cast<unsigned>(gtiles), kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        const dim3 g2(static_cast<unsigned>(gtiles));
+        if (hp && outer) bwd_dkv_kernel<true, true><<<g2, kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        else if (hp) bwd_dkv_kernel<true, false><<<g2, kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        else if (outer) bwd_dkv_kernel<false, true><<<g2, kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
+        else bwd_dkv_kernel<false, false><<<g2, kThreadsD, kDkvSmem, env.stream>>>(mq, mdo, mk2, mv2, p);
         e = cudaGetLastError();
         if (e != cudaSuccess) { *err = "backward pass 2"; return e; }
     }

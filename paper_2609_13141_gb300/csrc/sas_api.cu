@@ -655,8 +655,6 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
         (scores && !aligned4(scores)))
         return fail(h, SAS_ERR_INVALID_ARG, "misaligned pointer");
     if (c.d != 128) return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports d = 128");
-    if (c.gate_pos != SAS_GATE_INNER)
-        return fail(h, SAS_ERR_UNSUPPORTED, "the backward supports gates in the inner position");
     // the full scope and the hard gate's estimator gate every historical block
     const bool ste = c.mode == SAS_MODE_TRAIN_HARD_STE;
     const bool dense = h->full || ste;
@@ -754,6 +752,7 @@ sas_status sas_attention_bwd(sas_handle* h, const void* Q, const void* K, const 
     a.N = c.N; a.C = h->C; a.T = h->T; a.BH = h->BH; a.topk = c.topk; a.mode = c.mode; a.d = c.d;
     a.G = h->G;
     a.act = c.gate_act;
+    a.pos = c.gate_pos;
     a.sm_scale = h->sm_scale;
     if (h->varlen) {
         // the tile table of the last sas_attention_fwd_varlen (its union lists are per slot)

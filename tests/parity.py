@@ -120,7 +120,7 @@ def outer_logit_extra(Q, K, V, s, b, topk, mode, rows, act, pos):
     return 2.0 ** -8 * A
 
 
-def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None, act=OR.GATE_SOFTMAX):
+def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None, act=OR.GATE_SOFTMAX, pos=OR.GATE_INNER):
     """Derived extra bounds for the backward's dQ, dK, dV of one head.
 
     dV_j = sum_i P_ij dO_i, dK_j = scale sum_i dS_ij q_i and dQ_i = scale sum_j
@@ -134,22 +134,25 @@ def grad_extra(Q, K, V, s, dO, O_gpu, b, topk, mode, sm_scale=None, act=OR.GATE_
       dQ: scale E_S |K| + 2^-9 |dQ|,   dK: scale E_S^T |Q| + 2^-9 |dK|,
       dV: 2^-9 P^T |dO| + 2^-9 |dV|,
     each doubled to cover the second-order and fp32 terms.  P comes from the
-    oracle's materialised forward (Q, K, V [N, d]; s the head's scores)."""
+    oracle's materialised forward (Q, K, V [N, d]; s the head's scores).
+    Outer gate position: P is the plain softmax and each key carries its
+    block's gate w, so dV takes (P w)^T dO and dS = P (w dP - Delta)."""
     N, d = Q.shape
     if sm_scale is None:
         sm_scale = 1.0 / math.sqrt(d)
-    P = OR.sas_attention_materialized(Q, K, V, s, b, topk, mode, sm_scale, act=act)["P"]
+    mat = OR.sas_attention_materialized(Q, K, V, s, b, topk, mode, sm_scale, act=act, pos=pos)
+    P, W = mat["P"], mat["gate"]
     dP = dO @ V.T
-    Delta = (P * dP).sum(axis=1)
-    dS = P * (dP - Delta[:, None])
+    Delta = (P * W * dP).sum(axis=1)
+    dS = P * (W * dP - Delta[:, None])
     dDelta = 2.0 ** -8 * np.abs(dO * O_gpu).sum(axis=1)
     ES = 2.0 ** -9 * np.abs(dS) + P * dDelta[:, None]
     dQ = sm_scale * dS @ K
     dK = sm_scale * dS.T @ Q
-    dV = P.T @ dO
+    dV = (P * W).T @ dO
     return {"dQ": 2 * (sm_scale * ES @ np.abs(K) + 2.0 ** -9 * np.abs(dQ)),
             "dK": 2 * (sm_scale * ES.T @ np.abs(Q) + 2.0 ** -9 * np.abs(dK)),
-            "dV": 2 * (2.0 ** -9 * P.T @ np.abs(dO) + 2.0 ** -9 * np.abs(dV))}
+            "dV": 2 * (2.0 ** -9 * (P * W).T @ np.abs(dO) + 2.0 ** -9 * np.abs(dV))}
 
 
 def _flip_size(x, delta):

@@ -59,6 +59,9 @@ def test_status_strings(lib):
     (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, gate_pos=1), sas.SAS_ERR_UNSUPPORTED),   # full scope: inner only
     (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, gate_act=1), sas.SAS_ERR_UNSUPPORTED),   # full scope: softmax only
     (dict(B=1, H=2, N=128, d=64, topk=2, scope=1, max_seqs=2), sas.SAS_ERR_UNSUPPORTED),   # full scope: no packing
+    (dict(B=1, H=2, N=128, d=64, topk=2, mode=2, scope=1), sas.SAS_ERR_UNSUPPORTED),       # hard-STE: sparse scope
+    (dict(B=1, H=2, N=128, d=64, topk=2, mode=2, gate_act=1), sas.SAS_ERR_UNSUPPORTED),    # hard-STE: softmax gates
+    (dict(B=1, H=2, N=128, d=64, topk=2, mode=2, gate_pos=1), sas.SAS_ERR_UNSUPPORTED),    # hard-STE: inner position
 ])
 def test_create_rejects_bad_configs(lib, kw, expect):
     assert sas.sas_create_status(**kw) == expect

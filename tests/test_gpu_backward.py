@@ -21,7 +21,8 @@ def _delta_bound(O, dO):
     return 2.0 ** -8 * np.abs(P.f64(O) * P.f64(dO)).sum(axis=-1) + 1e-4
 
 
-def run_bwd(B, H, N, topk, mode, seed, learned=False, heads=None, rows=None, act=sas.SAS_GATE_SOFTMAX):
+def run_bwd(B, H, N, topk, mode, seed, learned=False, heads=None, rows=None, act=sas.SAS_GATE_SOFTMAX,
+            pos=sas.SAS_GATE_INNER):
     d = 128
     C = -(-N // 64)
     if learned:
@@ -32,7 +33,8 @@ def run_bwd(B, H, N, topk, mode, seed, learned=False, heads=None, rows=None, act
     else:
         Q, K, V = synth.qkv(B, H, N, d, seed=seed)
         S = synth.scores(B, H, N, C, seed=seed, regime="R1")
-        layer = sas.SasLayer(B, H, N, d, topk, mode=mode, selector=sas.SAS_SEL_SCORES_GIVEN, gate_act=act)
+        layer = sas.SasLayer(B, H, N, d, topk, mode=mode, selector=sas.SAS_SEL_SCORES_GIVEN, gate_act=act,
+                             gate_pos=pos)
     dO = synth.normal((B, H, N, d), seed + 5).to(torch.bfloat16)
     cu = lambda t: None if t is None else t.to(DEV).contiguous()
     Qd, Kd, Vd, dOd = cu(Q), cu(K), cu(V), cu(dO)
@@ -52,10 +54,10 @@ def run_bwd(B, H, N, topk, mode, seed, learned=False, heads=None, rows=None, act
         else:
             s = P.f64(S[bi, hi])
         ref = BO.sas_attention_bwd_head(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s,
-                                        P.f64(dO[bi, hi]), 64, topk, mode, act=act)
+                                        P.f64(dO[bi, hi]), 64, topk, mode, act=act, pos=pos)
         rr = np.arange(N) if rows is None else rows
         extra = P.grad_extra(P.f64(Q[bi, hi]), P.f64(K[bi, hi]), P.f64(V[bi, hi]), s, P.f64(dO[bi, hi]),
-                             P.f64(O[bi, hi].cpu()), 64, topk, mode, act=act)
+                             P.f64(O[bi, hi].cpu()), 64, topk, mode, act=act, pos=pos)
         for name, g in (("dQ", dQ), ("dK", dK), ("dV", dV)):
             r = ref[name][rr]
             P.compare_o(P.f64(g[bi, hi].cpu())[rr], r, f"{name}[{bi},{hi}]", extra[name][rr])
@@ -79,6 +81,13 @@ def test_backward_other_gate_activations(act):
     # Sec. 4.2 gate activation: the same passes on the forward's log-gates; the
     # score gradient reaches kept blocks only (sigmoid: dlogg (1 - g), raw logit: dlogg)
     run_bwd(1, 2, 700, 3, TRAIN, seed=15, act=act)
+
+
+@pytest.mark.parametrize("act", [sas.SAS_GATE_SOFTMAX, sas.SAS_GATE_SIGMOID])
+def test_backward_outer_gate_position(act):
+    # Sec. 4.2 gate position: o = softmax(z) (g . V); dV takes P g dO,
+    # dS = P (g dP - Delta), a block's dlogg is the row sum of P g dP
+    run_bwd(1, 2, 700, 3, TRAIN, seed=16, act=act, pos=sas.SAS_GATE_OUTER)
 
 
 def test_backward_inference_mode_has_no_gate_gradient():

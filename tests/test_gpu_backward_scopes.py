@@ -56,19 +56,20 @@ def _run(layer, Q, K, V, S, dO):
     return g
 
 
-def _check_qkv(g, Q, K, V, S, dO, topk, mode, rows=None):
+def _check_qkv(g, Q, K, V, S, dO, topk, mode, rows=None, act=sas.SAS_GATE_SOFTMAX, pos=sas.SAS_GATE_INNER):
     """dQ per head, dK and dV per group, each within the summed derived bounds."""
     H, Hkv = Q.shape[1], K.shape[1]
     G = H // Hkv
     N = Q.shape[2]
     rr = np.arange(N) if rows is None else rows
-    ref = BO.sas_attention_bwd_gqa(P.f64(Q[0]), P.f64(K[0]), P.f64(V[0]), P.f64(S[0]), P.f64(dO[0]), 64, topk, mode)
+    ref = BO.sas_attention_bwd_gqa(P.f64(Q[0]), P.f64(K[0]), P.f64(V[0]), P.f64(S[0]), P.f64(dO[0]), 64, topk, mode,
+                                   act=act, pos=pos)
     for gk in range(Hkv):
         ek = np.zeros((N, 128))
         ev = np.zeros((N, 128))
         for h in range(gk * G, (gk + 1) * G):
             ex = P.grad_extra(P.f64(Q[0, h]), P.f64(K[0, gk]), P.f64(V[0, gk]), P.f64(S[0, gk]), P.f64(dO[0, h]),
-                              P.f64(g["O"][0, h]), 64, topk, mode)
+                              P.f64(g["O"][0, h]), 64, topk, mode, act=act, pos=pos)
             P.compare_o(P.f64(g["dQ"][0, h])[rr], ref["dQ"][h][rr], f"dQ[{h}]", ex["dQ"][rr])
             ek += ex["dK"]
             ev += ex["dV"]
@@ -182,3 +183,51 @@ def test_ste_rejects_what_it_does_not_cover():
         sas.SasLayer(1, 2, 256, 128, 2, mode=STE, scope=sas.SAS_SCOPE_FULL)
     with pytest.raises(sas.SasError):
         sas.SasLayer(1, 2, 256, 128, 2, mode=STE, gate_act=sas.SAS_GATE_SIGMOID)
+
+
+# --------------------------------------------------------------------- full*
+
+def test_noisy_scope_backward_is_the_sparse_backward_at_the_noisy_scores():
+    # full* (Table 1 setting 11): s~ = s + eps chooses and gates the blocks, and
+    # ds = ds~, so the backward is the sparse one evaluated at s~ (passed as the
+    # scores); the oracle runs on fp32(s + eps)
+    H, N, topk = 2, 700, 3
+    Q, K, V, S, dO = _inputs(H, H, N, 21)
+    eps = (0.5 * synth.normal(tuple(S.shape), 77)).to(torch.float32)
+    St = (S + eps).to(torch.float32)                         # the fp32 sum the forward forms
+    d = lambda t: t.to(DEV).contiguous()
+    layer = sas.SasLayer(1, H, N, 128, topk)
+    Qd, Kd, Vd, dOd = d(Q), d(K), d(V), d(dO)
+    O, LSE, si, sl = layer.attention_noisy(Qd, Kd, Vd, d(eps), scores=d(S))
+    out = layer.attention_bwd(Qd, Kd, Vd, O, LSE, dOd, scores=d(St), sel_idx=si, sel_logg=sl, want_ds=True)
+    torch.cuda.synchronize()
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    g = dict(zip(("dQ", "dK", "dV", "dlogg", "ds"), (t.cpu() for t in out)))
+    g["O"] = O.cpu()
+    s_noisy = OR.noisy_scores(P.f64(S), P.f64(eps))
+    ref = _check_qkv(g, Q, K, V, torch.from_numpy(s_noisy), dO, topk, TRAIN)
+    for h in range(H):
+        tol = _delta_err(g["O"][0, h], dO[0, h]) + 1e-4
+        gl = g["dlogg"][0, h].numpy()[:, :topk]
+        assert np.all(np.abs(gl - ref["dlogg"][h]) <= tol[:, None]), "dlogg"
+        assert np.all(np.abs(g["ds"][0, h].numpy() - ref["ds"][h]) <= 2 * tol[:, None]), "ds"
+
+
+# ------------------------------------------------ outer gate position, GQA
+
+def test_outer_gate_position_gqa_backward():
+    # o = softmax(z) (g . V) under GQA (head-packed tiles in both passes): dK, dV
+    # and the group's d(log g) are sums over its heads; ds from the summed dlogg
+    H, Hkv, N, topk = 4, 2, 517, 2
+    Q, K, V, S, dO = _inputs(H, Hkv, N, 31)
+    layer = sas.SasLayer(1, H, N, 128, topk, Hkv=Hkv, gate_pos=sas.SAS_GATE_OUTER)
+    g = _run(layer, Q, K, V, S, dO)
+    assert g["status"] == 0
+    ref = _check_qkv(g, Q, K, V, S, dO, topk, TRAIN, pos=sas.SAS_GATE_OUTER)
+    G = H // Hkv
+    for gk in range(Hkv):
+        tol = sum(_delta_err(g["O"][0, h], dO[0, h]) for h in range(gk * G, (gk + 1) * G)) + 1e-4
+        gl = g["dlogg"][0, gk].numpy()[:, :topk]
+        assert np.all(np.abs(gl - ref["dlogg"][gk]) <= tol[:, None]), "dlogg"
+        assert np.all(np.abs(g["ds"][0, gk].numpy() - ref["ds"][gk]) <= 2 * tol[:, None]), "ds"
