@@ -231,3 +231,34 @@ def test_outer_gate_position_gqa_backward():
         gl = g["dlogg"][0, gk].numpy()[:, :topk]
         assert np.all(np.abs(gl - ref["dlogg"][gk]) <= tol[:, None]), "dlogg"
         assert np.all(np.abs(g["ds"][0, gk].numpy() - ref["ds"][gk]) <= 2 * tol[:, None]), "ds"
+
+
+def test_full_scope_backward_learned_selector():
+    # the learned selector's full scope: the handle's score table supplies the
+    # log-gates of every block (integer Q, K and sparse {-1, 0, 1} projections,
+    # so the kernel's scores are exact and equal the oracle's)
+    B, H, N, d = 1, 2, 900, 128
+    Q, K, V, Wq, Wk = synth.integer_selector_inputs(B, H, N, d, d, seed=8)
+    dO = synth.normal((B, H, N, d), 13).to(torch.bfloat16)
+    dv = lambda t: t.to(DEV).contiguous()
+    layer = sas.SasLayer(B, H, N, d, 4, selector=sas.SAS_SEL_MEANPOOL_PROJ, d_sel=d, scope=sas.SAS_SCOPE_FULL)
+    Qd, Kd, Vd, dOd = dv(Q), dv(K), dv(V), dv(dO)
+    O, LSE, _, _ = layer.attention(Qd, Kd, Vd, Wq=dv(Wq), Wk=dv(Wk))
+    dQ, dK, dV, dlogg, ds = layer.attention_bwd(Qd, Kd, Vd, O, LSE, dOd)
+    torch.cuda.synchronize()
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
+    C = -(-N // 64)
+    assert ds is None and dlogg.shape == (B, H, N, C)
+    for hi in range(H):
+        s = P.oracle_scores(Q, K, Wq, Wk, 0, hi)
+        args = (P.f64(Q[0, hi]), P.f64(K[0, hi]), P.f64(V[0, hi]), s, P.f64(dO[0, hi]))
+        ref = BO.sas_attention_bwd_full_head(*args, 64)
+        ex = P.grad_extra(*args, P.f64(O[0, hi].cpu()), 64, C, TRAIN)
+        for name, gt in (("dQ", dQ), ("dK", dK), ("dV", dV)):
+            P.compare_o(P.f64(gt[0, hi].cpu()), ref[name], f"{name}[{hi}]", ex[name])
+        tol = _delta_err(O[0, hi].cpu(), dO[0, hi]) + 1e-4
+        gl = dlogg[0, hi].cpu().numpy()
+        for i in range(N):
+            c = i // 64
+            assert np.all(np.abs(gl[i, :c] - ref["dlogg"][i, :c]) <= tol[i]), ("dlogg", hi, i)

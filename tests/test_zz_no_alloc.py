@@ -68,3 +68,27 @@ def test_noalloc_mlp_refuses_sizes_beyond_its_array():
     Y2 = torch.empty(T + 1, D, device=dev, dtype=torch.bfloat16)
     with pytest.raises(sas.SasError, match="exceeds"):
         sas.sas_mlp_fwd_noalloc(X2, W1, W2, Y2)
+
+
+def test_noalloc_mlp_captured_in_a_cuda_graph():
+    # the entry point's purpose: a CUDA graph capture fails on any allocation,
+    # so a call captured (after one warm-up call outside the capture, which sets
+    # the kernels' attributes) and replayed must reproduce the eager result
+    dev = torch.device("cuda:0")
+    T, D, F = 300, 256, 1024
+    X, W1, W2, b1, b2 = (t.to(dev) for t in synth.mlp(T, D, F, seed=6, bias=True))
+    Y = torch.empty(T, D, device=dev, dtype=torch.bfloat16)
+    sas.sas_mlp_fwd_noalloc(X, W1, W2, Y, b1, b2)
+    torch.cuda.synchronize()
+    assert sas.sas_mlp_noalloc_get_device_status() == sas.SAS_OK
+    eager = Y.clone()
+    Y.zero_()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        sas.sas_mlp_fwd_noalloc(X, W1, W2, Y, b1, b2)
+    for _ in range(2):
+        Y.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(Y, eager)
+    assert sas.sas_mlp_noalloc_get_device_status() == sas.SAS_OK
