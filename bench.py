@@ -424,7 +424,10 @@ def run_ours(args, w, rank, world):
     fl = packed_flops(w) if lens else algorithmic_flops(w, learned)
     tflop = fl["total"] / 1e12
     value = job_throughput(tflop, world, ms)
-    per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None)} for k, (n, t) in kt.items()}
+    # per kind: launches in the timed steps, time per launch and per step (a kind
+    # may launch twice a step: head-packed tiles add the segment unions to the selection)
+    per_kind = {k: {"launches": n, "ms_per_launch": (t / n if n else None), "ms_per_step": (t / args.steps if n else None)}
+                for k, (n, t) in kt.items()}
     flops_per_launch = {"attention": fl["attention"], "mlp_up_gelu": fl["mlp"] / 2, "mlp_down": fl["mlp"] / 2}
     dom = max((k for k in kt if kt[k][0] > 0), key=lambda k: kt[k][1])
     peaks = load_peaks()
@@ -466,7 +469,7 @@ def run_ours(args, w, rank, world):
         exe = work_blocks * 4 * 128 * 64 * d
         a_alg = fl["attention"] / (a_avg / 1e3) / 1e12
         a_exe = exe / (a_avg / 1e3) / 1e12
-        sas_ms = sum(kt[k][1] / max(kt[k][0], 1) for k in ("block_summaries", "selection", "attention"))
+        sas_ms = sum(kt[k][1] / args.steps for k in ("block_summaries", "selection", "attention"))
         out["attention_kernel"] = {
             "ms": round(a_avg, 4), "algorithmic_tflops": round(a_alg, 1),
             "frac_of_bf16_peak": round(a_alg / peaks["bf16"], 4),
@@ -477,8 +480,8 @@ def run_ours(args, w, rank, world):
             "mean_union_blocks_per_tile": round(sum(unions) / max(len(unions), 1), 2)}
         out["sas_layer"] = {"ms": round(sas_ms, 4),
                             "algorithmic_tflops": round((fl["attention"] + fl["selector"]) / (sas_ms / 1e3) / 1e12, 1),
-                            "selection_ms": round(kt["selection"][1] / max(kt["selection"][0], 1), 4),
-                            "block_summaries_ms": round(kt["block_summaries"][1] / max(kt["block_summaries"][0], 1), 4)}
+                            "selection_ms": round(kt["selection"][1] / args.steps, 4),
+                            "block_summaries_ms": round(kt["block_summaries"][1] / args.steps, 4)}
     if not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget, learned=learned, workload=args.workload,
                                            topk=args.topk)
@@ -653,7 +656,11 @@ def run_train(args, w, rank, world):
     the score gradient is produced too; GQA workloads share K, V, the kept
     sets and the gates per KV group, packed ones run every sequence as its own
     problem.  Algorithmic FLOPs: the forward's 4 d per attended (row, key)
-    pair plus the backward's 10 d (QK^T, dO V^T, dS K, dS^T Q, P^T dO)."""
+    pair plus the backward's 10 d (QK^T, dO V^T, dS K, dS^T Q, P^T dO).
+    --train-form full: the full training scope (every historical block kept
+    and gated: K = C_i in those counts).  --train-form ste: the hard Top-K gate
+    under the straight-through estimator (the hard forward and backward, plus
+    the gate gradient of every historical key: q.k and dO.v, 4 d a pair)."""
     import numpy as np
     import torch
 
@@ -671,12 +678,17 @@ def run_train(args, w, rank, world):
     S = synth.scores(B, Hkv, N, C, seed=rank, regime="R1")
     dO = synth.normal((B, H, N, d), rank + 5).to(torch.bfloat16)
     Qd, Kd, Vd, Sd, dOd = (t.to(dev) for t in (Q, Kk, V, S, dO))
+    form = args.train_form
+    if form != "sparse" and lens:
+        raise SystemExit("--train-form full / ste take [B, H, N, d] workloads")
     if lens:
         layer = sas.SasLayer(1, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv, max_seqs=len(lens),
                              max_seqlen=max(lens))
         cud = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
     else:
-        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv)
+        layer = sas.SasLayer(B, H, N, d, K, selector=sas.SAS_SEL_SCORES_GIVEN, Hkv=Hkv,
+                             mode=sas.SAS_MODE_TRAIN_HARD_STE if form == "ste" else sas.SAS_MODE_TRAIN_SOFT,
+                             scope=sas.SAS_SCOPE_FULL if form == "full" else sas.SAS_SCOPE_SPARSE)
     h = layer.h
     stream = torch.cuda.current_stream(dev)
     O = torch.empty_like(Qd)
@@ -684,8 +696,10 @@ def run_train(args, w, rank, world):
     si = torch.empty(B, Hkv, N, max(K, 1), device=dev, dtype=torch.int32)
     sl = torch.empty(B, Hkv, N, max(K, 1), device=dev, dtype=torch.float32)
     dQ, dK, dV = torch.empty_like(Qd), torch.empty_like(Kd), torch.empty_like(Vd)
-    dl = torch.empty_like(sl)
+    dl = torch.empty_like(sl) if form == "sparse" else torch.empty(B, Hkv, N, C, device=dev, dtype=torch.float32)
     ds = torch.empty_like(Sd)
+    if form == "full":
+        si = sl = None   # the full scope keeps no Top-K
     flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
 
     def step():
@@ -723,22 +737,29 @@ def run_train(args, w, rank, world):
         used = sum((n + 127) // 128 for n in lens)
         unions = [unions[g * Tt + k] for g in range(Hkv) for k in range(used)]
     layer.close()
-    fl = packed_flops(w) if lens else algorithmic_flops(w, learned=False)
+    fl = packed_flops(w) if lens else algorithmic_flops(dict(w, topk=C) if form == "full" else w, learned=False)
     f_fwd = fl["attention"]
     f_bwd = f_fwd * 10 // 4
+    if form == "ste":
+        # the estimator's gate pass: q.k and dO.v for every historical key of every row
+        hist = sum(min(64, N - 64 * c) * 64 * c for c in range((N + 63) // 64))
+        f_bwd += 4 * d * B * H * hist
     tflop = (f_fwd + f_bwd) / 1e12
     peaks = load_peaks()
-    bwd_ms = kt["attention_bwd"][1] / max(kt["attention_bwd"][0], 1)
-    fwd_ms = kt["attention"][1] / max(kt["attention"][0], 1)
-    sel_ms = kt["selection"][1] / max(kt["selection"][0], 1)
+    # per step (the hard-STE backward is two launches of its kind, head-packed
+    # selection two: the Top-K and the segment unions)
+    bwd_ms = kt["attention_bwd"][1] / args.steps
+    fwd_ms = kt["attention"][1] / args.steps
+    sel_ms = kt["selection"][1] / args.steps
     ach = f_bwd / (bwd_ms / 1e3) / 1e12
     return {
         "metric": TRAIN_METRIC, "value": round(tflop / (ms / 1e3), 2), "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 softmax and gradients of log g, s)",
         "data": "synthetic (seeded; R1 block-coherent scores given, N(0,1) Q/K/V/dO)",
-        "config": {"workload": w["name"] + " (attention only, forward + backward)", "B": B, "H": H, "Hkv": Hkv,
-                   "N": N, "d": d, "topk": K, "packed_lengths": lens,
+        "config": {"workload": w["name"] + " (attention only, forward + backward)"
+                   + {"sparse": "", "full": ", full training scope", "ste": ", hard Top-K gate with STE"}[form],
+                   "B": B, "H": H, "Hkv": Hkv, "N": N, "d": d, "topk": K, "packed_lengths": lens, "form": form,
                    "l2": "flushed between timed steps (256 MiB write)", "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "tensor", "kernel": "attention_bwd", "achieved": round(ach, 1), "peak": peaks["bf16"],
                      "unit": "TFLOP/s", "frac": round(ach / peaks["bf16"], 4), "traffic": None,
@@ -1002,6 +1023,8 @@ def main():
                     help="decode: run one arm only (for profiling)")
     ap.add_argument("--train", action="store_true",
                     help="time the attention training step (forward + backward) of the workload instead")
+    ap.add_argument("--train-form", choices=["sparse", "full", "ste"], default="sparse",
+                    help="--train: the sparse scope (SAS), the full training scope, or the hard Top-K gate with STE")
     ap.add_argument("--regime", choices=["R2", "R1"], default="R2",
                     help="R2: learned selector on block-correlated queries; R1: block-coherent scores given")
     ap.add_argument("--topk", type=int, default=None, help="override the workload's K")
