@@ -95,6 +95,28 @@ def algorithmic_flops(w, learned=True):
             "total": BH * (attn + sel) + mlp}
 
 
+def train_flops(w, form="sparse"):
+    """(forward, backward) algorithmic FLOPs of one attention training step:
+    the forward's 4 d per attended (row, key) pair and the backward's 10 d.
+    form "full": the full training scope (every historical block kept: K = C_i
+    in those counts); "ste": the hard Top-K gate under the straight-through
+    estimator, whose gate pass adds q.k and dO.v (4 d) for every historical
+    key of every row; "sparse": the SAS scope."""
+    lens = w.get("lens")
+    if lens:
+        fl = packed_flops(w)
+    else:
+        C = (w["N"] + 63) // 64
+        fl = algorithmic_flops(dict(w, topk=C) if form == "full" else w, learned=False)
+    f_fwd = fl["attention"]
+    f_bwd = f_fwd * 10 // 4
+    if form == "ste":
+        N, d = w["N"], w["d"]
+        hist = sum(min(64, N - 64 * c) * 64 * c for c in range((N + 63) // 64))
+        f_bwd += 4 * d * w["B"] * w["H"] * hist
+    return f_fwd, f_bwd
+
+
 def packed_flops(w, learned=False):
     """algorithmic_flops summed over the packed sequences (the MLP runs on all tokens)."""
     att = sel = 0
@@ -737,13 +759,7 @@ def run_train(args, w, rank, world):
         used = sum((n + 127) // 128 for n in lens)
         unions = [unions[g * Tt + k] for g in range(Hkv) for k in range(used)]
     layer.close()
-    fl = packed_flops(w) if lens else algorithmic_flops(dict(w, topk=C) if form == "full" else w, learned=False)
-    f_fwd = fl["attention"]
-    f_bwd = f_fwd * 10 // 4
-    if form == "ste":
-        # the estimator's gate pass: q.k and dO.v for every historical key of every row
-        hist = sum(min(64, N - 64 * c) * 64 * c for c in range((N + 63) // 64))
-        f_bwd += 4 * d * B * H * hist
+    f_fwd, f_bwd = train_flops(w, form)
     tflop = (f_fwd + f_bwd) / 1e12
     peaks = load_peaks()
     # per step (the hard-STE backward is two launches of its kind, head-packed

@@ -41,3 +41,17 @@ def test_backward_flops_are_ten_d_per_attended_pair():
     # the oracle's backward count equals 10/4 of the forward's attention count per head
     N, K, d = 900, 5, 128
     assert BO.backward_flops_head(N, 64, K, d) * 4 == _rows(N, K, d) * 10
+
+
+def test_training_flops_of_the_three_forms():
+    # sparse: 4 d + 10 d per attended pair; full scope: every key j <= i of row i
+    # attended (K = C_i); hard-STE: the sparse count plus 4 d per historical key
+    N, K, d, B, H = 700, 3, 128, 2, 3
+    w = dict(B=B, H=H, N=N, d=d, topk=K, d_sel=128, D=64, F=64)
+    fwd, bwd = bench.train_flops(w, "sparse")
+    assert fwd == B * H * _rows(N, K, d) and bwd * 4 == fwd * 10
+    fwd_f, bwd_f = bench.train_flops(w, "full")
+    assert fwd_f == B * H * sum(4 * d * (i + 1) for i in range(N)) and bwd_f * 4 == fwd_f * 10
+    fwd_s, bwd_s = bench.train_flops(w, "ste")
+    assert fwd_s == fwd
+    assert bwd_s - bwd == B * H * sum(4 * d * 64 * (i // 64) for i in range(N))
