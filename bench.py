@@ -355,7 +355,8 @@ def run_ours(args, w, rank, world):
         hX = X.pin_memory()
         hY = torch.empty(T, D, dtype=torch.bfloat16).pin_memory()
     G = H // Hkv if attn else 1
-    gk = Hkv if (not attn or lens) else next(k for k in range(1, Hkv + 1) if Hkv % k == 0 and B * Hkv // k <= 8)
+    max_groups = args.e2e_groups
+    gk = Hkv if (not attn or lens) else next(k for k in range(1, Hkv + 1) if Hkv % k == 0 and B * Hkv // k <= max_groups)
     groups = [(b, kv0) for b in range(B) for kv0 in range(0, Hkv, gk)] if attn else []
     ghandle = None
     if attn and not lens:
@@ -1050,6 +1051,7 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=4.0)
     ap.add_argument("--oracle-sample-only", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--e2e-groups", type=int, default=8, help=argparse.SUPPRESS)   # streamed head groups, at most
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
