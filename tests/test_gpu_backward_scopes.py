@@ -142,6 +142,7 @@ def test_full_scope_backward_beyond_64_blocks():
     (2, 2, 700, 3, 11),        # ragged, several tiles
     (4, 2, 517, 2, 12),        # GQA (head-packed tiles in the hard backward)
     (2, 2, 300, 0, 13),        # K = 0: every historical block is dropped
+    (2, 2, 250, 8, 14),        # K >= C_i: every historical block is kept (the gates are all 1)
 ])
 def test_ste_backward_matches_oracle(H, Hkv, N, topk, seed):
     Q, K, V, S, dO = _inputs(H, Hkv, N, seed)
@@ -183,6 +184,18 @@ def test_ste_rejects_what_it_does_not_cover():
         sas.SasLayer(1, 2, 256, 128, 2, mode=STE, scope=sas.SAS_SCOPE_FULL)
     with pytest.raises(sas.SasError):
         sas.SasLayer(1, 2, 256, 128, 2, mode=STE, gate_act=sas.SAS_GATE_SIGMOID)
+    # packed sequences: the forward runs, the estimator's backward is refused before any launch
+    N, d = 512, 128
+    layer = sas.SasLayer(1, 2, N, d, 2, mode=STE, max_seqs=2, max_seqlen=300)
+    Q, K, V = (t[0].to(DEV) for t in synth.qkv(1, 2, N, d, seed=3))
+    S = synth.scores(1, 2, N, 5, seed=3)[0].to(DEV)
+    cu = torch.tensor([0, 300, 512], dtype=torch.int32, device=DEV)
+    O, LSE, si, sl = layer.attention_varlen(cu, Q, K, V, S)
+    with pytest.raises(sas.SasError, match="take \\[B, H, N, d\\] inputs"):
+        layer.attention_bwd_varlen(Q, K, V, O, LSE, torch.zeros_like(Q), scores=S, sel_idx=si, sel_logg=sl)
+    torch.cuda.synchronize()
+    assert sas.sas_get_device_status(layer.h) == 0
+    layer.close()
 
 
 # --------------------------------------------------------------------- full*
